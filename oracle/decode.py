@@ -1,0 +1,231 @@
+"""Greedy self-speculative decoding and plain greedy AR decoding (oracle, float64).
+
+Test infrastructure only.  Follows the paper's round (Appendix "Self-Speculative
+Decoding and KV-Cache Update", steps State / Draft forward / Verify forward /
+Accept / Cache update / Next round; Sec. 4.3; Fig. "Self-speculative
+decoding"):
+
+* State: the cache holds causal KV states of every committed token except the
+  boundary token x0, the last committed one.  The first x0 is the argmax at
+  the prefill's last position.
+* Draft forward: window [x0, [M] x K] at slots n..n+K.  The boundary row
+  attends causally (keys 0..n); every mask row attends to the cache and to the
+  whole window (keys 0..n+K).  a0 = argmax of the boundary row, d_j = argmax of
+  mask row j (shifted alignment: the prediction for slot p is read from the
+  row at slot p-1, Sec. 4.2 and Appendix "Direct Block-Diffusion Decoding").
+* Verify forward: [a0, d_1..d_K] at slots n+1..n+K+1, token-level causal
+  (row i sees keys 0..n+1+i); it overwrites the draft's states of the mask
+  slots.  a_{i+1} = argmax of row i.
+* Accept: A = largest j <= K with d_1..d_j == a_1..a_j; commit a0, d_1..d_A,
+  a_{A+1}; keep slots 0..n+1+A (seq_len n+A+2); the next boundary is a_{A+1}.
+* Stop: the committed run is cut at the first stop token (or at the output
+  cap) and the rest of the round is dropped.
+
+Where the paper is silent the design notes fix the reading (architecture,
+[M] id = V-1, causal prefix attention, ties broken to the lowest token id,
+absolute RoPE positions of mask slots, output cap counting the prefill's x0).
+"""
+from __future__ import annotations
+
+import dataclasses
+from typing import List, Optional
+
+import numpy as np
+
+from synth import bf16_bits_to_f32
+
+from .model import Decoder, KVCache
+
+
+def argmax_rows(logits: np.ndarray) -> np.ndarray:
+    """Greedy token per row; ties go to the lowest token id (np.argmax is first-max)."""
+    return np.argmax(logits, axis=1).astype(np.int64)
+
+
+def top2_gap(logits: np.ndarray) -> np.ndarray:
+    """Top-1 minus top-2 logit per row (the near-tie margin)."""
+    part = np.partition(logits, -2, axis=1)
+    return part[:, -1] - part[:, -2]
+
+
+@dataclasses.dataclass
+class SeqState:
+    """Decoding state of one sequence between rounds."""
+    cache: KVCache
+    x0: int                 # boundary token (committed, not yet in the cache)
+    out: List[int]          # committed output tokens, x0 included
+    max_new: int            # cap on len(out)
+    eos: int = -1
+    done: bool = False
+
+    @property
+    def n(self) -> int:
+        return self.cache.seq_len
+
+
+@dataclasses.dataclass
+class RoundResult:
+    a0: int
+    d_draft: np.ndarray     # draft argmax d_1..d_K (before any forcing)
+    d: np.ndarray           # drafts fed to the verifier (after forcing)
+    a: np.ndarray           # verifier predictions a_1..a_{K+1}
+    A: int                  # accepted draft length
+    committed: List[int]    # tokens this round commits (after stop truncation)
+    draft_logits: np.ndarray
+    verify_logits: np.ndarray
+    draft_gap: np.ndarray   # top-2 gaps of the draft rows [K+1]
+    verify_gap: np.ndarray  # top-2 gaps of the verify rows [K+1]
+
+
+# ------------------------------------------------------------------ prefill
+def prefill(dec: Decoder, vis_bits: np.ndarray, text: np.ndarray, capacity: int,
+            max_new: int, eos: int = -1) -> SeqState:
+    """Causal forward over [visual embeddings; text tokens] at slots 0..P-1.
+
+    The visual rows replace token embeddings at positions 0..n_vis-1.  The
+    prefix is causal (the base decoder is a causal AR model, Sec. 3).  The
+    first boundary x0 is the argmax at the last prefix position; it is the
+    first committed output token (Appendix, step "State").
+    """
+    vis = bf16_bits_to_f32(vis_bits).astype(np.float64)
+    x = np.concatenate([vis, dec.embed_tokens(text)], axis=0)
+    P = x.shape[0]
+    cache = KVCache(dec.cfg, capacity)
+    slots = np.arange(P)
+    allowed = slots[None, :] <= slots[:, None]                     # causal
+    logits = dec.forward(x, slots, allowed, cache)
+    cache.seq_len = P
+    x0 = int(argmax_rows(logits[-1:])[0])
+    st = SeqState(cache=cache, x0=x0, out=[x0], max_new=max_new, eos=eos)
+    st.done = (x0 == eos) or (len(st.out) >= max_new)
+    return st
+
+
+# ------------------------------------------------------------------ forwards
+def draft_forward(dec: Decoder, cache: KVCache, x0: int, K: int) -> np.ndarray:
+    """Draft forward over [x0, [M] x K] at slots n..n+K (hybrid mask).
+
+    Row 0 (boundary) sees keys 0..n; rows 1..K see keys 0..n+K.  Writes the
+    window's KV states (x0's causal state at slot n; the mask slots get
+    bidirectional states that the verify forward overwrites).  Returns logits
+    [K+1, V].
+    """
+    n = cache.seq_len
+    ids = np.array([x0] + [dec.cfg.mask_token_id] * K)
+    slots = n + np.arange(K + 1)
+    keys = np.arange(n + K + 1)
+    allowed = np.empty((K + 1, n + K + 1), dtype=bool)
+    allowed[0] = keys <= n
+    allowed[1:] = True
+    return dec.forward(dec.embed_tokens(ids), slots, allowed, cache)
+
+
+def verify_forward(dec: Decoder, cache: KVCache, a0: int, d: np.ndarray) -> np.ndarray:
+    """Verify forward over [a0, d_1..d_K] at slots n+1..n+K+1, token-level causal.
+
+    Row i sees keys 0..n+1+i, i.e. the cache, x0 (written by the draft) and
+    the verify window up to itself.  Returns logits [K+1, V].
+    """
+    n = cache.seq_len
+    K = len(d)
+    ids = np.concatenate([[a0], np.asarray(d, dtype=np.int64)])
+    slots = n + 1 + np.arange(K + 1)
+    keys = np.arange(n + K + 2)
+    allowed = keys[None, :] <= slots[:, None]
+    return dec.forward(dec.embed_tokens(ids), slots, allowed, cache)
+
+
+def ar_step_forward(dec: Decoder, cache: KVCache, token: int) -> np.ndarray:
+    """One plain AR step: feed ``token`` at slot n (keys 0..n). Returns logits [1, V]."""
+    n = cache.seq_len
+    allowed = np.ones((1, n + 1), dtype=bool)
+    logits = dec.forward(dec.embed_tokens([token]), np.array([n]), allowed, cache)
+    cache.seq_len = n + 1
+    return logits
+
+
+# ------------------------------------------------------------------ accept
+def accept_length(d: np.ndarray, a: np.ndarray) -> int:
+    """A = length of the longest prefix with d_j == a_j (1 <= j <= K)."""
+    A = 0
+    for dj, aj in zip(d, a):
+        if int(dj) != int(aj):
+            break
+        A += 1
+    return A
+
+
+def forced_drafts(d: np.ndarray, teacher: np.ndarray, n: int, L: int, vocab: int) -> np.ndarray:
+    """Benchmark hook (not in the paper): force the accepted length to L.
+
+    ``teacher[p]`` is the greedy-AR token at absolute slot p.  Drafts d_j sit at
+    slot n+1+j, so d_j := teacher[n+1+j] for j <= L, and d_{L+1} :=
+    (teacher[n+2+L] + 1) mod V when L < K, so that the verifier rejects it.
+    """
+    d = np.array(d, dtype=np.int64)
+    K = len(d)
+    for j in range(1, min(L, K) + 1):
+        d[j - 1] = teacher[n + 1 + j]
+    if L < K:
+        d[L] = (int(teacher[n + 2 + L]) + 1) % vocab
+    return d
+
+
+# ------------------------------------------------------------------ round
+def self_spec_round(dec: Decoder, st: SeqState, K: int, teacher: Optional[np.ndarray] = None,
+                    L: Optional[int] = None) -> RoundResult:
+    """One greedy self-speculative round; updates ``st`` in place."""
+    assert not st.done
+    cache = st.cache
+    n = cache.seq_len
+    dl = draft_forward(dec, cache, st.x0, K)
+    tok = argmax_rows(dl)
+    a0, d_draft = int(tok[0]), tok[1:].copy()
+    d = d_draft if teacher is None else forced_drafts(d_draft, teacher, n, L, dec.cfg.vocab)
+    vl = verify_forward(dec, cache, a0, d)
+    a = argmax_rows(vl)                                    # a_1..a_{K+1}
+    A = accept_length(d, a[:K])
+    run = [a0] + [int(x) for x in d[:A]] + [int(a[A])]
+    # stop condition: cut at the first stop token or at the output cap
+    committed = []
+    for t in run:
+        committed.append(t)
+        if t == st.eos or len(st.out) + len(committed) >= st.max_new:
+            st.done = True
+            break
+    st.out.extend(committed)
+    # cache update: causal states of x0, a0, d_1..d_A stay (slots n..n+1+A)
+    cache.truncate(n + A + 2)
+    st.x0 = int(a[A])
+    return RoundResult(a0=a0, d_draft=d_draft, d=d, a=a, A=A, committed=committed,
+                       draft_logits=dl, verify_logits=vl,
+                       draft_gap=top2_gap(dl), verify_gap=top2_gap(vl))
+
+
+def self_spec_decode(dec: Decoder, st: SeqState, K: int, teacher: Optional[np.ndarray] = None,
+                     schedule: Optional[np.ndarray] = None, max_rounds: int = 1 << 30
+                     ) -> List[RoundResult]:
+    rounds = []
+    while not st.done and len(rounds) < max_rounds:
+        L = None if schedule is None else int(schedule[len(rounds)])
+        rounds.append(self_spec_round(dec, st, K, teacher, L))
+    return rounds
+
+
+def ar_decode(dec: Decoder, st: SeqState) -> List[int]:
+    """Plain greedy AR from the prefill state: one causal step per token (Eq. 1)."""
+    while not st.done:
+        logits = ar_step_forward(dec, st.cache, st.x0)
+        st.x0 = int(argmax_rows(logits)[0])
+        st.out.append(st.x0)
+        if st.x0 == st.eos or len(st.out) >= st.max_new:
+            st.done = True
+    return st.out
+
+
+def tokens_per_forward(committed_per_round: List[int]) -> float:
+    """TPF (Sec. 5 "Efficiency Measurement"): committed tokens / forwards, counting
+    the draft and the verify forward of every round separately, prefill excluded."""
+    if not committed_per_round:
+        return 0.0
+    return float(sum(committed_per_round)) / (2.0 * len(committed_per_round))
