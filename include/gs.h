@@ -1,0 +1,222 @@
+/*
+ * gs.h -- C ABI of libgs: greedy self-speculative draft/verify decoding with a
+ * shared-parameter AR / block-diffusion decoder on one GB300 (sm_103a).
+ *
+ * The method (paper Sec. 4.3 "Self-Speculative Decoding", Fig. "Self-speculative
+ * decoding", Appendix "Self-Speculative Decoding and KV-Cache Update"): every
+ * round runs one DRAFT forward over [x0, [M] x K] with the hybrid mask (the
+ * boundary row x0 causal to the cache, the K mask rows bidirectional inside
+ * the window), then one VERIFY forward over [a0, d_1..d_K] with token-level
+ * causal attention, accepts the longest prefix with d_j == a_j, commits
+ * a0, d_1..d_A, a_{A+1} and rolls the KV cache back to the accepted prefix.
+ * The first boundary x0 is the argmax at the prefill's last position.
+ *
+ * Conventions shared by every entry point
+ *  - Device pointers are CUDA global-memory addresses on the current device;
+ *    host pointers are ordinary process memory.  Each argument says which.
+ *  - The caller owns every buffer it passes (weights, workspace, inputs,
+ *    outputs) and the stream.  After gs_create the library allocates no
+ *    device memory; it carves everything from the caller's workspace.
+ *  - Work is enqueued asynchronously on the handle's stream unless stated.
+ *  - bf16 tensors are IEEE bfloat16 bit patterns, row-major.
+ *  - Return value: GS_OK (0) or one of the GS_ERR_* codes below; the message
+ *    of the last failure is available from gs_last_error().  Kernel-side
+ *    checks (slot ids, token ids, bounded waits) raise a device error word
+ *    that gs_sync_check() turns into GS_ERR_DEVICE_CHECK / GS_ERR_TIMEOUT.
+ */
+#ifndef GS_H_
+#define GS_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+enum {
+  GS_OK = 0,
+  GS_ERR_INVALID_ARG = 1,   /* bad pointer, size, slot or config value        */
+  GS_ERR_OOM = 2,           /* workspace too small / KV page pool exhausted    */
+  GS_ERR_UNSUPPORTED = 3,   /* valid request this build does not implement     */
+  GS_ERR_CUDA = 4,          /* a CUDA runtime call failed                      */
+  GS_ERR_DEVICE_CHECK = 5,  /* a kernel's bounds check fired                   */
+  GS_ERR_TIMEOUT = 6        /* a kernel's bounded wait ran out                 */
+};
+
+/* Acceptance rule (paper Sec. 3 "Speculative Decoding"): greedy accepts drafts
+ * while they equal the verifier's argmax; stochastic (rejection sampling) is
+ * named by the paper but not used in its experiments -> GS_ERR_UNSUPPORTED. */
+typedef enum { GS_ACCEPT_GREEDY = 0, GS_ACCEPT_STOCHASTIC = 1 } gs_accept_rule;
+
+/* Decoder shape and capacity.  The paper does not print the architecture; the
+ * library implements a pre-norm decoder: RMSNorm (learned gain, eps) ->
+ * grouped-query attention with rotate-half RoPE on all head dims at absolute
+ * positions -> RMSNorm -> SwiGLU FFN; untied input/output embeddings, no
+ * biases.  Requirements: head_dim 64, n_heads % n_kv_heads == 0,
+ * d_model % 128 == 0, (n_heads + 2 n_kv_heads) * 64 % 128 == 0,
+ * d_ffn % 64 == 0, vocab % 128 == 0. */
+typedef struct {
+  int n_layers, d_model, n_heads, n_kv_heads, head_dim, d_ffn, vocab;
+  float rope_theta, rms_eps;
+  int mask_token_id;   /* the [M] embedding row (paper Sec. 4, "AR-to-Diffusion Conversion") */
+  int eos_token_id;    /* stop token, -1 = none (Appendix step "Next round")              */
+  int max_batch;       /* sequence slots                                                  */
+  int max_ctx;         /* slots one sequence may reserve: prefix + max_new + max_K + 2   */
+  int max_K;           /* largest block size a round may use                              */
+  int max_prefill;     /* tokens per prefill chunk (longer prefixes run in chunks)        */
+  int kv_pages;        /* 64-token pages in the KV pool; 0 = max_batch * ceil(max_ctx/64) */
+  int split_pages;     /* attention pages per KV split (decode); 0 = automatic             */
+} gs_config;
+
+/* Weights: device pointers to bf16 arrays owned by the caller, row-major
+ * [out_features, in_features].  Per-layer fields are HOST arrays of n_layers
+ * device pointers (copied by gs_create).
+ *   embed [vocab, d]   lm_head [vocab, d]   final_norm [d]
+ *   attn_norm [d]   w_qkv [(Hq + 2 Hkv) * 64, d]  (q heads, then k heads, then v heads)
+ *   w_o [d, Hq * 64]   ffn_norm [d]   w_gate_up [2 d_ffn, d] (gate rows, then up rows)
+ *   w_down [d, d_ffn]
+ * Every pointer must be 16-byte aligned. */
+typedef struct {
+  const void *embed, *lm_head, *final_norm;
+  const void *const *attn_norm, *const *w_qkv, *const *w_o,
+             *const *ffn_norm, *const *w_gate_up, *const *w_down;
+} gs_weights;
+
+/* Forced acceptance (benchmark hook, not in the paper).  After the draft
+ * argmax, for the sequence in slot s at round r with L = L_sched[row * L_stride + r]
+ * (row = the sequence's index in this call's slot list, r = the number of
+ * rounds the sequence has run since its prefill):
+ *   d_j := teacher[row * teacher_stride + n + 1 + j]    for 1 <= j <= L
+ *   d_{L+1} := (teacher[row * teacher_stride + n + 2 + L] + 1) mod vocab  if L < K
+ * where n is the sequence's cached length at the round's start and teacher[p]
+ * is the greedy token at absolute slot p.  All pointers are device int32. */
+typedef struct {
+  const int32_t *teacher;
+  int64_t teacher_stride;
+  const int32_t *L_sched;
+  int64_t L_stride;
+} gs_force;
+
+/* Optional per-round diagnostics (device pointers, any may be NULL).  A round
+ * given a non-NULL gs_debug runs outside the CUDA-graph cache.
+ *   draft_tok  int32 [n_seq, K+1]   argmax of the draft rows (a0, d_1..d_K)
+ *   verify_in  int32 [n_seq, K+1]   verify inputs after forcing (a0, d_1..d_K)
+ *   verify_tok int32 [n_seq, K+1]   argmax of the verify rows (a_1..a_{K+1})
+ *   draft_logits / verify_logits fp32 [n_seq, K+1, vocab] */
+typedef struct {
+  int32_t *draft_tok, *verify_in, *verify_tok;
+  float *draft_logits, *verify_logits;
+} gs_debug;
+
+typedef struct gs_handle gs_handle;
+
+/* Bytes of device workspace gs_create needs for this config (KV page pool,
+ * page table, per-sequence state, activations, split scratch).  0 if the
+ * config is invalid. */
+size_t gs_workspace_bytes(const gs_config *cfg);
+
+/* Build a handle.  cfg, w: host structs (copied).  workspace: device memory of
+ * at least gs_workspace_bytes(cfg) bytes, 256-byte aligned, owned by the
+ * caller and not touched by anyone else until gs_destroy.  stream: a
+ * cudaStream_t (NULL = legacy default stream).  Zeroes the workspace and
+ * builds the TMA descriptors; synchronises the stream before returning.
+ * Errors: GS_ERR_INVALID_ARG, GS_ERR_UNSUPPORTED (shape), GS_ERR_OOM
+ * (workspace too small), GS_ERR_CUDA. */
+int gs_create(const gs_config *cfg, const gs_weights *w, void *workspace, size_t ws_bytes,
+              void *stream, gs_handle **out);
+
+/* Release the handle (graphs, host tables).  Frees no caller memory. */
+int gs_destroy(gs_handle *h);
+
+/* Message of the last failure on this handle ("" if none).  NULL handle gives
+ * the last failure of gs_create in this thread. */
+const char *gs_last_error(gs_handle *h);
+
+/* Prefill (paper Appendix step "State"; Sec. 3 task formulation: image I and
+ * prompt c).  Reserves KV pages for n_vis + n_text + max_new + max_K + 2
+ * slots in sequence slot `slot` (freeing whatever the slot held), runs a
+ * causal forward over the visual rows then the text tokens, sets the cached
+ * length to P = n_vis + n_text and the boundary x0 to the argmax at position
+ * P-1, which is the first committed output token.
+ *   vis_emb  device bf16 [n_vis, d_model] (may be NULL when n_vis == 0)
+ *   text     device int32 [n_text], ids in [0, vocab)
+ *   max_new  cap on committed output tokens, x0 included (>= 1)
+ *   x0_out   device int32 [1] or NULL
+ * Errors: GS_ERR_INVALID_ARG, GS_ERR_OOM (pool exhausted or ctx too long). */
+int gs_prefill(gs_handle *h, int slot, const void *vis_emb, int n_vis, const int32_t *text,
+               int n_text, int max_new, int32_t *x0_out);
+
+/* One self-speculative round for n_seq sequences (paper Appendix steps Draft
+ * forward / Verify forward / Accept / Cache update / Next round).
+ *   slots    device int32 [n_seq], distinct prefilled slots
+ *   K        block size, 0 <= K <= max_K (K = 0 is two plain AR steps)
+ *   rule     GS_ACCEPT_GREEDY
+ *   force    NULL for natural drafting, else the forcing hook above
+ *   out_tok  device int32 [n_seq, K+2]: committed tokens of this round
+ *   out_cnt  device int32 [n_seq]: how many (0 for a sequence already done)
+ *   out_done device int32 [n_seq]: 1 once the sequence hit EOS or max_new
+ *   dbg      NULL, or diagnostics (see gs_debug)
+ * Rounds with the same (n_seq, K, pointers) replay one cached CUDA graph; no
+ * host synchronisation happens inside or between rounds. */
+int gs_round(gs_handle *h, const int32_t *slots, int n_seq, int K, int rule, const gs_force *force,
+             int32_t *out_tok, int32_t *out_cnt, int32_t *out_done, const gs_debug *dbg);
+
+/* Overwrite a sequence's boundary token and output count (resume/checkpoint
+ * of the per-sequence state: the cache is described by its length alone).
+ *   seq_len   new cached length, 1 <= seq_len <= current cached length (rollback only)
+ *   x0        boundary token, n_out committed-token count (x0 included)
+ * Host values; enqueued on the stream.  Errors: GS_ERR_INVALID_ARG. */
+int gs_seq_restore(gs_handle *h, int slot, int seq_len, int x0, int n_out, int done);
+
+/* Read one slot's state (synchronises the stream).  Any out pointer may be NULL. */
+int gs_seq_state(gs_handle *h, int slot, int *seq_len, int *x0, int *n_out, int *done, int *rounds);
+
+/* Free the slot's KV pages (host bookkeeping only). */
+int gs_release(gs_handle *h, int slot);
+
+/* Synchronise the stream and report a kernel-side check or bounded-wait
+ * failure raised since the last call (then clear it). */
+int gs_sync_check(gs_handle *h);
+
+/* ---------------------------------------------------------------------------
+ * Sub-steps exposed for the attention-only sweep and kernel parity tests.
+ * ------------------------------------------------------------------------ */
+
+/* Hybrid-mask attention over a paged bf16 KV cache (paper Appendix steps
+ * Draft forward / Verify forward; mask semantics Sec. 4.2).  Standalone form
+ * of the kernel the rounds use.
+ *   mode 0 DRAFT:  query row i of sequence s sits at slot n_s + i;
+ *                  row 0 sees keys 0..n_s, rows i >= 1 see keys 0..n_s + W - 1
+ *   mode 1 VERIFY: query row i sits at slot n_s + 1 + i and sees keys 0..n_s + 1 + i
+ *   q        device bf16 [n_seq, W, n_heads, 64] (RoPE already applied)
+ *   kv       device bf16 page pool [n_pages][2 (K,V)][n_kv_heads][64 tokens][64]
+ *   page_table device int32 [n_seq, pt_stride]: logical page -> physical page
+ *   n        device int32 [n_seq]: n_s
+ *   out      device bf16 [n_seq, W, n_heads, 64]
+ *   scratch  device, >= gs_attention_scratch_bytes(...) bytes, zeroed before
+ *            its first use; the kernels leave it zeroed again
+ *   split_pages pages per KV split (>= 1)
+ *   stream   cudaStream_t */
+size_t gs_attention_scratch_bytes(int n_seq, int W, int n_heads, int n_kv_heads, int max_pages,
+                                  int split_pages);
+int gs_attention(int mode, const void *q, const void *kv, int n_pages, const int32_t *page_table,
+                 int pt_stride, const int32_t *n, int n_seq, int W, int n_heads, int n_kv_heads,
+                 void *out, void *scratch, size_t scratch_bytes, int split_pages, void *stream);
+
+/* Y = X . W^T on the tcgen05 GEMM the decoder uses.
+ *   x device bf16 [M, K] (row stride K), w device bf16 [N, K], y device [M, N]
+ *   epilogue 0: y bf16 = acc;  1: y fp32 += acc (residual);  2: SwiGLU: w is
+ *   [2N, K] (gate rows then up rows), y bf16 [M, N] = silu(gate) * up;
+ *   3: argmax: y is uint64 [M] packed (ordered fp32 bits << 32 | ~index),
+ *   combined with atomicMax (caller zeroes it first).
+ *   split_k: 1 or a divisor of K/64; scratch device >= gs_linear_scratch_bytes.
+ *   Requirements: K % 64 == 0, N % 128 == 0 (N % 64 for epilogue 2), M >= 1. */
+size_t gs_linear_scratch_bytes(int M, int N, int split_k);
+int gs_linear(const void *x, const void *w, void *y, int M, int N, int K, int epilogue, int split_k,
+              void *scratch, size_t scratch_bytes, void *stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* GS_H_ */

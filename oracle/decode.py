@@ -57,6 +57,7 @@ class SeqState:
     max_new: int            # cap on len(out)
     eos: int = -1
     done: bool = False
+    prefill_gap: float = float("inf")   # top-2 gap of the row that chose the first x0
 
     @property
     def n(self) -> int:
@@ -96,9 +97,27 @@ def prefill(dec: Decoder, vis_bits: np.ndarray, text: np.ndarray, capacity: int,
     logits = dec.forward(x, slots, allowed, cache)
     cache.seq_len = P
     x0 = int(argmax_rows(logits[-1:])[0])
-    st = SeqState(cache=cache, x0=x0, out=[x0], max_new=max_new, eos=eos)
+    st = SeqState(cache=cache, x0=x0, out=[x0], max_new=max_new, eos=eos,
+                  prefill_gap=float(top2_gap(logits[-1:])[0]))
     st.done = (x0 == eos) or (len(st.out) >= max_new)
     return st
+
+
+# ------------------------------------------------------------------ masks
+def draft_allowed(n: int, K: int) -> np.ndarray:
+    """Hybrid draft mask over keys 0..n+K: row 0 (boundary, slot n) sees 0..n;
+    mask rows 1..K see the cache and the whole window, 0..n+K."""
+    keys = np.arange(n + K + 1)
+    allowed = np.empty((K + 1, n + K + 1), dtype=bool)
+    allowed[0] = keys <= n
+    allowed[1:] = True
+    return allowed
+
+
+def verify_allowed(n: int, K: int) -> np.ndarray:
+    """Token-level causal verify mask over keys 0..n+K+1: row i (slot n+1+i) sees 0..n+1+i."""
+    slots = n + 1 + np.arange(K + 1)
+    return np.arange(n + K + 2)[None, :] <= slots[:, None]
 
 
 # ------------------------------------------------------------------ forwards
@@ -113,11 +132,7 @@ def draft_forward(dec: Decoder, cache: KVCache, x0: int, K: int) -> np.ndarray:
     n = cache.seq_len
     ids = np.array([x0] + [dec.cfg.mask_token_id] * K)
     slots = n + np.arange(K + 1)
-    keys = np.arange(n + K + 1)
-    allowed = np.empty((K + 1, n + K + 1), dtype=bool)
-    allowed[0] = keys <= n
-    allowed[1:] = True
-    return dec.forward(dec.embed_tokens(ids), slots, allowed, cache)
+    return dec.forward(dec.embed_tokens(ids), slots, draft_allowed(n, K), cache)
 
 
 def verify_forward(dec: Decoder, cache: KVCache, a0: int, d: np.ndarray) -> np.ndarray:
@@ -130,9 +145,7 @@ def verify_forward(dec: Decoder, cache: KVCache, a0: int, d: np.ndarray) -> np.n
     K = len(d)
     ids = np.concatenate([[a0], np.asarray(d, dtype=np.int64)])
     slots = n + 1 + np.arange(K + 1)
-    keys = np.arange(n + K + 2)
-    allowed = keys[None, :] <= slots[:, None]
-    return dec.forward(dec.embed_tokens(ids), slots, allowed, cache)
+    return dec.forward(dec.embed_tokens(ids), slots, verify_allowed(n, K), cache)
 
 
 def ar_step_forward(dec: Decoder, cache: KVCache, token: int) -> np.ndarray:

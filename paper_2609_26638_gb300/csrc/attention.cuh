@@ -1,0 +1,356 @@
+// attention.cuh -- hybrid-mask attention over the paged bf16 KV cache.
+//
+// One CTA = (query block b, KV head h, KV split c).  A query block is a run of
+// tokens of one sequence (the K+1 window of a decode forward, or 64 tokens of
+// a prefill chunk); its rows are (token, query head of the GQA group), so the
+// two query heads that share a KV head read each K/V page once.  Every query
+// token carries its own inclusive key limit, which encodes the mask: draft
+// boundary row n, draft mask rows n+K, verify row i n+1+i, prefill row p (paper
+// Appendix steps Draft forward / Verify forward).
+//
+// K and V pages (64 tokens x 64 dims, 8 KB each) are staged by TMA with
+// 128-byte swizzle into a ring of shared-memory stages; each warp owns 16 rows
+// and runs S = Q K^T and O += P V on mma.sync m16n8k16 (bf16 in, fp32 out),
+// with the online softmax in registers (exp2 with the 1/sqrt(64) scale folded).
+//
+// Splits cover fixed absolute page ranges [c*SP, (c+1)*SP), so a row's result
+// depends only on its own keys and not on the window it sits in; keys past a
+// row's limit contribute exact zeros.  With more than one split, each CTA
+// writes (O, m, l) partials and the last CTA of (b, h) merges them in split
+// order.
+#pragma once
+#include "ptx.cuh"
+
+namespace gs {
+
+struct AttnArgs {
+  const __nv_bfloat16* q;     // [T, Hq, 64]
+  const int32_t* lim;         // [T] inclusive key limit per query token
+  __nv_bfloat16* out;         // [T, Hq, 64]
+  const int32_t* page_table;  // [slots, pt_stride]
+  int pt_stride;
+  const int32_t* blk_slot;    // [n_blocks] page-table row per block, or null -> fixed_slot
+  const int32_t* blk_active;  // [n_blocks] nonzero = run, or null
+  int fixed_slot;
+  int T, QB;                  // tokens; tokens per query block
+  int Hq, Hkv, G;
+  long long kv_row_base;      // first KV-map row of this layer
+  int rows_per_page;          // 2 * Hkv * 64
+  int split_pages;            // SP
+  int max_splits;
+  int r_max;                  // QB * G rounded up to 16
+  float* part_o;              // [n_blocks][Hkv][max_splits][r_max][64]
+  float* part_ml;             // [n_blocks][Hkv][max_splits][r_max][2]
+  int* counters;              // [n_blocks][Hkv]
+  int* err;
+};
+
+constexpr int kAttnStages = 4;
+constexpr int kAttnPageBytes = 64 * 128;  // 64 tokens x 64 bf16
+
+__host__ __device__ inline int attn_smem_bytes(int r_max) {
+  return 1024 + kAttnStages * 2 * kAttnPageBytes + r_max * 128 + 64 /*barriers*/ + 64;
+}
+
+__device__ __forceinline__ uint32_t sw128(int row, int chunk) {
+  return static_cast<uint32_t>(row * 128 + ((chunk ^ (row & 7)) << 4));
+}
+
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
+                                        uint32_t& r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr));
+}
+
+__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
+                                          uint32_t& r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr));
+}
+
+__device__ __forceinline__ void mma_bf16_16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0,
+                                               uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, "
+      "{%8, %9}, {%0, %1, %2, %3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+  __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&v);
+}
+
+__global__ void __launch_bounds__(512)
+    attn_paged_kernel(const __grid_constant__ CUtensorMap tmKV, const AttnArgs a) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  uint8_t* sK = smem;                                     // [stages][64][128 B]
+  uint8_t* sV = smem + kAttnStages * kAttnPageBytes;      // [stages][64][128 B]
+  uint8_t* sQ = smem + 2 * kAttnStages * kAttnPageBytes;  // [r_max][128 B]
+  uint64_t* full = reinterpret_cast<uint64_t*>(sQ + a.r_max * 128);
+  __shared__ int s_maxlim;
+  __shared__ int s_last;
+
+  const int c = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int nthreads = blockDim.x;
+  if (a.blk_active != nullptr && a.blk_active[b] == 0) return;
+  const int tok0 = b * a.QB;
+  const int ntok = min(a.QB, a.T - tok0);
+  if (ntok <= 0) return;
+  const int R = ntok * a.G;
+  const int slot = a.blk_slot ? a.blk_slot[b] : a.fixed_slot;
+
+  if (warp == 0) {
+    int m = -1;
+    for (int i = lane; i < ntok; i += 32) m = max(m, a.lim[tok0 + i]);
+#pragma unroll
+    for (int o = 16; o >= 1; o >>= 1) m = max(m, __shfl_xor_sync(0xFFFFFFFFu, m, o));
+    if (lane == 0) s_maxlim = m;
+  }
+  __syncthreads();
+  const int maxlim = s_maxlim;
+  const int npages_blk = maxlim / 64 + 1;
+  const int SP = a.split_pages;
+  const int nsplit = (npages_blk + SP - 1) / SP;
+  if (c >= nsplit) return;
+  const int p_begin = c * SP;
+  const int p_end = min(npages_blk, p_begin + SP);
+  const int np = p_end - p_begin;
+  if (maxlim < 0 || npages_blk > a.pt_stride || slot < 0) {
+    if (threadIdx.x == 0) atomicExch(a.err, kErrBounds);
+    return;
+  }
+  const int32_t* pt = a.page_table + static_cast<size_t>(slot) * a.pt_stride;
+
+  if (threadIdx.x == 0) {
+    tma_prefetch_desc(&tmKV);
+    for (int s = 0; s < kAttnStages; ++s) mbar_init(smem_u32(&full[s]), 1);
+    fence_mbar_init();
+  }
+  __syncthreads();
+  const uint64_t pol = l2_policy_evict_first();
+  auto issue = [&](int i) {
+    const int s = i % kAttnStages;
+    int phys = pt[p_begin + i];
+    if (phys < 0) {  // unmapped page: the TMA box lands out of bounds and reads zeros
+      atomicExch(a.err, kErrBounds);
+      phys = 0x3FFFFFFF / a.rows_per_page;
+    }
+    const long long row = a.kv_row_base + static_cast<long long>(phys) * a.rows_per_page;
+    const uint32_t fb = smem_u32(&full[s]);
+    mbar_arrive_expect_tx(fb, 2 * kAttnPageBytes);
+    tma_load_2d(smem_u32(sK + s * kAttnPageBytes), &tmKV, 0, static_cast<int>(row + h * 64), fb, pol);
+    tma_load_2d(smem_u32(sV + s * kAttnPageBytes), &tmKV, 0,
+                static_cast<int>(row + (a.Hkv + h) * 64), fb, pol);
+  };
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < min(np, kAttnStages); ++i) issue(i);
+  }
+
+  // Q rows -> swizzled smem (zero rows past R)
+  const int nrows_pad = (nthreads / 32) * 16;
+  for (int idx = threadIdx.x; idx < nrows_pad * 8; idx += nthreads) {
+    const int r = idx >> 3, ch = idx & 7;
+    uint4 v = make_uint4(0, 0, 0, 0);
+    if (r < R) {
+      const int t = tok0 + r / a.G;
+      const int hq = h * a.G + r % a.G;
+      v = *reinterpret_cast<const uint4*>(a.q + (static_cast<size_t>(t) * a.Hq + hq) * 64 + ch * 8);
+    }
+    *reinterpret_cast<uint4*>(sQ + sw128(r, ch)) = v;
+  }
+  __syncthreads();
+
+  const bool has_rows = warp * 16 < R;
+  const int g = lane >> 2, tq = lane & 3;
+  const int r0 = warp * 16 + g, r1 = r0 + 8;
+  const int lim0 = r0 < R ? a.lim[tok0 + r0 / a.G] : -1;
+  const int lim1 = r1 < R ? a.lim[tok0 + r1 / a.G] : -1;
+
+  uint32_t qa[4][4];
+  if (has_rows) {
+#pragma unroll
+    for (int kk = 0; kk < 4; ++kk) {
+      const int row = warp * 16 + (lane & 15);
+      const int ch = 2 * kk + (lane >> 4);
+      ldsm_x4(smem_u32(sQ) + sw128(row, ch), qa[kk][0], qa[kk][1], qa[kk][2], qa[kk][3]);
+    }
+  }
+
+  const float kScaleLog2 = 0.125f * 1.4426950408889634f;
+  float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f;
+  float o[8][4];
+#pragma unroll
+  for (int j = 0; j < 8; ++j) o[j][0] = o[j][1] = o[j][2] = o[j][3] = 0.f;
+  bool ok = true;
+
+  for (int i = 0; i < np; ++i) {
+    const int s = i % kAttnStages;
+    if (ok && !mbar_wait(smem_u32(&full[s]), (i / kAttnStages) & 1, a.err)) ok = false;
+    if (ok && has_rows) {
+      const uint32_t kbase = smem_u32(sK + s * kAttnPageBytes);
+      const uint32_t vbase = smem_u32(sV + s * kAttnPageBytes);
+      float sacc[8][4];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) sacc[j][0] = sacc[j][1] = sacc[j][2] = sacc[j][3] = 0.f;
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+#pragma unroll
+        for (int kk = 0; kk < 4; kk += 2) {
+          uint32_t b0, b1, b2, b3;
+          const int row = 8 * j + (lane & 7);
+          const int ch = 2 * kk + (lane >> 3);
+          ldsm_x4(kbase + sw128(row, ch), b0, b1, b2, b3);
+          mma_bf16_16816(sacc[j], qa[kk], b0, b1);
+          mma_bf16_16816(sacc[j], qa[kk + 1], b2, b3);
+        }
+      }
+      // mask + online softmax (rows r0: elements 0,1; r1: elements 2,3)
+      const int kbase_abs = (p_begin + i) * 64;
+      float mx0 = -INFINITY, mx1 = -INFINITY;
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const int key = kbase_abs + 8 * j + 2 * tq;
+        sacc[j][0] = key <= lim0 ? sacc[j][0] * kScaleLog2 : -INFINITY;
+        sacc[j][1] = key + 1 <= lim0 ? sacc[j][1] * kScaleLog2 : -INFINITY;
+        sacc[j][2] = key <= lim1 ? sacc[j][2] * kScaleLog2 : -INFINITY;
+        sacc[j][3] = key + 1 <= lim1 ? sacc[j][3] * kScaleLog2 : -INFINITY;
+        mx0 = fmaxf(mx0, fmaxf(sacc[j][0], sacc[j][1]));
+        mx1 = fmaxf(mx1, fmaxf(sacc[j][2], sacc[j][3]));
+      }
+      mx0 = fmaxf(mx0, __shfl_xor_sync(0xFFFFFFFFu, mx0, 1));
+      mx0 = fmaxf(mx0, __shfl_xor_sync(0xFFFFFFFFu, mx0, 2));
+      mx1 = fmaxf(mx1, __shfl_xor_sync(0xFFFFFFFFu, mx1, 1));
+      mx1 = fmaxf(mx1, __shfl_xor_sync(0xFFFFFFFFu, mx1, 2));
+      const float mn0 = fmaxf(m0, mx0), mn1 = fmaxf(m1, mx1);
+      const float al0 = (mn0 == -INFINITY) ? 1.f : exp2f(m0 - mn0);
+      const float al1 = (mn1 == -INFINITY) ? 1.f : exp2f(m1 - mn1);
+      const float sub0 = (mn0 == -INFINITY) ? 0.f : mn0;
+      const float sub1 = (mn1 == -INFINITY) ? 0.f : mn1;
+      m0 = mn0;
+      m1 = mn1;
+      float ps0 = 0.f, ps1 = 0.f;
+      uint32_t pa[4][4];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const float p0 = exp2f(sacc[j][0] - sub0), p1 = exp2f(sacc[j][1] - sub0);
+        const float p2 = exp2f(sacc[j][2] - sub1), p3 = exp2f(sacc[j][3] - sub1);
+        ps0 += p0 + p1;
+        ps1 += p2 + p3;
+        pa[j >> 1][(j & 1) * 2 + 0] = pack_bf16x2(p0, p1);
+        pa[j >> 1][(j & 1) * 2 + 1] = pack_bf16x2(p2, p3);
+      }
+      l0 = l0 * al0 + ps0;
+      l1 = l1 * al1 + ps1;
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        o[j][0] *= al0;
+        o[j][1] *= al0;
+        o[j][2] *= al1;
+        o[j][3] *= al1;
+      }
+      // O += P V ; V stored [key][dim] -> transposed ldmatrix
+#pragma unroll
+      for (int kk = 0; kk < 4; ++kk) {
+#pragma unroll
+        for (int jn = 0; jn < 8; jn += 2) {
+          uint32_t b0, b1, b2, b3;
+          const int row = 16 * kk + (lane & 7) + ((lane >> 3) & 1) * 8;
+          const int ch = jn + (lane >> 4);
+          ldsm_x4_t(vbase + sw128(row, ch), b0, b1, b2, b3);
+          mma_bf16_16816(o[jn], pa[kk], b0, b1);
+          mma_bf16_16816(o[jn + 1], pa[kk], b2, b3);
+        }
+      }
+    }
+    __syncthreads();
+    if (threadIdx.x == 0 && ok && i + kAttnStages < np) issue(i + kAttnStages);
+  }
+  if (!__syncthreads_and(ok)) return;
+
+  // row sums across the quad
+  l0 += __shfl_xor_sync(0xFFFFFFFFu, l0, 1);
+  l0 += __shfl_xor_sync(0xFFFFFFFFu, l0, 2);
+  l1 += __shfl_xor_sync(0xFFFFFFFFu, l1, 1);
+  l1 += __shfl_xor_sync(0xFFFFFFFFu, l1, 2);
+
+  if (nsplit == 1) {
+    if (has_rows) {
+#pragma unroll
+      for (int half = 0; half < 2; ++half) {
+        const int r = half ? r1 : r0;
+        if (r >= R) continue;
+        const float inv = 1.0f / (half ? l1 : l0);
+        const int t = tok0 + r / a.G;
+        const int hq = h * a.G + r % a.G;
+        __nv_bfloat16* dst = a.out + (static_cast<size_t>(t) * a.Hq + hq) * 64;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          const float x0 = o[j][half * 2 + 0] * inv, x1 = o[j][half * 2 + 1] * inv;
+          *reinterpret_cast<__nv_bfloat162*>(dst + 8 * j + 2 * tq) = __floats2bfloat162_rn(x0, x1);
+        }
+      }
+    }
+    return;
+  }
+
+  // split partials
+  const size_t bh = static_cast<size_t>(b) * a.Hkv + h;
+  float* po = a.part_o + ((bh * a.max_splits + c) * a.r_max) * 64;
+  float* pml = a.part_ml + ((bh * a.max_splits + c) * a.r_max) * 2;
+  if (has_rows) {
+#pragma unroll
+    for (int half = 0; half < 2; ++half) {
+      const int r = half ? r1 : r0;
+      if (r >= R) continue;
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        *reinterpret_cast<float2*>(po + r * 64 + 8 * j + 2 * tq) =
+            make_float2(o[j][half * 2 + 0], o[j][half * 2 + 1]);
+      }
+      if (tq == 0) {
+        pml[r * 2 + 0] = half ? m1 : m0;
+        pml[r * 2 + 1] = half ? l1 : l0;
+      }
+    }
+  }
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    const int old = atomicAdd(a.counters + bh, 1);
+    s_last = (old == nsplit - 1);
+    if (s_last) a.counters[bh] = 0;
+  }
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+  const float* po0 = a.part_o + (bh * a.max_splits * a.r_max) * 64;
+  const float* pml0 = a.part_ml + (bh * a.max_splits * a.r_max) * 2;
+  for (int idx = threadIdx.x; idx < R * 32; idx += nthreads) {
+    const int r = idx >> 5, d2 = (idx & 31) * 2;
+    float M = -INFINITY;
+    for (int s = 0; s < nsplit; ++s) M = fmaxf(M, __ldcg(pml0 + (s * a.r_max + r) * 2));
+    float ox = 0.f, oy = 0.f, L = 0.f;
+    for (int s = 0; s < nsplit; ++s) {
+      const float ms = __ldcg(pml0 + (s * a.r_max + r) * 2);
+      const float w = (ms == -INFINITY) ? 0.f : exp2f(ms - M);
+      L += w * __ldcg(pml0 + (s * a.r_max + r) * 2 + 1);
+      const float2 v = __ldcg(reinterpret_cast<const float2*>(po0 + (s * a.r_max + r) * 64 + d2));
+      ox += w * v.x;
+      oy += w * v.y;
+    }
+    const float inv = 1.0f / L;
+    const int t = tok0 + r / a.G;
+    const int hq = h * a.G + r % a.G;
+    *reinterpret_cast<__nv_bfloat162*>(a.out + (static_cast<size_t>(t) * a.Hq + hq) * 64 + d2) =
+        __floats2bfloat162_rn(ox * inv, oy * inv);
+  }
+}
+
+}  // namespace gs

@@ -1,0 +1,913 @@
+// engine.cu -- libgs host side: workspace carving, paged-KV bookkeeping, the
+// decoder forward as a launch sequence, the round (draft -> force -> verify ->
+// accept) with a CUDA-graph cache, prefill, and the C ABI of include/gs.h.
+#include <algorithm>
+#include <cstdio>
+#include <cstring>
+#include <map>
+#include <string>
+#include <tuple>
+#include <vector>
+
+#include "attention.cuh"
+#include "gemm_tc.cuh"
+#include "internal.h"
+#include "small.cuh"
+#include "../../include/gs.h"
+
+using namespace gs;
+
+namespace {
+
+thread_local std::string g_create_error;
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn get_encode() {
+  static EncodeTiledFn fn = nullptr;
+  if (!fn) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  }
+  return fn;
+}
+
+// 2-D bf16 tensor map over a row-major [rows, cols] array, box {64, box_rows},
+// 128-byte swizzle, zero fill out of bounds.
+bool make_map(CUtensorMap* m, const void* base, uint64_t rows, uint64_t cols, uint32_t box_rows) {
+  EncodeTiledFn enc = get_encode();
+  if (!enc) return false;
+  cuuint64_t dims[2] = {cols, rows};
+  cuuint64_t strides[1] = {cols * 2};
+  cuuint32_t box[2] = {64, box_rows};
+  cuuint32_t es[2] = {1, 1};
+  CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides,
+                   box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+inline int cdiv(long long a, long long b) { return static_cast<int>((a + b - 1) / b); }
+inline int round16(int x) { return (x + 15) / 16 * 16; }
+
+// Sequential carving of the caller's workspace (also used to size it).
+struct Carver {
+  uint8_t* base;
+  size_t off = 0;
+  explicit Carver(void* b) : base(static_cast<uint8_t*>(b)) {}
+  template <class T>
+  T* take(size_t count) {
+    off = align_up(off, 256);
+    T* p = base ? reinterpret_cast<T*>(base + off) : nullptr;
+    off += count * sizeof(T);
+    return p;
+  }
+};
+
+struct GemmPlan {
+  int bn, tok_tiles, feat_tiles, splits;
+};
+
+// Token tile from T; split-K (decode only) so that about one wave of CTAs runs.
+GemmPlan plan_gemm(int weight_rows, int K, int T, bool allow_split) {
+  GemmPlan p;
+  p.bn = gemm_bn_for(T);
+  p.tok_tiles = cdiv(T, p.bn);
+  p.feat_tiles = weight_rows / 128;
+  p.splits = 1;
+  const int tiles = p.feat_tiles * p.tok_tiles;
+  const int nkb = K / 64;
+  if (allow_split && tiles < 152) {
+    const int want = cdiv(152, tiles);
+    for (int s = 1; s <= nkb; ++s)
+      if (nkb % s == 0 && s <= want) p.splits = s;
+  }
+  return p;
+}
+
+constexpr size_t kGemmPartialFloats = 12u << 20;  // 48 MB of split-K partials
+constexpr int kGemmCounters = 1 << 16;
+
+}  // namespace
+
+struct gs_handle {
+  gs_config cfg;
+  cudaStream_t stream = nullptr;
+  std::string err;
+
+  // weights
+  const __nv_bfloat16 *embed = nullptr, *lm_head = nullptr, *final_norm = nullptr;
+  std::vector<const __nv_bfloat16*> attn_norm, ffn_norm, w_qkv, w_o, w_gu, w_down;
+  std::vector<CUtensorMap> tm_qkv, tm_o, tm_gu, tm_down;
+  CUtensorMap tm_lm;
+  CUtensorMap tm_xn[4], tm_ao[4], tm_act[4];
+  CUtensorMap tm_kv;
+
+  // sizes
+  int qkv_dim = 0, G = 1, T_max = 0, pt_stride = 0, n_pages = 0, split_pages = 1;
+  int max_splits_dec = 1, r_max_dec = 16, W_max = 1;
+
+  // workspace
+  int* err_word = nullptr;
+  SeqStateDev st{};
+  int32_t* page_table = nullptr;
+  __nv_bfloat16* kv = nullptr;
+  float2* rope = nullptr;
+  int32_t *tok = nullptr, *pos = nullptr, *lim = nullptr, *tok_slot = nullptr;
+  int32_t *blk_slot = nullptr, *blk_active = nullptr;
+  float* hbuf = nullptr;
+  __nv_bfloat16 *xn = nullptr, *qkv = nullptr, *qr = nullptr, *ao = nullptr, *act = nullptr;
+  unsigned long long *packed_d = nullptr, *packed_v = nullptr;
+  int32_t *draft_tok = nullptr, *verify_in = nullptr, *verify_tok = nullptr;
+  float* gemm_partial = nullptr;
+  int* gemm_counters = nullptr;
+  float *attn_po = nullptr, *attn_pml = nullptr;
+  int* attn_counters = nullptr;
+
+  // host page bookkeeping
+  std::vector<int> free_pages;
+  std::vector<std::vector<int>> slot_pages;
+  std::vector<int> slot_reserved;  // slots (tokens) reserved per sequence slot
+  std::vector<int32_t> pt_host;
+
+  // graphs keyed by (n_seq, K, pointers)
+  typedef std::tuple<int, int, const void*, const void*, long long, const void*, long long,
+                     const void*, const void*, const void*>
+      GraphKey;
+  std::map<GraphKey, cudaGraphExec_t> graphs;
+};
+
+namespace {
+
+int fail(gs_handle* h, int code, const std::string& msg) {
+  if (h) h->err = msg;
+  else g_create_error = msg;
+  return code;
+}
+
+#define GS_CUDA(h, call)                                                              \
+  do {                                                                                \
+    cudaError_t e_ = (call);                                                          \
+    if (e_ != cudaSuccess)                                                            \
+      return fail(h, GS_ERR_CUDA, std::string(#call " -> ") + cudaGetErrorString(e_)); \
+  } while (0)
+
+int bn_index(int bn) { return bn == 32 ? 0 : (bn == 64 ? 1 : (bn == 128 ? 2 : 3)); }
+
+bool config_ok(const gs_config* c, std::string* why) {
+  auto bad = [&](const char* m) { *why = m; return false; };
+  if (!c) return bad("null config");
+  if (c->n_layers < 1 || c->d_model < 128 || c->vocab < 128) return bad("bad sizes");
+  if (c->head_dim != 64) return bad("head_dim must be 64");
+  if (c->n_heads < 1 || c->n_kv_heads < 1 || c->n_heads % c->n_kv_heads) return bad("bad heads");
+  if (c->n_heads / c->n_kv_heads > 8) return bad("GQA group > 8 unsupported");
+  if (c->d_model % 128) return bad("d_model % 128");
+  if (((c->n_heads + 2 * c->n_kv_heads) * 64) % 128) return bad("qkv rows % 128");
+  if ((c->n_heads * 64) % 64) return bad("attn dim % 64");
+  if (c->d_ffn % 64 || c->d_ffn < 64) return bad("d_ffn % 64");
+  if (c->vocab % 128) return bad("vocab % 128");
+  if (c->mask_token_id < 0 || c->mask_token_id >= c->vocab) return bad("mask_token_id");
+  if (c->eos_token_id >= c->vocab) return bad("eos_token_id");
+  if (c->max_batch < 1 || c->max_ctx < 64 || c->max_K < 0 || c->max_prefill < 1)
+    return bad("bad capacity");
+  if ((c->max_K + 1) * (c->n_heads / c->n_kv_heads) > 256) return bad("window rows > 256");
+  if (c->max_batch * (c->max_K + 1) > 65536) return bad("decode tokens > 65536");
+  return true;
+}
+
+// Carve the workspace; with base == nullptr only sizes it.
+size_t carve(gs_handle* h, const gs_config& c, void* base) {
+  Carver cv(base);
+  const int G = c.n_heads / c.n_kv_heads;
+  const int qkv_dim = (c.n_heads + 2 * c.n_kv_heads) * 64;
+  const int pt_stride = cdiv(c.max_ctx, 64);
+  const int n_pages = c.kv_pages > 0 ? c.kv_pages : c.max_batch * pt_stride;
+  const int W_max = c.max_K + 1;
+  int T_max = std::max(c.max_batch * W_max, c.max_prefill);
+  T_max = static_cast<int>(align_up(std::max(T_max, 256), 256));
+  int sp = c.split_pages;
+  if (sp <= 0) sp = std::max(1, cdiv(static_cast<long long>(pt_stride) * c.max_batch * c.n_kv_heads, 304));
+  const int max_splits = cdiv(pt_stride, sp);
+  const int r_max = round16(W_max * G);
+
+  int* err_word = cv.take<int>(64);
+  SeqStateDev st;
+  st.seq_len = cv.take<int32_t>(c.max_batch);
+  st.x0 = cv.take<int32_t>(c.max_batch);
+  st.n_out = cv.take<int32_t>(c.max_batch);
+  st.max_new = cv.take<int32_t>(c.max_batch);
+  st.done = cv.take<int32_t>(c.max_batch);
+  st.rounds = cv.take<int32_t>(c.max_batch);
+  int32_t* page_table = cv.take<int32_t>(static_cast<size_t>(c.max_batch) * pt_stride);
+  __nv_bfloat16* kv = cv.take<__nv_bfloat16>(static_cast<size_t>(c.n_layers) * n_pages * 2 *
+                                             c.n_kv_heads * 64 * 64);
+  float2* rope = cv.take<float2>(static_cast<size_t>(c.max_ctx) * 32);
+  int32_t* tok = cv.take<int32_t>(T_max);
+  int32_t* pos = cv.take<int32_t>(T_max);
+  int32_t* lim = cv.take<int32_t>(T_max);
+  int32_t* tok_slot = cv.take<int32_t>(T_max);
+  int32_t* blk_slot = cv.take<int32_t>(std::max(c.max_batch, T_max / 64 + 1));
+  int32_t* blk_active = cv.take<int32_t>(std::max(c.max_batch, T_max / 64 + 1));
+  float* hbuf = cv.take<float>(static_cast<size_t>(T_max) * c.d_model);
+  __nv_bfloat16* xn = cv.take<__nv_bfloat16>(static_cast<size_t>(T_max) * c.d_model);
+  __nv_bfloat16* qkv = cv.take<__nv_bfloat16>(static_cast<size_t>(T_max) * qkv_dim);
+  __nv_bfloat16* qr = cv.take<__nv_bfloat16>(static_cast<size_t>(T_max) * c.n_heads * 64);
+  __nv_bfloat16* ao = cv.take<__nv_bfloat16>(static_cast<size_t>(T_max) * c.n_heads * 64);
+  __nv_bfloat16* act = cv.take<__nv_bfloat16>(static_cast<size_t>(T_max) * c.d_ffn);
+  unsigned long long* packed_d = cv.take<unsigned long long>(T_max);
+  unsigned long long* packed_v = cv.take<unsigned long long>(T_max);
+  int32_t* draft_tok = cv.take<int32_t>(static_cast<size_t>(c.max_batch) * W_max);
+  int32_t* verify_in = cv.take<int32_t>(static_cast<size_t>(c.max_batch) * W_max);
+  int32_t* verify_tok = cv.take<int32_t>(static_cast<size_t>(c.max_batch) * W_max);
+  float* gemm_partial = cv.take<float>(kGemmPartialFloats);
+  int* gemm_counters = cv.take<int>(kGemmCounters);
+  const size_t bh = static_cast<size_t>(c.max_batch) * c.n_kv_heads;
+  float* attn_po = cv.take<float>(bh * max_splits * r_max * 64);
+  float* attn_pml = cv.take<float>(bh * max_splits * r_max * 2);
+  int* attn_counters = cv.take<int>(bh);
+
+  if (h) {
+    h->G = G;
+    h->qkv_dim = qkv_dim;
+    h->pt_stride = pt_stride;
+    h->n_pages = n_pages;
+    h->T_max = T_max;
+    h->W_max = W_max;
+    h->split_pages = sp;
+    h->max_splits_dec = max_splits;
+    h->r_max_dec = r_max;
+    h->err_word = err_word;
+    h->st = st;
+    h->page_table = page_table;
+    h->kv = kv;
+    h->rope = rope;
+    h->tok = tok;
+    h->pos = pos;
+    h->lim = lim;
+    h->tok_slot = tok_slot;
+    h->blk_slot = blk_slot;
+    h->blk_active = blk_active;
+    h->hbuf = hbuf;
+    h->xn = xn;
+    h->qkv = qkv;
+    h->qr = qr;
+    h->ao = ao;
+    h->act = act;
+    h->packed_d = packed_d;
+    h->packed_v = packed_v;
+    h->draft_tok = draft_tok;
+    h->verify_in = verify_in;
+    h->verify_tok = verify_tok;
+    h->gemm_partial = gemm_partial;
+    h->gemm_counters = gemm_counters;
+    h->attn_po = attn_po;
+    h->attn_pml = attn_pml;
+    h->attn_counters = attn_counters;
+  }
+  return align_up(cv.off, 256);
+}
+
+// ------------------------------------------------------------------ launches
+int run_gemm(gs_handle* h, const CUtensorMap& tw, int weight_rows, const CUtensorMap* tx_set, int K,
+             int T, int epi, void* y, int ldy, int N, float* logits, bool decode) {
+  const GemmPlan p = plan_gemm(weight_rows, K, T, decode);
+  GemmArgs a;
+  a.M = T;
+  a.N = N;
+  a.K = K;
+  a.splits = p.splits;
+  a.kb_per_split = (K / 64) / p.splits;
+  a.y = y;
+  a.ldy = ldy;
+  a.partial = h->gemm_partial;
+  a.counters = h->gemm_counters;
+  a.logits = logits;
+  a.err = h->err_word;
+  if (p.splits > 1) {
+    const size_t need = static_cast<size_t>(p.splits) * p.feat_tiles * p.tok_tiles * p.bn * 128;
+    if (need > kGemmPartialFloats || p.feat_tiles * p.tok_tiles > kGemmCounters)
+      return fail(h, GS_ERR_OOM, "split-K scratch too small");
+  }
+  GS_CUDA(h, launch_gemm(p.bn, epi, tw, tx_set[bn_index(p.bn)], a, p.feat_tiles, p.tok_tiles,
+                         h->stream));
+  return GS_OK;
+}
+
+int run_rmsnorm(gs_handle* h, const float* x, const __nv_bfloat16* g, __nv_bfloat16* y, int T,
+                unsigned long long* reset) {
+  const int rows_per_block = 4;
+  rmsnorm_kernel<<<cdiv(T, rows_per_block), 32 * rows_per_block, 0, h->stream>>>(
+      x, g, y, T, h->cfg.d_model, h->cfg.rms_eps, reset);
+  GS_CUDA(h, cudaGetLastError());
+  return GS_OK;
+}
+
+struct AttnLaunch {
+  int n_blocks, QB, max_splits, split_pages, r_max;
+  const int32_t* blk_slot;
+  const int32_t* blk_active;
+  int fixed_slot;
+};
+
+int run_attention(gs_handle* h, int layer, int T, const AttnLaunch& L) {
+  const gs_config& c = h->cfg;
+  AttnArgs a;
+  a.q = h->qr;
+  a.lim = h->lim;
+  a.out = h->ao;
+  a.page_table = h->page_table;
+  a.pt_stride = h->pt_stride;
+  a.blk_slot = L.blk_slot;
+  a.blk_active = L.blk_active;
+  a.fixed_slot = L.fixed_slot;
+  a.T = T;
+  a.QB = L.QB;
+  a.Hq = c.n_heads;
+  a.Hkv = c.n_kv_heads;
+  a.G = h->G;
+  a.rows_per_page = 2 * c.n_kv_heads * 64;
+  a.kv_row_base = static_cast<long long>(layer) * h->n_pages * a.rows_per_page;
+  a.split_pages = L.split_pages;
+  a.max_splits = L.max_splits;
+  a.r_max = L.r_max;
+  a.part_o = h->attn_po;
+  a.part_ml = h->attn_pml;
+  a.counters = h->attn_counters;
+  a.err = h->err_word;
+  dim3 grid(L.max_splits, c.n_kv_heads, L.n_blocks);
+  const int threads = (L.r_max / 16) * 32;
+  attn_paged_kernel<<<grid, threads, attn_smem_bytes(L.r_max), h->stream>>>(h->tm_kv, a);
+  GS_CUDA(h, cudaGetLastError());
+  return GS_OK;
+}
+
+// One decoder forward over T rows already described by tok/pos/lim/tok_slot.
+// Visual rows (prefill) come first when n_vis > 0.  The LM head runs on rows
+// [lm_row0, lm_row0 + n_lm) and leaves argmax keys in `packed`.
+int forward(gs_handle* h, int T, const int32_t* tok, const __nv_bfloat16* vis, int n_vis,
+            const AttnLaunch& AL, int lm_row0, int n_lm, unsigned long long* packed,
+            float* logits, bool decode) {
+  const gs_config& c = h->cfg;
+  const int d = c.d_model, F = c.d_ffn, HD = c.n_heads * 64;
+  embed_kernel<<<T, 128, 0, h->stream>>>(tok, h->embed, vis, n_vis, T, d, c.vocab, h->hbuf,
+                                         h->err_word);
+  GS_CUDA(h, cudaGetLastError());
+  const size_t layer_kv = static_cast<size_t>(h->n_pages) * 2 * c.n_kv_heads * 64 * 64;
+  int rc;
+  for (int l = 0; l < c.n_layers; ++l) {
+    if ((rc = run_rmsnorm(h, h->hbuf, h->attn_norm[l], h->xn, T, nullptr))) return rc;
+    if ((rc = run_gemm(h, h->tm_qkv[l], h->qkv_dim, h->tm_xn, d, T, kEpiStoreBf16, h->qkv,
+                       h->qkv_dim, h->qkv_dim, nullptr, decode)))
+      return rc;
+    RopeKvArgs r;
+    r.qkv = h->qkv;
+    r.pos = h->pos;
+    r.tok_slot = h->tok_slot;
+    r.rope = h->rope;
+    r.q_out = h->qr;
+    r.kv = h->kv + l * layer_kv;
+    r.page_table = h->page_table;
+    r.pt_stride = h->pt_stride;
+    r.n_pages = h->n_pages;
+    r.T = T;
+    r.Hq = c.n_heads;
+    r.Hkv = c.n_kv_heads;
+    r.max_ctx = c.max_ctx;
+    r.err = h->err_word;
+    const int warps = T * (c.n_heads + 2 * c.n_kv_heads);
+    rope_kv_kernel<<<cdiv(warps, 8), 256, 0, h->stream>>>(r);
+    GS_CUDA(h, cudaGetLastError());
+    if ((rc = run_attention(h, l, T, AL))) return rc;
+    if ((rc = run_gemm(h, h->tm_o[l], d, h->tm_ao, HD, T, kEpiResidF32, h->hbuf, d, d, nullptr,
+                       decode)))
+      return rc;
+    if ((rc = run_rmsnorm(h, h->hbuf, h->ffn_norm[l], h->xn, T, nullptr))) return rc;
+    if ((rc = run_gemm(h, h->tm_gu[l], 2 * F, h->tm_xn, d, T, kEpiSwiGLU, h->act, F, F, nullptr,
+                       decode)))
+      return rc;
+    if ((rc = run_gemm(h, h->tm_down[l], d, h->tm_act, F, T, kEpiResidF32, h->hbuf, d, d, nullptr,
+                       decode)))
+      return rc;
+  }
+  if ((rc = run_rmsnorm(h, h->hbuf + static_cast<size_t>(lm_row0) * d, h->final_norm, h->xn, n_lm,
+                        packed)))
+    return rc;
+  return run_gemm(h, h->tm_lm, c.vocab, h->tm_xn, d, n_lm, kEpiArgmax, packed, 0, c.vocab, logits,
+                  decode);
+}
+
+int enqueue_round(gs_handle* h, const int32_t* slots, int n_seq, int K, const gs_force* force,
+                  int32_t* out_tok, int32_t* out_cnt, int32_t* out_done, const gs_debug* dbg) {
+  const gs_config& c = h->cfg;
+  const int W = K + 1, T = n_seq * W;
+  WindowArgs w;
+  memset(&w, 0, sizeof(w));
+  w.slots = slots;
+  w.n_seq = n_seq;
+  w.K = K;
+  w.W = W;
+  w.mask_id = c.mask_token_id;
+  w.vocab = c.vocab;
+  w.st = h->st;
+  w.tok = h->tok;
+  w.pos = h->pos;
+  w.lim = h->lim;
+  w.tok_slot = h->tok_slot;
+  w.blk_slot = h->blk_slot;
+  w.blk_active = h->blk_active;
+  w.draft_packed = h->packed_d;
+  w.draft_tok = h->draft_tok;
+  w.verify_in = h->verify_in;
+  if (force) {
+    w.teacher = force->teacher;
+    w.teacher_stride = force->teacher_stride;
+    w.L_sched = force->L_sched;
+    w.L_stride = force->L_stride;
+  }
+  w.err = h->err_word;
+  const int nb = cdiv(T, 128);
+  AttnLaunch AL;
+  AL.n_blocks = n_seq;
+  AL.QB = W;
+  AL.max_splits = h->max_splits_dec;
+  AL.split_pages = h->split_pages;
+  AL.r_max = round16(W * h->G);
+  AL.blk_slot = h->blk_slot;
+  AL.blk_active = h->blk_active;
+  AL.fixed_slot = -1;
+
+  window_draft_kernel<<<nb, 128, 0, h->stream>>>(w);
+  GS_CUDA(h, cudaGetLastError());
+  int rc = forward(h, T, h->tok, nullptr, 0, AL, 0, T, h->packed_d,
+                   dbg ? dbg->draft_logits : nullptr, true);
+  if (rc) return rc;
+  window_verify_kernel<<<nb, 128, 0, h->stream>>>(w);
+  GS_CUDA(h, cudaGetLastError());
+  rc = forward(h, T, h->tok, nullptr, 0, AL, 0, T, h->packed_v, dbg ? dbg->verify_logits : nullptr,
+               true);
+  if (rc) return rc;
+  AcceptArgs ac;
+  ac.slots = slots;
+  ac.n_seq = n_seq;
+  ac.K = K;
+  ac.W = W;
+  ac.eos = c.eos_token_id;
+  ac.st = h->st;
+  ac.verify_in = h->verify_in;
+  ac.verify_packed = h->packed_v;
+  ac.verify_tok = h->verify_tok;
+  ac.out_tok = out_tok;
+  ac.out_cnt = out_cnt;
+  ac.out_done = out_done;
+  accept_commit_kernel<<<cdiv(n_seq, 64), 64, 0, h->stream>>>(ac);
+  GS_CUDA(h, cudaGetLastError());
+  if (dbg) {
+    if (dbg->draft_tok) copy_i32_kernel<<<nb, 128, 0, h->stream>>>(h->draft_tok, dbg->draft_tok, T);
+    if (dbg->verify_in) copy_i32_kernel<<<nb, 128, 0, h->stream>>>(h->verify_in, dbg->verify_in, T);
+    if (dbg->verify_tok)
+      copy_i32_kernel<<<nb, 128, 0, h->stream>>>(h->verify_tok, dbg->verify_tok, T);
+    GS_CUDA(h, cudaGetLastError());
+  }
+  return GS_OK;
+}
+
+}  // namespace
+
+// =================================================================== C ABI
+extern "C" {
+
+size_t gs_workspace_bytes(const gs_config* cfg) {
+  std::string why;
+  if (!config_ok(cfg, &why)) return 0;
+  return carve(nullptr, *cfg, nullptr);
+}
+
+int gs_create(const gs_config* cfg, const gs_weights* w, void* workspace, size_t ws_bytes,
+              void* stream, gs_handle** out) {
+  if (!out) return fail(nullptr, GS_ERR_INVALID_ARG, "out is null");
+  *out = nullptr;
+  std::string why;
+  if (!config_ok(cfg, &why)) return fail(nullptr, GS_ERR_INVALID_ARG, "config: " + why);
+  if (!w || !w->embed || !w->lm_head || !w->final_norm || !w->attn_norm || !w->w_qkv || !w->w_o ||
+      !w->ffn_norm || !w->w_gate_up || !w->w_down)
+    return fail(nullptr, GS_ERR_INVALID_ARG, "null weight pointer");
+  if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 255))
+    return fail(nullptr, GS_ERR_INVALID_ARG, "workspace null or not 256-byte aligned");
+  const size_t need = carve(nullptr, *cfg, nullptr);
+  if (ws_bytes < need)
+    return fail(nullptr, GS_ERR_OOM, "workspace too small: need " + std::to_string(need));
+  if (!get_encode()) return fail(nullptr, GS_ERR_CUDA, "cuTensorMapEncodeTiled unavailable");
+  static bool attrs_done = false;
+  if (!attrs_done) {
+    cudaError_t e = gemm_init_attributes();
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(attn_paged_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               attn_smem_bytes(256));
+    if (e != cudaSuccess)
+      return fail(nullptr, GS_ERR_CUDA, std::string("kernel attributes: ") + cudaGetErrorString(e));
+    attrs_done = true;
+  }
+
+  gs_handle* h = new gs_handle();
+  h->cfg = *cfg;
+  h->stream = static_cast<cudaStream_t>(stream);
+  carve(h, *cfg, workspace);
+  const gs_config& c = h->cfg;
+  const int L = c.n_layers, d = c.d_model, F = c.d_ffn;
+  auto chk = [&](const void* p) { return p && (reinterpret_cast<uintptr_t>(p) & 15) == 0; };
+  h->embed = static_cast<const __nv_bfloat16*>(w->embed);
+  h->lm_head = static_cast<const __nv_bfloat16*>(w->lm_head);
+  h->final_norm = static_cast<const __nv_bfloat16*>(w->final_norm);
+  bool ok = chk(w->embed) && chk(w->lm_head) && chk(w->final_norm);
+  h->tm_qkv.resize(L);
+  h->tm_o.resize(L);
+  h->tm_gu.resize(L);
+  h->tm_down.resize(L);
+  for (int l = 0; l < L && ok; ++l) {
+    h->attn_norm.push_back(static_cast<const __nv_bfloat16*>(w->attn_norm[l]));
+    h->ffn_norm.push_back(static_cast<const __nv_bfloat16*>(w->ffn_norm[l]));
+    h->w_qkv.push_back(static_cast<const __nv_bfloat16*>(w->w_qkv[l]));
+    h->w_o.push_back(static_cast<const __nv_bfloat16*>(w->w_o[l]));
+    h->w_gu.push_back(static_cast<const __nv_bfloat16*>(w->w_gate_up[l]));
+    h->w_down.push_back(static_cast<const __nv_bfloat16*>(w->w_down[l]));
+    ok = chk(w->attn_norm[l]) && chk(w->ffn_norm[l]) && chk(w->w_qkv[l]) && chk(w->w_o[l]) &&
+         chk(w->w_gate_up[l]) && chk(w->w_down[l]);
+    ok = ok && make_map(&h->tm_qkv[l], w->w_qkv[l], h->qkv_dim, d, 128) &&
+         make_map(&h->tm_o[l], w->w_o[l], d, c.n_heads * 64, 128) &&
+         make_map(&h->tm_gu[l], w->w_gate_up[l], 2 * F, d, 64) &&
+         make_map(&h->tm_down[l], w->w_down[l], d, F, 128);
+  }
+  ok = ok && make_map(&h->tm_lm, w->lm_head, c.vocab, d, 128);
+  const int bns[4] = {32, 64, 128, 256};
+  for (int i = 0; i < 4 && ok; ++i) {
+    ok = make_map(&h->tm_xn[i], h->xn, h->T_max, d, bns[i]) &&
+         make_map(&h->tm_ao[i], h->ao, h->T_max, c.n_heads * 64, bns[i]) &&
+         make_map(&h->tm_act[i], h->act, h->T_max, F, bns[i]);
+  }
+  const uint64_t kv_rows = static_cast<uint64_t>(L) * h->n_pages * 2 * c.n_kv_heads * 64;
+  ok = ok && kv_rows < (1ull << 31) && make_map(&h->tm_kv, h->kv, kv_rows, 64, 64);
+  if (!ok) {
+    delete h;
+    return fail(nullptr, GS_ERR_INVALID_ARG, "misaligned weight pointer or tensor-map encode failed");
+  }
+  // zero the workspace, page table -> -1, rope table
+  cudaError_t e = cudaMemsetAsync(workspace, 0, need, h->stream);
+  h->pt_host.assign(static_cast<size_t>(c.max_batch) * h->pt_stride, -1);
+  if (e == cudaSuccess)
+    e = cudaMemcpyAsync(h->page_table, h->pt_host.data(), h->pt_host.size() * 4,
+                        cudaMemcpyHostToDevice, h->stream);
+  if (e == cudaSuccess) {
+    rope_table_kernel<<<cdiv(static_cast<long long>(c.max_ctx) * 32, 256), 256, 0, h->stream>>>(
+        h->rope, c.max_ctx, static_cast<double>(c.rope_theta));
+    e = cudaGetLastError();
+  }
+  if (e == cudaSuccess) {
+    // sequences start "done" so a round over an unprefilled slot commits nothing
+    std::vector<int32_t> ones(c.max_batch, 1);
+    e = cudaMemcpyAsync(h->st.done, ones.data(), ones.size() * 4, cudaMemcpyHostToDevice, h->stream);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(h->stream);
+  }
+  if (e != cudaSuccess) {
+    delete h;
+    return fail(nullptr, GS_ERR_CUDA, std::string("workspace init: ") + cudaGetErrorString(e));
+  }
+  h->free_pages.reserve(h->n_pages);
+  for (int p = h->n_pages - 1; p >= 0; --p) h->free_pages.push_back(p);
+  h->slot_pages.assign(c.max_batch, {});
+  h->slot_reserved.assign(c.max_batch, 0);
+  *out = h;
+  return GS_OK;
+}
+
+int gs_destroy(gs_handle* h) {
+  if (!h) return GS_ERR_INVALID_ARG;
+  for (auto& kv : h->graphs) cudaGraphExecDestroy(kv.second);
+  delete h;
+  return GS_OK;
+}
+
+const char* gs_last_error(gs_handle* h) { return h ? h->err.c_str() : g_create_error.c_str(); }
+
+int gs_release(gs_handle* h, int slot) {
+  if (!h) return GS_ERR_INVALID_ARG;
+  if (slot < 0 || slot >= h->cfg.max_batch) return fail(h, GS_ERR_INVALID_ARG, "slot out of range");
+  for (int p : h->slot_pages[slot]) h->free_pages.push_back(p);
+  h->slot_pages[slot].clear();
+  h->slot_reserved[slot] = 0;
+  std::fill(h->pt_host.begin() + static_cast<size_t>(slot) * h->pt_stride,
+            h->pt_host.begin() + static_cast<size_t>(slot + 1) * h->pt_stride, -1);
+  GS_CUDA(h, cudaMemcpyAsync(h->page_table + static_cast<size_t>(slot) * h->pt_stride,
+                             h->pt_host.data() + static_cast<size_t>(slot) * h->pt_stride,
+                             h->pt_stride * 4, cudaMemcpyHostToDevice, h->stream));
+  const int one = 1;
+  GS_CUDA(h, cudaMemcpyAsync(h->st.done + slot, &one, 4, cudaMemcpyHostToDevice, h->stream));
+  GS_CUDA(h, cudaStreamSynchronize(h->stream));
+  return GS_OK;
+}
+
+int gs_prefill(gs_handle* h, int slot, const void* vis_emb, int n_vis, const int32_t* text,
+               int n_text, int max_new, int32_t* x0_out) {
+  if (!h) return GS_ERR_INVALID_ARG;
+  const gs_config& c = h->cfg;
+  if (slot < 0 || slot >= c.max_batch) return fail(h, GS_ERR_INVALID_ARG, "slot out of range");
+  if (n_vis < 0 || n_text < 0 || n_vis + n_text < 1 || max_new < 1)
+    return fail(h, GS_ERR_INVALID_ARG, "bad prefix or max_new");
+  if ((n_vis > 0 && !vis_emb) || (n_text > 0 && !text))
+    return fail(h, GS_ERR_INVALID_ARG, "null prefix pointer");
+  if (vis_emb && (reinterpret_cast<uintptr_t>(vis_emb) & 15))
+    return fail(h, GS_ERR_INVALID_ARG, "vis_emb not 16-byte aligned");
+  const long long P = static_cast<long long>(n_vis) + n_text;
+  const long long reserve = P + max_new + c.max_K + 2;
+  if (reserve > c.max_ctx) return fail(h, GS_ERR_OOM, "prefix + max_new + max_K + 2 > max_ctx");
+  // (re)reserve pages
+  int rc = gs_release(h, slot);
+  if (rc) return rc;
+  const int need = cdiv(reserve, 64);
+  if (need > static_cast<int>(h->free_pages.size()))
+    return fail(h, GS_ERR_OOM, "KV page pool exhausted");
+  for (int i = 0; i < need; ++i) {
+    const int p = h->free_pages.back();
+    h->free_pages.pop_back();
+    h->slot_pages[slot].push_back(p);
+    h->pt_host[static_cast<size_t>(slot) * h->pt_stride + i] = p;
+  }
+  h->slot_reserved[slot] = static_cast<int>(reserve);
+  GS_CUDA(h, cudaMemcpyAsync(h->page_table + static_cast<size_t>(slot) * h->pt_stride,
+                             h->pt_host.data() + static_cast<size_t>(slot) * h->pt_stride,
+                             h->pt_stride * 4, cudaMemcpyHostToDevice, h->stream));
+  // causal forward in chunks of max_prefill tokens
+  const int chunk = std::min(c.max_prefill, h->T_max);
+  const __nv_bfloat16* vis = static_cast<const __nv_bfloat16*>(vis_emb);
+  for (long long p0 = 0; p0 < P; p0 += chunk) {
+    const int T = static_cast<int>(std::min<long long>(chunk, P - p0));
+    const int vis_rows = static_cast<int>(std::max<long long>(0, std::min<long long>(n_vis - p0, T)));
+    const long long text0 = std::max<long long>(0, p0 - n_vis);
+    prefill_window_kernel<<<cdiv(T, 128), 128, 0, h->stream>>>(T, static_cast<int>(p0), slot,
+                                                               h->pos, h->lim, h->tok_slot);
+    GS_CUDA(h, cudaGetLastError());
+    AttnLaunch AL;
+    AL.QB = 64;
+    AL.n_blocks = cdiv(T, 64);
+    AL.max_splits = 1;
+    AL.split_pages = h->pt_stride;
+    AL.r_max = round16(64 * h->G);
+    AL.blk_slot = nullptr;
+    AL.blk_active = nullptr;
+    AL.fixed_slot = slot;
+    const bool last = p0 + T >= P;
+    rc = forward(h, T, text ? text + text0 : nullptr, vis ? vis + p0 * c.d_model : nullptr,
+                 vis_rows, AL, last ? T - 1 : 0, 1, h->packed_d, nullptr, false);
+    if (rc) return rc;
+  }
+  prefill_finish_kernel<<<1, 32, 0, h->stream>>>(h->packed_d, h->st, slot, static_cast<int>(P),
+                                                 max_new, c.eos_token_id, x0_out);
+  GS_CUDA(h, cudaGetLastError());
+  return GS_OK;
+}
+
+int gs_round(gs_handle* h, const int32_t* slots, int n_seq, int K, int rule, const gs_force* force,
+             int32_t* out_tok, int32_t* out_cnt, int32_t* out_done, const gs_debug* dbg) {
+  if (!h) return GS_ERR_INVALID_ARG;
+  const gs_config& c = h->cfg;
+  if (rule == GS_ACCEPT_STOCHASTIC)
+    return fail(h, GS_ERR_UNSUPPORTED, "stochastic acceptance is not implemented");
+  if (rule != GS_ACCEPT_GREEDY) return fail(h, GS_ERR_INVALID_ARG, "unknown acceptance rule");
+  if (!slots || !out_tok || !out_cnt || !out_done)
+    return fail(h, GS_ERR_INVALID_ARG, "null slots or output pointer");
+  if (n_seq < 1 || n_seq > c.max_batch) return fail(h, GS_ERR_INVALID_ARG, "n_seq out of range");
+  if (K < 0 || K > c.max_K) return fail(h, GS_ERR_INVALID_ARG, "K out of range");
+  if (force && (!force->teacher || !force->L_sched || force->teacher_stride < 1))
+    return fail(h, GS_ERR_INVALID_ARG, "incomplete force hook");
+  if (dbg || h->stream == nullptr)
+    return enqueue_round(h, slots, n_seq, K, force, out_tok, out_cnt, out_done, dbg);
+  gs_handle::GraphKey key(n_seq, K, slots, force ? force->teacher : nullptr,
+                          force ? force->teacher_stride : 0, force ? force->L_sched : nullptr,
+                          force ? force->L_stride : 0, out_tok, out_cnt, out_done);
+  auto it = h->graphs.find(key);
+  if (it == h->graphs.end()) {
+    cudaGraph_t g;
+    GS_CUDA(h, cudaStreamBeginCapture(h->stream, cudaStreamCaptureModeThreadLocal));
+    const int rc = enqueue_round(h, slots, n_seq, K, force, out_tok, out_cnt, out_done, nullptr);
+    cudaError_t e = cudaStreamEndCapture(h->stream, &g);
+    if (rc) {
+      if (e == cudaSuccess) cudaGraphDestroy(g);
+      return rc;
+    }
+    if (e != cudaSuccess) return fail(h, GS_ERR_CUDA, std::string("capture: ") + cudaGetErrorString(e));
+    cudaGraphExec_t ge;
+    e = cudaGraphInstantiate(&ge, g, 0);
+    cudaGraphDestroy(g);
+    if (e != cudaSuccess)
+      return fail(h, GS_ERR_CUDA, std::string("instantiate: ") + cudaGetErrorString(e));
+    if (h->graphs.size() >= 64) {
+      cudaGraphExecDestroy(h->graphs.begin()->second);
+      h->graphs.erase(h->graphs.begin());
+    }
+    it = h->graphs.emplace(key, ge).first;
+  }
+  GS_CUDA(h, cudaGraphLaunch(it->second, h->stream));
+  return GS_OK;
+}
+
+int gs_seq_restore(gs_handle* h, int slot, int seq_len, int x0, int n_out, int done) {
+  if (!h) return GS_ERR_INVALID_ARG;
+  const gs_config& c = h->cfg;
+  if (slot < 0 || slot >= c.max_batch || h->slot_reserved[slot] == 0)
+    return fail(h, GS_ERR_INVALID_ARG, "slot out of range or not prefilled");
+  if (seq_len < 1 || seq_len + c.max_K + 2 > h->slot_reserved[slot])
+    return fail(h, GS_ERR_INVALID_ARG, "seq_len outside the slot's reservation");
+  if (x0 < 0 || x0 >= c.vocab || n_out < 1) return fail(h, GS_ERR_INVALID_ARG, "bad x0 / n_out");
+  seq_restore_kernel<<<1, 32, 0, h->stream>>>(h->st, slot, seq_len, x0, n_out, done ? 1 : 0);
+  GS_CUDA(h, cudaGetLastError());
+  return GS_OK;
+}
+
+int gs_seq_state(gs_handle* h, int slot, int* seq_len, int* x0, int* n_out, int* done, int* rounds) {
+  if (!h) return GS_ERR_INVALID_ARG;
+  if (slot < 0 || slot >= h->cfg.max_batch) return fail(h, GS_ERR_INVALID_ARG, "slot out of range");
+  GS_CUDA(h, cudaStreamSynchronize(h->stream));
+  int v[6];
+  int32_t* src[6] = {h->st.seq_len, h->st.x0, h->st.n_out, h->st.done, h->st.rounds, h->st.max_new};
+  for (int i = 0; i < 6; ++i) GS_CUDA(h, cudaMemcpy(&v[i], src[i] + slot, 4, cudaMemcpyDeviceToHost));
+  if (seq_len) *seq_len = v[0];
+  if (x0) *x0 = v[1];
+  if (n_out) *n_out = v[2];
+  if (done) *done = v[3];
+  if (rounds) *rounds = v[4];
+  return GS_OK;
+}
+
+int gs_sync_check(gs_handle* h) {
+  if (!h) return GS_ERR_INVALID_ARG;
+  GS_CUDA(h, cudaStreamSynchronize(h->stream));
+  int word = 0;
+  GS_CUDA(h, cudaMemcpy(&word, h->err_word, 4, cudaMemcpyDeviceToHost));
+  if (word == 0) return GS_OK;
+  const int zero = 0;
+  GS_CUDA(h, cudaMemcpy(h->err_word, &zero, 4, cudaMemcpyHostToDevice));
+  if (word == kErrTimeout) return fail(h, GS_ERR_TIMEOUT, "a kernel's bounded wait ran out");
+  return fail(h, GS_ERR_DEVICE_CHECK, "a kernel bounds check fired");
+}
+
+// ------------------------------------------------------------ sub-step entry points
+size_t gs_attention_scratch_bytes(int n_seq, int W, int n_heads, int n_kv_heads, int max_pages,
+                                  int split_pages) {
+  if (n_seq < 1 || W < 1 || n_kv_heads < 1 || n_heads % n_kv_heads || max_pages < 1 ||
+      split_pages < 1)
+    return 0;
+  const int G = n_heads / n_kv_heads;
+  const int r_max = round16(W * G);
+  const int ms = cdiv(max_pages, split_pages);
+  Carver cv(nullptr);
+  cv.take<int>(64);                        // error word
+  cv.take<int32_t>(static_cast<size_t>(n_seq) * W);  // lim
+  cv.take<int32_t>(n_seq);                 // blk_slot
+  cv.take<int>(static_cast<size_t>(n_seq) * n_kv_heads);
+  cv.take<float>(static_cast<size_t>(n_seq) * n_kv_heads * ms * r_max * 2);
+  cv.take<float>(static_cast<size_t>(n_seq) * n_kv_heads * ms * r_max * 64);
+  return align_up(cv.off, 256);
+}
+
+}  // extern "C"
+
+namespace {
+__global__ void attn_standalone_prep(int mode, const int32_t* n, int n_seq, int W, int32_t* lim,
+                                     int32_t* blk_slot) {
+  const int idx = blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx >= n_seq * W) return;
+  const int b = idx / W, i = idx % W;
+  const int ns = n[b];
+  lim[idx] = mode == 0 ? (i == 0 ? ns : ns + W - 1) : ns + 1 + i;
+  if (i == 0) blk_slot[b] = b;
+}
+}  // namespace
+
+extern "C" {
+
+int gs_attention(int mode, const void* q, const void* kv, int n_pages, const int32_t* page_table,
+                 int pt_stride, const int32_t* n, int n_seq, int W, int n_heads, int n_kv_heads,
+                 void* out, void* scratch, size_t scratch_bytes, int split_pages, void* stream) {
+  if ((mode != 0 && mode != 1) || !q || !kv || !page_table || !n || !out || !scratch ||
+      n_pages < 1 || pt_stride < 1)
+    return GS_ERR_INVALID_ARG;
+  if (n_kv_heads < 1 || n_heads % n_kv_heads || W < 1 || n_seq < 1 || split_pages < 1)
+    return GS_ERR_INVALID_ARG;
+  const int G = n_heads / n_kv_heads;
+  if (W * G > 256) return GS_ERR_UNSUPPORTED;
+  if (scratch_bytes < gs_attention_scratch_bytes(n_seq, W, n_heads, n_kv_heads, pt_stride, split_pages))
+    return GS_ERR_OOM;
+  if ((reinterpret_cast<uintptr_t>(kv) & 15) || (reinterpret_cast<uintptr_t>(q) & 15))
+    return GS_ERR_INVALID_ARG;
+  static bool attr = false;
+  if (!attr) {
+    if (cudaFuncSetAttribute(attn_paged_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             attn_smem_bytes(256)) != cudaSuccess)
+      return GS_ERR_CUDA;
+    attr = true;
+  }
+  const int r_max = round16(W * G);
+  const int ms = cdiv(pt_stride, split_pages);
+  Carver cv(scratch);
+  int* err = cv.take<int>(64);
+  int32_t* lim = cv.take<int32_t>(static_cast<size_t>(n_seq) * W);
+  int32_t* blk_slot = cv.take<int32_t>(n_seq);
+  int* counters = cv.take<int>(static_cast<size_t>(n_seq) * n_kv_heads);
+  float* pml = cv.take<float>(static_cast<size_t>(n_seq) * n_kv_heads * ms * r_max * 2);
+  float* po = cv.take<float>(static_cast<size_t>(n_seq) * n_kv_heads * ms * r_max * 64);
+  CUtensorMap tm;
+  const uint64_t rows = static_cast<uint64_t>(n_pages) * 2 * n_kv_heads * 64;
+  if (rows >= (1ull << 31) || !make_map(&tm, kv, rows, 64, 64)) return GS_ERR_INVALID_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  attn_standalone_prep<<<cdiv(n_seq * W, 128), 128, 0, s>>>(mode, n, n_seq, W, lim, blk_slot);
+  AttnArgs a;
+  a.q = static_cast<const __nv_bfloat16*>(q);
+  a.lim = lim;
+  a.out = static_cast<__nv_bfloat16*>(out);
+  a.page_table = page_table;
+  a.pt_stride = pt_stride;
+  a.blk_slot = blk_slot;
+  a.blk_active = nullptr;
+  a.fixed_slot = -1;
+  a.T = n_seq * W;
+  a.QB = W;
+  a.Hq = n_heads;
+  a.Hkv = n_kv_heads;
+  a.G = G;
+  a.rows_per_page = 2 * n_kv_heads * 64;
+  a.kv_row_base = 0;
+  a.split_pages = split_pages;
+  a.max_splits = ms;
+  a.r_max = r_max;
+  a.part_o = po;
+  a.part_ml = pml;
+  a.counters = counters;
+  a.err = err;
+  dim3 grid(ms, n_kv_heads, n_seq);
+  attn_paged_kernel<<<grid, (r_max / 16) * 32, attn_smem_bytes(r_max), s>>>(tm, a);
+  return cudaGetLastError() == cudaSuccess ? GS_OK : GS_ERR_CUDA;
+}
+
+size_t gs_linear_scratch_bytes(int M, int N, int split_k) {
+  if (M < 1 || N < 64 || split_k < 1) return 0;
+  const int bn = gemm_bn_for(M);
+  const size_t tiles = static_cast<size_t>(cdiv(M, bn)) * cdiv(N, 64);
+  Carver cv(nullptr);
+  cv.take<int>(64);
+  cv.take<int>(tiles);
+  if (split_k > 1) cv.take<float>(static_cast<size_t>(split_k) * tiles * bn * 128);
+  return align_up(cv.off, 256);
+}
+
+int gs_linear(const void* x, const void* w, void* y, int M, int N, int K, int epilogue, int split_k,
+              void* scratch, size_t scratch_bytes, void* stream) {
+  if (!x || !w || !y || !scratch || M < 1 || K < 64 || K % 64 || split_k < 1 ||
+      (K / 64) % split_k)
+    return GS_ERR_INVALID_ARG;
+  if (epilogue < 0 || epilogue > 3) return GS_ERR_INVALID_ARG;
+  if (epilogue == kEpiSwiGLU ? (N % 64) : (N % 128)) return GS_ERR_INVALID_ARG;
+  if (M > 65536) return GS_ERR_UNSUPPORTED;
+  if (scratch_bytes < gs_linear_scratch_bytes(M, N, split_k)) return GS_ERR_OOM;
+  if ((reinterpret_cast<uintptr_t>(x) & 15) || (reinterpret_cast<uintptr_t>(w) & 15))
+    return GS_ERR_INVALID_ARG;
+  static bool attrs = false;
+  if (!attrs) {
+    if (gemm_init_attributes() != cudaSuccess) return GS_ERR_CUDA;
+    attrs = true;
+  }
+  const int bn = gemm_bn_for(M);
+  const int tok_tiles = cdiv(M, bn);
+  const int w_rows = epilogue == kEpiSwiGLU ? 2 * N : N;
+  const int feat_tiles = w_rows / 128;
+  CUtensorMap tw, tx;
+  if (!make_map(&tw, w, w_rows, K, epilogue == kEpiSwiGLU ? 64 : 128)) return GS_ERR_INVALID_ARG;
+  if (!make_map(&tx, x, M, K, bn)) return GS_ERR_INVALID_ARG;
+  Carver cv(scratch);
+  GemmArgs a;
+  a.err = cv.take<int>(64);
+  a.counters = cv.take<int>(static_cast<size_t>(tok_tiles) * cdiv(N, 64));
+  a.partial = split_k > 1
+                  ? cv.take<float>(static_cast<size_t>(split_k) * tok_tiles * feat_tiles * bn * 128)
+                  : nullptr;
+  a.M = M;
+  a.N = N;
+  a.K = K;
+  a.splits = split_k;
+  a.kb_per_split = (K / 64) / split_k;
+  a.y = y;
+  a.ldy = N;
+  a.logits = nullptr;
+  return launch_gemm(bn, epilogue, tw, tx, a, feat_tiles, tok_tiles,
+                     static_cast<cudaStream_t>(stream)) == cudaSuccess
+             ? GS_OK
+             : GS_ERR_CUDA;
+}
+
+}  // extern "C"

@@ -1,0 +1,63 @@
+// gemm.cu -- instantiations and launcher of the tcgen05 GEMM.
+#include "gemm_tc.cuh"
+#include "internal.h"
+
+namespace gs {
+
+template <int BN, int EPI>
+static cudaError_t launch_one(const CUtensorMap& tmW, const CUtensorMap& tmX, const GemmArgs& a,
+                              int feat_tiles, int tok_tiles, cudaStream_t s) {
+  dim3 grid(feat_tiles, tok_tiles, a.splits);
+  gemm_tc_kernel<BN, EPI><<<grid, 128, GemmShape<BN>::kSmemBytes, s>>>(tmW, tmX, a);
+  return cudaGetLastError();
+}
+
+template <int BN>
+static cudaError_t launch_bn(int epi, const CUtensorMap& tmW, const CUtensorMap& tmX,
+                             const GemmArgs& a, int ft, int tt, cudaStream_t s) {
+  switch (epi) {
+    case kEpiStoreBf16: return launch_one<BN, kEpiStoreBf16>(tmW, tmX, a, ft, tt, s);
+    case kEpiResidF32: return launch_one<BN, kEpiResidF32>(tmW, tmX, a, ft, tt, s);
+    case kEpiSwiGLU: return launch_one<BN, kEpiSwiGLU>(tmW, tmX, a, ft, tt, s);
+    case kEpiArgmax: return launch_one<BN, kEpiArgmax>(tmW, tmX, a, ft, tt, s);
+  }
+  return cudaErrorInvalidValue;
+}
+
+cudaError_t launch_gemm(int bn, int epi, const CUtensorMap& tmW, const CUtensorMap& tmX,
+                        const GemmArgs& a, int feat_tiles, int tok_tiles, cudaStream_t s) {
+  switch (bn) {
+    case 32: return launch_bn<32>(epi, tmW, tmX, a, feat_tiles, tok_tiles, s);
+    case 64: return launch_bn<64>(epi, tmW, tmX, a, feat_tiles, tok_tiles, s);
+    case 128: return launch_bn<128>(epi, tmW, tmX, a, feat_tiles, tok_tiles, s);
+    case 256: return launch_bn<256>(epi, tmW, tmX, a, feat_tiles, tok_tiles, s);
+  }
+  return cudaErrorInvalidValue;
+}
+
+template <int BN>
+static cudaError_t set_attr_bn() {
+  const int bytes = GemmShape<BN>::kSmemBytes;
+  cudaError_t e;
+  if ((e = cudaFuncSetAttribute(gemm_tc_kernel<BN, kEpiStoreBf16>,
+                                cudaFuncAttributeMaxDynamicSharedMemorySize, bytes)) != cudaSuccess)
+    return e;
+  if ((e = cudaFuncSetAttribute(gemm_tc_kernel<BN, kEpiResidF32>,
+                                cudaFuncAttributeMaxDynamicSharedMemorySize, bytes)) != cudaSuccess)
+    return e;
+  if ((e = cudaFuncSetAttribute(gemm_tc_kernel<BN, kEpiSwiGLU>,
+                                cudaFuncAttributeMaxDynamicSharedMemorySize, bytes)) != cudaSuccess)
+    return e;
+  return cudaFuncSetAttribute(gemm_tc_kernel<BN, kEpiArgmax>,
+                              cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+}
+
+cudaError_t gemm_init_attributes() {
+  cudaError_t e;
+  if ((e = set_attr_bn<32>()) != cudaSuccess) return e;
+  if ((e = set_attr_bn<64>()) != cudaSuccess) return e;
+  if ((e = set_attr_bn<128>()) != cudaSuccess) return e;
+  return set_attr_bn<256>();
+}
+
+}  // namespace gs

@@ -1,0 +1,261 @@
+// gemm_tc.cuh -- tcgen05/TMEM GEMM for the decoder's projections and LM head.
+//
+// Computes D[f, t] = sum_k W[f, k] X[t, k] with the weight rows on the MMA M
+// side (128 rows per CTA, "swap-AB") and the token rows on the MMA N side
+// (BN in {32, 64, 128, 256}), so a 17-token decode window and an 8192-token
+// prefill chunk use the same kernel.  Operands are K-major bf16 tiles staged by
+// TMA with 128-byte swizzle; one elected thread issues tcgen05.mma into a TMEM
+// fp32 accumulator of 128 lanes x BN columns; four warps read it back with
+// tcgen05.ld for the fused epilogue.
+//
+// Split-K: CTAs of one output tile that own different K ranges write fp32
+// partials; the last CTA to arrive (atomic counter, no spinning) sums the
+// partials in split order, so results do not depend on arrival order.
+//
+// Epilogues: bf16 store, fp32 residual add, SwiGLU (gate and up rows of the
+// same features share a tile), and LM-head argmax (packed 64-bit atomicMax,
+// ties to the lowest index) with an optional fp32 logit dump.
+#pragma once
+#include "ptx.cuh"
+
+namespace gs {
+
+enum GemmEpilogue : int { kEpiStoreBf16 = 0, kEpiResidF32 = 1, kEpiSwiGLU = 2, kEpiArgmax = 3 };
+
+struct GemmArgs {
+  int M;            // token rows
+  int N;            // output features (for SwiGLU: d_ffn, the weight has 2N rows)
+  int K;            // reduction length, multiple of 64
+  int splits;       // split-K factor (divides K / 64)
+  int kb_per_split; // (K / 64) / splits
+  void* y;          // output: bf16 [M, ldy] | fp32 [M, ldy] | uint64 [M] (argmax)
+  int ldy;
+  float* partial;   // split-K partials [splits][tiles][BN][128] fp32
+  int* counters;    // per output tile, zero between launches
+  float* logits;    // argmax only: optional fp32 [M, N] dump
+  int* err;
+};
+
+template <int BN>
+struct GemmShape {
+  static constexpr int kABytes = 128 * 128;        // 128 rows x 64 bf16
+  static constexpr int kBBytes = BN * 128;         // BN rows x 64 bf16
+  static constexpr int kStageBytes = kABytes + kBBytes;
+  // two CTAs per SM up to BN = 128 (<= ~97 KB each), one at BN = 256
+  static constexpr int kStages = BN <= 64 ? 4 : (BN <= 128 ? 3 : 4);
+  static constexpr int kTmemCols = BN < 32 ? 32 : BN;
+  static constexpr int kSmemBytes = kStages * kStageBytes + 1024 /*align*/ + 256 /*barriers*/;
+};
+
+template <int BN, int EPI>
+__device__ __forceinline__ void gemm_epilogue_chunk(const GemmArgs& a, float (&v)[32], int row,
+                                                    int feat_tile, int tok0, int chunk,
+                                                    float* xbuf) {
+  const int warp = threadIdx.x >> 5;
+  const int t0 = tok0 + chunk * 32;
+  const int nvalid = min(32, a.M - t0);
+  if constexpr (EPI == kEpiStoreBf16) {
+    __nv_bfloat16* y = static_cast<__nv_bfloat16*>(a.y);
+    const int f = feat_tile * 128 + row;
+#pragma unroll
+    for (int j = 0; j < 32; ++j)
+      if (j < nvalid) y[static_cast<size_t>(t0 + j) * a.ldy + f] = __float2bfloat16_rn(v[j]);
+  } else if constexpr (EPI == kEpiResidF32) {
+    float* y = static_cast<float*>(a.y);
+    const int f = feat_tile * 128 + row;
+#pragma unroll
+    for (int j = 0; j < 32; ++j)
+      if (j < nvalid) {
+        float* p = y + static_cast<size_t>(t0 + j) * a.ldy + f;
+        *p = *p + v[j];
+      }
+  } else if constexpr (EPI == kEpiSwiGLU) {
+    // rows 0..63: gate of features f0..f0+63; rows 64..127: up of the same features
+    if (warp >= 2) {
+#pragma unroll
+      for (int j = 0; j < 32; ++j) xbuf[j * 64 + (row - 64)] = v[j];
+    }
+    asm volatile("bar.sync 1, 128;" ::: "memory");
+    if (warp < 2) {
+      __nv_bfloat16* y = static_cast<__nv_bfloat16*>(a.y);
+      const int f = feat_tile * 64 + row;
+#pragma unroll
+      for (int j = 0; j < 32; ++j)
+        if (j < nvalid) {
+          const float g = v[j];
+          const float u = xbuf[j * 64 + row];
+          const float s = g / (1.0f + __expf(-g));
+          y[static_cast<size_t>(t0 + j) * a.ldy + f] = __float2bfloat16_rn(s * u);
+        }
+    }
+    asm volatile("bar.sync 1, 128;" ::: "memory");
+  } else {  // argmax over the vocabulary rows of this tile, per token
+    const uint32_t f = static_cast<uint32_t>(feat_tile * 128 + row);
+    unsigned long long* out = static_cast<unsigned long long*>(a.y);
+    if (a.logits != nullptr) {
+#pragma unroll
+      for (int j = 0; j < 32; ++j)
+        if (j < nvalid) a.logits[static_cast<size_t>(t0 + j) * a.N + f] = v[j];
+    }
+    const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int j = 0; j < 32; ++j) {
+      unsigned long long key = argmax_key(v[j], f);
+#pragma unroll
+      for (int m = 16; m >= 1; m >>= 1) {
+        const unsigned long long o = shfl_xor_u64(key, m);
+        key = o > key ? o : key;
+      }
+      if (lane == 0 && j < nvalid) atomicMax(out + t0 + j, key);
+    }
+  }
+}
+
+template <int BN, int EPI>
+__global__ void __launch_bounds__(128, 1)
+    gemm_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmX,
+                   const GemmArgs a) {
+  using S = GemmShape<BN>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  uint8_t* smA = smem;
+  uint8_t* smB = smem + S::kStages * S::kABytes;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + S::kStages * S::kStageBytes);
+  uint64_t* full = bars;
+  uint64_t* empty = bars + S::kStages;
+  uint64_t* accum = bars + 2 * S::kStages;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(accum + 1);
+  volatile int* flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const int feat_tile = blockIdx.x;
+  const int tok_tile = blockIdx.y;
+  const int split = blockIdx.z;
+  const int kb0 = split * a.kb_per_split;
+  const int nkb = a.kb_per_split;
+
+  if (threadIdx.x == 0) {
+    tma_prefetch_desc(&tmW);
+    tma_prefetch_desc(&tmX);
+    for (int s = 0; s < S::kStages; ++s) {
+      mbar_init(smem_u32(&full[s]), 1);
+      mbar_init(smem_u32(&empty[s]), 1);
+    }
+    mbar_init(smem_u32(accum), 1);
+    *flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 2) tmem_alloc(smem_u32(tmem_slot), S::kTmemCols);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0 && lane == 0) {
+    // TMA producer
+    const uint64_t pol_w = l2_policy_evict_first();
+    const uint64_t pol_x = l2_policy_evict_last();
+    for (int i = 0; i < nkb; ++i) {
+      const int s = i % S::kStages;
+      const uint32_t ph = (i / S::kStages) & 1;
+      if (!mbar_wait(smem_u32(&empty[s]), ph ^ 1, a.err)) { *flag = 1; break; }
+      const uint32_t fb = smem_u32(&full[s]);
+      mbar_arrive_expect_tx(fb, S::kStageBytes);
+      const int kx = (kb0 + i) * 64;
+      if constexpr (EPI == kEpiSwiGLU) {
+        tma_load_2d(smem_u32(smA + s * S::kABytes), &tmW, kx, feat_tile * 64, fb, pol_w);
+        tma_load_2d(smem_u32(smA + s * S::kABytes + 64 * 128), &tmW, kx, a.N + feat_tile * 64, fb,
+                    pol_w);
+      } else {
+        tma_load_2d(smem_u32(smA + s * S::kABytes), &tmW, kx, feat_tile * 128, fb, pol_w);
+      }
+      tma_load_2d(smem_u32(smB + s * S::kBBytes), &tmX, kx, tok_tile * BN, fb, pol_x);
+    }
+  } else if (warp == 1 && lane == 0) {
+    // MMA issuer
+    constexpr uint32_t idesc = umma_idesc_bf16(128, BN);
+    bool ok = true;
+    for (int i = 0; i < nkb; ++i) {
+      const int s = i % S::kStages;
+      const uint32_t ph = (i / S::kStages) & 1;
+      if (!mbar_wait(smem_u32(&full[s]), ph, a.err)) { ok = false; *flag = 1; break; }
+      tc_fence_after();
+      const uint64_t ad = umma_desc_sw128(smem_u32(smA + s * S::kABytes));
+      const uint64_t bd = umma_desc_sw128(smem_u32(smB + s * S::kBBytes));
+#pragma unroll
+      for (int k = 0; k < 4; ++k)
+        umma_bf16(tmem, ad + 2 * k, bd + 2 * k, idesc, (i > 0 || k > 0) ? 1u : 0u);
+      umma_commit(smem_u32(&empty[s]));
+    }
+    umma_commit(smem_u32(accum));
+    (void)ok;
+  }
+  __syncwarp();
+
+  // All four warps: wait for the accumulator, then the epilogue.
+  const bool acc_ok = mbar_wait(smem_u32(accum), 0, a.err);
+  tc_fence_after();
+  const int row = warp * 32 + lane;      // TMEM lane = weight row of the tile
+  const uint32_t trow = tmem + (static_cast<uint32_t>(warp * 32) << 16);
+  float* xbuf = reinterpret_cast<float*>(smA);   // pipeline smem is free after the accumulator
+  const int tok0 = tok_tile * BN;
+  const bool failed = !acc_ok || *flag;
+
+  if (a.splits == 1) {
+    if (!failed) {
+      for (int c = 0; c < BN / 32; ++c) {
+        if (tok0 + c * 32 >= a.M) break;   // uniform across the CTA
+        float v[32];
+        tmem_ld_32x32b_x32(trow + c * 32, v);
+        gemm_epilogue_chunk<BN, EPI>(a, v, row, feat_tile, tok0, c, xbuf);
+      }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 2) tmem_dealloc(tmem, S::kTmemCols);
+    return;
+  }
+
+  // split-K: write this split's partial tile, token-major [BN][128]
+  const int tiles = gridDim.x * gridDim.y;
+  const int tile = tok_tile * gridDim.x + feat_tile;
+  float* mine = a.partial + (static_cast<size_t>(split) * tiles + tile) * (BN * 128);
+  if (!failed) {
+    for (int c = 0; c < BN / 32; ++c) {
+      if (tok0 + c * 32 >= a.M) break;
+      float v[32];
+      tmem_ld_32x32b_x32(trow + c * 32, v);
+#pragma unroll
+      for (int j = 0; j < 32; ++j) mine[(c * 32 + j) * 128 + row] = v[j];
+    }
+  }
+  __threadfence();
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 2) tmem_dealloc(tmem, S::kTmemCols);
+  __shared__ int is_last;
+  if (threadIdx.x == 0) {
+    const int old = atomicAdd(a.counters + tile, 1);
+    is_last = (old == a.splits - 1);
+    if (is_last) a.counters[tile] = 0;
+  }
+  __syncthreads();
+  if (!is_last || failed) return;
+  __threadfence();
+  for (int c = 0; c < BN / 32; ++c) {
+    if (tok0 + c * 32 >= a.M) break;
+    float v[32];
+#pragma unroll
+    for (int j = 0; j < 32; ++j) v[j] = 0.0f;
+    for (int s = 0; s < a.splits; ++s) {
+      const float* p = a.partial + (static_cast<size_t>(s) * tiles + tile) * (BN * 128);
+#pragma unroll
+      for (int j = 0; j < 32; ++j) v[j] += __ldcg(p + (c * 32 + j) * 128 + row);
+    }
+    gemm_epilogue_chunk<BN, EPI>(a, v, row, feat_tile, tok0, c, xbuf);
+  }
+}
+
+}  // namespace gs

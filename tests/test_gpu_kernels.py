@@ -1,0 +1,183 @@
+"""Kernel-level GPU parity: the tcgen05 GEMM against a plain fp32 torch matmul,
+and the paged hybrid-mask attention against the oracle's float64 masked
+softmax (draft and verify masks from the oracle's mask builders)."""
+import math
+import types
+
+import numpy as np
+import pytest
+import torch
+
+import synth
+from oracle import decode as od
+from oracle.model import Decoder
+
+pytestmark = pytest.mark.gpu
+DEV = "cuda:0"
+
+
+@pytest.fixture(scope="module")
+def gs():
+    from paper_2609_26638_gb300 import gs as binding
+    return binding
+
+
+def _linear(gs, x, w, M, N, K, epi, split, y):
+    sb = gs.gs_linear_scratch_bytes(M, N, split)
+    scratch = torch.zeros(sb, dtype=torch.uint8, device=DEV)
+    gs.gs_linear(x.data_ptr(), w.data_ptr(), y.data_ptr(), M, N, K, epi, split, scratch.data_ptr(),
+                 sb, torch.cuda.current_stream().cuda_stream)
+    torch.cuda.synchronize()
+
+
+@pytest.mark.parametrize("M", [1, 17, 33, 100, 264, 544])
+@pytest.mark.parametrize("N,K,split", [(256, 256, 1), (2048, 1024, 8), (1024, 4096, 16)])
+def test_linear_store_and_residual(gs, M, N, K, split):
+    g = torch.Generator(device=DEV).manual_seed(M * 7 + N)
+    x = torch.randn(M, K, device=DEV, generator=g).bfloat16()
+    w = (0.02 * torch.randn(N, K, device=DEV, generator=g)).bfloat16()
+    ref = x.float() @ w.float().T
+    y = torch.zeros(M, N, dtype=torch.bfloat16, device=DEV)
+    _linear(gs, x, w, M, N, K, gs.EPI_STORE_BF16, split, y)
+    torch.testing.assert_close(y.float(), ref, rtol=1e-2, atol=1e-2 * ref.abs().max().item())
+    base = torch.randn(M, N, device=DEV, generator=g)
+    r = base.clone()
+    _linear(gs, x, w, M, N, K, gs.EPI_RESID_F32, split, r)
+    torch.testing.assert_close(r, base + ref, rtol=1e-4, atol=1e-4 * ref.abs().max().item())
+
+
+@pytest.mark.parametrize("M,split", [(9, 1), (17, 2), (200, 1)])
+def test_linear_swiglu(gs, M, split):
+    F, K = 1024, 256
+    g = torch.Generator(device=DEV).manual_seed(3)
+    x = torch.randn(M, K, device=DEV, generator=g).bfloat16()
+    w = (0.05 * torch.randn(2 * F, K, device=DEV, generator=g)).bfloat16()
+    gu = x.float() @ w.float().T
+    ref = torch.nn.functional.silu(gu[:, :F]) * gu[:, F:]
+    y = torch.zeros(M, F, dtype=torch.bfloat16, device=DEV)
+    _linear(gs, x, w, M, F, K, gs.EPI_SWIGLU, split, y)
+    torch.testing.assert_close(y.float(), ref, rtol=1.5e-2, atol=1e-2 * ref.abs().max().item())
+
+
+@pytest.mark.parametrize("M,V", [(1, 4096), (17, 59392), (70, 4096)])
+def test_linear_argmax(gs, M, V):
+    K = 1024
+    g = torch.Generator(device=DEV).manual_seed(M)
+    x = torch.randn(M, K, device=DEV, generator=g).bfloat16()
+    w = (0.02 * torch.randn(V, K, device=DEV, generator=g)).bfloat16()
+    ref = x.float() @ w.float().T
+    keys = torch.zeros(M, dtype=torch.int64, device=DEV)
+    _linear(gs, x, w, M, V, K, gs.EPI_ARGMAX, 1, keys)
+    idx = (0xFFFFFFFF - (keys & 0xFFFFFFFF)).cpu().numpy()
+    want = ref.argmax(dim=1).cpu().numpy()
+    top2 = ref.topk(2, dim=1).values
+    gap = (top2[:, 0] - top2[:, 1]).cpu().numpy()
+    for i in range(M):
+        if idx[i] != want[i]:
+            assert gap[i] < 1e-4, (i, idx[i], want[i], gap[i])
+    # ties resolve to the lowest index: duplicate the winning row further down
+    w2 = w.clone()
+    w2[V - 1] = w2[int(want[0])]
+    keys.zero_()
+    _linear(gs, x[:1].contiguous(), w2, 1, V, K, gs.EPI_ARGMAX, 1, keys)
+    got = int(0xFFFFFFFF - (int(keys[0].item()) & 0xFFFFFFFF))
+    assert got == min(int(want[0]), V - 1) or gap[0] < 1e-4
+
+
+def test_linear_rows_do_not_depend_on_batch(gs):
+    """Same token tile and split: a row's bits do not depend on the other rows."""
+    N, K = 2048, 1024
+    g = torch.Generator(device=DEV).manual_seed(5)
+    x = torch.randn(17, K, device=DEV, generator=g).bfloat16()
+    w = (0.02 * torch.randn(N, K, device=DEV, generator=g)).bfloat16()
+    y17 = torch.zeros(17, N, dtype=torch.bfloat16, device=DEV)
+    _linear(gs, x, w, 17, N, K, gs.EPI_STORE_BF16, 8, y17)
+    for r in (0, 5, 16):
+        y1 = torch.zeros(1, N, dtype=torch.bfloat16, device=DEV)
+        _linear(gs, x[r:r + 1].contiguous(), w, 1, N, K, gs.EPI_STORE_BF16, 8, y1)
+        assert torch.equal(y1[0], y17[r])
+
+
+# ------------------------------------------------------------------ attention
+def _paged(k, v, rng):
+    """Pack per-sequence K/V [B, ctx, Hkv, 64] into a shuffled page pool."""
+    B, ctx, Hkv, hd = k.shape
+    pages_per = math.ceil(ctx / 64)
+    n_pages = B * pages_per + 3
+    perm = rng.permutation(n_pages)[: B * pages_per].reshape(B, pages_per)
+    pool = np.zeros((n_pages, 2, Hkv, 64, 64), dtype=np.uint16)
+    for b in range(B):
+        for p in range(pages_per):
+            t0, t1 = p * 64, min(ctx, p * 64 + 64)
+            pool[perm[b, p], 0, :, : t1 - t0] = k[b, t0:t1].transpose(1, 0, 2)
+            pool[perm[b, p], 1, :, : t1 - t0] = v[b, t0:t1].transpose(1, 0, 2)
+    return pool, perm.astype(np.int32), n_pages
+
+
+def _oracle_attn(q, k, v, allowed, Hq, Hkv):
+    fake = types.SimpleNamespace(cfg=types.SimpleNamespace(n_heads=Hq, n_kv_heads=Hkv, head_dim=64))
+    return Decoder.attention(fake, q, k, v, allowed)
+
+
+def _run_attention(gs, mode, q_bits, pool, pt, n_arr, W, Hq, Hkv, split_pages):
+    B = q_bits.shape[0]
+    qd = torch.from_numpy(q_bits.view(np.int16)).to(DEV)
+    kvd = torch.from_numpy(pool.view(np.int16)).to(DEV)
+    ptd = torch.from_numpy(pt).to(DEV)
+    nd = torch.from_numpy(n_arr.astype(np.int32)).to(DEV)
+    out = torch.zeros(q_bits.shape, dtype=torch.int16, device=DEV)
+    sb = gs.gs_attention_scratch_bytes(B, W, Hq, Hkv, pt.shape[1], split_pages)
+    scratch = torch.zeros(sb, dtype=torch.uint8, device=DEV)
+    gs.gs_attention(mode, qd.data_ptr(), kvd.data_ptr(), pool.shape[0], ptd.data_ptr(), pt.shape[1],
+                    nd.data_ptr(), B, W, Hq, Hkv, out.data_ptr(), scratch.data_ptr(), sb,
+                    split_pages, torch.cuda.current_stream().cuda_stream)
+    torch.cuda.synchronize()
+    return synth.bf16_bits_to_f32(out.cpu().numpy().view(np.uint16)).astype(np.float64)
+
+
+@pytest.mark.parametrize("mode", [0, 1])
+@pytest.mark.parametrize("W,ns,Hq,Hkv,sp", [
+    (5, [1, 63, 64], 16, 8, 1),
+    (17, [2048, 2500], 16, 8, 2),
+    (33, [0, 127, 4000], 16, 8, 3),
+    (65, [190, 1030], 16, 8, 64),
+    (9, [440, 511], 4, 4, 2),
+])
+def test_attention_matches_oracle(gs, mode, W, ns, Hq, Hkv, sp):
+    rng = np.random.default_rng(W * 31 + mode)
+    B = len(ns)
+    ctx = max(ns) + W + 1
+    q, k, v = synth.attn_inputs(B, W, ctx, Hq, Hkv, index=W + mode)
+    pool, pt, n_pages = _paged(k, v, rng)
+    got = _run_attention(gs, mode, q, pool, pt, np.array(ns), W, Hq, Hkv, sp)
+    K = W - 1
+    for b, n in enumerate(ns):
+        allowed = od.draft_allowed(n, K) if mode == 0 else od.verify_allowed(n, K)
+        nk = allowed.shape[1]
+        qf = synth.bf16_bits_to_f32(q[b]).astype(np.float64)
+        kf = synth.bf16_bits_to_f32(k[b, :nk]).astype(np.float64)
+        vf = synth.bf16_bits_to_f32(v[b, :nk]).astype(np.float64)
+        want = _oracle_attn(qf, kf, vf, allowed, Hq, Hkv)
+        np.testing.assert_allclose(got[b], want, rtol=2e-2, atol=2e-2)
+
+
+@pytest.mark.parametrize("B,prefix,K", [(64, 8192, 64), (8, 4096, 16), (1, 1024, 4)])
+def test_attention_sweep_sizes_sampled(gs, B, prefix, K):
+    """Attention-sweep shapes; the oracle checks a seeded sample of sequences."""
+    W = K + 1
+    Hq, Hkv = 16, 8
+    rng = np.random.default_rng(prefix + B)
+    ns = [prefix] * B
+    ctx = prefix + W + 1
+    q, k, v = synth.attn_inputs(B, W, ctx, Hq, Hkv, index=B)
+    pool, pt, _ = _paged(k, v, rng)
+    sp = max(1, math.ceil(pt.shape[1] * B * Hkv / 304))
+    for mode in (0, 1):
+        got = _run_attention(gs, mode, q, pool, pt, np.array(ns), W, Hq, Hkv, sp)
+        for b in sorted(set([0, B - 1] + list(rng.integers(0, B, 2)))):
+            allowed = od.draft_allowed(prefix, K) if mode == 0 else od.verify_allowed(prefix, K)
+            nk = allowed.shape[1]
+            want = _oracle_attn(synth.bf16_bits_to_f32(q[b]).astype(np.float64),
+                                synth.bf16_bits_to_f32(k[b, :nk]).astype(np.float64),
+                                synth.bf16_bits_to_f32(v[b, :nk]).astype(np.float64), allowed, Hq, Hkv)
+            np.testing.assert_allclose(got[b], want, rtol=2e-2, atol=2e-2)

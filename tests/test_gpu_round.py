@@ -1,0 +1,202 @@
+"""GPU round parity against the oracle, batch invariance, forcing and edge cases."""
+import numpy as np
+import pytest
+import torch
+
+import synth
+from oracle import decode as od
+from oracle.model import Decoder
+from tests.gpu_util import NEAR_TIE, gpu_accept, lockstep, new_engine
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def tiny():
+    w = synth.make_weights(synth.TINY, seed=synth.WEIGHT_SEED)
+    return synth.TINY, w, Decoder(synth.TINY, w)
+
+
+@pytest.fixture(scope="module")
+def tiny_gain():
+    cfg = synth.TINY.with_(n_heads=8, n_kv_heads=4)   # GQA group 2 on the tiny decoder
+    w = synth.make_weights(cfg, seed=7, gain_std=0.1)
+    return cfg, w, Decoder(cfg, w)
+
+
+def test_tiny_workload_lockstep(tiny):
+    """Tiny decoder workload: prefix 448 visual + 64 text, K = 8, about 64 rounds."""
+    cfg, w, dec = tiny
+    wl = synth.WORKLOADS["tiny"]
+    prompt = wl.prompts()[0]
+    eng = new_engine(cfg, w, max_ctx=1024, max_K=8, max_prefill=512)
+    st, stats = lockstep(eng, dec, prompt, wl.K, wl.max_new, check_logits=True)
+    print(f"\ntiny lockstep: {stats}")
+    assert st.done and len(st.out) == wl.max_new
+    assert stats.rounds >= 30
+    assert stats.max_logit_err <= 3e-2
+    eng.close()
+
+
+@pytest.mark.parametrize("K,n_vis,n_text", [(0, 40, 23), (1, 64, 0), (4, 0, 65), (15, 100, 27),
+                                            (16, 127, 1)])
+def test_tiny_gqa_gains_lockstep(tiny_gain, K, n_vis, n_text):
+    """GQA group 2, non-unit norm gains, ragged prefixes around page edges, K in 0..16."""
+    cfg, w, dec = tiny_gain
+    prompt = synth.make_prompt(cfg, n_vis, n_text, index=K)
+    eng = new_engine(cfg, w, max_ctx=512, max_K=16, max_prefill=96)   # prefill in chunks
+    st, stats = lockstep(eng, dec, prompt, K, 48, check_logits=True)
+    print(f"\nK={K}: {stats}")
+    assert st.done and len(st.out) == 48
+    eng.close()
+
+
+def _decode_all(eng, slots, K, max_rounds, force=None):
+    dev = eng.device
+    n = slots.shape[0]
+    out_tok = torch.zeros((n, K + 2), dtype=torch.int32, device=dev)
+    cnt = torch.zeros(n, dtype=torch.int32, device=dev)
+    done = torch.zeros(n, dtype=torch.int32, device=dev)
+    outs = [[] for _ in range(n)]
+    torch.cuda.synchronize(dev)
+    for _ in range(max_rounds):
+        eng.round(slots, K, out_tok, cnt, done, force=force)
+        eng.stream.synchronize()
+        c = cnt.cpu().numpy()
+        t = out_tok.cpu().numpy()
+        for i in range(n):
+            outs[i].extend(t[i, :c[i]].tolist())
+        if done.cpu().numpy().all():
+            break
+    eng.check()
+    return outs
+
+
+def test_gpu_self_spec_equals_gpu_ar(tiny_gain):
+    """Batch-invariant kernels: the GPU's self-speculative output equals its own
+    greedy AR (K = 0) output token for token (the paper's AR-equivalence, here
+    exact because a row's arithmetic does not depend on the window it sits in)."""
+    cfg, w, _ = tiny_gain
+    eng = new_engine(cfg, w, max_ctx=1024, max_K=16, max_prefill=256)
+    prompt = synth.make_prompt(cfg, 200, 50, index=11)
+    slots = torch.tensor([0], dtype=torch.int32, device=eng.device)
+    outs = {}
+    for K in (0, 3, 8, 16):
+        x0 = eng.prefill(0, prompt.vis, prompt.text, 200)
+        outs[K] = [x0] + _decode_all(eng, slots, K, 400)[0]
+        assert len(outs[K]) == 200
+    assert outs[3] == outs[0] and outs[8] == outs[0] and outs[16] == outs[0]
+    eng.close()
+
+
+def test_forced_acceptance_hits_schedule(tiny_gain):
+    """Forcing d_1..d_L to the greedy continuation makes the verifier accept exactly L."""
+    cfg, w, _ = tiny_gain
+    K, max_new = 16, 300
+    eng = new_engine(cfg, w, max_ctx=2048, max_K=K, max_prefill=256)
+    prompt = synth.make_prompt(cfg, 300, 20, index=12)
+    slots = torch.tensor([0], dtype=torch.int32, device=eng.device)
+    x0 = eng.prefill(0, prompt.vis, prompt.text, max_new + K + 4)
+    ref = [x0] + _decode_all(eng, slots, K, 1000)[0]
+    P = prompt.length
+    teacher = np.full(P + len(ref) + 4, -1, np.int32)
+    teacher[P:P + len(ref)] = ref
+    sched = synth.accept_schedule("geometric", K, 1, 200)
+    from paper_2609_26638_gb300 import gs
+    t_dev = torch.from_numpy(teacher).to(eng.device)
+    s_dev = torch.from_numpy(sched).to(eng.device)
+    force = gs.gs_force(teacher=t_dev.data_ptr(), teacher_stride=teacher.shape[0],
+                        L_sched=s_dev.data_ptr(), L_stride=sched.shape[1])
+    x0b = eng.prefill(0, prompt.vis, prompt.text, max_new)
+    assert x0b == x0
+    dev = eng.device
+    out_tok = torch.zeros((1, K + 2), dtype=torch.int32, device=dev)
+    cnt = torch.zeros(1, dtype=torch.int32, device=dev)
+    done = torch.zeros(1, dtype=torch.int32, device=dev)
+    torch.cuda.synchronize(dev)
+    got = [x0]
+    r = 0
+    while True:
+        eng.round(slots, K, out_tok, cnt, done, force=force)
+        eng.stream.synchronize()
+        c = int(cnt.cpu()[0])
+        got.extend(out_tok.cpu().numpy()[0, :c].tolist())
+        if int(done.cpu()[0]):
+            break
+        assert c == int(sched[0, r]) + 2, (r, c, sched[0, r])
+        r += 1
+    assert got == ref[:max_new]
+    eng.check()
+    eng.close()
+
+
+def test_batch_equals_single_and_ragged_finish(tiny_gain):
+    """Three sequences with different prefixes and caps decoded as one batch give
+    the same tokens as each decoded alone; finished ones commit nothing more."""
+    cfg, w, _ = tiny_gain
+    K = 6
+    eng = new_engine(cfg, w, max_batch=4, max_ctx=1024, max_K=K, max_prefill=256)
+    prompts = [synth.make_prompt(cfg, nv, nt, index=20 + i)
+               for i, (nv, nt) in enumerate([(63, 2), (130, 5), (10, 1)])]
+    caps = [40, 17, 29]
+    single = []
+    for i, p in enumerate(prompts):
+        x0 = eng.prefill(i, p.vis, p.text, caps[i])
+        single.append([x0] + _decode_all(eng, torch.tensor([i], dtype=torch.int32, device=eng.device),
+                                         K, 100)[0])
+    x0s = [eng.prefill(i, p.vis, p.text, caps[i]) for i, p in enumerate(prompts)]
+    slots = torch.tensor([2, 0, 1], dtype=torch.int32, device=eng.device)   # any slot order
+    outs = _decode_all(eng, slots, K, 100)
+    batch = {2: outs[0], 0: outs[1], 1: outs[2]}
+    for i in range(3):
+        assert [x0s[i]] + batch[i] == single[i]
+        assert len(single[i]) == caps[i]
+    eng.close()
+
+
+def test_stop_token_truncates(tiny_gain):
+    cfg, w, dec = tiny_gain
+    prompt = synth.make_prompt(cfg, 50, 10, index=31)
+    ar = od.ar_decode(dec, od.prefill(dec, prompt.vis, prompt.text, 512, 40))
+    eos = ar[9]
+    eng = new_engine(cfg, w, max_ctx=512, max_K=8, max_prefill=128, eos=eos)
+    st, stats = lockstep(eng, dec, prompt, 8, 40, eos=eos)
+    assert st.done and st.out[-1] == eos and eos not in st.out[:-1]
+    eng.close()
+
+
+def test_bad_requests_raise(tiny):
+    from paper_2609_26638_gb300 import gs
+    cfg, w, _ = tiny
+    eng = new_engine(cfg, w, max_ctx=256, max_K=4, max_prefill=128)
+    dev = eng.device
+    slots = torch.tensor([0], dtype=torch.int32, device=dev)
+    o = torch.zeros((1, 8), dtype=torch.int32, device=dev)
+    c = torch.zeros(1, dtype=torch.int32, device=dev)
+    d = torch.zeros(1, dtype=torch.int32, device=dev)
+    with pytest.raises(gs.GsError) as e:
+        eng.round(slots, 5, o, c, d)                         # K > max_K
+    assert e.value.code == gs.GS_ERR_INVALID_ARG
+    with pytest.raises(gs.GsError) as e:
+        gs.gs_round(eng.handle, slots.data_ptr(), 1, 2, gs.GS_ACCEPT_STOCHASTIC, None,
+                    o.data_ptr(), c.data_ptr(), d.data_ptr())
+    assert e.value.code == gs.GS_ERR_UNSUPPORTED
+    p = synth.make_prompt(cfg, 200, 10)
+    with pytest.raises(gs.GsError) as e:
+        eng.prefill(0, p.vis, p.text, 100)                   # 210 + 100 + 6 > 256
+    assert e.value.code == gs.GS_ERR_OOM
+    with pytest.raises(gs.GsError):
+        eng.prefill(3, p.vis[:8], p.text[:2], 4)             # slot out of range
+    # an unprefilled slot is "done": a round commits nothing
+    eng.round(slots, 2, o, c, d)
+    eng.stream.synchronize()
+    assert int(c.cpu()[0]) == 0 and int(d.cpu()[0]) == 1
+    # out-of-range token id: the kernel clamps it and raises the device check
+    bad = p.text[:4].copy()
+    bad[1] = cfg.vocab + 5
+    eng.prefill(0, None, bad, 4)
+    with pytest.raises(gs.GsError) as e:
+        eng.check()
+    assert e.value.code == gs.GS_ERR_DEVICE_CHECK
+    eng.check()                                            # cleared
+    eng.close()
