@@ -1,0 +1,475 @@
+"""Benchmark: greedy self-speculative decoding rounds on one GB300 per rank.
+
+Workload (default ``glm_b1``): the GLM-OCR-scale synthetic decoder (24 layers,
+d_model 1024, 16 query / 8 KV heads, SwiGLU 4096, vocab 59392, random bf16
+weights), batch 1, prefix 2048 (1600 visual embeddings + 448 text tokens),
+block size K = 16, 512 output tokens, accepted draft lengths forced to a
+seeded censored-geometric schedule with mean 9.7.
+
+A step is one complete decode of the 512 output tokens: the sequence state is
+rolled back to the end of the prefill (the prefill itself is untimed, as in
+the paper's TPF accounting) and every round of the schedule runs as one CUDA
+graph (draft forward -> forcing -> verify forward -> accept/commit).  The
+metric is committed tokens per second; per-round latencies come from CUDA
+events.  The 876.6 MB of weights every forward streams exceed the 129 MB L2,
+so no flush is needed between steps.
+
+--impl reference times the float64 CPU oracle on this host's cores instead
+(one forced round per step).  Multi-GPU: replicas (one independent decode per
+rank, no collective on the data path).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import synth  # noqa: E402
+
+METRIC = "committed tokens/s (greedy self-speculative decode, 1 GB300 per rank)"
+UNIT = "tokens/s"
+
+
+def schedule_rounds(sched: np.ndarray, max_new: int) -> int:
+    n_out, r = 1, 0
+    while n_out < max_new:
+        n_out += int(sched[r]) + 2
+        r += 1
+    return r
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return d.get("hbm_gbs", 6800.0), d.get("bf16_tflops", 1900.0), "measured"
+    return 6800.0, 1900.0, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle sampling during the timed region."""
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.idx = gpu_index
+        self.proc = None
+        self.path = os.path.join("/tmp", f"gs_clocks_{os.getpid()}_{gpu_index}.csv")
+
+    def __enter__(self):
+        try:
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.idx), f"--query-gpu={self.Q}", "--format=csv,noheader",
+                 "-lms", "100"], stdout=self.f, stderr=subprocess.DEVNULL)
+            time.sleep(0.3)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+        return self
+
+    def __exit__(self, *a):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+            self.f.close()
+
+    def summary(self):
+        if self.proc is None or not os.path.exists(self.path):
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        mhz, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.path):
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                mhz.append(float(parts[1].split()[0]))
+                mx = float(parts[2].split()[0])
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not mhz:
+            return {"sm_mhz": None, "sm_max_mhz": mx, "reasons": ["no samples"]}
+        return {"sm_mhz": statistics.median(mhz), "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(mhz)}
+
+
+# ---------------------------------------------------------------------- GPU arm
+def gpu_arm(args, rank: int, world: int):
+    import torch
+    from paper_2609_26638_gb300 import gs
+    from paper_2609_26638_gb300.runtime import Engine
+
+    dev = torch.device("cuda", int(os.environ.get("LOCAL_RANK", 0)))
+    torch.cuda.set_device(dev)
+    wl = synth.WORKLOADS[args.workload]
+    cfg = wl.model
+    assert wl.batch == 1, "the bench decodes one sequence per rank"
+    K, max_new = wl.K, wl.max_new
+    prompt = wl.prompts()[0]
+    P = prompt.length
+    weights = synth.make_weights(cfg)
+    extra = K + 4
+    eng = Engine(cfg, weights, max_batch=1, max_ctx=P + max_new + extra + K + 2 + 64, max_K=K,
+                 max_prefill=2048, device=str(dev))
+    del weights
+    x0 = eng.prefill(0, prompt.vis, prompt.text, max_new + extra)
+
+    slots = torch.zeros(1, dtype=torch.int32, device=dev)
+    out_tok = torch.zeros((1, K + 2), dtype=torch.int32, device=dev)
+    out_cnt = torch.zeros(1, dtype=torch.int32, device=dev)
+    out_done = torch.zeros(1, dtype=torch.int32, device=dev)
+    torch.cuda.synchronize(dev)
+
+    # teacher: the greedy continuation, from natural rounds of the same shape
+    teacher_toks = [x0]
+    while True:
+        eng.round(slots, K, out_tok, out_cnt, out_done)
+        eng.stream.synchronize()
+        c = int(out_cnt.cpu()[0])
+        teacher_toks.extend(out_tok.cpu().numpy()[0, :c].tolist())
+        if int(out_done.cpu()[0]):
+            break
+    eng.check()
+    teacher = np.full(P + len(teacher_toks) + 8, -1, np.int32)
+    teacher[P:P + len(teacher_toks)] = teacher_toks
+    sched_all = wl.schedule()                       # [1, max_rounds]
+    R = schedule_rounds(sched_all[0], max_new)
+    sched = np.ascontiguousarray(sched_all[:, :R + 1])
+    t_dev = torch.from_numpy(teacher).to(dev)
+    s_dev = torch.from_numpy(sched).to(dev)
+    force = gs.gs_force(teacher=t_dev.data_ptr(), teacher_stride=teacher.shape[0],
+                        L_sched=s_dev.data_ptr(), L_stride=sched.shape[1])
+    ring_tok = torch.zeros((R, K + 2), dtype=torch.int32, device=dev)
+    ring_cnt = torch.zeros(R, dtype=torch.int32, device=dev)
+    torch.cuda.synchronize(dev)
+    stream = eng.stream
+
+    def one_decode(evs=None):
+        eng.restore(0, P, x0, 1, max_new, 0, 0)
+        for r in range(R):
+            if evs is not None:
+                evs[r][0].record(stream)
+            eng.round(slots, K, out_tok, out_cnt, out_done, force=force)
+            if evs is not None:
+                evs[r][1].record(stream)
+            with torch.cuda.stream(stream):
+                ring_tok[r].copy_(out_tok[0], non_blocking=True)
+                ring_cnt[r:r + 1].copy_(out_cnt, non_blocking=True)
+
+    for _ in range(args.warmup):
+        one_decode()
+    stream.synchronize()
+    launches_per_round = gs.gs_round_launches(eng.handle)
+
+    def barrier():
+        if world > 1:
+            import torch.distributed as dist
+            dist.barrier()
+        torch.cuda.synchronize(dev)
+
+    ev = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+           for _ in range(R)] for _ in range(args.steps)]
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    # GS_PROFILE_RANGE=1 marks the first timed decode as the profiler's capture
+    # range (ncu --profile-from-start off); it changes no work
+    prof = os.environ.get("GS_PROFILE_RANGE") == "1"
+    barrier()
+    with ClockSampler(dev.index) as clk:
+        t0.record(stream)
+        for s in range(args.steps):
+            if prof and s == 0:
+                torch.cuda.profiler.start()
+            one_decode(ev[s])
+            if prof and s == 0:
+                stream.synchronize()
+                torch.cuda.profiler.stop()
+        t1.record(stream)
+        stream.synchronize()
+    barrier()
+    elapsed = t0.elapsed_time(t1) / 1e3
+    round_ms = sorted(a.elapsed_time(b) for step in ev for (a, b) in step)
+    eng.check()
+
+    # every forced round committed exactly L + 2 tokens and the output is the greedy one
+    cnt = ring_cnt.cpu().numpy()
+    toks = ring_tok.cpu().numpy()
+    got = [x0]
+    for r in range(R):
+        got.extend(toks[r, :cnt[r]].tolist())
+    committed_per_decode = int(cnt.sum())
+    ok_sched = all(int(cnt[r]) == int(sched[0, r]) + 2 for r in range(R - 1))
+    ok_tokens = got == teacher_toks[:max_new]
+
+    # end to end: inputs from pinned host memory, outputs back to the host, every step
+    h_teacher = torch.from_numpy(teacher).pin_memory()
+    h_sched = torch.from_numpy(sched).pin_memory()
+    h_ring = torch.empty((R, K + 2), dtype=torch.int32).pin_memory()
+    h_cnt = torch.empty(R, dtype=torch.int32).pin_memory()
+    barrier()
+    e0 = time.perf_counter()
+    for s in range(args.steps):
+        with torch.cuda.stream(stream):
+            t_dev.copy_(h_teacher, non_blocking=True)
+            s_dev.copy_(h_sched, non_blocking=True)
+        one_decode()
+        with torch.cuda.stream(stream):
+            h_ring.copy_(ring_tok, non_blocking=True)
+            h_cnt.copy_(ring_cnt, non_blocking=True)
+        stream.synchronize()
+    barrier()
+    e_elapsed = time.perf_counter() - e0
+
+    # roofline: the LM-head GEMM (largest single kernel of the round), timed alone
+    roof = lm_head_roofline(eng, cfg, K, dev)
+    attn = attention_roofline(cfg, dev)
+    res = dict(elapsed=elapsed, e2e_elapsed=e_elapsed, tokens=committed_per_decode * args.steps,
+               round_ms=round_ms, rounds=R, launches_per_round=launches_per_round,
+               ok_sched=ok_sched, ok_tokens=ok_tokens, clocks=clk.summary(), roofline=roof,
+               attention=attn, h2d=int(teacher.nbytes + sched.nbytes),
+               d2h=int(R * (K + 2) * 4 + R * 4), P=P, K=K, max_new=max_new)
+    eng.close()
+    return res
+
+
+def _time_kernel(fn, stream, iters: int):
+    import torch
+    for _ in range(3):
+        fn()
+    a = torch.cuda.Event(enable_timing=True)
+    b = torch.cuda.Event(enable_timing=True)
+    a.record(stream)
+    for _ in range(iters):
+        fn()
+    b.record(stream)
+    b.synchronize()
+    return a.elapsed_time(b) / 1e3 / iters
+
+
+def lm_head_roofline(eng, cfg, K, dev):
+    """LM-head GEMM + argmax at the decode shape (17 rows x 59392 x 1024), the
+    same kernel instantiation the round launches, over rotating weight copies
+    (3 x 121.6 MB > L2)."""
+    import torch
+    from paper_2609_26638_gb300 import gs
+    hbm, _, src = load_peaks()
+    M, N, Kd = K + 1, cfg.vocab, cfg.d_model
+    g = torch.Generator(device=dev).manual_seed(0)
+    ws = [(0.02 * torch.randn(N, Kd, device=dev, generator=g)).bfloat16() for _ in range(3)]
+    x = torch.randn(M, Kd, device=dev, generator=g).bfloat16()
+    keys = torch.zeros(M, dtype=torch.int64, device=dev)
+    sb = gs.gs_linear_scratch_bytes(M, N, 1)
+    scratch = torch.zeros(sb, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    it = [0]
+
+    def fn():
+        w = ws[it[0] % 3]
+        it[0] += 1
+        gs.gs_linear(x.data_ptr(), w.data_ptr(), keys.data_ptr(), M, N, Kd, gs.EPI_ARGMAX, 1,
+                     scratch.data_ptr(), sb, stream.cuda_stream)
+
+    t = _time_kernel(fn, stream, 30)
+    algo = N * Kd * 2 + M * Kd * 2 + M * 8
+    achieved = algo / t / 1e9
+    return {"kernel": "gemm_tc_kernel<32, argmax> (LM head 17x59392x1024)", "bound": "hbm",
+            "achieved": round(achieved, 1), "peak": hbm, "unit": "GB/s",
+            "frac": round(achieved / hbm, 4), "peak_source": src, "algorithmic_bytes": algo,
+            "us_per_launch": round(t * 1e6, 2), "traffic": None}
+
+
+def attention_roofline(cfg, dev):
+    """Hybrid-mask draft attention at the serving shape (32 sequences, prefix
+    U[1024, 6144] -> mean ~3600, K = 16), the kernel alone over a paged pool
+    larger than L2."""
+    import torch
+    from paper_2609_26638_gb300 import gs
+    hbm, _, src = load_peaks()
+    rng = np.random.default_rng(5)
+    B, K = 32, 16
+    W = K + 1
+    Hq, Hkv = cfg.n_heads, cfg.n_kv_heads
+    ns = rng.integers(1024, 6145, size=B).astype(np.int32)
+    pages_per = [math.ceil((n + W + 1) / 64) for n in ns]
+    pt_stride = max(pages_per)
+    n_pages = sum(pages_per)
+    perm = rng.permutation(n_pages)
+    pt = np.full((B, pt_stride), -1, np.int32)
+    o = 0
+    for b in range(B):
+        pt[b, :pages_per[b]] = perm[o:o + pages_per[b]]
+        o += pages_per[b]
+    kv = torch.randn(n_pages * 2 * Hkv * 64 * 64, device=dev).bfloat16()
+    q = torch.randn(B * W * Hq * 64, device=dev).bfloat16()
+    out = torch.zeros_like(q)
+    ptd = torch.from_numpy(pt).to(dev)
+    nd = torch.from_numpy(ns).to(dev)
+    sp = max(1, math.ceil(pt_stride * B * Hkv / 304))
+    sb = gs.gs_attention_scratch_bytes(B, W, Hq, Hkv, pt_stride, sp)
+    scratch = torch.zeros(sb, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def fn():
+        gs.gs_attention(0, q.data_ptr(), kv.data_ptr(), n_pages, ptd.data_ptr(), pt_stride,
+                        nd.data_ptr(), B, W, Hq, Hkv, out.data_ptr(), scratch.data_ptr(), sb, sp,
+                        stream.cuda_stream)
+
+    t = _time_kernel(fn, stream, 20)
+    keys = int(sum(int(n) + W for n in ns))
+    algo = keys * Hkv * 64 * 2 * 2 + 2 * B * W * Hq * 64 * 2
+    achieved = algo / t / 1e9
+    return {"kernel": "attn_paged_kernel (draft, 32 seqs, ctx ~3.6k, K=16)", "bound": "hbm",
+            "achieved": round(achieved, 1), "peak": hbm, "unit": "GB/s",
+            "frac": round(achieved / hbm, 4), "kv_bytes": algo, "us_per_launch": round(t * 1e6, 2)}
+
+
+# ---------------------------------------------------------------------- oracle arm
+def oracle_sample(wl, n_rounds: int, warmup: int, budget_s: float):
+    """Forced self-speculative rounds of the float64 oracle on this host's cores.
+
+    The oracle's own greedy AR continuation is the forcing teacher; the sample
+    is the first rounds of the workload's decode (prefill and teacher untimed).
+    Returns (per-round seconds, committed tokens per timed round).
+    """
+    from oracle import decode as od
+    from oracle.model import Decoder
+    cfg = wl.model
+    K = wl.K
+    prompt = wl.prompts()[0]
+    dec = Decoder(cfg, synth.make_weights(cfg))
+    sched = wl.schedule()[0]
+    total = warmup + n_rounds
+    need = int(sum(int(sched[r]) + 2 for r in range(total))) + K + 4
+    cap = prompt.length + need + K + 8
+    ar_state = od.prefill(dec, prompt.vis, prompt.text, cap, need)
+    st = od.SeqState(cache=ar_state.cache.copy(), x0=ar_state.x0, out=[ar_state.x0],
+                     max_new=wl.max_new)
+    od.ar_decode(dec, ar_state)
+    P = prompt.length
+    teacher = np.full(P + len(ar_state.out) + 8, -1, np.int64)
+    teacher[P:P + len(ar_state.out)] = ar_state.out
+    times, counts = [], []
+    t_start = time.perf_counter()
+    for r in range(total):
+        t0 = time.perf_counter()
+        res = od.self_spec_round(dec, st, K, teacher, int(sched[r]))
+        dt = time.perf_counter() - t0
+        if r >= warmup:
+            times.append(dt)
+            counts.append(len(res.committed))
+            if time.perf_counter() - t_start > budget_s and len(times) >= 1:
+                break
+        if st.done:
+            break
+    return times, counts
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="gpu", choices=["gpu", "reference"])
+    ap.add_argument("--workload", default="glm_b1")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    wl = synth.WORKLOADS[args.workload]
+    config = {"workload": f"{wl.name}: GLM-OCR-scale synthetic decoder L24 d1024 H16/8 F4096 V59392, "
+                          f"batch 1, prefix {wl.prefix_min} (1600 visual + 448 text), K={wl.K}, "
+                          f"{wl.max_new} output tokens, forced acceptance censored geometric mean 9.7",
+              "model": "synthetic random-init bf16 (seed 0)", "global_batch": wl.batch * max(world, 1),
+              "K": wl.K, "max_new": wl.max_new,
+              "l2": "inputs larger than L2: 876.6 MB of weights streamed per forward",
+              "parallelism": f"replicas x{max(world, 1)}"}
+
+    if args.impl == "reference":
+        if rank != 0:
+            return
+        t0 = time.perf_counter()
+        times, counts = oracle_sample(wl, args.steps, args.warmup, budget_s=240.0)
+        value = sum(counts) / sum(times)
+        cores = os.cpu_count()
+        sample = (f"{len(times)} forced rounds of the {wl.name} decode (after {args.warmup} warm-up "
+                  f"rounds), float64 oracle, prefill and teacher untimed")
+        line = {"impl": "reference", "metric": METRIC, "value": round(value, 3), "unit": UNIT,
+                "n_gpus": args.gpus, "steps": len(times), "warmup": args.warmup,
+                "ms_per_step": round(1e3 * statistics.mean(times), 2), "higher_is_better": True,
+                "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+                "config": config,
+                "cpu_baseline": {"value": round(value, 3), "unit": UNIT, "cores": cores,
+                                 "kind": "oracle", "sample": sample},
+                "e2e": {"value": round(value, 3), "unit": UNIT, "h2d_bytes_per_step": 0,
+                        "d2h_bytes_per_step": 0},
+                "wall_s": round(time.perf_counter() - t0, 1)}
+        print(json.dumps(line))
+        return
+
+    import torch
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", int(os.environ["LOCAL_RANK"])))
+    res = gpu_arm(args, rank, world)
+    el = res["elapsed"]
+    ee = res["e2e_elapsed"]
+    if world > 1:
+        import torch.distributed as dist
+        t = torch.tensor([el, ee], dtype=torch.float64, device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        el, ee = float(t[0]), float(t[1])
+    tokens_all = res["tokens"] * max(world, 1)
+    value = tokens_all / el
+    rms = res["round_ms"]
+    line = {"metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": max(world, 1),
+            "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": round(1e3 * el / args.steps, 3), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": config,
+            "round_p50_ms": round(rms[len(rms) // 2], 4),
+            "round_p90_ms": round(rms[int(len(rms) * 0.9)], 4),
+            "rounds_per_step": res["rounds"],
+            "committed_per_round": round(res["tokens"] / (args.steps * res["rounds"]), 3),
+            "tpf": round(res["tokens"] / (args.steps * res["rounds"] * 2), 3),
+            "forced_schedule_hit": res["ok_sched"], "tokens_match_greedy": res["ok_tokens"],
+            "gpu_launches": res["launches_per_round"] * res["rounds"] * args.steps
+            + args.steps,
+            "e2e": {"value": round(tokens_all / ee, 1), "unit": UNIT,
+                    "h2d_bytes_per_step": res["h2d"], "d2h_bytes_per_step": res["d2h"]},
+            "clocks": res["clocks"], "roofline": res["roofline"],
+            "attention_roofline": res["attention"]}
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        times, counts = oracle_sample(synth.WORKLOADS[args.workload], 6, 1, budget_s=25.0)
+        line["cpu_baseline"] = {
+            "value": round(sum(counts) / sum(times), 3), "unit": UNIT, "cores": os.cpu_count(),
+            "kind": "oracle",
+            "sample": f"{len(times)} forced rounds (after 1 warm-up) of the same decode, float64 "
+                      f"oracle with numpy/OpenBLAS threads on all host cores"}
+    if rank == 0:
+        print(json.dumps(line))
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

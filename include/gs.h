@@ -162,15 +162,23 @@ int gs_prefill(gs_handle *h, int slot, const void *vis_emb, int n_vis, const int
 int gs_round(gs_handle *h, const int32_t *slots, int n_seq, int K, int rule, const gs_force *force,
              int32_t *out_tok, int32_t *out_cnt, int32_t *out_done, const gs_debug *dbg);
 
-/* Overwrite a sequence's boundary token and output count (resume/checkpoint
- * of the per-sequence state: the cache is described by its length alone).
- *   seq_len   new cached length, 1 <= seq_len <= current cached length (rollback only)
- *   x0        boundary token, n_out committed-token count (x0 included)
+/* Overwrite a sequence's per-slot state (resume/checkpoint: with the KV pages,
+ * which keep their contents, the state is the cached length, the boundary
+ * token, the output count and cap, the done flag and the round counter that
+ * indexes a forcing schedule).  Rolling the cached length back to a value the
+ * cache held before (e.g. the prefix length after a prefill) replays a decode.
+ *   seq_len   1 <= seq_len and seq_len + max_K + 2 <= the slot's reservation
+ *   x0        boundary token in [0, vocab); n_out >= 1 committed tokens (x0 included)
+ *   max_new   output cap (>= n_out); done 0/1; rounds >= 0
  * Host values; enqueued on the stream.  Errors: GS_ERR_INVALID_ARG. */
-int gs_seq_restore(gs_handle *h, int slot, int seq_len, int x0, int n_out, int done);
+int gs_seq_restore(gs_handle *h, int slot, int seq_len, int x0, int n_out, int max_new, int done,
+                   int rounds);
 
 /* Read one slot's state (synchronises the stream).  Any out pointer may be NULL. */
 int gs_seq_state(gs_handle *h, int slot, int *seq_len, int *x0, int *n_out, int *done, int *rounds);
+
+/* Number of kernel launches the most recent gs_round enqueued (or captured). */
+int gs_round_launches(gs_handle *h);
 
 /* Free the slot's KV pages (host bookkeeping only). */
 int gs_release(gs_handle *h, int slot);

@@ -143,6 +143,8 @@ struct gs_handle {
                      const void*, const void*, const void*>
       GraphKey;
   std::map<GraphKey, cudaGraphExec_t> graphs;
+  int launches = 0;             // kernel launches counted while enqueueing
+  int last_round_launches = 0;
 };
 
 namespace {
@@ -298,6 +300,7 @@ int run_gemm(gs_handle* h, const CUtensorMap& tw, int weight_rows, const CUtenso
   }
   GS_CUDA(h, launch_gemm(p.bn, epi, tw, tx_set[bn_index(p.bn)], a, p.feat_tiles, p.tok_tiles,
                          h->stream));
+  ++h->launches;
   return GS_OK;
 }
 
@@ -307,6 +310,7 @@ int run_rmsnorm(gs_handle* h, const float* x, const __nv_bfloat16* g, __nv_bfloa
   rmsnorm_kernel<<<cdiv(T, rows_per_block), 32 * rows_per_block, 0, h->stream>>>(
       x, g, y, T, h->cfg.d_model, h->cfg.rms_eps, reset);
   GS_CUDA(h, cudaGetLastError());
+  ++h->launches;
   return GS_OK;
 }
 
@@ -346,6 +350,7 @@ int run_attention(gs_handle* h, int layer, int T, const AttnLaunch& L) {
   const int threads = (L.r_max / 16) * 32;
   attn_paged_kernel<<<grid, threads, attn_smem_bytes(L.r_max), h->stream>>>(h->tm_kv, a);
   GS_CUDA(h, cudaGetLastError());
+  ++h->launches;
   return GS_OK;
 }
 
@@ -360,6 +365,7 @@ int forward(gs_handle* h, int T, const int32_t* tok, const __nv_bfloat16* vis, i
   embed_kernel<<<T, 128, 0, h->stream>>>(tok, h->embed, vis, n_vis, T, d, c.vocab, h->hbuf,
                                          h->err_word);
   GS_CUDA(h, cudaGetLastError());
+  ++h->launches;
   const size_t layer_kv = static_cast<size_t>(h->n_pages) * 2 * c.n_kv_heads * 64 * 64;
   int rc;
   for (int l = 0; l < c.n_layers; ++l) {
@@ -385,6 +391,7 @@ int forward(gs_handle* h, int T, const int32_t* tok, const __nv_bfloat16* vis, i
     const int warps = T * (c.n_heads + 2 * c.n_kv_heads);
     rope_kv_kernel<<<cdiv(warps, 8), 256, 0, h->stream>>>(r);
     GS_CUDA(h, cudaGetLastError());
+    ++h->launches;
     if ((rc = run_attention(h, l, T, AL))) return rc;
     if ((rc = run_gemm(h, h->tm_o[l], d, h->tm_ao, HD, T, kEpiResidF32, h->hbuf, d, d, nullptr,
                        decode)))
@@ -444,13 +451,16 @@ int enqueue_round(gs_handle* h, const int32_t* slots, int n_seq, int K, const gs
   AL.blk_active = h->blk_active;
   AL.fixed_slot = -1;
 
+  h->launches = 0;
   window_draft_kernel<<<nb, 128, 0, h->stream>>>(w);
   GS_CUDA(h, cudaGetLastError());
+  ++h->launches;
   int rc = forward(h, T, h->tok, nullptr, 0, AL, 0, T, h->packed_d,
                    dbg ? dbg->draft_logits : nullptr, true);
   if (rc) return rc;
   window_verify_kernel<<<nb, 128, 0, h->stream>>>(w);
   GS_CUDA(h, cudaGetLastError());
+  ++h->launches;
   rc = forward(h, T, h->tok, nullptr, 0, AL, 0, T, h->packed_v, dbg ? dbg->verify_logits : nullptr,
                true);
   if (rc) return rc;
@@ -469,13 +479,17 @@ int enqueue_round(gs_handle* h, const int32_t* slots, int n_seq, int K, const gs
   ac.out_done = out_done;
   accept_commit_kernel<<<cdiv(n_seq, 64), 64, 0, h->stream>>>(ac);
   GS_CUDA(h, cudaGetLastError());
+  ++h->launches;
   if (dbg) {
     if (dbg->draft_tok) copy_i32_kernel<<<nb, 128, 0, h->stream>>>(h->draft_tok, dbg->draft_tok, T);
     if (dbg->verify_in) copy_i32_kernel<<<nb, 128, 0, h->stream>>>(h->verify_in, dbg->verify_in, T);
     if (dbg->verify_tok)
       copy_i32_kernel<<<nb, 128, 0, h->stream>>>(h->verify_tok, dbg->verify_tok, T);
     GS_CUDA(h, cudaGetLastError());
+    h->launches += (dbg->draft_tok != nullptr) + (dbg->verify_in != nullptr) +
+                   (dbg->verify_tok != nullptr);
   }
+  h->last_round_launches = h->launches;
   return GS_OK;
 }
 
@@ -717,18 +731,26 @@ int gs_round(gs_handle* h, const int32_t* slots, int n_seq, int K, int rule, con
   return GS_OK;
 }
 
-int gs_seq_restore(gs_handle* h, int slot, int seq_len, int x0, int n_out, int done) {
+int gs_seq_restore(gs_handle* h, int slot, int seq_len, int x0, int n_out, int max_new, int done,
+                   int rounds) {
   if (!h) return GS_ERR_INVALID_ARG;
   const gs_config& c = h->cfg;
   if (slot < 0 || slot >= c.max_batch || h->slot_reserved[slot] == 0)
     return fail(h, GS_ERR_INVALID_ARG, "slot out of range or not prefilled");
   if (seq_len < 1 || seq_len + c.max_K + 2 > h->slot_reserved[slot])
     return fail(h, GS_ERR_INVALID_ARG, "seq_len outside the slot's reservation");
-  if (x0 < 0 || x0 >= c.vocab || n_out < 1) return fail(h, GS_ERR_INVALID_ARG, "bad x0 / n_out");
-  seq_restore_kernel<<<1, 32, 0, h->stream>>>(h->st, slot, seq_len, x0, n_out, done ? 1 : 0);
+  if (x0 < 0 || x0 >= c.vocab || n_out < 1 || max_new < n_out || rounds < 0)
+    return fail(h, GS_ERR_INVALID_ARG, "bad x0 / n_out / max_new / rounds");
+  // the cap must keep every reachable round inside the reservation
+  if (static_cast<long long>(seq_len) + (max_new - n_out) + c.max_K + 2 > h->slot_reserved[slot])
+    return fail(h, GS_ERR_INVALID_ARG, "max_new reaches past the slot's reservation");
+  seq_restore_kernel<<<1, 32, 0, h->stream>>>(h->st, slot, seq_len, x0, n_out, max_new,
+                                              done ? 1 : 0, rounds);
   GS_CUDA(h, cudaGetLastError());
   return GS_OK;
 }
+
+int gs_round_launches(gs_handle* h) { return h ? h->last_round_launches : 0; }
 
 int gs_seq_state(gs_handle* h, int slot, int* seq_len, int* x0, int* n_out, int* done, int* rounds) {
   if (!h) return GS_ERR_INVALID_ARG;

@@ -159,12 +159,14 @@ __global__ void prefill_finish_kernel(const unsigned long long* packed, SeqState
 }
 
 __global__ void seq_restore_kernel(SeqStateDev st, int slot, int seq_len, int x0, int n_out,
-                                   int done) {
+                                   int max_new, int done, int rounds) {
   if (threadIdx.x != 0 || blockIdx.x != 0) return;
   st.seq_len[slot] = seq_len;
   st.x0[slot] = x0;
   st.n_out[slot] = n_out;
+  st.max_new[slot] = max_new;
   st.done[slot] = done;
+  st.rounds[slot] = rounds;
 }
 
 // Prefill chunk positions: token t at slot p0 + t, causal limit p0 + t.

@@ -77,7 +77,8 @@ def _load():
         "gs_prefill": (i32, [vp, i32, vp, i32, vp, i32, i32, vp]),
         "gs_round": (i32, [vp, vp, i32, i32, i32, ctypes.POINTER(gs_force), vp, vp, vp,
                            ctypes.POINTER(gs_debug)]),
-        "gs_seq_restore": (i32, [vp, i32, i32, i32, i32, i32]),
+        "gs_seq_restore": (i32, [vp, i32, i32, i32, i32, i32, i32, i32]),
+        "gs_round_launches": (i32, [vp]),
         "gs_seq_state": (i32, [vp, i32] + [ctypes.POINTER(i32)] * 5),
         "gs_release": (i32, [vp, i32]),
         "gs_sync_check": (i32, [vp]),
@@ -96,7 +97,7 @@ def _load():
 
 _lib = _load()
 EXPORTED = ("gs_workspace_bytes", "gs_create", "gs_destroy", "gs_last_error", "gs_prefill",
-            "gs_round", "gs_seq_restore", "gs_seq_state", "gs_release", "gs_sync_check",
+            "gs_round", "gs_seq_restore", "gs_round_launches", "gs_seq_state", "gs_release", "gs_sync_check",
             "gs_attention_scratch_bytes", "gs_attention", "gs_linear_scratch_bytes", "gs_linear")
 
 
@@ -146,8 +147,13 @@ def gs_round(h, slots_ptr: int, n_seq: int, K: int, rule: int, force: gs_force |
                             ctypes.byref(dbg) if dbg is not None else None))
 
 
-def gs_seq_restore(h, slot: int, seq_len: int, x0: int, n_out: int, done: int) -> None:
-    _check(h, _lib.gs_seq_restore(h, slot, seq_len, x0, n_out, done))
+def gs_seq_restore(h, slot: int, seq_len: int, x0: int, n_out: int, max_new: int, done: int,
+                   rounds: int) -> None:
+    _check(h, _lib.gs_seq_restore(h, slot, seq_len, x0, n_out, max_new, done, rounds))
+
+
+def gs_round_launches(h) -> int:
+    return int(_lib.gs_round_launches(h))
 
 
 def gs_seq_state(h, slot: int) -> dict:

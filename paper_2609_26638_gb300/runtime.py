@@ -94,8 +94,9 @@ class Engine:
         gs.gs_round(self.handle, slots.data_ptr(), slots.shape[0], K, gs.GS_ACCEPT_GREEDY, force,
                     out_tok.data_ptr(), out_cnt.data_ptr(), out_done.data_ptr(), dbg)
 
-    def restore(self, slot: int, seq_len: int, x0: int, n_out: int, done: int = 0) -> None:
-        gs.gs_seq_restore(self.handle, slot, seq_len, x0, n_out, done)
+    def restore(self, slot: int, seq_len: int, x0: int, n_out: int, max_new: int, done: int = 0,
+                rounds: int = 0) -> None:
+        gs.gs_seq_restore(self.handle, slot, seq_len, x0, n_out, max_new, done, rounds)
 
     def state(self, slot: int) -> dict:
         return gs.gs_seq_state(self.handle, slot)

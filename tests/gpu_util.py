@@ -66,7 +66,7 @@ def lockstep(eng, dec, prompt, K: int, max_new: int, max_rounds: int = 1 << 30, 
     if x0 != st.x0:
         assert st.prefill_gap < NEAR_TIE, ("prefill x0 differs", x0, st.x0, st.prefill_gap)
         stats.near_tie_flips += 1
-        eng.restore(slot, st.n, st.x0, 1, int(st.done))
+        eng.restore(slot, st.n, st.x0, 1, max_new, int(st.done))
 
     slots = torch.tensor([slot], dtype=torch.int32, device=dev)
     out_tok = torch.zeros((1, K + 2), dtype=torch.int32, device=dev)
@@ -137,5 +137,5 @@ def lockstep(eng, dec, prompt, K: int, max_new: int, max_rounds: int = 1 << 30, 
             stats.resyncs += 1
             text = np.concatenate([prompt.text, np.asarray(st.out[:-1], dtype=np.int32)])
             eng.prefill(slot, prompt.vis, text, max_new)
-            eng.restore(slot, st.n, st.x0, len(st.out), int(st.done))
+            eng.restore(slot, st.n, st.x0, len(st.out), max_new, int(st.done))
     return st, stats
