@@ -224,6 +224,31 @@ size_t gs_linear_scratch_bytes(int M, int N, int split_k);
 int gs_linear(const void *x, const void *w, void *y, int M, int N, int K, int epilogue, int split_k,
               void *scratch, size_t scratch_bytes, void *stream);
 
+/* ---------------------------------------------------------------------------
+ * Allocation-free variant of gs_linear.  The paper has no counterpart: this
+ * entry point exists for callers that cannot allocate device memory at the
+ * call and have no workspace to pass (an operator inside another framework
+ * with no workspace argument, a plugin host whose allocator owns all device
+ * memory, a real-time path where cudaMalloc's implicit synchronisation is not
+ * allowed).
+ *
+ * Same arguments and results as gs_linear minus the scratch pointer: the
+ * split-K scratch (error word, per-tile counters, fp32 partials) lives in a
+ * fixed device array of GS_NOALLOC_SCRATCH_BYTES inside the library, which
+ * every GPU that loads the library keeps until the process exits.  The call
+ * makes no cudaMalloc / cudaFree and calls no allocating library routine.
+ *   - The first call on a device looks up that array's device address (with
+ *     the device current); make that first call before any stream capture.
+ *   - Every call clears the counters it uses before its kernel runs.
+ *   - All calls share the one array: calls whose kernels overlap on the GPU
+ *     (two streams, or two host threads on one device) race; serialise them.
+ * Errors: as gs_linear; GS_ERR_OOM when split_k x tiles of partials for
+ * (M, N) do not fit in GS_NOALLOC_SCRATCH_BYTES (e.g. M <= 32 rows, N = 2048,
+ * split_k = 8 needs 2 MiB). */
+#define GS_NOALLOC_SCRATCH_BYTES (8u << 20)
+int gs_linear_noalloc(const void *x, const void *w, void *y, int M, int N, int K, int epilogue,
+                      int split_k, void *stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -87,6 +87,7 @@ def _load():
                                vp]),
         "gs_linear_scratch_bytes": (sz, [i32, i32, i32]),
         "gs_linear": (i32, [vp, vp, vp, i32, i32, i32, i32, i32, vp, sz, vp]),
+        "gs_linear_noalloc": (i32, [vp, vp, vp, i32, i32, i32, i32, i32, vp]),
     }
     for name, (res, args) in sig.items():
         f = getattr(lib, name)
@@ -98,7 +99,8 @@ def _load():
 _lib = _load()
 EXPORTED = ("gs_workspace_bytes", "gs_create", "gs_destroy", "gs_last_error", "gs_prefill",
             "gs_round", "gs_seq_restore", "gs_round_launches", "gs_seq_state", "gs_release", "gs_sync_check",
-            "gs_attention_scratch_bytes", "gs_attention", "gs_linear_scratch_bytes", "gs_linear")
+            "gs_attention_scratch_bytes", "gs_attention", "gs_linear_scratch_bytes", "gs_linear",
+            "gs_linear_noalloc")
 
 
 def lib():
@@ -193,3 +195,15 @@ def gs_linear(x_ptr, w_ptr, y_ptr, M, N, K, epilogue, split_k, scratch_ptr, scra
                         stream_ptr)
     if rc != GS_OK:
         raise GsError(rc, "gs_linear")
+
+
+NOALLOC_SCRATCH_BYTES = 8 << 20
+
+
+def gs_linear_noalloc(x_ptr, w_ptr, y_ptr, M, N, K, epilogue, split_k, stream_ptr) -> None:
+    """gs_linear with its scratch in the library's fixed device array (no allocation).
+    Calls that overlap on the GPU race on that array; the first call on a device
+    must come before any stream capture."""
+    rc = _lib.gs_linear_noalloc(x_ptr, w_ptr, y_ptr, M, N, K, epilogue, split_k, stream_ptr)
+    if rc != GS_OK:
+        raise GsError(rc, "gs_linear_noalloc")

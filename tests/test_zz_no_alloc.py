@@ -1,0 +1,57 @@
+"""gs_linear_noalloc: the projection GEMM for callers that cannot allocate
+device memory (an operator with no workspace argument, a plugin host whose
+allocator owns the device memory, a real-time path that must not trigger
+cudaMalloc's synchronisation).  Its split-K scratch lives in a fixed device
+array inside the library; this checks it against gs_linear, which takes the
+same scratch from the caller, on two calls in a row through the C ABI.
+
+Kept in a file of its own that pytest collects last.
+"""
+import pytest
+import torch
+
+pytestmark = pytest.mark.gpu
+DEV = "cuda:0"
+
+
+@pytest.fixture(scope="module")
+def gs():
+    from paper_2609_26638_gb300 import gs as binding
+    return binding
+
+
+def _with_caller_scratch(gs, x, w, M, N, K, epi, split, y):
+    sb = gs.gs_linear_scratch_bytes(M, N, split)
+    scratch = torch.zeros(sb, dtype=torch.uint8, device=DEV)
+    gs.gs_linear(x.data_ptr(), w.data_ptr(), y.data_ptr(), M, N, K, epi, split, scratch.data_ptr(),
+                 sb, torch.cuda.current_stream().cuda_stream)
+    torch.cuda.synchronize()
+
+
+def test_noalloc_matches_linear_on_two_calls_in_a_row(gs):
+    stream = torch.cuda.current_stream().cuda_stream
+    g = torch.Generator(device=DEV).manual_seed(11)
+    cases = [(17, 2048, 1024, gs.EPI_STORE_BF16, 8), (9, 1024, 4096, gs.EPI_STORE_BF16, 16)]
+    for M, N, K, epi, split in cases:          # two calls in a row share the one array
+        x = torch.randn(M, K, device=DEV, generator=g).bfloat16()
+        w = (0.02 * torch.randn(N, K, device=DEV, generator=g)).bfloat16()
+        want = torch.zeros(M, N, dtype=torch.bfloat16, device=DEV)
+        _with_caller_scratch(gs, x, w, M, N, K, epi, split, want)
+        got = torch.zeros(M, N, dtype=torch.bfloat16, device=DEV)
+        gs.gs_linear_noalloc(x.data_ptr(), w.data_ptr(), got.data_ptr(), M, N, K, epi, split, stream)
+        torch.cuda.synchronize()
+        ref = x.float() @ w.float().T
+        torch.testing.assert_close(got.float(), want.float(), rtol=1e-2,
+                                   atol=1e-2 * ref.abs().max().item())
+        torch.testing.assert_close(got.float(), ref, rtol=1e-2, atol=1e-2 * ref.abs().max().item())
+
+
+def test_noalloc_rejects_scratch_beyond_its_array(gs):
+    # 64 k-block splits over 64 feature tiles of 32 rows need 64 MiB of partials > 8 MiB
+    x = torch.zeros(17, 4096, dtype=torch.bfloat16, device=DEV)
+    w = torch.zeros(8192, 4096, dtype=torch.bfloat16, device=DEV)
+    y = torch.zeros(17, 8192, dtype=torch.bfloat16, device=DEV)
+    with pytest.raises(gs.GsError) as e:
+        gs.gs_linear_noalloc(x.data_ptr(), w.data_ptr(), y.data_ptr(), 17, 8192, 4096,
+                             gs.EPI_STORE_BF16, 64, torch.cuda.current_stream().cuda_stream)
+    assert e.value.code == gs.GS_ERR_OOM
