@@ -48,8 +48,12 @@ struct AttnArgs {
 constexpr int kAttnStages = 4;
 constexpr int kAttnPageBytes = 64 * 128;  // 64 tokens x 64 bf16
 
+// Rows of Q staged in shared memory: at least 64 (four warps), so the split
+// merge always has 128 threads.
+__host__ __device__ inline int attn_rows_alloc(int r_max) { return r_max < 64 ? 64 : r_max; }
+__host__ __device__ inline int attn_threads(int r_max) { return attn_rows_alloc(r_max) / 16 * 32; }
 __host__ __device__ inline int attn_smem_bytes(int r_max) {
-  return 1024 + kAttnStages * 2 * kAttnPageBytes + r_max * 128 + 64 /*barriers*/ + 64;
+  return 1024 + kAttnStages * 2 * kAttnPageBytes + attn_rows_alloc(r_max) * 128 + 64 + 64;
 }
 
 __device__ __forceinline__ uint32_t sw128(int row, int chunk) {
@@ -92,13 +96,17 @@ __global__ void __launch_bounds__(512)
   uint8_t* sK = smem;                                     // [stages][64][128 B]
   uint8_t* sV = smem + kAttnStages * kAttnPageBytes;      // [stages][64][128 B]
   uint8_t* sQ = smem + 2 * kAttnStages * kAttnPageBytes;  // [r_max][128 B]
-  uint64_t* full = reinterpret_cast<uint64_t*>(sQ + a.r_max * 128);
+  uint64_t* full = reinterpret_cast<uint64_t*>(sQ + attn_rows_alloc(a.r_max) * 128);
   __shared__ int s_maxlim;
   __shared__ int s_last;
 
   const int c = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int nthreads = blockDim.x;
+  // Before griddepcontrol.wait this kernel reads only what the kernel right
+  // before it (RoPE + KV write) does not write: the window descriptors (key
+  // limits, block slots), the page table, and cache pages wholly before the
+  // current window.
   if (a.blk_active != nullptr && a.blk_active[b] == 0) return;
   const int tok0 = b * a.QB;
   const int ntok = min(a.QB, a.T - tok0);
@@ -134,6 +142,8 @@ __global__ void __launch_bounds__(512)
     fence_mbar_init();
   }
   __syncthreads();
+  // pages wholly before the block's first slot hold committed states only
+  const int safe_pages = a.blk_slot ? a.lim[tok0] / 64 : 0;
   const uint64_t pol = l2_policy_evict_first();
   auto issue = [&](int i) {
     const int s = i % kAttnStages;
@@ -149,8 +159,14 @@ __global__ void __launch_bounds__(512)
     tma_load_2d(smem_u32(sV + s * kAttnPageBytes), &tmKV, 0,
                 static_cast<int>(row + (a.Hkv + h) * 64), fb, pol);
   };
+  int issued = 0;
   if (threadIdx.x == 0) {
-    for (int i = 0; i < min(np, kAttnStages); ++i) issue(i);
+    while (issued < min(np, kAttnStages) && p_begin + issued < safe_pages) issue(issued++);
+  }
+  pdl_wait();
+  pdl_trigger();
+  if (threadIdx.x == 0) {
+    while (issued < min(np, kAttnStages)) issue(issued++);
   }
 
   // Q rows -> swizzled smem (zero rows past R)
@@ -330,26 +346,59 @@ __global__ void __launch_bounds__(512)
   __syncthreads();
   if (!s_last) return;
   __threadfence();
+  // Merge: stage (m, l) of every split for a group of rows in shared memory,
+  // turn them into weights exp2(m_s - M) / L per row, then each thread sums
+  // four output dims over the splits in order 0..S-1.  With one split holding
+  // all of a row's keys this reduces to O * (1 / l), the direct path's result.
   const float* po0 = a.part_o + (bh * a.max_splits * a.r_max) * 64;
   const float* pml0 = a.part_ml + (bh * a.max_splits * a.r_max) * 2;
-  for (int idx = threadIdx.x; idx < R * 32; idx += nthreads) {
-    const int r = idx >> 5, d2 = (idx & 31) * 2;
-    float M = -INFINITY;
-    for (int s = 0; s < nsplit; ++s) M = fmaxf(M, __ldcg(pml0 + (s * a.r_max + r) * 2));
-    float ox = 0.f, oy = 0.f, L = 0.f;
-    for (int s = 0; s < nsplit; ++s) {
-      const float ms = __ldcg(pml0 + (s * a.r_max + r) * 2);
-      const float w = (ms == -INFINITY) ? 0.f : exp2f(ms - M);
-      L += w * __ldcg(pml0 + (s * a.r_max + r) * 2 + 1);
-      const float2 v = __ldcg(reinterpret_cast<const float2*>(po0 + (s * a.r_max + r) * 64 + d2));
-      ox += w * v.x;
-      oy += w * v.y;
+  float* sm_m = reinterpret_cast<float*>(sK);                 // [nsplit][RG]
+  float* sm_w = sm_m + (kAttnStages * 2 * kAttnPageBytes / 4) / 2;   // [nsplit][RG]
+  const int cap = (kAttnStages * 2 * kAttnPageBytes / 4) / 2;
+  const int RG = min(R, cap / nsplit);
+  for (int rg0 = 0; rg0 < R; rg0 += RG) {
+    const int nr = min(RG, R - rg0);
+    for (int idx = threadIdx.x; idx < nsplit * nr; idx += nthreads) {
+      const int sp = idx / nr, rr = idx % nr;
+      const float2 ml = __ldcg(reinterpret_cast<const float2*>(pml0 + (sp * a.r_max + rg0 + rr) * 2));
+      sm_m[sp * RG + rr] = ml.x;
+      sm_w[sp * RG + rr] = ml.y;
     }
-    const float inv = 1.0f / L;
-    const int t = tok0 + r / a.G;
-    const int hq = h * a.G + r % a.G;
-    *reinterpret_cast<__nv_bfloat162*>(a.out + (static_cast<size_t>(t) * a.Hq + hq) * 64 + d2) =
-        __floats2bfloat162_rn(ox * inv, oy * inv);
+    __syncthreads();
+    for (int rr = threadIdx.x; rr < nr; rr += nthreads) {
+      float M = -INFINITY;
+      for (int sp = 0; sp < nsplit; ++sp) M = fmaxf(M, sm_m[sp * RG + rr]);
+      float L = 0.f;
+      for (int sp = 0; sp < nsplit; ++sp) {
+        const float ms = sm_m[sp * RG + rr];
+        const float w = (ms == -INFINITY) ? 0.f : exp2f(ms - M);
+        sm_m[sp * RG + rr] = w;
+        L += w * sm_w[sp * RG + rr];
+      }
+      const float inv = 1.0f / L;
+      for (int sp = 0; sp < nsplit; ++sp) sm_w[sp * RG + rr] = sm_m[sp * RG + rr] * inv;
+    }
+    __syncthreads();
+    for (int idx = threadIdx.x; idx < nr * 16; idx += nthreads) {
+      const int rr = idx >> 4, d4 = (idx & 15) * 4;
+      const int r = rg0 + rr;
+      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll 4
+      for (int sp = 0; sp < nsplit; ++sp) {
+        const float w = sm_w[sp * RG + rr];
+        const float4 v = __ldcg(reinterpret_cast<const float4*>(po0 + (sp * a.r_max + r) * 64 + d4));
+        acc.x += w * v.x;
+        acc.y += w * v.y;
+        acc.z += w * v.z;
+        acc.w += w * v.w;
+      }
+      const int t = tok0 + r / a.G;
+      const int hq = h * a.G + r % a.G;
+      __nv_bfloat16* dst = a.out + (static_cast<size_t>(t) * a.Hq + hq) * 64 + d4;
+      *reinterpret_cast<__nv_bfloat162*>(dst) = __floats2bfloat162_rn(acc.x, acc.y);
+      *reinterpret_cast<__nv_bfloat162*>(dst + 2) = __floats2bfloat162_rn(acc.z, acc.w);
+    }
+    __syncthreads();
   }
 }
 

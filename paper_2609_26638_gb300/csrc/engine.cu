@@ -86,7 +86,7 @@ GemmPlan plan_gemm(int weight_rows, int K, int T, bool allow_split) {
   const int tiles = p.feat_tiles * p.tok_tiles;
   const int nkb = K / 64;
   if (allow_split && tiles < 152) {
-    const int want = cdiv(152, tiles);
+    const int want = std::min(cdiv(152, tiles), kMaxClusterSplits);
     for (int s = 1; s <= nkb; ++s)
       if (nkb % s == 0 && s <= want) p.splits = s;
   }
@@ -287,6 +287,7 @@ int run_gemm(gs_handle* h, const CUtensorMap& tw, int weight_rows, const CUtenso
   a.K = K;
   a.splits = p.splits;
   a.kb_per_split = (K / 64) / p.splits;
+  a.cluster = p.splits > 1 ? 1 : 0;
   a.y = y;
   a.ldy = ldy;
   a.partial = h->gemm_partial;
@@ -299,7 +300,7 @@ int run_gemm(gs_handle* h, const CUtensorMap& tw, int weight_rows, const CUtenso
       return fail(h, GS_ERR_OOM, "split-K scratch too small");
   }
   GS_CUDA(h, launch_gemm(p.bn, epi, tw, tx_set[bn_index(p.bn)], a, p.feat_tiles, p.tok_tiles,
-                         h->stream));
+                         h->stream, true));
   ++h->launches;
   return GS_OK;
 }
@@ -307,9 +308,8 @@ int run_gemm(gs_handle* h, const CUtensorMap& tw, int weight_rows, const CUtenso
 int run_rmsnorm(gs_handle* h, const float* x, const __nv_bfloat16* g, __nv_bfloat16* y, int T,
                 unsigned long long* reset) {
   const int rows_per_block = 4;
-  rmsnorm_kernel<<<cdiv(T, rows_per_block), 32 * rows_per_block, 0, h->stream>>>(
-      x, g, y, T, h->cfg.d_model, h->cfg.rms_eps, reset);
-  GS_CUDA(h, cudaGetLastError());
+  GS_CUDA(h, launch_ex(rmsnorm_kernel, dim3(cdiv(T, rows_per_block)), dim3(32 * rows_per_block), 0,
+                       h->stream, true, 1, x, g, y, T, h->cfg.d_model, h->cfg.rms_eps, reset));
   ++h->launches;
   return GS_OK;
 }
@@ -347,9 +347,8 @@ int run_attention(gs_handle* h, int layer, int T, const AttnLaunch& L) {
   a.counters = h->attn_counters;
   a.err = h->err_word;
   dim3 grid(L.max_splits, c.n_kv_heads, L.n_blocks);
-  const int threads = (L.r_max / 16) * 32;
-  attn_paged_kernel<<<grid, threads, attn_smem_bytes(L.r_max), h->stream>>>(h->tm_kv, a);
-  GS_CUDA(h, cudaGetLastError());
+  GS_CUDA(h, launch_ex(attn_paged_kernel, grid, dim3(attn_threads(L.r_max)),
+                       attn_smem_bytes(L.r_max), h->stream, true, 1, h->tm_kv, a));
   ++h->launches;
   return GS_OK;
 }
@@ -362,9 +361,8 @@ int forward(gs_handle* h, int T, const int32_t* tok, const __nv_bfloat16* vis, i
             float* logits, bool decode) {
   const gs_config& c = h->cfg;
   const int d = c.d_model, F = c.d_ffn, HD = c.n_heads * 64;
-  embed_kernel<<<T, 128, 0, h->stream>>>(tok, h->embed, vis, n_vis, T, d, c.vocab, h->hbuf,
-                                         h->err_word);
-  GS_CUDA(h, cudaGetLastError());
+  GS_CUDA(h, launch_ex(embed_kernel, dim3(T), dim3(128), 0, h->stream, true, 1, tok, h->embed, vis,
+                       n_vis, T, d, c.vocab, h->hbuf, h->err_word));
   ++h->launches;
   const size_t layer_kv = static_cast<size_t>(h->n_pages) * 2 * c.n_kv_heads * 64 * 64;
   int rc;
@@ -389,8 +387,7 @@ int forward(gs_handle* h, int T, const int32_t* tok, const __nv_bfloat16* vis, i
     r.max_ctx = c.max_ctx;
     r.err = h->err_word;
     const int warps = T * (c.n_heads + 2 * c.n_kv_heads);
-    rope_kv_kernel<<<cdiv(warps, 8), 256, 0, h->stream>>>(r);
-    GS_CUDA(h, cudaGetLastError());
+    GS_CUDA(h, launch_ex(rope_kv_kernel, dim3(cdiv(warps, 8)), dim3(256), 0, h->stream, true, 1, r));
     ++h->launches;
     if ((rc = run_attention(h, l, T, AL))) return rc;
     if ((rc = run_gemm(h, h->tm_o[l], d, h->tm_ao, HD, T, kEpiResidF32, h->hbuf, d, d, nullptr,
@@ -452,14 +449,12 @@ int enqueue_round(gs_handle* h, const int32_t* slots, int n_seq, int K, const gs
   AL.fixed_slot = -1;
 
   h->launches = 0;
-  window_draft_kernel<<<nb, 128, 0, h->stream>>>(w);
-  GS_CUDA(h, cudaGetLastError());
+  GS_CUDA(h, launch_ex(window_draft_kernel, dim3(nb), dim3(128), 0, h->stream, true, 1, w));
   ++h->launches;
   int rc = forward(h, T, h->tok, nullptr, 0, AL, 0, T, h->packed_d,
                    dbg ? dbg->draft_logits : nullptr, true);
   if (rc) return rc;
-  window_verify_kernel<<<nb, 128, 0, h->stream>>>(w);
-  GS_CUDA(h, cudaGetLastError());
+  GS_CUDA(h, launch_ex(window_verify_kernel, dim3(nb), dim3(128), 0, h->stream, true, 1, w));
   ++h->launches;
   rc = forward(h, T, h->tok, nullptr, 0, AL, 0, T, h->packed_v, dbg ? dbg->verify_logits : nullptr,
                true);
@@ -477,8 +472,8 @@ int enqueue_round(gs_handle* h, const int32_t* slots, int n_seq, int K, const gs
   ac.out_tok = out_tok;
   ac.out_cnt = out_cnt;
   ac.out_done = out_done;
-  accept_commit_kernel<<<cdiv(n_seq, 64), 64, 0, h->stream>>>(ac);
-  GS_CUDA(h, cudaGetLastError());
+  GS_CUDA(h, launch_ex(accept_commit_kernel, dim3(cdiv(n_seq, 64)), dim3(64), 0, h->stream, true, 1,
+                       ac));
   ++h->launches;
   if (dbg) {
     if (dbg->draft_tok) copy_i32_kernel<<<nb, 128, 0, h->stream>>>(h->draft_tok, dbg->draft_tok, T);
@@ -873,7 +868,7 @@ int gs_attention(int mode, const void* q, const void* kv, int n_pages, const int
   a.counters = counters;
   a.err = err;
   dim3 grid(ms, n_kv_heads, n_seq);
-  attn_paged_kernel<<<grid, (r_max / 16) * 32, attn_smem_bytes(r_max), s>>>(tm, a);
+  attn_paged_kernel<<<grid, attn_threads(r_max), attn_smem_bytes(r_max), s>>>(tm, a);
   return cudaGetLastError() == cudaSuccess ? GS_OK : GS_ERR_CUDA;
 }
 
@@ -923,6 +918,7 @@ int gs_linear(const void* x, const void* w, void* y, int M, int N, int K, int ep
   a.K = K;
   a.splits = split_k;
   a.kb_per_split = (K / 64) / split_k;
+  a.cluster = (split_k > 1 && split_k <= kMaxClusterSplits) ? 1 : 0;
   a.y = y;
   a.ldy = N;
   a.logits = nullptr;

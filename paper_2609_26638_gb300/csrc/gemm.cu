@@ -6,31 +6,33 @@ namespace gs {
 
 template <int BN, int EPI>
 static cudaError_t launch_one(const CUtensorMap& tmW, const CUtensorMap& tmX, const GemmArgs& a,
-                              int feat_tiles, int tok_tiles, cudaStream_t s) {
+                              int feat_tiles, int tok_tiles, cudaStream_t s, bool pdl) {
   dim3 grid(feat_tiles, tok_tiles, a.splits);
-  gemm_tc_kernel<BN, EPI><<<grid, 128, GemmShape<BN>::kSmemBytes, s>>>(tmW, tmX, a);
-  return cudaGetLastError();
+  const int cz = (a.splits > 1 && a.cluster) ? a.splits : 1;
+  return launch_ex(gemm_tc_kernel<BN, EPI>, grid, dim3(128), GemmShape<BN>::kSmemBytes, s, pdl, cz,
+                   tmW, tmX, a);
 }
 
 template <int BN>
 static cudaError_t launch_bn(int epi, const CUtensorMap& tmW, const CUtensorMap& tmX,
-                             const GemmArgs& a, int ft, int tt, cudaStream_t s) {
+                             const GemmArgs& a, int ft, int tt, cudaStream_t s, bool pdl) {
   switch (epi) {
-    case kEpiStoreBf16: return launch_one<BN, kEpiStoreBf16>(tmW, tmX, a, ft, tt, s);
-    case kEpiResidF32: return launch_one<BN, kEpiResidF32>(tmW, tmX, a, ft, tt, s);
-    case kEpiSwiGLU: return launch_one<BN, kEpiSwiGLU>(tmW, tmX, a, ft, tt, s);
-    case kEpiArgmax: return launch_one<BN, kEpiArgmax>(tmW, tmX, a, ft, tt, s);
+    case kEpiStoreBf16: return launch_one<BN, kEpiStoreBf16>(tmW, tmX, a, ft, tt, s, pdl);
+    case kEpiResidF32: return launch_one<BN, kEpiResidF32>(tmW, tmX, a, ft, tt, s, pdl);
+    case kEpiSwiGLU: return launch_one<BN, kEpiSwiGLU>(tmW, tmX, a, ft, tt, s, pdl);
+    case kEpiArgmax: return launch_one<BN, kEpiArgmax>(tmW, tmX, a, ft, tt, s, pdl);
   }
   return cudaErrorInvalidValue;
 }
 
 cudaError_t launch_gemm(int bn, int epi, const CUtensorMap& tmW, const CUtensorMap& tmX,
-                        const GemmArgs& a, int feat_tiles, int tok_tiles, cudaStream_t s) {
+                        const GemmArgs& a, int feat_tiles, int tok_tiles, cudaStream_t s,
+                        bool pdl) {
   switch (bn) {
-    case 32: return launch_bn<32>(epi, tmW, tmX, a, feat_tiles, tok_tiles, s);
-    case 64: return launch_bn<64>(epi, tmW, tmX, a, feat_tiles, tok_tiles, s);
-    case 128: return launch_bn<128>(epi, tmW, tmX, a, feat_tiles, tok_tiles, s);
-    case 256: return launch_bn<256>(epi, tmW, tmX, a, feat_tiles, tok_tiles, s);
+    case 32: return launch_bn<32>(epi, tmW, tmX, a, feat_tiles, tok_tiles, s, pdl);
+    case 64: return launch_bn<64>(epi, tmW, tmX, a, feat_tiles, tok_tiles, s, pdl);
+    case 128: return launch_bn<128>(epi, tmW, tmX, a, feat_tiles, tok_tiles, s, pdl);
+    case 256: return launch_bn<256>(epi, tmW, tmX, a, feat_tiles, tok_tiles, s, pdl);
   }
   return cudaErrorInvalidValue;
 }

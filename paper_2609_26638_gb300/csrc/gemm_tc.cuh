@@ -8,9 +8,18 @@
 // fp32 accumulator of 128 lanes x BN columns; four warps read it back with
 // tcgen05.ld for the fused epilogue.
 //
-// Split-K: CTAs of one output tile that own different K ranges write fp32
-// partials; the last CTA to arrive (atomic counter, no spinning) sums the
-// partials in split order, so results do not depend on arrival order.
+// Launch overlap: weight tiles do not depend on the previous kernel, so the
+// producer issues the first stages' weight loads before griddepcontrol.wait
+// (programmatic dependent launch); activation loads and every global write
+// come after it.
+//
+// Split-K: the CTAs that own different K ranges of one output tile either
+// form a thread-block cluster and reduce their fp32 partials through
+// distributed shared memory (each CTA sums a slice of the tile's tokens over
+// all peers), or -- for split factors above the cluster limit -- write the
+// partials to global scratch, where the last CTA to arrive (atomic ticket, no
+// spinning) sums them.  Both sum the splits in order 0..S-1 from a zero
+// start, so the result does not depend on the path or on arrival order.
 //
 // Epilogues: bf16 store, fp32 residual add, SwiGLU (gate and up rows of the
 // same features share a tile), and LM-head argmax (packed 64-bit atomicMax,
@@ -28,10 +37,11 @@ struct GemmArgs {
   int K;            // reduction length, multiple of 64
   int splits;       // split-K factor (divides K / 64)
   int kb_per_split; // (K / 64) / splits
+  int cluster;      // 1: split-K partials reduced inside a cluster of `splits` CTAs
   void* y;          // output: bf16 [M, ldy] | fp32 [M, ldy] | uint64 [M] (argmax)
   int ldy;
-  float* partial;   // split-K partials [splits][tiles][BN][128] fp32
-  int* counters;    // per output tile, zero between launches
+  float* partial;   // global split-K partials [splits][tiles][BN][128] fp32 (cluster == 0)
+  int* counters;    // per output tile, zero between launches (cluster == 0)
   float* logits;    // argmax only: optional fp32 [M, N] dump
   int* err;
 };
@@ -44,28 +54,32 @@ struct GemmShape {
   // two CTAs per SM up to BN = 128 (<= ~97 KB each), one at BN = 256
   static constexpr int kStages = BN <= 64 ? 4 : (BN <= 128 ? 3 : 4);
   static constexpr int kTmemCols = BN < 32 ? 32 : BN;
+  static constexpr int kRedBytes = BN * 128 * 4;   // cluster reduction tile [BN][128] fp32
+  static constexpr int kXBufBytes = 32 * 64 * 4;   // SwiGLU gate/up exchange
+  static_assert(kRedBytes + kXBufBytes <= kStages * kStageBytes, "reduction smem");
   static constexpr int kSmemBytes = kStages * kStageBytes + 1024 /*align*/ + 256 /*barriers*/;
 };
 
+// Epilogue of 32 consecutive tokens (t0 .. t0+31) of feature row `row`;
+// only tokens j in [jlo, jhi) with t0 + j < M are produced.
 template <int BN, int EPI>
 __device__ __forceinline__ void gemm_epilogue_chunk(const GemmArgs& a, float (&v)[32], int row,
-                                                    int feat_tile, int tok0, int chunk,
+                                                    int feat_tile, int t0, int jlo, int jhi,
                                                     float* xbuf) {
   const int warp = threadIdx.x >> 5;
-  const int t0 = tok0 + chunk * 32;
-  const int nvalid = min(32, a.M - t0);
+  jhi = min(jhi, a.M - t0);
   if constexpr (EPI == kEpiStoreBf16) {
     __nv_bfloat16* y = static_cast<__nv_bfloat16*>(a.y);
     const int f = feat_tile * 128 + row;
 #pragma unroll
     for (int j = 0; j < 32; ++j)
-      if (j < nvalid) y[static_cast<size_t>(t0 + j) * a.ldy + f] = __float2bfloat16_rn(v[j]);
+      if (j >= jlo && j < jhi) y[static_cast<size_t>(t0 + j) * a.ldy + f] = __float2bfloat16_rn(v[j]);
   } else if constexpr (EPI == kEpiResidF32) {
     float* y = static_cast<float*>(a.y);
     const int f = feat_tile * 128 + row;
 #pragma unroll
     for (int j = 0; j < 32; ++j)
-      if (j < nvalid) {
+      if (j >= jlo && j < jhi) {
         float* p = y + static_cast<size_t>(t0 + j) * a.ldy + f;
         *p = *p + v[j];
       }
@@ -81,7 +95,7 @@ __device__ __forceinline__ void gemm_epilogue_chunk(const GemmArgs& a, float (&v
       const int f = feat_tile * 64 + row;
 #pragma unroll
       for (int j = 0; j < 32; ++j)
-        if (j < nvalid) {
+        if (j >= jlo && j < jhi) {
           const float g = v[j];
           const float u = xbuf[j * 64 + row];
           const float s = g / (1.0f + __expf(-g));
@@ -95,7 +109,7 @@ __device__ __forceinline__ void gemm_epilogue_chunk(const GemmArgs& a, float (&v
     if (a.logits != nullptr) {
 #pragma unroll
       for (int j = 0; j < 32; ++j)
-        if (j < nvalid) a.logits[static_cast<size_t>(t0 + j) * a.N + f] = v[j];
+        if (j >= jlo && j < jhi) a.logits[static_cast<size_t>(t0 + j) * a.N + f] = v[j];
     }
     const int lane = threadIdx.x & 31;
 #pragma unroll
@@ -106,7 +120,7 @@ __device__ __forceinline__ void gemm_epilogue_chunk(const GemmArgs& a, float (&v
         const unsigned long long o = shfl_xor_u64(key, m);
         key = o > key ? o : key;
       }
-      if (lane == 0 && j < nvalid) atomicMax(out + t0 + j, key);
+      if (lane == 0 && j >= jlo && j < jhi) atomicMax(out + t0 + j, key);
     }
   }
 }
@@ -154,15 +168,12 @@ __global__ void __launch_bounds__(128, 1)
   const uint32_t tmem = *tmem_slot;
 
   if (warp == 0 && lane == 0) {
-    // TMA producer
+    // TMA producer.  Weight tiles of the first stages go out before the
+    // dependency wait; activations only after it.
     const uint64_t pol_w = l2_policy_evict_first();
     const uint64_t pol_x = l2_policy_evict_last();
-    for (int i = 0; i < nkb; ++i) {
-      const int s = i % S::kStages;
-      const uint32_t ph = (i / S::kStages) & 1;
-      if (!mbar_wait(smem_u32(&empty[s]), ph ^ 1, a.err)) { *flag = 1; break; }
+    auto load_w = [&](int i, int s) {
       const uint32_t fb = smem_u32(&full[s]);
-      mbar_arrive_expect_tx(fb, S::kStageBytes);
       const int kx = (kb0 + i) * 64;
       if constexpr (EPI == kEpiSwiGLU) {
         tma_load_2d(smem_u32(smA + s * S::kABytes), &tmW, kx, feat_tile * 64, fb, pol_w);
@@ -171,26 +182,47 @@ __global__ void __launch_bounds__(128, 1)
       } else {
         tma_load_2d(smem_u32(smA + s * S::kABytes), &tmW, kx, feat_tile * 128, fb, pol_w);
       }
-      tma_load_2d(smem_u32(smB + s * S::kBBytes), &tmX, kx, tok_tile * BN, fb, pol_x);
+    };
+    auto load_x = [&](int i, int s) {
+      tma_load_2d(smem_u32(smB + s * S::kBBytes), &tmX, (kb0 + i) * 64, tok_tile * BN,
+                  smem_u32(&full[s]), pol_x);
+    };
+    const int npre = nkb < S::kStages ? nkb : S::kStages;
+    for (int i = 0; i < npre; ++i) {          // fresh stages: no empty-barrier wait needed
+      mbar_arrive_expect_tx(smem_u32(&full[i]), S::kStageBytes);
+      load_w(i, i);
     }
-  } else if (warp == 1 && lane == 0) {
-    // MMA issuer
-    constexpr uint32_t idesc = umma_idesc_bf16(128, BN);
-    bool ok = true;
-    for (int i = 0; i < nkb; ++i) {
+    pdl_wait();
+    pdl_trigger();
+    for (int i = 0; i < npre; ++i) load_x(i, i);
+    for (int i = npre; i < nkb; ++i) {
       const int s = i % S::kStages;
       const uint32_t ph = (i / S::kStages) & 1;
-      if (!mbar_wait(smem_u32(&full[s]), ph, a.err)) { ok = false; *flag = 1; break; }
-      tc_fence_after();
-      const uint64_t ad = umma_desc_sw128(smem_u32(smA + s * S::kABytes));
-      const uint64_t bd = umma_desc_sw128(smem_u32(smB + s * S::kBBytes));
-#pragma unroll
-      for (int k = 0; k < 4; ++k)
-        umma_bf16(tmem, ad + 2 * k, bd + 2 * k, idesc, (i > 0 || k > 0) ? 1u : 0u);
-      umma_commit(smem_u32(&empty[s]));
+      if (!mbar_wait(smem_u32(&empty[s]), ph ^ 1, a.err)) { *flag = 1; break; }
+      mbar_arrive_expect_tx(smem_u32(&full[s]), S::kStageBytes);
+      load_w(i, s);
+      load_x(i, s);
     }
-    umma_commit(smem_u32(accum));
-    (void)ok;
+  } else {
+    pdl_wait();
+    pdl_trigger();
+    if (warp == 1 && lane == 0) {
+      // MMA issuer
+      constexpr uint32_t idesc = umma_idesc_bf16(128, BN);
+      for (int i = 0; i < nkb; ++i) {
+        const int s = i % S::kStages;
+        const uint32_t ph = (i / S::kStages) & 1;
+        if (!mbar_wait(smem_u32(&full[s]), ph, a.err)) { *flag = 1; break; }
+        tc_fence_after();
+        const uint64_t ad = umma_desc_sw128(smem_u32(smA + s * S::kABytes));
+        const uint64_t bd = umma_desc_sw128(smem_u32(smB + s * S::kBBytes));
+#pragma unroll
+        for (int k = 0; k < 4; ++k)
+          umma_bf16(tmem, ad + 2 * k, bd + 2 * k, idesc, (i > 0 || k > 0) ? 1u : 0u);
+        umma_commit(smem_u32(&empty[s]));
+      }
+      umma_commit(smem_u32(accum));
+    }
   }
   __syncwarp();
 
@@ -199,17 +231,17 @@ __global__ void __launch_bounds__(128, 1)
   tc_fence_after();
   const int row = warp * 32 + lane;      // TMEM lane = weight row of the tile
   const uint32_t trow = tmem + (static_cast<uint32_t>(warp * 32) << 16);
-  float* xbuf = reinterpret_cast<float*>(smA);   // pipeline smem is free after the accumulator
   const int tok0 = tok_tile * BN;
   const bool failed = !acc_ok || *flag;
 
   if (a.splits == 1) {
+    float* xbuf = reinterpret_cast<float*>(smA);   // pipeline smem is free after the accumulator
     if (!failed) {
       for (int c = 0; c < BN / 32; ++c) {
         if (tok0 + c * 32 >= a.M) break;   // uniform across the CTA
         float v[32];
         tmem_ld_32x32b_x32(trow + c * 32, v);
-        gemm_epilogue_chunk<BN, EPI>(a, v, row, feat_tile, tok0, c, xbuf);
+        gemm_epilogue_chunk<BN, EPI>(a, v, row, feat_tile, tok0 + c * 32, 0, 32, xbuf);
       }
     }
     tc_fence_before();
@@ -218,7 +250,45 @@ __global__ void __launch_bounds__(128, 1)
     return;
   }
 
-  // split-K: write this split's partial tile, token-major [BN][128]
+  if (a.cluster) {
+    // Cluster split-K: partial tile -> own smem [BN][128]; after the cluster
+    // barrier, CTA `split` reduces tokens [split*BN/S, (split+1)*BN/S) over
+    // all peers in order 0..S-1 and runs the epilogue on them.
+    float* red = reinterpret_cast<float*>(smA);
+    float* xbuf = reinterpret_cast<float*>(smA + S::kRedBytes);
+    const int ntok = min(BN, a.M - tok0);
+    if (!failed) {
+      for (int c = 0; c < BN / 32; ++c) {
+        if (c * 32 >= ntok) break;
+        float v[32];
+        tmem_ld_32x32b_x32(trow + c * 32, v);
+#pragma unroll
+        for (int j = 0; j < 32; ++j) red[(c * 32 + j) * 128 + row] = v[j];
+      }
+    }
+    tc_fence_before();
+    cluster_sync_all();
+    if (warp == 2) tmem_dealloc(tmem, S::kTmemCols);
+    const int per = BN / a.splits;
+    const int lo = split * per, hi = min(lo + per, ntok);
+    for (int c = lo / 32; c * 32 < hi; ++c) {
+      const int jlo = max(lo - c * 32, 0), jhi = min(hi - c * 32, 32);
+      float v[32];
+#pragma unroll
+      for (int j = 0; j < 32; ++j) v[j] = 0.0f;
+      for (int s = 0; s < a.splits; ++s) {
+        const float* peer = cluster_peer_ptr(red, static_cast<uint32_t>(s));
+#pragma unroll
+        for (int j = 0; j < 32; ++j)
+          if (j >= jlo && j < jhi) v[j] += peer[(c * 32 + j) * 128 + row];
+      }
+      if (!failed) gemm_epilogue_chunk<BN, EPI>(a, v, row, feat_tile, tok0 + c * 32, jlo, jhi, xbuf);
+    }
+    cluster_sync_all();   // peers may still be reading this CTA's partial tile
+    return;
+  }
+
+  // global split-K: write this split's partial tile, token-major [BN][128]
   const int tiles = gridDim.x * gridDim.y;
   const int tile = tok_tile * gridDim.x + feat_tile;
   float* mine = a.partial + (static_cast<size_t>(split) * tiles + tile) * (BN * 128);
@@ -244,6 +314,7 @@ __global__ void __launch_bounds__(128, 1)
   __syncthreads();
   if (!is_last || failed) return;
   __threadfence();
+  float* xbuf = reinterpret_cast<float*>(smA);
   for (int c = 0; c < BN / 32; ++c) {
     if (tok0 + c * 32 >= a.M) break;
     float v[32];
@@ -254,7 +325,7 @@ __global__ void __launch_bounds__(128, 1)
 #pragma unroll
       for (int j = 0; j < 32; ++j) v[j] += __ldcg(p + (c * 32 + j) * 128 + row);
     }
-    gemm_epilogue_chunk<BN, EPI>(a, v, row, feat_tile, tok0, c, xbuf);
+    gemm_epilogue_chunk<BN, EPI>(a, v, row, feat_tile, tok0 + c * 32, 0, 32, xbuf);
   }
 }
 

@@ -4,17 +4,53 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <utility>
+
 namespace gs {
 
 struct GemmArgs;
+
+// cudaLaunchKernelEx with optional programmatic stream serialisation (PDL) and
+// a cluster along z.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_ex(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                      cudaStream_t s, bool pdl, int cluster_z, Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attrs[2];
+  int n = 0;
+  if (pdl) {
+    attrs[n].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attrs[n].val.programmaticStreamSerializationAllowed = 1;
+    ++n;
+  }
+  if (cluster_z > 1) {
+    attrs[n].id = cudaLaunchAttributeClusterDimension;
+    attrs[n].val.clusterDim.x = 1;
+    attrs[n].val.clusterDim.y = 1;
+    attrs[n].val.clusterDim.z = cluster_z;
+    ++n;
+  }
+  cfg.attrs = attrs;
+  cfg.numAttrs = n;
+  return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
 
 // Token tile for a GEMM over T token rows.
 inline int gemm_bn_for(int T) { return T <= 32 ? 32 : (T <= 64 ? 64 : (T <= 128 ? 128 : 256)); }
 
 // Launch Y = epilogue(W . X^T) for one weight matrix.  grid = (feat_tiles,
 // tok_tiles, splits).  Returns a cudaError_t.
+// Split-K partials are reduced through distributed shared memory inside a
+// cluster of the `splits` CTAs of a tile when splits <= kMaxClusterSplits,
+// else through global scratch by the last CTA to arrive (same order, same bits).
+constexpr int kMaxClusterSplits = 8;
 cudaError_t launch_gemm(int bn, int epi, const CUtensorMap& tmW, const CUtensorMap& tmX,
-                        const GemmArgs& args, int feat_tiles, int tok_tiles, cudaStream_t s);
+                        const GemmArgs& args, int feat_tiles, int tok_tiles, cudaStream_t s,
+                        bool pdl = false);
 
 // Sets the dynamic shared-memory limit of every GEMM instantiation once.
 cudaError_t gemm_init_attributes();

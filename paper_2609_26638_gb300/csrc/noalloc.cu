@@ -123,6 +123,7 @@ extern "C" int gs_linear_noalloc(const void* x, const void* w, void* y, int M, i
   a.N = N;
   a.K = K;
   a.splits = split_k;
+  a.cluster = 0;
   a.kb_per_split = (K / 64) / split_k;
   a.y = y;
   a.ldy = N;

@@ -178,6 +178,28 @@ __device__ __forceinline__ void tmem_ld_32x32b_x32(uint32_t taddr, float (&v)[32
   for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
 
+// ---------------------------------------------------------------- PDL / clusters
+// Programmatic dependent launch: wait until the preceding kernel in the stream
+// has completed and its writes are visible (a no-op when the kernel was not
+// launched with programmatic stream serialisation), and allow the next kernel
+// to start its pre-wait prologue.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;"
+               ::: "memory");
+}
+
+// Generic address of the same shared-memory location in CTA `rank` of the cluster.
+__device__ __forceinline__ const float* cluster_peer_ptr(const float* p, uint32_t rank) {
+  uint64_t g;
+  asm volatile("mapa.u64 %0, %1, %2;" : "=l"(g) : "l"(reinterpret_cast<uint64_t>(p)), "r"(rank));
+  return reinterpret_cast<const float*>(g);
+}
+
 // ---------------------------------------------------------------- misc
 // Total order on floats as unsigned keys (larger float -> larger key).
 __device__ __forceinline__ uint32_t float_order_key(float v) {

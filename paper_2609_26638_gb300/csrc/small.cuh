@@ -40,6 +40,8 @@ struct WindowArgs {
 
 // Draft window: [x0, [M] x K] at slots n..n+K; row 0 sees keys 0..n, mask rows 0..n+K.
 __global__ void window_draft_kernel(WindowArgs a) {
+  pdl_wait();
+  pdl_trigger();
   const int idx = blockIdx.x * blockDim.x + threadIdx.x;
   if (idx >= a.n_seq * a.W) return;
   const int b = idx / a.W, i = idx % a.W;
@@ -59,6 +61,8 @@ __global__ void window_draft_kernel(WindowArgs a) {
 // Verify window: [a0, d_1..d_K] at slots n+1..n+K+1, token-level causal.
 // Applies the forcing hook to the drafts when a teacher is given.
 __global__ void window_verify_kernel(WindowArgs a) {
+  pdl_wait();
+  pdl_trigger();
   const int idx = blockIdx.x * blockDim.x + threadIdx.x;
   if (idx >= a.n_seq * a.W) return;
   const int b = idx / a.W, i = idx % a.W;
@@ -109,6 +113,8 @@ struct AcceptArgs {
 };
 
 __global__ void accept_commit_kernel(AcceptArgs a) {
+  pdl_wait();
+  pdl_trigger();
   const int b = blockIdx.x * blockDim.x + threadIdx.x;
   if (b >= a.n_seq) return;
   const int slot = a.slots[b];
@@ -147,6 +153,8 @@ __global__ void accept_commit_kernel(AcceptArgs a) {
 // After a prefill: x0 = argmax at the last prefix position (paper Appendix step State).
 __global__ void prefill_finish_kernel(const unsigned long long* packed, SeqStateDev st, int slot,
                                       int P, int max_new, int eos, int32_t* x0_out) {
+  pdl_wait();
+  pdl_trigger();
   if (threadIdx.x != 0 || blockIdx.x != 0) return;
   const int x0 = argmax_key_index(packed[0]);
   st.seq_len[slot] = P;
@@ -160,6 +168,8 @@ __global__ void prefill_finish_kernel(const unsigned long long* packed, SeqState
 
 __global__ void seq_restore_kernel(SeqStateDev st, int slot, int seq_len, int x0, int n_out,
                                    int max_new, int done, int rounds) {
+  pdl_wait();
+  pdl_trigger();
   if (threadIdx.x != 0 || blockIdx.x != 0) return;
   st.seq_len[slot] = seq_len;
   st.x0[slot] = x0;
@@ -172,6 +182,8 @@ __global__ void seq_restore_kernel(SeqStateDev st, int slot, int seq_len, int x0
 // Prefill chunk positions: token t at slot p0 + t, causal limit p0 + t.
 __global__ void prefill_window_kernel(int T, int p0, int slot, int32_t* pos, int32_t* lim,
                                       int32_t* tok_slot) {
+  pdl_wait();
+  pdl_trigger();
   const int t = blockIdx.x * blockDim.x + threadIdx.x;
   if (t >= T) return;
   pos[t] = p0 + t;
@@ -182,6 +194,8 @@ __global__ void prefill_window_kernel(int T, int p0, int slot, int32_t* pos, int
 // h[t] = E[tok[t]] (fp32), or the visual row for t < n_vis.  d % 8 == 0.
 __global__ void embed_kernel(const int32_t* tok, const __nv_bfloat16* E, const __nv_bfloat16* vis,
                              int n_vis, int T, int d, int vocab, float* h, int* err) {
+  pdl_wait();
+  pdl_trigger();
   const int t = blockIdx.x;
   if (t >= T) return;
   const __nv_bfloat16* src;
@@ -214,6 +228,8 @@ __global__ void embed_kernel(const int32_t* tok, const __nv_bfloat16* E, const _
 // Optionally zeroes argmax keys of the row (the LM-head argmax accumulator).
 __global__ void rmsnorm_kernel(const float* x, const __nv_bfloat16* gain, __nv_bfloat16* y, int T,
                                int d, float eps, unsigned long long* reset_keys) {
+  pdl_wait();
+  pdl_trigger();
   const int row = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (row >= T) return;
@@ -257,6 +273,8 @@ struct RopeKvArgs {
 };
 
 __global__ void rope_kv_kernel(RopeKvArgs a) {
+  pdl_wait();
+  pdl_trigger();
   const int warps_per_block = blockDim.x >> 5;
   const int gw = blockIdx.x * warps_per_block + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
