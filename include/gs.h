@@ -53,9 +53,9 @@ typedef enum { GS_ACCEPT_GREEDY = 0, GS_ACCEPT_STOCHASTIC = 1 } gs_accept_rule;
  * library implements a pre-norm decoder: RMSNorm (learned gain, eps) ->
  * grouped-query attention with rotate-half RoPE on all head dims at absolute
  * positions -> RMSNorm -> SwiGLU FFN; untied input/output embeddings, no
- * biases.  Requirements: head_dim 64, n_heads % n_kv_heads == 0,
- * d_model % 128 == 0, (n_heads + 2 n_kv_heads) * 64 % 128 == 0,
- * d_ffn % 64 == 0, vocab % 128 == 0. */
+ * biases.  Requirements: head_dim 64, n_heads % n_kv_heads == 0, n_heads and
+ * n_kv_heads even (a 128-row projection tile holds two whole heads),
+ * d_model % 128 == 0, d_ffn % 64 == 0, vocab % 128 == 0. */
 typedef struct {
   int n_layers, d_model, n_heads, n_kv_heads, head_dim, d_ffn, vocab;
   float rope_theta, rms_eps;

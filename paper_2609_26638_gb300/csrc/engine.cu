@@ -108,7 +108,7 @@ struct gs_handle {
   std::vector<const __nv_bfloat16*> attn_norm, ffn_norm, w_qkv, w_o, w_gu, w_down;
   std::vector<CUtensorMap> tm_qkv, tm_o, tm_gu, tm_down;
   CUtensorMap tm_lm;
-  CUtensorMap tm_xn[4], tm_ao[4], tm_act[4];
+  CUtensorMap tm_hb[4], tm_ao[4], tm_act[4];
   CUtensorMap tm_kv;
 
   // sizes
@@ -124,7 +124,8 @@ struct gs_handle {
   int32_t *tok = nullptr, *pos = nullptr, *lim = nullptr, *tok_slot = nullptr;
   int32_t *blk_slot = nullptr, *blk_active = nullptr;
   float* hbuf = nullptr;
-  __nv_bfloat16 *xn = nullptr, *qkv = nullptr, *qr = nullptr, *ao = nullptr, *act = nullptr;
+  __nv_bfloat16 *hb = nullptr, *qr = nullptr, *ao = nullptr, *act = nullptr;
+  float* ssp = nullptr;   // per-token sums of h^2 per 128-feature block [T_max][d/128]
   unsigned long long *packed_d = nullptr, *packed_v = nullptr;
   int32_t *draft_tok = nullptr, *verify_in = nullptr, *verify_tok = nullptr;
   float* gemm_partial = nullptr;
@@ -172,7 +173,7 @@ bool config_ok(const gs_config* c, std::string* why) {
   if (c->n_heads < 1 || c->n_kv_heads < 1 || c->n_heads % c->n_kv_heads) return bad("bad heads");
   if (c->n_heads / c->n_kv_heads > 8) return bad("GQA group > 8 unsupported");
   if (c->d_model % 128) return bad("d_model % 128");
-  if (((c->n_heads + 2 * c->n_kv_heads) * 64) % 128) return bad("qkv rows % 128");
+  if (c->n_heads % 2 || c->n_kv_heads % 2) return bad("n_heads and n_kv_heads must be even");
   if ((c->n_heads * 64) % 64) return bad("attn dim % 64");
   if (c->d_ffn % 64 || c->d_ffn < 64) return bad("d_ffn % 64");
   if (c->vocab % 128) return bad("vocab % 128");
@@ -219,8 +220,8 @@ size_t carve(gs_handle* h, const gs_config& c, void* base) {
   int32_t* blk_slot = cv.take<int32_t>(std::max(c.max_batch, T_max / 64 + 1));
   int32_t* blk_active = cv.take<int32_t>(std::max(c.max_batch, T_max / 64 + 1));
   float* hbuf = cv.take<float>(static_cast<size_t>(T_max) * c.d_model);
-  __nv_bfloat16* xn = cv.take<__nv_bfloat16>(static_cast<size_t>(T_max) * c.d_model);
-  __nv_bfloat16* qkv = cv.take<__nv_bfloat16>(static_cast<size_t>(T_max) * qkv_dim);
+  __nv_bfloat16* hb = cv.take<__nv_bfloat16>(static_cast<size_t>(T_max) * c.d_model);
+  float* ssp = cv.take<float>(static_cast<size_t>(T_max) * (c.d_model / 128));
   __nv_bfloat16* qr = cv.take<__nv_bfloat16>(static_cast<size_t>(T_max) * c.n_heads * 64);
   __nv_bfloat16* ao = cv.take<__nv_bfloat16>(static_cast<size_t>(T_max) * c.n_heads * 64);
   __nv_bfloat16* act = cv.take<__nv_bfloat16>(static_cast<size_t>(T_max) * c.d_ffn);
@@ -258,8 +259,8 @@ size_t carve(gs_handle* h, const gs_config& c, void* base) {
     h->blk_slot = blk_slot;
     h->blk_active = blk_active;
     h->hbuf = hbuf;
-    h->xn = xn;
-    h->qkv = qkv;
+    h->hb = hb;
+    h->ssp = ssp;
     h->qr = qr;
     h->ao = ao;
     h->act = act;
@@ -278,38 +279,29 @@ size_t carve(gs_handle* h, const gs_config& c, void* base) {
 }
 
 // ------------------------------------------------------------------ launches
+// A GemmArgs with the fields every decoder GEMM shares; the caller adds the
+// epilogue's outputs.
+GemmArgs gemm_base(gs_handle* h) {
+  GemmArgs a = {};
+  a.partial = h->gemm_partial;
+  a.counters = h->gemm_counters;
+  a.err = h->err_word;
+  a.n_ssp = h->cfg.d_model / 128;
+  a.inv_d = 1.0f / static_cast<float>(h->cfg.d_model);
+  a.eps = h->cfg.rms_eps;
+  return a;
+}
+
 int run_gemm(gs_handle* h, const CUtensorMap& tw, int weight_rows, const CUtensorMap* tx_set, int K,
-             int T, int epi, void* y, int ldy, int N, float* logits, bool decode) {
+             int T, int epi, GemmArgs a, bool decode) {
   const GemmPlan p = plan_gemm(weight_rows, K, T, decode);
-  GemmArgs a;
   a.M = T;
-  a.N = N;
   a.K = K;
   a.splits = p.splits;
   a.kb_per_split = (K / 64) / p.splits;
   a.cluster = p.splits > 1 ? 1 : 0;
-  a.y = y;
-  a.ldy = ldy;
-  a.partial = h->gemm_partial;
-  a.counters = h->gemm_counters;
-  a.logits = logits;
-  a.err = h->err_word;
-  if (p.splits > 1) {
-    const size_t need = static_cast<size_t>(p.splits) * p.feat_tiles * p.tok_tiles * p.bn * 128;
-    if (need > kGemmPartialFloats || p.feat_tiles * p.tok_tiles > kGemmCounters)
-      return fail(h, GS_ERR_OOM, "split-K scratch too small");
-  }
   GS_CUDA(h, launch_gemm(p.bn, epi, tw, tx_set[bn_index(p.bn)], a, p.feat_tiles, p.tok_tiles,
                          h->stream, true));
-  ++h->launches;
-  return GS_OK;
-}
-
-int run_rmsnorm(gs_handle* h, const float* x, const __nv_bfloat16* g, __nv_bfloat16* y, int T,
-                unsigned long long* reset) {
-  const int rows_per_block = 4;
-  GS_CUDA(h, launch_ex(rmsnorm_kernel, dim3(cdiv(T, rows_per_block)), dim3(32 * rows_per_block), 0,
-                       h->stream, true, 1, x, g, y, T, h->cfg.d_model, h->cfg.rms_eps, reset));
   ++h->launches;
   return GS_OK;
 }
@@ -355,57 +347,69 @@ int run_attention(gs_handle* h, int layer, int T, const AttnLaunch& L) {
 
 // One decoder forward over T rows already described by tok/pos/lim/tok_slot.
 // Visual rows (prefill) come first when n_vis > 0.  The LM head runs on rows
-// [lm_row0, lm_row0 + n_lm) and leaves argmax keys in `packed`.
+// [lm_row0, lm_row0 + n_lm) (none if n_lm == 0) and leaves argmax keys in
+// `packed`.  Per layer: QKV (+norm scale, RoPE, KV write) -> attention ->
+// O (+residual, next norm's input) -> gate/up (+norm scale, SwiGLU) -> down
+// (+residual, next norm's input).
 int forward(gs_handle* h, int T, const int32_t* tok, const __nv_bfloat16* vis, int n_vis,
             const AttnLaunch& AL, int lm_row0, int n_lm, unsigned long long* packed,
             float* logits, bool decode) {
   const gs_config& c = h->cfg;
-  const int d = c.d_model, F = c.d_ffn, HD = c.n_heads * 64;
+  const int d = c.d_model, F = c.d_ffn, HD = c.n_heads * 64, L = c.n_layers;
   GS_CUDA(h, launch_ex(embed_kernel, dim3(T), dim3(128), 0, h->stream, true, 1, tok, h->embed, vis,
-                       n_vis, T, d, c.vocab, h->hbuf, h->err_word));
+                       n_vis, T, d, c.vocab, h->hbuf, h->hb, h->attn_norm[0], h->ssp, packed,
+                       h->err_word));
   ++h->launches;
   const size_t layer_kv = static_cast<size_t>(h->n_pages) * 2 * c.n_kv_heads * 64 * 64;
   int rc;
-  for (int l = 0; l < c.n_layers; ++l) {
-    if ((rc = run_rmsnorm(h, h->hbuf, h->attn_norm[l], h->xn, T, nullptr))) return rc;
-    if ((rc = run_gemm(h, h->tm_qkv[l], h->qkv_dim, h->tm_xn, d, T, kEpiStoreBf16, h->qkv,
-                       h->qkv_dim, h->qkv_dim, nullptr, decode)))
-      return rc;
-    RopeKvArgs r;
-    r.qkv = h->qkv;
-    r.pos = h->pos;
-    r.tok_slot = h->tok_slot;
-    r.rope = h->rope;
-    r.q_out = h->qr;
-    r.kv = h->kv + l * layer_kv;
-    r.page_table = h->page_table;
-    r.pt_stride = h->pt_stride;
-    r.n_pages = h->n_pages;
-    r.T = T;
-    r.Hq = c.n_heads;
-    r.Hkv = c.n_kv_heads;
-    r.max_ctx = c.max_ctx;
-    r.err = h->err_word;
-    const int warps = T * (c.n_heads + 2 * c.n_kv_heads);
-    GS_CUDA(h, launch_ex(rope_kv_kernel, dim3(cdiv(warps, 8)), dim3(256), 0, h->stream, true, 1, r));
-    ++h->launches;
+  for (int l = 0; l < L; ++l) {
+    GemmArgs q = gemm_base(h);
+    q.N = h->qkv_dim;
+    q.ssp_in = h->ssp;
+    q.q_out = h->qr;
+    q.kv_layer = h->kv + l * layer_kv;
+    q.pos = h->pos;
+    q.tok_slot = h->tok_slot;
+    q.page_table = h->page_table;
+    q.rope = h->rope;
+    q.pt_stride = h->pt_stride;
+    q.n_pages = h->n_pages;
+    q.max_ctx = c.max_ctx;
+    q.Hq = c.n_heads;
+    q.Hkv = c.n_kv_heads;
+    if ((rc = run_gemm(h, h->tm_qkv[l], h->qkv_dim, h->tm_hb, d, T, kEpiQKV, q, decode))) return rc;
     if ((rc = run_attention(h, l, T, AL))) return rc;
-    if ((rc = run_gemm(h, h->tm_o[l], d, h->tm_ao, HD, T, kEpiResidF32, h->hbuf, d, d, nullptr,
-                       decode)))
-      return rc;
-    if ((rc = run_rmsnorm(h, h->hbuf, h->ffn_norm[l], h->xn, T, nullptr))) return rc;
-    if ((rc = run_gemm(h, h->tm_gu[l], 2 * F, h->tm_xn, d, T, kEpiSwiGLU, h->act, F, F, nullptr,
-                       decode)))
-      return rc;
-    if ((rc = run_gemm(h, h->tm_down[l], d, h->tm_act, F, T, kEpiResidF32, h->hbuf, d, d, nullptr,
-                       decode)))
-      return rc;
+    GemmArgs o = gemm_base(h);
+    o.N = d;
+    o.y = h->hbuf;
+    o.ldy = d;
+    o.hb_out = h->hb;
+    o.g_next = h->ffn_norm[l];
+    o.ssp_out = h->ssp;
+    if ((rc = run_gemm(h, h->tm_o[l], d, h->tm_ao, HD, T, kEpiResidF32, o, decode))) return rc;
+    GemmArgs gu = gemm_base(h);
+    gu.N = F;
+    gu.y = h->act;
+    gu.ldy = F;
+    gu.ssp_in = h->ssp;
+    if ((rc = run_gemm(h, h->tm_gu[l], 2 * F, h->tm_hb, d, T, kEpiSwiGLU, gu, decode))) return rc;
+    GemmArgs dn = gemm_base(h);
+    dn.N = d;
+    dn.y = h->hbuf;
+    dn.ldy = d;
+    dn.hb_out = h->hb;
+    dn.g_next = l + 1 < L ? h->attn_norm[l + 1] : h->final_norm;
+    dn.ssp_out = h->ssp;
+    if ((rc = run_gemm(h, h->tm_down[l], d, h->tm_act, F, T, kEpiResidF32, dn, decode))) return rc;
   }
-  if ((rc = run_rmsnorm(h, h->hbuf + static_cast<size_t>(lm_row0) * d, h->final_norm, h->xn, n_lm,
-                        packed)))
-    return rc;
-  return run_gemm(h, h->tm_lm, c.vocab, h->tm_xn, d, n_lm, kEpiArgmax, packed, 0, c.vocab, logits,
-                  decode);
+  if (n_lm == 0) return GS_OK;
+  GemmArgs lm = gemm_base(h);
+  lm.N = c.vocab;
+  lm.y = packed;
+  lm.logits = logits;
+  lm.ssp_in = h->ssp;
+  lm.x_row0 = lm_row0;
+  return run_gemm(h, h->tm_lm, c.vocab, h->tm_hb, d, n_lm, kEpiArgmax, lm, decode);
 }
 
 int enqueue_round(gs_handle* h, const int32_t* slots, int n_seq, int K, const gs_force* force,
@@ -557,7 +561,7 @@ int gs_create(const gs_config* cfg, const gs_weights* w, void* workspace, size_t
   ok = ok && make_map(&h->tm_lm, w->lm_head, c.vocab, d, 128);
   const int bns[4] = {32, 64, 128, 256};
   for (int i = 0; i < 4 && ok; ++i) {
-    ok = make_map(&h->tm_xn[i], h->xn, h->T_max, d, bns[i]) &&
+    ok = make_map(&h->tm_hb[i], h->hb, h->T_max, d, bns[i]) &&
          make_map(&h->tm_ao[i], h->ao, h->T_max, c.n_heads * 64, bns[i]) &&
          make_map(&h->tm_act[i], h->act, h->T_max, F, bns[i]);
   }
@@ -673,7 +677,7 @@ int gs_prefill(gs_handle* h, int slot, const void* vis_emb, int n_vis, const int
     AL.fixed_slot = slot;
     const bool last = p0 + T >= P;
     rc = forward(h, T, text ? text + text0 : nullptr, vis ? vis + p0 * c.d_model : nullptr,
-                 vis_rows, AL, last ? T - 1 : 0, 1, h->packed_d, nullptr, false);
+                 vis_rows, AL, last ? T - 1 : 0, last ? 1 : 0, h->packed_d, nullptr, false);
     if (rc) return rc;
   }
   prefill_finish_kernel<<<1, 32, 0, h->stream>>>(h->packed_d, h->st, slot, static_cast<int>(P),
@@ -907,7 +911,7 @@ int gs_linear(const void* x, const void* w, void* y, int M, int N, int K, int ep
   if (!make_map(&tw, w, w_rows, K, epilogue == kEpiSwiGLU ? 64 : 128)) return GS_ERR_INVALID_ARG;
   if (!make_map(&tx, x, M, K, bn)) return GS_ERR_INVALID_ARG;
   Carver cv(scratch);
-  GemmArgs a;
+  GemmArgs a = {};
   a.err = cv.take<int>(64);
   a.counters = cv.take<int>(static_cast<size_t>(tok_tiles) * cdiv(N, 64));
   a.partial = split_k > 1

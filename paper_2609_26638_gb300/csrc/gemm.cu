@@ -21,6 +21,7 @@ static cudaError_t launch_bn(int epi, const CUtensorMap& tmW, const CUtensorMap&
     case kEpiResidF32: return launch_one<BN, kEpiResidF32>(tmW, tmX, a, ft, tt, s, pdl);
     case kEpiSwiGLU: return launch_one<BN, kEpiSwiGLU>(tmW, tmX, a, ft, tt, s, pdl);
     case kEpiArgmax: return launch_one<BN, kEpiArgmax>(tmW, tmX, a, ft, tt, s, pdl);
+    case kEpiQKV: return launch_one<BN, kEpiQKV>(tmW, tmX, a, ft, tt, s, pdl);
   }
   return cudaErrorInvalidValue;
 }
@@ -50,7 +51,10 @@ static cudaError_t set_attr_bn() {
   if ((e = cudaFuncSetAttribute(gemm_tc_kernel<BN, kEpiSwiGLU>,
                                 cudaFuncAttributeMaxDynamicSharedMemorySize, bytes)) != cudaSuccess)
     return e;
-  return cudaFuncSetAttribute(gemm_tc_kernel<BN, kEpiArgmax>,
+  if ((e = cudaFuncSetAttribute(gemm_tc_kernel<BN, kEpiArgmax>,
+                                cudaFuncAttributeMaxDynamicSharedMemorySize, bytes)) != cudaSuccess)
+    return e;
+  return cudaFuncSetAttribute(gemm_tc_kernel<BN, kEpiQKV>,
                               cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
 }
 

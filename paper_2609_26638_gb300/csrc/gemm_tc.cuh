@@ -22,14 +22,23 @@
 // start, so the result does not depend on the path or on arrival order.
 //
 // Epilogues: bf16 store, fp32 residual add, SwiGLU (gate and up rows of the
-// same features share a tile), and LM-head argmax (packed 64-bit atomicMax,
-// ties to the lowest index) with an optional fp32 logit dump.
+// same features share a tile), LM-head argmax (packed 64-bit atomicMax, ties
+// to the lowest index) with an optional fp32 logit dump, and the QKV epilogue
+// (RoPE on q and k, q to its buffer, k and v into the paged KV cache).
+//
+// RMSNorm is folded into the GEMMs: a residual epilogue also writes
+// hb = bf16(h * g) with the gain g of the norm that comes next, and the sum of
+// h^2 over its 128 features (one partial per feature tile, "ssp"); the GEMM
+// that consumes hb multiplies its accumulator by rsqrt(sum(ssp) / d + eps).
+// Since that factor is one scalar per token, this equals normalising first.
 #pragma once
 #include "ptx.cuh"
 
 namespace gs {
 
-enum GemmEpilogue : int { kEpiStoreBf16 = 0, kEpiResidF32 = 1, kEpiSwiGLU = 2, kEpiArgmax = 3 };
+enum GemmEpilogue : int {
+  kEpiStoreBf16 = 0, kEpiResidF32 = 1, kEpiSwiGLU = 2, kEpiArgmax = 3, kEpiQKV = 4
+};
 
 struct GemmArgs {
   int M;            // token rows
@@ -44,6 +53,23 @@ struct GemmArgs {
   int* counters;    // per output tile, zero between launches (cluster == 0)
   float* logits;    // argmax only: optional fp32 [M, N] dump
   int* err;
+  int x_row0;       // X (and ssp_in) row of token 0
+  // folded RMSNorm on the input: scale = rsqrt(sum_p ssp_in[t][p] * inv_d + eps)
+  const float* ssp_in;
+  int n_ssp;        // d / 128 partials per token
+  float inv_d, eps;
+  // residual epilogue extras: hb_out[t][f] = bf16(h[t][f] * g_next[f]); ssp_out[t][tile] = sum h^2
+  __nv_bfloat16* hb_out;
+  const __nv_bfloat16* g_next;
+  float* ssp_out;
+  // QKV epilogue
+  __nv_bfloat16* q_out;        // [M, Hq, 64]
+  __nv_bfloat16* kv_layer;     // this layer's page pool [pages][2][Hkv][64][64]
+  const int32_t* pos;          // [M] absolute slot
+  const int32_t* tok_slot;     // [M] page-table row, -1 = no KV write
+  const int32_t* page_table;
+  const float2* rope;          // [max_ctx][32] cos, sin
+  int pt_stride, n_pages, max_ctx, Hq, Hkv;
 };
 
 template <int BN>
@@ -55,9 +81,10 @@ struct GemmShape {
   static constexpr int kStages = BN <= 64 ? 4 : (BN <= 128 ? 3 : 4);
   static constexpr int kTmemCols = BN < 32 ? 32 : BN;
   static constexpr int kRedBytes = BN * 128 * 4;   // cluster reduction tile [BN][128] fp32
-  static constexpr int kXBufBytes = 32 * 64 * 4;   // SwiGLU gate/up exchange
+  static constexpr int kXBufBytes = 32 * 128 * 4;  // epilogue exchange (SwiGLU, RoPE, sums)
   static_assert(kRedBytes + kXBufBytes <= kStages * kStageBytes, "reduction smem");
-  static constexpr int kSmemBytes = kStages * kStageBytes + 1024 /*align*/ + 256 /*barriers*/;
+  // pipeline | barriers (256 B) | per-token norm scale (BN floats)
+  static constexpr int kSmemBytes = kStages * kStageBytes + 1024 /*align*/ + 256 + BN * 4;
 };
 
 // Epilogue of 32 consecutive tokens (t0 .. t0+31) of feature row `row`;
@@ -65,9 +92,14 @@ struct GemmShape {
 template <int BN, int EPI>
 __device__ __forceinline__ void gemm_epilogue_chunk(const GemmArgs& a, float (&v)[32], int row,
                                                     int feat_tile, int t0, int jlo, int jhi,
-                                                    float* xbuf) {
+                                                    float* xbuf, const float* rs) {
   const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
   jhi = min(jhi, a.M - t0);
+  if (rs != nullptr) {
+#pragma unroll
+    for (int j = 0; j < 32; ++j) v[j] *= rs[j];
+  }
   if constexpr (EPI == kEpiStoreBf16) {
     __nv_bfloat16* y = static_cast<__nv_bfloat16*>(a.y);
     const int f = feat_tile * 128 + row;
@@ -77,12 +109,87 @@ __device__ __forceinline__ void gemm_epilogue_chunk(const GemmArgs& a, float (&v
   } else if constexpr (EPI == kEpiResidF32) {
     float* y = static_cast<float*>(a.y);
     const int f = feat_tile * 128 + row;
+    const float g = a.hb_out ? __bfloat162float(a.g_next[f]) : 0.f;
 #pragma unroll
-    for (int j = 0; j < 32; ++j)
+    for (int j = 0; j < 32; ++j) {
+      float hsq = 0.f;
       if (j >= jlo && j < jhi) {
         float* p = y + static_cast<size_t>(t0 + j) * a.ldy + f;
-        *p = *p + v[j];
+        const float hn = *p + v[j];
+        *p = hn;
+        if (a.hb_out) a.hb_out[static_cast<size_t>(t0 + j) * a.ldy + f] = __float2bfloat16_rn(hn * g);
+        hsq = hn * hn;
       }
+      v[j] = hsq;
+    }
+    if (a.ssp_out != nullptr) {
+      // sum of h^2 over the tile's 128 features per token: warp tree, then 4 warps in order
+#pragma unroll
+      for (int j = 0; j < 32; ++j) {
+        float t = v[j];
+#pragma unroll
+        for (int m = 16; m >= 1; m >>= 1) t += __shfl_xor_sync(0xFFFFFFFFu, t, m);
+        if (lane == 0) xbuf[warp * 32 + j] = t;
+      }
+      asm volatile("bar.sync 2, 128;" ::: "memory");
+      if (threadIdx.x < 32) {
+        const int j = threadIdx.x;
+        if (j >= jlo && j < jhi)
+          a.ssp_out[static_cast<size_t>(t0 + j) * a.n_ssp + feat_tile] =
+              ((xbuf[j] + xbuf[32 + j]) + xbuf[64 + j]) + xbuf[96 + j];
+      }
+      asm volatile("bar.sync 2, 128;" ::: "memory");
+    }
+  } else if constexpr (EPI == kEpiQKV) {
+    // rows of this tile: two heads of 64; RoPE pairs row r with row r ^ 32
+    const int rbase = feat_tile * 128;
+    const int region = rbase < a.Hq * 64 ? 0 : (rbase < (a.Hq + a.Hkv) * 64 ? 1 : 2);
+    const int d = row & 63;
+    if (region < 2) {
+#pragma unroll
+      for (int j = 0; j < 32; ++j) xbuf[j * 128 + row] = v[j];
+      asm volatile("bar.sync 1, 128;" ::: "memory");
+#pragma unroll
+      for (int j = 0; j < 32; ++j) {
+        if (j >= jlo && j < jhi) {
+          const int p = a.pos[t0 + j];
+          if (p >= 0 && p < a.max_ctx) {
+            const float2 cs = a.rope[static_cast<size_t>(p) * 32 + (d & 31)];
+            const float pr = xbuf[j * 128 + (row ^ 32)];
+            v[j] = d < 32 ? v[j] * cs.x - pr * cs.y : v[j] * cs.x + pr * cs.y;
+          } else if (lane == 0) {
+            atomicExch(a.err, kErrBounds);
+          }
+        }
+      }
+      asm volatile("bar.sync 1, 128;" ::: "memory");
+    }
+    const int head = (rbase + row) / 64 - (region == 0 ? 0 : (region == 1 ? a.Hq : a.Hq + a.Hkv));
+    if (region == 0) {
+#pragma unroll
+      for (int j = 0; j < 32; ++j)
+        if (j >= jlo && j < jhi)
+          a.q_out[(static_cast<size_t>(t0 + j) * a.Hq + head) * 64 + d] = __float2bfloat16_rn(v[j]);
+    } else {
+      const int isv = region == 2 ? 1 : 0;
+#pragma unroll
+      for (int j = 0; j < 32; ++j) {
+        if (j >= jlo && j < jhi) {
+          const int slot = a.tok_slot[t0 + j];
+          const int p = a.pos[t0 + j];
+          if (slot < 0) continue;
+          const int lp = p >> 6;
+          const int phys = (p >= 0 && lp < a.pt_stride)
+                               ? a.page_table[static_cast<size_t>(slot) * a.pt_stride + lp] : -1;
+          if (phys < 0 || phys >= a.n_pages) {
+            atomicExch(a.err, kErrBounds);
+            continue;
+          }
+          a.kv_layer[((((static_cast<size_t>(phys) * 2 + isv) * a.Hkv + head) * 64 + (p & 63)) * 64) +
+                     d] = __float2bfloat16_rn(v[j]);
+        }
+      }
+    }
   } else if constexpr (EPI == kEpiSwiGLU) {
     // rows 0..63: gate of features f0..f0+63; rows 64..127: up of the same features
     if (warp >= 2) {
@@ -111,7 +218,6 @@ __device__ __forceinline__ void gemm_epilogue_chunk(const GemmArgs& a, float (&v
       for (int j = 0; j < 32; ++j)
         if (j >= jlo && j < jhi) a.logits[static_cast<size_t>(t0 + j) * a.N + f] = v[j];
     }
-    const int lane = threadIdx.x & 31;
 #pragma unroll
     for (int j = 0; j < 32; ++j) {
       unsigned long long key = argmax_key(v[j], f);
@@ -184,7 +290,7 @@ __global__ void __launch_bounds__(128, 1)
       }
     };
     auto load_x = [&](int i, int s) {
-      tma_load_2d(smem_u32(smB + s * S::kBBytes), &tmX, (kb0 + i) * 64, tok_tile * BN,
+      tma_load_2d(smem_u32(smB + s * S::kBBytes), &tmX, (kb0 + i) * 64, a.x_row0 + tok_tile * BN,
                   smem_u32(&full[s]), pol_x);
     };
     const int npre = nkb < S::kStages ? nkb : S::kStages;
@@ -233,6 +339,20 @@ __global__ void __launch_bounds__(128, 1)
   const uint32_t trow = tmem + (static_cast<uint32_t>(warp * 32) << 16);
   const int tok0 = tok_tile * BN;
   const bool failed = !acc_ok || *flag;
+  // folded RMSNorm: per-token scale of the input rows
+  float* rs_s = reinterpret_cast<float*>(smem + S::kStages * S::kStageBytes + 256);
+  if (a.ssp_in != nullptr) {
+    for (int t = threadIdx.x; t < BN; t += 128) {
+      float ss = 0.f;
+      if (tok0 + t < a.M) {
+        const float* sp = a.ssp_in + static_cast<size_t>(a.x_row0 + tok0 + t) * a.n_ssp;
+        for (int p = 0; p < a.n_ssp; ++p) ss += sp[p];
+      }
+      rs_s[t] = rsqrtf(ss * a.inv_d + a.eps);
+    }
+    __syncthreads();
+  }
+  auto rs_of = [&](int c) -> const float* { return a.ssp_in ? rs_s + c * 32 : nullptr; };
 
   if (a.splits == 1) {
     float* xbuf = reinterpret_cast<float*>(smA);   // pipeline smem is free after the accumulator
@@ -241,7 +361,7 @@ __global__ void __launch_bounds__(128, 1)
         if (tok0 + c * 32 >= a.M) break;   // uniform across the CTA
         float v[32];
         tmem_ld_32x32b_x32(trow + c * 32, v);
-        gemm_epilogue_chunk<BN, EPI>(a, v, row, feat_tile, tok0 + c * 32, 0, 32, xbuf);
+        gemm_epilogue_chunk<BN, EPI>(a, v, row, feat_tile, tok0 + c * 32, 0, 32, xbuf, rs_of(c));
       }
     }
     tc_fence_before();
@@ -282,7 +402,8 @@ __global__ void __launch_bounds__(128, 1)
         for (int j = 0; j < 32; ++j)
           if (j >= jlo && j < jhi) v[j] += peer[(c * 32 + j) * 128 + row];
       }
-      if (!failed) gemm_epilogue_chunk<BN, EPI>(a, v, row, feat_tile, tok0 + c * 32, jlo, jhi, xbuf);
+      if (!failed)
+        gemm_epilogue_chunk<BN, EPI>(a, v, row, feat_tile, tok0 + c * 32, jlo, jhi, xbuf, rs_of(c));
     }
     cluster_sync_all();   // peers may still be reading this CTA's partial tile
     return;
@@ -325,7 +446,7 @@ __global__ void __launch_bounds__(128, 1)
 #pragma unroll
       for (int j = 0; j < 32; ++j) v[j] += __ldcg(p + (c * 32 + j) * 128 + row);
     }
-    gemm_epilogue_chunk<BN, EPI>(a, v, row, feat_tile, tok0 + c * 32, 0, 32, xbuf);
+    gemm_epilogue_chunk<BN, EPI>(a, v, row, feat_tile, tok0 + c * 32, 0, 32, xbuf, rs_of(c));
   }
 }
 

@@ -115,7 +115,7 @@ extern "C" int gs_linear_noalloc(const void* x, const void* w, void* y, int M, i
   uint8_t* b = static_cast<uint8_t*>(base);
   // the split-K counters must start at zero; the array keeps the last call's contents
   if (cudaMemsetAsync(b, 0, err_bytes + cnt_bytes, s) != cudaSuccess) return GS_ERR_CUDA;
-  GemmArgs a;
+  GemmArgs a = {};
   a.err = reinterpret_cast<int*>(b);
   a.counters = reinterpret_cast<int*>(b + err_bytes);
   a.partial = split_k > 1 ? reinterpret_cast<float*>(b + err_bytes + cnt_bytes) : nullptr;

@@ -1,5 +1,5 @@
 // small.cuh -- bandwidth-trivial kernels of the round: window build, forcing,
-// embedding gather, RMSNorm, RoPE + paged KV write, accept/commit.
+// embedding gather (with the first norm's inputs), accept/commit.
 #pragma once
 #include "ptx.cuh"
 
@@ -191,9 +191,15 @@ __global__ void prefill_window_kernel(int T, int p0, int slot, int32_t* pos, int
   tok_slot[t] = slot;
 }
 
-// h[t] = E[tok[t]] (fp32), or the visual row for t < n_vis.  d % 8 == 0.
+// Row t of the residual stream: h[t] = E[tok[t]] (fp32), or the visual row for
+// t < n_vis.  Also writes what the first QKV GEMM consumes for its folded
+// RMSNorm -- hb[t] = bf16(h[t] * g0) and the per-128-feature sums of h^2 --
+// and zeroes the LM-head argmax key of the row.  One CTA of 128 threads per
+// row, 8 features per thread; d % 128 == 0.
 __global__ void embed_kernel(const int32_t* tok, const __nv_bfloat16* E, const __nv_bfloat16* vis,
-                             int n_vis, int T, int d, int vocab, float* h, int* err) {
+                             int n_vis, int T, int d, int vocab, float* h, __nv_bfloat16* hb,
+                             const __nv_bfloat16* g0, float* ssp, unsigned long long* keys,
+                             int* err) {
   pdl_wait();
   pdl_trigger();
   const int t = blockIdx.x;
@@ -209,116 +215,39 @@ __global__ void embed_kernel(const int32_t* tok, const __nv_bfloat16* E, const _
     }
     src = E + static_cast<size_t>(id) * d;
   }
+  const int n_ssp = d / 128;
   for (int c = threadIdx.x * 8; c < d; c += blockDim.x * 8) {
     const uint4 raw = *reinterpret_cast<const uint4*>(src + c);
+    const uint4 graw = *reinterpret_cast<const uint4*>(g0 + c);
     const __nv_bfloat162* p = reinterpret_cast<const __nv_bfloat162*>(&raw);
-    float4 lo, hi;
-    float2 f;
-    f = __bfloat1622float2(p[0]); lo.x = f.x; lo.y = f.y;
-    f = __bfloat1622float2(p[1]); lo.z = f.x; lo.w = f.y;
-    f = __bfloat1622float2(p[2]); hi.x = f.x; hi.y = f.y;
-    f = __bfloat1622float2(p[3]); hi.z = f.x; hi.w = f.y;
-    float* dst = h + static_cast<size_t>(t) * d + c;
-    *reinterpret_cast<float4*>(dst) = lo;
-    *reinterpret_cast<float4*>(dst + 4) = hi;
-  }
-}
-
-// RMSNorm, one warp per row: y = x / sqrt(mean(x^2) + eps) * gain -> bf16.
-// Optionally zeroes argmax keys of the row (the LM-head argmax accumulator).
-__global__ void rmsnorm_kernel(const float* x, const __nv_bfloat16* gain, __nv_bfloat16* y, int T,
-                               int d, float eps, unsigned long long* reset_keys) {
-  pdl_wait();
-  pdl_trigger();
-  const int row = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
-  const int lane = threadIdx.x & 31;
-  if (row >= T) return;
-  const float* xr = x + static_cast<size_t>(row) * d;
-  float ss = 0.f;
-  for (int c = lane * 4; c < d; c += 128) {
-    const float4 v = *reinterpret_cast<const float4*>(xr + c);
-    ss += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
-  }
+    const __nv_bfloat162* gp = reinterpret_cast<const __nv_bfloat162*>(&graw);
+    float x[8], o[8];
+    float sq = 0.f;
 #pragma unroll
-  for (int o = 16; o >= 1; o >>= 1) ss += __shfl_xor_sync(0xFFFFFFFFu, ss, o);
-  const float r = rsqrtf(ss / static_cast<float>(d) + eps);
-  __nv_bfloat16* yr = y + static_cast<size_t>(row) * d;
-  for (int c = lane * 4; c < d; c += 128) {
-    const float4 v = *reinterpret_cast<const float4*>(xr + c);
-    const __nv_bfloat162* g2 = reinterpret_cast<const __nv_bfloat162*>(gain + c);
-    const float2 ga = __bfloat1622float2(g2[0]), gb = __bfloat1622float2(g2[1]);
-    __nv_bfloat162 o0 = __floats2bfloat162_rn(v.x * r * ga.x, v.y * r * ga.y);
-    __nv_bfloat162 o1 = __floats2bfloat162_rn(v.z * r * gb.x, v.w * r * gb.y);
-    uint2 pk;
-    pk.x = *reinterpret_cast<uint32_t*>(&o0);
-    pk.y = *reinterpret_cast<uint32_t*>(&o1);
-    *reinterpret_cast<uint2*>(yr + c) = pk;
-  }
-  if (reset_keys != nullptr && lane == 0) reset_keys[row] = 0ull;
-}
-
-// RoPE (rotate-half, pairs (i, i+32)) on q and k at absolute positions, then
-// k and v written into the paged cache at the token's slot.  One warp per
-// (token, head) of the fused qkv row; lane i owns dims i and i+32.
-struct RopeKvArgs {
-  const __nv_bfloat16* qkv;   // [T, (Hq + 2 Hkv) * 64]
-  const int32_t* pos;         // [T]
-  const int32_t* tok_slot;    // [T] page-table row or -1
-  const float2* rope;         // [max_ctx][32] (cos, sin)
-  __nv_bfloat16* q_out;       // [T, Hq, 64]
-  __nv_bfloat16* kv;          // page pool of this layer: [pages][2][Hkv][64][64]
-  const int32_t* page_table;
-  int pt_stride, n_pages, T, Hq, Hkv, max_ctx;
-  int* err;
-};
-
-__global__ void rope_kv_kernel(RopeKvArgs a) {
-  pdl_wait();
-  pdl_trigger();
-  const int warps_per_block = blockDim.x >> 5;
-  const int gw = blockIdx.x * warps_per_block + (threadIdx.x >> 5);
-  const int lane = threadIdx.x & 31;
-  const int nh = a.Hq + 2 * a.Hkv;
-  if (gw >= a.T * nh) return;
-  const int t = gw / nh, hh = gw % nh;
-  const int p = a.pos[t];
-  const __nv_bfloat16* src = a.qkv + static_cast<size_t>(t) * nh * 64 + hh * 64;
-  const float x1 = __bfloat162float(src[lane]);
-  const float x2 = __bfloat162float(src[lane + 32]);
-  float y1 = x1, y2 = x2;
-  if (hh < a.Hq + a.Hkv) {
-    if (p < 0 || p >= a.max_ctx) {
-      if (lane == 0) atomicExch(a.err, kErrBounds);
-      return;
+    for (int i = 0; i < 4; ++i) {
+      const float2 f = __bfloat1622float2(p[i]);
+      const float2 g = __bfloat1622float2(gp[i]);
+      x[2 * i] = f.x;
+      x[2 * i + 1] = f.y;
+      o[2 * i] = f.x * g.x;
+      o[2 * i + 1] = f.y * g.y;
     }
-    const float2 cs = a.rope[static_cast<size_t>(p) * 32 + lane];
-    y1 = x1 * cs.x - x2 * cs.y;
-    y2 = x2 * cs.x + x1 * cs.y;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) sq += x[i] * x[i];
+    float* dst = h + static_cast<size_t>(t) * d + c;
+    *reinterpret_cast<float4*>(dst) = make_float4(x[0], x[1], x[2], x[3]);
+    *reinterpret_cast<float4*>(dst + 4) = make_float4(x[4], x[5], x[6], x[7]);
+    uint4 ob;
+    __nv_bfloat162* op = reinterpret_cast<__nv_bfloat162*>(&ob);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) op[i] = __floats2bfloat162_rn(o[2 * i], o[2 * i + 1]);
+    *reinterpret_cast<uint4*>(hb + static_cast<size_t>(t) * d + c) = ob;
+    // 16 consecutive threads cover one 128-feature block
+#pragma unroll
+    for (int m = 8; m >= 1; m >>= 1) sq += __shfl_xor_sync(0xFFFFFFFFu, sq, m);
+    if ((threadIdx.x & 15) == 0) ssp[static_cast<size_t>(t) * n_ssp + c / 128] = sq;
   }
-  if (hh < a.Hq) {
-    __nv_bfloat16* dst = a.q_out + (static_cast<size_t>(t) * a.Hq + hh) * 64;
-    dst[lane] = __float2bfloat16_rn(y1);
-    dst[lane + 32] = __float2bfloat16_rn(y2);
-    return;
-  }
-  const int slot = a.tok_slot[t];
-  if (slot < 0) return;
-  const int lp = p >> 6;
-  if (lp >= a.pt_stride) {
-    if (lane == 0) atomicExch(a.err, kErrBounds);
-    return;
-  }
-  const int phys = a.page_table[static_cast<size_t>(slot) * a.pt_stride + lp];
-  if (phys < 0 || phys >= a.n_pages) {
-    if (lane == 0) atomicExch(a.err, kErrBounds);
-    return;
-  }
-  const int is_v = hh >= a.Hq + a.Hkv;
-  const int kh = is_v ? hh - a.Hq - a.Hkv : hh - a.Hq;
-  __nv_bfloat16* dst = a.kv + ((((static_cast<size_t>(phys) * 2 + is_v) * a.Hkv + kh) * 64 +
-                                (p & 63)) * 64);
-  dst[lane] = __float2bfloat16_rn(y1);
-  dst[lane + 32] = __float2bfloat16_rn(y2);
+  if (threadIdx.x == 0 && keys != nullptr) keys[t] = 0ull;
 }
 
 // cos/sin table: angle p * theta^(-2i/64), computed in double precision.
