@@ -202,9 +202,12 @@ int gs_sync_check(gs_handle *h);
  *   page_table device int32 [n_seq, pt_stride]: logical page -> physical page
  *   n        device int32 [n_seq]: n_s
  *   out      device bf16 [n_seq, W, n_heads, 64]
- *   scratch  device, >= gs_attention_scratch_bytes(...) bytes, zeroed before
- *            its first use; the kernels leave it zeroed again
- *   split_pages pages per KV split (>= 1)
+ *   scratch  device, >= gs_attention_scratch_bytes(...) bytes (key limits and
+ *            the block -> page-table map; no split partials: the KV splits of a
+ *            (sequence, head) form one thread-block cluster and merge through
+ *            distributed shared memory)
+ *   split_pages pages per KV split (>= 1); raised to ceil(pt_stride / 8) when
+ *            a sequence would otherwise need more than 8 splits
  *   stream   cudaStream_t */
 size_t gs_attention_scratch_bytes(int n_seq, int W, int n_heads, int n_kv_heads, int max_pages,
                                   int split_pages);

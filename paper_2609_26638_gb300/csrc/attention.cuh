@@ -1,9 +1,9 @@
 // attention.cuh -- hybrid-mask attention over the paged bf16 KV cache.
 //
-// One CTA = (query block b, KV head h, KV split c).  A query block is a run of
+// One CTA = (KV split c, KV head h, query block b).  A query block is a run of
 // tokens of one sequence (the K+1 window of a decode forward, or 64 tokens of
 // a prefill chunk); its rows are (token, query head of the GQA group), so the
-// two query heads that share a KV head read each K/V page once.  Every query
+// query heads that share a KV head read each K/V page once.  Every query
 // token carries its own inclusive key limit, which encodes the mask: draft
 // boundary row n, draft mask rows n+K, verify row i n+1+i, prefill row p (paper
 // Appendix steps Draft forward / Verify forward).
@@ -15,13 +15,19 @@
 //
 // Splits cover fixed absolute page ranges [c*SP, (c+1)*SP), so a row's result
 // depends only on its own keys and not on the window it sits in; keys past a
-// row's limit contribute exact zeros.  With more than one split, each CTA
-// writes (O, m, l) partials and the last CTA of (b, h) merges them in split
-// order.
+// row's limit contribute exact zeros.  The splits of one (block, head) are one
+// thread-block cluster (at most kAttnMaxSplits CTAs): each CTA leaves its
+// (O, m, l) partial in its own shared memory and, after a cluster barrier,
+// merges a share of the rows over all peers through distributed shared memory
+// in split order.  A block whose keys fit in one split writes directly.
 #pragma once
 #include "ptx.cuh"
 
 namespace gs {
+
+constexpr int kAttnMaxSplits = 8;
+constexpr int kAttnStages = 4;
+constexpr int kAttnPageBytes = 64 * 128;  // 64 tokens x 64 bf16
 
 struct AttnArgs {
   const __nv_bfloat16* q;     // [T, Hq, 64]
@@ -36,24 +42,19 @@ struct AttnArgs {
   int Hq, Hkv, G;
   long long kv_row_base;      // first KV-map row of this layer
   int rows_per_page;          // 2 * Hkv * 64
-  int split_pages;            // SP
-  int max_splits;
-  int r_max;                  // QB * G rounded up to 16
-  float* part_o;              // [n_blocks][Hkv][max_splits][r_max][64]
-  float* part_ml;             // [n_blocks][Hkv][max_splits][r_max][2]
-  int* counters;              // [n_blocks][Hkv]
+  int split_pages;            // SP; gridDim.x (the cluster) * SP covers the block's pages
   int* err;
 };
 
-constexpr int kAttnStages = 4;
-constexpr int kAttnPageBytes = 64 * 128;  // 64 tokens x 64 bf16
-
-// Rows of Q staged in shared memory: at least 64 (four warps), so the split
-// merge always has 128 threads.
+// Rows of Q staged in shared memory: at least 64 (four warps).
 __host__ __device__ inline int attn_rows_alloc(int r_max) { return r_max < 64 ? 64 : r_max; }
 __host__ __device__ inline int attn_threads(int r_max) { return attn_rows_alloc(r_max) / 16 * 32; }
 __host__ __device__ inline int attn_smem_bytes(int r_max) {
   return 1024 + kAttnStages * 2 * kAttnPageBytes + attn_rows_alloc(r_max) * 128 + 64 + 64;
+}
+// Pages per split so that a sequence of `pages` pages needs at most kAttnMaxSplits splits.
+__host__ __device__ inline int attn_min_split_pages(int pages) {
+  return (pages + kAttnMaxSplits - 1) / kAttnMaxSplits;
 }
 
 __device__ __forceinline__ uint32_t sw128(int row, int chunk) {
@@ -95,18 +96,20 @@ __global__ void __launch_bounds__(512)
                                              ~static_cast<uintptr_t>(1023));
   uint8_t* sK = smem;                                     // [stages][64][128 B]
   uint8_t* sV = smem + kAttnStages * kAttnPageBytes;      // [stages][64][128 B]
-  uint8_t* sQ = smem + 2 * kAttnStages * kAttnPageBytes;  // [r_max][128 B]
-  uint64_t* full = reinterpret_cast<uint64_t*>(sQ + attn_rows_alloc(a.r_max) * 128);
+  uint8_t* sQ = smem + 2 * kAttnStages * kAttnPageBytes;  // [rows][128 B]
+  const int nthreads = blockDim.x;
+  const int rows_alloc = nthreads / 32 * 16;
+  uint64_t* full = reinterpret_cast<uint64_t*>(sQ + rows_alloc * 128);
   __shared__ int s_maxlim;
-  __shared__ int s_last;
 
   const int c = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
+  const int C = gridDim.x;                  // split slots = cluster size
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int nthreads = blockDim.x;
   // Before griddepcontrol.wait this kernel reads only what the kernel right
-  // before it (RoPE + KV write) does not write: the window descriptors (key
-  // limits, block slots), the page table, and cache pages wholly before the
-  // current window.
+  // before it (the QKV GEMM, which writes q and the window's K/V) does not
+  // write: the window descriptors (key limits, block slots), the page table,
+  // and cache pages wholly before the current window.  Every branch that
+  // leaves early is uniform across the cluster.
   if (a.blk_active != nullptr && a.blk_active[b] == 0) return;
   const int tok0 = b * a.QB;
   const int ntok = min(a.QB, a.T - tok0);
@@ -126,14 +129,13 @@ __global__ void __launch_bounds__(512)
   const int npages_blk = maxlim / 64 + 1;
   const int SP = a.split_pages;
   const int nsplit = (npages_blk + SP - 1) / SP;
-  if (c >= nsplit) return;
-  const int p_begin = c * SP;
-  const int p_end = min(npages_blk, p_begin + SP);
-  const int np = p_end - p_begin;
-  if (maxlim < 0 || npages_blk > a.pt_stride || slot < 0) {
+  if (maxlim < 0 || npages_blk > a.pt_stride || slot < 0 || nsplit > C) {
     if (threadIdx.x == 0) atomicExch(a.err, kErrBounds);
     return;
   }
+  if (nsplit == 1 && c > 0) return;         // direct path: CTA 0 alone
+  const int p_begin = c * SP;
+  const int np = c < nsplit ? min(npages_blk, p_begin + SP) - p_begin : 0;
   const int32_t* pt = a.page_table + static_cast<size_t>(slot) * a.pt_stride;
 
   if (threadIdx.x == 0) {
@@ -170,8 +172,7 @@ __global__ void __launch_bounds__(512)
   }
 
   // Q rows -> swizzled smem (zero rows past R)
-  const int nrows_pad = (nthreads / 32) * 16;
-  for (int idx = threadIdx.x; idx < nrows_pad * 8; idx += nthreads) {
+  for (int idx = threadIdx.x; idx < rows_alloc * 8; idx += nthreads) {
     const int r = idx >> 3, ch = idx & 7;
     uint4 v = make_uint4(0, 0, 0, 0);
     if (r < R) {
@@ -288,7 +289,7 @@ __global__ void __launch_bounds__(512)
     __syncthreads();
     if (threadIdx.x == 0 && ok && i + kAttnStages < np) issue(i + kAttnStages);
   }
-  if (!__syncthreads_and(ok)) return;
+  const bool all_ok = __syncthreads_and(ok);
 
   // row sums across the quad
   l0 += __shfl_xor_sync(0xFFFFFFFFu, l0, 1);
@@ -297,7 +298,7 @@ __global__ void __launch_bounds__(512)
   l1 += __shfl_xor_sync(0xFFFFFFFFu, l1, 2);
 
   if (nsplit == 1) {
-    if (has_rows) {
+    if (has_rows && all_ok) {
 #pragma unroll
       for (int half = 0; half < 2; ++half) {
         const int r = half ? r1 : r0;
@@ -316,90 +317,84 @@ __global__ void __launch_bounds__(512)
     return;
   }
 
-  // split partials
-  const size_t bh = static_cast<size_t>(b) * a.Hkv + h;
-  float* po = a.part_o + ((bh * a.max_splits + c) * a.r_max) * 64;
-  float* pml = a.part_ml + ((bh * a.max_splits + c) * a.r_max) * 2;
+  // ---- cluster merge.  Partials in this CTA's shared memory (stage buffers are free):
+  //      so [rows_alloc][64] fp32, sml [rows_alloc][2] = (m, l); empty rows: (0, -inf, 0).
+  float* so = reinterpret_cast<float*>(sK);
+  float* sml = so + rows_alloc * 64;
   if (has_rows) {
 #pragma unroll
     for (int half = 0; half < 2; ++half) {
       const int r = half ? r1 : r0;
-      if (r >= R) continue;
 #pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        *reinterpret_cast<float2*>(po + r * 64 + 8 * j + 2 * tq) =
+      for (int j = 0; j < 8; ++j)
+        *reinterpret_cast<float2*>(so + r * 64 + 8 * j + 2 * tq) =
             make_float2(o[j][half * 2 + 0], o[j][half * 2 + 1]);
-      }
       if (tq == 0) {
-        pml[r * 2 + 0] = half ? m1 : m0;
-        pml[r * 2 + 1] = half ? l1 : l0;
+        sml[r * 2 + 0] = half ? m1 : m0;
+        sml[r * 2 + 1] = half ? l1 : l0;
       }
+    }
+  } else {
+    for (int idx = lane; idx < 16 * 64; idx += 32) so[(warp * 16 + idx / 64) * 64 + idx % 64] = 0.f;
+    if (lane < 16) {
+      sml[(warp * 16 + lane) * 2 + 0] = -INFINITY;
+      sml[(warp * 16 + lane) * 2 + 1] = 0.f;
     }
   }
-  __threadfence();
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    const int old = atomicAdd(a.counters + bh, 1);
-    s_last = (old == nsplit - 1);
-    if (s_last) a.counters[bh] = 0;
-  }
-  __syncthreads();
-  if (!s_last) return;
-  __threadfence();
-  // Merge: stage (m, l) of every split for a group of rows in shared memory,
-  // turn them into weights exp2(m_s - M) / L per row, then each thread sums
-  // four output dims over the splits in order 0..S-1.  With one split holding
-  // all of a row's keys this reduces to O * (1 / l), the direct path's result.
-  const float* po0 = a.part_o + (bh * a.max_splits * a.r_max) * 64;
-  const float* pml0 = a.part_ml + (bh * a.max_splits * a.r_max) * 2;
-  float* sm_m = reinterpret_cast<float*>(sK);                 // [nsplit][RG]
-  float* sm_w = sm_m + (kAttnStages * 2 * kAttnPageBytes / 4) / 2;   // [nsplit][RG]
-  const int cap = (kAttnStages * 2 * kAttnPageBytes / 4) / 2;
-  const int RG = min(R, cap / nsplit);
-  for (int rg0 = 0; rg0 < R; rg0 += RG) {
-    const int nr = min(RG, R - rg0);
-    for (int idx = threadIdx.x; idx < nsplit * nr; idx += nthreads) {
-      const int sp = idx / nr, rr = idx % nr;
-      const float2 ml = __ldcg(reinterpret_cast<const float2*>(pml0 + (sp * a.r_max + rg0 + rr) * 2));
-      sm_m[sp * RG + rr] = ml.x;
-      sm_w[sp * RG + rr] = ml.y;
-    }
-    __syncthreads();
-    for (int rr = threadIdx.x; rr < nr; rr += nthreads) {
-      float M = -INFINITY;
-      for (int sp = 0; sp < nsplit; ++sp) M = fmaxf(M, sm_m[sp * RG + rr]);
-      float L = 0.f;
-      for (int sp = 0; sp < nsplit; ++sp) {
-        const float ms = sm_m[sp * RG + rr];
-        const float w = (ms == -INFINITY) ? 0.f : exp2f(ms - M);
-        sm_m[sp * RG + rr] = w;
-        L += w * sm_w[sp * RG + rr];
+  cluster_sync_all();
+  // CTA c merges rows c, c + C, c + 2C, ...; one thread per (row, 4 dims).
+  // Weights exp2(m_s - M) / L are summed over splits in order 0..C-1; with
+  // one split holding all of a row's keys this is O * (1 / l), the direct
+  // path's result.
+  const int my_rows = (R - c + C - 1) / C;
+  for (int idx = threadIdx.x; idx < my_rows * 16; idx += nthreads) {
+    const int r = c + (idx >> 4) * C;
+    const int d4 = (idx & 15) * 4;
+    float ms[kAttnMaxSplits], ls[kAttnMaxSplits];
+    float4 os[kAttnMaxSplits];
+#pragma unroll
+    for (int sp = 0; sp < kAttnMaxSplits; ++sp) {
+      if (sp < C) {
+        const float* pml = cluster_peer_ptr(sml + r * 2, static_cast<uint32_t>(sp));
+        const float* po = cluster_peer_ptr(so + r * 64 + d4, static_cast<uint32_t>(sp));
+        ms[sp] = pml[0];
+        ls[sp] = pml[1];
+        os[sp] = *reinterpret_cast<const float4*>(po);
       }
-      const float inv = 1.0f / L;
-      for (int sp = 0; sp < nsplit; ++sp) sm_w[sp * RG + rr] = sm_m[sp * RG + rr] * inv;
     }
-    __syncthreads();
-    for (int idx = threadIdx.x; idx < nr * 16; idx += nthreads) {
-      const int rr = idx >> 4, d4 = (idx & 15) * 4;
-      const int r = rg0 + rr;
-      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll 4
-      for (int sp = 0; sp < nsplit; ++sp) {
-        const float w = sm_w[sp * RG + rr];
-        const float4 v = __ldcg(reinterpret_cast<const float4*>(po0 + (sp * a.r_max + r) * 64 + d4));
-        acc.x += w * v.x;
-        acc.y += w * v.y;
-        acc.z += w * v.z;
-        acc.w += w * v.w;
+    float M = -INFINITY;
+#pragma unroll
+    for (int sp = 0; sp < kAttnMaxSplits; ++sp)
+      if (sp < C) M = fmaxf(M, ms[sp]);
+    float L = 0.f;
+#pragma unroll
+    for (int sp = 0; sp < kAttnMaxSplits; ++sp) {
+      if (sp < C) {
+        ms[sp] = (ms[sp] == -INFINITY) ? 0.f : exp2f(ms[sp] - M);
+        L += ms[sp] * ls[sp];
       }
+    }
+    const float inv = 1.0f / L;
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+    for (int sp = 0; sp < kAttnMaxSplits; ++sp) {
+      if (sp < C) {
+        const float w = ms[sp] * inv;
+        acc.x += w * os[sp].x;
+        acc.y += w * os[sp].y;
+        acc.z += w * os[sp].z;
+        acc.w += w * os[sp].w;
+      }
+    }
+    if (all_ok) {
       const int t = tok0 + r / a.G;
       const int hq = h * a.G + r % a.G;
       __nv_bfloat16* dst = a.out + (static_cast<size_t>(t) * a.Hq + hq) * 64 + d4;
       *reinterpret_cast<__nv_bfloat162*>(dst) = __floats2bfloat162_rn(acc.x, acc.y);
       *reinterpret_cast<__nv_bfloat162*>(dst + 2) = __floats2bfloat162_rn(acc.z, acc.w);
     }
-    __syncthreads();
   }
+  cluster_sync_all();   // peers may still be reading this CTA's partials
 }
 
 }  // namespace gs

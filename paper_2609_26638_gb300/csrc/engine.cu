@@ -130,8 +130,6 @@ struct gs_handle {
   int32_t *draft_tok = nullptr, *verify_in = nullptr, *verify_tok = nullptr;
   float* gemm_partial = nullptr;
   int* gemm_counters = nullptr;
-  float *attn_po = nullptr, *attn_pml = nullptr;
-  int* attn_counters = nullptr;
 
   // host page bookkeeping
   std::vector<int> free_pages;
@@ -196,8 +194,10 @@ size_t carve(gs_handle* h, const gs_config& c, void* base) {
   const int W_max = c.max_K + 1;
   int T_max = std::max(c.max_batch * W_max, c.max_prefill);
   T_max = static_cast<int>(align_up(std::max(T_max, 256), 256));
+  // attention splits: fixed page ranges, at most kAttnMaxSplits per sequence (one cluster)
   int sp = c.split_pages;
   if (sp <= 0) sp = std::max(1, cdiv(static_cast<long long>(pt_stride) * c.max_batch * c.n_kv_heads, 304));
+  sp = std::max(sp, attn_min_split_pages(pt_stride));
   const int max_splits = cdiv(pt_stride, sp);
   const int r_max = round16(W_max * G);
 
@@ -232,10 +232,6 @@ size_t carve(gs_handle* h, const gs_config& c, void* base) {
   int32_t* verify_tok = cv.take<int32_t>(static_cast<size_t>(c.max_batch) * W_max);
   float* gemm_partial = cv.take<float>(kGemmPartialFloats);
   int* gemm_counters = cv.take<int>(kGemmCounters);
-  const size_t bh = static_cast<size_t>(c.max_batch) * c.n_kv_heads;
-  float* attn_po = cv.take<float>(bh * max_splits * r_max * 64);
-  float* attn_pml = cv.take<float>(bh * max_splits * r_max * 2);
-  int* attn_counters = cv.take<int>(bh);
 
   if (h) {
     h->G = G;
@@ -271,9 +267,6 @@ size_t carve(gs_handle* h, const gs_config& c, void* base) {
     h->verify_tok = verify_tok;
     h->gemm_partial = gemm_partial;
     h->gemm_counters = gemm_counters;
-    h->attn_po = attn_po;
-    h->attn_pml = attn_pml;
-    h->attn_counters = attn_counters;
   }
   return align_up(cv.off, 256);
 }
@@ -332,15 +325,11 @@ int run_attention(gs_handle* h, int layer, int T, const AttnLaunch& L) {
   a.rows_per_page = 2 * c.n_kv_heads * 64;
   a.kv_row_base = static_cast<long long>(layer) * h->n_pages * a.rows_per_page;
   a.split_pages = L.split_pages;
-  a.max_splits = L.max_splits;
-  a.r_max = L.r_max;
-  a.part_o = h->attn_po;
-  a.part_ml = h->attn_pml;
-  a.counters = h->attn_counters;
   a.err = h->err_word;
   dim3 grid(L.max_splits, c.n_kv_heads, L.n_blocks);
   GS_CUDA(h, launch_ex(attn_paged_kernel, grid, dim3(attn_threads(L.r_max)),
-                       attn_smem_bytes(L.r_max), h->stream, true, 1, h->tm_kv, a));
+                       attn_smem_bytes(L.r_max), h->stream, true, dim3(L.max_splits, 1, 1), h->tm_kv,
+                       a));
   ++h->launches;
   return GS_OK;
 }
@@ -356,7 +345,7 @@ int forward(gs_handle* h, int T, const int32_t* tok, const __nv_bfloat16* vis, i
             float* logits, bool decode) {
   const gs_config& c = h->cfg;
   const int d = c.d_model, F = c.d_ffn, HD = c.n_heads * 64, L = c.n_layers;
-  GS_CUDA(h, launch_ex(embed_kernel, dim3(T), dim3(128), 0, h->stream, true, 1, tok, h->embed, vis,
+  GS_CUDA(h, launch_ex(embed_kernel, dim3(T), dim3(128), 0, h->stream, true, dim3(1), tok, h->embed, vis,
                        n_vis, T, d, c.vocab, h->hbuf, h->hb, h->attn_norm[0], h->ssp, packed,
                        h->err_word));
   ++h->launches;
@@ -453,12 +442,12 @@ int enqueue_round(gs_handle* h, const int32_t* slots, int n_seq, int K, const gs
   AL.fixed_slot = -1;
 
   h->launches = 0;
-  GS_CUDA(h, launch_ex(window_draft_kernel, dim3(nb), dim3(128), 0, h->stream, true, 1, w));
+  GS_CUDA(h, launch_ex(window_draft_kernel, dim3(nb), dim3(128), 0, h->stream, true, dim3(1), w));
   ++h->launches;
   int rc = forward(h, T, h->tok, nullptr, 0, AL, 0, T, h->packed_d,
                    dbg ? dbg->draft_logits : nullptr, true);
   if (rc) return rc;
-  GS_CUDA(h, launch_ex(window_verify_kernel, dim3(nb), dim3(128), 0, h->stream, true, 1, w));
+  GS_CUDA(h, launch_ex(window_verify_kernel, dim3(nb), dim3(128), 0, h->stream, true, dim3(1), w));
   ++h->launches;
   rc = forward(h, T, h->tok, nullptr, 0, AL, 0, T, h->packed_v, dbg ? dbg->verify_logits : nullptr,
                true);
@@ -476,7 +465,7 @@ int enqueue_round(gs_handle* h, const int32_t* slots, int n_seq, int K, const gs
   ac.out_tok = out_tok;
   ac.out_cnt = out_cnt;
   ac.out_done = out_done;
-  GS_CUDA(h, launch_ex(accept_commit_kernel, dim3(cdiv(n_seq, 64)), dim3(64), 0, h->stream, true, 1,
+  GS_CUDA(h, launch_ex(accept_commit_kernel, dim3(cdiv(n_seq, 64)), dim3(64), 0, h->stream, true, dim3(1),
                        ac));
   ++h->launches;
   if (dbg) {
@@ -784,16 +773,10 @@ size_t gs_attention_scratch_bytes(int n_seq, int W, int n_heads, int n_kv_heads,
   if (n_seq < 1 || W < 1 || n_kv_heads < 1 || n_heads % n_kv_heads || max_pages < 1 ||
       split_pages < 1)
     return 0;
-  const int G = n_heads / n_kv_heads;
-  const int r_max = round16(W * G);
-  const int ms = cdiv(max_pages, split_pages);
   Carver cv(nullptr);
-  cv.take<int>(64);                        // error word
-  cv.take<int32_t>(static_cast<size_t>(n_seq) * W);  // lim
-  cv.take<int32_t>(n_seq);                 // blk_slot
-  cv.take<int>(static_cast<size_t>(n_seq) * n_kv_heads);
-  cv.take<float>(static_cast<size_t>(n_seq) * n_kv_heads * ms * r_max * 2);
-  cv.take<float>(static_cast<size_t>(n_seq) * n_kv_heads * ms * r_max * 64);
+  cv.take<int>(64);                                   // error word
+  cv.take<int32_t>(static_cast<size_t>(n_seq) * W);  // key limits
+  cv.take<int32_t>(n_seq);                            // block -> page-table row
   return align_up(cv.off, 256);
 }
 
@@ -835,14 +818,12 @@ int gs_attention(int mode, const void* q, const void* kv, int n_pages, const int
     attr = true;
   }
   const int r_max = round16(W * G);
-  const int ms = cdiv(pt_stride, split_pages);
+  const int sp = std::max(split_pages, attn_min_split_pages(pt_stride));
+  const int ms = cdiv(pt_stride, sp);
   Carver cv(scratch);
   int* err = cv.take<int>(64);
   int32_t* lim = cv.take<int32_t>(static_cast<size_t>(n_seq) * W);
   int32_t* blk_slot = cv.take<int32_t>(n_seq);
-  int* counters = cv.take<int>(static_cast<size_t>(n_seq) * n_kv_heads);
-  float* pml = cv.take<float>(static_cast<size_t>(n_seq) * n_kv_heads * ms * r_max * 2);
-  float* po = cv.take<float>(static_cast<size_t>(n_seq) * n_kv_heads * ms * r_max * 64);
   CUtensorMap tm;
   const uint64_t rows = static_cast<uint64_t>(n_pages) * 2 * n_kv_heads * 64;
   if (rows >= (1ull << 31) || !make_map(&tm, kv, rows, 64, 64)) return GS_ERR_INVALID_ARG;
@@ -864,16 +845,13 @@ int gs_attention(int mode, const void* q, const void* kv, int n_pages, const int
   a.G = G;
   a.rows_per_page = 2 * n_kv_heads * 64;
   a.kv_row_base = 0;
-  a.split_pages = split_pages;
-  a.max_splits = ms;
-  a.r_max = r_max;
-  a.part_o = po;
-  a.part_ml = pml;
-  a.counters = counters;
+  a.split_pages = sp;
   a.err = err;
   dim3 grid(ms, n_kv_heads, n_seq);
-  attn_paged_kernel<<<grid, attn_threads(r_max), attn_smem_bytes(r_max), s>>>(tm, a);
-  return cudaGetLastError() == cudaSuccess ? GS_OK : GS_ERR_CUDA;
+  return launch_ex(attn_paged_kernel, grid, dim3(attn_threads(r_max)), attn_smem_bytes(r_max), s,
+                   false, dim3(ms, 1, 1), tm, a) == cudaSuccess
+             ? GS_OK
+             : GS_ERR_CUDA;
 }
 
 size_t gs_linear_scratch_bytes(int M, int N, int split_k) {

@@ -83,16 +83,28 @@ struct GemmShape {
   static constexpr int kRedBytes = BN * 128 * 4;   // cluster reduction tile [BN][128] fp32
   static constexpr int kXBufBytes = 32 * 128 * 4;  // epilogue exchange (SwiGLU, RoPE, sums)
   static_assert(kRedBytes + kXBufBytes <= kStages * kStageBytes, "reduction smem");
-  // pipeline | barriers (256 B) | per-token norm scale (BN floats)
-  static constexpr int kSmemBytes = kStages * kStageBytes + 1024 /*align*/ + 256 + BN * 4;
+  // pipeline | barriers (256 B) | per token: norm scale (4 B), KV destination (8 B), position (4 B)
+  static constexpr int kSmemBytes = kStages * kStageBytes + 1024 /*align*/ + 256 + 16 * BN;
 };
 
 // Epilogue of 32 consecutive tokens (t0 .. t0+31) of feature row `row`;
 // only tokens j in [jlo, jhi) with t0 + j < M are produced.
+__device__ __forceinline__ int isv_of(int region) { return region == 2 ? 1 : 0; }
+
+// Per-token data the epilogue needs, staged in shared memory while the
+// mainloop runs: rs = folded-norm scale, kvdst = element offset of the token's
+// row in its KV page (-1: no write), pos = absolute slot.
+struct TokMeta {
+  const float* rs;
+  const long long* kvdst;
+  const int* pos;
+};
+
 template <int BN, int EPI>
 __device__ __forceinline__ void gemm_epilogue_chunk(const GemmArgs& a, float (&v)[32], int row,
                                                     int feat_tile, int t0, int jlo, int jhi,
-                                                    float* xbuf, const float* rs) {
+                                                    float* xbuf, TokMeta tm) {
+  const float* rs = tm.rs;
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   jhi = min(jhi, a.M - t0);
@@ -110,13 +122,16 @@ __device__ __forceinline__ void gemm_epilogue_chunk(const GemmArgs& a, float (&v
     float* y = static_cast<float*>(a.y);
     const int f = feat_tile * 128 + row;
     const float g = a.hb_out ? __bfloat162float(a.g_next[f]) : 0.f;
+    float hv[32];
+#pragma unroll
+    for (int j = 0; j < 32; ++j)   // all loads first: one round trip, not 32
+      hv[j] = (j >= jlo && j < jhi) ? y[static_cast<size_t>(t0 + j) * a.ldy + f] : 0.f;
 #pragma unroll
     for (int j = 0; j < 32; ++j) {
       float hsq = 0.f;
       if (j >= jlo && j < jhi) {
-        float* p = y + static_cast<size_t>(t0 + j) * a.ldy + f;
-        const float hn = *p + v[j];
-        *p = hn;
+        const float hn = hv[j] + v[j];
+        y[static_cast<size_t>(t0 + j) * a.ldy + f] = hn;
         if (a.hb_out) a.hb_out[static_cast<size_t>(t0 + j) * a.ldy + f] = __float2bfloat16_rn(hn * g);
         hsq = hn * hn;
       }
@@ -149,17 +164,18 @@ __device__ __forceinline__ void gemm_epilogue_chunk(const GemmArgs& a, float (&v
 #pragma unroll
       for (int j = 0; j < 32; ++j) xbuf[j * 128 + row] = v[j];
       asm volatile("bar.sync 1, 128;" ::: "memory");
+      float2 cs[32];
+#pragma unroll
+      for (int j = 0; j < 32; ++j) {   // all table loads first
+        const int p = tm.pos[j];
+        cs[j] = (j >= jlo && j < jhi && p >= 0 && p < a.max_ctx)
+                    ? a.rope[static_cast<size_t>(p) * 32 + (d & 31)] : make_float2(1.f, 0.f);
+      }
 #pragma unroll
       for (int j = 0; j < 32; ++j) {
         if (j >= jlo && j < jhi) {
-          const int p = a.pos[t0 + j];
-          if (p >= 0 && p < a.max_ctx) {
-            const float2 cs = a.rope[static_cast<size_t>(p) * 32 + (d & 31)];
-            const float pr = xbuf[j * 128 + (row ^ 32)];
-            v[j] = d < 32 ? v[j] * cs.x - pr * cs.y : v[j] * cs.x + pr * cs.y;
-          } else if (lane == 0) {
-            atomicExch(a.err, kErrBounds);
-          }
+          const float pr = xbuf[j * 128 + (row ^ 32)];
+          v[j] = d < 32 ? v[j] * cs[j].x - pr * cs[j].y : v[j] * cs[j].x + pr * cs[j].y;
         }
       }
       asm volatile("bar.sync 1, 128;" ::: "memory");
@@ -171,23 +187,12 @@ __device__ __forceinline__ void gemm_epilogue_chunk(const GemmArgs& a, float (&v
         if (j >= jlo && j < jhi)
           a.q_out[(static_cast<size_t>(t0 + j) * a.Hq + head) * 64 + d] = __float2bfloat16_rn(v[j]);
     } else {
-      const int isv = region == 2 ? 1 : 0;
+      // kvdst[j]: offset of (page, K, head 0, row p & 63, dim 0); V is Hkv * 4096 further
+      const long long off = (static_cast<long long>(isv_of(region)) * a.Hkv + head) * 4096 + d;
 #pragma unroll
       for (int j = 0; j < 32; ++j) {
-        if (j >= jlo && j < jhi) {
-          const int slot = a.tok_slot[t0 + j];
-          const int p = a.pos[t0 + j];
-          if (slot < 0) continue;
-          const int lp = p >> 6;
-          const int phys = (p >= 0 && lp < a.pt_stride)
-                               ? a.page_table[static_cast<size_t>(slot) * a.pt_stride + lp] : -1;
-          if (phys < 0 || phys >= a.n_pages) {
-            atomicExch(a.err, kErrBounds);
-            continue;
-          }
-          a.kv_layer[((((static_cast<size_t>(phys) * 2 + isv) * a.Hkv + head) * 64 + (p & 63)) * 64) +
-                     d] = __float2bfloat16_rn(v[j]);
-        }
+        const long long base = tm.kvdst[j];
+        if (j >= jlo && j < jhi && base >= 0) a.kv_layer[base + off] = __float2bfloat16_rn(v[j]);
       }
     }
   } else if constexpr (EPI == kEpiSwiGLU) {
@@ -312,6 +317,41 @@ __global__ void __launch_bounds__(128, 1)
   } else {
     pdl_wait();
     pdl_trigger();
+    if (warp >= 2) {
+      // idle during the mainloop: stage the epilogue's per-token inputs
+      float* rs_s = reinterpret_cast<float*>(smem + S::kStages * S::kStageBytes + 256);
+      long long* kvdst_s = reinterpret_cast<long long*>(rs_s + BN);
+      int* pos_s = reinterpret_cast<int*>(kvdst_s + BN);
+      const int tok0 = tok_tile * BN;
+      for (int t = threadIdx.x - 64; t < BN; t += 64) {
+        const bool valid = tok0 + t < a.M;
+        if (a.ssp_in != nullptr) {
+          float ss = 0.f;
+          if (valid) {
+            const float* sp = a.ssp_in + static_cast<size_t>(a.x_row0 + tok0 + t) * a.n_ssp;
+            for (int p = 0; p < a.n_ssp; ++p) ss += sp[p];
+          }
+          rs_s[t] = rsqrtf(ss * a.inv_d + a.eps);
+        }
+        if constexpr (EPI == kEpiQKV) {
+          long long dst = -1;
+          int p = -1;
+          if (valid) {
+            p = a.pos[tok0 + t];
+            const int slot = a.tok_slot[tok0 + t];
+            if (slot >= 0) {
+              const int lp = p >> 6;
+              const int phys = (p >= 0 && p < a.max_ctx && lp < a.pt_stride)
+                                   ? a.page_table[static_cast<size_t>(slot) * a.pt_stride + lp] : -1;
+              if (phys < 0 || phys >= a.n_pages) atomicExch(a.err, kErrBounds);
+              else dst = static_cast<long long>(phys) * 2 * a.Hkv * 4096 + (p & 63) * 64;
+            }
+          }
+          kvdst_s[t] = dst;
+          pos_s[t] = p;
+        }
+      }
+    }
     if (warp == 1 && lane == 0) {
       // MMA issuer
       constexpr uint32_t idesc = umma_idesc_bf16(128, BN);
@@ -339,20 +379,14 @@ __global__ void __launch_bounds__(128, 1)
   const uint32_t trow = tmem + (static_cast<uint32_t>(warp * 32) << 16);
   const int tok0 = tok_tile * BN;
   const bool failed = !acc_ok || *flag;
-  // folded RMSNorm: per-token scale of the input rows
-  float* rs_s = reinterpret_cast<float*>(smem + S::kStages * S::kStageBytes + 256);
-  if (a.ssp_in != nullptr) {
-    for (int t = threadIdx.x; t < BN; t += 128) {
-      float ss = 0.f;
-      if (tok0 + t < a.M) {
-        const float* sp = a.ssp_in + static_cast<size_t>(a.x_row0 + tok0 + t) * a.n_ssp;
-        for (int p = 0; p < a.n_ssp; ++p) ss += sp[p];
-      }
-      rs_s[t] = rsqrtf(ss * a.inv_d + a.eps);
-    }
-    __syncthreads();
-  }
-  auto rs_of = [&](int c) -> const float* { return a.ssp_in ? rs_s + c * 32 : nullptr; };
+  // per-token epilogue inputs staged by warps 2-3 during the mainloop
+  __syncthreads();
+  const float* rs_s = reinterpret_cast<const float*>(smem + S::kStages * S::kStageBytes + 256);
+  const long long* kvdst_s = reinterpret_cast<const long long*>(rs_s + BN);
+  const int* pos_s = reinterpret_cast<const int*>(kvdst_s + BN);
+  auto rs_of = [&](int c) -> TokMeta {
+    return TokMeta{a.ssp_in ? rs_s + c * 32 : nullptr, kvdst_s + c * 32, pos_s + c * 32};
+  };
 
   if (a.splits == 1) {
     float* xbuf = reinterpret_cast<float*>(smA);   // pipeline smem is free after the accumulator

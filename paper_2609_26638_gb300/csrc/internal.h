@@ -11,10 +11,10 @@ namespace gs {
 struct GemmArgs;
 
 // cudaLaunchKernelEx with optional programmatic stream serialisation (PDL) and
-// a cluster along z.
+// an optional thread-block cluster shape.
 template <typename... KArgs, typename... Args>
 cudaError_t launch_ex(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
-                      cudaStream_t s, bool pdl, int cluster_z, Args&&... args) {
+                      cudaStream_t s, bool pdl, dim3 cluster, Args&&... args) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = grid;
   cfg.blockDim = block;
@@ -27,11 +27,11 @@ cudaError_t launch_ex(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t sm
     attrs[n].val.programmaticStreamSerializationAllowed = 1;
     ++n;
   }
-  if (cluster_z > 1) {
+  if (cluster.x * cluster.y * cluster.z > 1) {
     attrs[n].id = cudaLaunchAttributeClusterDimension;
-    attrs[n].val.clusterDim.x = 1;
-    attrs[n].val.clusterDim.y = 1;
-    attrs[n].val.clusterDim.z = cluster_z;
+    attrs[n].val.clusterDim.x = cluster.x;
+    attrs[n].val.clusterDim.y = cluster.y;
+    attrs[n].val.clusterDim.z = cluster.z;
     ++n;
   }
   cfg.attrs = attrs;
