@@ -9,9 +9,14 @@
 // Appendix steps Draft forward / Verify forward).
 //
 // K and V pages (64 tokens x 64 dims, 8 KB each) are staged by TMA with
-// 128-byte swizzle into a ring of shared-memory stages; each warp owns 16 rows
-// and runs S = Q K^T and O += P V on mma.sync m16n8k16 (bf16 in, fp32 out),
-// with the online softmax in registers (exp2 with the 1/sqrt(64) scale folded).
+// 128-byte swizzle into a ring of shared-memory stages.  Warps form NG groups
+// of one warp per 16 rows; group g takes the split's pages g, g+NG, ... so NG
+// pages are in work at once.  Each warp runs S = Q K^T and O += P V on
+// mma.sync m16n8k16 (bf16 in, fp32 out) with the online softmax in registers
+// (exp2 with the 1/sqrt(64) scale folded); the groups' partials merge in
+// shared memory in group order.  NG depends only on the row count (4 up to 64
+// rows, 2 up to 128, else 1), so windows with the same group count give
+// bit-identical rows.
 //
 // Splits cover fixed absolute page ranges [c*SP, (c+1)*SP), so a row's result
 // depends only on its own keys and not on the window it sits in; keys past a
@@ -26,7 +31,7 @@
 namespace gs {
 
 constexpr int kAttnMaxSplits = 8;
-constexpr int kAttnStages = 4;
+constexpr int kAttnStages = 8;
 constexpr int kAttnPageBytes = 64 * 128;  // 64 tokens x 64 bf16
 
 struct AttnArgs {
@@ -46,11 +51,16 @@ struct AttnArgs {
   int* err;
 };
 
-// Rows of Q staged in shared memory: at least 64 (four warps).
-__host__ __device__ inline int attn_rows_alloc(int r_max) { return r_max < 64 ? 64 : r_max; }
-__host__ __device__ inline int attn_threads(int r_max) { return attn_rows_alloc(r_max) / 16 * 32; }
+// Rows (16 per warp), warp groups and threads for a block of r_max rows.
+__host__ __device__ inline int attn_mtiles(int r_max) { return (r_max + 15) / 16; }
+__host__ __device__ inline int attn_groups(int r_max) {
+  return attn_mtiles(r_max) <= 4 ? 4 : (attn_mtiles(r_max) <= 8 ? 2 : 1);
+}
+__host__ __device__ inline int attn_threads(int r_max) {
+  return attn_mtiles(r_max) * attn_groups(r_max) * 32;
+}
 __host__ __device__ inline int attn_smem_bytes(int r_max) {
-  return 1024 + kAttnStages * 2 * kAttnPageBytes + attn_rows_alloc(r_max) * 128 + 64 + 64;
+  return 1024 + kAttnStages * 2 * kAttnPageBytes + attn_mtiles(r_max) * 16 * 128 + 128 + 64;
 }
 // Pages per split so that a sequence of `pages` pages needs at most kAttnMaxSplits splits.
 __host__ __device__ inline int attn_min_split_pages(int pages) {
@@ -98,13 +108,16 @@ __global__ void __launch_bounds__(512)
   uint8_t* sV = smem + kAttnStages * kAttnPageBytes;      // [stages][64][128 B]
   uint8_t* sQ = smem + 2 * kAttnStages * kAttnPageBytes;  // [rows][128 B]
   const int nthreads = blockDim.x;
-  const int rows_alloc = nthreads / 32 * 16;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int mtiles = attn_mtiles(a.QB * a.G);
+  const int NG = nthreads / 32 / mtiles;    // warp groups
+  const int grp = warp / mtiles, mt = warp % mtiles;
+  const int rows_alloc = mtiles * 16;
   uint64_t* full = reinterpret_cast<uint64_t*>(sQ + rows_alloc * 128);
   __shared__ int s_maxlim;
 
   const int c = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
   const int C = gridDim.x;                  // split slots = cluster size
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   // Before griddepcontrol.wait this kernel reads only what the kernel right
   // before it (the QKV GEMM, which writes q and the window's K/V) does not
   // write: the window descriptors (key limits, block slots), the page table,
@@ -184,9 +197,9 @@ __global__ void __launch_bounds__(512)
   }
   __syncthreads();
 
-  const bool has_rows = warp * 16 < R;
+  const bool has_rows = mt * 16 < R;
   const int g = lane >> 2, tq = lane & 3;
-  const int r0 = warp * 16 + g, r1 = r0 + 8;
+  const int r0 = mt * 16 + g, r1 = r0 + 8;
   const int lim0 = r0 < R ? a.lim[tok0 + r0 / a.G] : -1;
   const int lim1 = r1 < R ? a.lim[tok0 + r1 / a.G] : -1;
 
@@ -194,7 +207,7 @@ __global__ void __launch_bounds__(512)
   if (has_rows) {
 #pragma unroll
     for (int kk = 0; kk < 4; ++kk) {
-      const int row = warp * 16 + (lane & 15);
+      const int row = mt * 16 + (lane & 15);
       const int ch = 2 * kk + (lane >> 4);
       ldsm_x4(smem_u32(sQ) + sw128(row, ch), qa[kk][0], qa[kk][1], qa[kk][2], qa[kk][3]);
     }
@@ -207,10 +220,12 @@ __global__ void __launch_bounds__(512)
   for (int j = 0; j < 8; ++j) o[j][0] = o[j][1] = o[j][2] = o[j][3] = 0.f;
   bool ok = true;
 
-  for (int i = 0; i < np; ++i) {
+  for (int it = 0; it * NG < np; ++it) {
+    const int i = it * NG + grp;              // this group's page of the iteration
     const int s = i % kAttnStages;
-    if (ok && !mbar_wait(smem_u32(&full[s]), (i / kAttnStages) & 1, a.err)) ok = false;
-    if (ok && has_rows) {
+    const bool mine = i < np;
+    if (ok && mine && !mbar_wait(smem_u32(&full[s]), (i / kAttnStages) & 1, a.err)) ok = false;
+    if (ok && mine && has_rows) {
       const uint32_t kbase = smem_u32(sK + s * kAttnPageBytes);
       const uint32_t vbase = smem_u32(sV + s * kAttnPageBytes);
       float sacc[8][4];
@@ -287,7 +302,10 @@ __global__ void __launch_bounds__(512)
       }
     }
     __syncthreads();
-    if (threadIdx.x == 0 && ok && i + kAttnStages < np) issue(i + kAttnStages);
+    if (threadIdx.x == 0 && ok) {
+      for (int q = it * NG; q < it * NG + NG; ++q)
+        if (q + kAttnStages < np) issue(q + kAttnStages);
+    }
   }
   const bool all_ok = __syncthreads_and(ok);
 
@@ -297,8 +315,66 @@ __global__ void __launch_bounds__(512)
   l1 += __shfl_xor_sync(0xFFFFFFFFu, l1, 1);
   l1 += __shfl_xor_sync(0xFFFFFFFFu, l1, 2);
 
+  if (NG > 1) {
+    // groups 1..NG-1 hand their (O, m, l) to group 0 through shared memory
+    // (the stage ring is idle now); group 0 merges them in group order.
+    float* gp = reinterpret_cast<float*>(sK);            // [NG][rows_alloc][66]
+    if (grp > 0 && has_rows) {
+#pragma unroll
+      for (int half = 0; half < 2; ++half) {
+        float* dst = gp + (static_cast<size_t>(grp) * rows_alloc + (half ? r1 : r0)) * 66;
+#pragma unroll
+        for (int j = 0; j < 8; ++j)
+          *reinterpret_cast<float2*>(dst + 8 * j + 2 * tq) =
+              make_float2(o[j][half * 2 + 0], o[j][half * 2 + 1]);
+        if (tq == 0) {
+          dst[64] = half ? m1 : m0;
+          dst[65] = half ? l1 : l0;
+        }
+      }
+    }
+    __syncthreads();
+    if (grp == 0 && has_rows) {
+#pragma unroll
+      for (int half = 0; half < 2; ++half) {
+        const int r = half ? r1 : r0;
+        float M = half ? m1 : m0;
+        for (int q = 1; q < NG; ++q) M = fmaxf(M, gp[(static_cast<size_t>(q) * rows_alloc + r) * 66 + 64]);
+        const float mself = half ? m1 : m0;
+        const float w0 = (mself == -INFINITY) ? 0.f : exp2f(mself - M);
+        float L = w0 * (half ? l1 : l0);
+        float acc[16];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          acc[2 * j] = w0 * o[j][half * 2 + 0];
+          acc[2 * j + 1] = w0 * o[j][half * 2 + 1];
+        }
+        for (int q = 1; q < NG; ++q) {
+          const float* src = gp + (static_cast<size_t>(q) * rows_alloc + r) * 66;
+          const float mq = src[64];
+          const float wq = (mq == -INFINITY) ? 0.f : exp2f(mq - M);
+          L += wq * src[65];
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            const float2 v = *reinterpret_cast<const float2*>(src + 8 * j + 2 * tq);
+            acc[2 * j] += wq * v.x;
+            acc[2 * j + 1] += wq * v.y;
+          }
+        }
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          o[j][half * 2 + 0] = acc[2 * j];
+          o[j][half * 2 + 1] = acc[2 * j + 1];
+        }
+        if (half) { m1 = M; l1 = L; } else { m0 = M; l0 = L; }
+      }
+    }
+    __syncthreads();   // group partials consumed; the region is reused below
+  }
+  const bool lead = grp == 0 && has_rows;     // warps that hold the CTA's result rows
+
   if (nsplit == 1) {
-    if (has_rows && all_ok) {
+    if (lead && all_ok) {
 #pragma unroll
       for (int half = 0; half < 2; ++half) {
         const int r = half ? r1 : r0;
@@ -321,7 +397,7 @@ __global__ void __launch_bounds__(512)
   //      so [rows_alloc][64] fp32, sml [rows_alloc][2] = (m, l); empty rows: (0, -inf, 0).
   float* so = reinterpret_cast<float*>(sK);
   float* sml = so + rows_alloc * 64;
-  if (has_rows) {
+  if (lead) {
 #pragma unroll
     for (int half = 0; half < 2; ++half) {
       const int r = half ? r1 : r0;
@@ -334,11 +410,11 @@ __global__ void __launch_bounds__(512)
         sml[r * 2 + 1] = half ? l1 : l0;
       }
     }
-  } else {
-    for (int idx = lane; idx < 16 * 64; idx += 32) so[(warp * 16 + idx / 64) * 64 + idx % 64] = 0.f;
+  } else if (grp == 0) {   // row tiles past R: empty partials
+    for (int idx = lane; idx < 16 * 64; idx += 32) so[(mt * 16 + idx / 64) * 64 + idx % 64] = 0.f;
     if (lane < 16) {
-      sml[(warp * 16 + lane) * 2 + 0] = -INFINITY;
-      sml[(warp * 16 + lane) * 2 + 1] = 0.f;
+      sml[(mt * 16 + lane) * 2 + 0] = -INFINITY;
+      sml[(mt * 16 + lane) * 2 + 1] = 0.f;
     }
   }
   cluster_sync_all();

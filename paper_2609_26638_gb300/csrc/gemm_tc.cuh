@@ -36,6 +36,9 @@
 
 namespace gs {
 
+// Split-K factors up to this many reduce inside a cluster (portable cluster size).
+constexpr int kGemmMaxClusterSplits = 8;
+
 enum GemmEpilogue : int {
   kEpiStoreBf16 = 0, kEpiResidF32 = 1, kEpiSwiGLU = 2, kEpiArgmax = 3, kEpiQKV = 4
 };
@@ -83,8 +86,13 @@ struct GemmShape {
   static constexpr int kRedBytes = BN * 128 * 4;   // cluster reduction tile [BN][128] fp32
   static constexpr int kXBufBytes = 32 * 128 * 4;  // epilogue exchange (SwiGLU, RoPE, sums)
   static_assert(kRedBytes + kXBufBytes <= kStages * kStageBytes, "reduction smem");
+  // RoPE cos/sin rows of the tile's tokens, staged while the mainloop runs (decode tiles)
+  static constexpr bool kStageRope = BN <= 64;
+  static constexpr int kRopeBytes = kStageRope ? BN * 32 * 8 : 0;
   // pipeline | barriers (256 B) | per token: norm scale (4 B), KV destination (8 B), position (4 B)
-  static constexpr int kSmemBytes = kStages * kStageBytes + 1024 /*align*/ + 256 + 16 * BN;
+  // | RoPE rows
+  static constexpr int kSmemBytes =
+      kStages * kStageBytes + 1024 /*align*/ + 256 + 16 * BN + kRopeBytes;
 };
 
 // Epilogue of 32 consecutive tokens (t0 .. t0+31) of feature row `row`;
@@ -98,6 +106,7 @@ struct TokMeta {
   const float* rs;
   const long long* kvdst;
   const int* pos;
+  const float2* cs;   // [32 tokens][32] cos/sin, or null: read the table
 };
 
 template <int BN, int EPI>
@@ -141,10 +150,12 @@ __device__ __forceinline__ void gemm_epilogue_chunk(const GemmArgs& a, float (&v
       // sum of h^2 over the tile's 128 features per token: warp tree, then 4 warps in order
 #pragma unroll
       for (int j = 0; j < 32; ++j) {
-        float t = v[j];
+        if (j >= jlo && j < jhi) {   // uniform across the CTA
+          float t = v[j];
 #pragma unroll
-        for (int m = 16; m >= 1; m >>= 1) t += __shfl_xor_sync(0xFFFFFFFFu, t, m);
-        if (lane == 0) xbuf[warp * 32 + j] = t;
+          for (int m = 16; m >= 1; m >>= 1) t += __shfl_xor_sync(0xFFFFFFFFu, t, m);
+          if (lane == 0) xbuf[warp * 32 + j] = t;
+        }
       }
       asm volatile("bar.sync 2, 128;" ::: "memory");
       if (threadIdx.x < 32) {
@@ -162,14 +173,17 @@ __device__ __forceinline__ void gemm_epilogue_chunk(const GemmArgs& a, float (&v
     const int d = row & 63;
     if (region < 2) {
 #pragma unroll
-      for (int j = 0; j < 32; ++j) xbuf[j * 128 + row] = v[j];
+      for (int j = 0; j < 32; ++j)
+        if (j >= jlo && j < jhi) xbuf[j * 128 + row] = v[j];
       asm volatile("bar.sync 1, 128;" ::: "memory");
       float2 cs[32];
 #pragma unroll
-      for (int j = 0; j < 32; ++j) {   // all table loads first
+      for (int j = 0; j < 32; ++j) {   // staged rows, else all table loads first
         const int p = tm.pos[j];
-        cs[j] = (j >= jlo && j < jhi && p >= 0 && p < a.max_ctx)
-                    ? a.rope[static_cast<size_t>(p) * 32 + (d & 31)] : make_float2(1.f, 0.f);
+        const bool ok = j >= jlo && j < jhi && p >= 0 && p < a.max_ctx;
+        cs[j] = !ok ? make_float2(1.f, 0.f)
+                    : (tm.cs ? tm.cs[j * 32 + (d & 31)]
+                             : a.rope[static_cast<size_t>(p) * 32 + (d & 31)]);
       }
 #pragma unroll
       for (int j = 0; j < 32; ++j) {
@@ -199,7 +213,8 @@ __device__ __forceinline__ void gemm_epilogue_chunk(const GemmArgs& a, float (&v
     // rows 0..63: gate of features f0..f0+63; rows 64..127: up of the same features
     if (warp >= 2) {
 #pragma unroll
-      for (int j = 0; j < 32; ++j) xbuf[j * 64 + (row - 64)] = v[j];
+      for (int j = 0; j < 32; ++j)
+        if (j >= jlo && j < jhi) xbuf[j * 64 + (row - 64)] = v[j];
     }
     asm volatile("bar.sync 1, 128;" ::: "memory");
     if (warp < 2) {
@@ -225,13 +240,15 @@ __device__ __forceinline__ void gemm_epilogue_chunk(const GemmArgs& a, float (&v
     }
 #pragma unroll
     for (int j = 0; j < 32; ++j) {
-      unsigned long long key = argmax_key(v[j], f);
+      if (j >= jlo && j < jhi) {   // uniform across the CTA
+        unsigned long long key = argmax_key(v[j], f);
 #pragma unroll
-      for (int m = 16; m >= 1; m >>= 1) {
-        const unsigned long long o = shfl_xor_u64(key, m);
-        key = o > key ? o : key;
+        for (int m = 16; m >= 1; m >>= 1) {
+          const unsigned long long o = shfl_xor_u64(key, m);
+          key = o > key ? o : key;
+        }
+        if (lane == 0) atomicMax(out + t0 + j, key);
       }
-      if (lane == 0 && j >= jlo && j < jhi) atomicMax(out + t0 + j, key);
     }
   }
 }
@@ -349,6 +366,15 @@ __global__ void __launch_bounds__(128, 1)
           }
           kvdst_s[t] = dst;
           pos_s[t] = p;
+          if constexpr (S::kStageRope) {
+            float2* cs_s = reinterpret_cast<float2*>(pos_s + BN);
+            if (p >= 0 && p < a.max_ctx) {
+              const float4* src = reinterpret_cast<const float4*>(a.rope + static_cast<size_t>(p) * 32);
+              float4* dstv = reinterpret_cast<float4*>(cs_s + t * 32);
+#pragma unroll
+              for (int q = 0; q < 16; ++q) dstv[q] = src[q];
+            }
+          }
         }
       }
     }
@@ -384,8 +410,10 @@ __global__ void __launch_bounds__(128, 1)
   const float* rs_s = reinterpret_cast<const float*>(smem + S::kStages * S::kStageBytes + 256);
   const long long* kvdst_s = reinterpret_cast<const long long*>(rs_s + BN);
   const int* pos_s = reinterpret_cast<const int*>(kvdst_s + BN);
+  const float2* cs_s = S::kStageRope ? reinterpret_cast<const float2*>(pos_s + BN) : nullptr;
   auto rs_of = [&](int c) -> TokMeta {
-    return TokMeta{a.ssp_in ? rs_s + c * 32 : nullptr, kvdst_s + c * 32, pos_s + c * 32};
+    return TokMeta{a.ssp_in ? rs_s + c * 32 : nullptr, kvdst_s + c * 32, pos_s + c * 32,
+                   cs_s ? cs_s + c * 32 * 32 : nullptr};
   };
 
   if (a.splits == 1) {
@@ -430,11 +458,14 @@ __global__ void __launch_bounds__(128, 1)
       float v[32];
 #pragma unroll
       for (int j = 0; j < 32; ++j) v[j] = 0.0f;
-      for (int s = 0; s < a.splits; ++s) {
-        const float* peer = cluster_peer_ptr(red, static_cast<uint32_t>(s));
 #pragma unroll
-        for (int j = 0; j < 32; ++j)
-          if (j >= jlo && j < jhi) v[j] += peer[(c * 32 + j) * 128 + row];
+      for (int s = 0; s < kGemmMaxClusterSplits; ++s) {
+        if (s < a.splits) {
+          const float* peer = cluster_peer_ptr(red, static_cast<uint32_t>(s));
+#pragma unroll
+          for (int j = 0; j < 32; ++j)
+            if (j >= jlo && j < jhi) v[j] += peer[(c * 32 + j) * 128 + row];
+        }
       }
       if (!failed)
         gemm_epilogue_chunk<BN, EPI>(a, v, row, feat_tile, tok0 + c * 32, jlo, jhi, xbuf, rs_of(c));
