@@ -428,14 +428,14 @@ __global__ void __launch_bounds__(512)
     const int d4 = (idx & 15) * 4;
     float ms[kAttnMaxSplits], ls[kAttnMaxSplits];
     float4 os[kAttnMaxSplits];
+    const uint32_t ml_addr = smem_u32(sml + r * 2), o_addr = smem_u32(so + r * 64 + d4);
 #pragma unroll
-    for (int sp = 0; sp < kAttnMaxSplits; ++sp) {
+    for (int sp = 0; sp < kAttnMaxSplits; ++sp) {   // every peer's loads before any use
       if (sp < C) {
-        const float* pml = cluster_peer_ptr(sml + r * 2, static_cast<uint32_t>(sp));
-        const float* po = cluster_peer_ptr(so + r * 64 + d4, static_cast<uint32_t>(sp));
-        ms[sp] = pml[0];
-        ls[sp] = pml[1];
-        os[sp] = *reinterpret_cast<const float4*>(po);
+        const float2 ml = ld_cluster_f32x2(cluster_map(ml_addr, static_cast<uint32_t>(sp)));
+        ms[sp] = ml.x;
+        ls[sp] = ml.y;
+        os[sp] = ld_cluster_f32x4(cluster_map(o_addr, static_cast<uint32_t>(sp)));
       }
     }
     float M = -INFINITY;

@@ -332,30 +332,21 @@ __global__ void __launch_bounds__(128, 1)
       load_x(i, s);
     }
   } else {
-    pdl_wait();
-    pdl_trigger();
-    if (warp >= 2) {
-      // idle during the mainloop: stage the epilogue's per-token inputs
-      float* rs_s = reinterpret_cast<float*>(smem + S::kStages * S::kStageBytes + 256);
-      long long* kvdst_s = reinterpret_cast<long long*>(rs_s + BN);
-      int* pos_s = reinterpret_cast<int*>(kvdst_s + BN);
-      const int tok0 = tok_tile * BN;
-      for (int t = threadIdx.x - 64; t < BN; t += 64) {
-        const bool valid = tok0 + t < a.M;
-        if (a.ssp_in != nullptr) {
-          float ss = 0.f;
-          if (valid) {
-            const float* sp = a.ssp_in + static_cast<size_t>(a.x_row0 + tok0 + t) * a.n_ssp;
-            for (int p = 0; p < a.n_ssp; ++p) ss += sp[p];
-          }
-          rs_s[t] = rsqrtf(ss * a.inv_d + a.eps);
-        }
-        if constexpr (EPI == kEpiQKV) {
+    float* rs_s = reinterpret_cast<float*>(smem + S::kStages * S::kStageBytes + 256);
+    long long* kvdst_s = reinterpret_cast<long long*>(rs_s + BN);
+    int* pos_s = reinterpret_cast<int*>(kvdst_s + BN);
+    const int tok0s = tok_tile * BN;
+    if constexpr (EPI == kEpiQKV) {
+      // Positions, page-table rows and the RoPE table are written by kernels
+      // that completed before the previous one started: stage them before the
+      // dependency wait.
+      if (warp >= 2) {
+        for (int t = threadIdx.x - 64; t < BN; t += 64) {
           long long dst = -1;
           int p = -1;
-          if (valid) {
-            p = a.pos[tok0 + t];
-            const int slot = a.tok_slot[tok0 + t];
+          if (tok0s + t < a.M) {
+            p = a.pos[tok0s + t];
+            const int slot = a.tok_slot[tok0s + t];
             if (slot >= 0) {
               const int lp = p >> 6;
               const int phys = (p >= 0 && p < a.max_ctx && lp < a.pt_stride)
@@ -371,11 +362,32 @@ __global__ void __launch_bounds__(128, 1)
             if (p >= 0 && p < a.max_ctx) {
               const float4* src = reinterpret_cast<const float4*>(a.rope + static_cast<size_t>(p) * 32);
               float4* dstv = reinterpret_cast<float4*>(cs_s + t * 32);
+              float4 buf[16];
 #pragma unroll
-              for (int q = 0; q < 16; ++q) dstv[q] = src[q];
+              for (int q = 0; q < 16; ++q) buf[q] = src[q];
+#pragma unroll
+              for (int q = 0; q < 16; ++q) dstv[q] = buf[q];
             }
           }
         }
+      }
+    }
+    pdl_wait();
+    pdl_trigger();
+    if (warp >= 2 && a.ssp_in != nullptr) {
+      // folded-norm scale from the previous kernel's per-tile sums of h^2
+      for (int t = threadIdx.x - 64; t < BN; t += 64) {
+        float ss = 0.f;
+        if (tok0s + t < a.M) {
+          const float* sp = a.ssp_in + static_cast<size_t>(a.x_row0 + tok0s + t) * a.n_ssp;
+          float part[16];
+#pragma unroll
+          for (int q = 0; q < 16; ++q) part[q] = q < a.n_ssp ? sp[q] : 0.f;
+#pragma unroll
+          for (int q = 0; q < 16; ++q) ss += part[q];
+          for (int q = 16; q < a.n_ssp; ++q) ss += sp[q];
+        }
+        rs_s[t] = rsqrtf(ss * a.inv_d + a.eps);
       }
     }
     if (warp == 1 && lane == 0) {
@@ -458,13 +470,26 @@ __global__ void __launch_bounds__(128, 1)
       float v[32];
 #pragma unroll
       for (int j = 0; j < 32; ++j) v[j] = 0.0f;
+      const uint32_t red_base = smem_u32(red) + static_cast<uint32_t>(((c * 32) * 128 + row) * 4);
 #pragma unroll
-      for (int s = 0; s < kGemmMaxClusterSplits; ++s) {
-        if (s < a.splits) {
-          const float* peer = cluster_peer_ptr(red, static_cast<uint32_t>(s));
+      for (int j0 = 0; j0 < 32; j0 += 4) {
+        if (j0 + 4 > jlo && j0 < jhi) {   // uniform across the CTA
+          float t[kGemmMaxClusterSplits][4];
 #pragma unroll
-          for (int j = 0; j < 32; ++j)
-            if (j >= jlo && j < jhi) v[j] += peer[(c * 32 + j) * 128 + row];
+          for (int s = 0; s < kGemmMaxClusterSplits; ++s) {
+            if (s < a.splits) {
+              const uint32_t pb = cluster_map(red_base, static_cast<uint32_t>(s));
+#pragma unroll
+              for (int q = 0; q < 4; ++q)
+                t[s][q] = (j0 + q >= jlo && j0 + q < jhi) ? ld_cluster_f32(pb + (j0 + q) * 512) : 0.f;
+            }
+          }
+#pragma unroll
+          for (int s = 0; s < kGemmMaxClusterSplits; ++s)
+            if (s < a.splits) {
+#pragma unroll
+              for (int q = 0; q < 4; ++q) v[j0 + q] += t[s][q];
+            }
         }
       }
       if (!failed)
