@@ -76,10 +76,7 @@ struct GemmPlan {
   int bn, tok_tiles, feat_tiles, splits;
 };
 
-// Token tile from T.  Decode GEMMs with fewer tiles than SMs split K so that a
-// CTA's K slice fits its stage ring (8 x 64 at BN <= 64): the CTA then issues
-// every weight load before the dependency wait, while the previous kernel
-// still runs.  Splits stay within one cluster.
+// Token tile from T; split-K (decode only) so that about one wave of CTAs runs.
 GemmPlan plan_gemm(int weight_rows, int K, int T, bool allow_split) {
   GemmPlan p;
   p.bn = gemm_bn_for(T);
@@ -88,11 +85,10 @@ GemmPlan plan_gemm(int weight_rows, int K, int T, bool allow_split) {
   p.splits = 1;
   const int tiles = p.feat_tiles * p.tok_tiles;
   const int nkb = K / 64;
-  const int stages = p.bn <= 64 ? 8 : (p.bn <= 128 ? 3 : 4);
-  if (allow_split && tiles < 152 && nkb > stages) {
-    const int want = std::min(cdiv(nkb, stages), kMaxClusterSplits);
-    for (int s = 1; s <= nkb && s <= kMaxClusterSplits; ++s)
-      if (nkb % s == 0 && s >= want) { p.splits = s; break; }
+  if (allow_split && tiles < 152) {
+    const int want = std::min(cdiv(152, tiles), kMaxClusterSplits);
+    for (int s = 1; s <= nkb; ++s)
+      if (nkb % s == 0 && s <= want) p.splits = s;
   }
   return p;
 }

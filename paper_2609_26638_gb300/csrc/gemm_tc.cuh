@@ -80,10 +80,8 @@ struct GemmShape {
   static constexpr int kABytes = 128 * 128;        // 128 rows x 64 bf16
   static constexpr int kBBytes = BN * 128;         // BN rows x 64 bf16
   static constexpr int kStageBytes = kABytes + kBBytes;
-  // Decode tiles (BN <= 64) hold 8 stages, so a CTA whose K slice is 512 has
-  // its whole weight slice in flight before the dependency wait; prefill
-  // tiles (BN 128, 256) pipeline 3-4 stages.
-  static constexpr int kStages = BN <= 64 ? 8 : (BN <= 128 ? 3 : 4);
+  // two CTAs per SM up to BN = 128 (<= ~97 KB each), one at BN = 256
+  static constexpr int kStages = BN <= 64 ? 4 : (BN <= 128 ? 3 : 4);
   static constexpr int kTmemCols = BN < 32 ? 32 : BN;
   static constexpr int kRedBytes = BN * 128 * 4;   // cluster reduction tile [BN][128] fp32
   static constexpr int kXBufBytes = 32 * 128 * 4;  // epilogue exchange (SwiGLU, RoPE, sums)
