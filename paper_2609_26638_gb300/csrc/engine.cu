@@ -86,7 +86,8 @@ GemmPlan plan_gemm(int weight_rows, int K, int T, bool allow_split) {
   const int tiles = p.feat_tiles * p.tok_tiles;
   const int nkb = K / 64;
   if (allow_split && tiles < 152) {
-    const int want = std::min(cdiv(152, tiles), kMaxClusterSplits);
+    // about one wave, and split CTAs owning at most 8 tokens (BN / splits <= 8)
+    const int want = std::min(std::max(cdiv(152, tiles), p.bn / 8), kMaxClusterSplits);
     for (int s = 1; s <= nkb; ++s)
       if (nkb % s == 0 && s <= want) p.splits = s;
   }

@@ -109,8 +109,11 @@ struct TokMeta {
   const float2* cs;   // [32 tokens][32] cos/sin, or null: read the table
 };
 
-template <int BN, int EPI>
-__device__ __forceinline__ void gemm_epilogue_chunk(const GemmArgs& a, float (&v)[32], int row,
+// Epilogue of EW consecutive token slots t0 .. t0+EW-1 of feature row `row`;
+// slots q in [jlo, jhi) with t0 + q < M are produced.  Split CTAs own at most
+// 8 tokens and use EW = 8; whole tiles use EW = 32.
+template <int BN, int EPI, int EW>
+__device__ __forceinline__ void gemm_epilogue_chunk(const GemmArgs& a, float (&v)[EW], int row,
                                                     int feat_tile, int t0, int jlo, int jhi,
                                                     float* xbuf, TokMeta tm) {
   const float* rs = tm.rs;
@@ -119,24 +122,24 @@ __device__ __forceinline__ void gemm_epilogue_chunk(const GemmArgs& a, float (&v
   jhi = min(jhi, a.M - t0);
   if (rs != nullptr) {
 #pragma unroll
-    for (int j = 0; j < 32; ++j) v[j] *= rs[j];
+    for (int j = 0; j < EW; ++j) v[j] *= rs[j];
   }
   if constexpr (EPI == kEpiStoreBf16) {
     __nv_bfloat16* y = static_cast<__nv_bfloat16*>(a.y);
     const int f = feat_tile * 128 + row;
 #pragma unroll
-    for (int j = 0; j < 32; ++j)
+    for (int j = 0; j < EW; ++j)
       if (j >= jlo && j < jhi) y[static_cast<size_t>(t0 + j) * a.ldy + f] = __float2bfloat16_rn(v[j]);
   } else if constexpr (EPI == kEpiResidF32) {
     float* y = static_cast<float*>(a.y);
     const int f = feat_tile * 128 + row;
     const float g = a.hb_out ? __bfloat162float(a.g_next[f]) : 0.f;
-    float hv[32];
+    float hv[EW];
 #pragma unroll
-    for (int j = 0; j < 32; ++j)   // all loads first: one round trip, not 32
+    for (int j = 0; j < EW; ++j)   // all loads first: one round trip, not 32
       hv[j] = (j >= jlo && j < jhi) ? y[static_cast<size_t>(t0 + j) * a.ldy + f] : 0.f;
 #pragma unroll
-    for (int j = 0; j < 32; ++j) {
+    for (int j = 0; j < EW; ++j) {
       float hsq = 0.f;
       if (j >= jlo && j < jhi) {
         const float hn = hv[j] + v[j];
@@ -149,7 +152,7 @@ __device__ __forceinline__ void gemm_epilogue_chunk(const GemmArgs& a, float (&v
     if (a.ssp_out != nullptr) {
       // sum of h^2 over the tile's 128 features per token: warp tree, then 4 warps in order
 #pragma unroll
-      for (int j = 0; j < 32; ++j) {
+      for (int j = 0; j < EW; ++j) {
         if (j >= jlo && j < jhi) {   // uniform across the CTA
           float t = v[j];
 #pragma unroll
@@ -173,12 +176,12 @@ __device__ __forceinline__ void gemm_epilogue_chunk(const GemmArgs& a, float (&v
     const int d = row & 63;
     if (region < 2) {
 #pragma unroll
-      for (int j = 0; j < 32; ++j)
+      for (int j = 0; j < EW; ++j)
         if (j >= jlo && j < jhi) xbuf[j * 128 + row] = v[j];
       asm volatile("bar.sync 1, 128;" ::: "memory");
-      float2 cs[32];
+      float2 cs[EW];
 #pragma unroll
-      for (int j = 0; j < 32; ++j) {   // staged rows, else all table loads first
+      for (int j = 0; j < EW; ++j) {   // staged rows, else all table loads first
         const int p = tm.pos[j];
         const bool ok = j >= jlo && j < jhi && p >= 0 && p < a.max_ctx;
         cs[j] = !ok ? make_float2(1.f, 0.f)
@@ -186,7 +189,7 @@ __device__ __forceinline__ void gemm_epilogue_chunk(const GemmArgs& a, float (&v
                              : a.rope[static_cast<size_t>(p) * 32 + (d & 31)]);
       }
 #pragma unroll
-      for (int j = 0; j < 32; ++j) {
+      for (int j = 0; j < EW; ++j) {
         if (j >= jlo && j < jhi) {
           const float pr = xbuf[j * 128 + (row ^ 32)];
           v[j] = d < 32 ? v[j] * cs[j].x - pr * cs[j].y : v[j] * cs[j].x + pr * cs[j].y;
@@ -197,14 +200,14 @@ __device__ __forceinline__ void gemm_epilogue_chunk(const GemmArgs& a, float (&v
     const int head = (rbase + row) / 64 - (region == 0 ? 0 : (region == 1 ? a.Hq : a.Hq + a.Hkv));
     if (region == 0) {
 #pragma unroll
-      for (int j = 0; j < 32; ++j)
+      for (int j = 0; j < EW; ++j)
         if (j >= jlo && j < jhi)
           a.q_out[(static_cast<size_t>(t0 + j) * a.Hq + head) * 64 + d] = __float2bfloat16_rn(v[j]);
     } else {
       // kvdst[j]: offset of (page, K, head 0, row p & 63, dim 0); V is Hkv * 4096 further
       const long long off = (static_cast<long long>(isv_of(region)) * a.Hkv + head) * 4096 + d;
 #pragma unroll
-      for (int j = 0; j < 32; ++j) {
+      for (int j = 0; j < EW; ++j) {
         const long long base = tm.kvdst[j];
         if (j >= jlo && j < jhi && base >= 0) a.kv_layer[base + off] = __float2bfloat16_rn(v[j]);
       }
@@ -213,7 +216,7 @@ __device__ __forceinline__ void gemm_epilogue_chunk(const GemmArgs& a, float (&v
     // rows 0..63: gate of features f0..f0+63; rows 64..127: up of the same features
     if (warp >= 2) {
 #pragma unroll
-      for (int j = 0; j < 32; ++j)
+      for (int j = 0; j < EW; ++j)
         if (j >= jlo && j < jhi) xbuf[j * 64 + (row - 64)] = v[j];
     }
     asm volatile("bar.sync 1, 128;" ::: "memory");
@@ -221,7 +224,7 @@ __device__ __forceinline__ void gemm_epilogue_chunk(const GemmArgs& a, float (&v
       __nv_bfloat16* y = static_cast<__nv_bfloat16*>(a.y);
       const int f = feat_tile * 64 + row;
 #pragma unroll
-      for (int j = 0; j < 32; ++j)
+      for (int j = 0; j < EW; ++j)
         if (j >= jlo && j < jhi) {
           const float g = v[j];
           const float u = xbuf[j * 64 + row];
@@ -235,11 +238,11 @@ __device__ __forceinline__ void gemm_epilogue_chunk(const GemmArgs& a, float (&v
     unsigned long long* out = static_cast<unsigned long long*>(a.y);
     if (a.logits != nullptr) {
 #pragma unroll
-      for (int j = 0; j < 32; ++j)
+      for (int j = 0; j < EW; ++j)
         if (j >= jlo && j < jhi) a.logits[static_cast<size_t>(t0 + j) * a.N + f] = v[j];
     }
 #pragma unroll
-    for (int j = 0; j < 32; ++j) {
+    for (int j = 0; j < EW; ++j) {
       if (j >= jlo && j < jhi) {   // uniform across the CTA
         unsigned long long key = argmax_key(v[j], f);
 #pragma unroll
@@ -435,7 +438,7 @@ __global__ void __launch_bounds__(128, 1)
         if (tok0 + c * 32 >= a.M) break;   // uniform across the CTA
         float v[32];
         tmem_ld_32x32b_x32(trow + c * 32, v);
-        gemm_epilogue_chunk<BN, EPI>(a, v, row, feat_tile, tok0 + c * 32, 0, 32, xbuf, rs_of(c));
+        gemm_epilogue_chunk<BN, EPI, 32>(a, v, row, feat_tile, tok0 + c * 32, 0, 32, xbuf, rs_of(c));
       }
     }
     tc_fence_before();
@@ -465,35 +468,66 @@ __global__ void __launch_bounds__(128, 1)
     if (warp == 2) tmem_dealloc(tmem, S::kTmemCols);
     const int per = BN / a.splits;
     const int lo = split * per, hi = min(lo + per, ntok);
-    for (int c = lo / 32; c * 32 < hi; ++c) {
-      const int jlo = max(lo - c * 32, 0), jhi = min(hi - c * 32, 32);
-      float v[32];
+    if (per <= 8) {
+      // this CTA's <= 8 tokens: every peer's values for them, then the epilogue
+      if (hi > lo) {
+        const int nq = hi - lo;
+        const uint32_t base = smem_u32(red) + static_cast<uint32_t>((lo * 128 + row) * 4);
+        float t[kGemmMaxClusterSplits][8];
 #pragma unroll
-      for (int j = 0; j < 32; ++j) v[j] = 0.0f;
-      const uint32_t red_base = smem_u32(red) + static_cast<uint32_t>(((c * 32) * 128 + row) * 4);
+        for (int s = 0; s < kGemmMaxClusterSplits; ++s) {
+          if (s < a.splits) {
+            const uint32_t pb = cluster_map(base, static_cast<uint32_t>(s));
 #pragma unroll
-      for (int j0 = 0; j0 < 32; j0 += 4) {
-        if (j0 + 4 > jlo && j0 < jhi) {   // uniform across the CTA
-          float t[kGemmMaxClusterSplits][4];
-#pragma unroll
-          for (int s = 0; s < kGemmMaxClusterSplits; ++s) {
-            if (s < a.splits) {
-              const uint32_t pb = cluster_map(red_base, static_cast<uint32_t>(s));
-#pragma unroll
-              for (int q = 0; q < 4; ++q)
-                t[s][q] = (j0 + q >= jlo && j0 + q < jhi) ? ld_cluster_f32(pb + (j0 + q) * 512) : 0.f;
-            }
+            for (int q = 0; q < 8; ++q) t[s][q] = q < nq ? ld_cluster_f32(pb + q * 512) : 0.f;
           }
-#pragma unroll
-          for (int s = 0; s < kGemmMaxClusterSplits; ++s)
-            if (s < a.splits) {
-#pragma unroll
-              for (int q = 0; q < 4; ++q) v[j0 + q] += t[s][q];
-            }
         }
+        float v[8];
+#pragma unroll
+        for (int q = 0; q < 8; ++q) v[q] = 0.0f;
+#pragma unroll
+        for (int s = 0; s < kGemmMaxClusterSplits; ++s)
+          if (s < a.splits) {
+#pragma unroll
+            for (int q = 0; q < 8; ++q) v[q] += t[s][q];
+          }
+        const TokMeta m = rs_of(0);
+        const TokMeta tm{m.rs ? m.rs + lo : nullptr, m.kvdst + lo, m.pos + lo,
+                         m.cs ? m.cs + lo * 32 : nullptr};
+        if (!failed) gemm_epilogue_chunk<BN, EPI, 8>(a, v, row, feat_tile, tok0 + lo, 0, nq, xbuf, tm);
       }
-      if (!failed)
-        gemm_epilogue_chunk<BN, EPI>(a, v, row, feat_tile, tok0 + c * 32, jlo, jhi, xbuf, rs_of(c));
+    } else {
+      for (int c = lo / 32; c * 32 < hi; ++c) {
+        const int jlo = max(lo - c * 32, 0), jhi = min(hi - c * 32, 32);
+        float v[32];
+#pragma unroll
+        for (int j = 0; j < 32; ++j) v[j] = 0.0f;
+        const uint32_t red_base = smem_u32(red) + static_cast<uint32_t>(((c * 32) * 128 + row) * 4);
+#pragma unroll
+        for (int j0 = 0; j0 < 32; j0 += 4) {
+          if (j0 + 4 > jlo && j0 < jhi) {   // uniform across the CTA
+            float t[kGemmMaxClusterSplits][4];
+#pragma unroll
+            for (int s = 0; s < kGemmMaxClusterSplits; ++s) {
+              if (s < a.splits) {
+                const uint32_t pb = cluster_map(red_base, static_cast<uint32_t>(s));
+#pragma unroll
+                for (int q = 0; q < 4; ++q)
+                  t[s][q] = (j0 + q >= jlo && j0 + q < jhi) ? ld_cluster_f32(pb + (j0 + q) * 512) : 0.f;
+              }
+            }
+#pragma unroll
+            for (int s = 0; s < kGemmMaxClusterSplits; ++s)
+              if (s < a.splits) {
+#pragma unroll
+                for (int q = 0; q < 4; ++q) v[j0 + q] += t[s][q];
+              }
+          }
+        }
+        if (!failed)
+          gemm_epilogue_chunk<BN, EPI, 32>(a, v, row, feat_tile, tok0 + c * 32, jlo, jhi, xbuf,
+                                           rs_of(c));
+      }
     }
     cluster_sync_all();   // peers may still be reading this CTA's partial tile
     return;
@@ -536,7 +570,7 @@ __global__ void __launch_bounds__(128, 1)
 #pragma unroll
       for (int j = 0; j < 32; ++j) v[j] += __ldcg(p + (c * 32 + j) * 128 + row);
     }
-    gemm_epilogue_chunk<BN, EPI>(a, v, row, feat_tile, tok0 + c * 32, 0, 32, xbuf, rs_of(c));
+    gemm_epilogue_chunk<BN, EPI, 32>(a, v, row, feat_tile, tok0 + c * 32, 0, 32, xbuf, rs_of(c));
   }
 }
 
