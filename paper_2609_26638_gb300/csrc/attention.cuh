@@ -13,25 +13,26 @@
 // of one warp per 16 rows; group g takes the split's pages g, g+NG, ... so NG
 // pages are in work at once.  Each warp runs S = Q K^T and O += P V on
 // mma.sync m16n8k16 (bf16 in, fp32 out) with the online softmax in registers
-// (exp2 with the 1/sqrt(64) scale folded); the groups' partials merge in
-// shared memory in group order.  NG depends only on the row count (4 up to 64
-// rows, 2 up to 128, else 1), so windows with the same group count give
-// bit-identical rows.
+// (exp2 with the 1/sqrt(64) scale folded).  NG depends only on the row count
+// (4 up to 64 rows, 2 up to 128, else 1), so windows with the same group
+// count give bit-identical rows.
 //
 // Splits cover fixed absolute page ranges [c*SP, (c+1)*SP), so a row's result
 // depends only on its own keys and not on the window it sits in; keys past a
 // row's limit contribute exact zeros.  The splits of one (block, head) are one
-// thread-block cluster (at most kAttnMaxSplits CTAs): each CTA leaves its
-// (O, m, l) partial in its own shared memory and, after a cluster barrier,
-// merges a share of the rows over all peers through distributed shared memory
-// in split order.  A block whose keys fit in one split writes directly.
+// thread-block cluster (at most kAttnMaxSplits CTAs).  Row r is owned by CTA
+// r mod C: every warp pushes the (O, m, l) partial of its rows into the
+// owner's receive buffer (distributed-shared-memory stores), one cluster
+// barrier follows, and each owner merges its rows over all (split, group)
+// sources in that order.  A block whose keys fit in one split runs in CTA 0
+// alone and merges its groups the same way.
 #pragma once
 #include "ptx.cuh"
 
 namespace gs {
 
 constexpr int kAttnMaxSplits = 8;
-constexpr int kAttnStages = 8;
+constexpr int kAttnStages = 6;
 constexpr int kAttnPageBytes = 64 * 128;  // 64 tokens x 64 bf16
 
 struct AttnArgs {
@@ -59,8 +60,13 @@ __host__ __device__ inline int attn_groups(int r_max) {
 __host__ __device__ inline int attn_threads(int r_max) {
   return attn_mtiles(r_max) * attn_groups(r_max) * 32;
 }
+// receive buffer: per (split, group) source, ceil(rows / C) rows of 66 floats (O, m, l)
+__host__ __device__ inline int attn_recv_floats(int r_max) {
+  return attn_groups(r_max) * (attn_mtiles(r_max) * 16 + kAttnMaxSplits) * 66;
+}
 __host__ __device__ inline int attn_smem_bytes(int r_max) {
-  return 1024 + kAttnStages * 2 * kAttnPageBytes + attn_mtiles(r_max) * 16 * 128 + 128 + 64;
+  return 1024 + kAttnStages * 2 * kAttnPageBytes + attn_mtiles(r_max) * 16 * 128 + 128 +
+         attn_recv_floats(r_max) * 4;
 }
 // Pages per split so that a sequence of `pages` pages needs at most kAttnMaxSplits splits.
 __host__ __device__ inline int attn_min_split_pages(int pages) {
@@ -147,6 +153,7 @@ __global__ void __launch_bounds__(512)
     return;
   }
   if (nsplit == 1 && c > 0) return;         // direct path: CTA 0 alone
+  if (nsplit > 1) cluster_arrive_relaxed();  // completed by cluster_wait() before the pushes
   const int p_begin = c * SP;
   const int np = c < nsplit ? min(npages_blk, p_begin + SP) - p_begin : 0;
   const int32_t* pt = a.page_table + static_cast<size_t>(slot) * a.pt_stride;
@@ -315,152 +322,70 @@ __global__ void __launch_bounds__(512)
   l1 += __shfl_xor_sync(0xFFFFFFFFu, l1, 1);
   l1 += __shfl_xor_sync(0xFFFFFFFFu, l1, 2);
 
-  if (NG > 1) {
-    // groups 1..NG-1 hand their (O, m, l) to group 0 through shared memory
-    // (the stage ring is idle now); group 0 merges them in group order.
-    float* gp = reinterpret_cast<float*>(sK);            // [NG][rows_alloc][66]
-    if (grp > 0 && has_rows) {
+  // ---- merge.  Sources: (split c, group g), src = c * NG + g; Ceff splits take part.
+  const int Ceff = nsplit == 1 ? 1 : C;
+  const int cself = nsplit == 1 ? 0 : c;
+  const int rpo = (rows_alloc + Ceff - 1) / Ceff;          // rows per owner
+  float* recv = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(full) + 128);  // [src][rpo][66]
+  if (Ceff > 1) cluster_wait();   // every CTA of the cluster runs: peers' shared memory exists
+  if (has_rows) {
+    const int src = cself * NG + grp;
 #pragma unroll
-      for (int half = 0; half < 2; ++half) {
-        float* dst = gp + (static_cast<size_t>(grp) * rows_alloc + (half ? r1 : r0)) * 66;
+    for (int half = 0; half < 2; ++half) {
+      const int r = half ? r1 : r0;
+      if (r >= R) continue;
+      const int owner = r % Ceff, slot = r / Ceff;
+      const uint32_t base = smem_u32(recv + (src * rpo + slot) * 66);
+      const float mm = half ? m1 : m0, ll = half ? l1 : l0;
+      if (Ceff == 1) {
+        float* dst = recv + (src * rpo + slot) * 66;
 #pragma unroll
         for (int j = 0; j < 8; ++j)
           *reinterpret_cast<float2*>(dst + 8 * j + 2 * tq) =
               make_float2(o[j][half * 2 + 0], o[j][half * 2 + 1]);
         if (tq == 0) {
-          dst[64] = half ? m1 : m0;
-          dst[65] = half ? l1 : l0;
+          dst[64] = mm;
+          dst[65] = ll;
         }
+      } else {
+        const uint32_t rb = cluster_map(base, static_cast<uint32_t>(owner));
+#pragma unroll
+        for (int j = 0; j < 8; ++j)
+          st_cluster_f32x2(rb + (8 * j + 2 * tq) * 4, make_float2(o[j][half * 2 + 0], o[j][half * 2 + 1]));
+        if (tq == 0) st_cluster_f32x2(rb + 64 * 4, make_float2(mm, ll));
       }
     }
-    __syncthreads();
-    if (grp == 0 && has_rows) {
-#pragma unroll
-      for (int half = 0; half < 2; ++half) {
-        const int r = half ? r1 : r0;
-        float M = half ? m1 : m0;
-        for (int q = 1; q < NG; ++q) M = fmaxf(M, gp[(static_cast<size_t>(q) * rows_alloc + r) * 66 + 64]);
-        const float mself = half ? m1 : m0;
-        const float w0 = (mself == -INFINITY) ? 0.f : exp2f(mself - M);
-        float L = w0 * (half ? l1 : l0);
-        float acc[16];
-#pragma unroll
-        for (int j = 0; j < 8; ++j) {
-          acc[2 * j] = w0 * o[j][half * 2 + 0];
-          acc[2 * j + 1] = w0 * o[j][half * 2 + 1];
-        }
-        for (int q = 1; q < NG; ++q) {
-          const float* src = gp + (static_cast<size_t>(q) * rows_alloc + r) * 66;
-          const float mq = src[64];
-          const float wq = (mq == -INFINITY) ? 0.f : exp2f(mq - M);
-          L += wq * src[65];
-#pragma unroll
-          for (int j = 0; j < 8; ++j) {
-            const float2 v = *reinterpret_cast<const float2*>(src + 8 * j + 2 * tq);
-            acc[2 * j] += wq * v.x;
-            acc[2 * j + 1] += wq * v.y;
-          }
-        }
-#pragma unroll
-        for (int j = 0; j < 8; ++j) {
-          o[j][half * 2 + 0] = acc[2 * j];
-          o[j][half * 2 + 1] = acc[2 * j + 1];
-        }
-        if (half) { m1 = M; l1 = L; } else { m0 = M; l0 = L; }
-      }
-    }
-    __syncthreads();   // group partials consumed; the region is reused below
   }
-  const bool lead = grp == 0 && has_rows;     // warps that hold the CTA's result rows
+  if (Ceff == 1) __syncthreads();
+  else cluster_sync_all();   // every partial has landed at its owner
 
-  if (nsplit == 1) {
-    if (lead && all_ok) {
-#pragma unroll
-      for (int half = 0; half < 2; ++half) {
-        const int r = half ? r1 : r0;
-        if (r >= R) continue;
-        const float inv = 1.0f / (half ? l1 : l0);
-        const int t = tok0 + r / a.G;
-        const int hq = h * a.G + r % a.G;
-        __nv_bfloat16* dst = a.out + (static_cast<size_t>(t) * a.Hq + hq) * 64;
-#pragma unroll
-        for (int j = 0; j < 8; ++j) {
-          const float x0 = o[j][half * 2 + 0] * inv, x1 = o[j][half * 2 + 1] * inv;
-          *reinterpret_cast<__nv_bfloat162*>(dst + 8 * j + 2 * tq) = __floats2bfloat162_rn(x0, x1);
-        }
-      }
-    }
-    return;
-  }
-
-  // ---- cluster merge.  Partials in this CTA's shared memory (stage buffers are free):
-  //      so [rows_alloc][64] fp32, sml [rows_alloc][2] = (m, l); empty rows: (0, -inf, 0).
-  float* so = reinterpret_cast<float*>(sK);
-  float* sml = so + rows_alloc * 64;
-  if (lead) {
-#pragma unroll
-    for (int half = 0; half < 2; ++half) {
-      const int r = half ? r1 : r0;
-#pragma unroll
-      for (int j = 0; j < 8; ++j)
-        *reinterpret_cast<float2*>(so + r * 64 + 8 * j + 2 * tq) =
-            make_float2(o[j][half * 2 + 0], o[j][half * 2 + 1]);
-      if (tq == 0) {
-        sml[r * 2 + 0] = half ? m1 : m0;
-        sml[r * 2 + 1] = half ? l1 : l0;
-      }
-    }
-  } else if (grp == 0) {   // row tiles past R: empty partials
-    for (int idx = lane; idx < 16 * 64; idx += 32) so[(mt * 16 + idx / 64) * 64 + idx % 64] = 0.f;
-    if (lane < 16) {
-      sml[(mt * 16 + lane) * 2 + 0] = -INFINITY;
-      sml[(mt * 16 + lane) * 2 + 1] = 0.f;
-    }
-  }
-  cluster_sync_all();
-  // CTA c merges rows c, c + C, c + 2C, ...; one thread per (row, 4 dims).
-  // Weights exp2(m_s - M) / L are summed over splits in order 0..C-1; with
-  // one split holding all of a row's keys this is O * (1 / l), the direct
-  // path's result.
-  const int my_rows = (R - c + C - 1) / C;
+  // owner: rows r = cself + k * Ceff; one thread per (row, 4 dims); weights
+  // exp2(m_src - M) / L over the sources in order.  With one source holding
+  // all of a row's keys this is O * (1 / l).
+  const int nsrc = Ceff * NG;
+  const int my_rows = (R - cself + Ceff - 1) / Ceff;
   for (int idx = threadIdx.x; idx < my_rows * 16; idx += nthreads) {
-    const int r = c + (idx >> 4) * C;
-    const int d4 = (idx & 15) * 4;
-    float ms[kAttnMaxSplits], ls[kAttnMaxSplits];
-    float4 os[kAttnMaxSplits];
-    const uint32_t ml_addr = smem_u32(sml + r * 2), o_addr = smem_u32(so + r * 64 + d4);
-#pragma unroll
-    for (int sp = 0; sp < kAttnMaxSplits; ++sp) {   // every peer's loads before any use
-      if (sp < C) {
-        const float2 ml = ld_cluster_f32x2(cluster_map(ml_addr, static_cast<uint32_t>(sp)));
-        ms[sp] = ml.x;
-        ls[sp] = ml.y;
-        os[sp] = ld_cluster_f32x4(cluster_map(o_addr, static_cast<uint32_t>(sp)));
-      }
-    }
+    const int k = idx >> 4, d4 = (idx & 15) * 4;
+    const int r = cself + k * Ceff;
+    const float* rowp = recv + k * 66;
     float M = -INFINITY;
-#pragma unroll
-    for (int sp = 0; sp < kAttnMaxSplits; ++sp)
-      if (sp < C) M = fmaxf(M, ms[sp]);
+    for (int sidx = 0; sidx < nsrc; ++sidx) M = fmaxf(M, rowp[sidx * rpo * 66 + 64]);
     float L = 0.f;
-#pragma unroll
-    for (int sp = 0; sp < kAttnMaxSplits; ++sp) {
-      if (sp < C) {
-        ms[sp] = (ms[sp] == -INFINITY) ? 0.f : exp2f(ms[sp] - M);
-        L += ms[sp] * ls[sp];
-      }
+    for (int sidx = 0; sidx < nsrc; ++sidx) {
+      const float ms = rowp[sidx * rpo * 66 + 64];
+      const float w = (ms == -INFINITY) ? 0.f : exp2f(ms - M);
+      L += w * rowp[sidx * rpo * 66 + 65];
     }
     const float inv = 1.0f / L;
     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll
-    for (int sp = 0; sp < kAttnMaxSplits; ++sp) {
-      if (sp < C) {
-        const float w = ms[sp] * inv;
-        acc.x += w * os[sp].x;
-        acc.y += w * os[sp].y;
-        acc.z += w * os[sp].z;
-        acc.w += w * os[sp].w;
-      }
+    for (int sidx = 0; sidx < nsrc; ++sidx) {
+      const float ms = rowp[sidx * rpo * 66 + 64];
+      const float w = ((ms == -INFINITY) ? 0.f : exp2f(ms - M)) * inv;
+      const float4 v = *reinterpret_cast<const float4*>(rowp + sidx * rpo * 66 + d4);
+      acc.x += w * v.x;
+      acc.y += w * v.y;
+      acc.z += w * v.z;
+      acc.w += w * v.w;
     }
     if (all_ok) {
       const int t = tok0 + r / a.G;
@@ -470,7 +395,6 @@ __global__ void __launch_bounds__(512)
       *reinterpret_cast<__nv_bfloat162*>(dst + 2) = __floats2bfloat162_rn(acc.z, acc.w);
     }
   }
-  cluster_sync_all();   // peers may still be reading this CTA's partials
 }
 
 }  // namespace gs

@@ -72,6 +72,9 @@ struct Carver {
   }
 };
 
+constexpr size_t kGemmPartialFloats = 12u << 20;  // 48 MB of split-K partials
+constexpr int kGemmCounters = 1 << 16;
+
 struct GemmPlan {
   int bn, tok_tiles, feat_tiles, splits;
 };
@@ -86,16 +89,24 @@ GemmPlan plan_gemm(int weight_rows, int K, int T, bool allow_split) {
   const int tiles = p.feat_tiles * p.tok_tiles;
   const int nkb = K / 64;
   if (allow_split && tiles < 152) {
-    // about one wave, and split CTAs owning at most 8 tokens (BN / splits <= 8)
-    const int want = std::min(std::max(cdiv(152, tiles), p.bn / 8), kMaxClusterSplits);
+    // about one wave; cluster-reduced decode tiles (BN <= 64) also keep each
+    // split CTA at <= 8 tokens (BN / splits <= 8)
+    int want = cdiv(152, tiles);
+    if (p.bn <= 64) want = std::max(want, p.bn / 8);
+    want = std::min(want, kMaxClusterSplits);
     for (int s = 1; s <= nkb; ++s)
       if (nkb % s == 0 && s <= want) p.splits = s;
+    // wider tiles reduce through global scratch: stay within it
+    while (p.bn > 64 && p.splits > 1 &&
+           static_cast<size_t>(p.splits) * tiles * p.bn * 128 > kGemmPartialFloats) {
+      int s = p.splits - 1;
+      while (s > 1 && nkb % s) --s;
+      p.splits = s;
+    }
   }
   return p;
 }
 
-constexpr size_t kGemmPartialFloats = 12u << 20;  // 48 MB of split-K partials
-constexpr int kGemmCounters = 1 << 16;
 
 }  // namespace
 
@@ -293,7 +304,11 @@ int run_gemm(gs_handle* h, const CUtensorMap& tw, int weight_rows, const CUtenso
   a.K = K;
   a.splits = p.splits;
   a.kb_per_split = (K / 64) / p.splits;
-  a.cluster = p.splits > 1 ? 1 : 0;
+  a.cluster = (p.splits > 1 && p.bn <= 64) ? 1 : 0;
+  if (p.splits > 1 && !a.cluster &&
+      (static_cast<size_t>(p.splits) * p.feat_tiles * p.tok_tiles * p.bn * 128 > kGemmPartialFloats ||
+       p.feat_tiles * p.tok_tiles > kGemmCounters))
+    return fail(h, GS_ERR_OOM, "split-K scratch too small");
   GS_CUDA(h, launch_gemm(p.bn, epi, tw, tx_set[bn_index(p.bn)], a, p.feat_tiles, p.tok_tiles,
                          h->stream, true));
   ++h->launches;
@@ -901,7 +916,7 @@ int gs_linear(const void* x, const void* w, void* y, int M, int N, int K, int ep
   a.K = K;
   a.splits = split_k;
   a.kb_per_split = (K / 64) / split_k;
-  a.cluster = (split_k > 1 && split_k <= kMaxClusterSplits) ? 1 : 0;
+  a.cluster = (split_k > 1 && split_k <= kMaxClusterSplits && bn <= 64) ? 1 : 0;
   a.y = y;
   a.ldy = N;
   a.logits = nullptr;

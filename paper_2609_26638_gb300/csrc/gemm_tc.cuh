@@ -14,12 +14,13 @@
 // come after it.
 //
 // Split-K: the CTAs that own different K ranges of one output tile either
-// form a thread-block cluster and reduce their fp32 partials through
-// distributed shared memory (each CTA sums a slice of the tile's tokens over
-// all peers), or -- for split factors above the cluster limit -- write the
-// partials to global scratch, where the last CTA to arrive (atomic ticket, no
-// spinning) sums them.  Both sum the splits in order 0..S-1 from a zero
-// start, so the result does not depend on the path or on arrival order.
+// form a thread-block cluster (decode tiles, BN <= 64) -- each CTA owns a
+// slice of the tile's tokens, every CTA pushes its fp32 partials for that
+// slice into the owner's receive buffer with distributed-shared-memory
+// stores, and after one cluster barrier the owner sums them locally -- or
+// write the partials to global scratch, where the last CTA to arrive (atomic
+// ticket, no spinning) sums them.  Both sum the splits in order 0..S-1 from a
+// zero start, so the result does not depend on the path or on arrival order.
 //
 // Epilogues: bf16 store, fp32 residual add, SwiGLU (gate and up rows of the
 // same features share a tile), LM-head argmax (packed 64-bit atomicMax, ties
@@ -89,10 +90,13 @@ struct GemmShape {
   // RoPE cos/sin rows of the tile's tokens, staged while the mainloop runs (decode tiles)
   static constexpr bool kStageRope = BN <= 64;
   static constexpr int kRopeBytes = kStageRope ? BN * 32 * 8 : 0;
+  // cluster split-K receive buffer [S][BN / S][128] fp32 (decode tiles only)
+  static constexpr bool kClusterOk = BN <= 64;
+  static constexpr int kRecvBytes = kClusterOk ? BN * 128 * 4 : 0;
   // pipeline | barriers (256 B) | per token: norm scale (4 B), KV destination (8 B), position (4 B)
-  // | RoPE rows
-  static constexpr int kSmemBytes =
-      kStages * kStageBytes + 1024 /*align*/ + 256 + 16 * BN + kRopeBytes;
+  // | RoPE rows | receive buffer
+  static constexpr int kRecvOffset = kStages * kStageBytes + 256 + 16 * BN + kRopeBytes;
+  static constexpr int kSmemBytes = kRecvOffset + kRecvBytes + 1024 /*align*/;
 };
 
 // Epilogue of 32 consecutive tokens (t0 .. t0+31) of feature row `row`;
@@ -297,6 +301,7 @@ __global__ void __launch_bounds__(128, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
+  if (a.cluster) cluster_arrive_relaxed();   // completed by cluster_wait() before the pushes
 
   if (warp == 0 && lane == 0) {
     // TMA producer.  Weight tiles of the first stages go out before the
@@ -447,90 +452,67 @@ __global__ void __launch_bounds__(128, 1)
     return;
   }
 
-  if (a.cluster) {
-    // Cluster split-K: partial tile -> own smem [BN][128]; after the cluster
-    // barrier, CTA `split` reduces tokens [split*BN/S, (split+1)*BN/S) over
-    // all peers in order 0..S-1 and runs the epilogue on them.
-    float* red = reinterpret_cast<float*>(smA);
-    float* xbuf = reinterpret_cast<float*>(smA + S::kRedBytes);
-    const int ntok = min(BN, a.M - tok0);
-    if (!failed) {
-      for (int c = 0; c < BN / 32; ++c) {
-        if (c * 32 >= ntok) break;
-        float v[32];
-        tmem_ld_32x32b_x32(trow + c * 32, v);
+  if constexpr (S::kClusterOk) {
+    if (a.cluster) {
+      // Cluster split-K.  CTA q owns tokens [q*per, (q+1)*per) of the tile;
+      // every CTA pushes its partials for them into q's receive buffer
+      // recv[s][jj][row] (s = pushing split), then one cluster barrier, then
+      // each owner sums its tokens over s = 0..S-1 and runs the epilogue.
+      float* recv = reinterpret_cast<float*>(smem + S::kRecvOffset);
+      float* xbuf = reinterpret_cast<float*>(smA);
+      const int per = BN / a.splits;
+      const int ntok = min(BN, a.M - tok0);
+      cluster_wait();       // every CTA of the cluster runs: peers' shared memory exists
+      if (!failed) {
+        const uint32_t recv0 = smem_u32(recv) + static_cast<uint32_t>(row * 4);
+        for (int c = 0; c < BN / 32; ++c) {
+          if (c * 32 >= ntok) break;
+          float v[32];
+          tmem_ld_32x32b_x32(trow + c * 32, v);
 #pragma unroll
-        for (int j = 0; j < 32; ++j) red[(c * 32 + j) * 128 + row] = v[j];
-      }
-    }
-    tc_fence_before();
-    cluster_sync_all();
-    if (warp == 2) tmem_dealloc(tmem, S::kTmemCols);
-    const int per = BN / a.splits;
-    const int lo = split * per, hi = min(lo + per, ntok);
-    if (per <= 8) {
-      // this CTA's <= 8 tokens: every peer's values for them, then the epilogue
-      if (hi > lo) {
-        const int nq = hi - lo;
-        const uint32_t base = smem_u32(red) + static_cast<uint32_t>((lo * 128 + row) * 4);
-        float t[kGemmMaxClusterSplits][8];
-#pragma unroll
-        for (int s = 0; s < kGemmMaxClusterSplits; ++s) {
-          if (s < a.splits) {
-            const uint32_t pb = cluster_map(base, static_cast<uint32_t>(s));
-#pragma unroll
-            for (int q = 0; q < 8; ++q) t[s][q] = q < nq ? ld_cluster_f32(pb + q * 512) : 0.f;
-          }
-        }
-        float v[8];
-#pragma unroll
-        for (int q = 0; q < 8; ++q) v[q] = 0.0f;
-#pragma unroll
-        for (int s = 0; s < kGemmMaxClusterSplits; ++s)
-          if (s < a.splits) {
-#pragma unroll
-            for (int q = 0; q < 8; ++q) v[q] += t[s][q];
-          }
-        const TokMeta m = rs_of(0);
-        const TokMeta tm{m.rs ? m.rs + lo : nullptr, m.kvdst + lo, m.pos + lo,
-                         m.cs ? m.cs + lo * 32 : nullptr};
-        if (!failed) gemm_epilogue_chunk<BN, EPI, 8>(a, v, row, feat_tile, tok0 + lo, 0, nq, xbuf, tm);
-      }
-    } else {
-      for (int c = lo / 32; c * 32 < hi; ++c) {
-        const int jlo = max(lo - c * 32, 0), jhi = min(hi - c * 32, 32);
-        float v[32];
-#pragma unroll
-        for (int j = 0; j < 32; ++j) v[j] = 0.0f;
-        const uint32_t red_base = smem_u32(red) + static_cast<uint32_t>(((c * 32) * 128 + row) * 4);
-#pragma unroll
-        for (int j0 = 0; j0 < 32; j0 += 4) {
-          if (j0 + 4 > jlo && j0 < jhi) {   // uniform across the CTA
-            float t[kGemmMaxClusterSplits][4];
-#pragma unroll
-            for (int s = 0; s < kGemmMaxClusterSplits; ++s) {
-              if (s < a.splits) {
-                const uint32_t pb = cluster_map(red_base, static_cast<uint32_t>(s));
-#pragma unroll
-                for (int q = 0; q < 4; ++q)
-                  t[s][q] = (j0 + q >= jlo && j0 + q < jhi) ? ld_cluster_f32(pb + (j0 + q) * 512) : 0.f;
-              }
+          for (int j = 0; j < 32; ++j) {
+            const int t = c * 32 + j;
+            if (t < ntok) {
+              const int q = t / per, jj = t - q * per;
+              st_cluster_f32(cluster_map(recv0 + static_cast<uint32_t>(((split * per + jj) * 128) * 4),
+                                         static_cast<uint32_t>(q)), v[j]);
             }
-#pragma unroll
-            for (int s = 0; s < kGemmMaxClusterSplits; ++s)
-              if (s < a.splits) {
-#pragma unroll
-                for (int q = 0; q < 4; ++q) v[j0 + q] += t[s][q];
-              }
           }
         }
-        if (!failed)
-          gemm_epilogue_chunk<BN, EPI, 32>(a, v, row, feat_tile, tok0 + c * 32, jlo, jhi, xbuf,
-                                           rs_of(c));
       }
+      tc_fence_before();
+      cluster_sync_all();   // every push has landed
+      if (warp == 2) tmem_dealloc(tmem, S::kTmemCols);
+      const int lo = split * per, hi = min(lo + per, ntok);
+      if (hi > lo && !failed) {
+        const int nq = hi - lo;
+        if (per <= 8) {
+          float v[8];
+#pragma unroll
+          for (int q = 0; q < 8; ++q) v[q] = 0.0f;
+          for (int sp = 0; sp < a.splits; ++sp)
+#pragma unroll
+            for (int q = 0; q < 8; ++q)
+              if (q < nq) v[q] += recv[(sp * per + q) * 128 + row];
+          const TokMeta m = rs_of(0);
+          const TokMeta tm{m.rs ? m.rs + lo : nullptr, m.kvdst + lo, m.pos + lo,
+                           m.cs ? m.cs + lo * 32 : nullptr};
+          gemm_epilogue_chunk<BN, EPI, 8>(a, v, row, feat_tile, tok0 + lo, 0, nq, xbuf, tm);
+        } else {   // per in {16, 32}: one 32-token chunk
+          const int c = lo / 32, jlo = lo - c * 32;
+          float v[32];
+#pragma unroll
+          for (int j = 0; j < 32; ++j) v[j] = 0.0f;
+          for (int sp = 0; sp < a.splits; ++sp)
+#pragma unroll
+            for (int j = 0; j < 32; ++j)
+              if (j >= jlo && j < jlo + nq) v[j] += recv[(sp * per + (j - jlo)) * 128 + row];
+          gemm_epilogue_chunk<BN, EPI, 32>(a, v, row, feat_tile, tok0 + c * 32, jlo, jlo + nq, xbuf,
+                                           rs_of(c));
+        }
+      }
+      return;
     }
-    cluster_sync_all();   // peers may still be reading this CTA's partial tile
-    return;
   }
 
   // global split-K: write this split's partial tile, token-major [BN][128]
