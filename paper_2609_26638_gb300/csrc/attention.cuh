@@ -60,9 +60,11 @@ __host__ __device__ inline int attn_groups(int r_max) {
 __host__ __device__ inline int attn_threads(int r_max) {
   return attn_mtiles(r_max) * attn_groups(r_max) * 32;
 }
-// receive buffer: per (split, group) source, ceil(rows / C) rows of 66 floats (O, m, l)
+// receive buffer: per (split, group) source, ceil(rows / C) rows of kAttnRecvRow floats:
+// O[64], m, l, 2 pad (272 B keeps every row 16-byte aligned for float4 reads)
+constexpr int kAttnRecvRow = 68;
 __host__ __device__ inline int attn_recv_floats(int r_max) {
-  return attn_groups(r_max) * (attn_mtiles(r_max) * 16 + kAttnMaxSplits) * 66;
+  return attn_groups(r_max) * (attn_mtiles(r_max) * 16 + kAttnMaxSplits) * kAttnRecvRow;
 }
 __host__ __device__ inline int attn_smem_bytes(int r_max) {
   return 1024 + kAttnStages * 2 * kAttnPageBytes + attn_mtiles(r_max) * 16 * 128 + 128 +
@@ -326,7 +328,7 @@ __global__ void __launch_bounds__(512)
   const int Ceff = nsplit == 1 ? 1 : C;
   const int cself = nsplit == 1 ? 0 : c;
   const int rpo = (rows_alloc + Ceff - 1) / Ceff;          // rows per owner
-  float* recv = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(full) + 128);  // [src][rpo][66]
+  float* recv = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(full) + 128);  // [src][rpo][68]
   if (Ceff > 1) cluster_wait();   // every CTA of the cluster runs: peers' shared memory exists
   if (has_rows) {
     const int src = cself * NG + grp;
@@ -335,10 +337,10 @@ __global__ void __launch_bounds__(512)
       const int r = half ? r1 : r0;
       if (r >= R) continue;
       const int owner = r % Ceff, slot = r / Ceff;
-      const uint32_t base = smem_u32(recv + (src * rpo + slot) * 66);
+      const uint32_t base = smem_u32(recv + (src * rpo + slot) * kAttnRecvRow);
       const float mm = half ? m1 : m0, ll = half ? l1 : l0;
       if (Ceff == 1) {
-        float* dst = recv + (src * rpo + slot) * 66;
+        float* dst = recv + (src * rpo + slot) * kAttnRecvRow;
 #pragma unroll
         for (int j = 0; j < 8; ++j)
           *reinterpret_cast<float2*>(dst + 8 * j + 2 * tq) =
@@ -367,21 +369,21 @@ __global__ void __launch_bounds__(512)
   for (int idx = threadIdx.x; idx < my_rows * 16; idx += nthreads) {
     const int k = idx >> 4, d4 = (idx & 15) * 4;
     const int r = cself + k * Ceff;
-    const float* rowp = recv + k * 66;
+    const float* rowp = recv + k * kAttnRecvRow;
     float M = -INFINITY;
-    for (int sidx = 0; sidx < nsrc; ++sidx) M = fmaxf(M, rowp[sidx * rpo * 66 + 64]);
+    for (int sidx = 0; sidx < nsrc; ++sidx) M = fmaxf(M, rowp[sidx * rpo * kAttnRecvRow + 64]);
     float L = 0.f;
     for (int sidx = 0; sidx < nsrc; ++sidx) {
-      const float ms = rowp[sidx * rpo * 66 + 64];
+      const float ms = rowp[sidx * rpo * kAttnRecvRow + 64];
       const float w = (ms == -INFINITY) ? 0.f : exp2f(ms - M);
-      L += w * rowp[sidx * rpo * 66 + 65];
+      L += w * rowp[sidx * rpo * kAttnRecvRow + 65];
     }
     const float inv = 1.0f / L;
     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
     for (int sidx = 0; sidx < nsrc; ++sidx) {
-      const float ms = rowp[sidx * rpo * 66 + 64];
+      const float ms = rowp[sidx * rpo * kAttnRecvRow + 64];
       const float w = ((ms == -INFINITY) ? 0.f : exp2f(ms - M)) * inv;
-      const float4 v = *reinterpret_cast<const float4*>(rowp + sidx * rpo * 66 + d4);
+      const float4 v = *reinterpret_cast<const float4*>(rowp + sidx * rpo * kAttnRecvRow + d4);
       acc.x += w * v.x;
       acc.y += w * v.y;
       acc.z += w * v.z;
