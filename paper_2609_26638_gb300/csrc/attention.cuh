@@ -21,11 +21,12 @@
 // depends only on its own keys and not on the window it sits in; keys past a
 // row's limit contribute exact zeros.  The splits of one (block, head) are one
 // thread-block cluster (at most kAttnMaxSplits CTAs).  Row r is owned by CTA
-// r mod C: every warp pushes the (O, m, l) partial of its rows into the
-// owner's receive buffer (distributed-shared-memory stores), one cluster
-// barrier follows, and each owner merges its rows over all (split, group)
-// sources in that order.  A block whose keys fit in one split runs in CTA 0
-// alone and merges its groups the same way.
+// r mod C: every warp stages the (O, m, l) partial of its rows, grouped by
+// owner, in its CTA's shared memory; one thread sends each owner its block
+// with a bulk async copy that completes on the owner's mbarrier; each owner
+// then merges its rows over all (split, group) sources in that order.  A
+// block whose keys fit in one split runs in CTA 0 alone and merges its groups
+// the same way without copies.
 #pragma once
 #include "ptx.cuh"
 
@@ -70,6 +71,8 @@ __host__ __device__ inline int attn_smem_bytes(int r_max) {
   return 1024 + kAttnStages * 2 * kAttnPageBytes + attn_mtiles(r_max) * 16 * 128 + 128 +
          attn_recv_floats(r_max) * 4;
 }
+static_assert(kAttnStages * 2 * kAttnPageBytes >= 4 * (64 + kAttnMaxSplits) * 68 * 4,
+              "the K/V ring must hold the largest merge staging block");
 // Pages per split so that a sequence of `pages` pages needs at most kAttnMaxSplits splits.
 __host__ __device__ inline int attn_min_split_pages(int pages) {
   return (pages + kAttnMaxSplits - 1) / kAttnMaxSplits;
@@ -160,9 +163,17 @@ __global__ void __launch_bounds__(512)
   const int np = c < nsplit ? min(npages_blk, p_begin + SP) - p_begin : 0;
   const int32_t* pt = a.page_table + static_cast<size_t>(slot) * a.pt_stride;
 
+  const int Ceff = nsplit == 1 ? 1 : C;          // CTAs taking part in the merge
+  const int rpo = (rows_alloc + Ceff - 1) / Ceff;  // rows per owner
+  const int blk_floats = NG * rpo * kAttnRecvRow;  // one source CTA's block for one owner
+  uint64_t* recv_bar = full + kAttnStages;
   if (threadIdx.x == 0) {
     tma_prefetch_desc(&tmKV);
     for (int s = 0; s < kAttnStages; ++s) mbar_init(smem_u32(&full[s]), 1);
+    if (Ceff > 1) {
+      mbar_init(smem_u32(recv_bar), 1);
+      mbar_arrive_expect_tx(smem_u32(recv_bar), static_cast<uint32_t>(Ceff * blk_floats * 4));
+    }
     fence_mbar_init();
   }
   __syncthreads();
@@ -325,41 +336,45 @@ __global__ void __launch_bounds__(512)
   l1 += __shfl_xor_sync(0xFFFFFFFFu, l1, 2);
 
   // ---- merge.  Sources: (split c, group g), src = c * NG + g; Ceff splits take part.
-  const int Ceff = nsplit == 1 ? 1 : C;
+  // stage [owner][g][slot][68] in the idle K/V ring; recv [src CTA][g][slot][68].
   const int cself = nsplit == 1 ? 0 : c;
-  const int rpo = (rows_alloc + Ceff - 1) / Ceff;          // rows per owner
-  float* recv = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(full) + 128);  // [src][rpo][68]
-  if (Ceff > 1) cluster_wait();   // every CTA of the cluster runs: peers' shared memory exists
+  float* recv = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(full) + 128);
+  float* stage = Ceff > 1 ? reinterpret_cast<float*>(sK) : recv;
   if (has_rows) {
-    const int src = cself * NG + grp;
 #pragma unroll
     for (int half = 0; half < 2; ++half) {
       const int r = half ? r1 : r0;
       if (r >= R) continue;
-      const int owner = r % Ceff, slot = r / Ceff;
-      const uint32_t base = smem_u32(recv + (src * rpo + slot) * kAttnRecvRow);
-      const float mm = half ? m1 : m0, ll = half ? l1 : l0;
-      if (Ceff == 1) {
-        float* dst = recv + (src * rpo + slot) * kAttnRecvRow;
+      float* dst = stage + (static_cast<size_t>(r % Ceff) * blk_floats) +
+                   (static_cast<size_t>(grp) * rpo + r / Ceff) * kAttnRecvRow;
 #pragma unroll
-        for (int j = 0; j < 8; ++j)
-          *reinterpret_cast<float2*>(dst + 8 * j + 2 * tq) =
-              make_float2(o[j][half * 2 + 0], o[j][half * 2 + 1]);
-        if (tq == 0) {
-          dst[64] = mm;
-          dst[65] = ll;
-        }
-      } else {
-        const uint32_t rb = cluster_map(base, static_cast<uint32_t>(owner));
-#pragma unroll
-        for (int j = 0; j < 8; ++j)
-          st_cluster_f32x2(rb + (8 * j + 2 * tq) * 4, make_float2(o[j][half * 2 + 0], o[j][half * 2 + 1]));
-        if (tq == 0) st_cluster_f32x2(rb + 64 * 4, make_float2(mm, ll));
+      for (int j = 0; j < 8; ++j)
+        *reinterpret_cast<float2*>(dst + 8 * j + 2 * tq) =
+            make_float2(o[j][half * 2 + 0], o[j][half * 2 + 1]);
+      if (tq == 0) {
+        dst[64] = half ? m1 : m0;
+        dst[65] = half ? l1 : l0;
       }
     }
   }
-  if (Ceff == 1) __syncthreads();
-  else cluster_sync_all();   // every partial has landed at its owner
+  bool got = true;
+  if (Ceff == 1) {
+    __syncthreads();
+  } else {
+    fence_proxy_async_smem();
+    __syncthreads();
+    cluster_wait();   // every CTA of the cluster runs: peers' buffers and barriers exist
+    if (threadIdx.x == 0) {
+      const uint32_t bytes = static_cast<uint32_t>(blk_floats * 4);
+      const uint32_t dst_local = smem_u32(recv) + static_cast<uint32_t>(c) * bytes;
+      for (int q = 0; q < Ceff; ++q)
+        bulk_copy_to_peer(cluster_map(dst_local, static_cast<uint32_t>(q)),
+                          smem_u32(stage) + static_cast<uint32_t>(q) * bytes, bytes,
+                          cluster_map(smem_u32(recv_bar), static_cast<uint32_t>(q)));
+      bulk_commit();
+    }
+    got = mbar_wait(smem_u32(recv_bar), 0, a.err);
+  }
 
   // owner: rows r = cself + k * Ceff; one thread per (row, 4 dims); weights
   // exp2(m_src - M) / L over the sources in order.  With one source holding
@@ -369,6 +384,8 @@ __global__ void __launch_bounds__(512)
   for (int idx = threadIdx.x; idx < my_rows * 16; idx += nthreads) {
     const int k = idx >> 4, d4 = (idx & 15) * 4;
     const int r = cself + k * Ceff;
+    // source sidx = c * NG + g lives at recv + c * blk_floats + (g * rpo + k) * 68 =
+    // recv + sidx * rpo * 68 + k * 68
     const float* rowp = recv + k * kAttnRecvRow;
     float M = -INFINITY;
     for (int sidx = 0; sidx < nsrc; ++sidx) M = fmaxf(M, rowp[sidx * rpo * kAttnRecvRow + 64]);
@@ -389,7 +406,7 @@ __global__ void __launch_bounds__(512)
       acc.z += w * v.z;
       acc.w += w * v.w;
     }
-    if (all_ok) {
+    if (all_ok && got) {
       const int t = tok0 + r / a.G;
       const int hq = h * a.G + r % a.G;
       __nv_bfloat16* dst = a.out + (static_cast<size_t>(t) * a.Hq + hq) * 64 + d4;
@@ -397,6 +414,7 @@ __global__ void __launch_bounds__(512)
       *reinterpret_cast<__nv_bfloat162*>(dst + 2) = __floats2bfloat162_rn(acc.z, acc.w);
     }
   }
+  if (Ceff > 1 && threadIdx.x == 0) bulk_wait_read_all();   // outgoing blocks have left `stage`
 }
 
 }  // namespace gs

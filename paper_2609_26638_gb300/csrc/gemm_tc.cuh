@@ -15,9 +15,10 @@
 //
 // Split-K: the CTAs that own different K ranges of one output tile either
 // form a thread-block cluster (decode tiles, BN <= 64) -- each CTA owns a
-// slice of the tile's tokens, every CTA pushes its fp32 partials for that
-// slice into the owner's receive buffer with distributed-shared-memory
-// stores, and after one cluster barrier the owner sums them locally -- or
+// slice of the tile's tokens; every CTA stages its fp32 partials slice by
+// slice in its own shared memory and one thread sends each slice to its
+// owner with a bulk async copy that completes on the owner's mbarrier; the
+// owner then sums the received slices locally -- or
 // write the partials to global scratch, where the last CTA to arrive (atomic
 // ticket, no spinning) sums them.  Both sum the splits in order 0..S-1 from a
 // zero start, so the result does not depend on the path or on arrival order.
@@ -87,6 +88,7 @@ struct GemmShape {
   static constexpr int kRedBytes = BN * 128 * 4;   // cluster reduction tile [BN][128] fp32
   static constexpr int kXBufBytes = 32 * 128 * 4;  // epilogue exchange (SwiGLU, RoPE, sums)
   static_assert(kRedBytes + kXBufBytes <= kStages * kStageBytes, "reduction smem");
+  static_assert(!(BN <= 64) || kXBufBytes + BN * 128 * 4 <= kStages * kStageBytes, "staging smem");
   // RoPE cos/sin rows of the tile's tokens, staged while the mainloop runs (decode tiles)
   static constexpr bool kStageRope = BN <= 64;
   static constexpr int kRopeBytes = kStageRope ? BN * 32 * 8 : 0;
@@ -276,6 +278,7 @@ __global__ void __launch_bounds__(128, 1)
   uint64_t* accum = bars + 2 * S::kStages;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(accum + 1);
   volatile int* flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  uint64_t* recv_bar = accum + 3;   // cluster split-K: partial slices received
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -294,6 +297,13 @@ __global__ void __launch_bounds__(128, 1)
     }
     mbar_init(smem_u32(accum), 1);
     *flag = 0;
+    if constexpr (S::kClusterOk) {
+      if (a.cluster) {
+        mbar_init(smem_u32(recv_bar), 1);
+        // S slices of BN / S tokens x 128 rows of fp32 will arrive
+        mbar_arrive_expect_tx(smem_u32(recv_bar), BN * 128 * 4);
+      }
+    }
     fence_mbar_init();
   }
   if (warp == 2) tmem_alloc(smem_u32(tmem_slot), S::kTmemCols);
@@ -454,37 +464,42 @@ __global__ void __launch_bounds__(128, 1)
 
   if constexpr (S::kClusterOk) {
     if (a.cluster) {
-      // Cluster split-K.  CTA q owns tokens [q*per, (q+1)*per) of the tile;
-      // every CTA pushes its partials for them into q's receive buffer
-      // recv[s][jj][row] (s = pushing split), then one cluster barrier, then
-      // each owner sums its tokens over s = 0..S-1 and runs the epilogue.
-      float* recv = reinterpret_cast<float*>(smem + S::kRecvOffset);
+      // Cluster split-K.  CTA q owns tokens [q*per, (q+1)*per) of the tile.
+      // Stage this CTA's partials token-major in its own shared memory (slice
+      // q contiguous), send slice q to CTA q's receive buffer at position
+      // [split] with one bulk copy, and wait for the S slices of our own
+      // tokens on recv_bar; then sum them over s = 0..S-1.
+      float* recv = reinterpret_cast<float*>(smem + S::kRecvOffset);   // [S][per][128]
+      float* stage = reinterpret_cast<float*>(smA + S::kXBufBytes);   // [BN][128], after xbuf
       float* xbuf = reinterpret_cast<float*>(smA);
       const int per = BN / a.splits;
       const int ntok = min(BN, a.M - tok0);
-      cluster_wait();       // every CTA of the cluster runs: peers' shared memory exists
       if (!failed) {
-        const uint32_t recv0 = smem_u32(recv) + static_cast<uint32_t>(row * 4);
         for (int c = 0; c < BN / 32; ++c) {
           if (c * 32 >= ntok) break;
           float v[32];
           tmem_ld_32x32b_x32(trow + c * 32, v);
 #pragma unroll
-          for (int j = 0; j < 32; ++j) {
-            const int t = c * 32 + j;
-            if (t < ntok) {
-              const int q = t / per, jj = t - q * per;
-              st_cluster_f32(cluster_map(recv0 + static_cast<uint32_t>(((split * per + jj) * 128) * 4),
-                                         static_cast<uint32_t>(q)), v[j]);
-            }
-          }
+          for (int j = 0; j < 32; ++j) stage[(c * 32 + j) * 128 + row] = v[j];
         }
       }
+      fence_proxy_async_smem();
       tc_fence_before();
-      cluster_sync_all();   // every push has landed
+      __syncthreads();
       if (warp == 2) tmem_dealloc(tmem, S::kTmemCols);
+      const uint32_t slice_bytes = static_cast<uint32_t>(per * 128 * 4);
+      cluster_wait();       // every CTA of the cluster runs: peers' buffers and barriers exist
+      if (threadIdx.x == 0) {
+        const uint32_t dst_local = smem_u32(recv) + static_cast<uint32_t>(split) * slice_bytes;
+        for (int q = 0; q < a.splits; ++q)
+          bulk_copy_to_peer(cluster_map(dst_local, static_cast<uint32_t>(q)),
+                            smem_u32(stage) + static_cast<uint32_t>(q) * slice_bytes, slice_bytes,
+                            cluster_map(smem_u32(recv_bar), static_cast<uint32_t>(q)));
+        bulk_commit();
+      }
+      const bool got = mbar_wait(smem_u32(recv_bar), 0, a.err);
       const int lo = split * per, hi = min(lo + per, ntok);
-      if (hi > lo && !failed) {
+      if (hi > lo && !failed && got) {
         const int nq = hi - lo;
         if (per <= 8) {
           float v[8];
@@ -511,6 +526,7 @@ __global__ void __launch_bounds__(128, 1)
                                            rs_of(c));
         }
       }
+      if (threadIdx.x == 0) bulk_wait_read_all();   // our outgoing slices have left `stage`
       return;
     }
   }
