@@ -19,20 +19,20 @@
 //
 // Splits cover fixed absolute page ranges [c*SP, (c+1)*SP), so a row's result
 // depends only on its own keys and not on the window it sits in; keys past a
-// row's limit contribute exact zeros.  The splits of one (block, head) are one
-// thread-block cluster (at most kAttnMaxSplits CTAs).  Row r is owned by CTA
-// r mod C: every warp stages the (O, m, l) partial of its rows, grouped by
-// owner, in its CTA's shared memory; one thread sends each owner its block
-// with a bulk async copy that completes on the owner's mbarrier; each owner
-// then merges its rows over all (split, group) sources in that order.  A
-// block whose keys fit in one split runs in CTA 0 alone and merges its groups
-// the same way without copies.
+// row's limit contribute exact zeros.  The warp groups of a CTA first merge
+// their partials in shared memory (group order).  The splits of one (block,
+// head) are one thread-block cluster (at most kAttnMaxSplits CTAs, a
+// non-portable size above 8).  Row r is owned by CTA r mod C: each CTA stages
+// its (O, m, l) rows grouped by owner and one thread sends each owner its
+// block with a bulk async copy completing on the owner's mbarrier; each owner
+// merges its rows over the splits in order.  A block whose keys fit in one
+// split runs in CTA 0 alone and writes after the group merge.
 #pragma once
 #include "ptx.cuh"
 
 namespace gs {
 
-constexpr int kAttnMaxSplits = 8;
+constexpr int kAttnMaxSplits = 16;
 constexpr int kAttnStages = 6;
 constexpr int kAttnPageBytes = 64 * 128;  // 64 tokens x 64 bf16
 
@@ -61,18 +61,19 @@ __host__ __device__ inline int attn_groups(int r_max) {
 __host__ __device__ inline int attn_threads(int r_max) {
   return attn_mtiles(r_max) * attn_groups(r_max) * 32;
 }
-// receive buffer: per (split, group) source, ceil(rows / C) rows of kAttnRecvRow floats:
+// receive buffer: per source split, ceil(rows / C) rows of kAttnRecvRow floats:
 // O[64], m, l, 2 pad (272 B keeps every row 16-byte aligned for float4 reads)
 constexpr int kAttnRecvRow = 68;
 __host__ __device__ inline int attn_recv_floats(int r_max) {
-  return attn_groups(r_max) * (attn_mtiles(r_max) * 16 + kAttnMaxSplits) * kAttnRecvRow;
+  return (attn_mtiles(r_max) * 16 + kAttnMaxSplits) * kAttnRecvRow;
 }
 __host__ __device__ inline int attn_smem_bytes(int r_max) {
   return 1024 + kAttnStages * 2 * kAttnPageBytes + attn_mtiles(r_max) * 16 * 128 + 128 +
          attn_recv_floats(r_max) * 4;
 }
-static_assert(kAttnStages * 2 * kAttnPageBytes >= 4 * (64 + kAttnMaxSplits) * 68 * 4,
-              "the K/V ring must hold the largest merge staging block");
+static_assert(kAttnStages * 2 * kAttnPageBytes >= 4 * 64 * 68 * 4 &&
+                  kAttnStages * 2 * kAttnPageBytes >= (256 + kAttnMaxSplits) * 68 * 4,
+              "the K/V ring must hold the group partials and the merge staging");
 // Pages per split so that a sequence of `pages` pages needs at most kAttnMaxSplits splits.
 __host__ __device__ inline int attn_min_split_pages(int pages) {
   return (pages + kAttnMaxSplits - 1) / kAttnMaxSplits;
@@ -165,7 +166,7 @@ __global__ void __launch_bounds__(512)
 
   const int Ceff = nsplit == 1 ? 1 : C;          // CTAs taking part in the merge
   const int rpo = (rows_alloc + Ceff - 1) / Ceff;  // rows per owner
-  const int blk_floats = NG * rpo * kAttnRecvRow;  // one source CTA's block for one owner
+  const int blk_floats = rpo * kAttnRecvRow;       // one source CTA's block for one owner
   uint64_t* recv_bar = full + kAttnStages;
   if (threadIdx.x == 0) {
     tma_prefetch_desc(&tmKV);
@@ -335,18 +336,89 @@ __global__ void __launch_bounds__(512)
   l1 += __shfl_xor_sync(0xFFFFFFFFu, l1, 1);
   l1 += __shfl_xor_sync(0xFFFFFFFFu, l1, 2);
 
-  // ---- merge.  Sources: (split c, group g), src = c * NG + g; Ceff splits take part.
-  // stage [owner][g][slot][68] in the idle K/V ring; recv [src CTA][g][slot][68].
-  const int cself = nsplit == 1 ? 0 : c;
+  // ---- 1. groups -> group 0 (shared memory, group order): O = sum w_g O_g,
+  //         L = sum w_g l_g, w_g = exp2(m_g - M).  gp [g][row][68] in the idle K/V ring.
+  float* ring = reinterpret_cast<float*>(sK);
+  if (NG > 1) {
+    if (grp > 0 && has_rows) {
+#pragma unroll
+      for (int half = 0; half < 2; ++half) {
+        float* dst = ring + (static_cast<size_t>(grp) * rows_alloc + (half ? r1 : r0)) * kAttnRecvRow;
+#pragma unroll
+        for (int j = 0; j < 8; ++j)
+          *reinterpret_cast<float2*>(dst + 8 * j + 2 * tq) =
+              make_float2(o[j][half * 2 + 0], o[j][half * 2 + 1]);
+        if (tq == 0) {
+          dst[64] = half ? m1 : m0;
+          dst[65] = half ? l1 : l0;
+        }
+      }
+    }
+    __syncthreads();
+    if (grp == 0 && has_rows) {
+#pragma unroll
+      for (int half = 0; half < 2; ++half) {
+        const int r = half ? r1 : r0;
+        const float mself = half ? m1 : m0;
+        float M = mself;
+        for (int q = 1; q < NG; ++q)
+          M = fmaxf(M, ring[(static_cast<size_t>(q) * rows_alloc + r) * kAttnRecvRow + 64]);
+        const float w0 = (mself == -INFINITY) ? 0.f : exp2f(mself - M);
+        float L = w0 * (half ? l1 : l0);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          o[j][half * 2 + 0] *= w0;
+          o[j][half * 2 + 1] *= w0;
+        }
+        for (int q = 1; q < NG; ++q) {
+          const float* src = ring + (static_cast<size_t>(q) * rows_alloc + r) * kAttnRecvRow;
+          const float mq = src[64];
+          const float wq = (mq == -INFINITY) ? 0.f : exp2f(mq - M);
+          L += wq * src[65];
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            const float2 v = *reinterpret_cast<const float2*>(src + 8 * j + 2 * tq);
+            o[j][half * 2 + 0] += wq * v.x;
+            o[j][half * 2 + 1] += wq * v.y;
+          }
+        }
+        if (half) { m1 = M; l1 = L; } else { m0 = M; l0 = L; }
+      }
+    }
+    __syncthreads();   // group partials consumed; the ring is reused below
+  }
+  const bool lead = grp == 0 && has_rows;
+
+  if (Ceff == 1) {   // one split: the CTA's merged rows are final
+    if (lead && all_ok) {
+#pragma unroll
+      for (int half = 0; half < 2; ++half) {
+        const int r = half ? r1 : r0;
+        if (r >= R) continue;
+        const float inv = 1.0f / (half ? l1 : l0);
+        const int t = tok0 + r / a.G;
+        const int hq = h * a.G + r % a.G;
+        __nv_bfloat16* dst = a.out + (static_cast<size_t>(t) * a.Hq + hq) * 64;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          const float x0 = o[j][half * 2 + 0] * inv, x1 = o[j][half * 2 + 1] * inv;
+          *reinterpret_cast<__nv_bfloat162*>(dst + 8 * j + 2 * tq) = __floats2bfloat162_rn(x0, x1);
+        }
+      }
+    }
+    return;
+  }
+
+  // ---- 2. splits -> owners (cluster).  stage [owner][slot][68] in the ring,
+  //         recv [source split][slot][68].
   float* recv = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(full) + 128);
-  float* stage = Ceff > 1 ? reinterpret_cast<float*>(sK) : recv;
-  if (has_rows) {
+  float* stage = ring;
+  if (lead) {
 #pragma unroll
     for (int half = 0; half < 2; ++half) {
       const int r = half ? r1 : r0;
       if (r >= R) continue;
-      float* dst = stage + (static_cast<size_t>(r % Ceff) * blk_floats) +
-                   (static_cast<size_t>(grp) * rpo + r / Ceff) * kAttnRecvRow;
+      float* dst = stage + static_cast<size_t>(r % Ceff) * blk_floats + (r / Ceff) * kAttnRecvRow;
 #pragma unroll
       for (int j = 0; j < 8; ++j)
         *reinterpret_cast<float2*>(dst + 8 * j + 2 * tq) =
@@ -357,50 +429,51 @@ __global__ void __launch_bounds__(512)
       }
     }
   }
-  bool got = true;
-  if (Ceff == 1) {
-    __syncthreads();
-  } else {
-    fence_proxy_async_smem();
-    __syncthreads();
-    cluster_wait();   // every CTA of the cluster runs: peers' buffers and barriers exist
-    if (threadIdx.x == 0) {
-      const uint32_t bytes = static_cast<uint32_t>(blk_floats * 4);
-      const uint32_t dst_local = smem_u32(recv) + static_cast<uint32_t>(c) * bytes;
-      for (int q = 0; q < Ceff; ++q)
-        bulk_copy_to_peer(cluster_map(dst_local, static_cast<uint32_t>(q)),
-                          smem_u32(stage) + static_cast<uint32_t>(q) * bytes, bytes,
-                          cluster_map(smem_u32(recv_bar), static_cast<uint32_t>(q)));
-      bulk_commit();
-    }
-    got = mbar_wait(smem_u32(recv_bar), 0, a.err);
+  fence_proxy_async_smem();
+  __syncthreads();
+  cluster_wait();   // every CTA of the cluster runs: peers' buffers and barriers exist
+  if (threadIdx.x == 0) {
+    const uint32_t bytes = static_cast<uint32_t>(blk_floats * 4);
+    const uint32_t dst_local = smem_u32(recv) + static_cast<uint32_t>(c) * bytes;
+    for (int q = 0; q < Ceff; ++q)
+      bulk_copy_to_peer(cluster_map(dst_local, static_cast<uint32_t>(q)),
+                        smem_u32(stage) + static_cast<uint32_t>(q) * bytes, bytes,
+                        cluster_map(smem_u32(recv_bar), static_cast<uint32_t>(q)));
+    bulk_commit();
   }
+  const bool got = mbar_wait(smem_u32(recv_bar), 0, a.err);
 
-  // owner: rows r = cself + k * Ceff; one thread per (row, 4 dims); weights
-  // exp2(m_src - M) / L over the sources in order.  With one source holding
-  // all of a row's keys this is O * (1 / l).
-  const int nsrc = Ceff * NG;
-  const int my_rows = (R - cself + Ceff - 1) / Ceff;
-  for (int idx = threadIdx.x; idx < my_rows * 16; idx += nthreads) {
-    const int k = idx >> 4, d4 = (idx & 15) * 4;
-    const int r = cself + k * Ceff;
-    // source sidx = c * NG + g lives at recv + c * blk_floats + (g * rpo + k) * 68 =
-    // recv + sidx * rpo * 68 + k * 68
-    const float* rowp = recv + k * kAttnRecvRow;
+  // ---- 3. owner merge of rows r = c + k * C over the splits in order:
+  //         per row the weights w_s = exp2(m_s - M) / L (one thread per row),
+  //         then one thread per (row, 4 dims) sums w_s O_s.  With one split
+  //         holding all of a row's keys this is O * (1 / l), the direct path.
+  const int my_rows = (R - c + Ceff - 1) / Ceff;
+  for (int k = threadIdx.x; k < my_rows; k += nthreads) {
     float M = -INFINITY;
-    for (int sidx = 0; sidx < nsrc; ++sidx) M = fmaxf(M, rowp[sidx * rpo * kAttnRecvRow + 64]);
+    for (int sidx = 0; sidx < Ceff; ++sidx)
+      M = fmaxf(M, recv[(sidx * rpo + k) * kAttnRecvRow + 64]);
     float L = 0.f;
-    for (int sidx = 0; sidx < nsrc; ++sidx) {
-      const float ms = rowp[sidx * rpo * kAttnRecvRow + 64];
-      const float w = (ms == -INFINITY) ? 0.f : exp2f(ms - M);
-      L += w * rowp[sidx * rpo * kAttnRecvRow + 65];
+    for (int sidx = 0; sidx < Ceff; ++sidx) {
+      float* p = recv + (sidx * rpo + k) * kAttnRecvRow;
+      const float w = (p[64] == -INFINITY) ? 0.f : exp2f(p[64] - M);
+      p[66] = w;
+      L += w * p[65];
     }
     const float inv = 1.0f / L;
+    for (int sidx = 0; sidx < Ceff; ++sidx) {
+      float* p = recv + (sidx * rpo + k) * kAttnRecvRow;
+      p[66] = p[66] * inv;
+    }
+  }
+  __syncthreads();
+  for (int idx = threadIdx.x; idx < my_rows * 16; idx += nthreads) {
+    const int k = idx >> 4, d4 = (idx & 15) * 4;
+    const int r = c + k * Ceff;
     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-    for (int sidx = 0; sidx < nsrc; ++sidx) {
-      const float ms = rowp[sidx * rpo * kAttnRecvRow + 64];
-      const float w = ((ms == -INFINITY) ? 0.f : exp2f(ms - M)) * inv;
-      const float4 v = *reinterpret_cast<const float4*>(rowp + sidx * rpo * kAttnRecvRow + d4);
+    for (int sidx = 0; sidx < Ceff; ++sidx) {
+      const float* p = recv + (sidx * rpo + k) * kAttnRecvRow;
+      const float w = p[66];
+      const float4 v = *reinterpret_cast<const float4*>(p + d4);
       acc.x += w * v.x;
       acc.y += w * v.y;
       acc.z += w * v.z;
@@ -414,7 +487,7 @@ __global__ void __launch_bounds__(512)
       *reinterpret_cast<__nv_bfloat162*>(dst + 2) = __floats2bfloat162_rn(acc.z, acc.w);
     }
   }
-  if (Ceff > 1 && threadIdx.x == 0) bulk_wait_read_all();   // outgoing blocks have left `stage`
+  if (threadIdx.x == 0) bulk_wait_read_all();   // outgoing blocks have left `stage`
 }
 
 }  // namespace gs
