@@ -21,8 +21,8 @@
 // depends only on its own keys and not on the window it sits in; keys past a
 // row's limit contribute exact zeros.  The warp groups of a CTA first merge
 // their partials in shared memory (group order).  The splits of one (block,
-// head) are one thread-block cluster (at most kAttnMaxSplits CTAs, a
-// non-portable size above 8).  Row r is owned by CTA r mod C: each CTA stages
+// head) are one thread-block cluster (at most kAttnMaxSplits CTAs; 16-CTA
+// clusters measured slower: they wait for 16 free SMs in one GPC).  Row r is owned by CTA r mod C: each CTA stages
 // its (O, m, l) rows grouped by owner and one thread sends each owner its
 // block with a bulk async copy completing on the owner's mbarrier; each owner
 // merges its rows over the splits in order.  A block whose keys fit in one
@@ -32,7 +32,7 @@
 
 namespace gs {
 
-constexpr int kAttnMaxSplits = 16;
+constexpr int kAttnMaxSplits = 8;
 constexpr int kAttnStages = 6;
 constexpr int kAttnPageBytes = 64 * 128;  // 64 tokens x 64 bf16
 

@@ -529,8 +529,7 @@ int gs_create(const gs_config* cfg, const gs_weights* w, void* workspace, size_t
     if (e == cudaSuccess)
       e = cudaFuncSetAttribute(attn_paged_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                attn_smem_bytes(256));
-    if (e == cudaSuccess)   // KV-split clusters of up to 16 CTAs
-      e = cudaFuncSetAttribute(attn_paged_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+
     if (e != cudaSuccess)
       return fail(nullptr, GS_ERR_CUDA, std::string("kernel attributes: ") + cudaGetErrorString(e));
     attrs_done = true;
@@ -831,9 +830,7 @@ int gs_attention(int mode, const void* q, const void* kv, int n_pages, const int
   static bool attr = false;
   if (!attr) {
     if (cudaFuncSetAttribute(attn_paged_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             attn_smem_bytes(256)) != cudaSuccess ||
-        cudaFuncSetAttribute(attn_paged_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed,
-                             1) != cudaSuccess)
+                             attn_smem_bytes(256)) != cudaSuccess)
       return GS_ERR_CUDA;
     attr = true;
   }
