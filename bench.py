@@ -112,6 +112,37 @@ class ClockSampler:
                 "samples": len(mhz)}
 
 
+def kernel_bytes(cfg, kind: str, T: int, ctx: list) -> int | None:
+    """Algorithmic HBM bytes of one launch of `kind` over T window rows.
+
+    Each operand counted once at its storage width: bf16 weights, bf16
+    activations, float32 residual stream (read and written), float32 per-128
+    feature sums of squares (the folded RMSNorm), 8-byte argmax keys.  For
+    attention, ctx[i] is sequence i's visible keys (cached prefix + window):
+    K and V rows of every KV head, plus the bf16 queries read and outputs
+    written.  None for the small window / accept kernels (no bandwidth model).
+    """
+    d, F, V = cfg.d_model, cfg.d_ffn, cfg.vocab
+    Hq, Hkv, hd = cfg.n_heads, cfg.n_kv_heads, cfg.head_dim
+    HD, qkv = Hq * hd, cfg.qkv_dim
+    ssp = T * (d // 128) * 4
+    if kind == "qkv":
+        return 2 * qkv * d + 2 * T * d + ssp + 2 * T * HD + 2 * T * 2 * Hkv * hd
+    if kind == "attention":
+        return sum(c * Hkv * hd * 2 * 2 for c in ctx) + 2 * (2 * T * HD)
+    if kind == "o_proj":
+        return 2 * d * HD + 2 * T * HD + 2 * 4 * T * d + 2 * T * d + ssp
+    if kind == "gate_up":
+        return 2 * 2 * F * d + 2 * T * d + ssp + 2 * T * F
+    if kind == "down":
+        return 2 * d * F + 2 * T * F + 2 * 4 * T * d + 2 * T * d + ssp
+    if kind == "lm_head":
+        return 2 * V * d + 2 * T * d + ssp + 8 * T
+    if kind == "embed":
+        return 2 * T * d + 4 * T * d + 2 * T * d + ssp
+    return None
+
+
 # ---------------------------------------------------------------------- GPU arm
 def gpu_arm(args, rank: int, world: int):
     import torch
@@ -239,13 +270,44 @@ def gpu_arm(args, rank: int, world: int):
     barrier()
     e_elapsed = time.perf_counter() - e0
 
-    # roofline: the LM-head GEMM (largest single kernel of the round), timed alone
-    roof = lm_head_roofline(eng, cfg, K, dev)
+    # per-kernel device times: the same forced decode once more, every round
+    # enqueued eagerly with a CUDA event after each launch (gs_round_profile)
+    hbm, _, src = load_peaks()
+    W = K + 1
+    per = {}
+    eng.restore(0, P, x0, 1, max_new, 0, 0)
+    for r in range(R):
+        ctx = [eng.state(0)["seq_len"] + W]
+        for name, ms in eng.round_profile(slots, K, out_tok, out_cnt, out_done, force=force):
+            e = per.setdefault(name, [0, 0.0, 0])
+            e[0] += 1
+            e[1] += ms
+            b = kernel_bytes(cfg, name, W, ctx)
+            e[2] += b or 0
+    eng.check()
+    kernels = {}
+    for name, (n, ms, b) in sorted(per.items(), key=lambda kv: -kv[1][1]):
+        k = {"launches": n, "total_ms": round(ms, 3), "us_per_launch": round(1e3 * ms / n, 2)}
+        if b:
+            k["bytes_per_launch"] = b // n
+            k["gb_s"] = round(b / (ms * 1e-3) / 1e9, 1)
+            k["frac_hbm"] = round(b / (ms * 1e-3) / 1e9 / hbm, 4)
+        kernels[name] = k
+    dom = max((n for n in kernels if "gb_s" in kernels[n]), key=lambda n: kernels[n]["total_ms"])
+    dk = kernels[dom]
+    roof = {"kernel": f"{dom} (gemm_tc_kernel / attn_paged_kernel by kind), decode shape "
+                      f"{W} rows", "bound": "hbm", "achieved": dk["gb_s"], "peak": hbm,
+            "unit": "GB/s", "frac": dk["frac_hbm"], "peak_source": src,
+            "algorithmic_bytes_per_launch": dk["bytes_per_launch"],
+            "us_per_launch": dk["us_per_launch"], "launches_per_step": dk["launches"],
+            "timing": "CUDA events around each launch of one eagerly enqueued decode "
+                      "(no launch overlap)", "traffic": None}
+    lm = lm_head_roofline(eng, cfg, K, dev)
     attn = attention_roofline(cfg, dev)
     res = dict(elapsed=elapsed, e2e_elapsed=e_elapsed, tokens=committed_per_decode * args.steps,
                round_ms=round_ms, rounds=R, launches_per_round=launches_per_round,
                ok_sched=ok_sched, ok_tokens=ok_tokens, clocks=clk.summary(), roofline=roof,
-               attention=attn, h2d=int(teacher.nbytes + sched.nbytes),
+               kernels=kernels, lm_head=lm, attention=attn, h2d=int(teacher.nbytes + sched.nbytes),
                d2h=int(R * (K + 2) * 4 + R * 4), P=P, K=K, max_new=max_new)
     eng.close()
     return res
@@ -455,8 +517,8 @@ def main():
             + args.steps,
             "e2e": {"value": round(tokens_all / ee, 1), "unit": UNIT,
                     "h2d_bytes_per_step": res["h2d"], "d2h_bytes_per_step": res["d2h"]},
-            "clocks": res["clocks"], "roofline": res["roofline"],
-            "attention_roofline": res["attention"]}
+            "clocks": res["clocks"], "roofline": res["roofline"], "kernels": res["kernels"],
+            "lm_head_alone": res["lm_head"], "attention_roofline": res["attention"]}
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         times, counts = oracle_sample(synth.WORKLOADS[args.workload], 6, 1, budget_s=25.0)
         line["cpu_baseline"] = {

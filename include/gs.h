@@ -180,6 +180,38 @@ int gs_seq_state(gs_handle *h, int slot, int *seq_len, int *x0, int *n_out, int 
 /* Number of kernel launches the most recent gs_round enqueued (or captured). */
 int gs_round_launches(gs_handle *h);
 
+/* Kinds of kernel reported by gs_round_profile (one per launch). */
+enum {
+  GS_KIND_WINDOW = 0,    /* draft window build or verify input build (Sec. 3.2) */
+  GS_KIND_EMBED = 1,     /* token embedding + first RMSNorm input */
+  GS_KIND_QKV = 2,       /* QKV projection + RoPE + KV-cache write */
+  GS_KIND_ATTENTION = 3, /* hybrid-mask paged attention (Eq. 3 / Eq. 5 masks) */
+  GS_KIND_O_PROJ = 4,    /* output projection + residual */
+  GS_KIND_GATE_UP = 5,   /* gate/up projection + SwiGLU */
+  GS_KIND_DOWN = 6,      /* down projection + residual */
+  GS_KIND_LM_HEAD = 7,   /* LM head + greedy argmax */
+  GS_KIND_ACCEPT = 8     /* longest-prefix acceptance and commit (Sec. 3.3) */
+};
+
+/* Measurement aid: one greedy round, with the same arguments and effects as
+ * gs_round(h, slots, n_seq, K, GS_ACCEPT_GREEDY, force, out_tok, out_cnt,
+ * out_done, NULL), enqueued eagerly (never from the graph cache) with a CUDA
+ * event recorded after every kernel launch.  The paper has no counterpart.
+ *   ms[i]       device milliseconds between launch i-1's end event and launch
+ *               i's end event (for i = 0, from an event recorded before the
+ *               round).  An event between two kernels stops the second from
+ *               starting early, so each figure is the kernel alone plus the
+ *               gap the front end needs to start it.
+ *   kind[i]     GS_KIND_* of launch i.
+ *   n_launches  number of launches written.
+ * ms and kind are host arrays of max_launches entries.  Synchronises the
+ * handle's stream (which must not be the default stream).
+ * Errors: GS_ERR_INVALID_ARG (bad arguments, max_launches too small — the
+ * round has then run), GS_ERR_CUDA. */
+int gs_round_profile(gs_handle *h, const int32_t *slots, int n_seq, int K, const gs_force *force,
+                     int32_t *out_tok, int32_t *out_cnt, int32_t *out_done, int max_launches,
+                     float *ms, int *kind, int *n_launches);
+
 /* Free the slot's KV pages (host bookkeeping only). */
 int gs_release(gs_handle *h, int slot);
 

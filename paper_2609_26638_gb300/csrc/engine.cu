@@ -156,6 +156,12 @@ struct gs_handle {
   std::map<GraphKey, cudaGraphExec_t> graphs;
   int launches = 0;             // kernel launches counted while enqueueing
   int last_round_launches = 0;
+
+  // gs_round_profile: an event after every launch and the launch's kind
+  bool profiling = false;
+  cudaError_t prof_err = cudaSuccess;
+  std::vector<cudaEvent_t> prof_ev;
+  std::vector<int> prof_kind;
 };
 
 namespace {
@@ -172,6 +178,26 @@ int fail(gs_handle* h, int code, const std::string& msg) {
     if (e_ != cudaSuccess)                                                            \
       return fail(h, GS_ERR_CUDA, std::string(#call " -> ") + cudaGetErrorString(e_)); \
   } while (0)
+
+// Counts one kernel launch; under gs_round_profile also records an event
+// behind it on the handle's stream and remembers what kind of kernel it was.
+void note_launch(gs_handle* h, int kind) {
+  ++h->launches;
+  if (!h->profiling) return;
+  const size_t i = h->prof_kind.size() + 1;  // event 0 marks the start of the round
+  while (h->prof_ev.size() <= i) {
+    cudaEvent_t e;
+    cudaError_t r = cudaEventCreate(&e);
+    if (r != cudaSuccess) {
+      if (h->prof_err == cudaSuccess) h->prof_err = r;
+      return;
+    }
+    h->prof_ev.push_back(e);
+  }
+  cudaError_t r = cudaEventRecord(h->prof_ev[i], h->stream);
+  if (r != cudaSuccess && h->prof_err == cudaSuccess) h->prof_err = r;
+  h->prof_kind.push_back(kind);
+}
 
 int bn_index(int bn) { return bn == 32 ? 0 : (bn == 64 ? 1 : (bn == 128 ? 2 : 3)); }
 
@@ -298,7 +324,7 @@ GemmArgs gemm_base(gs_handle* h) {
 }
 
 int run_gemm(gs_handle* h, const CUtensorMap& tw, int weight_rows, const CUtensorMap* tx_set, int K,
-             int T, int epi, GemmArgs a, bool decode) {
+             int T, int epi, GemmArgs a, bool decode, int kind) {
   const GemmPlan p = plan_gemm(weight_rows, K, T, decode);
   a.M = T;
   a.K = K;
@@ -311,7 +337,7 @@ int run_gemm(gs_handle* h, const CUtensorMap& tw, int weight_rows, const CUtenso
     return fail(h, GS_ERR_OOM, "split-K scratch too small");
   GS_CUDA(h, launch_gemm(p.bn, epi, tw, tx_set[bn_index(p.bn)], a, p.feat_tiles, p.tok_tiles,
                          h->stream, true));
-  ++h->launches;
+  note_launch(h, kind);
   return GS_OK;
 }
 
@@ -346,7 +372,7 @@ int run_attention(gs_handle* h, int layer, int T, const AttnLaunch& L) {
   GS_CUDA(h, launch_ex(attn_paged_kernel, grid, dim3(attn_threads(L.r_max)),
                        attn_smem_bytes(L.r_max), h->stream, true, dim3(L.max_splits, 1, 1), h->tm_kv,
                        a));
-  ++h->launches;
+  note_launch(h, GS_KIND_ATTENTION);
   return GS_OK;
 }
 
@@ -364,7 +390,7 @@ int forward(gs_handle* h, int T, const int32_t* tok, const __nv_bfloat16* vis, i
   GS_CUDA(h, launch_ex(embed_kernel, dim3(T), dim3(128), 0, h->stream, true, dim3(1), tok, h->embed, vis,
                        n_vis, T, d, c.vocab, h->hbuf, h->hb, h->attn_norm[0], h->ssp, packed,
                        h->err_word));
-  ++h->launches;
+  note_launch(h, GS_KIND_EMBED);
   const size_t layer_kv = static_cast<size_t>(h->n_pages) * 2 * c.n_kv_heads * 64 * 64;
   int rc;
   for (int l = 0; l < L; ++l) {
@@ -382,7 +408,9 @@ int forward(gs_handle* h, int T, const int32_t* tok, const __nv_bfloat16* vis, i
     q.max_ctx = c.max_ctx;
     q.Hq = c.n_heads;
     q.Hkv = c.n_kv_heads;
-    if ((rc = run_gemm(h, h->tm_qkv[l], h->qkv_dim, h->tm_hb, d, T, kEpiQKV, q, decode))) return rc;
+    if ((rc = run_gemm(h, h->tm_qkv[l], h->qkv_dim, h->tm_hb, d, T, kEpiQKV, q, decode,
+                       GS_KIND_QKV)))
+      return rc;
     if ((rc = run_attention(h, l, T, AL))) return rc;
     GemmArgs o = gemm_base(h);
     o.N = d;
@@ -391,13 +419,17 @@ int forward(gs_handle* h, int T, const int32_t* tok, const __nv_bfloat16* vis, i
     o.hb_out = h->hb;
     o.g_next = h->ffn_norm[l];
     o.ssp_out = h->ssp;
-    if ((rc = run_gemm(h, h->tm_o[l], d, h->tm_ao, HD, T, kEpiResidF32, o, decode))) return rc;
+    if ((rc = run_gemm(h, h->tm_o[l], d, h->tm_ao, HD, T, kEpiResidF32, o, decode,
+                       GS_KIND_O_PROJ)))
+      return rc;
     GemmArgs gu = gemm_base(h);
     gu.N = F;
     gu.y = h->act;
     gu.ldy = F;
     gu.ssp_in = h->ssp;
-    if ((rc = run_gemm(h, h->tm_gu[l], 2 * F, h->tm_hb, d, T, kEpiSwiGLU, gu, decode))) return rc;
+    if ((rc = run_gemm(h, h->tm_gu[l], 2 * F, h->tm_hb, d, T, kEpiSwiGLU, gu, decode,
+                       GS_KIND_GATE_UP)))
+      return rc;
     GemmArgs dn = gemm_base(h);
     dn.N = d;
     dn.y = h->hbuf;
@@ -405,7 +437,9 @@ int forward(gs_handle* h, int T, const int32_t* tok, const __nv_bfloat16* vis, i
     dn.hb_out = h->hb;
     dn.g_next = l + 1 < L ? h->attn_norm[l + 1] : h->final_norm;
     dn.ssp_out = h->ssp;
-    if ((rc = run_gemm(h, h->tm_down[l], d, h->tm_act, F, T, kEpiResidF32, dn, decode))) return rc;
+    if ((rc = run_gemm(h, h->tm_down[l], d, h->tm_act, F, T, kEpiResidF32, dn, decode,
+                       GS_KIND_DOWN)))
+      return rc;
   }
   if (n_lm == 0) return GS_OK;
   GemmArgs lm = gemm_base(h);
@@ -414,7 +448,8 @@ int forward(gs_handle* h, int T, const int32_t* tok, const __nv_bfloat16* vis, i
   lm.logits = logits;
   lm.ssp_in = h->ssp;
   lm.x_row0 = lm_row0;
-  return run_gemm(h, h->tm_lm, c.vocab, h->tm_hb, d, n_lm, kEpiArgmax, lm, decode);
+  return run_gemm(h, h->tm_lm, c.vocab, h->tm_hb, d, n_lm, kEpiArgmax, lm, decode,
+                  GS_KIND_LM_HEAD);
 }
 
 int enqueue_round(gs_handle* h, const int32_t* slots, int n_seq, int K, const gs_force* force,
@@ -459,12 +494,12 @@ int enqueue_round(gs_handle* h, const int32_t* slots, int n_seq, int K, const gs
 
   h->launches = 0;
   GS_CUDA(h, launch_ex(window_draft_kernel, dim3(nb), dim3(128), 0, h->stream, true, dim3(1), w));
-  ++h->launches;
+  note_launch(h, GS_KIND_WINDOW);
   int rc = forward(h, T, h->tok, nullptr, 0, AL, 0, T, h->packed_d,
                    dbg ? dbg->draft_logits : nullptr, true);
   if (rc) return rc;
   GS_CUDA(h, launch_ex(window_verify_kernel, dim3(nb), dim3(128), 0, h->stream, true, dim3(1), w));
-  ++h->launches;
+  note_launch(h, GS_KIND_WINDOW);
   rc = forward(h, T, h->tok, nullptr, 0, AL, 0, T, h->packed_v, dbg ? dbg->verify_logits : nullptr,
                true);
   if (rc) return rc;
@@ -483,7 +518,7 @@ int enqueue_round(gs_handle* h, const int32_t* slots, int n_seq, int K, const gs
   ac.out_done = out_done;
   GS_CUDA(h, launch_ex(accept_commit_kernel, dim3(cdiv(n_seq, 64)), dim3(64), 0, h->stream, true, dim3(1),
                        ac));
-  ++h->launches;
+  note_launch(h, GS_KIND_ACCEPT);
   if (dbg) {
     if (dbg->draft_tok) copy_i32_kernel<<<nb, 128, 0, h->stream>>>(h->draft_tok, dbg->draft_tok, T);
     if (dbg->verify_in) copy_i32_kernel<<<nb, 128, 0, h->stream>>>(h->verify_in, dbg->verify_in, T);
@@ -609,6 +644,7 @@ int gs_create(const gs_config* cfg, const gs_weights* w, void* workspace, size_t
 int gs_destroy(gs_handle* h) {
   if (!h) return GS_ERR_INVALID_ARG;
   for (auto& kv : h->graphs) cudaGraphExecDestroy(kv.second);
+  for (cudaEvent_t e : h->prof_ev) cudaEventDestroy(e);
   delete h;
   return GS_OK;
 }
@@ -756,6 +792,46 @@ int gs_seq_restore(gs_handle* h, int slot, int seq_len, int x0, int n_out, int m
 }
 
 int gs_round_launches(gs_handle* h) { return h ? h->last_round_launches : 0; }
+
+int gs_round_profile(gs_handle* h, const int32_t* slots, int n_seq, int K, const gs_force* force,
+                     int32_t* out_tok, int32_t* out_cnt, int32_t* out_done, int max_launches,
+                     float* ms, int* kind, int* n_launches) {
+  if (!h) return GS_ERR_INVALID_ARG;
+  if (!ms || !kind || !n_launches || max_launches < 1)
+    return fail(h, GS_ERR_INVALID_ARG, "null or empty profile output");
+  if (!h->stream) return fail(h, GS_ERR_INVALID_ARG, "profiling needs a non-default stream");
+  const gs_config& c = h->cfg;
+  if (!slots || !out_tok || !out_cnt || !out_done)
+    return fail(h, GS_ERR_INVALID_ARG, "null slots or output pointer");
+  if (n_seq < 1 || n_seq > c.max_batch) return fail(h, GS_ERR_INVALID_ARG, "n_seq out of range");
+  if (K < 0 || K > c.max_K) return fail(h, GS_ERR_INVALID_ARG, "K out of range");
+  if (force && (!force->teacher || !force->L_sched || force->teacher_stride < 1))
+    return fail(h, GS_ERR_INVALID_ARG, "incomplete force hook");
+  *n_launches = 0;
+  if (h->prof_ev.empty()) {
+    cudaEvent_t e;
+    GS_CUDA(h, cudaEventCreate(&e));
+    h->prof_ev.push_back(e);
+  }
+  h->prof_kind.clear();
+  h->prof_err = cudaSuccess;
+  GS_CUDA(h, cudaEventRecord(h->prof_ev[0], h->stream));
+  h->profiling = true;
+  const int rc = enqueue_round(h, slots, n_seq, K, force, out_tok, out_cnt, out_done, nullptr);
+  h->profiling = false;
+  if (rc) return rc;
+  if (h->prof_err != cudaSuccess)
+    return fail(h, GS_ERR_CUDA, std::string("profile events: ") + cudaGetErrorString(h->prof_err));
+  GS_CUDA(h, cudaStreamSynchronize(h->stream));
+  const int n = static_cast<int>(h->prof_kind.size());
+  if (n > max_launches) return fail(h, GS_ERR_INVALID_ARG, "max_launches below the round's launches");
+  for (int i = 0; i < n; ++i) {
+    GS_CUDA(h, cudaEventElapsedTime(&ms[i], h->prof_ev[i], h->prof_ev[i + 1]));
+    kind[i] = h->prof_kind[i];
+  }
+  *n_launches = n;
+  return GS_OK;
+}
 
 int gs_seq_state(gs_handle* h, int slot, int* seq_len, int* x0, int* n_out, int* done, int* rounds) {
   if (!h) return GS_ERR_INVALID_ARG;

@@ -24,6 +24,8 @@ GS_ACCEPT_GREEDY = 0
 GS_ACCEPT_STOCHASTIC = 1
 EPI_STORE_BF16, EPI_RESID_F32, EPI_SWIGLU, EPI_ARGMAX = 0, 1, 2, 3
 ATTN_DRAFT, ATTN_VERIFY = 0, 1
+KIND_NAMES = ("window", "embed", "qkv", "attention", "o_proj", "gate_up", "down", "lm_head",
+              "accept")
 
 ERROR_NAMES = {0: "GS_OK", 1: "GS_ERR_INVALID_ARG", 2: "GS_ERR_OOM", 3: "GS_ERR_UNSUPPORTED",
                4: "GS_ERR_CUDA", 5: "GS_ERR_DEVICE_CHECK", 6: "GS_ERR_TIMEOUT"}
@@ -79,6 +81,9 @@ def _load():
                            ctypes.POINTER(gs_debug)]),
         "gs_seq_restore": (i32, [vp, i32, i32, i32, i32, i32, i32, i32]),
         "gs_round_launches": (i32, [vp]),
+        "gs_round_profile": (i32, [vp, vp, i32, i32, ctypes.POINTER(gs_force), vp, vp, vp, i32,
+                                   ctypes.POINTER(ctypes.c_float), ctypes.POINTER(i32),
+                                   ctypes.POINTER(i32)]),
         "gs_seq_state": (i32, [vp, i32] + [ctypes.POINTER(i32)] * 5),
         "gs_release": (i32, [vp, i32]),
         "gs_sync_check": (i32, [vp]),
@@ -98,7 +103,8 @@ def _load():
 
 _lib = _load()
 EXPORTED = ("gs_workspace_bytes", "gs_create", "gs_destroy", "gs_last_error", "gs_prefill",
-            "gs_round", "gs_seq_restore", "gs_round_launches", "gs_seq_state", "gs_release", "gs_sync_check",
+            "gs_round", "gs_seq_restore", "gs_round_launches", "gs_round_profile", "gs_seq_state",
+            "gs_release", "gs_sync_check",
             "gs_attention_scratch_bytes", "gs_attention", "gs_linear_scratch_bytes", "gs_linear",
             "gs_linear_noalloc")
 
@@ -156,6 +162,20 @@ def gs_seq_restore(h, slot: int, seq_len: int, x0: int, n_out: int, max_new: int
 
 def gs_round_launches(h) -> int:
     return int(_lib.gs_round_launches(h))
+
+
+def gs_round_profile(h, slots_ptr: int, n_seq: int, K: int, force: gs_force | None,
+                     out_tok_ptr: int, out_cnt_ptr: int, out_done_ptr: int,
+                     max_launches: int = 4096) -> list[tuple[int, float]]:
+    """(kind, device ms) per kernel launch of one eagerly enqueued round."""
+    ms = (ctypes.c_float * max_launches)()
+    kind = (ctypes.c_int * max_launches)()
+    n = ctypes.c_int()
+    _check(h, _lib.gs_round_profile(h, slots_ptr, n_seq, K,
+                                    ctypes.byref(force) if force is not None else None,
+                                    out_tok_ptr, out_cnt_ptr, out_done_ptr, max_launches, ms, kind,
+                                    ctypes.byref(n)))
+    return [(int(kind[i]), float(ms[i])) for i in range(n.value)]
 
 
 def gs_seq_state(h, slot: int) -> dict:

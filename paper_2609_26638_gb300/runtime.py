@@ -94,6 +94,15 @@ class Engine:
         gs.gs_round(self.handle, slots.data_ptr(), slots.shape[0], K, gs.GS_ACCEPT_GREEDY, force,
                     out_tok.data_ptr(), out_cnt.data_ptr(), out_done.data_ptr(), dbg)
 
+    def round_profile(self, slots: torch.Tensor, K: int, out_tok: torch.Tensor,
+                      out_cnt: torch.Tensor, out_done: torch.Tensor,
+                      force: Optional[gs.gs_force] = None) -> list:
+        """One round enqueued eagerly with an event after every kernel:
+        [(kind name, device ms)] per launch (see gs_round_profile)."""
+        prof = gs.gs_round_profile(self.handle, slots.data_ptr(), slots.shape[0], K, force,
+                                   out_tok.data_ptr(), out_cnt.data_ptr(), out_done.data_ptr())
+        return [(gs.KIND_NAMES[k], ms) for k, ms in prof]
+
     def restore(self, slot: int, seq_len: int, x0: int, n_out: int, max_new: int, done: int = 0,
                 rounds: int = 0) -> None:
         gs.gs_seq_restore(self.handle, slot, seq_len, x0, n_out, max_new, done, rounds)

@@ -200,3 +200,44 @@ def test_bad_requests_raise(tiny):
     assert e.value.code == gs.GS_ERR_DEVICE_CHECK
     eng.check()                                            # cleared
     eng.close()
+
+
+def test_round_profile_matches_round(tiny_gain):
+    """gs_round_profile runs the same round as gs_round (same committed tokens
+    and state) and reports one timed entry per kernel launch, in launch order:
+    window, embed, per layer QKV / attention / O / gate-up / down, LM head, for
+    the draft and the verify forward, then accept."""
+    cfg, w, _ = tiny_gain
+    eng = new_engine(cfg, w, max_ctx=1024, max_K=16, max_prefill=256)
+    prompt = synth.make_prompt(cfg, 120, 30, index=3)
+    dev = eng.device
+    slots = torch.tensor([0], dtype=torch.int32, device=dev)
+    K = 6
+    bufs = [torch.zeros((1, K + 2), dtype=torch.int32, device=dev),
+            torch.zeros(1, dtype=torch.int32, device=dev),
+            torch.zeros(1, dtype=torch.int32, device=dev)]
+    eng.prefill(0, prompt.vis, prompt.text, 100)
+    ref = []
+    for _ in range(3):
+        eng.round(slots, K, *bufs)
+        eng.stream.synchronize()
+        ref.append(bufs[0].cpu().numpy()[0, :int(bufs[1].cpu()[0])].tolist())
+    ref_state = eng.state(0)
+    eng.prefill(0, prompt.vis, prompt.text, 100)
+    got = []
+    for _ in range(3):
+        prof = eng.round_profile(slots, K, *bufs)
+        got.append(bufs[0].cpu().numpy()[0, :int(bufs[1].cpu()[0])].tolist())
+    assert got == ref
+    assert eng.state(0) == ref_state
+    fwd = ["embed"] + ["qkv", "attention", "o_proj", "gate_up", "down"] * cfg.n_layers + ["lm_head"]
+    assert [k for k, _ in prof] == ["window"] + fwd + ["window"] + fwd + ["accept"]
+    assert len(prof) == gs_launches(eng)
+    assert all(ms > 0 for _, ms in prof)
+    eng.check()
+    eng.close()
+
+
+def gs_launches(eng):
+    from paper_2609_26638_gb300 import gs
+    return gs.gs_round_launches(eng.handle)
