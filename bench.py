@@ -115,11 +115,11 @@ class ClockSampler:
 def kernel_bytes(cfg, kind: str, T: int, ctx: list) -> int | None:
     """Algorithmic HBM bytes of one launch of `kind` over T window rows.
 
-    Each operand counted once at its storage width: bf16 weights, bf16
+    Each operand counted once at its storage width: fp16 weight copies, fp16
     activations, float32 residual stream (read and written), float32 per-128
     feature sums of squares (the folded RMSNorm), 8-byte argmax keys.  For
     attention, ctx[i] is sequence i's visible keys (cached prefix + window):
-    K and V rows of every KV head, plus the bf16 queries read and outputs
+    K and V rows of every KV head, plus the fp16 queries read and outputs
     written.  None for the small window / accept kernels (no bandwidth model).
     """
     d, F, V = cfg.d_model, cfg.d_ffn, cfg.vocab
@@ -336,8 +336,8 @@ def lm_head_roofline(eng, cfg, K, dev):
     hbm, _, src = load_peaks()
     M, N, Kd = K + 1, cfg.vocab, cfg.d_model
     g = torch.Generator(device=dev).manual_seed(0)
-    ws = [(0.02 * torch.randn(N, Kd, device=dev, generator=g)).bfloat16() for _ in range(3)]
-    x = torch.randn(M, Kd, device=dev, generator=g).bfloat16()
+    ws = [(0.02 * torch.randn(N, Kd, device=dev, generator=g)).half() for _ in range(3)]
+    x = torch.randn(M, Kd, device=dev, generator=g).half()
     keys = torch.zeros(M, dtype=torch.int64, device=dev)
     sb = gs.gs_linear_scratch_bytes(M, N, 1)
     scratch = torch.zeros(sb, dtype=torch.uint8, device=dev)
@@ -380,12 +380,12 @@ def attention_roofline(cfg, dev):
     for b in range(B):
         pt[b, :pages_per[b]] = perm[o:o + pages_per[b]]
         o += pages_per[b]
-    kv = torch.randn(n_pages * 2 * Hkv * 64 * 64, device=dev).bfloat16()
-    q = torch.randn(B * W * Hq * 64, device=dev).bfloat16()
+    kv = torch.randn(n_pages * 2 * Hkv * 64 * 64, device=dev).half()
+    q = torch.randn(B * W * Hq * 64, device=dev).half()
     out = torch.zeros_like(q)
     ptd = torch.from_numpy(pt).to(dev)
     nd = torch.from_numpy(ns).to(dev)
-    sp = max(1, math.ceil(pt_stride * B * Hkv / 304))
+    sp = min(32, max(2, math.ceil(pt_stride * B * Hkv / (152 * 16))))
     sb = gs.gs_attention_scratch_bytes(B, W, Hq, Hkv, pt_stride, sp)
     scratch = torch.zeros(sb, dtype=torch.uint8, device=dev)
     stream = torch.cuda.current_stream(dev)
@@ -505,7 +505,7 @@ def main():
     line = {"metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": max(world, 1),
             "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": round(1e3 * el / args.steps, 3), "higher_is_better": True,
-            "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "scaling": "weak", "vs_baseline": None, "dtype": "f16", "data": "synthetic",
             "config": config,
             "round_p50_ms": round(rms[len(rms) // 2], 4),
             "round_p90_ms": round(rms[int(len(rms) * 0.9)], 4),

@@ -18,7 +18,15 @@
  *    outputs) and the stream.  After gs_create the library allocates no
  *    device memory; it carves everything from the caller's workspace.
  *  - Work is enqueued asynchronously on the handle's stream unless stated.
- *  - bf16 tensors are IEEE bfloat16 bit patterns, row-major.
+ *  - bf16 tensors are bfloat16 bit patterns, fp16 tensors IEEE binary16
+ *    bit patterns; all row-major.
+ *  - Arithmetic: the model's weights arrive as bf16; gs_create re-encodes each
+ *    matrix as an fp16 copy scaled by a power of two (exact for every weight
+ *    whose magnitude is above 2^-31 of the tensor's largest).  Activations
+ *    between kernels and the KV cache are fp16 (11 significant bits, against
+ *    8 for bf16); every contraction accumulates in fp32; the residual stream
+ *    and the softmax statistics are fp32.  A kernel that would store a value
+ *    beyond the fp16 range raises the device error word (GS_ERR_DEVICE_CHECK).
  *  - Return value: GS_OK (0) or one of the GS_ERR_* codes below; the message
  *    of the last failure is available from gs_last_error().  Kernel-side
  *    checks (slot ids, token ids, bounded waits) raise a device error word
@@ -66,7 +74,7 @@ typedef struct {
   int max_K;           /* largest block size a round may use                              */
   int max_prefill;     /* tokens per prefill chunk (longer prefixes run in chunks)        */
   int kv_pages;        /* 64-token pages in the KV pool; 0 = max_batch * ceil(max_ctx/64) */
-  int split_pages;     /* attention pages per KV split (decode); 0 = automatic             */
+  int split_pages;     /* attention pages per work item (decode); 0 = automatic           */
 } gs_config;
 
 /* Weights: device pointers to bf16 arrays owned by the caller, row-major
@@ -111,16 +119,19 @@ typedef struct {
 
 typedef struct gs_handle gs_handle;
 
-/* Bytes of device workspace gs_create needs for this config (KV page pool,
- * page table, per-sequence state, activations, split scratch).  0 if the
- * config is invalid. */
+/* Bytes of device workspace gs_create needs for this config (fp16 weight
+ * copies, KV page pool, page table, per-sequence state, activations, split
+ * scratch).  0 if the config is invalid. */
 size_t gs_workspace_bytes(const gs_config *cfg);
 
 /* Build a handle.  cfg, w: host structs (copied).  workspace: device memory of
  * at least gs_workspace_bytes(cfg) bytes, 256-byte aligned, owned by the
  * caller and not touched by anyone else until gs_destroy.  stream: a
- * cudaStream_t (NULL = legacy default stream).  Zeroes the workspace and
- * builds the TMA descriptors; synchronises the stream before returning.
+ * cudaStream_t (NULL = legacy default stream).  Zeroes the workspace, writes
+ * the scaled fp16 copies of the weight matrices into it (the caller's bf16
+ * matrices are not read again; embed and the norm gains are read at every
+ * forward) and builds the TMA descriptors; synchronises the stream before
+ * returning.
  * Errors: GS_ERR_INVALID_ARG, GS_ERR_UNSUPPORTED (shape), GS_ERR_OOM
  * (workspace too small), GS_ERR_CUDA. */
 int gs_create(const gs_config *cfg, const gs_weights *w, void *workspace, size_t ws_bytes,
@@ -223,23 +234,26 @@ int gs_sync_check(gs_handle *h);
  * Sub-steps exposed for the attention-only sweep and kernel parity tests.
  * ------------------------------------------------------------------------ */
 
-/* Hybrid-mask attention over a paged bf16 KV cache (paper Appendix steps
+/* Hybrid-mask attention over a paged fp16 KV cache (paper Appendix steps
  * Draft forward / Verify forward; mask semantics Sec. 4.2).  Standalone form
  * of the kernel the rounds use.
  *   mode 0 DRAFT:  query row i of sequence s sits at slot n_s + i;
  *                  row 0 sees keys 0..n_s, rows i >= 1 see keys 0..n_s + W - 1
  *   mode 1 VERIFY: query row i sits at slot n_s + 1 + i and sees keys 0..n_s + 1 + i
- *   q        device bf16 [n_seq, W, n_heads, 64] (RoPE already applied)
- *   kv       device bf16 page pool [n_pages][2 (K,V)][n_kv_heads][64 tokens][64]
+ *   q        device fp16 [n_seq, W, n_heads, 64] (RoPE already applied)
+ *   kv       device fp16 page pool [n_pages][2 (K,V)][n_kv_heads][64 tokens][64]
  *   page_table device int32 [n_seq, pt_stride]: logical page -> physical page
  *   n        device int32 [n_seq]: n_s
- *   out      device bf16 [n_seq, W, n_heads, 64]
- *   scratch  device, >= gs_attention_scratch_bytes(...) bytes (key limits and
- *            the block -> page-table map; no split partials: the KV splits of a
- *            (sequence, head) form one thread-block cluster and merge through
- *            distributed shared memory)
- *   split_pages pages per KV split (>= 1); raised to ceil(pt_stride / 8) when
- *            a sequence would otherwise need more than 8 splits
+ *   out      device fp16 [n_seq, W, n_heads, 64]
+ *   scratch  device, >= gs_attention_scratch_bytes(...) bytes: key limits, the
+ *            block -> page-table map, merge tickets and the fp32 partial rows
+ *            (O, m, l) of every work item
+ *   split_pages pages per work item (>= 1): item i of a sequence covers its
+ *            logical pages [i * split_pages, (i + 1) * split_pages); items are
+ *            reduced independently and merged in item order, so results depend
+ *            on split_pages but not on n_seq, W or the other sequences.
+ *            GS_ERR_UNSUPPORTED if ceil(pt_stride / split_pages) items exceed
+ *            what the merge holds (12288 / (16 * ceil(W * G / 16))).
  *   stream   cudaStream_t */
 size_t gs_attention_scratch_bytes(int n_seq, int W, int n_heads, int n_kv_heads, int max_pages,
                                   int split_pages);
@@ -248,9 +262,9 @@ int gs_attention(int mode, const void *q, const void *kv, int n_pages, const int
                  void *out, void *scratch, size_t scratch_bytes, int split_pages, void *stream);
 
 /* Y = X . W^T on the tcgen05 GEMM the decoder uses.
- *   x device bf16 [M, K] (row stride K), w device bf16 [N, K], y device [M, N]
- *   epilogue 0: y bf16 = acc;  1: y fp32 += acc (residual);  2: SwiGLU: w is
- *   [2N, K] (gate rows then up rows), y bf16 [M, N] = silu(gate) * up;
+ *   x device fp16 [M, K] (row stride K), w device fp16 [N, K], y device [M, N]
+ *   epilogue 0: y fp16 = acc;  1: y fp32 += acc (residual);  2: SwiGLU: w is
+ *   [2N, K] (gate rows then up rows), y fp16 [M, N] = silu(gate) * up;
  *   3: argmax: y is uint64 [M] packed (ordered fp32 bits << 32 | ~index),
  *   combined with atomicMax (caller zeroes it first).
  *   split_k: 1 or a divisor of K/64; scratch device >= gs_linear_scratch_bytes.

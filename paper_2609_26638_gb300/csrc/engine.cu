@@ -2,6 +2,7 @@
 // decoder forward as a launch sequence, the round (draft -> force -> verify ->
 // accept) with a CUDA-graph cache, prefill, and the C ABI of include/gs.h.
 #include <algorithm>
+#include <cmath>
 #include <cstdio>
 #include <cstring>
 #include <map>
@@ -39,7 +40,7 @@ EncodeTiledFn get_encode() {
   return fn;
 }
 
-// 2-D bf16 tensor map over a row-major [rows, cols] array, box {64, box_rows},
+// 2-D fp16 tensor map over a row-major [rows, cols] array, box {64, box_rows},
 // 128-byte swizzle, zero fill out of bounds.
 bool make_map(CUtensorMap* m, const void* base, uint64_t rows, uint64_t cols, uint32_t box_rows) {
   EncodeTiledFn enc = get_encode();
@@ -48,7 +49,7 @@ bool make_map(CUtensorMap* m, const void* base, uint64_t rows, uint64_t cols, ui
   cuuint64_t strides[1] = {cols * 2};
   cuuint32_t box[2] = {64, box_rows};
   cuuint32_t es[2] = {1, 1};
-  CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides,
+  CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void*>(base), dims, strides,
                    box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                    CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;
@@ -72,41 +73,54 @@ struct Carver {
   }
 };
 
-constexpr size_t kGemmPartialFloats = 12u << 20;  // 48 MB of split-K partials
 constexpr int kGemmCounters = 1 << 16;
 
 struct GemmPlan {
   int bn, tok_tiles, feat_tiles, splits;
 };
 
-// Token tile from T; split-K (decode only) so that about one wave of CTAs runs.
-GemmPlan plan_gemm(int weight_rows, int K, int T, bool allow_split) {
+// Split-K factor of a weight matrix in decode rounds.  It depends on the
+// weight's shape only, never on the token count: every split sums its K range
+// from zero and the splits are added in order 0..S-1, and the MMA's per-column
+// arithmetic does not depend on the tile width, so a token row gets the same
+// bits in any window and any batch.  About one wave of CTAs for a one-tile
+// window, at least 4 splits (cluster split CTAs own at most 8 of 32 tokens),
+// at most one cluster; matrices with a wave of feature tiles are not split.
+int decode_splits(int weight_rows, int K) {
+  const int feat_tiles = weight_rows / 128;
+  const int nkb = K / 64;
+  if (feat_tiles >= 152) return 1;
+  const int want = std::min(std::max(cdiv(152, feat_tiles), 4), kMaxClusterSplits);
+  int s = 1;
+  for (int k = 1; k <= nkb; ++k)
+    if (nkb % k == 0 && k <= want) s = k;
+  return s;
+}
+
+GemmPlan plan_gemm(int weight_rows, int K, int T, bool decode) {
   GemmPlan p;
   p.bn = gemm_bn_for(T);
   p.tok_tiles = cdiv(T, p.bn);
   p.feat_tiles = weight_rows / 128;
-  p.splits = 1;
-  const int tiles = p.feat_tiles * p.tok_tiles;
-  const int nkb = K / 64;
-  if (allow_split && tiles < 152) {
-    // about one wave; cluster-reduced decode tiles (BN <= 64) also keep each
-    // split CTA at <= 8 tokens (BN / splits <= 8)
-    int want = cdiv(152, tiles);
-    if (p.bn <= 64) want = std::max(want, p.bn / 8);
-    want = std::min(want, kMaxClusterSplits);
-    for (int s = 1; s <= nkb; ++s)
-      if (nkb % s == 0 && s <= want) p.splits = s;
-    // wider tiles reduce through global scratch: stay within it
-    while (p.bn > 64 && p.splits > 1 &&
-           static_cast<size_t>(p.splits) * tiles * p.bn * 128 > kGemmPartialFloats) {
-      int s = p.splits - 1;
-      while (s > 1 && nkb % s) --s;
-      p.splits = s;
-    }
-  }
+  p.splits = decode ? decode_splits(weight_rows, K) : 1;
   return p;
 }
 
+// fp32 partials the widest decode tiles (BN > 64, reduced through global
+// scratch) need: splits x feature tiles x token columns (T + 255 bounds the
+// padded token count) x 128, over the decoder's five weight shapes.
+size_t gemm_partial_floats(const gs_config& c, int qkv_dim, int T_dec) {
+  const int HD = c.n_heads * 64;
+  const int shapes[5][2] = {{qkv_dim, c.d_model}, {c.d_model, HD}, {2 * c.d_ffn, c.d_model},
+                            {c.d_model, c.d_ffn}, {c.vocab, c.d_model}};
+  size_t need = 0;
+  for (const auto& sh : shapes) {
+    const int S = decode_splits(sh[0], sh[1]);
+    if (S > 1)
+      need = std::max(need, static_cast<size_t>(S) * (sh[0] / 128) * (T_dec + 255) * 128);
+  }
+  return need;
+}
 
 }  // namespace
 
@@ -116,31 +130,43 @@ struct gs_handle {
   std::string err;
 
   // weights
-  const __nv_bfloat16 *embed = nullptr, *lm_head = nullptr, *final_norm = nullptr;
-  std::vector<const __nv_bfloat16*> attn_norm, ffn_norm, w_qkv, w_o, w_gu, w_down;
+  const __nv_bfloat16 *embed = nullptr, *final_norm = nullptr;
+  std::vector<const __nv_bfloat16*> attn_norm, ffn_norm;
+  // fp16 copies of the matrices, each scaled by 2^s (w_scale = 2^-s undoes it)
+  std::vector<const __half*> w_qkv, w_o, w_gu, w_down;
+  const __half* lm_head = nullptr;
+  std::vector<float> sc_qkv, sc_o, sc_gu, sc_down;
+  float sc_lm = 1.f;
+  __half* wcopy = nullptr;
   std::vector<CUtensorMap> tm_qkv, tm_o, tm_gu, tm_down;
   CUtensorMap tm_lm;
   CUtensorMap tm_hb[4], tm_ao[4], tm_act[4];
   CUtensorMap tm_kv;
 
   // sizes
-  int qkv_dim = 0, G = 1, T_max = 0, pt_stride = 0, n_pages = 0, split_pages = 1;
-  int max_splits_dec = 1, r_max_dec = 16, W_max = 1;
+  int qkv_dim = 0, G = 1, T_max = 0, pt_stride = 0, n_pages = 0, W_max = 1;
+  // attention work items: pages per item and item slots, decode and prefill
+  int split_pages = 1, items_dec = 1, r_max_dec = 16;
+  int split_pages_pf = 8, items_pf = 1, qb_pf = 64;
+  float* attn_part = nullptr;
+  size_t attn_part_floats = 0;
+  int* attn_ticket = nullptr;
 
   // workspace
   int* err_word = nullptr;
   SeqStateDev st{};
   int32_t* page_table = nullptr;
-  __nv_bfloat16* kv = nullptr;
+  __half* kv = nullptr;
   float2* rope = nullptr;
   int32_t *tok = nullptr, *pos = nullptr, *lim = nullptr, *tok_slot = nullptr;
   int32_t *blk_slot = nullptr, *blk_active = nullptr;
   float* hbuf = nullptr;
-  __nv_bfloat16 *hb = nullptr, *qr = nullptr, *ao = nullptr, *act = nullptr;
+  __half *hb = nullptr, *qr = nullptr, *ao = nullptr, *act = nullptr;
   float* ssp = nullptr;   // per-token sums of h^2 per 128-feature block [T_max][d/128]
   unsigned long long *packed_d = nullptr, *packed_v = nullptr;
   int32_t *draft_tok = nullptr, *verify_in = nullptr, *verify_tok = nullptr;
   float* gemm_partial = nullptr;
+  size_t partial_floats = 0;
   int* gemm_counters = nullptr;
 
   // host page bookkeeping
@@ -232,12 +258,26 @@ size_t carve(gs_handle* h, const gs_config& c, void* base) {
   const int W_max = c.max_K + 1;
   int T_max = std::max(c.max_batch * W_max, c.max_prefill);
   T_max = static_cast<int>(align_up(std::max(T_max, 256), 256));
-  // attention splits: fixed page ranges, at most kAttnMaxSplits per sequence (one cluster)
-  int sp = c.split_pages;
-  if (sp <= 0) sp = std::max(1, cdiv(static_cast<long long>(pt_stride) * c.max_batch * c.n_kv_heads, 304));
-  sp = std::max(sp, attn_min_split_pages(pt_stride));
-  const int max_splits = cdiv(pt_stride, sp);
+  // attention work items (fixed absolute page ranges).  Decode: about 16
+  // items per SM over a full batch at full context, at least 2 pages each;
+  // prefill: 8 pages or more.  Either way the last item's merge keeps one
+  // coefficient per (item, row) in shared memory.
   const int r_max = round16(W_max * G);
+  const int qb_pf = std::max(1, 128 / G);
+  const int r_pf = round16(qb_pf * G);
+  int sp = c.split_pages;
+  if (sp <= 0)
+    sp = std::min(32, std::max(2, cdiv(static_cast<long long>(pt_stride) * c.max_batch * c.n_kv_heads,
+                                       152 * 16)));
+  sp = std::max(sp, cdiv(pt_stride, attn_max_merge_items(r_max)));
+  const int items_dec = cdiv(pt_stride, sp);
+  const int sp_pf = std::max(8, cdiv(pt_stride, attn_max_merge_items(r_pf)));
+  const int items_pf = cdiv(pt_stride, sp_pf);
+  const int chunk = std::min(c.max_prefill, T_max);
+  const int blocks_pf = cdiv(chunk, qb_pf);
+  const size_t attn_part_floats =
+      std::max(static_cast<size_t>(c.max_batch) * c.n_kv_heads * items_dec * r_max,
+               static_cast<size_t>(blocks_pf) * c.n_kv_heads * items_pf * r_pf) * kAttnRow;
 
   int* err_word = cv.take<int>(64);
   SeqStateDev st;
@@ -248,8 +288,8 @@ size_t carve(gs_handle* h, const gs_config& c, void* base) {
   st.done = cv.take<int32_t>(c.max_batch);
   st.rounds = cv.take<int32_t>(c.max_batch);
   int32_t* page_table = cv.take<int32_t>(static_cast<size_t>(c.max_batch) * pt_stride);
-  __nv_bfloat16* kv = cv.take<__nv_bfloat16>(static_cast<size_t>(c.n_layers) * n_pages * 2 *
-                                             c.n_kv_heads * 64 * 64);
+  __half* kv = cv.take<__half>(static_cast<size_t>(c.n_layers) * n_pages * 2 * c.n_kv_heads * 64 *
+                               64);
   float2* rope = cv.take<float2>(static_cast<size_t>(c.max_ctx) * 32);
   int32_t* tok = cv.take<int32_t>(T_max);
   int32_t* pos = cv.take<int32_t>(T_max);
@@ -258,18 +298,28 @@ size_t carve(gs_handle* h, const gs_config& c, void* base) {
   int32_t* blk_slot = cv.take<int32_t>(std::max(c.max_batch, T_max / 64 + 1));
   int32_t* blk_active = cv.take<int32_t>(std::max(c.max_batch, T_max / 64 + 1));
   float* hbuf = cv.take<float>(static_cast<size_t>(T_max) * c.d_model);
-  __nv_bfloat16* hb = cv.take<__nv_bfloat16>(static_cast<size_t>(T_max) * c.d_model);
+  __half* hb = cv.take<__half>(static_cast<size_t>(T_max) * c.d_model);
   float* ssp = cv.take<float>(static_cast<size_t>(T_max) * (c.d_model / 128));
-  __nv_bfloat16* qr = cv.take<__nv_bfloat16>(static_cast<size_t>(T_max) * c.n_heads * 64);
-  __nv_bfloat16* ao = cv.take<__nv_bfloat16>(static_cast<size_t>(T_max) * c.n_heads * 64);
-  __nv_bfloat16* act = cv.take<__nv_bfloat16>(static_cast<size_t>(T_max) * c.d_ffn);
+  __half* qr = cv.take<__half>(static_cast<size_t>(T_max) * c.n_heads * 64);
+  __half* ao = cv.take<__half>(static_cast<size_t>(T_max) * c.n_heads * 64);
+  __half* act = cv.take<__half>(static_cast<size_t>(T_max) * c.d_ffn);
   unsigned long long* packed_d = cv.take<unsigned long long>(T_max);
   unsigned long long* packed_v = cv.take<unsigned long long>(T_max);
   int32_t* draft_tok = cv.take<int32_t>(static_cast<size_t>(c.max_batch) * W_max);
   int32_t* verify_in = cv.take<int32_t>(static_cast<size_t>(c.max_batch) * W_max);
   int32_t* verify_tok = cv.take<int32_t>(static_cast<size_t>(c.max_batch) * W_max);
-  float* gemm_partial = cv.take<float>(kGemmPartialFloats);
+  const size_t partial_floats = gemm_partial_floats(c, qkv_dim, c.max_batch * W_max);
+  float* gemm_partial = cv.take<float>(partial_floats);
   int* gemm_counters = cv.take<int>(kGemmCounters);
+  float* attn_part = cv.take<float>(attn_part_floats);
+  int* attn_ticket = cv.take<int>(static_cast<size_t>(std::max(c.max_batch, blocks_pf)) * c.n_kv_heads);
+  // fp16 weight copies: per layer qkv | o | gate_up | down, then the LM head
+  const size_t per_layer = static_cast<size_t>(qkv_dim) * c.d_model +
+                           static_cast<size_t>(c.d_model) * c.n_heads * 64 +
+                           2 * static_cast<size_t>(c.d_ffn) * c.d_model +
+                           static_cast<size_t>(c.d_model) * c.d_ffn;
+  // (every tensor's element count is a multiple of 64 * 64, so the copies pack without padding)
+  __half* wcopy = cv.take<__half>(per_layer * c.n_layers + static_cast<size_t>(c.vocab) * c.d_model);
 
   if (h) {
     h->G = G;
@@ -279,9 +329,17 @@ size_t carve(gs_handle* h, const gs_config& c, void* base) {
     h->T_max = T_max;
     h->W_max = W_max;
     h->split_pages = sp;
-    h->max_splits_dec = max_splits;
+    h->items_dec = items_dec;
     h->r_max_dec = r_max;
+    h->split_pages_pf = sp_pf;
+    h->items_pf = items_pf;
+    h->qb_pf = qb_pf;
+    h->attn_part = attn_part;
+    h->attn_part_floats = attn_part_floats;
+    h->attn_ticket = attn_ticket;
     h->err_word = err_word;
+    h->wcopy = wcopy;
+    h->partial_floats = partial_floats;
     h->st = st;
     h->page_table = page_table;
     h->kv = kv;
@@ -320,6 +378,7 @@ GemmArgs gemm_base(gs_handle* h) {
   a.n_ssp = h->cfg.d_model / 128;
   a.inv_d = 1.0f / static_cast<float>(h->cfg.d_model);
   a.eps = h->cfg.rms_eps;
+  a.w_scale = 1.f;
   return a;
 }
 
@@ -330,9 +389,9 @@ int run_gemm(gs_handle* h, const CUtensorMap& tw, int weight_rows, const CUtenso
   a.K = K;
   a.splits = p.splits;
   a.kb_per_split = (K / 64) / p.splits;
-  a.cluster = (p.splits > 1 && p.bn <= 64) ? 1 : 0;
+  a.cluster = gemm_cluster_ok(p.bn, p.splits) ? 1 : 0;
   if (p.splits > 1 && !a.cluster &&
-      (static_cast<size_t>(p.splits) * p.feat_tiles * p.tok_tiles * p.bn * 128 > kGemmPartialFloats ||
+      (static_cast<size_t>(p.splits) * p.feat_tiles * p.tok_tiles * p.bn * 128 > h->partial_floats ||
        p.feat_tiles * p.tok_tiles > kGemmCounters))
     return fail(h, GS_ERR_OOM, "split-K scratch too small");
   GS_CUDA(h, launch_gemm(p.bn, epi, tw, tx_set[bn_index(p.bn)], a, p.feat_tiles, p.tok_tiles,
@@ -342,7 +401,7 @@ int run_gemm(gs_handle* h, const CUtensorMap& tw, int weight_rows, const CUtenso
 }
 
 struct AttnLaunch {
-  int n_blocks, QB, max_splits, split_pages, r_max;
+  int n_blocks, QB, split_pages, max_items, r_max;
   const int32_t* blk_slot;
   const int32_t* blk_active;
   int fixed_slot;
@@ -367,11 +426,19 @@ int run_attention(gs_handle* h, int layer, int T, const AttnLaunch& L) {
   a.rows_per_page = 2 * c.n_kv_heads * 64;
   a.kv_row_base = static_cast<long long>(layer) * h->n_pages * a.rows_per_page;
   a.split_pages = L.split_pages;
+  a.max_items = L.max_items;
+  a.r_pad = L.r_max;
+  a.part = h->attn_part;
+  a.ticket = h->attn_ticket;
   a.err = h->err_word;
-  dim3 grid(L.max_splits, c.n_kv_heads, L.n_blocks);
-  GS_CUDA(h, launch_ex(attn_paged_kernel, grid, dim3(attn_threads(L.r_max)),
-                       attn_smem_bytes(L.r_max), h->stream, true, dim3(L.max_splits, 1, 1), h->tm_kv,
-                       a));
+  if (static_cast<size_t>(L.n_blocks) * c.n_kv_heads * L.max_items * L.r_max * kAttnRow >
+          h->attn_part_floats ||
+      L.max_items > attn_max_merge_items(L.r_max))
+    return fail(h, GS_ERR_OOM, "attention item scratch too small");
+  const int ng = attn_groups_for(L.r_max, L.max_items * c.n_kv_heads * L.n_blocks);
+  dim3 grid(cdiv(L.max_items, ng), c.n_kv_heads, L.n_blocks);
+  GS_CUDA(h, launch_ex(attn_paged_kernel, grid, dim3(attn_threads(L.r_max, ng)),
+                       attn_smem_bytes(L.r_max, ng), h->stream, true, dim3(1, 1, 1), h->tm_kv, a));
   note_launch(h, GS_KIND_ATTENTION);
   return GS_OK;
 }
@@ -395,6 +462,7 @@ int forward(gs_handle* h, int T, const int32_t* tok, const __nv_bfloat16* vis, i
   int rc;
   for (int l = 0; l < L; ++l) {
     GemmArgs q = gemm_base(h);
+    q.w_scale = h->sc_qkv[l];
     q.N = h->qkv_dim;
     q.ssp_in = h->ssp;
     q.q_out = h->qr;
@@ -413,6 +481,7 @@ int forward(gs_handle* h, int T, const int32_t* tok, const __nv_bfloat16* vis, i
       return rc;
     if ((rc = run_attention(h, l, T, AL))) return rc;
     GemmArgs o = gemm_base(h);
+    o.w_scale = h->sc_o[l];
     o.N = d;
     o.y = h->hbuf;
     o.ldy = d;
@@ -423,6 +492,7 @@ int forward(gs_handle* h, int T, const int32_t* tok, const __nv_bfloat16* vis, i
                        GS_KIND_O_PROJ)))
       return rc;
     GemmArgs gu = gemm_base(h);
+    gu.w_scale = h->sc_gu[l];
     gu.N = F;
     gu.y = h->act;
     gu.ldy = F;
@@ -431,6 +501,7 @@ int forward(gs_handle* h, int T, const int32_t* tok, const __nv_bfloat16* vis, i
                        GS_KIND_GATE_UP)))
       return rc;
     GemmArgs dn = gemm_base(h);
+    dn.w_scale = h->sc_down[l];
     dn.N = d;
     dn.y = h->hbuf;
     dn.ldy = d;
@@ -443,6 +514,7 @@ int forward(gs_handle* h, int T, const int32_t* tok, const __nv_bfloat16* vis, i
   }
   if (n_lm == 0) return GS_OK;
   GemmArgs lm = gemm_base(h);
+  lm.w_scale = h->sc_lm;
   lm.N = c.vocab;
   lm.y = packed;
   lm.logits = logits;
@@ -485,8 +557,8 @@ int enqueue_round(gs_handle* h, const int32_t* slots, int n_seq, int K, const gs
   AttnLaunch AL;
   AL.n_blocks = n_seq;
   AL.QB = W;
-  AL.max_splits = h->max_splits_dec;
   AL.split_pages = h->split_pages;
+  AL.max_items = h->items_dec;
   AL.r_max = round16(W * h->G);
   AL.blk_slot = h->blk_slot;
   AL.blk_active = h->blk_active;
@@ -563,7 +635,7 @@ int gs_create(const gs_config* cfg, const gs_weights* w, void* workspace, size_t
     cudaError_t e = gemm_init_attributes();
     if (e == cudaSuccess)
       e = cudaFuncSetAttribute(attn_paged_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                               attn_smem_bytes(256));
+                               attn_max_smem_bytes());
 
     if (e != cudaSuccess)
       return fail(nullptr, GS_ERR_CUDA, std::string("kernel attributes: ") + cudaGetErrorString(e));
@@ -575,43 +647,23 @@ int gs_create(const gs_config* cfg, const gs_weights* w, void* workspace, size_t
   h->stream = static_cast<cudaStream_t>(stream);
   carve(h, *cfg, workspace);
   const gs_config& c = h->cfg;
-  const int L = c.n_layers, d = c.d_model, F = c.d_ffn;
+  const int L = c.n_layers, d = c.d_model, F = c.d_ffn, HD = c.n_heads * 64;
   auto chk = [&](const void* p) { return p && (reinterpret_cast<uintptr_t>(p) & 15) == 0; };
-  h->embed = static_cast<const __nv_bfloat16*>(w->embed);
-  h->lm_head = static_cast<const __nv_bfloat16*>(w->lm_head);
-  h->final_norm = static_cast<const __nv_bfloat16*>(w->final_norm);
   bool ok = chk(w->embed) && chk(w->lm_head) && chk(w->final_norm);
-  h->tm_qkv.resize(L);
-  h->tm_o.resize(L);
-  h->tm_gu.resize(L);
-  h->tm_down.resize(L);
-  for (int l = 0; l < L && ok; ++l) {
-    h->attn_norm.push_back(static_cast<const __nv_bfloat16*>(w->attn_norm[l]));
-    h->ffn_norm.push_back(static_cast<const __nv_bfloat16*>(w->ffn_norm[l]));
-    h->w_qkv.push_back(static_cast<const __nv_bfloat16*>(w->w_qkv[l]));
-    h->w_o.push_back(static_cast<const __nv_bfloat16*>(w->w_o[l]));
-    h->w_gu.push_back(static_cast<const __nv_bfloat16*>(w->w_gate_up[l]));
-    h->w_down.push_back(static_cast<const __nv_bfloat16*>(w->w_down[l]));
+  for (int l = 0; l < L && ok; ++l)
     ok = chk(w->attn_norm[l]) && chk(w->ffn_norm[l]) && chk(w->w_qkv[l]) && chk(w->w_o[l]) &&
          chk(w->w_gate_up[l]) && chk(w->w_down[l]);
-    ok = ok && make_map(&h->tm_qkv[l], w->w_qkv[l], h->qkv_dim, d, 128) &&
-         make_map(&h->tm_o[l], w->w_o[l], d, c.n_heads * 64, 128) &&
-         make_map(&h->tm_gu[l], w->w_gate_up[l], 2 * F, d, 64) &&
-         make_map(&h->tm_down[l], w->w_down[l], d, F, 128);
-  }
-  ok = ok && make_map(&h->tm_lm, w->lm_head, c.vocab, d, 128);
-  const int bns[4] = {32, 64, 128, 256};
-  for (int i = 0; i < 4 && ok; ++i) {
-    ok = make_map(&h->tm_hb[i], h->hb, h->T_max, d, bns[i]) &&
-         make_map(&h->tm_ao[i], h->ao, h->T_max, c.n_heads * 64, bns[i]) &&
-         make_map(&h->tm_act[i], h->act, h->T_max, F, bns[i]);
-  }
-  const uint64_t kv_rows = static_cast<uint64_t>(L) * h->n_pages * 2 * c.n_kv_heads * 64;
-  ok = ok && kv_rows < (1ull << 31) && make_map(&h->tm_kv, h->kv, kv_rows, 64, 64);
   if (!ok) {
     delete h;
-    return fail(nullptr, GS_ERR_INVALID_ARG, "misaligned weight pointer or tensor-map encode failed");
+    return fail(nullptr, GS_ERR_INVALID_ARG, "null or misaligned weight pointer");
   }
+  h->embed = static_cast<const __nv_bfloat16*>(w->embed);
+  h->final_norm = static_cast<const __nv_bfloat16*>(w->final_norm);
+  for (int l = 0; l < L; ++l) {
+    h->attn_norm.push_back(static_cast<const __nv_bfloat16*>(w->attn_norm[l]));
+    h->ffn_norm.push_back(static_cast<const __nv_bfloat16*>(w->ffn_norm[l]));
+  }
+
   // zero the workspace, page table -> -1, rope table
   cudaError_t e = cudaMemsetAsync(workspace, 0, need, h->stream);
   h->pt_host.assign(static_cast<size_t>(c.max_batch) * h->pt_stride, -1);
@@ -629,9 +681,87 @@ int gs_create(const gs_config* cfg, const gs_weights* w, void* workspace, size_t
     e = cudaMemcpyAsync(h->st.done, ones.data(), ones.size() * 4, cudaMemcpyHostToDevice, h->stream);
     if (e == cudaSuccess) e = cudaStreamSynchronize(h->stream);
   }
+
+  // fp16 weight copies.  Per tensor: the largest |w| (into the zeroed split-K
+  // counters), then w * 2^s with 2^s putting that maximum just below 2^15.
+  struct Src { const void* p; size_t n; };
+  std::vector<Src> src;
+  for (int l = 0; l < L; ++l) {
+    src.push_back({w->w_qkv[l], static_cast<size_t>(h->qkv_dim) * d});
+    src.push_back({w->w_o[l], static_cast<size_t>(d) * HD});
+    src.push_back({w->w_gate_up[l], 2 * static_cast<size_t>(F) * d});
+    src.push_back({w->w_down[l], static_cast<size_t>(d) * F});
+  }
+  src.push_back({w->lm_head, static_cast<size_t>(c.vocab) * d});
+  unsigned int* amax = reinterpret_cast<unsigned int*>(h->gemm_counters);
+  for (size_t t = 0; t < src.size() && e == cudaSuccess; ++t) {
+    absmax_bf16_kernel<<<304, 256, 0, h->stream>>>(static_cast<const __nv_bfloat16*>(src[t].p),
+                                                    src[t].n, amax + t);
+    e = cudaGetLastError();
+  }
+  std::vector<unsigned int> amax_host(src.size(), 0);
+  if (e == cudaSuccess)
+    e = cudaMemcpyAsync(amax_host.data(), amax, src.size() * 4, cudaMemcpyDeviceToHost, h->stream);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(h->stream);
+  std::vector<float> scales(src.size(), 1.f);
+  __half* dst = h->wcopy;
+  std::vector<const __half*> copies(src.size());
+  for (size_t t = 0; t < src.size() && e == cudaSuccess; ++t) {
+    float m;
+    std::memcpy(&m, &amax_host[t], 4);
+    int s_exp = 0;
+    if (m > 0.f && std::isfinite(m)) {
+      int ex = 0;
+      std::frexp(m, &ex);                // m = f * 2^ex, f in [0.5, 1)
+      s_exp = std::min(100, std::max(-100, 15 - ex));
+    }
+    scales[t] = std::ldexp(1.f, -s_exp);
+    scale_to_f16_kernel<<<304, 256, 0, h->stream>>>(static_cast<const __nv_bfloat16*>(src[t].p),
+                                                     src[t].n, std::ldexp(1.f, s_exp), dst);
+    e = cudaGetLastError();
+    copies[t] = dst;
+    dst += src[t].n;
+  }
+  if (e == cudaSuccess) e = cudaMemsetAsync(amax, 0, src.size() * 4, h->stream);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(h->stream);
   if (e != cudaSuccess) {
     delete h;
     return fail(nullptr, GS_ERR_CUDA, std::string("workspace init: ") + cudaGetErrorString(e));
+  }
+  for (int l = 0; l < L; ++l) {
+    h->w_qkv.push_back(copies[4 * l + 0]);
+    h->w_o.push_back(copies[4 * l + 1]);
+    h->w_gu.push_back(copies[4 * l + 2]);
+    h->w_down.push_back(copies[4 * l + 3]);
+    h->sc_qkv.push_back(scales[4 * l + 0]);
+    h->sc_o.push_back(scales[4 * l + 1]);
+    h->sc_gu.push_back(scales[4 * l + 2]);
+    h->sc_down.push_back(scales[4 * l + 3]);
+  }
+  h->lm_head = copies[4 * L];
+  h->sc_lm = scales[4 * L];
+
+  h->tm_qkv.resize(L);
+  h->tm_o.resize(L);
+  h->tm_gu.resize(L);
+  h->tm_down.resize(L);
+  for (int l = 0; l < L && ok; ++l)
+    ok = make_map(&h->tm_qkv[l], h->w_qkv[l], h->qkv_dim, d, 128) &&
+         make_map(&h->tm_o[l], h->w_o[l], d, HD, 128) &&
+         make_map(&h->tm_gu[l], h->w_gu[l], 2 * F, d, 64) &&
+         make_map(&h->tm_down[l], h->w_down[l], d, F, 128);
+  ok = ok && make_map(&h->tm_lm, h->lm_head, c.vocab, d, 128);
+  const int bns[4] = {32, 64, 128, 256};
+  for (int i = 0; i < 4 && ok; ++i) {
+    ok = make_map(&h->tm_hb[i], h->hb, h->T_max, d, bns[i]) &&
+         make_map(&h->tm_ao[i], h->ao, h->T_max, HD, bns[i]) &&
+         make_map(&h->tm_act[i], h->act, h->T_max, F, bns[i]);
+  }
+  const uint64_t kv_rows = static_cast<uint64_t>(L) * h->n_pages * 2 * c.n_kv_heads * 64;
+  ok = ok && kv_rows < (1ull << 31) && make_map(&h->tm_kv, h->kv, kv_rows, 64, 64);
+  if (!ok) {
+    delete h;
+    return fail(nullptr, GS_ERR_INVALID_ARG, "tensor-map encode failed");
   }
   h->free_pages.reserve(h->n_pages);
   for (int p = h->n_pages - 1; p >= 0; --p) h->free_pages.push_back(p);
@@ -709,11 +839,11 @@ int gs_prefill(gs_handle* h, int slot, const void* vis_emb, int n_vis, const int
                                                                h->pos, h->lim, h->tok_slot);
     GS_CUDA(h, cudaGetLastError());
     AttnLaunch AL;
-    AL.QB = 64;
-    AL.n_blocks = cdiv(T, 64);
-    AL.max_splits = 1;
-    AL.split_pages = h->pt_stride;
-    AL.r_max = round16(64 * h->G);
+    AL.QB = h->qb_pf;
+    AL.n_blocks = cdiv(T, h->qb_pf);
+    AL.split_pages = h->split_pages_pf;
+    AL.max_items = h->items_pf;
+    AL.r_max = round16(h->qb_pf * h->G);
     AL.blk_slot = nullptr;
     AL.blk_active = nullptr;
     AL.fixed_slot = slot;
@@ -866,10 +996,14 @@ size_t gs_attention_scratch_bytes(int n_seq, int W, int n_heads, int n_kv_heads,
   if (n_seq < 1 || W < 1 || n_kv_heads < 1 || n_heads % n_kv_heads || max_pages < 1 ||
       split_pages < 1)
     return 0;
+  const int r_max = round16(W * (n_heads / n_kv_heads));
+  const int items = cdiv(max_pages, split_pages);
   Carver cv(nullptr);
   cv.take<int>(64);                                   // error word
   cv.take<int32_t>(static_cast<size_t>(n_seq) * W);  // key limits
   cv.take<int32_t>(n_seq);                            // block -> page-table row
+  cv.take<int>(static_cast<size_t>(n_seq) * n_kv_heads);  // merge tickets
+  cv.take<float>(static_cast<size_t>(n_seq) * n_kv_heads * items * r_max * kAttnRow);  // items
   return align_up(cv.off, 256);
 }
 
@@ -906,26 +1040,32 @@ int gs_attention(int mode, const void* q, const void* kv, int n_pages, const int
   static bool attr = false;
   if (!attr) {
     if (cudaFuncSetAttribute(attn_paged_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             attn_smem_bytes(256)) != cudaSuccess)
+                             attn_max_smem_bytes()) != cudaSuccess)
       return GS_ERR_CUDA;
     attr = true;
   }
   const int r_max = round16(W * G);
-  const int sp = std::max(split_pages, attn_min_split_pages(pt_stride));
-  const int ms = cdiv(pt_stride, sp);
+  const int items = cdiv(pt_stride, split_pages);
+  if (items > attn_max_merge_items(r_max)) return GS_ERR_UNSUPPORTED;
   Carver cv(scratch);
   int* err = cv.take<int>(64);
   int32_t* lim = cv.take<int32_t>(static_cast<size_t>(n_seq) * W);
   int32_t* blk_slot = cv.take<int32_t>(n_seq);
+  int* ticket = cv.take<int>(static_cast<size_t>(n_seq) * n_kv_heads);
+  float* part = cv.take<float>(static_cast<size_t>(n_seq) * n_kv_heads * items * r_max * kAttnRow);
   CUtensorMap tm;
   const uint64_t rows = static_cast<uint64_t>(n_pages) * 2 * n_kv_heads * 64;
   if (rows >= (1ull << 31) || !make_map(&tm, kv, rows, 64, 64)) return GS_ERR_INVALID_ARG;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
+  // the merge tickets start at zero (the kernel leaves them at zero)
+  if (cudaMemsetAsync(ticket, 0, static_cast<size_t>(n_seq) * n_kv_heads * sizeof(int), s) !=
+      cudaSuccess)
+    return GS_ERR_CUDA;
   attn_standalone_prep<<<cdiv(n_seq * W, 128), 128, 0, s>>>(mode, n, n_seq, W, lim, blk_slot);
   AttnArgs a;
-  a.q = static_cast<const __nv_bfloat16*>(q);
+  a.q = static_cast<const __half*>(q);
   a.lim = lim;
-  a.out = static_cast<__nv_bfloat16*>(out);
+  a.out = static_cast<__half*>(out);
   a.page_table = page_table;
   a.pt_stride = pt_stride;
   a.blk_slot = blk_slot;
@@ -938,11 +1078,16 @@ int gs_attention(int mode, const void* q, const void* kv, int n_pages, const int
   a.G = G;
   a.rows_per_page = 2 * n_kv_heads * 64;
   a.kv_row_base = 0;
-  a.split_pages = sp;
+  a.split_pages = split_pages;
+  a.max_items = items;
+  a.r_pad = r_max;
+  a.part = part;
+  a.ticket = ticket;
   a.err = err;
-  dim3 grid(ms, n_kv_heads, n_seq);
-  return launch_ex(attn_paged_kernel, grid, dim3(attn_threads(r_max)), attn_smem_bytes(r_max), s,
-                   false, dim3(ms, 1, 1), tm, a) == cudaSuccess
+  const int ng = attn_groups_for(r_max, items * n_kv_heads * n_seq);
+  dim3 grid(cdiv(items, ng), n_kv_heads, n_seq);
+  return launch_ex(attn_paged_kernel, grid, dim3(attn_threads(r_max, ng)),
+                   attn_smem_bytes(r_max, ng), s, false, dim3(1, 1, 1), tm, a) == cudaSuccess
              ? GS_OK
              : GS_ERR_CUDA;
 }
@@ -993,10 +1138,11 @@ int gs_linear(const void* x, const void* w, void* y, int M, int N, int K, int ep
   a.K = K;
   a.splits = split_k;
   a.kb_per_split = (K / 64) / split_k;
-  a.cluster = (split_k > 1 && split_k <= kMaxClusterSplits && bn <= 64) ? 1 : 0;
+  a.cluster = gemm_cluster_ok(bn, split_k) ? 1 : 0;
   a.y = y;
   a.ldy = N;
   a.logits = nullptr;
+  a.w_scale = 1.f;
   return launch_gemm(bn, epilogue, tw, tx, a, feat_tiles, tok_tiles,
                      static_cast<cudaStream_t>(stream)) == cudaSuccess
              ? GS_OK

@@ -17,7 +17,7 @@ template <int BN>
 static cudaError_t launch_bn(int epi, const CUtensorMap& tmW, const CUtensorMap& tmX,
                              const GemmArgs& a, int ft, int tt, cudaStream_t s, bool pdl) {
   switch (epi) {
-    case kEpiStoreBf16: return launch_one<BN, kEpiStoreBf16>(tmW, tmX, a, ft, tt, s, pdl);
+    case kEpiStoreF16: return launch_one<BN, kEpiStoreF16>(tmW, tmX, a, ft, tt, s, pdl);
     case kEpiResidF32: return launch_one<BN, kEpiResidF32>(tmW, tmX, a, ft, tt, s, pdl);
     case kEpiSwiGLU: return launch_one<BN, kEpiSwiGLU>(tmW, tmX, a, ft, tt, s, pdl);
     case kEpiArgmax: return launch_one<BN, kEpiArgmax>(tmW, tmX, a, ft, tt, s, pdl);
@@ -42,7 +42,7 @@ template <int BN>
 static cudaError_t set_attr_bn() {
   const int bytes = GemmShape<BN>::kSmemBytes;
   cudaError_t e;
-  if ((e = cudaFuncSetAttribute(gemm_tc_kernel<BN, kEpiStoreBf16>,
+  if ((e = cudaFuncSetAttribute(gemm_tc_kernel<BN, kEpiStoreF16>,
                                 cudaFuncAttributeMaxDynamicSharedMemorySize, bytes)) != cudaSuccess)
     return e;
   if ((e = cudaFuncSetAttribute(gemm_tc_kernel<BN, kEpiResidF32>,

@@ -3,7 +3,7 @@
 // Computes D[f, t] = sum_k W[f, k] X[t, k] with the weight rows on the MMA M
 // side (128 rows per CTA, "swap-AB") and the token rows on the MMA N side
 // (BN in {32, 64, 128, 256}), so a 17-token decode window and an 8192-token
-// prefill chunk use the same kernel.  Operands are K-major bf16 tiles staged by
+// prefill chunk use the same kernel.  Operands are K-major fp16 tiles staged by
 // TMA with 128-byte swizzle; one elected thread issues tcgen05.mma into a TMEM
 // fp32 accumulator of 128 lanes x BN columns; four warps read it back with
 // tcgen05.ld for the fused epilogue.
@@ -23,13 +23,18 @@
 // ticket, no spinning) sums them.  Both sum the splits in order 0..S-1 from a
 // zero start, so the result does not depend on the path or on arrival order.
 //
-// Epilogues: bf16 store, fp32 residual add, SwiGLU (gate and up rows of the
+// Weights arrive as fp16 copies scaled by a power of two 2^s per tensor (an
+// exact re-encoding of the model's bf16 values); the epilogue multiplies the
+// fp32 accumulator by w_scale = 2^-s, which is exact, so the result equals
+// the product with the unscaled weights.
+//
+// Epilogues: fp16 store, fp32 residual add, SwiGLU (gate and up rows of the
 // same features share a tile), LM-head argmax (packed 64-bit atomicMax, ties
 // to the lowest index) with an optional fp32 logit dump, and the QKV epilogue
 // (RoPE on q and k, q to its buffer, k and v into the paged KV cache).
 //
 // RMSNorm is folded into the GEMMs: a residual epilogue also writes
-// hb = bf16(h * g) with the gain g of the norm that comes next, and the sum of
+// hb = fp16(h * g) with the gain g of the norm that comes next, and the sum of
 // h^2 over its 128 features (one partial per feature tile, "ssp"); the GEMM
 // that consumes hb multiplies its accumulator by rsqrt(sum(ssp) / d + eps).
 // Since that factor is one scalar per token, this equals normalising first.
@@ -42,7 +47,7 @@ namespace gs {
 constexpr int kGemmMaxClusterSplits = 8;
 
 enum GemmEpilogue : int {
-  kEpiStoreBf16 = 0, kEpiResidF32 = 1, kEpiSwiGLU = 2, kEpiArgmax = 3, kEpiQKV = 4
+  kEpiStoreF16 = 0, kEpiResidF32 = 1, kEpiSwiGLU = 2, kEpiArgmax = 3, kEpiQKV = 4
 };
 
 struct GemmArgs {
@@ -52,24 +57,25 @@ struct GemmArgs {
   int splits;       // split-K factor (divides K / 64)
   int kb_per_split; // (K / 64) / splits
   int cluster;      // 1: split-K partials reduced inside a cluster of `splits` CTAs
-  void* y;          // output: bf16 [M, ldy] | fp32 [M, ldy] | uint64 [M] (argmax)
+  void* y;          // output: fp16 [M, ldy] | fp32 [M, ldy] | uint64 [M] (argmax)
   int ldy;
   float* partial;   // global split-K partials [splits][tiles][BN][128] fp32 (cluster == 0)
   int* counters;    // per output tile, zero between launches (cluster == 0)
   float* logits;    // argmax only: optional fp32 [M, N] dump
   int* err;
+  float w_scale;    // 2^-s of the weight copy (1 for unscaled weights)
   int x_row0;       // X (and ssp_in) row of token 0
   // folded RMSNorm on the input: scale = rsqrt(sum_p ssp_in[t][p] * inv_d + eps)
   const float* ssp_in;
   int n_ssp;        // d / 128 partials per token
   float inv_d, eps;
-  // residual epilogue extras: hb_out[t][f] = bf16(h[t][f] * g_next[f]); ssp_out[t][tile] = sum h^2
-  __nv_bfloat16* hb_out;
+  // residual epilogue extras: hb_out[t][f] = fp16(h[t][f] * g_next[f]); ssp_out[t][tile] = sum h^2
+  __half* hb_out;
   const __nv_bfloat16* g_next;
   float* ssp_out;
   // QKV epilogue
-  __nv_bfloat16* q_out;        // [M, Hq, 64]
-  __nv_bfloat16* kv_layer;     // this layer's page pool [pages][2][Hkv][64][64]
+  __half* q_out;               // [M, Hq, 64]
+  __half* kv_layer;            // this layer's page pool [pages][2][Hkv][64][64]
   const int32_t* pos;          // [M] absolute slot
   const int32_t* tok_slot;     // [M] page-table row, -1 = no KV write
   const int32_t* page_table;
@@ -79,8 +85,8 @@ struct GemmArgs {
 
 template <int BN>
 struct GemmShape {
-  static constexpr int kABytes = 128 * 128;        // 128 rows x 64 bf16
-  static constexpr int kBBytes = BN * 128;         // BN rows x 64 bf16
+  static constexpr int kABytes = 128 * 128;        // 128 rows x 64 fp16
+  static constexpr int kBBytes = BN * 128;         // BN rows x 64 fp16
   static constexpr int kStageBytes = kABytes + kBBytes;
   // two CTAs per SM up to BN = 128 (<= ~97 KB each), one at BN = 256
   static constexpr int kStages = BN <= 64 ? 4 : (BN <= 128 ? 3 : 4);
@@ -128,14 +134,17 @@ __device__ __forceinline__ void gemm_epilogue_chunk(const GemmArgs& a, float (&v
   jhi = min(jhi, a.M - t0);
   if (rs != nullptr) {
 #pragma unroll
-    for (int j = 0; j < EW; ++j) v[j] *= rs[j];
+    for (int j = 0; j < EW; ++j) v[j] *= rs[j] * a.w_scale;
+  } else {
+#pragma unroll
+    for (int j = 0; j < EW; ++j) v[j] *= a.w_scale;
   }
-  if constexpr (EPI == kEpiStoreBf16) {
-    __nv_bfloat16* y = static_cast<__nv_bfloat16*>(a.y);
+  if constexpr (EPI == kEpiStoreF16) {
+    __half* y = static_cast<__half*>(a.y);
     const int f = feat_tile * 128 + row;
 #pragma unroll
     for (int j = 0; j < EW; ++j)
-      if (j >= jlo && j < jhi) y[static_cast<size_t>(t0 + j) * a.ldy + f] = __float2bfloat16_rn(v[j]);
+      if (j >= jlo && j < jhi) y[static_cast<size_t>(t0 + j) * a.ldy + f] = to_f16(v[j], a.err);
   } else if constexpr (EPI == kEpiResidF32) {
     float* y = static_cast<float*>(a.y);
     const int f = feat_tile * 128 + row;
@@ -150,7 +159,7 @@ __device__ __forceinline__ void gemm_epilogue_chunk(const GemmArgs& a, float (&v
       if (j >= jlo && j < jhi) {
         const float hn = hv[j] + v[j];
         y[static_cast<size_t>(t0 + j) * a.ldy + f] = hn;
-        if (a.hb_out) a.hb_out[static_cast<size_t>(t0 + j) * a.ldy + f] = __float2bfloat16_rn(hn * g);
+        if (a.hb_out) a.hb_out[static_cast<size_t>(t0 + j) * a.ldy + f] = to_f16(hn * g, a.err);
         hsq = hn * hn;
       }
       v[j] = hsq;
@@ -208,14 +217,14 @@ __device__ __forceinline__ void gemm_epilogue_chunk(const GemmArgs& a, float (&v
 #pragma unroll
       for (int j = 0; j < EW; ++j)
         if (j >= jlo && j < jhi)
-          a.q_out[(static_cast<size_t>(t0 + j) * a.Hq + head) * 64 + d] = __float2bfloat16_rn(v[j]);
+          a.q_out[(static_cast<size_t>(t0 + j) * a.Hq + head) * 64 + d] = to_f16(v[j], a.err);
     } else {
       // kvdst[j]: offset of (page, K, head 0, row p & 63, dim 0); V is Hkv * 4096 further
       const long long off = (static_cast<long long>(isv_of(region)) * a.Hkv + head) * 4096 + d;
 #pragma unroll
       for (int j = 0; j < EW; ++j) {
         const long long base = tm.kvdst[j];
-        if (j >= jlo && j < jhi && base >= 0) a.kv_layer[base + off] = __float2bfloat16_rn(v[j]);
+        if (j >= jlo && j < jhi && base >= 0) a.kv_layer[base + off] = to_f16(v[j], a.err);
       }
     }
   } else if constexpr (EPI == kEpiSwiGLU) {
@@ -227,7 +236,7 @@ __device__ __forceinline__ void gemm_epilogue_chunk(const GemmArgs& a, float (&v
     }
     asm volatile("bar.sync 1, 128;" ::: "memory");
     if (warp < 2) {
-      __nv_bfloat16* y = static_cast<__nv_bfloat16*>(a.y);
+      __half* y = static_cast<__half*>(a.y);
       const int f = feat_tile * 64 + row;
 #pragma unroll
       for (int j = 0; j < EW; ++j)
@@ -235,7 +244,7 @@ __device__ __forceinline__ void gemm_epilogue_chunk(const GemmArgs& a, float (&v
           const float g = v[j];
           const float u = xbuf[j * 64 + row];
           const float s = g / (1.0f + __expf(-g));
-          y[static_cast<size_t>(t0 + j) * a.ldy + f] = __float2bfloat16_rn(s * u);
+          y[static_cast<size_t>(t0 + j) * a.ldy + f] = to_f16(s * u, a.err);
         }
     }
     asm volatile("bar.sync 1, 128;" ::: "memory");
@@ -410,7 +419,7 @@ __global__ void __launch_bounds__(128, 1)
     }
     if (warp == 1 && lane == 0) {
       // MMA issuer
-      constexpr uint32_t idesc = umma_idesc_bf16(128, BN);
+      constexpr uint32_t idesc = umma_idesc_f16(128, BN);
       for (int i = 0; i < nkb; ++i) {
         const int s = i % S::kStages;
         const uint32_t ph = (i / S::kStages) & 1;
@@ -420,7 +429,7 @@ __global__ void __launch_bounds__(128, 1)
         const uint64_t bd = umma_desc_sw128(smem_u32(smB + s * S::kBBytes));
 #pragma unroll
         for (int k = 0; k < 4; ++k)
-          umma_bf16(tmem, ad + 2 * k, bd + 2 * k, idesc, (i > 0 || k > 0) ? 1u : 0u);
+          umma_f16(tmem, ad + 2 * k, bd + 2 * k, idesc, (i > 0 || k > 0) ? 1u : 0u);
         umma_commit(smem_u32(&empty[s]));
       }
       umma_commit(smem_u32(accum));

@@ -48,6 +48,14 @@ inline int gemm_bn_for(int T) { return T <= 32 ? 32 : (T <= 64 ? 64 : (T <= 128 
 // cluster of the `splits` CTAs of a tile when splits <= kMaxClusterSplits,
 // else through global scratch by the last CTA to arrive (same order, same bits).
 constexpr int kMaxClusterSplits = 8;
+// The cluster reduction gives split CTA q the tokens [q*per, (q+1)*per) of a
+// BN-token tile, per = BN / splits, and its epilogue handles per <= 8 or a
+// per that divides 32 (a slice never straddles a 32-token chunk).
+inline bool gemm_cluster_ok(int bn, int splits) {
+  if (splits < 2 || splits > kMaxClusterSplits || bn > 64 || bn % splits) return false;
+  const int per = bn / splits;
+  return per <= 8 || 32 % per == 0;
+}
 cudaError_t launch_gemm(int bn, int epi, const CUtensorMap& tmW, const CUtensorMap& tmX,
                         const GemmArgs& args, int feat_tiles, int tok_tiles, cudaStream_t s,
                         bool pdl = false);

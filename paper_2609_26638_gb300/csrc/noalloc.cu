@@ -52,7 +52,7 @@ typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t,
                                   const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
                                   CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
 
-bool encode_bf16_rows(CUtensorMap* m, const void* base, uint64_t rows, uint64_t cols,
+bool encode_f16_rows(CUtensorMap* m, const void* base, uint64_t rows, uint64_t cols,
                       uint32_t box_rows) {
   static EncodeTiledFn fn = nullptr;
   if (!fn) {
@@ -68,7 +68,7 @@ bool encode_bf16_rows(CUtensorMap* m, const void* base, uint64_t rows, uint64_t 
   cuuint64_t strides[1] = {cols * 2};
   cuuint32_t box[2] = {64, box_rows};
   cuuint32_t es[2] = {1, 1};
-  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, es,
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void*>(base), dims, strides, box, es,
             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
@@ -108,9 +108,9 @@ extern "C" int gs_linear_noalloc(const void* x, const void* w, void* y, int M, i
   int rc = scratch_for_current_device(&base);
   if (rc != GS_OK) return rc;
   CUtensorMap tw, tx;
-  if (!encode_bf16_rows(&tw, w, w_rows, K, epilogue == kEpiSwiGLU ? 64 : 128))
+  if (!encode_f16_rows(&tw, w, w_rows, K, epilogue == kEpiSwiGLU ? 64 : 128))
     return GS_ERR_INVALID_ARG;
-  if (!encode_bf16_rows(&tx, x, M, K, bn)) return GS_ERR_INVALID_ARG;
+  if (!encode_f16_rows(&tx, x, M, K, bn)) return GS_ERR_INVALID_ARG;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   uint8_t* b = static_cast<uint8_t*>(base);
   // the split-K counters must start at zero; the array keeps the last call's contents
@@ -128,6 +128,7 @@ extern "C" int gs_linear_noalloc(const void* x, const void* w, void* y, int M, i
   a.y = y;
   a.ldy = N;
   a.logits = nullptr;
+  a.w_scale = 1.f;
   return launch_gemm(bn, epilogue, tw, tx, a, feat_tiles, tok_tiles, s) == cudaSuccess ? GS_OK
                                                                                         : GS_ERR_CUDA;
 }

@@ -3,13 +3,14 @@
 #pragma once
 #include <cuda.h>
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
 namespace gs {
 
 // Device error word codes (written with atomicExch, read by gs_sync_check).
-enum : int { kErrNone = 0, kErrBounds = 1, kErrTimeout = 2 };
+enum : int { kErrNone = 0, kErrBounds = 1, kErrTimeout = 2, kErrRange = 3 };
 
 // Bounded waits give up after this many nanoseconds of %globaltimer.
 constexpr uint64_t kWaitLimitNs = 2000000000ull;
@@ -135,15 +136,15 @@ __device__ __forceinline__ uint64_t umma_desc_sw128(uint32_t smem_addr) {
   return d;
 }
 
-// Instruction descriptor for kind::f16: D fp32, A and B bf16, both K-major,
-// N >> 3 at bits 17-22, M >> 4 at bits 24-28.
-__host__ __device__ constexpr uint32_t umma_idesc_bf16(int M, int N) {
-  return (1u << 4) | (1u << 7) | (1u << 10) | (static_cast<uint32_t>(N >> 3) << 17) |
-         (static_cast<uint32_t>(M >> 4) << 24);
+// Instruction descriptor for kind::f16: D fp32 (bit 4), A and B fp16 (format
+// 0 at bits 7-9 and 10-12), both K-major, N >> 3 at bits 17-22, M >> 4 at
+// bits 24-28.
+__host__ __device__ constexpr uint32_t umma_idesc_f16(int M, int N) {
+  return (1u << 4) | (static_cast<uint32_t>(N >> 3) << 17) | (static_cast<uint32_t>(M >> 4) << 24);
 }
 
-__device__ __forceinline__ void umma_bf16(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc,
-                                          uint32_t idesc, uint32_t accumulate) {
+__device__ __forceinline__ void umma_f16(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc,
+                                         uint32_t idesc, uint32_t accumulate) {
   asm volatile(
       "{\n\t.reg .pred p;\n\t"
       "setp.ne.b32 p, %4, 0;\n\t"
@@ -262,6 +263,15 @@ __device__ __forceinline__ const float* cluster_peer_ptr(const float* p, uint32_
   uint64_t g;
   asm volatile("mapa.u64 %0, %1, %2;" : "=l"(g) : "l"(reinterpret_cast<uint64_t>(p)), "r"(rank));
   return reinterpret_cast<const float*>(g);
+}
+
+// ---------------------------------------------------------------- fp16 stores
+// Activations and cached keys/values are stored as fp16.  A value whose
+// magnitude exceeds the fp16 range (or a NaN) sets kErrRange; the store then
+// holds the saturated infinity, so a range failure never passes silently.
+__device__ __forceinline__ __half to_f16(float x, int* err) {
+  if (!(fabsf(x) <= 65504.0f)) atomicExch(err, kErrRange);
+  return __float2half_rn(x);
 }
 
 // ---------------------------------------------------------------- misc

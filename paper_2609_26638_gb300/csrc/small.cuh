@@ -193,11 +193,11 @@ __global__ void prefill_window_kernel(int T, int p0, int slot, int32_t* pos, int
 
 // Row t of the residual stream: h[t] = E[tok[t]] (fp32), or the visual row for
 // t < n_vis.  Also writes what the first QKV GEMM consumes for its folded
-// RMSNorm -- hb[t] = bf16(h[t] * g0) and the per-128-feature sums of h^2 --
+// RMSNorm -- hb[t] = fp16(h[t] * g0) and the per-128-feature sums of h^2 --
 // and zeroes the LM-head argmax key of the row.  One CTA of 128 threads per
 // row, 8 features per thread; d % 128 == 0.
 __global__ void embed_kernel(const int32_t* tok, const __nv_bfloat16* E, const __nv_bfloat16* vis,
-                             int n_vis, int T, int d, int vocab, float* h, __nv_bfloat16* hb,
+                             int n_vis, int T, int d, int vocab, float* h, __half* hb,
                              const __nv_bfloat16* g0, float* ssp, unsigned long long* keys,
                              int* err) {
   pdl_wait();
@@ -238,9 +238,9 @@ __global__ void embed_kernel(const int32_t* tok, const __nv_bfloat16* E, const _
     *reinterpret_cast<float4*>(dst) = make_float4(x[0], x[1], x[2], x[3]);
     *reinterpret_cast<float4*>(dst + 4) = make_float4(x[4], x[5], x[6], x[7]);
     uint4 ob;
-    __nv_bfloat162* op = reinterpret_cast<__nv_bfloat162*>(&ob);
+    __half* op = reinterpret_cast<__half*>(&ob);
 #pragma unroll
-    for (int i = 0; i < 4; ++i) op[i] = __floats2bfloat162_rn(o[2 * i], o[2 * i + 1]);
+    for (int i = 0; i < 8; ++i) op[i] = to_f16(o[i], err);
     *reinterpret_cast<uint4*>(hb + static_cast<size_t>(t) * d + c) = ob;
     // 16 consecutive threads cover one 128-feature block
 #pragma unroll
@@ -248,6 +248,46 @@ __global__ void embed_kernel(const int32_t* tok, const __nv_bfloat16* E, const _
     if ((threadIdx.x & 15) == 0) ssp[static_cast<size_t>(t) * n_ssp + c / 128] = sq;
   }
   if (threadIdx.x == 0 && keys != nullptr) keys[t] = 0ull;
+}
+
+// Largest |w| over a bf16 tensor of n elements (n % 8 == 0, 16-byte aligned),
+// folded into *out as float bits (non-negative floats order like their bits).
+__global__ void absmax_bf16_kernel(const __nv_bfloat16* w, size_t n, unsigned int* out) {
+  float m = 0.f;
+  const size_t n8 = n / 8;
+  for (size_t i = blockIdx.x * static_cast<size_t>(blockDim.x) + threadIdx.x; i < n8;
+       i += static_cast<size_t>(gridDim.x) * blockDim.x) {
+    const uint4 raw = reinterpret_cast<const uint4*>(w)[i];
+    const __nv_bfloat162* p = reinterpret_cast<const __nv_bfloat162*>(&raw);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const float2 f = __bfloat1622float2(p[k]);
+      m = fmaxf(m, fmaxf(fabsf(f.x), fabsf(f.y)));
+    }
+  }
+#pragma unroll
+  for (int o = 16; o >= 1; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xFFFFFFFFu, m, o));
+  if ((threadIdx.x & 31) == 0) atomicMax(out, __float_as_uint(m));
+}
+
+// dst = fp16(w * 2^s): the weight copy the GEMMs read.  With 2^s chosen so the
+// largest |w| * 2^s stays below 2^15, every bf16 value down to 2^-(16 + s) in
+// magnitude converts exactly (fp16 keeps 8 significant bits to 2^-16).
+__global__ void scale_to_f16_kernel(const __nv_bfloat16* w, size_t n, float scale, __half* dst) {
+  const size_t n8 = n / 8;
+  for (size_t i = blockIdx.x * static_cast<size_t>(blockDim.x) + threadIdx.x; i < n8;
+       i += static_cast<size_t>(gridDim.x) * blockDim.x) {
+    const uint4 raw = reinterpret_cast<const uint4*>(w)[i];
+    const __nv_bfloat162* p = reinterpret_cast<const __nv_bfloat162*>(&raw);
+    uint4 ob;
+    __half2* op = reinterpret_cast<__half2*>(&ob);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const float2 f = __bfloat1622float2(p[k]);
+      op[k] = __floats2half2_rn(f.x * scale, f.y * scale);
+    }
+    reinterpret_cast<uint4*>(dst)[i] = ob;
+  }
 }
 
 // cos/sin table: angle p * theta^(-2i/64), computed in double precision.

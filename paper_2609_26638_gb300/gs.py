@@ -22,7 +22,7 @@ GS_ERR_DEVICE_CHECK = 5
 GS_ERR_TIMEOUT = 6
 GS_ACCEPT_GREEDY = 0
 GS_ACCEPT_STOCHASTIC = 1
-EPI_STORE_BF16, EPI_RESID_F32, EPI_SWIGLU, EPI_ARGMAX = 0, 1, 2, 3
+EPI_STORE_F16, EPI_RESID_F32, EPI_SWIGLU, EPI_ARGMAX = 0, 1, 2, 3
 ATTN_DRAFT, ATTN_VERIFY = 0, 1
 KIND_NAMES = ("window", "embed", "qkv", "attention", "o_proj", "gate_up", "down", "lm_head",
               "accept")

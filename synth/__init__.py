@@ -272,9 +272,10 @@ SWEEP_PREFIX = (1024, 4096, 8192)
 
 def attn_inputs(batch: int, W: int, ctx: int, n_heads: int = 16, n_kv_heads: int = 8,
                 head_dim: int = 64, seed: int = INPUT_SEED, index: int = 0):
-    """Q [batch, W, Hq, hd] and K/V [batch, ctx, Hkv, hd], N(0,1) as bf16 bits."""
+    """Q [batch, W, Hq, hd] and K/V [batch, ctx, Hkv, hd]: N(0,1) draws rounded
+    to fp16 (the attention kernel's operand type), as np.float16 arrays."""
     rng = _rng(seed, 400, index)
-    q = _normal_bf16(rng, (batch, W, n_heads, head_dim), 1.0)
-    k = _normal_bf16(rng, (batch, ctx, n_kv_heads, head_dim), 1.0)
-    v = _normal_bf16(rng, (batch, ctx, n_kv_heads, head_dim), 1.0)
+    q = rng.standard_normal((batch, W, n_heads, head_dim), dtype=np.float32).astype(np.float16)
+    k = rng.standard_normal((batch, ctx, n_kv_heads, head_dim), dtype=np.float32).astype(np.float16)
+    v = rng.standard_normal((batch, ctx, n_kv_heads, head_dim), dtype=np.float32).astype(np.float16)
     return q, k, v

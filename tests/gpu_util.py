@@ -25,7 +25,7 @@ import torch
 from oracle import decode as od
 
 NEAR_TIE = 0.1          # nats, top-2 logit gap under which a flip is allowed
-LOGIT_TOL = 3e-2        # max-abs logit error, bf16 path vs float64 oracle
+LOGIT_TOL = 3e-2        # max-abs logit error, 16-bit GPU path vs float64 oracle
 
 
 @dataclasses.dataclass
@@ -54,14 +54,16 @@ def gpu_accept(vin: np.ndarray, vt: np.ndarray, K: int) -> int:
 
 
 def lockstep(eng, dec, prompt, K: int, max_new: int, max_rounds: int = 1 << 30, slot: int = 0,
-             eos: int = -1, check_logits: bool = False, logit_tol: float = LOGIT_TOL):
+             eos: int = -1, check_logits: bool = False, logit_tol: float = LOGIT_TOL,
+             oracle_state=None):
     from paper_2609_26638_gb300 import gs
     dev = eng.device
     V = dec.cfg.vocab
     W = K + 1
     stats = LockstepStats()
     cap = prompt.length + 2 * max_new + K + 8
-    st = od.prefill(dec, prompt.vis, prompt.text, cap, max_new, eos)
+    st = oracle_state if oracle_state is not None else od.prefill(dec, prompt.vis, prompt.text,
+                                                                   cap, max_new, eos)
     x0 = eng.prefill(slot, prompt.vis, prompt.text, max_new)
     if x0 != st.x0:
         assert st.prefill_gap < NEAR_TIE, ("prefill x0 differs", x0, st.x0, st.prefill_gap)
@@ -139,3 +141,26 @@ def lockstep(eng, dec, prompt, K: int, max_new: int, max_rounds: int = 1 << 30, 
             eng.prefill(slot, prompt.vis, text, max_new)
             eng.restore(slot, st.n, st.x0, len(st.out), max_new, int(st.done))
     return st, stats
+
+
+def decode_all(eng, slots, K, max_rounds, force=None):
+    """Rounds (graph launches) until every sequence in `slots` is done: per
+    sequence the committed tokens after its prefill's x0."""
+    dev = eng.device
+    n = slots.shape[0]
+    out_tok = torch.zeros((n, K + 2), dtype=torch.int32, device=dev)
+    cnt = torch.zeros(n, dtype=torch.int32, device=dev)
+    done = torch.zeros(n, dtype=torch.int32, device=dev)
+    outs = [[] for _ in range(n)]
+    torch.cuda.synchronize(dev)
+    for _ in range(max_rounds):
+        eng.round(slots, K, out_tok, cnt, done, force=force)
+        eng.stream.synchronize()
+        c = cnt.cpu().numpy()
+        t = out_tok.cpu().numpy()
+        for i in range(n):
+            outs[i].extend(t[i, :c[i]].tolist())
+        if done.cpu().numpy().all():
+            break
+    eng.check()
+    return outs

@@ -1,6 +1,13 @@
-"""Kernel-level GPU parity: the tcgen05 GEMM against a plain fp32 torch matmul,
-and the paged hybrid-mask attention against the oracle's float64 masked
-softmax (draft and verify masks from the oracle's mask builders)."""
+"""Kernel-level GPU parity: the tcgen05 GEMM against a plain fp32 torch matmul
+of the same fp16 operands, and the paged hybrid-mask attention against the
+oracle's float64 masked softmax (draft and verify masks from the oracle's mask
+builders).
+
+Tolerances follow from the arithmetic: products are exact in fp32 and
+accumulate in fp32 (relative error ~K * 2^-24), so a GEMM output carries the
+fp16 rounding of its store, 2^-11 relative; attention carries the fp16
+rounding of the probabilities fed to P.V (each p within 2^-11 relative, so
+the output within 2^-11 * max|v|) plus the fp16 store of the output."""
 import math
 import types
 
@@ -34,12 +41,12 @@ def _linear(gs, x, w, M, N, K, epi, split, y):
 @pytest.mark.parametrize("N,K,split", [(256, 256, 1), (2048, 1024, 8), (1024, 4096, 16)])
 def test_linear_store_and_residual(gs, M, N, K, split):
     g = torch.Generator(device=DEV).manual_seed(M * 7 + N)
-    x = torch.randn(M, K, device=DEV, generator=g).bfloat16()
-    w = (0.02 * torch.randn(N, K, device=DEV, generator=g)).bfloat16()
+    x = torch.randn(M, K, device=DEV, generator=g).half()
+    w = (0.02 * torch.randn(N, K, device=DEV, generator=g)).half()
     ref = x.float() @ w.float().T
-    y = torch.zeros(M, N, dtype=torch.bfloat16, device=DEV)
-    _linear(gs, x, w, M, N, K, gs.EPI_STORE_BF16, split, y)
-    torch.testing.assert_close(y.float(), ref, rtol=1e-2, atol=1e-2 * ref.abs().max().item())
+    y = torch.zeros(M, N, dtype=torch.float16, device=DEV)
+    _linear(gs, x, w, M, N, K, gs.EPI_STORE_F16, split, y)
+    torch.testing.assert_close(y.float(), ref, rtol=2e-3, atol=1e-3 * ref.abs().max().item())
     base = torch.randn(M, N, device=DEV, generator=g)
     r = base.clone()
     _linear(gs, x, w, M, N, K, gs.EPI_RESID_F32, split, r)
@@ -50,21 +57,21 @@ def test_linear_store_and_residual(gs, M, N, K, split):
 def test_linear_swiglu(gs, M, split):
     F, K = 1024, 256
     g = torch.Generator(device=DEV).manual_seed(3)
-    x = torch.randn(M, K, device=DEV, generator=g).bfloat16()
-    w = (0.05 * torch.randn(2 * F, K, device=DEV, generator=g)).bfloat16()
+    x = torch.randn(M, K, device=DEV, generator=g).half()
+    w = (0.05 * torch.randn(2 * F, K, device=DEV, generator=g)).half()
     gu = x.float() @ w.float().T
     ref = torch.nn.functional.silu(gu[:, :F]) * gu[:, F:]
-    y = torch.zeros(M, F, dtype=torch.bfloat16, device=DEV)
+    y = torch.zeros(M, F, dtype=torch.float16, device=DEV)
     _linear(gs, x, w, M, F, K, gs.EPI_SWIGLU, split, y)
-    torch.testing.assert_close(y.float(), ref, rtol=1.5e-2, atol=1e-2 * ref.abs().max().item())
+    torch.testing.assert_close(y.float(), ref, rtol=2e-3, atol=1e-3 * ref.abs().max().item())
 
 
 @pytest.mark.parametrize("M,V", [(1, 4096), (17, 59392), (70, 4096)])
 def test_linear_argmax(gs, M, V):
     K = 1024
     g = torch.Generator(device=DEV).manual_seed(M)
-    x = torch.randn(M, K, device=DEV, generator=g).bfloat16()
-    w = (0.02 * torch.randn(V, K, device=DEV, generator=g)).bfloat16()
+    x = torch.randn(M, K, device=DEV, generator=g).half()
+    w = (0.02 * torch.randn(V, K, device=DEV, generator=g)).half()
     ref = x.float() @ w.float().T
     keys = torch.zeros(M, dtype=torch.int64, device=DEV)
     _linear(gs, x, w, M, V, K, gs.EPI_ARGMAX, 1, keys)
@@ -88,14 +95,35 @@ def test_linear_rows_do_not_depend_on_batch(gs):
     """Same token tile and split: a row's bits do not depend on the other rows."""
     N, K = 2048, 1024
     g = torch.Generator(device=DEV).manual_seed(5)
-    x = torch.randn(17, K, device=DEV, generator=g).bfloat16()
-    w = (0.02 * torch.randn(N, K, device=DEV, generator=g)).bfloat16()
-    y17 = torch.zeros(17, N, dtype=torch.bfloat16, device=DEV)
-    _linear(gs, x, w, 17, N, K, gs.EPI_STORE_BF16, 8, y17)
+    x = torch.randn(17, K, device=DEV, generator=g).half()
+    w = (0.02 * torch.randn(N, K, device=DEV, generator=g)).half()
+    y17 = torch.zeros(17, N, dtype=torch.float16, device=DEV)
+    _linear(gs, x, w, 17, N, K, gs.EPI_STORE_F16, 8, y17)
     for r in (0, 5, 16):
-        y1 = torch.zeros(1, N, dtype=torch.bfloat16, device=DEV)
-        _linear(gs, x[r:r + 1].contiguous(), w, 1, N, K, gs.EPI_STORE_BF16, 8, y1)
+        y1 = torch.zeros(1, N, dtype=torch.float16, device=DEV)
+        _linear(gs, x[r:r + 1].contiguous(), w, 1, N, K, gs.EPI_STORE_F16, 8, y1)
         assert torch.equal(y1[0], y17[r])
+
+
+@pytest.mark.parametrize("split", [1, 2, 8])
+def test_linear_rows_do_not_depend_on_tile_width(gs, split):
+    """Same split-K factor, different token counts (token tiles of 32, 64, 128
+    and 256 columns): the first rows' bits are the same."""
+    N, K = 1024, 1024
+    g = torch.Generator(device=DEV).manual_seed(11)
+    x = torch.randn(300, K, device=DEV, generator=g).half()
+    w = (0.02 * torch.randn(N, K, device=DEV, generator=g)).half()
+    ys = {}
+    for M in (17, 40, 100, 300):
+        y = torch.zeros(M, N, dtype=torch.float16, device=DEV)
+        _linear(gs, x[:M].contiguous(), w, M, N, K, gs.EPI_STORE_F16, split, y)
+        ys[M] = y
+        r = torch.zeros(M, N, dtype=torch.float32, device=DEV)
+        _linear(gs, x[:M].contiguous(), w, M, N, K, gs.EPI_RESID_F32, split, r)
+        ys[(M, "f32")] = r
+    for M in (40, 100, 300):
+        assert torch.equal(ys[M][:17], ys[17]), M
+        assert torch.equal(ys[(M, "f32")][:17], ys[(17, "f32")]), M
 
 
 # ------------------------------------------------------------------ attention
@@ -105,7 +133,7 @@ def _paged(k, v, rng):
     pages_per = math.ceil(ctx / 64)
     n_pages = B * pages_per + 3
     perm = rng.permutation(n_pages)[: B * pages_per].reshape(B, pages_per)
-    pool = np.zeros((n_pages, 2, Hkv, 64, 64), dtype=np.uint16)
+    pool = np.zeros((n_pages, 2, Hkv, 64, 64), dtype=np.float16)
     for b in range(B):
         for p in range(pages_per):
             t0, t1 = p * 64, min(ctx, p * 64 + 64)
@@ -119,20 +147,20 @@ def _oracle_attn(q, k, v, allowed, Hq, Hkv):
     return Decoder.attention(fake, q, k, v, allowed)
 
 
-def _run_attention(gs, mode, q_bits, pool, pt, n_arr, W, Hq, Hkv, split_pages):
-    B = q_bits.shape[0]
-    qd = torch.from_numpy(q_bits.view(np.int16)).to(DEV)
-    kvd = torch.from_numpy(pool.view(np.int16)).to(DEV)
+def _run_attention(gs, mode, q, pool, pt, n_arr, W, Hq, Hkv, split_pages):
+    B = q.shape[0]
+    qd = torch.from_numpy(q).to(DEV)
+    kvd = torch.from_numpy(pool).to(DEV)
     ptd = torch.from_numpy(pt).to(DEV)
     nd = torch.from_numpy(n_arr.astype(np.int32)).to(DEV)
-    out = torch.zeros(q_bits.shape, dtype=torch.int16, device=DEV)
+    out = torch.zeros(q.shape, dtype=torch.float16, device=DEV)
     sb = gs.gs_attention_scratch_bytes(B, W, Hq, Hkv, pt.shape[1], split_pages)
     scratch = torch.zeros(sb, dtype=torch.uint8, device=DEV)
     gs.gs_attention(mode, qd.data_ptr(), kvd.data_ptr(), pool.shape[0], ptd.data_ptr(), pt.shape[1],
                     nd.data_ptr(), B, W, Hq, Hkv, out.data_ptr(), scratch.data_ptr(), sb,
                     split_pages, torch.cuda.current_stream().cuda_stream)
     torch.cuda.synchronize()
-    return synth.bf16_bits_to_f32(out.cpu().numpy().view(np.uint16)).astype(np.float64)
+    return out.cpu().numpy().astype(np.float64)
 
 
 @pytest.mark.parametrize("mode", [0, 1])
@@ -154,11 +182,9 @@ def test_attention_matches_oracle(gs, mode, W, ns, Hq, Hkv, sp):
     for b, n in enumerate(ns):
         allowed = od.draft_allowed(n, K) if mode == 0 else od.verify_allowed(n, K)
         nk = allowed.shape[1]
-        qf = synth.bf16_bits_to_f32(q[b]).astype(np.float64)
-        kf = synth.bf16_bits_to_f32(k[b, :nk]).astype(np.float64)
-        vf = synth.bf16_bits_to_f32(v[b, :nk]).astype(np.float64)
-        want = _oracle_attn(qf, kf, vf, allowed, Hq, Hkv)
-        np.testing.assert_allclose(got[b], want, rtol=2e-2, atol=2e-2)
+        want = _oracle_attn(q[b].astype(np.float64), k[b, :nk].astype(np.float64),
+                            v[b, :nk].astype(np.float64), allowed, Hq, Hkv)
+        np.testing.assert_allclose(got[b], want, rtol=5e-3, atol=5e-3)
 
 
 @pytest.mark.parametrize("B,prefix,K", [(64, 8192, 64), (8, 4096, 16), (1, 1024, 4)])
@@ -171,13 +197,12 @@ def test_attention_sweep_sizes_sampled(gs, B, prefix, K):
     ctx = prefix + W + 1
     q, k, v = synth.attn_inputs(B, W, ctx, Hq, Hkv, index=B)
     pool, pt, _ = _paged(k, v, rng)
-    sp = max(1, math.ceil(pt.shape[1] * B * Hkv / 304))
+    sp = min(32, max(2, math.ceil(pt.shape[1] * B * Hkv / (152 * 16))))
     for mode in (0, 1):
         got = _run_attention(gs, mode, q, pool, pt, np.array(ns), W, Hq, Hkv, sp)
         for b in sorted(set([0, B - 1] + list(rng.integers(0, B, 2)))):
             allowed = od.draft_allowed(prefix, K) if mode == 0 else od.verify_allowed(prefix, K)
             nk = allowed.shape[1]
-            want = _oracle_attn(synth.bf16_bits_to_f32(q[b]).astype(np.float64),
-                                synth.bf16_bits_to_f32(k[b, :nk]).astype(np.float64),
-                                synth.bf16_bits_to_f32(v[b, :nk]).astype(np.float64), allowed, Hq, Hkv)
-            np.testing.assert_allclose(got[b], want, rtol=2e-2, atol=2e-2)
+            want = _oracle_attn(q[b].astype(np.float64), k[b, :nk].astype(np.float64),
+                                v[b, :nk].astype(np.float64), allowed, Hq, Hkv)
+            np.testing.assert_allclose(got[b], want, rtol=5e-3, atol=5e-3)

@@ -6,7 +6,7 @@ import torch
 import synth
 from oracle import decode as od
 from oracle.model import Decoder
-from tests.gpu_util import NEAR_TIE, gpu_accept, lockstep, new_engine
+from tests.gpu_util import NEAR_TIE, decode_all, gpu_accept, lockstep, new_engine
 
 pytestmark = pytest.mark.gpu
 
@@ -51,27 +51,6 @@ def test_tiny_gqa_gains_lockstep(tiny_gain, K, n_vis, n_text):
     eng.close()
 
 
-def _decode_all(eng, slots, K, max_rounds, force=None):
-    dev = eng.device
-    n = slots.shape[0]
-    out_tok = torch.zeros((n, K + 2), dtype=torch.int32, device=dev)
-    cnt = torch.zeros(n, dtype=torch.int32, device=dev)
-    done = torch.zeros(n, dtype=torch.int32, device=dev)
-    outs = [[] for _ in range(n)]
-    torch.cuda.synchronize(dev)
-    for _ in range(max_rounds):
-        eng.round(slots, K, out_tok, cnt, done, force=force)
-        eng.stream.synchronize()
-        c = cnt.cpu().numpy()
-        t = out_tok.cpu().numpy()
-        for i in range(n):
-            outs[i].extend(t[i, :c[i]].tolist())
-        if done.cpu().numpy().all():
-            break
-    eng.check()
-    return outs
-
-
 def test_gpu_self_spec_equals_gpu_ar(tiny_gain):
     """Batch-invariant kernels: the GPU's self-speculative output equals its own
     greedy AR (K = 0) output token for token (the paper's AR-equivalence, here
@@ -83,7 +62,7 @@ def test_gpu_self_spec_equals_gpu_ar(tiny_gain):
     outs = {}
     for K in (0, 3, 8, 16):
         x0 = eng.prefill(0, prompt.vis, prompt.text, 200)
-        outs[K] = [x0] + _decode_all(eng, slots, K, 400)[0]
+        outs[K] = [x0] + decode_all(eng, slots, K, 400)[0]
         assert len(outs[K]) == 200
     assert outs[3] == outs[0] and outs[8] == outs[0] and outs[16] == outs[0]
     eng.close()
@@ -97,7 +76,7 @@ def test_forced_acceptance_hits_schedule(tiny_gain):
     prompt = synth.make_prompt(cfg, 300, 20, index=12)
     slots = torch.tensor([0], dtype=torch.int32, device=eng.device)
     x0 = eng.prefill(0, prompt.vis, prompt.text, max_new + K + 4)
-    ref = [x0] + _decode_all(eng, slots, K, 1000)[0]
+    ref = [x0] + decode_all(eng, slots, K, 1000)[0]
     P = prompt.length
     teacher = np.full(P + len(ref) + 4, -1, np.int32)
     teacher[P:P + len(ref)] = ref
@@ -142,11 +121,11 @@ def test_batch_equals_single_and_ragged_finish(tiny_gain):
     single = []
     for i, p in enumerate(prompts):
         x0 = eng.prefill(i, p.vis, p.text, caps[i])
-        single.append([x0] + _decode_all(eng, torch.tensor([i], dtype=torch.int32, device=eng.device),
+        single.append([x0] + decode_all(eng, torch.tensor([i], dtype=torch.int32, device=eng.device),
                                          K, 100)[0])
     x0s = [eng.prefill(i, p.vis, p.text, caps[i]) for i, p in enumerate(prompts)]
     slots = torch.tensor([2, 0, 1], dtype=torch.int32, device=eng.device)   # any slot order
-    outs = _decode_all(eng, slots, K, 100)
+    outs = decode_all(eng, slots, K, 100)
     batch = {2: outs[0], 0: outs[1], 1: outs[2]}
     for i in range(3):
         assert [x0s[i]] + batch[i] == single[i]

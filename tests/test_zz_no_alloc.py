@@ -31,13 +31,13 @@ def _with_caller_scratch(gs, x, w, M, N, K, epi, split, y):
 def test_noalloc_matches_linear_on_two_calls_in_a_row(gs):
     stream = torch.cuda.current_stream().cuda_stream
     g = torch.Generator(device=DEV).manual_seed(11)
-    cases = [(17, 2048, 1024, gs.EPI_STORE_BF16, 8), (9, 1024, 4096, gs.EPI_STORE_BF16, 16)]
+    cases = [(17, 2048, 1024, gs.EPI_STORE_F16, 8), (9, 1024, 4096, gs.EPI_STORE_F16, 16)]
     for M, N, K, epi, split in cases:          # two calls in a row share the one array
-        x = torch.randn(M, K, device=DEV, generator=g).bfloat16()
-        w = (0.02 * torch.randn(N, K, device=DEV, generator=g)).bfloat16()
-        want = torch.zeros(M, N, dtype=torch.bfloat16, device=DEV)
+        x = torch.randn(M, K, device=DEV, generator=g).half()
+        w = (0.02 * torch.randn(N, K, device=DEV, generator=g)).half()
+        want = torch.zeros(M, N, dtype=torch.float16, device=DEV)
         _with_caller_scratch(gs, x, w, M, N, K, epi, split, want)
-        got = torch.zeros(M, N, dtype=torch.bfloat16, device=DEV)
+        got = torch.zeros(M, N, dtype=torch.float16, device=DEV)
         gs.gs_linear_noalloc(x.data_ptr(), w.data_ptr(), got.data_ptr(), M, N, K, epi, split, stream)
         torch.cuda.synchronize()
         ref = x.float() @ w.float().T
@@ -48,10 +48,10 @@ def test_noalloc_matches_linear_on_two_calls_in_a_row(gs):
 
 def test_noalloc_rejects_scratch_beyond_its_array(gs):
     # 64 k-block splits over 64 feature tiles of 32 rows need 64 MiB of partials > 8 MiB
-    x = torch.zeros(17, 4096, dtype=torch.bfloat16, device=DEV)
-    w = torch.zeros(8192, 4096, dtype=torch.bfloat16, device=DEV)
-    y = torch.zeros(17, 8192, dtype=torch.bfloat16, device=DEV)
+    x = torch.zeros(17, 4096, dtype=torch.float16, device=DEV)
+    w = torch.zeros(8192, 4096, dtype=torch.float16, device=DEV)
+    y = torch.zeros(17, 8192, dtype=torch.float16, device=DEV)
     with pytest.raises(gs.GsError) as e:
         gs.gs_linear_noalloc(x.data_ptr(), w.data_ptr(), y.data_ptr(), 17, 8192, 4096,
-                             gs.EPI_STORE_BF16, 64, torch.cuda.current_stream().cuda_stream)
+                             gs.EPI_STORE_F16, 64, torch.cuda.current_stream().cuda_stream)
     assert e.value.code == gs.GS_ERR_OOM
