@@ -385,7 +385,7 @@ def attention_roofline(cfg, dev):
     out = torch.zeros_like(q)
     ptd = torch.from_numpy(pt).to(dev)
     nd = torch.from_numpy(ns).to(dev)
-    sp = min(32, max(2, math.ceil(pt_stride * B * Hkv / (152 * 16))))
+    sp = max(2, math.ceil(pt_stride / 8))   # the engine's default: at most 8 items
     sb = gs.gs_attention_scratch_bytes(B, W, Hq, Hkv, pt_stride, sp)
     scratch = torch.zeros(sb, dtype=torch.uint8, device=dev)
     stream = torch.cuda.current_stream(dev)

@@ -1,41 +1,50 @@
 // attention.cuh -- hybrid-mask attention over the paged fp16 KV cache.
 //
-// A query block is a run of tokens of one sequence (the K+1 window of a decode
-// forward, or 64 tokens of a prefill chunk); its rows are (token, query head
-// of the GQA group), so the query heads that share a KV head read each K/V
-// page once.  Every query token carries its own inclusive key limit, which
-// encodes the mask: draft boundary row n, draft mask rows n+K, verify row i
-// n+1+i, prefill row p (paper Appendix steps Draft forward / Verify forward).
+// A query block is a run of at most kAttnMaxRows / G tokens of one sequence
+// (a decode window, cut into sub-blocks when K+1 tokens carry more than 128
+// rows, or a slice of a prefill chunk); its rows are (token, query head of the
+// GQA group), so the query heads that share a KV head read each K/V page once.
+// Every query token carries its own inclusive key limit, which encodes the
+// mask: draft boundary row n, draft mask rows n+K, verify row i n+1+i, prefill
+// row p (paper Appendix steps Draft forward / Verify forward).
 //
 // Work items.  The block's pages are cut into fixed absolute ranges of SP
-// pages ("items"): item i covers pages [i*SP, (i+1)*SP).  One warp group (one
-// warp per 16 rows) reduces one item: it streams the item's K and V pages
-// (64 tokens x 64 dims, 8 KB each) through its own ring of TMA stages with
-// 128-byte swizzle, and each warp runs S = Q K^T and O += P V on mma.sync
-// m16n8k16 (fp16 in, fp32 out) with the online softmax in registers (exp2,
-// the 1/sqrt(64) scale folded), pages in order.  A CTA = (item group, KV
-// head, query block) holds NG warp groups on consecutive items and shares the
-// block's Q tile among them.
+// pages ("items"): item i covers pages [i*SP, (i+1)*SP); one CTA reduces one
+// item.  Inside an item the pages are dealt to two lanes by parity (lane l
+// takes the item's pages l, l+2, ...); each lane is a warp group (one warp per
+// 16 rows) with its own ring of TMA stages (K and V pages, 64 tokens x 64
+// dims, 8 KB each, 128-byte swizzle).  Each warp runs S = Q K^T and O += P V
+// on mma.sync m16n8k16 (fp16 in, fp32 out) with the online softmax in
+// registers (exp2, the 1/sqrt(64) scale folded), its lane's pages in order.
+// The two lanes' (O, m, l) then merge in shared memory, lane 0 first.
 //
-// Merge.  A block with one item writes its rows directly.  Otherwise each item
-// writes its rows' (O, m, l) to global scratch, and the last item to finish
-// (atomic ticket per (block, head), no spinning) merges the items in order
-// 0, 1, ...: M = max m_i, w_i = exp2(m_i - M), O = sum w_i O_i / sum w_i l_i.
+// Merge over items, item order 0, 1, ...: M = max m_i, w_i = exp2(m_i - M),
+// coef_i = w_i / sum_j w_j l_j, O = sum coef_i O_i.  A block with one item
+// writes its rows directly.  With at most 8 items the items of a (block, head)
+// form one thread-block cluster: each CTA sends the rows that CTA (r mod n)
+// owns to it with one bulk async copy into its shared memory, completing on
+// its mbarrier, and each owner merges its rows.  With more items every item
+// writes its rows to global scratch and the last one to finish (atomic ticket
+// per (block, head), no spinning) merges them.  Both paths run the same
+// arithmetic in the same order.
 //
-// Invariance.  Item boundaries are absolute page numbers fixed by SP, each
-// item is reduced page by page in one warp, and the merge runs in item order,
-// so a row's result depends only on its own query, keys and limit: not on the
-// other rows of its window, the window size, the batch, or how many groups a
-// CTA holds.  Keys past a row's limit contribute exact zeros.
+// Invariance.  Item boundaries are absolute page numbers fixed by SP, the
+// lanes deal pages by parity, and the merges run in fixed order, so a row's
+// result depends only on its query, keys, limit and SP: not on the other rows
+// of its block, the window size, the batch, or the merge path.  Keys past a
+// row's limit contribute exact zeros.
 #pragma once
 #include "ptx.cuh"
 
 namespace gs {
 
-constexpr int kAttnStages = 3;             // K/V pages in flight per warp group
+constexpr int kAttnStages = 2;             // K/V pages in flight per lane
+constexpr int kAttnLanes = 2;
 constexpr int kAttnPageBytes = 64 * 128;  // 64 tokens x 64 fp16
 constexpr int kAttnRow = 68;              // partial row: O[64], m, l, 2 pad (272 B)
-constexpr int kAttnMaxGroups = 4;
+constexpr int kAttnMaxRows = 128;         // rows of one query block
+constexpr int kAttnMaxCluster = 8;        // items merged inside a cluster
+constexpr int kAttnRingBytes = kAttnLanes * kAttnStages * 2 * kAttnPageBytes;
 
 struct AttnArgs {
   const __half* q;            // [T, Hq, 64]
@@ -43,42 +52,42 @@ struct AttnArgs {
   __half* out;                // [T, Hq, 64]
   const int32_t* page_table;  // [slots, pt_stride]
   int pt_stride;
-  const int32_t* blk_slot;    // [n_blocks] page-table row per block, or null -> fixed_slot
-  const int32_t* blk_active;  // [n_blocks] nonzero = run, or null
+  const int32_t* blk_slot;    // [n_seq] page-table row per sequence, or null -> fixed_slot
+  const int32_t* blk_active;  // [n_seq] nonzero = run, or null
   int fixed_slot;
-  int T, QB;                  // tokens; tokens per query block
+  int T;                      // tokens
+  int QB;                     // tokens per sequence window (prefill: per block)
+  int QS, n_sub;              // tokens per query block; blocks per window
   int Hq, Hkv, G;
   long long kv_row_base;      // first KV-map row of this layer
   int rows_per_page;          // 2 * Hkv * 64
   int split_pages;            // SP: pages per item
-  int max_items;              // item slots per (block, head) in `part`
-  int r_pad;                  // row slots per item in `part` (>= rows of a block)
-  float* part;                // [n_blocks][Hkv][max_items][r_pad][kAttnRow]
-  int* ticket;                // [n_blocks][Hkv], zero between launches
+  int max_items;              // items per (block, head) the grid covers
+  int cluster;                // 1: the grid's x dimension is one cluster (max_items <= 8)
+  float* part;                // global merge: [n_blocks][Hkv][max_items][rows][kAttnRow]
+  int* ticket;                // global merge: [n_blocks][Hkv], zero between launches
   int* err;
 };
 
-// Rows (16 per warp) and launch shape for a block of r_max rows and ng groups.
-__host__ __device__ inline int attn_mtiles(int r_max) { return (r_max + 15) / 16; }
-__host__ __device__ inline int attn_threads(int r_max, int ng) { return attn_mtiles(r_max) * ng * 32; }
-__host__ __device__ inline int attn_smem_bytes(int r_max, int ng) {
-  return 1024 + attn_mtiles(r_max) * 16 * 128 + ng * kAttnStages * 2 * kAttnPageBytes +
-         ng * kAttnStages * 8 + 64;
+__host__ __device__ inline int attn_mtiles(int rows) { return (rows + 15) / 16; }
+__host__ __device__ inline int attn_threads(int rows) {
+  return kAttnLanes * attn_mtiles(rows) * 32;
 }
-// Warp groups per CTA: two when the launch has several waves of single-group
-// CTAs and two groups fit in 512 threads, else one.  Does not change results.
-__host__ __device__ inline int attn_groups_for(int r_max, int ctas_one_group) {
-  return (ctas_one_group >= 4 * 152 && attn_threads(r_max, 2) <= 512) ? 2 : 1;
+// receive buffer of an owner: n sources x ceil(rows / n) rows, at most rows + 8
+__host__ __device__ inline int attn_recv_floats(int rows) {
+  return (attn_mtiles(rows) * 16 + kAttnMaxCluster) * kAttnRow;
 }
-// Largest dynamic shared memory any launch asks for (rows <= 256).
-__host__ __device__ inline int attn_max_smem_bytes() {
-  const int a = attn_smem_bytes(256, 1), b = attn_smem_bytes(128, 2);
-  return a > b ? a : b;
+__host__ __device__ inline int attn_smem_bytes(int rows) {
+  return 1024 + attn_mtiles(rows) * 16 * 128 + kAttnRingBytes + attn_recv_floats(rows) * 4 + 128;
 }
-// The merge keeps one coefficient per (item, row) in the merging group's ring.
-__host__ __device__ inline int attn_max_merge_items(int r_max) {
-  return kAttnStages * 2 * kAttnPageBytes / 4 / (attn_mtiles(r_max) * 16);
+__host__ __device__ inline int attn_max_smem_bytes() { return attn_smem_bytes(kAttnMaxRows); }
+// The merge keeps m and l of every (item, row) in the idle ring.
+__host__ __device__ inline int attn_max_merge_items(int rows) {
+  return kAttnRingBytes / 4 / (2 * attn_mtiles(rows) * 16);
 }
+static_assert(kAttnRingBytes >= kAttnMaxRows * kAttnRow * 4 &&
+                  kAttnRingBytes >= (kAttnMaxRows + kAttnMaxCluster) * kAttnRow * 4,
+              "the idle ring holds a lane's partial rows and the owner-grouped rows");
 
 __device__ __forceinline__ uint32_t sw128(int row, int chunk) {
   return static_cast<uint32_t>(row * 128 + ((chunk ^ (row & 7)) << 4));
@@ -112,9 +121,9 @@ __device__ __forceinline__ uint32_t pack_f16x2(float lo, float hi) {
   return *reinterpret_cast<uint32_t*>(&v);
 }
 
-// Barrier over the warps of one group (ids 1..kAttnMaxGroups; 0 is __syncthreads).
-__device__ __forceinline__ void group_sync(int grp, int nthreads) {
-  asm volatile("bar.sync %0, %1;" ::"r"(grp + 1), "r"(nthreads) : "memory");
+// Barrier over the warps of one lane (ids 1, 2; 0 is __syncthreads).
+__device__ __forceinline__ void lane_sync(int lane_id, int nthreads) {
+  asm volatile("bar.sync %0, %1;" ::"r"(lane_id + 1), "r"(nthreads) : "memory");
 }
 
 __global__ void __launch_bounds__(512)
@@ -123,32 +132,34 @@ __global__ void __launch_bounds__(512)
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int mtiles = attn_mtiles(a.QB * a.G);
-  const int NG = blockDim.x / 32 / mtiles;    // warp groups of this CTA
-  const int grp = warp / mtiles, mt = warp % mtiles;
-  const int gthreads = mtiles * 32;
-  const int gtid = threadIdx.x - grp * gthreads;
+  const int mtiles = attn_mtiles(a.QS * a.G);
+  const int ln = warp / mtiles, mt = warp % mtiles;   // page lane, row tile
+  const int lthreads = mtiles * 32;
+  const int ltid = threadIdx.x - ln * lthreads;
   const int rows_alloc = mtiles * 16;
-  uint8_t* sQ = smem;                                              // [rows][128 B]
-  uint8_t* ring = smem + rows_alloc * 128;                         // [NG][stages][K | V]
-  uint8_t* sK = ring + grp * kAttnStages * 2 * kAttnPageBytes;     // this group's stages
+  uint8_t* sQ = smem;                                   // [rows][128 B]
+  uint8_t* ring = smem + rows_alloc * 128;              // [lane][stage][K | V]
+  uint8_t* sK = ring + ln * kAttnStages * 2 * kAttnPageBytes;
   uint8_t* sV = sK + kAttnStages * kAttnPageBytes;
-  uint64_t* full = reinterpret_cast<uint64_t*>(ring + NG * kAttnStages * 2 * kAttnPageBytes);
-  uint64_t* gfull = full + grp * kAttnStages;
-  int* s_int = reinterpret_cast<int*>(full + NG * kAttnStages);   // [0] max limit, [1+g] last flag
+  float* recv = reinterpret_cast<float*>(ring + kAttnRingBytes);   // [source][slot][kAttnRow]
+  uint64_t* full = reinterpret_cast<uint64_t*>(recv + attn_recv_floats(rows_alloc));
+  uint64_t* lfull = full + ln * kAttnStages;
+  uint64_t* recv_bar = full + kAttnLanes * kAttnStages;
+  int* s_int = reinterpret_cast<int*>(recv_bar + 1);    // [0] max limit, [1] last-item flag
 
-  const int h = blockIdx.y, b = blockIdx.z;
+  const int c = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
+  const int seq = b / a.n_sub, sub = b % a.n_sub;
   // Before griddepcontrol.wait this kernel reads only what the kernel right
   // before it (the QKV GEMM, which writes q and the window's K/V) does not
   // write: the window descriptors (key limits, block slots), the page table,
   // and cache pages wholly before the current window.  Every early exit is
-  // uniform across the CTA.
-  if (a.blk_active != nullptr && a.blk_active[b] == 0) return;
-  const int tok0 = b * a.QB;
-  const int ntok = min(a.QB, a.T - tok0);
+  // uniform across the CTA, and across the cluster before its barrier.
+  if (a.blk_active != nullptr && a.blk_active[seq] == 0) return;
+  const int tok0 = seq * a.QB + sub * a.QS;
+  const int ntok = min(min(a.QS, a.QB - sub * a.QS), a.T - tok0);
   if (ntok <= 0) return;
   const int R = ntok * a.G;
-  const int slot = a.blk_slot ? a.blk_slot[b] : a.fixed_slot;
+  const int slot = a.blk_slot ? a.blk_slot[seq] : a.fixed_slot;
 
   if (warp == 0) {
     int m = -1;
@@ -162,38 +173,46 @@ __global__ void __launch_bounds__(512)
   const int npages_blk = maxlim / 64 + 1;
   const int SP = a.split_pages;
   const int nitems = (npages_blk + SP - 1) / SP;
-  if (maxlim < 0 || npages_blk > a.pt_stride || slot < 0 || nitems > a.max_items ||
-      R > a.r_pad) {
+  if (maxlim < 0 || npages_blk > a.pt_stride || slot < 0 || nitems > a.max_items) {
     if (threadIdx.x == 0) atomicExch(a.err, kErrBounds);
     return;
   }
-  const int item0 = blockIdx.x * NG;
-  if (item0 >= nitems) return;
-  const int item = item0 + grp;
-  const bool has_item = item < nitems;
-  const int p_begin = item * SP;
-  const int np = has_item ? min(npages_blk, p_begin + SP) - p_begin : 0;
-  const int32_t* pt = a.page_table + static_cast<size_t>(slot) * a.pt_stride;
+  if (c >= nitems && (nitems == 1 || !a.cluster)) return;
+  const bool in_cluster = a.cluster && nitems > 1;
 
   if (threadIdx.x == 0) {
     tma_prefetch_desc(&tmKV);
-    for (int s = 0; s < NG * kAttnStages; ++s) mbar_init(smem_u32(&full[s]), 1);
+    for (int s = 0; s < kAttnLanes * kAttnStages; ++s) mbar_init(smem_u32(&full[s]), 1);
+    if (in_cluster) {
+      mbar_init(smem_u32(recv_bar), 1);
+      // nitems sources, ceil(rows / nitems) rows each, arrive by bulk copy
+      const int rpo = (rows_alloc + nitems - 1) / nitems;
+      mbar_arrive_expect_tx(smem_u32(recv_bar), static_cast<uint32_t>(nitems * rpo * kAttnRow * 4));
+    }
     fence_mbar_init();
   }
   __syncthreads();
-  const bool producer = gtid == 0;
+  if (in_cluster) cluster_arrive_release();   // waited on before the first remote access
+  if (c >= nitems) return;                     // idle cluster member: arrived, owns nothing
+
+  const int p_begin = c * SP;
+  const int np = min(npages_blk, p_begin + SP) - p_begin;
+  const int npl = np > ln ? (np - ln + 1) / kAttnLanes : 0;   // this lane's pages
+  const int32_t* pt = a.page_table + static_cast<size_t>(slot) * a.pt_stride;
+  const bool producer = ltid == 0;
   // pages wholly before the block's first slot hold committed states only
   const int safe_pages = a.blk_slot ? a.lim[tok0] / 64 : 0;
   const uint64_t pol = l2_policy_evict_first();
+  auto page_of = [&](int i) { return p_begin + ln + kAttnLanes * i; };
   auto issue = [&](int i) {
     const int s = i % kAttnStages;
-    int phys = pt[p_begin + i];
+    int phys = pt[page_of(i)];
     if (phys < 0) {  // unmapped page: the TMA box lands out of bounds and reads zeros
       atomicExch(a.err, kErrBounds);
       phys = 0x3FFFFFFF / a.rows_per_page;
     }
     const long long row = a.kv_row_base + static_cast<long long>(phys) * a.rows_per_page;
-    const uint32_t fb = smem_u32(&gfull[s]);
+    const uint32_t fb = smem_u32(&lfull[s]);
     mbar_arrive_expect_tx(fb, 2 * kAttnPageBytes);
     tma_load_2d(smem_u32(sK + s * kAttnPageBytes), &tmKV, 0, static_cast<int>(row + h * 64), fb, pol);
     tma_load_2d(smem_u32(sV + s * kAttnPageBytes), &tmKV, 0,
@@ -201,12 +220,12 @@ __global__ void __launch_bounds__(512)
   };
   int issued = 0;
   if (producer) {
-    while (issued < min(np, kAttnStages) && p_begin + issued < safe_pages) issue(issued++);
+    while (issued < min(npl, kAttnStages) && page_of(issued) < safe_pages) issue(issued++);
   }
   pdl_wait();
   pdl_trigger();
   if (producer) {
-    while (issued < min(np, kAttnStages)) issue(issued++);
+    while (issued < min(npl, kAttnStages)) issue(issued++);
   }
 
   // Q rows -> swizzled smem (zero rows past R)
@@ -221,7 +240,6 @@ __global__ void __launch_bounds__(512)
     *reinterpret_cast<uint4*>(sQ + sw128(r, ch)) = v;
   }
   __syncthreads();
-  if (!has_item) return;
 
   const bool has_rows = mt * 16 < R;
   const int g = lane >> 2, tq = lane & 3;
@@ -246,9 +264,9 @@ __global__ void __launch_bounds__(512)
   for (int j = 0; j < 8; ++j) o[j][0] = o[j][1] = o[j][2] = o[j][3] = 0.f;
   bool ok = true;
 
-  for (int i = 0; i < np; ++i) {
+  for (int i = 0; i < npl; ++i) {
     const int s = i % kAttnStages;
-    if (ok && !mbar_wait(smem_u32(&gfull[s]), (i / kAttnStages) & 1, a.err)) ok = false;
+    if (ok && !mbar_wait(smem_u32(&lfull[s]), (i / kAttnStages) & 1, a.err)) ok = false;
     if (ok && has_rows) {
       const uint32_t kbase = smem_u32(sK + s * kAttnPageBytes);
       const uint32_t vbase = smem_u32(sV + s * kAttnPageBytes);
@@ -268,7 +286,7 @@ __global__ void __launch_bounds__(512)
         }
       }
       // mask + online softmax (rows r0: elements 0,1; r1: elements 2,3)
-      const int kbase_abs = (p_begin + i) * 64;
+      const int kbase_abs = page_of(i) * 64;
       float mx0 = -INFINITY, mx1 = -INFINITY;
 #pragma unroll
       for (int j = 0; j < 8; ++j) {
@@ -325,9 +343,10 @@ __global__ void __launch_bounds__(512)
         }
       }
     }
-    group_sync(grp, gthreads);   // every warp of the group is done with stage s
-    if (producer && ok && i + kAttnStages < np) issue(i + kAttnStages);
+    lane_sync(ln, lthreads);   // every warp of the lane is done with stage s
+    if (producer && ok && i + kAttnStages < npl) issue(i + kAttnStages);
   }
+  const bool all_ok = __syncthreads_and(ok);   // both lanes done: the ring is idle
 
   // row sums across the quad
   l0 += __shfl_xor_sync(0xFFFFFFFFu, l0, 1);
@@ -335,8 +354,44 @@ __global__ void __launch_bounds__(512)
   l1 += __shfl_xor_sync(0xFFFFFFFFu, l1, 1);
   l1 += __shfl_xor_sync(0xFFFFFFFFu, l1, 2);
 
+  // ---- lane 1 -> lane 0 (shared memory): M = max, w = exp2(m - M) per lane,
+  //      O = w0 O0 + w1 O1, l = w0 l0 + w1 l1.  lp [row][kAttnRow] in the ring.
+  float* lp = reinterpret_cast<float*>(ring);
+  if (ln == 1 && has_rows) {
+#pragma unroll
+    for (int half = 0; half < 2; ++half) {
+      float* dst = lp + (half ? r1 : r0) * kAttnRow;
+#pragma unroll
+      for (int j = 0; j < 8; ++j)
+        *reinterpret_cast<float2*>(dst + 8 * j + 2 * tq) =
+            make_float2(o[j][half * 2 + 0], o[j][half * 2 + 1]);
+      if (tq == 0) *reinterpret_cast<float2*>(dst + 64) = half ? make_float2(m1, l1) : make_float2(m0, l0);
+    }
+  }
+  __syncthreads();
+  if (ln == 0 && has_rows) {
+#pragma unroll
+    for (int half = 0; half < 2; ++half) {
+      const float* src = lp + (half ? r1 : r0) * kAttnRow;
+      const float2 ml = *reinterpret_cast<const float2*>(src + 64);
+      const float ma = half ? m1 : m0;
+      const float M = fmaxf(ma, ml.x);
+      const float wa = (ma == -INFINITY) ? 0.f : exp2f(ma - M);
+      const float wb = (ml.x == -INFINITY) ? 0.f : exp2f(ml.x - M);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const float2 v = *reinterpret_cast<const float2*>(src + 8 * j + 2 * tq);
+        o[j][half * 2 + 0] = wa * o[j][half * 2 + 0] + wb * v.x;
+        o[j][half * 2 + 1] = wa * o[j][half * 2 + 1] + wb * v.y;
+      }
+      if (half) { l1 = wa * l1 + wb * ml.y; m1 = M; } else { l0 = wa * l0 + wb * ml.y; m0 = M; }
+    }
+  }
+  __syncthreads();   // lp consumed; the ring is reused below
+  const bool lead = ln == 0 && has_rows;
+
   if (nitems == 1) {   // the block's only item: its rows are final
-    if (has_rows && ok) {
+    if (lead && all_ok) {
 #pragma unroll
       for (int half = 0; half < 2; ++half) {
         const int r = half ? r1 : r0;
@@ -355,75 +410,150 @@ __global__ void __launch_bounds__(512)
     return;
   }
 
-  // ---- partial rows of this item -> global scratch
+  // Merged rows of one item: source `it`, row r -> float pointer (O[64], m, l).
+  // Cluster: recv[it][k] with r = c + k * nitems.  Global: part[b][h][it][r].
   const size_t bh = static_cast<size_t>(b) * a.Hkv + h;
-  float* part_bh = a.part + bh * a.max_items * a.r_pad * kAttnRow;
-  if (has_rows) {
+  float* part_bh = a.part + bh * a.max_items * rows_alloc * kAttnRow;
+  const int rpo = (rows_alloc + nitems - 1) / nitems;   // cluster: rows per owner
+  bool got = true;
+  int my_rows;
+  if (in_cluster) {
+    // ---- items -> owners.  stage [owner][slot][kAttnRow] in the ring.
+    float* stage = reinterpret_cast<float*>(ring);
+    const int blk_floats = rpo * kAttnRow;
+    if (lead) {
 #pragma unroll
-    for (int half = 0; half < 2; ++half) {
-      const int r = half ? r1 : r0;
-      if (r >= R) continue;
-      float* dst = part_bh + (static_cast<size_t>(item) * a.r_pad + r) * kAttnRow;
+      for (int half = 0; half < 2; ++half) {
+        const int r = half ? r1 : r0;
+        if (r >= R) continue;
+        float* dst = stage + static_cast<size_t>(r % nitems) * blk_floats + (r / nitems) * kAttnRow;
 #pragma unroll
-      for (int j = 0; j < 8; ++j)
-        *reinterpret_cast<float2*>(dst + 8 * j + 2 * tq) =
-            make_float2(o[j][half * 2 + 0], o[j][half * 2 + 1]);
-      if (tq == 0)
-        *reinterpret_cast<float2*>(dst + 64) = half ? make_float2(m1, l1) : make_float2(m0, l0);
+        for (int j = 0; j < 8; ++j)
+          *reinterpret_cast<float2*>(dst + 8 * j + 2 * tq) =
+              make_float2(o[j][half * 2 + 0], o[j][half * 2 + 1]);
+        if (tq == 0)
+          *reinterpret_cast<float2*>(dst + 64) = half ? make_float2(m1, l1) : make_float2(m0, l0);
+      }
+    }
+    fence_proxy_async_smem();
+    __syncthreads();
+    cluster_wait();   // every CTA of the cluster runs: peers' buffers and barriers exist
+    if (threadIdx.x == 0) {
+      const uint32_t bytes = static_cast<uint32_t>(blk_floats * 4);
+      const uint32_t dst_local = smem_u32(recv) + static_cast<uint32_t>(c) * bytes;
+      for (int q = 0; q < nitems; ++q)
+        bulk_copy_to_peer(cluster_map(dst_local, static_cast<uint32_t>(q)),
+                          smem_u32(stage) + static_cast<uint32_t>(q) * bytes, bytes,
+                          cluster_map(smem_u32(recv_bar), static_cast<uint32_t>(q)));
+      bulk_commit();
+    }
+    got = mbar_wait(smem_u32(recv_bar), 0, a.err);
+    my_rows = (R - c + nitems - 1) / nitems;
+  } else {
+    // ---- item rows -> global scratch; the last item to arrive merges
+    if (lead) {
+#pragma unroll
+      for (int half = 0; half < 2; ++half) {
+        const int r = half ? r1 : r0;
+        if (r >= R) continue;
+        float* dst = part_bh + (static_cast<size_t>(c) * rows_alloc + r) * kAttnRow;
+#pragma unroll
+        for (int j = 0; j < 8; ++j)
+          *reinterpret_cast<float2*>(dst + 8 * j + 2 * tq) =
+              make_float2(o[j][half * 2 + 0], o[j][half * 2 + 1]);
+        if (tq == 0)
+          *reinterpret_cast<float2*>(dst + 64) = half ? make_float2(m1, l1) : make_float2(m0, l0);
+      }
+    }
+    __threadfence();
+    __syncthreads();
+    if (threadIdx.x == 0) s_int[1] = (atomicAdd(a.ticket + bh, 1) == nitems - 1) ? 1 : 0;
+    __syncthreads();
+    if (!s_int[1]) return;
+    __threadfence();
+    if (threadIdx.x == 0) a.ticket[bh] = 0;   // every item of this launch has arrived
+    my_rows = R;
+  }
+  auto row_of = [&](int k) { return in_cluster ? c + k * nitems : k; };
+  // source rows: the owner's receive buffer (shared) or the global scratch
+  // (written by other SMs in this launch: read at L2, never from L1)
+  auto src_of = [&](int it, int k) -> const float* {
+    return in_cluster ? recv + (static_cast<size_t>(it) * rpo + k) * kAttnRow
+                      : part_bh + (static_cast<size_t>(it) * rows_alloc + k) * kAttnRow;
+  };
+  auto ld2 = [&](const float* p) {
+    return in_cluster ? *reinterpret_cast<const float2*>(p) : __ldcg(reinterpret_cast<const float2*>(p));
+  };
+  auto ld4 = [&](const float* p) {
+    return in_cluster ? *reinterpret_cast<const float4*>(p) : __ldcg(reinterpret_cast<const float4*>(p));
+  };
+
+  // ---- merge of items 0..nitems-1 in order for rows row_of(k), k < my_rows.
+  //      mb/lb [item][k] hold m and l, then mb the coefficients w_it / L (one
+  //      thread per row); then one thread per (row, 4 dims) sums coef * O_it.
+  //      Both live in the idle ring (in a cluster once this CTA's outgoing
+  //      copies have read it).
+  if (in_cluster && threadIdx.x == 0) bulk_wait_read_all();
+  __syncthreads();
+  float* mb = reinterpret_cast<float*>(ring);
+  float* lb = mb + static_cast<size_t>(nitems) * rows_alloc;
+  const bool fits = 2 * nitems * rows_alloc <= kAttnRingBytes / 4;
+  if (!fits && threadIdx.x == 0) atomicExch(a.err, kErrBounds);
+  if (fits) {
+    for (int idx = threadIdx.x; idx < nitems * my_rows; idx += blockDim.x) {
+      const int it = idx / my_rows, k = idx - it * my_rows;
+      const float2 ml = ld2(src_of(it, k) + 64);
+      mb[it * rows_alloc + k] = ml.x;
+      lb[it * rows_alloc + k] = ml.y;
     }
   }
-  __threadfence();
-  group_sync(grp, gthreads);
-  if (producer) s_int[1 + grp] = (atomicAdd(a.ticket + bh, 1) == nitems - 1) ? 1 : 0;
-  group_sync(grp, gthreads);
-  if (!s_int[1 + grp]) return;
-
-  // ---- last item of (block, head): merge items 0..nitems-1 in order.
-  //      coef[i][r] = w_i / L (one thread per row), then one thread per
-  //      (row, 4 dims) sums coef * O_i.
-  __threadfence();
-  float* coef = reinterpret_cast<float*>(sK);   // [nitems][rows_alloc], the group's idle ring
-  const bool fits = nitems <= attn_max_merge_items(a.QB * a.G);
-  if (!fits && gtid == 0) atomicExch(a.err, kErrBounds);
+  __syncthreads();
   if (fits) {
-    for (int r = gtid; r < R; r += gthreads) {
+    for (int k = threadIdx.x; k < my_rows; k += blockDim.x) {
       float M = -INFINITY;
-      for (int it = 0; it < nitems; ++it)
-        M = fmaxf(M, __ldcg(part_bh + (static_cast<size_t>(it) * a.r_pad + r) * kAttnRow + 64));
+      for (int it = 0; it < nitems; ++it) M = fmaxf(M, mb[it * rows_alloc + k]);
       float L = 0.f;
       for (int it = 0; it < nitems; ++it) {
-        const float2 ml = __ldcg(reinterpret_cast<const float2*>(
-            part_bh + (static_cast<size_t>(it) * a.r_pad + r) * kAttnRow + 64));
-        const float w = (ml.x == -INFINITY) ? 0.f : exp2f(ml.x - M);
-        coef[it * rows_alloc + r] = w;
-        L += w * ml.y;
+        const float mi = mb[it * rows_alloc + k];
+        const float w = (mi == -INFINITY) ? 0.f : exp2f(mi - M);
+        mb[it * rows_alloc + k] = w;
+        L += w * lb[it * rows_alloc + k];
       }
       const float inv = 1.0f / L;
-      for (int it = 0; it < nitems; ++it) coef[it * rows_alloc + r] *= inv;
+      for (int it = 0; it < nitems; ++it) mb[it * rows_alloc + k] *= inv;
     }
   }
-  group_sync(grp, gthreads);
+  __syncthreads();
   if (fits) {
-    for (int idx = gtid; idx < R * 16; idx += gthreads) {
-      const int r = idx >> 4, d4 = (idx & 15) * 4;
+    for (int idx = threadIdx.x; idx < my_rows * 16; idx += blockDim.x) {
+      const int k = idx >> 4, d4 = (idx & 15) * 4;
       float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-      for (int it = 0; it < nitems; ++it) {
-        const float w = coef[it * rows_alloc + r];
-        const float4 v = __ldcg(reinterpret_cast<const float4*>(
-            part_bh + (static_cast<size_t>(it) * a.r_pad + r) * kAttnRow + d4));
-        acc.x += w * v.x;
-        acc.y += w * v.y;
-        acc.z += w * v.z;
-        acc.w += w * v.w;
+      for (int it0 = 0; it0 < nitems; it0 += 8) {   // 8 loads in flight, summed in order
+        const int n8 = min(8, nitems - it0);
+        float4 v[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u)
+          if (u < n8) v[u] = ld4(src_of(it0 + u, k) + d4);
+#pragma unroll
+        for (int u = 0; u < 8; ++u)
+          if (u < n8) {
+            const float w = mb[(it0 + u) * rows_alloc + k];
+            acc.x += w * v[u].x;
+            acc.y += w * v[u].y;
+            acc.z += w * v[u].z;
+            acc.w += w * v[u].w;
+          }
       }
-      const int t = tok0 + r / a.G;
-      const int hq = h * a.G + r % a.G;
-      __half* dst = a.out + (static_cast<size_t>(t) * a.Hq + hq) * 64 + d4;
-      *reinterpret_cast<__half2*>(dst) = __floats2half2_rn(acc.x, acc.y);
-      *reinterpret_cast<__half2*>(dst + 2) = __floats2half2_rn(acc.z, acc.w);
+      if (all_ok && got) {
+        const int r = row_of(k);
+        const int t = tok0 + r / a.G;
+        const int hq = h * a.G + r % a.G;
+        __half* dst = a.out + (static_cast<size_t>(t) * a.Hq + hq) * 64 + d4;
+        *reinterpret_cast<__half2*>(dst) = __floats2half2_rn(acc.x, acc.y);
+        *reinterpret_cast<__half2*>(dst + 2) = __floats2half2_rn(acc.z, acc.w);
+      }
     }
   }
-  if (gtid == 0) a.ticket[bh] = 0;   // every item of this launch has arrived
 }
 
 }  // namespace gs

@@ -75,6 +75,24 @@ struct Carver {
 
 constexpr int kGemmCounters = 1 << 16;
 
+// Query blocks of a window of W tokens: at most kAttnMaxRows rows (QS tokens
+// of G rows) each, n_sub blocks per window, `rows` row slots per block.
+struct AttnGeom {
+  int QS, n_sub, rows;
+};
+AttnGeom attn_geom(int W, int G) {
+  const int qs = std::min(W, kAttnMaxRows / G);
+  return {qs, cdiv(W, qs), attn_mtiles(qs * G) * 16};
+}
+
+cudaError_t launch_attention(const CUtensorMap& tm, const AttnArgs& a, int n_blocks,
+                             cudaStream_t s, bool pdl) {
+  const int rows = attn_mtiles(a.QS * a.G) * 16;
+  dim3 grid(a.max_items, a.Hkv, n_blocks);
+  return launch_ex(attn_paged_kernel, grid, dim3(attn_threads(rows)), attn_smem_bytes(rows), s, pdl,
+                   dim3(a.cluster ? a.max_items : 1, 1, 1), tm, a);
+}
+
 struct GemmPlan {
   int bn, tok_tiles, feat_tiles, splits;
 };
@@ -258,27 +276,22 @@ size_t carve(gs_handle* h, const gs_config& c, void* base) {
   const int W_max = c.max_K + 1;
   int T_max = std::max(c.max_batch * W_max, c.max_prefill);
   T_max = static_cast<int>(align_up(std::max(T_max, 256), 256));
-  // attention work items (fixed absolute page ranges).  Decode: about 16
-  // items per SM over a full batch at full context, at least 2 pages each;
-  // prefill: 8 pages or more.  Either way the last item's merge keeps one
-  // coefficient per (item, row) in shared memory.
+  // attention work items (fixed absolute page ranges).  Decode: at most 8
+  // items per sequence (one cluster) unless the config asks for smaller
+  // items; prefill: at least 8 pages per item, at most 8 items.
   const int r_max = round16(W_max * G);
-  const int qb_pf = std::max(1, 128 / G);
-  const int r_pf = round16(qb_pf * G);
-  int sp = c.split_pages;
-  if (sp <= 0)
-    sp = std::min(32, std::max(2, cdiv(static_cast<long long>(pt_stride) * c.max_batch * c.n_kv_heads,
-                                       152 * 16)));
-  sp = std::max(sp, cdiv(pt_stride, attn_max_merge_items(r_max)));
+  const AttnGeom g_dec = attn_geom(W_max, G);
+  const int qb_pf = std::max(1, kAttnMaxRows / G);
+  int sp = c.split_pages > 0 ? c.split_pages : std::max(2, cdiv(pt_stride, kAttnMaxCluster));
+  sp = std::max(sp, cdiv(pt_stride, attn_max_merge_items(g_dec.rows)));
   const int items_dec = cdiv(pt_stride, sp);
-  const int sp_pf = std::max(8, cdiv(pt_stride, attn_max_merge_items(r_pf)));
+  const int sp_pf = std::max(8, cdiv(pt_stride, kAttnMaxCluster));
   const int items_pf = cdiv(pt_stride, sp_pf);
-  const int chunk = std::min(c.max_prefill, T_max);
-  const int blocks_pf = cdiv(chunk, qb_pf);
+  const size_t attn_blocks = static_cast<size_t>(c.max_batch) * g_dec.n_sub;
   const size_t attn_part_floats =
-      std::max(static_cast<size_t>(c.max_batch) * c.n_kv_heads * items_dec * r_max,
-               static_cast<size_t>(blocks_pf) * c.n_kv_heads * items_pf * r_pf) * kAttnRow;
-
+      items_dec > kAttnMaxCluster
+          ? attn_blocks * c.n_kv_heads * items_dec * g_dec.rows * kAttnRow
+          : 0;
   int* err_word = cv.take<int>(64);
   SeqStateDev st;
   st.seq_len = cv.take<int32_t>(c.max_batch);
@@ -312,7 +325,7 @@ size_t carve(gs_handle* h, const gs_config& c, void* base) {
   float* gemm_partial = cv.take<float>(partial_floats);
   int* gemm_counters = cv.take<int>(kGemmCounters);
   float* attn_part = cv.take<float>(attn_part_floats);
-  int* attn_ticket = cv.take<int>(static_cast<size_t>(std::max(c.max_batch, blocks_pf)) * c.n_kv_heads);
+  int* attn_ticket = cv.take<int>(attn_blocks * c.n_kv_heads);
   // fp16 weight copies: per layer qkv | o | gate_up | down, then the LM head
   const size_t per_layer = static_cast<size_t>(qkv_dim) * c.d_model +
                            static_cast<size_t>(c.d_model) * c.n_heads * 64 +
@@ -401,7 +414,7 @@ int run_gemm(gs_handle* h, const CUtensorMap& tw, int weight_rows, const CUtenso
 }
 
 struct AttnLaunch {
-  int n_blocks, QB, split_pages, max_items, r_max;
+  int n_seq, QB, split_pages, max_items;
   const int32_t* blk_slot;
   const int32_t* blk_active;
   int fixed_slot;
@@ -409,6 +422,7 @@ struct AttnLaunch {
 
 int run_attention(gs_handle* h, int layer, int T, const AttnLaunch& L) {
   const gs_config& c = h->cfg;
+  const AttnGeom g = attn_geom(L.QB, h->G);
   AttnArgs a;
   a.q = h->qr;
   a.lim = h->lim;
@@ -420,6 +434,8 @@ int run_attention(gs_handle* h, int layer, int T, const AttnLaunch& L) {
   a.fixed_slot = L.fixed_slot;
   a.T = T;
   a.QB = L.QB;
+  a.QS = g.QS;
+  a.n_sub = g.n_sub;
   a.Hq = c.n_heads;
   a.Hkv = c.n_kv_heads;
   a.G = h->G;
@@ -427,18 +443,17 @@ int run_attention(gs_handle* h, int layer, int T, const AttnLaunch& L) {
   a.kv_row_base = static_cast<long long>(layer) * h->n_pages * a.rows_per_page;
   a.split_pages = L.split_pages;
   a.max_items = L.max_items;
-  a.r_pad = L.r_max;
+  a.cluster = L.max_items <= kAttnMaxCluster ? 1 : 0;
   a.part = h->attn_part;
   a.ticket = h->attn_ticket;
   a.err = h->err_word;
-  if (static_cast<size_t>(L.n_blocks) * c.n_kv_heads * L.max_items * L.r_max * kAttnRow >
-          h->attn_part_floats ||
-      L.max_items > attn_max_merge_items(L.r_max))
+  const int n_blocks = L.n_seq * g.n_sub;
+  if (!a.cluster &&
+      (static_cast<size_t>(n_blocks) * c.n_kv_heads * L.max_items * g.rows * kAttnRow >
+           h->attn_part_floats ||
+       L.max_items > attn_max_merge_items(g.rows)))
     return fail(h, GS_ERR_OOM, "attention item scratch too small");
-  const int ng = attn_groups_for(L.r_max, L.max_items * c.n_kv_heads * L.n_blocks);
-  dim3 grid(cdiv(L.max_items, ng), c.n_kv_heads, L.n_blocks);
-  GS_CUDA(h, launch_ex(attn_paged_kernel, grid, dim3(attn_threads(L.r_max, ng)),
-                       attn_smem_bytes(L.r_max, ng), h->stream, true, dim3(1, 1, 1), h->tm_kv, a));
+  GS_CUDA(h, launch_attention(h->tm_kv, a, n_blocks, h->stream, true));
   note_launch(h, GS_KIND_ATTENTION);
   return GS_OK;
 }
@@ -555,11 +570,10 @@ int enqueue_round(gs_handle* h, const int32_t* slots, int n_seq, int K, const gs
   w.err = h->err_word;
   const int nb = cdiv(T, 128);
   AttnLaunch AL;
-  AL.n_blocks = n_seq;
+  AL.n_seq = n_seq;
   AL.QB = W;
   AL.split_pages = h->split_pages;
   AL.max_items = h->items_dec;
-  AL.r_max = round16(W * h->G);
   AL.blk_slot = h->blk_slot;
   AL.blk_active = h->blk_active;
   AL.fixed_slot = -1;
@@ -840,10 +854,9 @@ int gs_prefill(gs_handle* h, int slot, const void* vis_emb, int n_vis, const int
     GS_CUDA(h, cudaGetLastError());
     AttnLaunch AL;
     AL.QB = h->qb_pf;
-    AL.n_blocks = cdiv(T, h->qb_pf);
+    AL.n_seq = cdiv(T, h->qb_pf);   // prefill blocks (one per QB tokens)
     AL.split_pages = h->split_pages_pf;
     AL.max_items = h->items_pf;
-    AL.r_max = round16(h->qb_pf * h->G);
     AL.blk_slot = nullptr;
     AL.blk_active = nullptr;
     AL.fixed_slot = slot;
@@ -996,14 +1009,16 @@ size_t gs_attention_scratch_bytes(int n_seq, int W, int n_heads, int n_kv_heads,
   if (n_seq < 1 || W < 1 || n_kv_heads < 1 || n_heads % n_kv_heads || max_pages < 1 ||
       split_pages < 1)
     return 0;
-  const int r_max = round16(W * (n_heads / n_kv_heads));
+  const AttnGeom g = attn_geom(W, n_heads / n_kv_heads);
   const int items = cdiv(max_pages, split_pages);
+  const size_t blocks = static_cast<size_t>(n_seq) * g.n_sub;
   Carver cv(nullptr);
   cv.take<int>(64);                                   // error word
   cv.take<int32_t>(static_cast<size_t>(n_seq) * W);  // key limits
-  cv.take<int32_t>(n_seq);                            // block -> page-table row
-  cv.take<int>(static_cast<size_t>(n_seq) * n_kv_heads);  // merge tickets
-  cv.take<float>(static_cast<size_t>(n_seq) * n_kv_heads * items * r_max * kAttnRow);  // items
+  cv.take<int32_t>(n_seq);                            // sequence -> page-table row
+  cv.take<int>(blocks * n_kv_heads);                  // merge tickets
+  if (items > kAttnMaxCluster)                        // item rows of the global merge
+    cv.take<float>(blocks * n_kv_heads * items * g.rows * kAttnRow);
   return align_up(cv.off, 256);
 }
 
@@ -1032,7 +1047,7 @@ int gs_attention(int mode, const void* q, const void* kv, int n_pages, const int
   if (n_kv_heads < 1 || n_heads % n_kv_heads || W < 1 || n_seq < 1 || split_pages < 1)
     return GS_ERR_INVALID_ARG;
   const int G = n_heads / n_kv_heads;
-  if (W * G > 256) return GS_ERR_UNSUPPORTED;
+  if (G > kAttnMaxRows) return GS_ERR_UNSUPPORTED;
   if (scratch_bytes < gs_attention_scratch_bytes(n_seq, W, n_heads, n_kv_heads, pt_stride, split_pages))
     return GS_ERR_OOM;
   if ((reinterpret_cast<uintptr_t>(kv) & 15) || (reinterpret_cast<uintptr_t>(q) & 15))
@@ -1044,22 +1059,24 @@ int gs_attention(int mode, const void* q, const void* kv, int n_pages, const int
       return GS_ERR_CUDA;
     attr = true;
   }
-  const int r_max = round16(W * G);
+  const AttnGeom g = attn_geom(W, G);
   const int items = cdiv(pt_stride, split_pages);
-  if (items > attn_max_merge_items(r_max)) return GS_ERR_UNSUPPORTED;
+  if (items > attn_max_merge_items(g.rows)) return GS_ERR_UNSUPPORTED;
+  const size_t blocks = static_cast<size_t>(n_seq) * g.n_sub;
   Carver cv(scratch);
   int* err = cv.take<int>(64);
   int32_t* lim = cv.take<int32_t>(static_cast<size_t>(n_seq) * W);
   int32_t* blk_slot = cv.take<int32_t>(n_seq);
-  int* ticket = cv.take<int>(static_cast<size_t>(n_seq) * n_kv_heads);
-  float* part = cv.take<float>(static_cast<size_t>(n_seq) * n_kv_heads * items * r_max * kAttnRow);
+  int* ticket = cv.take<int>(blocks * n_kv_heads);
+  float* part = items > kAttnMaxCluster
+                    ? cv.take<float>(blocks * n_kv_heads * items * g.rows * kAttnRow)
+                    : nullptr;
   CUtensorMap tm;
   const uint64_t rows = static_cast<uint64_t>(n_pages) * 2 * n_kv_heads * 64;
   if (rows >= (1ull << 31) || !make_map(&tm, kv, rows, 64, 64)) return GS_ERR_INVALID_ARG;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   // the merge tickets start at zero (the kernel leaves them at zero)
-  if (cudaMemsetAsync(ticket, 0, static_cast<size_t>(n_seq) * n_kv_heads * sizeof(int), s) !=
-      cudaSuccess)
+  if (cudaMemsetAsync(ticket, 0, blocks * n_kv_heads * sizeof(int), s) != cudaSuccess)
     return GS_ERR_CUDA;
   attn_standalone_prep<<<cdiv(n_seq * W, 128), 128, 0, s>>>(mode, n, n_seq, W, lim, blk_slot);
   AttnArgs a;
@@ -1073,6 +1090,8 @@ int gs_attention(int mode, const void* q, const void* kv, int n_pages, const int
   a.fixed_slot = -1;
   a.T = n_seq * W;
   a.QB = W;
+  a.QS = g.QS;
+  a.n_sub = g.n_sub;
   a.Hq = n_heads;
   a.Hkv = n_kv_heads;
   a.G = G;
@@ -1080,16 +1099,12 @@ int gs_attention(int mode, const void* q, const void* kv, int n_pages, const int
   a.kv_row_base = 0;
   a.split_pages = split_pages;
   a.max_items = items;
-  a.r_pad = r_max;
+  a.cluster = items <= kAttnMaxCluster ? 1 : 0;
   a.part = part;
   a.ticket = ticket;
   a.err = err;
-  const int ng = attn_groups_for(r_max, items * n_kv_heads * n_seq);
-  dim3 grid(cdiv(items, ng), n_kv_heads, n_seq);
-  return launch_ex(attn_paged_kernel, grid, dim3(attn_threads(r_max, ng)),
-                   attn_smem_bytes(r_max, ng), s, false, dim3(1, 1, 1), tm, a) == cudaSuccess
-             ? GS_OK
-             : GS_ERR_CUDA;
+  return launch_attention(tm, a, static_cast<int>(blocks), s, false) == cudaSuccess ? GS_OK
+                                                                                   : GS_ERR_CUDA;
 }
 
 size_t gs_linear_scratch_bytes(int M, int N, int split_k) {

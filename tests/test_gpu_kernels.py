@@ -197,7 +197,7 @@ def test_attention_sweep_sizes_sampled(gs, B, prefix, K):
     ctx = prefix + W + 1
     q, k, v = synth.attn_inputs(B, W, ctx, Hq, Hkv, index=B)
     pool, pt, _ = _paged(k, v, rng)
-    sp = min(32, max(2, math.ceil(pt.shape[1] * B * Hkv / (152 * 16))))
+    sp = max(2, math.ceil(pt.shape[1] / 8))   # the engine's default: at most 8 items
     for mode in (0, 1):
         got = _run_attention(gs, mode, q, pool, pt, np.array(ns), W, Hq, Hkv, sp)
         for b in sorted(set([0, B - 1] + list(rng.integers(0, B, 2)))):
@@ -206,3 +206,23 @@ def test_attention_sweep_sizes_sampled(gs, B, prefix, K):
             want = _oracle_attn(q[b].astype(np.float64), k[b, :nk].astype(np.float64),
                                 v[b, :nk].astype(np.float64), allowed, Hq, Hkv)
             np.testing.assert_allclose(got[b], want, rtol=5e-3, atol=5e-3)
+
+
+@pytest.mark.parametrize("sp", [3, 1])
+def test_attention_rows_do_not_depend_on_window(gs, sp):
+    """Verify mode: the rows of a 17-token window and the first 17 rows of a
+    33- and a 65-token window (two query blocks of 128 rows) over the same
+    cache have the same limits and queries, so the same bits -- with the
+    items merged in a cluster (sp = 3: at most 8 items) or through global
+    scratch (sp = 1: 11 items)."""
+    Hq, Hkv, n = 16, 8, 620
+    rng = np.random.default_rng(3)
+    q, k, v = synth.attn_inputs(1, 65, n + 67, Hq, Hkv, index=77)
+    pool, pt, _ = _paged(k, v, rng)
+    outs = {}
+    for W in (17, 33, 65):
+        outs[W] = _run_attention(gs, 1, np.ascontiguousarray(q[:, :W]), pool, pt, np.array([n]), W,
+                                 Hq, Hkv, sp)
+    assert np.array_equal(outs[33][:, :17], outs[17])
+    assert np.array_equal(outs[65][:, :17], outs[17])
+    assert np.array_equal(outs[65][:, :33], outs[33])
