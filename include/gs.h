@@ -241,7 +241,8 @@ int gs_sync_check(gs_handle *h);
  *                  row 0 sees keys 0..n_s, rows i >= 1 see keys 0..n_s + W - 1
  *   mode 1 VERIFY: query row i sits at slot n_s + 1 + i and sees keys 0..n_s + 1 + i
  *   q        device fp16 [n_seq, W, n_heads, 64] (RoPE already applied)
- *   kv       device fp16 page pool [n_pages][2 (K,V)][n_kv_heads][64 tokens][64]
+ *   kv       device fp16 page pool [n_pages][2][n_kv_heads][64][64]: per page and
+ *            KV head, K as [64 tokens][64 dims] and V transposed, [64 dims][64 tokens]
  *   page_table device int32 [n_seq, pt_stride]: logical page -> physical page
  *   n        device int32 [n_seq]: n_s
  *   out      device fp16 [n_seq, W, n_heads, 64]
@@ -252,8 +253,8 @@ int gs_sync_check(gs_handle *h);
  *            logical pages [i * split_pages, (i + 1) * split_pages); items are
  *            reduced independently and merged in item order, so results depend
  *            on split_pages but not on n_seq, W or the other sequences.
- *            GS_ERR_UNSUPPORTED if ceil(pt_stride / split_pages) items exceed
- *            what the merge holds (12288 / (16 * ceil(W * G / 16))).
+ *            GS_ERR_UNSUPPORTED if ceil(pt_stride / split_pages) > 96 (the
+ *            merge's limit).
  *   stream   cudaStream_t */
 size_t gs_attention_scratch_bytes(int n_seq, int W, int n_heads, int n_kv_heads, int max_pages,
                                   int split_pages);

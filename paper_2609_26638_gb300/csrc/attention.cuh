@@ -1,50 +1,68 @@
-// attention.cuh -- hybrid-mask attention over the paged fp16 KV cache.
+// attention.cuh -- hybrid-mask attention over the paged fp16 KV cache, on
+// the tcgen05 tensor cores.
 //
-// A query block is a run of at most kAttnMaxRows / G tokens of one sequence
-// (a decode window, cut into sub-blocks when K+1 tokens carry more than 128
-// rows, or a slice of a prefill chunk); its rows are (token, query head of the
-// GQA group), so the query heads that share a KV head read each K/V page once.
+// A query block is a run of at most 128 / G tokens of one sequence (a decode
+// window, cut into sub-blocks when K+1 tokens carry more than 128 rows, or a
+// slice of a prefill chunk); its rows are (token, query head of the GQA
+// group), so the query heads that share a KV head read each K/V page once.
 // Every query token carries its own inclusive key limit, which encodes the
 // mask: draft boundary row n, draft mask rows n+K, verify row i n+1+i, prefill
 // row p (paper Appendix steps Draft forward / Verify forward).
 //
 // Work items.  The block's pages are cut into fixed absolute ranges of SP
 // pages ("items"): item i covers pages [i*SP, (i+1)*SP); one CTA reduces one
-// item.  Inside an item the pages are dealt to two lanes by parity (lane l
-// takes the item's pages l, l+2, ...); each lane is a warp group (one warp per
-// 16 rows) with its own ring of TMA stages (K and V pages, 64 tokens x 64
-// dims, 8 KB each, 128-byte swizzle).  Each warp runs S = Q K^T and O += P V
-// on mma.sync m16n8k16 (fp16 in, fp32 out) with the online softmax in
-// registers (exp2, the 1/sqrt(64) scale folded), its lane's pages in order.
-// The two lanes' (O, m, l) then merge in shared memory, lane 0 first.
+// item, pages in order.  A page holds K as [64 tokens][64 dims] and V
+// transposed, [64 dims][64 tokens] (8 KB each), so both are K-major operands.
+// Per page j:
+//   S_j = Q K_j^T      tcgen05.mma M=128 (rows) N=64 (keys) K=64, into TMEM
+//   softmax            one thread per row: m, l, p = exp2(s*scale - m) (fp32),
+//                      P_j (fp16) into shared memory as the next A operand
+//   PV_j = P_j V_j     tcgen05.mma M=128 N=64 (dims) K=64 (keys), into TMEM
+//   O = alpha_j O + PV_j  in the row's registers
+// Warps 0-3 own rows 0-127 (TMEM lanes); warp 4 streams K/V pages by TMA
+// (128-byte swizzle) through a ring of stages; warp 5 issues the MMAs, one
+// page of S ahead of the softmax, with S and PV double-buffered in TMEM.
 //
 // Merge over items, item order 0, 1, ...: M = max m_i, w_i = exp2(m_i - M),
 // coef_i = w_i / sum_j w_j l_j, O = sum coef_i O_i.  A block with one item
-// writes its rows directly.  With at most 8 items the items of a (block, head)
-// form one thread-block cluster: each CTA sends the rows that CTA (r mod n)
-// owns to it with one bulk async copy into its shared memory, completing on
-// its mbarrier, and each owner merges its rows.  With more items every item
-// writes its rows to global scratch and the last one to finish (atomic ticket
-// per (block, head), no spinning) merges them.  Both paths run the same
-// arithmetic in the same order.
+// writes its rows directly.  A (block, head) with at most 8 items may form one
+// thread-block cluster: each CTA sends the rows that CTA (r mod n) owns to it
+// with one bulk async copy into its shared memory, completing on its
+// mbarrier, and each owner merges its rows.  Otherwise every item writes its
+// rows to global scratch and the last one to finish (atomic ticket per (block,
+// head), no spinning) merges them.  Both paths run the same arithmetic in the
+// same order.
 //
-// Invariance.  Item boundaries are absolute page numbers fixed by SP, the
-// lanes deal pages by parity, and the merges run in fixed order, so a row's
-// result depends only on its query, keys, limit and SP: not on the other rows
-// of its block, the window size, the batch, or the merge path.  Keys past a
-// row's limit contribute exact zeros.
+// Invariance.  Item boundaries are absolute page numbers fixed by SP, pages
+// are reduced in order, the MMA's arithmetic for a row does not depend on the
+// other rows, and the merges run in fixed order, so a row's result depends
+// only on its query, keys, limit and SP: not on the other rows of its block,
+// the window size, the batch, or the merge path.  Keys past a row's limit
+// contribute exact zeros.
 #pragma once
 #include "ptx.cuh"
 
 namespace gs {
 
-constexpr int kAttnStages = 2;             // K/V pages in flight per lane
-constexpr int kAttnLanes = 2;
-constexpr int kAttnPageBytes = 64 * 128;  // 64 tokens x 64 fp16
+constexpr int kAttnStages = 6;             // K/V page pairs in flight
+constexpr int kAttnPageBytes = 64 * 128;  // 64 x 64 fp16
+constexpr int kAttnStageBytes = 2 * kAttnPageBytes;
 constexpr int kAttnRow = 68;              // partial row: O[64], m, l, 2 pad (272 B)
-constexpr int kAttnMaxRows = 128;         // rows of one query block
+constexpr int kAttnMaxRows = 128;         // rows of one query block (the MMA's M)
 constexpr int kAttnMaxCluster = 8;        // items merged inside a cluster
-constexpr int kAttnRingBytes = kAttnLanes * kAttnStages * 2 * kAttnPageBytes;
+constexpr int kAttnThreads = 192;         // 4 softmax warps, TMA warp, MMA warp
+constexpr int kAttnTmemCols = 256;        // S[2] at 0, 64; PV[2] at 128, 192
+constexpr int kAttnRingBytes = kAttnStages * kAttnStageBytes;
+// Q [128][128 B] | ring | P[2] [128][128 B] | receive buffer | barriers
+constexpr int kAttnQOff = 0;
+constexpr int kAttnRingOff = kAttnMaxRows * 128;
+constexpr int kAttnPOff = kAttnRingOff + kAttnRingBytes;
+constexpr int kAttnRecvOff = kAttnPOff + 2 * kAttnMaxRows * 128;
+constexpr int kAttnRecvFloats = (kAttnMaxRows + kAttnMaxCluster) * kAttnRow;
+constexpr int kAttnBarOff = kAttnRecvOff + kAttnRecvFloats * 4;
+constexpr int kAttnSmemBytes = 1024 + kAttnBarOff + 256;
+static_assert(kAttnRingBytes >= (kAttnMaxRows + kAttnMaxCluster) * kAttnRow * 4,
+              "the idle ring holds the owner-grouped rows");
 
 struct AttnArgs {
   const __half* q;            // [T, Hq, 64]
@@ -64,88 +82,63 @@ struct AttnArgs {
   int split_pages;            // SP: pages per item
   int max_items;              // items per (block, head) the grid covers
   int cluster;                // 1: the grid's x dimension is one cluster (max_items <= 8)
-  float* part;                // global merge: [n_blocks][Hkv][max_items][rows][kAttnRow]
+  float* part;                // global merge: [n_blocks][Hkv][max_items][128][kAttnRow]
   int* ticket;                // global merge: [n_blocks][Hkv], zero between launches
   int* err;
 };
 
 __host__ __device__ inline int attn_mtiles(int rows) { return (rows + 15) / 16; }
-__host__ __device__ inline int attn_threads(int rows) {
-  return kAttnLanes * attn_mtiles(rows) * 32;
+__host__ __device__ inline int attn_max_smem_bytes() { return kAttnSmemBytes; }
+// The global merge keeps m and l of every (item, row) in the idle ring.
+__host__ __device__ inline int attn_max_merge_items(int /*rows*/) {
+  return kAttnRingBytes / 4 / (2 * kAttnMaxRows);
 }
-// receive buffer of an owner: n sources x ceil(rows / n) rows, at most rows + 8
-__host__ __device__ inline int attn_recv_floats(int rows) {
-  return (attn_mtiles(rows) * 16 + kAttnMaxCluster) * kAttnRow;
-}
-__host__ __device__ inline int attn_smem_bytes(int rows) {
-  return 1024 + attn_mtiles(rows) * 16 * 128 + kAttnRingBytes + attn_recv_floats(rows) * 4 + 128;
-}
-__host__ __device__ inline int attn_max_smem_bytes() { return attn_smem_bytes(kAttnMaxRows); }
-// The merge keeps m and l of every (item, row) in the idle ring.
-__host__ __device__ inline int attn_max_merge_items(int rows) {
-  return kAttnRingBytes / 4 / (2 * attn_mtiles(rows) * 16);
-}
-static_assert(kAttnRingBytes >= kAttnMaxRows * kAttnRow * 4 &&
-                  kAttnRingBytes >= (kAttnMaxRows + kAttnMaxCluster) * kAttnRow * 4,
-              "the idle ring holds a lane's partial rows and the owner-grouped rows");
 
 __device__ __forceinline__ uint32_t sw128(int row, int chunk) {
   return static_cast<uint32_t>(row * 128 + ((chunk ^ (row & 7)) << 4));
 }
 
-__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
-                                        uint32_t& r3) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
-               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
-               : "r"(addr));
-}
-
-__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
-                                          uint32_t& r3) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
-               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
-               : "r"(addr));
-}
-
-__device__ __forceinline__ void mma_f16_16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0,
-                                              uint32_t b1) {
+// 32 lanes x 32 fp32 columns without the wait (issue several, then tmem_wait_ld).
+__device__ __forceinline__ void tmem_ld32_nowait(uint32_t taddr, uint32_t (&r)[32]) {
   asm volatile(
-      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, "
-      "{%8, %9}, {%0, %1, %2, %3};"
-      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
-      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
+      "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]),
+        "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]),
+        "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+}
+__device__ __forceinline__ void tmem_wait_ld() {
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
 
-__device__ __forceinline__ uint32_t pack_f16x2(float lo, float hi) {
-  __half2 v = __floats2half2_rn(lo, hi);
-  return *reinterpret_cast<uint32_t*>(&v);
-}
-
-// Barrier over the warps of one lane (ids 1, 2; 0 is __syncthreads).
-__device__ __forceinline__ void lane_sync(int lane_id, int nthreads) {
-  asm volatile("bar.sync %0, %1;" ::"r"(lane_id + 1), "r"(nthreads) : "memory");
-}
-
-__global__ void __launch_bounds__(512)
+__global__ void __launch_bounds__(kAttnThreads, 1)
     attn_paged_kernel(const __grid_constant__ CUtensorMap tmKV, const AttnArgs a) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int mtiles = attn_mtiles(a.QS * a.G);
-  const int ln = warp / mtiles, mt = warp % mtiles;   // page lane, row tile
-  const int lthreads = mtiles * 32;
-  const int ltid = threadIdx.x - ln * lthreads;
-  const int rows_alloc = mtiles * 16;
-  uint8_t* sQ = smem;                                   // [rows][128 B]
-  uint8_t* ring = smem + rows_alloc * 128;              // [lane][stage][K | V]
-  uint8_t* sK = ring + ln * kAttnStages * 2 * kAttnPageBytes;
-  uint8_t* sV = sK + kAttnStages * kAttnPageBytes;
-  float* recv = reinterpret_cast<float*>(ring + kAttnRingBytes);   // [source][slot][kAttnRow]
-  uint64_t* full = reinterpret_cast<uint64_t*>(recv + attn_recv_floats(rows_alloc));
-  uint64_t* lfull = full + ln * kAttnStages;
-  uint64_t* recv_bar = full + kAttnLanes * kAttnStages;
-  int* s_int = reinterpret_cast<int*>(recv_bar + 1);    // [0] max limit, [1] last-item flag
+  constexpr int rows_alloc = kAttnMaxRows;
+  uint8_t* sQ = smem + kAttnQOff;
+  uint8_t* ring = smem + kAttnRingOff;                   // [stage][K | V^T]
+  uint8_t* sP = smem + kAttnPOff;                        // [2][128][128 B]
+  float* recv = reinterpret_cast<float*>(smem + kAttnRecvOff);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kAttnBarOff);
+  uint64_t* full = bars;                                 // [stages] TMA landed
+  uint64_t* empty = bars + kAttnStages;                  // [stages] PV of the page done
+  uint64_t* s_full = bars + 2 * kAttnStages;             // [2] S in TMEM
+  uint64_t* s_free = s_full + 2;                         // [2] S read by all 128 threads
+  uint64_t* p_full = s_full + 4;                         // [2] P in smem (128 arrivals)
+  uint64_t* pv_full = s_full + 6;                        // [2] PV in TMEM
+  uint64_t* mma_done = s_full + 8;                       // every MMA of this CTA retired
+  uint64_t* recv_bar = s_full + 9;
+  uint64_t* q_full = s_full + 10;                        // Q tile in smem (128 arrivals)
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(s_full + 11);
+  // [0] max limit, [1] last-item flag, [2] pages the MMA warp took, [3] pages issued
+  int* s_int = reinterpret_cast<int*>(s_full + 12);
 
   const int c = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
   const int seq = b / a.n_sub, sub = b % a.n_sub;
@@ -173,7 +166,8 @@ __global__ void __launch_bounds__(512)
   const int npages_blk = maxlim / 64 + 1;
   const int SP = a.split_pages;
   const int nitems = (npages_blk + SP - 1) / SP;
-  if (maxlim < 0 || npages_blk > a.pt_stride || slot < 0 || nitems > a.max_items) {
+  if (maxlim < 0 || npages_blk > a.pt_stride || slot < 0 || nitems > a.max_items ||
+      R > kAttnMaxRows) {
     if (threadIdx.x == 0) atomicExch(a.err, kErrBounds);
     return;
   }
@@ -182,233 +176,265 @@ __global__ void __launch_bounds__(512)
 
   if (threadIdx.x == 0) {
     tma_prefetch_desc(&tmKV);
-    for (int s = 0; s < kAttnLanes * kAttnStages; ++s) mbar_init(smem_u32(&full[s]), 1);
+    for (int s = 0; s < kAttnStages; ++s) {
+      mbar_init(smem_u32(&full[s]), 1);
+      mbar_init(smem_u32(&empty[s]), 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(smem_u32(&s_full[i]), 1);
+      mbar_init(smem_u32(&s_free[i]), 128);
+      mbar_init(smem_u32(&p_full[i]), 128);
+      mbar_init(smem_u32(&pv_full[i]), 1);
+    }
+    mbar_init(smem_u32(mma_done), 1);
+    mbar_init(smem_u32(q_full), 128);
     if (in_cluster) {
       mbar_init(smem_u32(recv_bar), 1);
-      // nitems sources, ceil(rows / nitems) rows each, arrive by bulk copy
+      // nitems sources, ceil(128 / nitems) rows each, arrive by bulk copy
       const int rpo = (rows_alloc + nitems - 1) / nitems;
       mbar_arrive_expect_tx(smem_u32(recv_bar), static_cast<uint32_t>(nitems * rpo * kAttnRow * 4));
     }
+    s_int[2] = 0;
+    s_int[3] = 0;
     fence_mbar_init();
   }
+  if (in_cluster) {
+    __syncthreads();
+    cluster_arrive_release();   // waited on before the first remote access
+    if (c >= nitems) return;    // idle cluster member: arrived, owns nothing
+  }
+  if (warp == 5) tmem_alloc(smem_u32(tmem_slot), kAttnTmemCols);
+  tc_fence_before();
   __syncthreads();
-  if (in_cluster) cluster_arrive_release();   // waited on before the first remote access
-  if (c >= nitems) return;                     // idle cluster member: arrived, owns nothing
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
 
   const int p_begin = c * SP;
   const int np = min(npages_blk, p_begin + SP) - p_begin;
-  const int npl = np > ln ? (np - ln + 1) / kAttnLanes : 0;   // this lane's pages
   const int32_t* pt = a.page_table + static_cast<size_t>(slot) * a.pt_stride;
-  const bool producer = ltid == 0;
-  // pages wholly before the block's first slot hold committed states only
-  const int safe_pages = a.blk_slot ? a.lim[tok0] / 64 : 0;
-  const uint64_t pol = l2_policy_evict_first();
-  auto page_of = [&](int i) { return p_begin + ln + kAttnLanes * i; };
-  auto issue = [&](int i) {
-    const int s = i % kAttnStages;
-    int phys = pt[page_of(i)];
-    if (phys < 0) {  // unmapped page: the TMA box lands out of bounds and reads zeros
-      atomicExch(a.err, kErrBounds);
-      phys = 0x3FFFFFFF / a.rows_per_page;
-    }
-    const long long row = a.kv_row_base + static_cast<long long>(phys) * a.rows_per_page;
-    const uint32_t fb = smem_u32(&lfull[s]);
-    mbar_arrive_expect_tx(fb, 2 * kAttnPageBytes);
-    tma_load_2d(smem_u32(sK + s * kAttnPageBytes), &tmKV, 0, static_cast<int>(row + h * 64), fb, pol);
-    tma_load_2d(smem_u32(sV + s * kAttnPageBytes), &tmKV, 0,
-                static_cast<int>(row + (a.Hkv + h) * 64), fb, pol);
-  };
-  int issued = 0;
-  if (producer) {
-    while (issued < min(npl, kAttnStages) && page_of(issued) < safe_pages) issue(issued++);
-  }
-  pdl_wait();
-  pdl_trigger();
-  if (producer) {
-    while (issued < min(npl, kAttnStages)) issue(issued++);
-  }
-
-  // Q rows -> swizzled smem (zero rows past R)
-  for (int idx = threadIdx.x; idx < rows_alloc * 8; idx += blockDim.x) {
-    const int r = idx >> 3, ch = idx & 7;
-    uint4 v = make_uint4(0, 0, 0, 0);
-    if (r < R) {
-      const int t = tok0 + r / a.G;
-      const int hq = h * a.G + r % a.G;
-      v = *reinterpret_cast<const uint4*>(a.q + (static_cast<size_t>(t) * a.Hq + hq) * 64 + ch * 8);
-    }
-    *reinterpret_cast<uint4*>(sQ + sw128(r, ch)) = v;
-  }
-  __syncthreads();
-
-  const bool has_rows = mt * 16 < R;
-  const int g = lane >> 2, tq = lane & 3;
-  const int r0 = mt * 16 + g, r1 = r0 + 8;
-  const int lim0 = r0 < R ? a.lim[tok0 + r0 / a.G] : -1;
-  const int lim1 = r1 < R ? a.lim[tok0 + r1 / a.G] : -1;
-
-  uint32_t qa[4][4];
-  if (has_rows) {
-#pragma unroll
-    for (int kk = 0; kk < 4; ++kk) {
-      const int row = mt * 16 + (lane & 15);
-      const int ch = 2 * kk + (lane >> 4);
-      ldsm_x4(smem_u32(sQ) + sw128(row, ch), qa[kk][0], qa[kk][1], qa[kk][2], qa[kk][3]);
-    }
-  }
-
-  const float kScaleLog2 = 0.125f * 1.4426950408889634f;
-  float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f;
-  float o[8][4];
-#pragma unroll
-  for (int j = 0; j < 8; ++j) o[j][0] = o[j][1] = o[j][2] = o[j][3] = 0.f;
   bool ok = true;
+  // the row's state (softmax threads): O (unnormalised), running max m (log2
+  // units), running sum l
+  float o[64];
+#pragma unroll
+  for (int k = 0; k < 64; ++k) o[k] = 0.f;
+  float m = -INFINITY, l = 0.f;
 
-  for (int i = 0; i < npl; ++i) {
-    const int s = i % kAttnStages;
-    if (ok && !mbar_wait(smem_u32(&lfull[s]), (i / kAttnStages) & 1, a.err)) ok = false;
-    if (ok && has_rows) {
-      const uint32_t kbase = smem_u32(sK + s * kAttnPageBytes);
-      const uint32_t vbase = smem_u32(sV + s * kAttnPageBytes);
-      float sacc[8][4];
-#pragma unroll
-      for (int j = 0; j < 8; ++j) sacc[j][0] = sacc[j][1] = sacc[j][2] = sacc[j][3] = 0.f;
-#pragma unroll
-      for (int j = 0; j < 8; ++j) {
-#pragma unroll
-        for (int kk = 0; kk < 4; kk += 2) {
-          uint32_t b0, b1, b2, b3;
-          const int row = 8 * j + (lane & 7);
-          const int ch = 2 * kk + (lane >> 3);
-          ldsm_x4(kbase + sw128(row, ch), b0, b1, b2, b3);
-          mma_f16_16816(sacc[j], qa[kk], b0, b1);
-          mma_f16_16816(sacc[j], qa[kk + 1], b2, b3);
+  if (warp == 4) {
+    // ---- TMA producer: K and V^T pages of the item, in order
+    if (lane == 0) {
+      const int safe_pages = a.blk_slot ? a.lim[tok0] / 64 : 0;   // wholly committed pages
+      const uint64_t pol = l2_policy_evict_first();
+      int issued = 0;
+      auto issue = [&](int i) {
+        const int s = i % kAttnStages;
+        int phys = pt[p_begin + i];
+        if (phys < 0) {  // unmapped page: the TMA box lands out of bounds and reads zeros
+          atomicExch(a.err, kErrBounds);
+          phys = 0x3FFFFFFF / a.rows_per_page;
         }
-      }
-      // mask + online softmax (rows r0: elements 0,1; r1: elements 2,3)
-      const int kbase_abs = page_of(i) * 64;
-      float mx0 = -INFINITY, mx1 = -INFINITY;
-#pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        const int key = kbase_abs + 8 * j + 2 * tq;
-        sacc[j][0] = key <= lim0 ? sacc[j][0] * kScaleLog2 : -INFINITY;
-        sacc[j][1] = key + 1 <= lim0 ? sacc[j][1] * kScaleLog2 : -INFINITY;
-        sacc[j][2] = key <= lim1 ? sacc[j][2] * kScaleLog2 : -INFINITY;
-        sacc[j][3] = key + 1 <= lim1 ? sacc[j][3] * kScaleLog2 : -INFINITY;
-        mx0 = fmaxf(mx0, fmaxf(sacc[j][0], sacc[j][1]));
-        mx1 = fmaxf(mx1, fmaxf(sacc[j][2], sacc[j][3]));
-      }
-      mx0 = fmaxf(mx0, __shfl_xor_sync(0xFFFFFFFFu, mx0, 1));
-      mx0 = fmaxf(mx0, __shfl_xor_sync(0xFFFFFFFFu, mx0, 2));
-      mx1 = fmaxf(mx1, __shfl_xor_sync(0xFFFFFFFFu, mx1, 1));
-      mx1 = fmaxf(mx1, __shfl_xor_sync(0xFFFFFFFFu, mx1, 2));
-      const float mn0 = fmaxf(m0, mx0), mn1 = fmaxf(m1, mx1);
-      const float al0 = (mn0 == -INFINITY) ? 1.f : exp2f(m0 - mn0);
-      const float al1 = (mn1 == -INFINITY) ? 1.f : exp2f(m1 - mn1);
-      const float sub0 = (mn0 == -INFINITY) ? 0.f : mn0;
-      const float sub1 = (mn1 == -INFINITY) ? 0.f : mn1;
-      m0 = mn0;
-      m1 = mn1;
-      float ps0 = 0.f, ps1 = 0.f;
-      uint32_t pa[4][4];
-#pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        const float p0 = exp2f(sacc[j][0] - sub0), p1 = exp2f(sacc[j][1] - sub0);
-        const float p2 = exp2f(sacc[j][2] - sub1), p3 = exp2f(sacc[j][3] - sub1);
-        ps0 += p0 + p1;
-        ps1 += p2 + p3;
-        pa[j >> 1][(j & 1) * 2 + 0] = pack_f16x2(p0, p1);
-        pa[j >> 1][(j & 1) * 2 + 1] = pack_f16x2(p2, p3);
-      }
-      l0 = l0 * al0 + ps0;
-      l1 = l1 * al1 + ps1;
-#pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        o[j][0] *= al0;
-        o[j][1] *= al0;
-        o[j][2] *= al1;
-        o[j][3] *= al1;
-      }
-      // O += P V ; V stored [key][dim] -> transposed ldmatrix
-#pragma unroll
-      for (int kk = 0; kk < 4; ++kk) {
-#pragma unroll
-        for (int jn = 0; jn < 8; jn += 2) {
-          uint32_t b0, b1, b2, b3;
-          const int row = 16 * kk + (lane & 7) + ((lane >> 3) & 1) * 8;
-          const int ch = jn + (lane >> 4);
-          ldsm_x4_t(vbase + sw128(row, ch), b0, b1, b2, b3);
-          mma_f16_16816(o[jn], pa[kk], b0, b1);
-          mma_f16_16816(o[jn + 1], pa[kk], b2, b3);
+        const long long row = a.kv_row_base + static_cast<long long>(phys) * a.rows_per_page;
+        const uint32_t fb = smem_u32(&full[s]);
+        mbar_arrive_expect_tx(fb, kAttnStageBytes);
+        uint8_t* st = ring + s * kAttnStageBytes;
+        tma_load_2d(smem_u32(st), &tmKV, 0, static_cast<int>(row + h * 64), fb, pol);
+        tma_load_2d(smem_u32(st + kAttnPageBytes), &tmKV, 0, static_cast<int>(row + (a.Hkv + h) * 64),
+                    fb, pol);
+      };
+      while (issued < min(np, kAttnStages) && p_begin + issued < safe_pages) issue(issued++);
+      pdl_wait();
+      pdl_trigger();
+      while (issued < np && ok) {
+        const int s = issued % kAttnStages;
+        if (issued >= kAttnStages &&
+            !mbar_wait(smem_u32(&empty[s]), ((issued / kAttnStages) + 1) & 1, a.err)) {
+          ok = false;
+          break;
         }
+        issue(issued++);
       }
+      s_int[3] = issued;
+    } else {
+      pdl_wait();
+      pdl_trigger();
     }
-    lane_sync(ln, lthreads);   // every warp of the lane is done with stage s
-    if (producer && ok && i + kAttnStages < npl) issue(i + kAttnStages);
+  } else if (warp == 5) {
+    // ---- MMA issuer: S one page ahead of the softmax, PV after each P
+    pdl_wait();
+    pdl_trigger();
+    if (lane == 0) {
+      constexpr uint32_t idesc = umma_idesc_f16(128, 64);
+      const uint64_t qdesc = umma_desc_sw128(smem_u32(sQ));
+      auto issue_s = [&](int j) -> bool {
+        const int s = j % kAttnStages, buf = j & 1;
+        if (!mbar_wait(smem_u32(&full[s]), (j / kAttnStages) & 1, a.err)) return false;
+        s_int[2] = j + 1;
+        if (j >= 2 && !mbar_wait(smem_u32(&s_free[buf]), ((j >> 1) + 1) & 1, a.err)) return false;
+        tc_fence_after();
+        const uint64_t kdesc = umma_desc_sw128(smem_u32(ring + s * kAttnStageBytes));
+#pragma unroll
+        for (int k = 0; k < 4; ++k)
+          umma_f16(tmem + buf * 64, qdesc + 2 * k, kdesc + 2 * k, idesc, k > 0 ? 1u : 0u);
+        umma_commit(smem_u32(&s_full[buf]));
+        return true;
+      };
+      if (!mbar_wait(smem_u32(q_full), 0, a.err)) ok = false;   // Q tile written
+      if (ok) ok = issue_s(0);
+      for (int j = 0; j < np && ok; ++j) {
+        if (j + 1 < np && !(ok = issue_s(j + 1))) break;
+        const int s = j % kAttnStages, buf = j & 1;
+        if (!mbar_wait(smem_u32(&p_full[buf]), (j >> 1) & 1, a.err)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint64_t pdesc = umma_desc_sw128(smem_u32(sP + buf * kAttnMaxRows * 128));
+        const uint64_t vdesc = umma_desc_sw128(smem_u32(ring + s * kAttnStageBytes + kAttnPageBytes));
+#pragma unroll
+        for (int k = 0; k < 4; ++k)
+          umma_f16(tmem + 128 + buf * 64, pdesc + 2 * k, vdesc + 2 * k, idesc, k > 0 ? 1u : 0u);
+        umma_commit(smem_u32(&pv_full[buf]));
+        umma_commit(smem_u32(&empty[s]));
+      }
+      umma_commit(smem_u32(mma_done));   // retires once every MMA above has
+    }
+  } else {
+    // ---- softmax warps: thread r owns row r (TMEM lane r)
+    const int r = threadIdx.x;
+    // Q rows -> swizzled smem (zero rows past R); the MMA reads all 128 rows
+    pdl_wait();
+    pdl_trigger();
+    for (int idx = threadIdx.x; idx < rows_alloc * 8; idx += 128) {
+      const int rr = idx >> 3, ch = idx & 7;
+      uint4 v = make_uint4(0, 0, 0, 0);
+      if (rr < R) {
+        const int t = tok0 + rr / a.G;
+        const int hq = h * a.G + rr % a.G;
+        v = *reinterpret_cast<const uint4*>(a.q + (static_cast<size_t>(t) * a.Hq + hq) * 64 + ch * 8);
+      }
+      *reinterpret_cast<uint4*>(sQ + sw128(rr, ch)) = v;
+    }
+    fence_proxy_async_smem();
+    mbar_arrive(smem_u32(q_full));
+    const int lim_r = r < R ? a.lim[tok0 + r / a.G] : -1;
+    const uint32_t trow = tmem + (static_cast<uint32_t>(warp * 32) << 16);
+    const float kScaleLog2 = 0.125f * 1.4426950408889634f;   // 1/sqrt(64) in log2 units
+    float alpha_prev = 1.f;
+    // O = alpha O + PV_j, PV_j from TMEM buffer j & 1
+    auto apply_pv = [&](int j, float alpha) -> bool {
+      if (!mbar_wait(smem_u32(&pv_full[j & 1]), (j >> 1) & 1, a.err)) return false;
+      tc_fence_after();
+      uint32_t v0[32], v1[32];
+      tmem_ld32_nowait(trow + 128 + (j & 1) * 64, v0);
+      tmem_ld32_nowait(trow + 128 + (j & 1) * 64 + 32, v1);
+      tmem_wait_ld();
+#pragma unroll
+      for (int k = 0; k < 32; ++k) {
+        o[k] = alpha * o[k] + __uint_as_float(v0[k]);
+        o[32 + k] = alpha * o[32 + k] + __uint_as_float(v1[k]);
+      }
+      return true;
+    };
+    for (int j = 0; j < np; ++j) {
+      const int buf = j & 1;
+      // 1. S_j row from TMEM; the buffer is free again once all 128 rows are read
+      if (ok && !mbar_wait(smem_u32(&s_full[buf]), (j >> 1) & 1, a.err)) ok = false;
+      if (!ok) break;
+      tc_fence_after();
+      uint32_t s0[32], s1[32];
+      tmem_ld32_nowait(trow + buf * 64, s0);
+      tmem_ld32_nowait(trow + buf * 64 + 32, s1);
+      tmem_wait_ld();
+      tc_fence_before();
+      mbar_arrive(smem_u32(&s_free[buf]));
+      // 2. mask (keys past the row's limit), scale, running max, probabilities
+      const int key0 = (p_begin + j) * 64;
+      float sv[64];
+      float mx = -INFINITY;
+#pragma unroll
+      for (int k = 0; k < 64; ++k) {
+        const float x = __uint_as_float(k < 32 ? s0[k] : s1[k - 32]);
+        sv[k] = key0 + k <= lim_r ? x * kScaleLog2 : -INFINITY;
+        mx = fmaxf(mx, sv[k]);
+      }
+      const float m_new = fmaxf(m, mx);
+      const float alpha = (m_new == -INFINITY) ? 1.f : exp2f(m - m_new);
+      const float sub = (m_new == -INFINITY) ? 0.f : m_new;
+      uint32_t pk[32];
+      float ps[8];
+#pragma unroll
+      for (int cch = 0; cch < 8; ++cch) {
+        float p[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) p[e] = exp2f(sv[8 * cch + e] - sub);
+        ps[cch] = ((p[0] + p[1]) + (p[2] + p[3])) + ((p[4] + p[5]) + (p[6] + p[7]));
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          __half2 hv = __floats2half2_rn(p[2 * e], p[2 * e + 1]);
+          pk[4 * cch + e] = *reinterpret_cast<uint32_t*>(&hv);
+        }
+      }
+      l = l * alpha + (((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7])));
+      m = m_new;
+      // 3. PV_{j-1} into O (it and everything before it retired: P buffer `buf` is free)
+      if (j >= 1 && !(ok = apply_pv(j - 1, alpha_prev))) break;
+      // 4. P_j (fp16) as the A operand of PV_j: row r, 128-byte swizzle
+      uint8_t* prow = sP + buf * kAttnMaxRows * 128;
+#pragma unroll
+      for (int cch = 0; cch < 8; ++cch)
+        *reinterpret_cast<uint4*>(prow + sw128(r, cch)) =
+            make_uint4(pk[4 * cch], pk[4 * cch + 1], pk[4 * cch + 2], pk[4 * cch + 3]);
+      fence_proxy_async_smem();
+      tc_fence_before();
+      mbar_arrive(smem_u32(&p_full[buf]));
+      alpha_prev = alpha;
+    }
+    if (ok && np > 0) ok = apply_pv(np - 1, alpha_prev);
   }
-  const bool all_ok = __syncthreads_and(ok);   // both lanes done: the ring is idle
 
-  // row sums across the quad
-  l0 += __shfl_xor_sync(0xFFFFFFFFu, l0, 1);
-  l0 += __shfl_xor_sync(0xFFFFFFFFu, l0, 2);
-  l1 += __shfl_xor_sync(0xFFFFFFFFu, l1, 1);
-  l1 += __shfl_xor_sync(0xFFFFFFFFu, l1, 2);
-
-  // ---- lane 1 -> lane 0 (shared memory): M = max, w = exp2(m - M) per lane,
-  //      O = w0 O0 + w1 O1, l = w0 l0 + w1 l1.  lp [row][kAttnRow] in the ring.
-  float* lp = reinterpret_cast<float*>(ring);
-  if (ln == 1 && has_rows) {
-#pragma unroll
-    for (int half = 0; half < 2; ++half) {
-      float* dst = lp + (half ? r1 : r0) * kAttnRow;
-#pragma unroll
-      for (int j = 0; j < 8; ++j)
-        *reinterpret_cast<float2*>(dst + 8 * j + 2 * tq) =
-            make_float2(o[j][half * 2 + 0], o[j][half * 2 + 1]);
-      if (tq == 0) *reinterpret_cast<float2*>(dst + 64) = half ? make_float2(m1, l1) : make_float2(m0, l0);
-    }
+  const bool all_ok = __syncthreads_and(ok);
+  // every MMA retired and every TMA copy landed before TMEM and the ring are released
+  if (warp == 5) {
+    if (lane == 0) mbar_wait(smem_u32(mma_done), 0, a.err);
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc(tmem, kAttnTmemCols);
+  }
+  if (warp == 4 && lane == 0) {
+    for (int i = s_int[2]; i < s_int[3]; ++i)
+      mbar_wait(smem_u32(&full[i % kAttnStages]), (i / kAttnStages) & 1, a.err);
   }
   __syncthreads();
-  if (ln == 0 && has_rows) {
-#pragma unroll
-    for (int half = 0; half < 2; ++half) {
-      const float* src = lp + (half ? r1 : r0) * kAttnRow;
-      const float2 ml = *reinterpret_cast<const float2*>(src + 64);
-      const float ma = half ? m1 : m0;
-      const float M = fmaxf(ma, ml.x);
-      const float wa = (ma == -INFINITY) ? 0.f : exp2f(ma - M);
-      const float wb = (ml.x == -INFINITY) ? 0.f : exp2f(ml.x - M);
-#pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        const float2 v = *reinterpret_cast<const float2*>(src + 8 * j + 2 * tq);
-        o[j][half * 2 + 0] = wa * o[j][half * 2 + 0] + wb * v.x;
-        o[j][half * 2 + 1] = wa * o[j][half * 2 + 1] + wb * v.y;
-      }
-      if (half) { l1 = wa * l1 + wb * ml.y; m1 = M; } else { l0 = wa * l0 + wb * ml.y; m0 = M; }
-    }
-  }
-  __syncthreads();   // lp consumed; the ring is reused below
-  const bool lead = ln == 0 && has_rows;
+  const int r = threadIdx.x;
+  const bool row_thread = r < R;
 
   if (nitems == 1) {   // the block's only item: its rows are final
-    if (lead && all_ok) {
+    if (row_thread && all_ok) {
+      const float inv = 1.0f / l;
+      const int t = tok0 + r / a.G;
+      const int hq = h * a.G + r % a.G;
+      __half* dst = a.out + (static_cast<size_t>(t) * a.Hq + hq) * 64;
 #pragma unroll
-      for (int half = 0; half < 2; ++half) {
-        const int r = half ? r1 : r0;
-        if (r >= R) continue;
-        const float inv = 1.0f / (half ? l1 : l0);
-        const int t = tok0 + r / a.G;
-        const int hq = h * a.G + r % a.G;
-        __half* dst = a.out + (static_cast<size_t>(t) * a.Hq + hq) * 64;
+      for (int cch = 0; cch < 8; ++cch) {
+        uint32_t w4[4];
 #pragma unroll
-        for (int j = 0; j < 8; ++j) {
-          const float x0 = o[j][half * 2 + 0] * inv, x1 = o[j][half * 2 + 1] * inv;
-          *reinterpret_cast<__half2*>(dst + 8 * j + 2 * tq) = __floats2half2_rn(x0, x1);
+        for (int e = 0; e < 4; ++e) {
+          __half2 hv = __floats2half2_rn(o[8 * cch + 2 * e] * inv, o[8 * cch + 2 * e + 1] * inv);
+          w4[e] = *reinterpret_cast<uint32_t*>(&hv);
         }
+        *reinterpret_cast<uint4*>(dst + 8 * cch) = make_uint4(w4[0], w4[1], w4[2], w4[3]);
       }
     }
     return;
   }
+
+  // this thread's row (O, m, l) -> a [kAttnRow] slot
+  auto put_row = [&](float* dst) {
+#pragma unroll
+    for (int k = 0; k < 64; k += 4)
+      *reinterpret_cast<float4*>(dst + k) = make_float4(o[k], o[k + 1], o[k + 2], o[k + 3]);
+    *reinterpret_cast<float2*>(dst + 64) = make_float2(m, l);
+  };
 
   // Merged rows of one item: source `it`, row r -> float pointer (O[64], m, l).
   // Cluster: recv[it][k] with r = c + k * nitems.  Global: part[b][h][it][r].
@@ -421,20 +447,8 @@ __global__ void __launch_bounds__(512)
     // ---- items -> owners.  stage [owner][slot][kAttnRow] in the ring.
     float* stage = reinterpret_cast<float*>(ring);
     const int blk_floats = rpo * kAttnRow;
-    if (lead) {
-#pragma unroll
-      for (int half = 0; half < 2; ++half) {
-        const int r = half ? r1 : r0;
-        if (r >= R) continue;
-        float* dst = stage + static_cast<size_t>(r % nitems) * blk_floats + (r / nitems) * kAttnRow;
-#pragma unroll
-        for (int j = 0; j < 8; ++j)
-          *reinterpret_cast<float2*>(dst + 8 * j + 2 * tq) =
-              make_float2(o[j][half * 2 + 0], o[j][half * 2 + 1]);
-        if (tq == 0)
-          *reinterpret_cast<float2*>(dst + 64) = half ? make_float2(m1, l1) : make_float2(m0, l0);
-      }
-    }
+    if (row_thread)
+      put_row(stage + static_cast<size_t>(r % nitems) * blk_floats + (r / nitems) * kAttnRow);
     fence_proxy_async_smem();
     __syncthreads();
     cluster_wait();   // every CTA of the cluster runs: peers' buffers and barriers exist
@@ -451,20 +465,7 @@ __global__ void __launch_bounds__(512)
     my_rows = (R - c + nitems - 1) / nitems;
   } else {
     // ---- item rows -> global scratch; the last item to arrive merges
-    if (lead) {
-#pragma unroll
-      for (int half = 0; half < 2; ++half) {
-        const int r = half ? r1 : r0;
-        if (r >= R) continue;
-        float* dst = part_bh + (static_cast<size_t>(c) * rows_alloc + r) * kAttnRow;
-#pragma unroll
-        for (int j = 0; j < 8; ++j)
-          *reinterpret_cast<float2*>(dst + 8 * j + 2 * tq) =
-              make_float2(o[j][half * 2 + 0], o[j][half * 2 + 1]);
-        if (tq == 0)
-          *reinterpret_cast<float2*>(dst + 64) = half ? make_float2(m1, l1) : make_float2(m0, l0);
-      }
-    }
+    if (row_thread) put_row(part_bh + (static_cast<size_t>(c) * rows_alloc + r) * kAttnRow);
     __threadfence();
     __syncthreads();
     if (threadIdx.x == 0) s_int[1] = (atomicAdd(a.ticket + bh, 1) == nitems - 1) ? 1 : 0;
@@ -545,9 +546,9 @@ __global__ void __launch_bounds__(512)
           }
       }
       if (all_ok && got) {
-        const int r = row_of(k);
-        const int t = tok0 + r / a.G;
-        const int hq = h * a.G + r % a.G;
+        const int rr = row_of(k);
+        const int t = tok0 + rr / a.G;
+        const int hq = h * a.G + rr % a.G;
         __half* dst = a.out + (static_cast<size_t>(t) * a.Hq + hq) * 64 + d4;
         *reinterpret_cast<__half2*>(dst) = __floats2half2_rn(acc.x, acc.y);
         *reinterpret_cast<__half2*>(dst + 2) = __floats2half2_rn(acc.z, acc.w);

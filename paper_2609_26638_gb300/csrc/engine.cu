@@ -82,14 +82,21 @@ struct AttnGeom {
 };
 AttnGeom attn_geom(int W, int G) {
   const int qs = std::min(W, kAttnMaxRows / G);
-  return {qs, cdiv(W, qs), attn_mtiles(qs * G) * 16};
+  return {qs, cdiv(W, qs), kAttnMaxRows};
+}
+
+// Items merge inside a cluster when there are at most 8 of them and the
+// launch is about one wave (clusters of 8 CTAs wait for 8 free SMs of one GPC
+// and fragment larger grids); otherwise through global scratch.  Both give
+// the same bits.
+bool attn_use_cluster(int items, int blocks_x_heads) {
+  return items <= kAttnMaxCluster && items * blocks_x_heads <= 2 * 152;
 }
 
 cudaError_t launch_attention(const CUtensorMap& tm, const AttnArgs& a, int n_blocks,
                              cudaStream_t s, bool pdl) {
-  const int rows = attn_mtiles(a.QS * a.G) * 16;
   dim3 grid(a.max_items, a.Hkv, n_blocks);
-  return launch_ex(attn_paged_kernel, grid, dim3(attn_threads(rows)), attn_smem_bytes(rows), s, pdl,
+  return launch_ex(attn_paged_kernel, grid, dim3(kAttnThreads), kAttnSmemBytes, s, pdl,
                    dim3(a.cluster ? a.max_items : 1, 1, 1), tm, a);
 }
 
@@ -287,11 +294,15 @@ size_t carve(gs_handle* h, const gs_config& c, void* base) {
   const int items_dec = cdiv(pt_stride, sp);
   const int sp_pf = std::max(8, cdiv(pt_stride, kAttnMaxCluster));
   const int items_pf = cdiv(pt_stride, sp_pf);
-  const size_t attn_blocks = static_cast<size_t>(c.max_batch) * g_dec.n_sub;
+  const AttnGeom g_pf = attn_geom(qb_pf, G);
+  const int blocks_pf = cdiv(std::min(c.max_prefill, T_max), qb_pf);
+  const size_t attn_blocks = std::max(static_cast<size_t>(c.max_batch) * g_dec.n_sub,
+                                      static_cast<size_t>(blocks_pf));
+  // item rows of the global merge (used when a launch is too large for clusters)
   const size_t attn_part_floats =
-      items_dec > kAttnMaxCluster
-          ? attn_blocks * c.n_kv_heads * items_dec * g_dec.rows * kAttnRow
-          : 0;
+      std::max(static_cast<size_t>(c.max_batch) * g_dec.n_sub * items_dec * g_dec.rows,
+               static_cast<size_t>(blocks_pf) * items_pf * g_pf.rows) *
+      c.n_kv_heads * kAttnRow;
   int* err_word = cv.take<int>(64);
   SeqStateDev st;
   st.seq_len = cv.take<int32_t>(c.max_batch);
@@ -443,7 +454,7 @@ int run_attention(gs_handle* h, int layer, int T, const AttnLaunch& L) {
   a.kv_row_base = static_cast<long long>(layer) * h->n_pages * a.rows_per_page;
   a.split_pages = L.split_pages;
   a.max_items = L.max_items;
-  a.cluster = L.max_items <= kAttnMaxCluster ? 1 : 0;
+  a.cluster = attn_use_cluster(L.max_items, L.n_seq * g.n_sub * c.n_kv_heads) ? 1 : 0;
   a.part = h->attn_part;
   a.ticket = h->attn_ticket;
   a.err = h->err_word;
@@ -1017,7 +1028,7 @@ size_t gs_attention_scratch_bytes(int n_seq, int W, int n_heads, int n_kv_heads,
   cv.take<int32_t>(static_cast<size_t>(n_seq) * W);  // key limits
   cv.take<int32_t>(n_seq);                            // sequence -> page-table row
   cv.take<int>(blocks * n_kv_heads);                  // merge tickets
-  if (items > kAttnMaxCluster)                        // item rows of the global merge
+  if (!attn_use_cluster(items, static_cast<int>(blocks) * n_kv_heads))   // global merge rows
     cv.take<float>(blocks * n_kv_heads * items * g.rows * kAttnRow);
   return align_up(cv.off, 256);
 }
@@ -1068,9 +1079,9 @@ int gs_attention(int mode, const void* q, const void* kv, int n_pages, const int
   int32_t* lim = cv.take<int32_t>(static_cast<size_t>(n_seq) * W);
   int32_t* blk_slot = cv.take<int32_t>(n_seq);
   int* ticket = cv.take<int>(blocks * n_kv_heads);
-  float* part = items > kAttnMaxCluster
-                    ? cv.take<float>(blocks * n_kv_heads * items * g.rows * kAttnRow)
-                    : nullptr;
+  float* part = attn_use_cluster(items, static_cast<int>(blocks) * n_kv_heads)
+                    ? nullptr
+                    : cv.take<float>(blocks * n_kv_heads * items * g.rows * kAttnRow);
   CUtensorMap tm;
   const uint64_t rows = static_cast<uint64_t>(n_pages) * 2 * n_kv_heads * 64;
   if (rows >= (1ull << 31) || !make_map(&tm, kv, rows, 64, 64)) return GS_ERR_INVALID_ARG;
@@ -1099,7 +1110,7 @@ int gs_attention(int mode, const void* q, const void* kv, int n_pages, const int
   a.kv_row_base = 0;
   a.split_pages = split_pages;
   a.max_items = items;
-  a.cluster = items <= kAttnMaxCluster ? 1 : 0;
+  a.cluster = attn_use_cluster(items, static_cast<int>(blocks) * n_kv_heads) ? 1 : 0;
   a.part = part;
   a.ticket = ticket;
   a.err = err;

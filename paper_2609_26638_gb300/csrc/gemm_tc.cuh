@@ -109,7 +109,6 @@ struct GemmShape {
 
 // Epilogue of 32 consecutive tokens (t0 .. t0+31) of feature row `row`;
 // only tokens j in [jlo, jhi) with t0 + j < M are produced.
-__device__ __forceinline__ int isv_of(int region) { return region == 2 ? 1 : 0; }
 
 // Per-token data the epilogue needs, staged in shared memory while the
 // mainloop runs: rs = folded-norm scale, kvdst = element offset of the token's
@@ -218,13 +217,24 @@ __device__ __forceinline__ void gemm_epilogue_chunk(const GemmArgs& a, float (&v
       for (int j = 0; j < EW; ++j)
         if (j >= jlo && j < jhi)
           a.q_out[(static_cast<size_t>(t0 + j) * a.Hq + head) * 64 + d] = to_f16(v[j], a.err);
-    } else {
-      // kvdst[j]: offset of (page, K, head 0, row p & 63, dim 0); V is Hkv * 4096 further
-      const long long off = (static_cast<long long>(isv_of(region)) * a.Hkv + head) * 4096 + d;
+    } else if (region == 1) {
+      // K: kvdst[j] = offset of (page, K, head 0, token p & 63, dim 0); K is [token][dim]
+      const long long off = static_cast<long long>(head) * 4096 + d;
 #pragma unroll
       for (int j = 0; j < EW; ++j) {
         const long long base = tm.kvdst[j];
         if (j >= jlo && j < jhi && base >= 0) a.kv_layer[base + off] = to_f16(v[j], a.err);
+      }
+    } else {
+      // V is stored transposed, [dim][token]: (page, V, head, dim d, token p & 63)
+      const long long off = (static_cast<long long>(a.Hkv) + head) * 4096 + d * 64;
+#pragma unroll
+      for (int j = 0; j < EW; ++j) {
+        const long long base = tm.kvdst[j];
+        if (j >= jlo && j < jhi && base >= 0) {
+          const int tok = tm.pos[j] & 63;
+          a.kv_layer[base - tok * 64 + off + tok] = to_f16(v[j], a.err);
+        }
       }
     }
   } else if constexpr (EPI == kEpiSwiGLU) {

@@ -128,7 +128,8 @@ def test_linear_rows_do_not_depend_on_tile_width(gs, split):
 
 # ------------------------------------------------------------------ attention
 def _paged(k, v, rng):
-    """Pack per-sequence K/V [B, ctx, Hkv, 64] into a shuffled page pool."""
+    """Pack per-sequence K/V [B, ctx, Hkv, 64] into a shuffled page pool: per
+    page and KV head, K as [token][dim] and V transposed as [dim][token]."""
     B, ctx, Hkv, hd = k.shape
     pages_per = math.ceil(ctx / 64)
     n_pages = B * pages_per + 3
@@ -137,8 +138,8 @@ def _paged(k, v, rng):
     for b in range(B):
         for p in range(pages_per):
             t0, t1 = p * 64, min(ctx, p * 64 + 64)
-            pool[perm[b, p], 0, :, : t1 - t0] = k[b, t0:t1].transpose(1, 0, 2)
-            pool[perm[b, p], 1, :, : t1 - t0] = v[b, t0:t1].transpose(1, 0, 2)
+            pool[perm[b, p], 0, :, : t1 - t0] = k[b, t0:t1].transpose(1, 0, 2)      # [head][tok][dim]
+            pool[perm[b, p], 1, :, :, : t1 - t0] = v[b, t0:t1].transpose(1, 2, 0)   # [head][dim][tok]
     return pool, perm.astype(np.int32), n_pages
 
 
