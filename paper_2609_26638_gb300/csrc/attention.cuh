@@ -14,24 +14,28 @@
 // item, pages in order.  A page holds K as [64 tokens][64 dims] and V
 // transposed, [64 dims][64 tokens] (8 KB each), so both are K-major operands.
 // Per page j:
-//   S_j = Q K_j^T      tcgen05.mma M=128 (rows) N=64 (keys) K=64, into TMEM
-//   softmax            one thread per row: m, l, p = exp2(s*scale - m) (fp32),
-//                      P_j (fp16) into shared memory as the next A operand
-//   PV_j = P_j V_j     tcgen05.mma M=128 N=64 (dims) K=64 (keys), into TMEM
-//   O = alpha_j O + PV_j  in the row's registers
-// Warps 0-3 own rows 0-127 (TMEM lanes); warp 4 streams K/V pages by TMA
-// (128-byte swizzle) through a ring of stages; warp 5 issues the MMAs, one
-// page of S ahead of the softmax, with S and PV double-buffered in TMEM.
+//   S_j = Q K_j^T       tcgen05.mma M=128 (rows) N=64 (keys) K=64 into TMEM
+//   softmax             one thread per row: running max m (log2 units) and
+//                       sum l in fp32, P_j = exp2(s*scale - m) as fp16 into
+//                       shared memory (the A operand of the next MMA)
+//   O += P_j V_j        tcgen05.mma M=128 N=64 (dims) K=64 (keys), O in TMEM
+// The max only moves when a page raises it by more than 2^8: then the thread
+// first rescales its O row in TMEM (and l) by exp2(m_old - m_new).  Smaller
+// rises keep the old m, so P stays <= 2^8 (well inside fp16).  Either way
+// O / l is the softmax-weighted sum.  Warps 0-3 own rows 0-127 (TMEM lanes;
+// warps whose rows are all padding only keep the barriers' pace); warp 4
+// streams K/V pages by TMA (128-byte swizzle) through a ring of stages; warp
+// 5 issues the MMAs, S one page ahead of the softmax, S double-buffered.
 //
 // Merge over items, item order 0, 1, ...: M = max m_i, w_i = exp2(m_i - M),
 // coef_i = w_i / sum_j w_j l_j, O = sum coef_i O_i.  A block with one item
 // writes its rows directly.  A (block, head) with at most 8 items may form one
-// thread-block cluster: each CTA sends the rows that CTA (r mod n) owns to it
-// with one bulk async copy into its shared memory, completing on its
-// mbarrier, and each owner merges its rows.  Otherwise every item writes its
-// rows to global scratch and the last one to finish (atomic ticket per (block,
-// head), no spinning) merges them.  Both paths run the same arithmetic in the
-// same order.
+// thread-block cluster: once every CTA of the cluster has finished its pages,
+// each sends the rows that CTA (r mod n) owns to it with one bulk async copy
+// into its shared memory, completing on its mbarrier, and each owner merges
+// its rows.  Otherwise every item writes its rows to global scratch and the
+// last one to finish (atomic ticket per (block, head), no spinning) merges
+// them.  Both paths run the same arithmetic in the same order.
 //
 // Invariance.  Item boundaries are absolute page numbers fixed by SP, pages
 // are reduced in order, the MMA's arithmetic for a row does not depend on the
@@ -44,25 +48,30 @@
 
 namespace gs {
 
-constexpr int kAttnStages = 6;             // K/V page pairs in flight
+constexpr int kAttnStages = 3;             // K/V page pairs in flight
 constexpr int kAttnPageBytes = 64 * 128;  // 64 x 64 fp16
 constexpr int kAttnStageBytes = 2 * kAttnPageBytes;
 constexpr int kAttnRow = 68;              // partial row: O[64], m, l, 2 pad (272 B)
 constexpr int kAttnMaxRows = 128;         // rows of one query block (the MMA's M)
 constexpr int kAttnMaxCluster = 8;        // items merged inside a cluster
-constexpr int kAttnThreads = 192;         // 4 softmax warps, TMA warp, MMA warp
-constexpr int kAttnTmemCols = 256;        // S[2] at 0, 64; PV[2] at 128, 192
+constexpr int kAttnSoftWarps = 8;         // two warps per TMEM lane quarter
+constexpr int kAttnSoftThreads = kAttnSoftWarps * 32;
+constexpr int kAttnThreads = kAttnSoftThreads + 64;   // + TMA warp, MMA warp
+constexpr int kAttnTmaWarp = kAttnSoftWarps, kAttnMmaWarp = kAttnSoftWarps + 1;
+constexpr int kAttnTmemCols = 256;        // S[2] at columns 0, 64; O at 128
+constexpr float kAttnRescale = 8.0f;      // log2 growth of the max that forces a rescale
 constexpr int kAttnRingBytes = kAttnStages * kAttnStageBytes;
-// Q [128][128 B] | ring | P[2] [128][128 B] | receive buffer | barriers
+// Q [128][128 B] | P[2] [128][128 B] | ring | barriers.  After the pages are
+// done, Q and P hold the owner-grouped rows (cluster) and the ring the
+// received rows or the merge's (m, l) tables.
 constexpr int kAttnQOff = 0;
-constexpr int kAttnRingOff = kAttnMaxRows * 128;
-constexpr int kAttnPOff = kAttnRingOff + kAttnRingBytes;
-constexpr int kAttnRecvOff = kAttnPOff + 2 * kAttnMaxRows * 128;
-constexpr int kAttnRecvFloats = (kAttnMaxRows + kAttnMaxCluster) * kAttnRow;
-constexpr int kAttnBarOff = kAttnRecvOff + kAttnRecvFloats * 4;
-constexpr int kAttnSmemBytes = 1024 + kAttnBarOff + 256;
-static_assert(kAttnRingBytes >= (kAttnMaxRows + kAttnMaxCluster) * kAttnRow * 4,
-              "the idle ring holds the owner-grouped rows");
+constexpr int kAttnPOff = kAttnMaxRows * 128;
+constexpr int kAttnRingOff = kAttnPOff + 2 * kAttnMaxRows * 128;
+constexpr int kAttnBarOff = kAttnRingOff + kAttnRingBytes;
+constexpr int kAttnSmemBytes = 1024 + kAttnBarOff + 256 + (2 * kAttnSoftThreads + 8 * kAttnMaxRows) * 4;
+constexpr int kAttnRowsFloats = (kAttnMaxRows + kAttnMaxCluster) * kAttnRow;
+static_assert(kAttnRingOff >= kAttnRowsFloats * 4 && kAttnRingBytes >= kAttnRowsFloats * 4,
+              "Q + P hold the owner-grouped rows, the ring the received rows");
 
 struct AttnArgs {
   const __half* q;            // [T, Hq, 64]
@@ -87,9 +96,8 @@ struct AttnArgs {
   int* err;
 };
 
-__host__ __device__ inline int attn_mtiles(int rows) { return (rows + 15) / 16; }
 __host__ __device__ inline int attn_max_smem_bytes() { return kAttnSmemBytes; }
-// The global merge keeps m and l of every (item, row) in the idle ring.
+// The merge keeps m and l of every (item, row) in the idle ring.
 __host__ __device__ inline int attn_max_merge_items(int /*rows*/) {
   return kAttnRingBytes / 4 / (2 * kAttnMaxRows);
 }
@@ -114,8 +122,170 @@ __device__ __forceinline__ void tmem_ld32_nowait(uint32_t taddr, uint32_t (&r)[3
 __device__ __forceinline__ void tmem_wait_ld() {
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
+__device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], "
+      "{%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16, "
+      "%17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32};" ::"r"(taddr),
+      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
+      "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]),
+      "r"(r[15]), "r"(r[16]), "r"(r[17]), "r"(r[18]), "r"(r[19]), "r"(r[20]), "r"(r[21]),
+      "r"(r[22]), "r"(r[23]), "r"(r[24]), "r"(r[25]), "r"(r[26]), "r"(r[27]), "r"(r[28]),
+      "r"(r[29]), "r"(r[30]), "r"(r[31])
+      : "memory");
+}
+__device__ __forceinline__ void tmem_wait_st() {
+  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
 
-__global__ void __launch_bounds__(kAttnThreads, 1)
+__device__ __forceinline__ void tmem_ld16_nowait(uint32_t taddr, uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
+}
+
+// Barriers and buffers the softmax warps share with the MMA warp.
+struct AttnSync {
+  uint64_t *s_full, *s_free, *p_full, *pv_done;
+  uint64_t* mx_bar;  // [2] every thread of a row-holding warp posted its page max
+  uint8_t* sP;       // [2][128][128 B]
+  float* red;        // [2][128] per-thread page maxima
+};
+
+__device__ __forceinline__ void tmem_ld8_nowait(uint32_t taddr, uint32_t (&r)[8]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%8];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7])
+      : "r"(taddr));
+}
+
+// Online softmax over the item's pages for the rows one thread sees.  DUP
+// copies of each block row sit in the MMA's 128 rows (copy k of row rr at MMA
+// row k * 128 / DUP + rr, so every TMEM lane quarter -- and every SM
+// sub-partition -- holds rows), and two warps share each lane quarter: the
+// thread of (copy k, warp half s) takes the columns of part 2k + s, NC =
+// 64 / (2 DUP) columns of every page.  Per page: S from TMEM, mask and scale,
+// the row max over its parts (shared memory), an O rescale when the max rises
+// by more than 2^8 (the two copy-0 threads of the row, 32 columns each; the
+// previous O += P V must have retired), P into shared memory, and the row sum
+// kept as eight 8-column partials, so the arithmetic of a row is the same for
+// every DUP.  Returns false if a wait ran out.
+template <int DUP>
+__device__ __forceinline__ bool attn_softmax(const AttnArgs& a, const AttnSync& y, uint32_t tmem,
+                                             int np, int p_begin, int R, int tok0, float& m,
+                                             float (&lc)[8]) {
+  constexpr int RPC = kAttnMaxRows / DUP;   // MMA rows per copy
+  constexpr int NC = 64 / (2 * DUP);        // columns per thread
+  constexpr int NCH = NC / 8;               // 8-column chunks per thread
+  const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
+  const int quarter = warp & 3, half = warp >> 2;
+  const int mrow = quarter * 32 + lane;     // MMA row = TMEM lane
+  const int cp = mrow / RPC, rr = mrow % RPC;
+  const int part = 2 * cp + half, col0 = part * NC;
+  const bool busy = ((quarter * 32) % RPC) < R;   // the warp holds at least one real row
+  const int lim_r = rr < R ? a.lim[tok0 + rr / a.G] : -1;
+  const uint32_t trow = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
+  const float kScaleLog2 = 0.125f * 1.4426950408889634f;   // 1/sqrt(64) in log2 units
+  // waits are warp-uniform, so a warp that gives up leaves together
+  auto wwait = [&](uint64_t* bar, uint32_t parity) {
+    return __all_sync(0xFFFFFFFFu, mbar_wait(smem_u32(bar), parity, a.err)) != 0;
+  };
+  for (int j = 0; j < np; ++j) {
+    const int buf = j & 1;
+    if (!wwait(&y.s_full[buf], (j >> 1) & 1)) return false;
+    if (!busy) {   // padding rows only: release S, hand over an (unused) P
+      if (lane == 0) {
+        mbar_arrive(smem_u32(&y.s_free[buf]));
+        mbar_arrive(smem_u32(&y.p_full[buf]));
+      }
+      continue;
+    }
+    // 1. this thread's columns of S_j; the buffer is free once every warp has read
+    tc_fence_after();
+    uint32_t sr[NC];
+    if constexpr (NC == 8) {
+      tmem_ld8_nowait(trow + buf * 64 + col0, *reinterpret_cast<uint32_t(*)[8]>(sr));
+    } else if constexpr (NC == 16) {
+      tmem_ld16_nowait(trow + buf * 64 + col0, *reinterpret_cast<uint32_t(*)[16]>(sr));
+    } else {
+      tmem_ld32_nowait(trow + buf * 64 + col0, *reinterpret_cast<uint32_t(*)[32]>(sr));
+    }
+    tmem_wait_ld();
+    tc_fence_before();
+    __syncwarp();
+    if (lane == 0) mbar_arrive(smem_u32(&y.s_free[buf]));
+    // 2. mask (keys past the row's limit), scale, this thread's maximum
+    const int key0 = (p_begin + j) * 64 + col0;
+    float sv[NC];
+    float pmx = -INFINITY;
+#pragma unroll
+    for (int k = 0; k < NC; ++k) {
+      sv[k] = key0 + k <= lim_r ? __uint_as_float(sr[k]) * kScaleLog2 : -INFINITY;
+      pmx = fmaxf(pmx, sv[k]);
+    }
+    // 3. the row's page max over its 2 DUP parts (thread of part p: MMA row
+    //    (p / 2) * RPC + rr, warp half p % 2)
+    float* red = y.red + buf * kAttnSoftThreads;
+    red[t] = pmx;
+    __syncwarp();
+    if (lane == 0) mbar_arrive(smem_u32(&y.mx_bar[buf]));
+    if (!wwait(&y.mx_bar[buf], (j >> 1) & 1)) return false;
+    float mx = -INFINITY;
+#pragma unroll
+    for (int pp = 0; pp < 2 * DUP; ++pp) {
+      const int mr = (pp >> 1) * RPC + rr;
+      mx = fmaxf(mx, red[((pp & 1) * 4 + (mr >> 5)) * 32 + (mr & 31)]);
+    }
+    // 4. a rise by more than 2^8 rescales O and the row sums first
+    if (mx > m + kAttnRescale) {
+      const float alpha = (m == -INFINITY) ? 0.f : exp2f(m - mx);
+      if (cp == 0 && j > 0) {
+        if (!wwait(y.pv_done, (j - 1) & 1)) return false;
+        tc_fence_after();
+        uint32_t o32[32];
+        tmem_ld32_nowait(trow + 128 + half * 32, o32);
+        tmem_wait_ld();
+#pragma unroll
+        for (int k = 0; k < 32; ++k) o32[k] = __float_as_uint(alpha * __uint_as_float(o32[k]));
+        tmem_st32(trow + 128 + half * 32, o32);
+        tmem_wait_st();
+      }
+#pragma unroll
+      for (int c = 0; c < NCH; ++c) lc[c] *= alpha;
+      m = mx;
+    }
+    // 5. P_j = exp2(s - m) (fp16) into row rr of the P tile; 8-column sums
+    const float sub = (m == -INFINITY) ? 0.f : m;
+    uint8_t* prow = y.sP + buf * kAttnMaxRows * 128;
+#pragma unroll
+    for (int c = 0; c < NCH; ++c) {
+      float p[8];
+#pragma unroll
+      for (int e = 0; e < 8; ++e) p[e] = exp2f(sv[8 * c + e] - sub);
+      lc[c] += ((p[0] + p[1]) + (p[2] + p[3])) + ((p[4] + p[5]) + (p[6] + p[7]));
+      uint32_t w4[4];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        __half2 hv = __floats2half2_rn(p[2 * e], p[2 * e + 1]);
+        w4[e] = *reinterpret_cast<uint32_t*>(&hv);
+      }
+      *reinterpret_cast<uint4*>(prow + sw128(rr, col0 / 8 + c)) =
+          make_uint4(w4[0], w4[1], w4[2], w4[3]);
+    }
+    fence_proxy_async_smem();
+    tc_fence_before();
+    __syncwarp();
+    if (lane == 0) mbar_arrive(smem_u32(&y.p_full[buf]));
+  }
+  return true;
+}
+
+__global__ void __launch_bounds__(kAttnThreads, 2)
     attn_paged_kernel(const __grid_constant__ CUtensorMap tmKV, const AttnArgs a) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -123,22 +293,22 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   constexpr int rows_alloc = kAttnMaxRows;
   uint8_t* sQ = smem + kAttnQOff;
-  uint8_t* ring = smem + kAttnRingOff;                   // [stage][K | V^T]
   uint8_t* sP = smem + kAttnPOff;                        // [2][128][128 B]
-  float* recv = reinterpret_cast<float*>(smem + kAttnRecvOff);
+  uint8_t* ring = smem + kAttnRingOff;                   // [stage][K | V^T]
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kAttnBarOff);
   uint64_t* full = bars;                                 // [stages] TMA landed
   uint64_t* empty = bars + kAttnStages;                  // [stages] PV of the page done
   uint64_t* s_full = bars + 2 * kAttnStages;             // [2] S in TMEM
-  uint64_t* s_free = s_full + 2;                         // [2] S read by all 128 threads
-  uint64_t* p_full = s_full + 4;                         // [2] P in smem (128 arrivals)
-  uint64_t* pv_full = s_full + 6;                        // [2] PV in TMEM
-  uint64_t* mma_done = s_full + 8;                       // every MMA of this CTA retired
-  uint64_t* recv_bar = s_full + 9;
-  uint64_t* q_full = s_full + 10;                        // Q tile in smem (128 arrivals)
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(s_full + 11);
+  uint64_t* s_free = s_full + 2;                         // [2] S read by the 4 softmax warps
+  uint64_t* p_full = s_full + 4;                         // [2] P in smem (4 warp arrivals)
+  uint64_t* pv_done = s_full + 6;                        // O += P_j V_j retired (phase j)
+  uint64_t* mma_done = s_full + 7;                       // every MMA of this CTA retired
+  uint64_t* recv_bar = s_full + 8;
+  uint64_t* q_full = s_full + 9;                         // Q tile in smem (4 warp arrivals)
+  uint64_t* mx_bar = s_full + 10;                        // [2] page maxima exchanged
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(s_full + 12);
   // [0] max limit, [1] last-item flag, [2] pages the MMA warp took, [3] pages issued
-  int* s_int = reinterpret_cast<int*>(s_full + 12);
+  int* s_int = reinterpret_cast<int*>(s_full + 13);
 
   const int c = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
   const int seq = b / a.n_sub, sub = b % a.n_sub;
@@ -155,11 +325,11 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
   const int slot = a.blk_slot ? a.blk_slot[seq] : a.fixed_slot;
 
   if (warp == 0) {
-    int m = -1;
-    for (int i = lane; i < ntok; i += 32) m = max(m, a.lim[tok0 + i]);
+    int mxl = -1;
+    for (int i = lane; i < ntok; i += 32) mxl = max(mxl, a.lim[tok0 + i]);
 #pragma unroll
-    for (int o = 16; o >= 1; o >>= 1) m = max(m, __shfl_xor_sync(0xFFFFFFFFu, m, o));
-    if (lane == 0) s_int[0] = m;
+    for (int o = 16; o >= 1; o >>= 1) mxl = max(mxl, __shfl_xor_sync(0xFFFFFFFFu, mxl, o));
+    if (lane == 0) s_int[0] = mxl;
   }
   __syncthreads();
   const int maxlim = s_int[0];
@@ -173,6 +343,10 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
   }
   if (c >= nitems && (nitems == 1 || !a.cluster)) return;
   const bool in_cluster = a.cluster && nitems > 1;
+  if (c >= nitems) {   // idle cluster member: counts in the cluster barrier, owns nothing
+    cluster_arrive_release();
+    return;
+  }
 
   if (threadIdx.x == 0) {
     tma_prefetch_desc(&tmKV);
@@ -182,12 +356,19 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(smem_u32(&s_full[i]), 1);
-      mbar_init(smem_u32(&s_free[i]), 128);
-      mbar_init(smem_u32(&p_full[i]), 128);
-      mbar_init(smem_u32(&pv_full[i]), 1);
+      mbar_init(smem_u32(&s_free[i]), kAttnSoftWarps);   // one arrival per softmax warp
+      mbar_init(smem_u32(&p_full[i]), kAttnSoftWarps);
     }
+    mbar_init(smem_u32(pv_done), 1);
     mbar_init(smem_u32(mma_done), 1);
-    mbar_init(smem_u32(q_full), 128);
+    mbar_init(smem_u32(q_full), kAttnSoftWarps);
+    {
+      const int rpc = kAttnMaxRows / (R <= 32 ? 4 : (R <= 64 ? 2 : 1));
+      int nbusy = 0;   // softmax warps that hold rows
+      for (int w = 0; w < kAttnSoftWarps; ++w) nbusy += (((w & 3) * 32) % rpc) < R ? 1 : 0;
+      mbar_init(smem_u32(&mx_bar[0]), nbusy);
+      mbar_init(smem_u32(&mx_bar[1]), nbusy);
+    }
     if (in_cluster) {
       mbar_init(smem_u32(recv_bar), 1);
       // nitems sources, ceil(128 / nitems) rows each, arrive by bulk copy
@@ -198,12 +379,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     s_int[3] = 0;
     fence_mbar_init();
   }
-  if (in_cluster) {
-    __syncthreads();
-    cluster_arrive_release();   // waited on before the first remote access
-    if (c >= nitems) return;    // idle cluster member: arrived, owns nothing
-  }
-  if (warp == 5) tmem_alloc(smem_u32(tmem_slot), kAttnTmemCols);
+  if (warp == kAttnMmaWarp) tmem_alloc(smem_u32(tmem_slot), kAttnTmemCols);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -213,14 +389,12 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
   const int np = min(npages_blk, p_begin + SP) - p_begin;
   const int32_t* pt = a.page_table + static_cast<size_t>(slot) * a.pt_stride;
   bool ok = true;
-  // the row's state (softmax threads): O (unnormalised), running max m (log2
-  // units), running sum l
-  float o[64];
-#pragma unroll
-  for (int k = 0; k < 64; ++k) o[k] = 0.f;
-  float m = -INFINITY, l = 0.f;
+  float m = -INFINITY, l = 0.f;   // the row's running max (log2 units) and sum
+  float lc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};   // row sum, 8-column partials
+  float* red = reinterpret_cast<float*>(s_int + 8);        // [2][softmax threads] page maxima
+  float* lsum = red + 2 * kAttnSoftThreads;                // [8][128] partial sums
 
-  if (warp == 4) {
+  if (warp == kAttnTmaWarp) {
     // ---- TMA producer: K and V^T pages of the item, in order
     if (lane == 0) {
       const int safe_pages = a.blk_slot ? a.lim[tok0] / 64 : 0;   // wholly committed pages
@@ -258,8 +432,8 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
       pdl_wait();
       pdl_trigger();
     }
-  } else if (warp == 5) {
-    // ---- MMA issuer: S one page ahead of the softmax, PV after each P
+  } else if (warp == kAttnMmaWarp) {
+    // ---- MMA issuer: S one page ahead of the softmax, O += P V after each P
     pdl_wait();
     pdl_trigger();
     if (lane == 0) {
@@ -292,121 +466,76 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
         const uint64_t vdesc = umma_desc_sw128(smem_u32(ring + s * kAttnStageBytes + kAttnPageBytes));
 #pragma unroll
         for (int k = 0; k < 4; ++k)
-          umma_f16(tmem + 128 + buf * 64, pdesc + 2 * k, vdesc + 2 * k, idesc, k > 0 ? 1u : 0u);
-        umma_commit(smem_u32(&pv_full[buf]));
+          umma_f16(tmem + 128, pdesc + 2 * k, vdesc + 2 * k, idesc, (j > 0 || k > 0) ? 1u : 0u);
+        umma_commit(smem_u32(pv_done));
         umma_commit(smem_u32(&empty[s]));
       }
       umma_commit(smem_u32(mma_done));   // retires once every MMA above has
     }
   } else {
-    // ---- softmax warps: thread r owns row r (TMEM lane r)
-    const int r = threadIdx.x;
-    // Q rows -> swizzled smem (zero rows past R); the MMA reads all 128 rows
+    // ---- softmax warps: DUP copies of each row across the 128 MMA rows
+    const int dup = R <= 32 ? 4 : (R <= 64 ? 2 : 1);
+    const int rpc = kAttnMaxRows / dup;
+    // Q rows -> swizzled smem: MMA row i holds block row i % rpc (zero past R)
     pdl_wait();
     pdl_trigger();
-    for (int idx = threadIdx.x; idx < rows_alloc * 8; idx += 128) {
-      const int rr = idx >> 3, ch = idx & 7;
+    for (int idx = threadIdx.x; idx < rows_alloc * 8; idx += kAttnSoftThreads) {
+      const int i = idx >> 3, ch = idx & 7, rr = i % rpc;
       uint4 v = make_uint4(0, 0, 0, 0);
       if (rr < R) {
         const int t = tok0 + rr / a.G;
         const int hq = h * a.G + rr % a.G;
         v = *reinterpret_cast<const uint4*>(a.q + (static_cast<size_t>(t) * a.Hq + hq) * 64 + ch * 8);
       }
-      *reinterpret_cast<uint4*>(sQ + sw128(rr, ch)) = v;
+      *reinterpret_cast<uint4*>(sQ + sw128(i, ch)) = v;
     }
     fence_proxy_async_smem();
-    mbar_arrive(smem_u32(q_full));
-    const int lim_r = r < R ? a.lim[tok0 + r / a.G] : -1;
-    const uint32_t trow = tmem + (static_cast<uint32_t>(warp * 32) << 16);
-    const float kScaleLog2 = 0.125f * 1.4426950408889634f;   // 1/sqrt(64) in log2 units
-    float alpha_prev = 1.f;
-    // O = alpha O + PV_j, PV_j from TMEM buffer j & 1
-    auto apply_pv = [&](int j, float alpha) -> bool {
-      if (!mbar_wait(smem_u32(&pv_full[j & 1]), (j >> 1) & 1, a.err)) return false;
-      tc_fence_after();
-      uint32_t v0[32], v1[32];
-      tmem_ld32_nowait(trow + 128 + (j & 1) * 64, v0);
-      tmem_ld32_nowait(trow + 128 + (j & 1) * 64 + 32, v1);
-      tmem_wait_ld();
-#pragma unroll
-      for (int k = 0; k < 32; ++k) {
-        o[k] = alpha * o[k] + __uint_as_float(v0[k]);
-        o[32 + k] = alpha * o[32 + k] + __uint_as_float(v1[k]);
-      }
-      return true;
-    };
-    for (int j = 0; j < np; ++j) {
-      const int buf = j & 1;
-      // 1. S_j row from TMEM; the buffer is free again once all 128 rows are read
-      if (ok && !mbar_wait(smem_u32(&s_full[buf]), (j >> 1) & 1, a.err)) ok = false;
-      if (!ok) break;
-      tc_fence_after();
-      uint32_t s0[32], s1[32];
-      tmem_ld32_nowait(trow + buf * 64, s0);
-      tmem_ld32_nowait(trow + buf * 64 + 32, s1);
-      tmem_wait_ld();
-      tc_fence_before();
-      mbar_arrive(smem_u32(&s_free[buf]));
-      // 2. mask (keys past the row's limit), scale, running max, probabilities
-      const int key0 = (p_begin + j) * 64;
-      float sv[64];
-      float mx = -INFINITY;
-#pragma unroll
-      for (int k = 0; k < 64; ++k) {
-        const float x = __uint_as_float(k < 32 ? s0[k] : s1[k - 32]);
-        sv[k] = key0 + k <= lim_r ? x * kScaleLog2 : -INFINITY;
-        mx = fmaxf(mx, sv[k]);
-      }
-      const float m_new = fmaxf(m, mx);
-      const float alpha = (m_new == -INFINITY) ? 1.f : exp2f(m - m_new);
-      const float sub = (m_new == -INFINITY) ? 0.f : m_new;
-      uint32_t pk[32];
-      float ps[8];
-#pragma unroll
-      for (int cch = 0; cch < 8; ++cch) {
-        float p[8];
-#pragma unroll
-        for (int e = 0; e < 8; ++e) p[e] = exp2f(sv[8 * cch + e] - sub);
-        ps[cch] = ((p[0] + p[1]) + (p[2] + p[3])) + ((p[4] + p[5]) + (p[6] + p[7]));
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          __half2 hv = __floats2half2_rn(p[2 * e], p[2 * e + 1]);
-          pk[4 * cch + e] = *reinterpret_cast<uint32_t*>(&hv);
-        }
-      }
-      l = l * alpha + (((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7])));
-      m = m_new;
-      // 3. PV_{j-1} into O (it and everything before it retired: P buffer `buf` is free)
-      if (j >= 1 && !(ok = apply_pv(j - 1, alpha_prev))) break;
-      // 4. P_j (fp16) as the A operand of PV_j: row r, 128-byte swizzle
-      uint8_t* prow = sP + buf * kAttnMaxRows * 128;
-#pragma unroll
-      for (int cch = 0; cch < 8; ++cch)
-        *reinterpret_cast<uint4*>(prow + sw128(r, cch)) =
-            make_uint4(pk[4 * cch], pk[4 * cch + 1], pk[4 * cch + 2], pk[4 * cch + 3]);
-      fence_proxy_async_smem();
-      tc_fence_before();
-      mbar_arrive(smem_u32(&p_full[buf]));
-      alpha_prev = alpha;
-    }
-    if (ok && np > 0) ok = apply_pv(np - 1, alpha_prev);
-  }
+    __syncwarp();
+    if (lane == 0) mbar_arrive(smem_u32(q_full));
+    AttnSync y{s_full, s_free, p_full, pv_done, mx_bar, sP, red};
+    if (dup == 4) ok = attn_softmax<4>(a, y, tmem, np, p_begin, R, tok0, m, lc);
+    else if (dup == 2) ok = attn_softmax<2>(a, y, tmem, np, p_begin, R, tok0, m, lc);
+    else ok = attn_softmax<1>(a, y, tmem, np, p_begin, R, tok0, m, lc);
+    // the row's eight 8-column partial sums -> shared memory [chunk][row]
+    const int mrow = (warp & 3) * 32 + lane;
+    const int part = 2 * (mrow / rpc) + (warp >> 2), nch = 8 / (2 * dup);
+    for (int cc = 0; cc < nch; ++cc) lsum[(part * nch + cc) * kAttnMaxRows + mrow % rpc] = lc[cc];  }
 
   const bool all_ok = __syncthreads_and(ok);
-  // every MMA retired and every TMA copy landed before TMEM and the ring are released
-  if (warp == 5) {
-    if (lane == 0) mbar_wait(smem_u32(mma_done), 0, a.err);
-    __syncwarp();
-    tc_fence_after();
-    tmem_dealloc(tmem, kAttnTmemCols);
-  }
-  if (warp == 4 && lane == 0) {
+  // every MMA retired and every TMA copy landed before TMEM and the ring are reused
+  if (warp == kAttnMmaWarp && lane == 0) mbar_wait(smem_u32(mma_done), 0, a.err);
+  if (warp == kAttnTmaWarp && lane == 0) {
     for (int i = s_int[2]; i < s_int[3]; ++i)
       mbar_wait(smem_u32(&full[i % kAttnStages]), (i / kAttnStages) & 1, a.err);
   }
   __syncthreads();
+  // the row's O from TMEM and its sum from the four partials (rows < R)
   const int r = threadIdx.x;
   const bool row_thread = r < R;
+  if (row_thread) {
+    const float* ls = lsum + r;
+    l = ((ls[0 * kAttnMaxRows] + ls[1 * kAttnMaxRows]) + (ls[2 * kAttnMaxRows] + ls[3 * kAttnMaxRows])) +
+        ((ls[4 * kAttnMaxRows] + ls[5 * kAttnMaxRows]) + (ls[6 * kAttnMaxRows] + ls[7 * kAttnMaxRows]));
+  }
+  float o[64];
+  if (warp < 4) {
+    tc_fence_after();
+    uint32_t o0[32], o1[32];
+    tmem_ld32_nowait(tmem + (static_cast<uint32_t>(warp * 32) << 16) + 128, o0);
+    tmem_ld32_nowait(tmem + (static_cast<uint32_t>(warp * 32) << 16) + 128 + 32, o1);
+    tmem_wait_ld();
+#pragma unroll
+    for (int k = 0; k < 32; ++k) {
+      o[k] = __uint_as_float(o0[k]);
+      o[32 + k] = __uint_as_float(o1[k]);
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == kAttnMmaWarp) {
+    tc_fence_after();
+    tmem_dealloc(tmem, kAttnTmemCols);
+  }
 
   if (nitems == 1) {   // the block's only item: its rows are final
     if (row_thread && all_ok) {
@@ -437,21 +566,24 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
   };
 
   // Merged rows of one item: source `it`, row r -> float pointer (O[64], m, l).
-  // Cluster: recv[it][k] with r = c + k * nitems.  Global: part[b][h][it][r].
+  // Cluster: recv[it][k] (in the ring) with r = c + k * nitems.  Global:
+  // part[b][h][it][r].
   const size_t bh = static_cast<size_t>(b) * a.Hkv + h;
   float* part_bh = a.part + bh * a.max_items * rows_alloc * kAttnRow;
+  float* recv = reinterpret_cast<float*>(ring);
   const int rpo = (rows_alloc + nitems - 1) / nitems;   // cluster: rows per owner
   bool got = true;
   int my_rows;
   if (in_cluster) {
-    // ---- items -> owners.  stage [owner][slot][kAttnRow] in the ring.
-    float* stage = reinterpret_cast<float*>(ring);
+    // ---- items -> owners.  stage [owner][slot][kAttnRow] over Q and P.
+    float* stage = reinterpret_cast<float*>(sQ);
     const int blk_floats = rpo * kAttnRow;
     if (row_thread)
       put_row(stage + static_cast<size_t>(r % nitems) * blk_floats + (r / nitems) * kAttnRow);
     fence_proxy_async_smem();
     __syncthreads();
-    cluster_wait();   // every CTA of the cluster runs: peers' buffers and barriers exist
+    cluster_arrive_release();
+    cluster_wait();   // every CTA of the cluster is done with its pages: receive buffers idle
     if (threadIdx.x == 0) {
       const uint32_t bytes = static_cast<uint32_t>(blk_floats * 4);
       const uint32_t dst_local = smem_u32(recv) + static_cast<uint32_t>(c) * bytes;
@@ -496,9 +628,11 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
   //      copies have read it).
   if (in_cluster && threadIdx.x == 0) bulk_wait_read_all();
   __syncthreads();
-  float* mb = reinterpret_cast<float*>(ring);
+  // cluster: the received rows fill the ring, the tables go over Q and P (the
+  // outgoing copies have read them); global: the tables go in the ring
+  float* mb = reinterpret_cast<float*>(in_cluster ? sQ : ring);
   float* lb = mb + static_cast<size_t>(nitems) * rows_alloc;
-  const bool fits = 2 * nitems * rows_alloc <= kAttnRingBytes / 4;
+  const bool fits = 2 * nitems * rows_alloc * 4 <= (in_cluster ? kAttnRingOff : kAttnRingBytes);
   if (!fits && threadIdx.x == 0) atomicExch(a.err, kErrBounds);
   if (fits) {
     for (int idx = threadIdx.x; idx < nitems * my_rows; idx += blockDim.x) {
