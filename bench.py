@@ -1,22 +1,28 @@
-"""Benchmark: greedy self-speculative decoding rounds on one GB300 per rank.
+"""Benchmark: greedy self-speculative decoding on one GB300 per rank.
 
-Workload (default ``glm_b1``): the GLM-OCR-scale synthetic decoder (24 layers,
+Default workload ``glm_b1``: the GLM-OCR-scale synthetic decoder (24 layers,
 d_model 1024, 16 query / 8 KV heads, SwiGLU 4096, vocab 59392, random bf16
 weights), batch 1, prefix 2048 (1600 visual embeddings + 448 text tokens),
 block size K = 16, 512 output tokens, accepted draft lengths forced to a
-seeded censored-geometric schedule with mean 9.7.
+seeded censored-geometric schedule with mean 9.7.  ``--workload serve_b32``
+(32 sequences, prefixes U[1024, 6144]) and ``--workload long_b8`` (8 x prefix
+8192, K = 32, heavy-tailed acceptance) time the other configurations;
+``--K`` and ``--accept-mean`` override the block size and the forced mean
+(``--K 32 --accept-mean 17.4`` is the paper's TPF-9.7 operating point).
 
-A step is one complete decode of the 512 output tokens: the sequence state is
+A step is one complete decode of every sequence: the sequence states are
 rolled back to the end of the prefill (the prefill itself is untimed, as in
 the paper's TPF accounting) and every round of the schedule runs as one CUDA
 graph (draft forward -> forcing -> verify forward -> accept/commit).  The
-metric is committed tokens per second; per-round latencies come from CUDA
-events.  The 876.6 MB of weights every forward streams exceed the 129 MB L2,
-so no flush is needed between steps.
+metric is committed tokens per second over all sequences; per-round latencies
+come from CUDA events.  The 876.6 MB of weights every forward streams exceed
+the 129 MB L2, so no flush is needed between steps.  The same decode with
+K = 0 rounds (plain greedy AR, one token per forward) is timed on the same
+kernels for the speed-up the method buys.
 
 --impl reference times the float64 CPU oracle on this host's cores instead
-(one forced round per step).  Multi-GPU: replicas (one independent decode per
-rank, no collective on the data path).
+(forced rounds of the workload's shortest sequence).  Multi-GPU: replicas
+(one independent decode per rank, no collective on the data path).
 """
 from __future__ import annotations
 
@@ -144,6 +150,14 @@ def kernel_bytes(cfg, kind: str, T: int, ctx: list) -> int | None:
 
 
 # ---------------------------------------------------------------------- GPU arm
+def gemm_flops(cfg, kind: str, T: int) -> int | None:
+    """Multiply-add flops (x2) of one projection launch over T rows."""
+    d, F, V, HD = cfg.d_model, cfg.d_ffn, cfg.vocab, cfg.n_heads * cfg.head_dim
+    rows_k = {"qkv": (cfg.qkv_dim, d), "o_proj": (d, HD), "gate_up": (2 * F, d),
+              "down": (d, F), "lm_head": (V, d)}.get(kind)
+    return None if rows_k is None else 2 * T * rows_k[0] * rows_k[1]
+
+
 def gpu_arm(args, rank: int, world: int):
     import torch
     from paper_2609_26638_gb300 import gs
@@ -153,58 +167,72 @@ def gpu_arm(args, rank: int, world: int):
     torch.cuda.set_device(dev)
     wl = synth.WORKLOADS[args.workload]
     cfg = wl.model
-    assert wl.batch == 1, "the bench decodes one sequence per rank"
-    K, max_new = wl.K, wl.max_new
-    prompt = wl.prompts()[0]
-    P = prompt.length
+    K = wl.K if args.K is None else args.K
+    mean = wl.accept_mean if args.accept_mean is None else args.accept_mean
+    max_new = wl.max_new
+    prompts = wl.prompts()
+    B = len(prompts)
+    P = [p.length for p in prompts]
     weights = synth.make_weights(cfg)
     extra = K + 4
-    eng = Engine(cfg, weights, max_batch=1, max_ctx=P + max_new + extra + K + 2 + 64, max_K=K,
+    eng = Engine(cfg, weights, max_batch=B, max_ctx=max(P) + max_new + extra + K + 2 + 64, max_K=K,
                  max_prefill=2048, device=str(dev))
     del weights
-    x0 = eng.prefill(0, prompt.vis, prompt.text, max_new + extra)
+    stream = eng.stream
+    slots = torch.arange(B, dtype=torch.int32, device=dev)
+    out_tok = torch.zeros((B, K + 2), dtype=torch.int32, device=dev)
+    out_cnt = torch.zeros(B, dtype=torch.int32, device=dev)
+    out_done = torch.zeros(B, dtype=torch.int32, device=dev)
 
-    slots = torch.zeros(1, dtype=torch.int32, device=dev)
-    out_tok = torch.zeros((1, K + 2), dtype=torch.int32, device=dev)
-    out_cnt = torch.zeros(1, dtype=torch.int32, device=dev)
-    out_done = torch.zeros(1, dtype=torch.int32, device=dev)
-    torch.cuda.synchronize(dev)
+    def prefill_all(cap):
+        return [eng.prefill(i, p.vis, p.text, cap) for i, p in enumerate(prompts)]
 
-    # teacher: the greedy continuation, from natural rounds of the same shape
-    teacher_toks = [x0]
-    while True:
+    # teacher: the greedy continuation of every sequence, from natural rounds
+    x0 = prefill_all(max_new + extra)
+    teacher_toks = [[x] for x in x0]
+    for _ in range(max_new + extra):
         eng.round(slots, K, out_tok, out_cnt, out_done)
-        eng.stream.synchronize()
-        c = int(out_cnt.cpu()[0])
-        teacher_toks.extend(out_tok.cpu().numpy()[0, :c].tolist())
-        if int(out_done.cpu()[0]):
+        stream.synchronize()
+        c = out_cnt.cpu().numpy()
+        t = out_tok.cpu().numpy()
+        for i in range(B):
+            teacher_toks[i].extend(t[i, :c[i]].tolist())
+        if out_done.cpu().numpy().all():
             break
     eng.check()
-    teacher = np.full(P + len(teacher_toks) + 8, -1, np.int32)
-    teacher[P:P + len(teacher_toks)] = teacher_toks
-    sched_all = wl.schedule()                       # [1, max_rounds]
-    R = schedule_rounds(sched_all[0], max_new)
+    stride = max(P) + max_new + extra + K + 8
+    teacher = np.full((B, stride), -1, np.int32)
+    for i in range(B):
+        teacher[i, P[i]:P[i] + len(teacher_toks[i])] = teacher_toks[i]
+    kind = "geometric" if wl.accept in ("geometric", "natural") else wl.accept
+    sched_all = synth.accept_schedule(kind, K, B, wl.max_rounds(), mean)
+    Rb = [schedule_rounds(sched_all[i], max_new) for i in range(B)]
+    R = max(Rb)
     sched = np.ascontiguousarray(sched_all[:, :R + 1])
     t_dev = torch.from_numpy(teacher).to(dev)
     s_dev = torch.from_numpy(sched).to(dev)
-    force = gs.gs_force(teacher=t_dev.data_ptr(), teacher_stride=teacher.shape[0],
-                        L_sched=s_dev.data_ptr(), L_stride=sched.shape[1])
-    ring_tok = torch.zeros((R, K + 2), dtype=torch.int32, device=dev)
-    ring_cnt = torch.zeros(R, dtype=torch.int32, device=dev)
+    force = gs.gs_force(teacher=t_dev.data_ptr(), teacher_stride=stride, L_sched=s_dev.data_ptr(),
+                        L_stride=sched.shape[1])
+    ring_tok = torch.zeros((R, B, K + 2), dtype=torch.int32, device=dev)
+    ring_cnt = torch.zeros((R, B), dtype=torch.int32, device=dev)
     torch.cuda.synchronize(dev)
-    stream = eng.stream
 
-    def one_decode(evs=None):
-        eng.restore(0, P, x0, 1, max_new, 0, 0)
-        for r in range(R):
+    def restore_all():
+        for i in range(B):
+            eng.restore(i, P[i], x0[i], 1, max_new, 0, 0)
+
+    def one_decode(evs=None, Kr=K, frc=force, rounds=R, rt=ring_tok, rc=ring_cnt):
+        restore_all()
+        for r in range(rounds):
             if evs is not None:
                 evs[r][0].record(stream)
-            eng.round(slots, K, out_tok, out_cnt, out_done, force=force)
+            eng.round(slots, Kr, out_tok, out_cnt, out_done, force=frc)
             if evs is not None:
                 evs[r][1].record(stream)
-            with torch.cuda.stream(stream):
-                ring_tok[r].copy_(out_tok[0], non_blocking=True)
-                ring_cnt[r:r + 1].copy_(out_cnt, non_blocking=True)
+            if rt is not None:
+                with torch.cuda.stream(stream):
+                    rt[r].copy_(out_tok, non_blocking=True)
+                    rc[r].copy_(out_cnt, non_blocking=True)
 
     for _ in range(args.warmup):
         one_decode()
@@ -241,21 +269,24 @@ def gpu_arm(args, rank: int, world: int):
     round_ms = sorted(a.elapsed_time(b) for step in ev for (a, b) in step)
     eng.check()
 
-    # every forced round committed exactly L + 2 tokens and the output is the greedy one
+    # every forced round committed exactly L + 2 tokens (until the cap) and the
+    # output of every sequence is its greedy continuation
     cnt = ring_cnt.cpu().numpy()
     toks = ring_tok.cpu().numpy()
-    got = [x0]
-    for r in range(R):
-        got.extend(toks[r, :cnt[r]].tolist())
+    ok_sched, ok_tokens = True, True
+    for i in range(B):
+        got = [x0[i]]
+        for r in range(R):
+            got.extend(toks[r, i, :cnt[r, i]].tolist())
+        ok_tokens &= got == teacher_toks[i][:max_new]
+        ok_sched &= all(int(cnt[r, i]) == int(sched[i, r]) + 2 for r in range(Rb[i] - 1))
     committed_per_decode = int(cnt.sum())
-    ok_sched = all(int(cnt[r]) == int(sched[0, r]) + 2 for r in range(R - 1))
-    ok_tokens = got == teacher_toks[:max_new]
 
     # end to end: inputs from pinned host memory, outputs back to the host, every step
     h_teacher = torch.from_numpy(teacher).pin_memory()
     h_sched = torch.from_numpy(sched).pin_memory()
-    h_ring = torch.empty((R, K + 2), dtype=torch.int32).pin_memory()
-    h_cnt = torch.empty(R, dtype=torch.int32).pin_memory()
+    h_ring = torch.empty((R, B, K + 2), dtype=torch.int32).pin_memory()
+    h_cnt = torch.empty((R, B), dtype=torch.int32).pin_memory()
     barrier()
     e0 = time.perf_counter()
     for s in range(args.steps):
@@ -270,45 +301,87 @@ def gpu_arm(args, rank: int, world: int):
     barrier()
     e_elapsed = time.perf_counter() - e0
 
-    # per-kernel device times: the same forced decode once more, every round
+    # plain greedy AR on the same kernels (K = 0 rounds: two one-token forwards,
+    # two tokens per round), for the speed-up the method buys on this GPU
+    ar = None
+    if args.compare_ar:
+        R_ar = (max_new + 1) // 2
+        one_decode(Kr=0, frc=None, rounds=R_ar, rt=None)
+        stream.synchronize()
+        a0 = torch.cuda.Event(enable_timing=True)
+        a1 = torch.cuda.Event(enable_timing=True)
+        n_ar = max(1, min(args.steps, 3))
+        a0.record(stream)
+        for _ in range(n_ar):
+            one_decode(Kr=0, frc=None, rounds=R_ar, rt=None)
+        a1.record(stream)
+        stream.synchronize()
+        eng.check()
+        ar_s = a0.elapsed_time(a1) / 1e3 / n_ar
+        ar = {"value": round(B * (max_new - 1) / ar_s, 1), "unit": UNIT,
+              "ms_per_step": round(1e3 * ar_s, 3), "steps": n_ar, "rounds_per_step": R_ar}
+
+    # per-kernel device times: the forced decode once more, every round
     # enqueued eagerly with a CUDA event after each launch (gs_round_profile)
-    hbm, _, src = load_peaks()
+    hbm, bf16_tf, src = load_peaks()
     W = K + 1
+    T = B * W
     per = {}
-    eng.restore(0, P, x0, 1, max_new, 0, 0)
+    restore_all()
     for r in range(R):
-        ctx = [eng.state(0)["seq_len"] + W]
+        ctx = []
+        for i in range(B):
+            st = eng.state(i)
+            if not st["done"]:
+                ctx.append(st["seq_len"] + W)
         for name, ms in eng.round_profile(slots, K, out_tok, out_cnt, out_done, force=force):
-            e = per.setdefault(name, [0, 0.0, 0])
+            e = per.setdefault(name, [0, 0.0, 0, 0])
             e[0] += 1
             e[1] += ms
-            b = kernel_bytes(cfg, name, W, ctx)
-            e[2] += b or 0
+            e[2] += kernel_bytes(cfg, name, T, ctx) or 0
+            e[3] += gemm_flops(cfg, name, T) or 0
     eng.check()
     kernels = {}
-    for name, (n, ms, b) in sorted(per.items(), key=lambda kv: -kv[1][1]):
+    ridge = bf16_tf * 1e12 / (hbm * 1e9)
+    for name, (n, ms, b, f) in sorted(per.items(), key=lambda kv: -kv[1][1]):
         k = {"launches": n, "total_ms": round(ms, 3), "us_per_launch": round(1e3 * ms / n, 2)}
         if b:
             k["bytes_per_launch"] = b // n
             k["gb_s"] = round(b / (ms * 1e-3) / 1e9, 1)
             k["frac_hbm"] = round(b / (ms * 1e-3) / 1e9 / hbm, 4)
+        if f:
+            k["flops_per_launch"] = f // n
+            k["tflop_s"] = round(f / (ms * 1e-3) / 1e12, 1)
+            k["frac_tensor"] = round(f / (ms * 1e-3) / 1e12 / bf16_tf, 4)
+            k["bound"] = "tensor" if b and f / b > ridge else "hbm"
+        elif b:
+            k["bound"] = "hbm"
         kernels[name] = k
-    dom = max((n for n in kernels if "gb_s" in kernels[n]), key=lambda n: kernels[n]["total_ms"])
+    dom = max((n for n in kernels if "bound" in kernels[n]), key=lambda n: kernels[n]["total_ms"])
     dk = kernels[dom]
-    roof = {"kernel": f"{dom} (gemm_tc_kernel / attn_paged_kernel by kind), decode shape "
-                      f"{W} rows", "bound": "hbm", "achieved": dk["gb_s"], "peak": hbm,
-            "unit": "GB/s", "frac": dk["frac_hbm"], "peak_source": src,
-            "algorithmic_bytes_per_launch": dk["bytes_per_launch"],
-            "us_per_launch": dk["us_per_launch"], "launches_per_step": dk["launches"],
-            "timing": "CUDA events around each launch of one eagerly enqueued decode "
-                      "(no launch overlap)", "traffic": None}
-    lm = lm_head_roofline(eng, cfg, K, dev)
+    timing = "CUDA events around each launch of one eagerly enqueued decode (no launch overlap)"
+    if dk["bound"] == "tensor":
+        roof = {"kernel": f"{dom} (gemm_tc_kernel), {T} rows", "bound": "tensor",
+                "achieved": dk["tflop_s"], "peak": bf16_tf, "unit": "TFLOP/s",
+                "frac": dk["frac_tensor"], "peak_source": src + " bf16 burst (fp16 runs at the same rate)",
+                "algorithmic_flops_per_launch": dk["flops_per_launch"],
+                "us_per_launch": dk["us_per_launch"], "launches_per_step": dk["launches"],
+                "timing": timing, "traffic": None}
+    else:
+        roof = {"kernel": f"{dom} (gemm_tc_kernel / attn_paged_kernel by kind), {T} rows",
+                "bound": "hbm", "achieved": dk["gb_s"], "peak": hbm, "unit": "GB/s",
+                "frac": dk["frac_hbm"], "peak_source": src,
+                "algorithmic_bytes_per_launch": dk["bytes_per_launch"],
+                "us_per_launch": dk["us_per_launch"], "launches_per_step": dk["launches"],
+                "timing": timing, "traffic": None}
+    lm = lm_head_roofline(eng, cfg, K, dev) if B == 1 else None
     attn = attention_roofline(cfg, dev)
     res = dict(elapsed=elapsed, e2e_elapsed=e_elapsed, tokens=committed_per_decode * args.steps,
                round_ms=round_ms, rounds=R, launches_per_round=launches_per_round,
                ok_sched=ok_sched, ok_tokens=ok_tokens, clocks=clk.summary(), roofline=roof,
-               kernels=kernels, lm_head=lm, attention=attn, h2d=int(teacher.nbytes + sched.nbytes),
-               d2h=int(R * (K + 2) * 4 + R * 4), P=P, K=K, max_new=max_new)
+               kernels=kernels, lm_head=lm, attention=attn, ar=ar, B=B, K=K, mean=mean,
+               h2d=int(teacher.nbytes + sched.nbytes),
+               d2h=int(R * B * (K + 2) * 4 + R * B * 4), max_new=max_new)
     eng.close()
     return res
 
@@ -405,20 +478,24 @@ def attention_roofline(cfg, dev):
 
 
 # ---------------------------------------------------------------------- oracle arm
-def oracle_sample(wl, n_rounds: int, warmup: int, budget_s: float):
+def oracle_sample(wl, n_rounds: int, warmup: int, budget_s: float, K: int, mean: float):
     """Forced self-speculative rounds of the float64 oracle on this host's cores.
 
-    The oracle's own greedy AR continuation is the forcing teacher; the sample
-    is the first rounds of the workload's decode (prefill and teacher untimed).
-    Returns (per-round seconds, committed tokens per timed round).
+    The sample is the workload's shortest-prefix sequence (the oracle decodes
+    one sequence at a time, so its tokens/s is the same for any batch): its
+    own greedy AR continuation is the forcing teacher, the timed rounds are the
+    first rounds of its forced decode (prefill and teacher untimed).  Returns
+    (per-round seconds, committed tokens per timed round, prefix length).
     """
     from oracle import decode as od
     from oracle.model import Decoder
     cfg = wl.model
-    K = wl.K
-    prompt = wl.prompts()[0]
+    prompts = wl.prompts()
+    idx = min(range(len(prompts)), key=lambda i: prompts[i].length)
+    prompt = prompts[idx]
     dec = Decoder(cfg, synth.make_weights(cfg))
-    sched = wl.schedule()[0]
+    kind = "geometric" if wl.accept in ("geometric", "natural") else wl.accept
+    sched = synth.accept_schedule(kind, K, len(prompts), wl.max_rounds(), mean)[idx]
     total = warmup + n_rounds
     need = int(sum(int(sched[r]) + 2 for r in range(total))) + K + 4
     cap = prompt.length + need + K + 8
@@ -442,7 +519,27 @@ def oracle_sample(wl, n_rounds: int, warmup: int, budget_s: float):
                 break
         if st.done:
             break
-    return times, counts
+    return times, counts, P
+
+
+def describe(wl, K: int, mean: float, world: int) -> dict:
+    prompts = wl.prompts()
+    if wl.prefix_min == wl.prefix_max:
+        n_vis = int(prompts[0].vis.shape[0])
+        prefix = f"prefix {wl.prefix_min} ({n_vis} visual + {wl.prefix_min - n_vis} text)"
+    else:
+        prefix = (f"prefixes U[{wl.prefix_min}, {wl.prefix_max}] ({round(100 * wl.vis_frac)}% visual, "
+                  f"64-token pages, ragged)")
+    accept = {"geometric": f"censored geometric, mean accepted length {mean}",
+              "heavy": f"10% L=K, 10% L=0, else geometric; mean accepted length {mean}",
+              "natural": f"censored geometric, mean accepted length {mean}"}[wl.accept]
+    return {"workload": f"{wl.name}: GLM-OCR-scale synthetic decoder L24 d1024 H16/8 F4096 V59392, "
+                        f"batch {wl.batch}, {prefix}, K={K}, {wl.max_new} output tokens per "
+                        f"sequence, forced acceptance ({accept})",
+            "model": "synthetic random-init bf16 weights (seed 0)",
+            "global_batch": wl.batch * max(world, 1), "K": K, "max_new": wl.max_new,
+            "l2": "inputs larger than L2: 876.6 MB of weights streamed per forward",
+            "parallelism": f"replicas x{max(world, 1)}"}
 
 
 def main():
@@ -451,29 +548,31 @@ def main():
     ap.add_argument("--steps", type=int, default=10)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="gpu", choices=["gpu", "reference"])
-    ap.add_argument("--workload", default="glm_b1")
+    ap.add_argument("--workload", default="glm_b1", choices=sorted(synth.WORKLOADS))
+    ap.add_argument("--K", type=int, default=None, help="block size (default: the workload's)")
+    ap.add_argument("--accept-mean", type=float, default=None,
+                    help="mean forced accepted length (default: the workload's)")
+    ap.add_argument("--no-compare-ar", dest="compare_ar", action="store_false",
+                    help="skip timing plain greedy AR (K = 0 rounds) on the same workload")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     args = ap.parse_args()
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     wl = synth.WORKLOADS[args.workload]
-    config = {"workload": f"{wl.name}: GLM-OCR-scale synthetic decoder L24 d1024 H16/8 F4096 V59392, "
-                          f"batch 1, prefix {wl.prefix_min} (1600 visual + 448 text), K={wl.K}, "
-                          f"{wl.max_new} output tokens, forced acceptance censored geometric mean 9.7",
-              "model": "synthetic random-init bf16 (seed 0)", "global_batch": wl.batch * max(world, 1),
-              "K": wl.K, "max_new": wl.max_new,
-              "l2": "inputs larger than L2: 876.6 MB of weights streamed per forward",
-              "parallelism": f"replicas x{max(world, 1)}"}
+    K = wl.K if args.K is None else args.K
+    mean = wl.accept_mean if args.accept_mean is None else args.accept_mean
+    config = describe(wl, K, mean, world)
 
     if args.impl == "reference":
         if rank != 0:
             return
         t0 = time.perf_counter()
-        times, counts = oracle_sample(wl, args.steps, args.warmup, budget_s=240.0)
+        times, counts, P0 = oracle_sample(wl, args.steps, args.warmup, 240.0, K, mean)
         value = sum(counts) / sum(times)
         cores = os.cpu_count()
-        sample = (f"{len(times)} forced rounds of the {wl.name} decode (after {args.warmup} warm-up "
-                  f"rounds), float64 oracle, prefill and teacher untimed")
+        sample = (f"{len(times)} forced rounds (after {args.warmup} warm-up rounds) of the "
+                  f"prefix-{P0} sequence of {wl.name}, float64 oracle on all host cores "
+                  f"(numpy/OpenBLAS), prefill and teacher untimed")
         line = {"impl": "reference", "metric": METRIC, "value": round(value, 3), "unit": UNIT,
                 "n_gpus": args.gpus, "steps": len(times), "warmup": args.warmup,
                 "ms_per_step": round(1e3 * statistics.mean(times), 2), "higher_is_better": True,
@@ -502,6 +601,7 @@ def main():
     tokens_all = res["tokens"] * max(world, 1)
     value = tokens_all / el
     rms = res["round_ms"]
+    B = res["B"]
     line = {"metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": max(world, 1),
             "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": round(1e3 * el / args.steps, 3), "higher_is_better": True,
@@ -510,22 +610,28 @@ def main():
             "round_p50_ms": round(rms[len(rms) // 2], 4),
             "round_p90_ms": round(rms[int(len(rms) * 0.9)], 4),
             "rounds_per_step": res["rounds"],
-            "committed_per_round": round(res["tokens"] / (args.steps * res["rounds"]), 3),
-            "tpf": round(res["tokens"] / (args.steps * res["rounds"] * 2), 3),
+            "committed_per_round_per_seq": round(res["tokens"] / (args.steps * res["rounds"] * B), 3),
+            "tpf": round(res["tokens"] / (args.steps * res["rounds"] * 2 * B), 3),
             "forced_schedule_hit": res["ok_sched"], "tokens_match_greedy": res["ok_tokens"],
             "gpu_launches": res["launches_per_round"] * res["rounds"] * args.steps
-            + args.steps,
+            + args.steps * B,
             "e2e": {"value": round(tokens_all / ee, 1), "unit": UNIT,
                     "h2d_bytes_per_step": res["h2d"], "d2h_bytes_per_step": res["d2h"]},
             "clocks": res["clocks"], "roofline": res["roofline"], "kernels": res["kernels"],
-            "lm_head_alone": res["lm_head"], "attention_roofline": res["attention"]}
+            "attention_roofline": res["attention"]}
+    if res["lm_head"] is not None:
+        line["lm_head_alone"] = res["lm_head"]
+    if res["ar"] is not None:
+        line["greedy_ar"] = res["ar"]
+        line["speedup_vs_greedy_ar"] = round(value / (res["ar"]["value"] * max(world, 1)), 3)
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        times, counts = oracle_sample(synth.WORKLOADS[args.workload], 6, 1, budget_s=25.0)
+        times, counts, P0 = oracle_sample(wl, 6, 1, 25.0, K, mean)
         line["cpu_baseline"] = {
             "value": round(sum(counts) / sum(times), 3), "unit": UNIT, "cores": os.cpu_count(),
             "kind": "oracle",
-            "sample": f"{len(times)} forced rounds (after 1 warm-up) of the same decode, float64 "
-                      f"oracle with numpy/OpenBLAS threads on all host cores"}
+            "sample": f"{len(times)} forced rounds (after 1 warm-up) of the prefix-{P0} sequence "
+                      f"of the same workload, float64 oracle with numpy/OpenBLAS threads on all "
+                      f"host cores"}
     if rank == 0:
         print(json.dumps(line))
     if world > 1:

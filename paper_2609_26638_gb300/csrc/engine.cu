@@ -101,7 +101,7 @@ cudaError_t launch_attention(const CUtensorMap& tm, const AttnArgs& a, int n_blo
 }
 
 struct GemmPlan {
-  int bn, tok_tiles, feat_tiles, splits;
+  int bn, tok_tiles, feat_tiles, splits, chunks;
 };
 
 // Split-K factor of a weight matrix in decode rounds.  It depends on the
@@ -122,13 +122,28 @@ int decode_splits(int weight_rows, int K) {
   return s;
 }
 
-GemmPlan plan_gemm(int weight_rows, int K, int T, bool decode) {
+// Decode windows of up to 64 tokens split K across the CTAs of a cluster;
+// wider decode launches reduce the same K chunks inside each CTA (one TMEM
+// accumulator per chunk, summed in chunk order), with the token tile shrunk
+// until the launch covers about one wave.  Prefill does not split K.
+GemmPlan plan_split(int weight_rows, int T, int S) {
   GemmPlan p;
-  p.bn = gemm_bn_for(T);
-  p.tok_tiles = cdiv(T, p.bn);
   p.feat_tiles = weight_rows / 128;
-  p.splits = decode ? decode_splits(weight_rows, K) : 1;
+  p.chunks = 1;
+  p.splits = S;
+  p.bn = gemm_bn_for(T);
+  if (S > 1 && T > 64 && S * 32 <= 512) {
+    p.chunks = S;
+    p.splits = 1;
+    p.bn = std::min(128, 512 / S);
+    while (p.bn > 32 && p.feat_tiles * cdiv(T, p.bn) < 148) p.bn /= 2;
+  }
+  p.tok_tiles = cdiv(T, p.bn);
   return p;
+}
+
+GemmPlan plan_gemm(int weight_rows, int K, int T, bool decode) {
+  return plan_split(weight_rows, T, decode ? decode_splits(weight_rows, K) : 1);
 }
 
 // fp32 partials the widest decode tiles (BN > 64, reduced through global
@@ -412,6 +427,7 @@ int run_gemm(gs_handle* h, const CUtensorMap& tw, int weight_rows, const CUtenso
   a.M = T;
   a.K = K;
   a.splits = p.splits;
+  a.chunks = p.chunks;
   a.kb_per_split = (K / 64) / p.splits;
   a.cluster = gemm_cluster_ok(p.bn, p.splits) ? 1 : 0;
   if (p.splits > 1 && !a.cluster &&
@@ -1120,12 +1136,19 @@ int gs_attention(int mode, const void* q, const void* kv, int n_pages, const int
 
 size_t gs_linear_scratch_bytes(int M, int N, int split_k) {
   if (M < 1 || N < 64 || split_k < 1) return 0;
-  const int bn = gemm_bn_for(M);
-  const size_t tiles = static_cast<size_t>(cdiv(M, bn)) * cdiv(N, 64);
+  // the larger of the plans for an N-row and a 2N-row (SwiGLU) weight
+  size_t counters = 0, partial = 0;
+  for (int w_rows : {N, 2 * N}) {
+    const GemmPlan p = plan_split(w_rows, M, split_k);
+    counters = std::max(counters, static_cast<size_t>(p.tok_tiles) * p.feat_tiles);
+    if (p.splits > 1 && !gemm_cluster_ok(p.bn, p.splits))
+      partial = std::max(partial, static_cast<size_t>(p.splits) * p.tok_tiles * p.feat_tiles *
+                                      p.bn * 128);
+  }
   Carver cv(nullptr);
   cv.take<int>(64);
-  cv.take<int>(tiles);
-  if (split_k > 1) cv.take<float>(static_cast<size_t>(split_k) * tiles * bn * 128);
+  cv.take<int>(counters);
+  if (partial) cv.take<float>(partial);
   return align_up(cv.off, 256);
 }
 
@@ -1145,26 +1168,28 @@ int gs_linear(const void* x, const void* w, void* y, int M, int N, int K, int ep
     if (gemm_init_attributes() != cudaSuccess) return GS_ERR_CUDA;
     attrs = true;
   }
-  const int bn = gemm_bn_for(M);
-  const int tok_tiles = cdiv(M, bn);
+  // split-K as the decoder plans it: across the CTAs of a cluster (up to 64
+  // rows), as chunks inside each CTA (wider), else through global scratch
   const int w_rows = epilogue == kEpiSwiGLU ? 2 * N : N;
-  const int feat_tiles = w_rows / 128;
+  const GemmPlan p = plan_split(w_rows, M, split_k);
+  const int bn = p.bn, tok_tiles = p.tok_tiles, feat_tiles = p.feat_tiles;
   CUtensorMap tw, tx;
   if (!make_map(&tw, w, w_rows, K, epilogue == kEpiSwiGLU ? 64 : 128)) return GS_ERR_INVALID_ARG;
   if (!make_map(&tx, x, M, K, bn)) return GS_ERR_INVALID_ARG;
   Carver cv(scratch);
   GemmArgs a = {};
   a.err = cv.take<int>(64);
-  a.counters = cv.take<int>(static_cast<size_t>(tok_tiles) * cdiv(N, 64));
-  a.partial = split_k > 1
-                  ? cv.take<float>(static_cast<size_t>(split_k) * tok_tiles * feat_tiles * bn * 128)
+  a.counters = cv.take<int>(static_cast<size_t>(tok_tiles) * feat_tiles);
+  a.cluster = p.splits > 1 && gemm_cluster_ok(bn, p.splits) ? 1 : 0;
+  a.partial = p.splits > 1 && !a.cluster
+                  ? cv.take<float>(static_cast<size_t>(p.splits) * tok_tiles * feat_tiles * bn * 128)
                   : nullptr;
   a.M = M;
   a.N = N;
   a.K = K;
-  a.splits = split_k;
-  a.kb_per_split = (K / 64) / split_k;
-  a.cluster = gemm_cluster_ok(bn, split_k) ? 1 : 0;
+  a.splits = p.splits;
+  a.chunks = p.chunks;
+  a.kb_per_split = (K / 64) / a.splits;
   a.y = y;
   a.ldy = N;
   a.logits = nullptr;

@@ -7,7 +7,7 @@ namespace gs {
 template <int BN, int EPI>
 static cudaError_t launch_one(const CUtensorMap& tmW, const CUtensorMap& tmX, const GemmArgs& a,
                               int feat_tiles, int tok_tiles, cudaStream_t s, bool pdl) {
-  dim3 grid(feat_tiles, tok_tiles, a.splits);
+  dim3 grid(tok_tiles, feat_tiles, a.splits);
   const int cz = (a.splits > 1 && a.cluster) ? a.splits : 1;
   return launch_ex(gemm_tc_kernel<BN, EPI>, grid, dim3(128), GemmShape<BN>::kSmemBytes, s, pdl,
                    dim3(1, 1, cz), tmW, tmX, a);

@@ -57,6 +57,7 @@ struct GemmArgs {
   int splits;       // split-K factor (divides K / 64)
   int kb_per_split; // (K / 64) / splits
   int cluster;      // 1: split-K partials reduced inside a cluster of `splits` CTAs
+  int chunks;       // splits == 1: K reduced in this many chunks inside the CTA (>= 1)
   void* y;          // output: fp16 [M, ldy] | fp32 [M, ldy] | uint64 [M] (argmax)
   int ldy;
   float* partial;   // global split-K partials [splits][tiles][BN][128] fp32 (cluster == 0)
@@ -95,6 +96,8 @@ struct GemmShape {
   static constexpr int kXBufBytes = 32 * 128 * 4;  // epilogue exchange (SwiGLU, RoPE, sums)
   static_assert(kRedBytes + kXBufBytes <= kStages * kStageBytes, "reduction smem");
   static_assert(!(BN <= 64) || kXBufBytes + BN * 128 * 4 <= kStages * kStageBytes, "staging smem");
+  // argmax epilogue: keys [128][33] and quarter maxima [4][32], 8 bytes each
+  static_assert((128 * 33 + 4 * 32) * 8 <= kStages * kStageBytes, "argmax smem");
   // RoPE cos/sin rows of the tile's tokens, staged while the mainloop runs (decode tiles)
   static constexpr bool kStageRope = BN <= 64;
   static constexpr int kRopeBytes = kStageRope ? BN * 32 * 8 : 0;
@@ -266,18 +269,33 @@ __device__ __forceinline__ void gemm_epilogue_chunk(const GemmArgs& a, float (&v
       for (int j = 0; j < EW; ++j)
         if (j >= jlo && j < jhi) a.logits[static_cast<size_t>(t0 + j) * a.N + f] = v[j];
     }
+    // keys [row][slot] in shared memory (row stride EW + 1 keys), then thread
+    // (slot j, row quarter q) takes the max over its 32 rows, and the first
+    // warp the max over the four quarters: one atomicMax per token per CTA
+    unsigned long long* kb = reinterpret_cast<unsigned long long*>(xbuf);
+    constexpr int LD = EW + 1;
 #pragma unroll
-    for (int j = 0; j < EW; ++j) {
-      if (j >= jlo && j < jhi) {   // uniform across the CTA
-        unsigned long long key = argmax_key(v[j], f);
-#pragma unroll
-        for (int m = 16; m >= 1; m >>= 1) {
-          const unsigned long long o = shfl_xor_u64(key, m);
-          key = o > key ? o : key;
-        }
-        if (lane == 0) atomicMax(out + t0 + j, key);
+    for (int j = 0; j < EW; ++j) kb[row * LD + j] = argmax_key(v[j], f);
+    asm volatile("bar.sync 2, 128;" ::: "memory");
+    unsigned long long* qb = kb + 128 * LD;   // [4][EW] quarter maxima
+    if (threadIdx.x < 4 * EW) {
+      const int j = threadIdx.x % EW, q = threadIdx.x / EW;
+      unsigned long long best = 0;
+      for (int rr = 0; rr < 32; ++rr) {
+        const unsigned long long k = kb[(q * 32 + rr) * LD + j];
+        best = k > best ? k : best;
       }
+      qb[q * EW + j] = best;
     }
+    asm volatile("bar.sync 2, 128;" ::: "memory");
+    if (threadIdx.x < EW) {
+      const int j = threadIdx.x;
+      unsigned long long best = qb[j];
+#pragma unroll
+      for (int q = 1; q < 4; ++q) best = qb[q * EW + j] > best ? qb[q * EW + j] : best;
+      if (j >= jlo && j < jhi) atomicMax(out + t0 + j, best);
+    }
+    asm volatile("bar.sync 2, 128;" ::: "memory");
   }
 }
 
@@ -301,8 +319,10 @@ __global__ void __launch_bounds__(128, 1)
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  const int feat_tile = blockIdx.x;
-  const int tok_tile = blockIdx.y;
+  // token tiles vary fastest, so the CTAs that share a weight tile run together
+  // and read it from DRAM once
+  const int tok_tile = blockIdx.x;
+  const int feat_tile = blockIdx.y;
   const int split = blockIdx.z;
   const int kb0 = split * a.kb_per_split;
   const int nkb = a.kb_per_split;
@@ -325,7 +345,10 @@ __global__ void __launch_bounds__(128, 1)
     }
     fence_mbar_init();
   }
-  if (warp == 2) tmem_alloc(smem_u32(tmem_slot), S::kTmemCols);
+  // chunked K: one TMEM accumulator of BN columns per chunk
+  const int nchunk = a.chunks > 1 ? a.chunks : 1;
+  const uint32_t tmem_cols = static_cast<uint32_t>(S::kTmemCols * nchunk);
+  if (warp == 2) tmem_alloc(smem_u32(tmem_slot), tmem_cols);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -428,8 +451,10 @@ __global__ void __launch_bounds__(128, 1)
       }
     }
     if (warp == 1 && lane == 0) {
-      // MMA issuer
+      // MMA issuer.  Chunked K: chunk c (k-blocks [c*kpc, (c+1)*kpc)) starts a
+      // fresh accumulator at TMEM column c * BN.
       constexpr uint32_t idesc = umma_idesc_f16(128, BN);
+      const int kpc = nkb / nchunk;
       for (int i = 0; i < nkb; ++i) {
         const int s = i % S::kStages;
         const uint32_t ph = (i / S::kStages) & 1;
@@ -437,9 +462,11 @@ __global__ void __launch_bounds__(128, 1)
         tc_fence_after();
         const uint64_t ad = umma_desc_sw128(smem_u32(smA + s * S::kABytes));
         const uint64_t bd = umma_desc_sw128(smem_u32(smB + s * S::kBBytes));
+        const uint32_t dst = tmem + static_cast<uint32_t>((i / kpc) * BN);
+        const bool fresh = (i % kpc) == 0;
 #pragma unroll
         for (int k = 0; k < 4; ++k)
-          umma_f16(tmem, ad + 2 * k, bd + 2 * k, idesc, (i > 0 || k > 0) ? 1u : 0u);
+          umma_f16(dst, ad + 2 * k, bd + 2 * k, idesc, (!fresh || k > 0) ? 1u : 0u);
         umma_commit(smem_u32(&empty[s]));
       }
       umma_commit(smem_u32(accum));
@@ -453,9 +480,9 @@ __global__ void __launch_bounds__(128, 1)
   const int row = warp * 32 + lane;      // TMEM lane = weight row of the tile
   const uint32_t trow = tmem + (static_cast<uint32_t>(warp * 32) << 16);
   const int tok0 = tok_tile * BN;
-  const bool failed = !acc_ok || *flag;
-  // per-token epilogue inputs staged by warps 2-3 during the mainloop
-  __syncthreads();
+  // per-token epilogue inputs staged by warps 2-3 during the mainloop; the
+  // failure flag is made uniform so every barrier below is reached by all
+  const bool failed = __syncthreads_or(!acc_ok || *flag) != 0;
   const float* rs_s = reinterpret_cast<const float*>(smem + S::kStages * S::kStageBytes + 256);
   const long long* kvdst_s = reinterpret_cast<const long long*>(rs_s + BN);
   const int* pos_s = reinterpret_cast<const int*>(kvdst_s + BN);
@@ -471,13 +498,26 @@ __global__ void __launch_bounds__(128, 1)
       for (int c = 0; c < BN / 32; ++c) {
         if (tok0 + c * 32 >= a.M) break;   // uniform across the CTA
         float v[32];
-        tmem_ld_32x32b_x32(trow + c * 32, v);
+        if (nchunk == 1) {
+          tmem_ld_32x32b_x32(trow + c * 32, v);
+        } else {
+          // the chunks' partial sums in chunk order from zero: the same sums,
+          // in the same order, as split-K across CTAs
+#pragma unroll
+          for (int j = 0; j < 32; ++j) v[j] = 0.0f;
+          for (int ch = 0; ch < nchunk; ++ch) {
+            float w[32];
+            tmem_ld_32x32b_x32(trow + ch * BN + c * 32, w);
+#pragma unroll
+            for (int j = 0; j < 32; ++j) v[j] += w[j];
+          }
+        }
         gemm_epilogue_chunk<BN, EPI, 32>(a, v, row, feat_tile, tok0 + c * 32, 0, 32, xbuf, rs_of(c));
       }
     }
     tc_fence_before();
     __syncthreads();
-    if (warp == 2) tmem_dealloc(tmem, S::kTmemCols);
+    if (warp == 2) tmem_dealloc(tmem, tmem_cols);
     return;
   }
 
@@ -505,7 +545,7 @@ __global__ void __launch_bounds__(128, 1)
       fence_proxy_async_smem();
       tc_fence_before();
       __syncthreads();
-      if (warp == 2) tmem_dealloc(tmem, S::kTmemCols);
+      if (warp == 2) tmem_dealloc(tmem, tmem_cols);
       const uint32_t slice_bytes = static_cast<uint32_t>(per * 128 * 4);
       cluster_wait();       // every CTA of the cluster runs: peers' buffers and barriers exist
       if (threadIdx.x == 0) {
@@ -516,7 +556,9 @@ __global__ void __launch_bounds__(128, 1)
                             cluster_map(smem_u32(recv_bar), static_cast<uint32_t>(q)));
         bulk_commit();
       }
-      const bool got = mbar_wait(smem_u32(recv_bar), 0, a.err);
+      const bool got = __syncthreads_and(mbar_wait(smem_u32(recv_bar), 0, a.err)) != 0;
+      if (threadIdx.x == 0) bulk_wait_read_all();   // our outgoing slices have left `stage`
+      __syncthreads();                              // (the epilogue reuses that memory)
       const int lo = split * per, hi = min(lo + per, ntok);
       if (hi > lo && !failed && got) {
         const int nq = hi - lo;
@@ -545,14 +587,13 @@ __global__ void __launch_bounds__(128, 1)
                                            rs_of(c));
         }
       }
-      if (threadIdx.x == 0) bulk_wait_read_all();   // our outgoing slices have left `stage`
       return;
     }
   }
 
   // global split-K: write this split's partial tile, token-major [BN][128]
   const int tiles = gridDim.x * gridDim.y;
-  const int tile = tok_tile * gridDim.x + feat_tile;
+  const int tile = feat_tile * gridDim.x + tok_tile;
   float* mine = a.partial + (static_cast<size_t>(split) * tiles + tile) * (BN * 128);
   if (!failed) {
     for (int c = 0; c < BN / 32; ++c) {
@@ -566,7 +607,7 @@ __global__ void __launch_bounds__(128, 1)
   __threadfence();
   tc_fence_before();
   __syncthreads();
-  if (warp == 2) tmem_dealloc(tmem, S::kTmemCols);
+  if (warp == 2) tmem_dealloc(tmem, tmem_cols);
   __shared__ int is_last;
   if (threadIdx.x == 0) {
     const int old = atomicAdd(a.counters + tile, 1);

@@ -78,4 +78,6 @@ def test_entry_points_validate_before_launch(gs):
         gs.GS_ERR_INVALID_ARG
     assert gs.gs_attention_scratch_bytes(2, 17, 16, 8, 40, 2) > 0
     assert gs.gs_attention_scratch_bytes(2, 17, 16, 7, 40, 2) == 0
-    assert gs.gs_linear_scratch_bytes(17, 2048, 8) > gs.gs_linear_scratch_bytes(17, 2048, 1)
+    # cluster split-K (<= 8 splits at <= 64 rows) needs no partials; 32 splits reduce through scratch
+    assert gs.gs_linear_scratch_bytes(17, 2048, 8) == gs.gs_linear_scratch_bytes(17, 2048, 1)
+    assert gs.gs_linear_scratch_bytes(17, 2048, 32) > gs.gs_linear_scratch_bytes(17, 2048, 1)

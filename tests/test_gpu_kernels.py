@@ -38,7 +38,8 @@ def _linear(gs, x, w, M, N, K, epi, split, y):
 
 
 @pytest.mark.parametrize("M", [1, 17, 33, 100, 264, 544])
-@pytest.mark.parametrize("N,K,split", [(256, 256, 1), (2048, 1024, 8), (1024, 4096, 16)])
+@pytest.mark.parametrize("N,K,split", [(256, 256, 1), (2048, 1024, 8), (1024, 4096, 16),
+                                       (1024, 4096, 32)])
 def test_linear_store_and_residual(gs, M, N, K, split):
     g = torch.Generator(device=DEV).manual_seed(M * 7 + N)
     x = torch.randn(M, K, device=DEV, generator=g).half()
