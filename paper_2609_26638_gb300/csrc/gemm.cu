@@ -5,11 +5,18 @@
 namespace gs {
 
 template <int BN, int EPI>
-static cudaError_t launch_one(const CUtensorMap& tmW, const CUtensorMap& tmX, const GemmArgs& a,
+static cudaError_t launch_one(const CUtensorMap& tmW, const CUtensorMap& tmX, GemmArgs a,
                               int feat_tiles, int tok_tiles, cudaStream_t s, bool pdl) {
+  using S = GemmShape<BN>;
+  // stages: a depth that leaves room for a second resident CTA per SM (it
+  // starts as soon as the first releases TMEM, with no launch gap), never more
+  // than the k-blocks one CTA loads
+  const int want = S::kStagesDefault;
+  const int kb = a.kb_per_split;
+  a.stages = kb < S::kStagesMin ? S::kStagesMin : (kb > want ? want : kb);
   dim3 grid(tok_tiles, feat_tiles, a.splits);
   const int cz = (a.splits > 1 && a.cluster) ? a.splits : 1;
-  return launch_ex(gemm_tc_kernel<BN, EPI>, grid, dim3(128), GemmShape<BN>::kSmemBytes, s, pdl,
+  return launch_ex(gemm_tc_kernel<BN, EPI>, grid, dim3(128), S::smem_bytes(a.stages), s, pdl,
                    dim3(1, 1, cz), tmW, tmX, a);
 }
 
@@ -40,7 +47,7 @@ cudaError_t launch_gemm(int bn, int epi, const CUtensorMap& tmW, const CUtensorM
 
 template <int BN>
 static cudaError_t set_attr_bn() {
-  const int bytes = GemmShape<BN>::kSmemBytes;
+  const int bytes = GemmShape<BN>::smem_bytes(GemmShape<BN>::kStagesMax);
   cudaError_t e;
   if ((e = cudaFuncSetAttribute(gemm_tc_kernel<BN, kEpiStoreF16>,
                                 cudaFuncAttributeMaxDynamicSharedMemorySize, bytes)) != cudaSuccess)

@@ -58,6 +58,7 @@ struct GemmArgs {
   int kb_per_split; // (K / 64) / splits
   int cluster;      // 1: split-K partials reduced inside a cluster of `splits` CTAs
   int chunks;       // splits == 1: K reduced in this many chunks inside the CTA (>= 1)
+  int stages;       // pipeline stages (GemmShape::kStagesMin..kStagesMax)
   void* y;          // output: fp16 [M, ldy] | fp32 [M, ldy] | uint64 [M] (argmax)
   int ldy;
   float* partial;   // global split-K partials [splits][tiles][BN][128] fp32 (cluster == 0)
@@ -89,15 +90,19 @@ struct GemmShape {
   static constexpr int kABytes = 128 * 128;        // 128 rows x 64 fp16
   static constexpr int kBBytes = BN * 128;         // BN rows x 64 fp16
   static constexpr int kStageBytes = kABytes + kBBytes;
-  // two CTAs per SM up to BN = 128 (<= ~97 KB each), one at BN = 256
-  static constexpr int kStages = BN <= 64 ? 4 : (BN <= 128 ? 3 : 4);
+  // Pipeline depth is chosen per launch (GemmArgs::stages): two stages for a
+  // split CTA that loads two k-blocks, up to kStagesMax (about 190 KB) for
+  // CTAs that stream the whole K.
+  static constexpr int kStagesMax = BN <= 32 ? 8 : (BN <= 128 ? 6 : 4);
+  static constexpr int kStagesMin = 2;
+  static constexpr int kStagesDefault = BN <= 64 ? 4 : (BN <= 128 ? 3 : 4);
   static constexpr int kTmemCols = BN < 32 ? 32 : BN;
   static constexpr int kRedBytes = BN * 128 * 4;   // cluster reduction tile [BN][128] fp32
   static constexpr int kXBufBytes = 32 * 128 * 4;  // epilogue exchange (SwiGLU, RoPE, sums)
-  static_assert(kRedBytes + kXBufBytes <= kStages * kStageBytes, "reduction smem");
-  static_assert(!(BN <= 64) || kXBufBytes + BN * 128 * 4 <= kStages * kStageBytes, "staging smem");
+  static_assert(!(BN <= 64) || kXBufBytes + kRedBytes <= kStagesMin * kStageBytes,
+                "cluster staging smem");
   // argmax epilogue: keys [128][33] and quarter maxima [4][32], 8 bytes each
-  static_assert((128 * 33 + 4 * 32) * 8 <= kStages * kStageBytes, "argmax smem");
+  static_assert((128 * 33 + 4 * 32) * 8 <= kStagesMin * kStageBytes, "argmax smem");
   // RoPE cos/sin rows of the tile's tokens, staged while the mainloop runs (decode tiles)
   static constexpr bool kStageRope = BN <= 64;
   static constexpr int kRopeBytes = kStageRope ? BN * 32 * 8 : 0;
@@ -106,8 +111,13 @@ struct GemmShape {
   static constexpr int kRecvBytes = kClusterOk ? BN * 128 * 4 : 0;
   // pipeline | barriers (256 B) | per token: norm scale (4 B), KV destination (8 B), position (4 B)
   // | RoPE rows | receive buffer
-  static constexpr int kRecvOffset = kStages * kStageBytes + 256 + 16 * BN + kRopeBytes;
-  static constexpr int kSmemBytes = kRecvOffset + kRecvBytes + 1024 /*align*/;
+  __host__ __device__ static constexpr int recv_offset(int stages) {
+    return stages * kStageBytes + 256 + 16 * BN + kRopeBytes;
+  }
+  __host__ __device__ static constexpr int smem_bytes(int stages) {
+    return recv_offset(stages) + kRecvBytes + 1024 /*align*/;
+  }
+  static_assert(smem_bytes(kStagesMax) <= 227 * 1024, "deepest pipeline fits one CTA's smem");
 };
 
 // Epilogue of 32 consecutive tokens (t0 .. t0+31) of feature row `row`;
@@ -308,11 +318,12 @@ __global__ void __launch_bounds__(128, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
   uint8_t* smA = smem;
-  uint8_t* smB = smem + S::kStages * S::kABytes;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + S::kStages * S::kStageBytes);
+  const int NS = a.stages;   // pipeline stages of this launch
+  uint8_t* smB = smem + NS * S::kABytes;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + NS * S::kStageBytes);
   uint64_t* full = bars;
-  uint64_t* empty = bars + S::kStages;
-  uint64_t* accum = bars + 2 * S::kStages;
+  uint64_t* empty = bars + NS;
+  uint64_t* accum = bars + 2 * NS;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(accum + 1);
   volatile int* flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   uint64_t* recv_bar = accum + 3;   // cluster split-K: partial slices received
@@ -330,7 +341,7 @@ __global__ void __launch_bounds__(128, 1)
   if (threadIdx.x == 0) {
     tma_prefetch_desc(&tmW);
     tma_prefetch_desc(&tmX);
-    for (int s = 0; s < S::kStages; ++s) {
+    for (int s = 0; s < NS; ++s) {
       mbar_init(smem_u32(&full[s]), 1);
       mbar_init(smem_u32(&empty[s]), 1);
     }
@@ -375,7 +386,7 @@ __global__ void __launch_bounds__(128, 1)
       tma_load_2d(smem_u32(smB + s * S::kBBytes), &tmX, (kb0 + i) * 64, a.x_row0 + tok_tile * BN,
                   smem_u32(&full[s]), pol_x);
     };
-    const int npre = nkb < S::kStages ? nkb : S::kStages;
+    const int npre = nkb < NS ? nkb : NS;
     for (int i = 0; i < npre; ++i) {          // fresh stages: no empty-barrier wait needed
       mbar_arrive_expect_tx(smem_u32(&full[i]), S::kStageBytes);
       load_w(i, i);
@@ -384,15 +395,15 @@ __global__ void __launch_bounds__(128, 1)
     pdl_trigger();
     for (int i = 0; i < npre; ++i) load_x(i, i);
     for (int i = npre; i < nkb; ++i) {
-      const int s = i % S::kStages;
-      const uint32_t ph = (i / S::kStages) & 1;
+      const int s = i % NS;
+      const uint32_t ph = (i / NS) & 1;
       if (!mbar_wait(smem_u32(&empty[s]), ph ^ 1, a.err)) { *flag = 1; break; }
       mbar_arrive_expect_tx(smem_u32(&full[s]), S::kStageBytes);
       load_w(i, s);
       load_x(i, s);
     }
   } else {
-    float* rs_s = reinterpret_cast<float*>(smem + S::kStages * S::kStageBytes + 256);
+    float* rs_s = reinterpret_cast<float*>(smem + NS * S::kStageBytes + 256);
     long long* kvdst_s = reinterpret_cast<long long*>(rs_s + BN);
     int* pos_s = reinterpret_cast<int*>(kvdst_s + BN);
     const int tok0s = tok_tile * BN;
@@ -456,8 +467,8 @@ __global__ void __launch_bounds__(128, 1)
       constexpr uint32_t idesc = umma_idesc_f16(128, BN);
       const int kpc = nkb / nchunk;
       for (int i = 0; i < nkb; ++i) {
-        const int s = i % S::kStages;
-        const uint32_t ph = (i / S::kStages) & 1;
+        const int s = i % NS;
+        const uint32_t ph = (i / NS) & 1;
         if (!mbar_wait(smem_u32(&full[s]), ph, a.err)) { *flag = 1; break; }
         tc_fence_after();
         const uint64_t ad = umma_desc_sw128(smem_u32(smA + s * S::kABytes));
@@ -483,7 +494,7 @@ __global__ void __launch_bounds__(128, 1)
   // per-token epilogue inputs staged by warps 2-3 during the mainloop; the
   // failure flag is made uniform so every barrier below is reached by all
   const bool failed = __syncthreads_or(!acc_ok || *flag) != 0;
-  const float* rs_s = reinterpret_cast<const float*>(smem + S::kStages * S::kStageBytes + 256);
+  const float* rs_s = reinterpret_cast<const float*>(smem + NS * S::kStageBytes + 256);
   const long long* kvdst_s = reinterpret_cast<const long long*>(rs_s + BN);
   const int* pos_s = reinterpret_cast<const int*>(kvdst_s + BN);
   const float2* cs_s = S::kStageRope ? reinterpret_cast<const float2*>(pos_s + BN) : nullptr;
@@ -528,7 +539,7 @@ __global__ void __launch_bounds__(128, 1)
       // q contiguous), send slice q to CTA q's receive buffer at position
       // [split] with one bulk copy, and wait for the S slices of our own
       // tokens on recv_bar; then sum them over s = 0..S-1.
-      float* recv = reinterpret_cast<float*>(smem + S::kRecvOffset);   // [S][per][128]
+      float* recv = reinterpret_cast<float*>(smem + S::recv_offset(NS));   // [S][per][128]
       float* stage = reinterpret_cast<float*>(smA + S::kXBufBytes);   // [BN][128], after xbuf
       float* xbuf = reinterpret_cast<float*>(smA);
       const int per = BN / a.splits;
