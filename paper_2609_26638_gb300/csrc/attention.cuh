@@ -222,12 +222,19 @@ __device__ __forceinline__ bool attn_softmax(const AttnArgs& a, const AttnSync& 
     // 2. mask (keys past the row's limit), scale, this thread's maximum
     const int key0 = (p_begin + j) * 64 + col0;
     float sv[NC];
-    float pmx = -INFINITY;
 #pragma unroll
-    for (int k = 0; k < NC; ++k) {
+    for (int k = 0; k < NC; ++k)
       sv[k] = key0 + k <= lim_r ? __uint_as_float(sr[k]) * kScaleLog2 : -INFINITY;
-      pmx = fmaxf(pmx, sv[k]);
+    // max as a tree (a chain of NC dependent fmax would dominate the page)
+    float mt[8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+      mt[e] = sv[e];
+#pragma unroll
+      for (int k = e + 8; k < NC; k += 8) mt[e] = fmaxf(mt[e], sv[k]);
     }
+    const float pmx = fmaxf(fmaxf(fmaxf(mt[0], mt[1]), fmaxf(mt[2], mt[3])),
+                            fmaxf(fmaxf(mt[4], mt[5]), fmaxf(mt[6], mt[7])));
     // 3. the row's page max over its 2 DUP parts (thread of part p: MMA row
     //    (p / 2) * RPC + rr, warp half p % 2)
     float* red = y.red + buf * kAttnSoftThreads;

@@ -568,8 +568,10 @@ __global__ void __launch_bounds__(128, 1)
         bulk_commit();
       }
       const bool got = __syncthreads_and(mbar_wait(smem_u32(recv_bar), 0, a.err)) != 0;
-      if (threadIdx.x == 0) bulk_wait_read_all();   // our outgoing slices have left `stage`
-      __syncthreads();                              // (the epilogue reuses that memory)
+      if constexpr (EPI == kEpiArgmax) {   // its key table overlaps `stage`
+        if (threadIdx.x == 0) bulk_wait_read_all();
+        __syncthreads();
+      }
       const int lo = split * per, hi = min(lo + per, ntok);
       if (hi > lo && !failed && got) {
         const int nq = hi - lo;
@@ -598,6 +600,7 @@ __global__ void __launch_bounds__(128, 1)
                                            rs_of(c));
         }
       }
+      if (threadIdx.x == 0) bulk_wait_read_all();   // our outgoing slices have left `stage`
       return;
     }
   }
