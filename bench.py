@@ -374,7 +374,7 @@ def gpu_arm(args, rank: int, world: int):
                 "algorithmic_bytes_per_launch": dk["bytes_per_launch"],
                 "us_per_launch": dk["us_per_launch"], "launches_per_step": dk["launches"],
                 "timing": timing, "traffic": None}
-    lm = lm_head_roofline(eng, cfg, K, dev) if B == 1 else None
+    lm = lm_head_roofline(cfg, K, dev) if B == 1 else None
     attn = attention_roofline(cfg, dev)
     res = dict(elapsed=elapsed, e2e_elapsed=e_elapsed, tokens=committed_per_decode * args.steps,
                round_ms=round_ms, rounds=R, launches_per_round=launches_per_round,
@@ -400,7 +400,7 @@ def _time_kernel(fn, stream, iters: int):
     return a.elapsed_time(b) / 1e3 / iters
 
 
-def lm_head_roofline(eng, cfg, K, dev):
+def lm_head_roofline(cfg, K, dev):
     """LM-head GEMM + argmax at the decode shape (17 rows x 59392 x 1024), the
     same kernel instantiation the round launches, over rotating weight copies
     (3 x 121.6 MB > L2)."""
@@ -432,18 +432,20 @@ def lm_head_roofline(eng, cfg, K, dev):
             "us_per_launch": round(t * 1e6, 2), "traffic": None}
 
 
-def attention_roofline(cfg, dev):
-    """Hybrid-mask draft attention at the serving shape (32 sequences, prefix
-    U[1024, 6144] -> mean ~3600, K = 16), the kernel alone over a paged pool
-    larger than L2."""
+def attention_roofline(cfg, dev, ns=None, K=16):
+    """Hybrid-mask draft attention alone over a paged pool.  Default shape: the
+    serving one (32 sequences, prefix U[1024, 6144] -> mean ~3600, K = 16, a
+    pool larger than L2); `ns` gives other cached lengths (one per sequence)."""
     import torch
     from paper_2609_26638_gb300 import gs
     hbm, _, src = load_peaks()
     rng = np.random.default_rng(5)
-    B, K = 32, 16
+    if ns is None:
+        ns = rng.integers(1024, 6145, size=32).astype(np.int32)
+    ns = np.asarray(ns, np.int32)
+    B = len(ns)
     W = K + 1
     Hq, Hkv = cfg.n_heads, cfg.n_kv_heads
-    ns = rng.integers(1024, 6145, size=B).astype(np.int32)
     pages_per = [math.ceil((n + W + 1) / 64) for n in ns]
     pt_stride = max(pages_per)
     n_pages = sum(pages_per)
@@ -453,7 +455,9 @@ def attention_roofline(cfg, dev):
     for b in range(B):
         pt[b, :pages_per[b]] = perm[o:o + pages_per[b]]
         o += pages_per[b]
-    kv = torch.randn(n_pages * 2 * Hkv * 64 * 64, device=dev).half()
+    # enough pool copies (rotated per launch) that every launch reads from DRAM
+    n_copy = max(1, min(64, math.ceil(300e6 / (n_pages * 2 * Hkv * 4096 * 2))))
+    kvs = [torch.randn(n_pages * 2 * Hkv * 64 * 64, device=dev).half() for _ in range(n_copy)]
     q = torch.randn(B * W * Hq * 64, device=dev).half()
     out = torch.zeros_like(q)
     ptd = torch.from_numpy(pt).to(dev)
@@ -463,7 +467,11 @@ def attention_roofline(cfg, dev):
     scratch = torch.zeros(sb, dtype=torch.uint8, device=dev)
     stream = torch.cuda.current_stream(dev)
 
+    it = [0]
+
     def fn():
+        kv = kvs[it[0] % n_copy]
+        it[0] += 1
         gs.gs_attention(0, q.data_ptr(), kv.data_ptr(), n_pages, ptd.data_ptr(), pt_stride,
                         nd.data_ptr(), B, W, Hq, Hkv, out.data_ptr(), scratch.data_ptr(), sb, sp,
                         stream.cuda_stream)
@@ -472,7 +480,8 @@ def attention_roofline(cfg, dev):
     keys = int(sum(int(n) + W for n in ns))
     algo = keys * Hkv * 64 * 2 * 2 + 2 * B * W * Hq * 64 * 2
     achieved = algo / t / 1e9
-    return {"kernel": "attn_paged_kernel (draft, 32 seqs, ctx ~3.6k, K=16)", "bound": "hbm",
+    return {"kernel": f"attn_paged_kernel (draft, {B} seqs, mean cached {int(ns.mean())}, K={K}, "
+                      f"{sp} pages per item)", "bound": "hbm",
             "achieved": round(achieved, 1), "peak": hbm, "unit": "GB/s",
             "frac": round(achieved / hbm, 4), "kv_bytes": algo, "us_per_launch": round(t * 1e6, 2)}
 
@@ -555,7 +564,25 @@ def main():
     ap.add_argument("--no-compare-ar", dest="compare_ar", action="store_false",
                     help="skip timing plain greedy AR (K = 0 rounds) on the same workload")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--kernel", default=None, choices=["attention", "lm_head"],
+                    help="time one kernel alone at its serving / decode shape and print its "
+                         "roofline line (the single-kernel ncu captures run this)")
     args = ap.parse_args()
+    if args.kernel is not None:
+        import torch
+        dev = torch.device("cuda", 0)
+        torch.cuda.set_device(dev)
+        cfg = synth.WORKLOADS[args.workload].model
+        K = synth.WORKLOADS[args.workload].K if args.K is None else args.K
+        wl = synth.WORKLOADS[args.workload]
+        if args.kernel == "lm_head":
+            r = lm_head_roofline(cfg, K, dev)
+        elif wl.batch == 1:   # mid-decode of the single-sequence workload
+            r = attention_roofline(cfg, dev, [wl.prefix_min + wl.max_new // 2], K)
+        else:
+            r = attention_roofline(cfg, dev)
+        print(json.dumps(r))
+        return
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     wl = synth.WORKLOADS[args.workload]

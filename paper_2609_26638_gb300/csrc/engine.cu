@@ -90,7 +90,7 @@ AttnGeom attn_geom(int W, int G) {
 // and fragment larger grids); otherwise through global scratch.  Both give
 // the same bits.
 bool attn_use_cluster(int items, int blocks_x_heads) {
-  return items <= kAttnMaxCluster && items * blocks_x_heads <= 2 * 152;
+  return items <= kAttnMaxCluster && items * blocks_x_heads <= 2 * kNumSMs;
 }
 
 cudaError_t launch_attention(const CUtensorMap& tm, const AttnArgs& a, int n_blocks,
@@ -114,8 +114,8 @@ struct GemmPlan {
 int decode_splits(int weight_rows, int K) {
   const int feat_tiles = weight_rows / 128;
   const int nkb = K / 64;
-  if (feat_tiles >= 152) return 1;
-  const int want = std::min(std::max(cdiv(152, feat_tiles), 4), kMaxClusterSplits);
+  if (feat_tiles >= kNumSMs) return 1;
+  const int want = std::min(std::max(cdiv(kNumSMs, feat_tiles), 4), kMaxClusterSplits);
   int s = 1;
   for (int k = 1; k <= nkb; ++k)
     if (nkb % k == 0 && k <= want) s = k;
@@ -124,18 +124,19 @@ int decode_splits(int weight_rows, int K) {
 
 // Decode windows of up to 64 tokens split K across the CTAs of a cluster;
 // wider decode launches reduce the same K chunks inside each CTA (one TMEM
-// accumulator per chunk, summed in chunk order), with the token tile shrunk
-// until the launch covers about one wave.  Prefill does not split K.
+// accumulator per chunk, summed in chunk order).  The chunks' accumulators
+// take at most 256 TMEM columns, so two CTAs share an SM, and the token tile
+// shrinks until the launch covers about one wave.  Prefill does not split K.
 GemmPlan plan_split(int weight_rows, int T, int S) {
   GemmPlan p;
   p.feat_tiles = weight_rows / 128;
   p.chunks = 1;
   p.splits = S;
   p.bn = gemm_bn_for(T);
-  if (S > 1 && T > 64 && S * 32 <= 512) {
+  if (S > 1 && T > 64 && S * 32 <= 256) {
     p.chunks = S;
     p.splits = 1;
-    p.bn = std::min(128, 512 / S);
+    p.bn = std::min(128, 256 / S);
     while (p.bn > 32 && p.feat_tiles * cdiv(T, p.bn) < 148) p.bn /= 2;
   }
   p.tok_tiles = cdiv(T, p.bn);

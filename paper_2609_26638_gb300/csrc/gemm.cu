@@ -8,16 +8,24 @@ template <int BN, int EPI>
 static cudaError_t launch_one(const CUtensorMap& tmW, const CUtensorMap& tmX, GemmArgs a,
                               int feat_tiles, int tok_tiles, cudaStream_t s, bool pdl) {
   using S = GemmShape<BN>;
-  // stages: a depth that leaves room for a second resident CTA per SM (it
-  // starts as soon as the first releases TMEM, with no launch gap), never more
-  // than the k-blocks one CTA loads
-  const int want = S::kStagesDefault;
+  // Pipeline depth, never more than the k-blocks one CTA loads.  Decode
+  // windows (up to 64 rows, unchunked): a fixed depth that leaves room for a
+  // second resident CTA and for the neighbouring kernels' CTAs that overlap it
+  // under programmatic dependent launch.  Wider launches stream K through
+  // each CTA: the deepest pipeline that still fits the CTAs one SM holds
+  // (one when the grid is at most one CTA per SM, else two), since bytes in
+  // flight per SM set their load rate.
+  const bool cl = a.splits > 1 && a.cluster;
+  int want = S::kStagesDefault;
+  if (a.chunks > 1 || a.M > 64)
+    want = S::stages_fitting(static_cast<long>(feat_tiles) * tok_tiles * a.splits <= kNumSMs ? 1 : 2,
+                             EPI, cl);
   const int kb = a.kb_per_split;
   a.stages = kb < S::kStagesMin ? S::kStagesMin : (kb > want ? want : kb);
   dim3 grid(tok_tiles, feat_tiles, a.splits);
-  const int cz = (a.splits > 1 && a.cluster) ? a.splits : 1;
-  return launch_ex(gemm_tc_kernel<BN, EPI>, grid, dim3(128), S::smem_bytes(a.stages), s, pdl,
-                   dim3(1, 1, cz), tmW, tmX, a);
+  const int cz = cl ? a.splits : 1;
+  return launch_ex(gemm_tc_kernel<BN, EPI>, grid, dim3(128), S::smem_bytes(a.stages, EPI, cl), s,
+                   pdl, dim3(1, 1, cz), tmW, tmX, a);
 }
 
 template <int BN>
@@ -47,7 +55,7 @@ cudaError_t launch_gemm(int bn, int epi, const CUtensorMap& tmW, const CUtensorM
 
 template <int BN>
 static cudaError_t set_attr_bn() {
-  const int bytes = GemmShape<BN>::smem_bytes(GemmShape<BN>::kStagesMax);
+  const int bytes = GemmShape<BN>::kSmemMax;
   cudaError_t e;
   if ((e = cudaFuncSetAttribute(gemm_tc_kernel<BN, kEpiStoreF16>,
                                 cudaFuncAttributeMaxDynamicSharedMemorySize, bytes)) != cudaSuccess)

@@ -103,21 +103,32 @@ struct GemmShape {
                 "cluster staging smem");
   // argmax epilogue: keys [128][33] and quarter maxima [4][32], 8 bytes each
   static_assert((128 * 33 + 4 * 32) * 8 <= kStagesMin * kStageBytes, "argmax smem");
-  // RoPE cos/sin rows of the tile's tokens, staged while the mainloop runs (decode tiles)
+  // RoPE cos/sin rows of the tile's tokens, staged while the mainloop runs
+  // (QKV launches, decode tiles)
   static constexpr bool kStageRope = BN <= 64;
-  static constexpr int kRopeBytes = kStageRope ? BN * 32 * 8 : 0;
+  __host__ __device__ static constexpr int rope_bytes(int epi) {
+    return (kStageRope && epi == kEpiQKV) ? BN * 32 * 8 : 0;
+  }
   // cluster split-K receive buffer [S][BN / S][128] fp32 (decode tiles only)
   static constexpr bool kClusterOk = BN <= 64;
   static constexpr int kRecvBytes = kClusterOk ? BN * 128 * 4 : 0;
   // pipeline | barriers (256 B) | per token: norm scale (4 B), KV destination (8 B), position (4 B)
   // | RoPE rows | receive buffer
-  __host__ __device__ static constexpr int recv_offset(int stages) {
-    return stages * kStageBytes + 256 + 16 * BN + kRopeBytes;
+  __host__ __device__ static constexpr int recv_offset(int stages, int epi) {
+    return stages * kStageBytes + 256 + 16 * BN + rope_bytes(epi);
   }
-  __host__ __device__ static constexpr int smem_bytes(int stages) {
-    return recv_offset(stages) + kRecvBytes + 1024 /*align*/;
+  __host__ __device__ static constexpr int smem_bytes(int stages, int epi, bool cluster) {
+    return recv_offset(stages, epi) + (cluster ? kRecvBytes : 0) + 1024 /*align*/;
   }
-  static_assert(smem_bytes(kStagesMax) <= 227 * 1024, "deepest pipeline fits one CTA's smem");
+  static constexpr int kSmemMax = smem_bytes(kStagesMax, kEpiQKV, true);
+  static_assert(kSmemMax <= 227 * 1024, "deepest pipeline fits one CTA's smem");
+  // Deepest pipeline with which `per_sm` CTAs share one SM's 228 KB (each CTA
+  // also holds 1 KB of system smem and 16 B of static smem).
+  static int stages_fitting(int per_sm, int epi, bool cluster) {
+    for (int st = kStagesMax; st > kStagesMin; --st)
+      if ((smem_bytes(st, epi, cluster) + 1024 + 16) * per_sm <= 228 * 1024) return st;
+    return kStagesMin;
+  }
 };
 
 // Epilogue of 32 consecutive tokens (t0 .. t0+31) of feature row `row`;
@@ -539,7 +550,7 @@ __global__ void __launch_bounds__(128, 1)
       // q contiguous), send slice q to CTA q's receive buffer at position
       // [split] with one bulk copy, and wait for the S slices of our own
       // tokens on recv_bar; then sum them over s = 0..S-1.
-      float* recv = reinterpret_cast<float*>(smem + S::recv_offset(NS));   // [S][per][128]
+      float* recv = reinterpret_cast<float*>(smem + S::recv_offset(NS, EPI));   // [S][per][128]
       float* stage = reinterpret_cast<float*>(smA + S::kXBufBytes);   // [BN][128], after xbuf
       float* xbuf = reinterpret_cast<float*>(smA);
       const int per = BN / a.splits;

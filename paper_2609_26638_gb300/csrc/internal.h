@@ -40,6 +40,10 @@ cudaError_t launch_ex(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t sm
 }
 
 // Token tile for a GEMM over T token rows.
+// SMs of one GB300 (two dies x 76).  Work decompositions that must not depend
+// on the device (the split-K factors) use this constant, not a query.
+constexpr int kNumSMs = 152;
+
 inline int gemm_bn_for(int T) { return T <= 32 ? 32 : (T <= 64 ? 64 : (T <= 128 ? 128 : 256)); }
 
 // Launch Y = epilogue(W . X^T) for one weight matrix.  grid = (feat_tiles,
