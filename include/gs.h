@@ -253,8 +253,9 @@ int gs_sync_check(gs_handle *h);
  *            logical pages [i * split_pages, (i + 1) * split_pages); items are
  *            reduced independently and merged in item order, so results depend
  *            on split_pages but not on n_seq, W or the other sequences.
- *            GS_ERR_UNSUPPORTED if ceil(pt_stride / split_pages) > 96 (the
- *            merge's limit).
+ *            GS_ERR_UNSUPPORTED if ceil(pt_stride / split_pages) > 48 (the
+ *            merge keeps each item's running max and sum of every row in
+ *            shared memory).
  *   stream   cudaStream_t */
 size_t gs_attention_scratch_bytes(int n_seq, int W, int n_heads, int n_kv_heads, int max_pages,
                                   int split_pages);

@@ -348,6 +348,12 @@ __global__ void __launch_bounds__(128, 1)
   const int split = blockIdx.z;
   const int kb0 = split * a.kb_per_split;
   const int nkb = a.kb_per_split;
+  // Chunked K: step i works on k-block t of chunk c, c = i % nchunk and
+  // t = i / nchunk, so consecutive MMAs go to different accumulators and do
+  // not wait on each other; each chunk still sums its k-blocks in order.
+  const int nchunk = a.chunks > 1 ? a.chunks : 1;
+  const int kpc = nkb / nchunk;
+  auto kblock = [&](int i) { return nchunk > 1 ? (i % nchunk) * kpc + i / nchunk : i; };
 
   if (threadIdx.x == 0) {
     tma_prefetch_desc(&tmW);
@@ -368,7 +374,6 @@ __global__ void __launch_bounds__(128, 1)
     fence_mbar_init();
   }
   // chunked K: one TMEM accumulator of BN columns per chunk
-  const int nchunk = a.chunks > 1 ? a.chunks : 1;
   const uint32_t tmem_cols = static_cast<uint32_t>(S::kTmemCols * nchunk);
   if (warp == 2) tmem_alloc(smem_u32(tmem_slot), tmem_cols);
   tc_fence_before();
@@ -384,7 +389,7 @@ __global__ void __launch_bounds__(128, 1)
     const uint64_t pol_x = l2_policy_evict_last();
     auto load_w = [&](int i, int s) {
       const uint32_t fb = smem_u32(&full[s]);
-      const int kx = (kb0 + i) * 64;
+      const int kx = (kb0 + kblock(i)) * 64;
       if constexpr (EPI == kEpiSwiGLU) {
         tma_load_2d(smem_u32(smA + s * S::kABytes), &tmW, kx, feat_tile * 64, fb, pol_w);
         tma_load_2d(smem_u32(smA + s * S::kABytes + 64 * 128), &tmW, kx, a.N + feat_tile * 64, fb,
@@ -394,8 +399,8 @@ __global__ void __launch_bounds__(128, 1)
       }
     };
     auto load_x = [&](int i, int s) {
-      tma_load_2d(smem_u32(smB + s * S::kBBytes), &tmX, (kb0 + i) * 64, a.x_row0 + tok_tile * BN,
-                  smem_u32(&full[s]), pol_x);
+      tma_load_2d(smem_u32(smB + s * S::kBBytes), &tmX, (kb0 + kblock(i)) * 64,
+                  a.x_row0 + tok_tile * BN, smem_u32(&full[s]), pol_x);
     };
     const int npre = nkb < NS ? nkb : NS;
     for (int i = 0; i < npre; ++i) {          // fresh stages: no empty-barrier wait needed
@@ -473,10 +478,9 @@ __global__ void __launch_bounds__(128, 1)
       }
     }
     if (warp == 1 && lane == 0) {
-      // MMA issuer.  Chunked K: chunk c (k-blocks [c*kpc, (c+1)*kpc)) starts a
-      // fresh accumulator at TMEM column c * BN.
+      // MMA issuer.  Chunked K: chunk c (k-blocks [c*kpc, (c+1)*kpc)) has its
+      // accumulator at TMEM column c * BN, fresh at its first k-block.
       constexpr uint32_t idesc = umma_idesc_f16(128, BN);
-      const int kpc = nkb / nchunk;
       for (int i = 0; i < nkb; ++i) {
         const int s = i % NS;
         const uint32_t ph = (i / NS) & 1;
@@ -484,8 +488,8 @@ __global__ void __launch_bounds__(128, 1)
         tc_fence_after();
         const uint64_t ad = umma_desc_sw128(smem_u32(smA + s * S::kABytes));
         const uint64_t bd = umma_desc_sw128(smem_u32(smB + s * S::kBBytes));
-        const uint32_t dst = tmem + static_cast<uint32_t>((i / kpc) * BN);
-        const bool fresh = (i % kpc) == 0;
+        const uint32_t dst = tmem + static_cast<uint32_t>((i % nchunk) * BN);
+        const bool fresh = i < nchunk;
 #pragma unroll
         for (int k = 0; k < 4; ++k)
           umma_f16(dst, ad + 2 * k, bd + 2 * k, idesc, (!fresh || k > 0) ? 1u : 0u);
