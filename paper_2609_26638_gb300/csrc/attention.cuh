@@ -29,7 +29,7 @@
 //
 // Merge over items, item order 0, 1, ...: M = max m_i, w_i = exp2(m_i - M),
 // coef_i = w_i / sum_j w_j l_j, O = sum coef_i O_i.  A block with one item
-// writes its rows directly.  A (block, head) with at most 8 items may form one
+// writes its rows directly.  A (block, head) with at most 16 items may form one
 // thread-block cluster: once every CTA of the cluster has finished its pages,
 // each sends the rows that CTA (r mod n) owns to it with one bulk async copy
 // into its shared memory, completing on its mbarrier, and each owner merges
@@ -53,7 +53,7 @@ constexpr int kAttnPageBytes = 64 * 128;  // 64 x 64 fp16
 constexpr int kAttnStageBytes = 2 * kAttnPageBytes;
 constexpr int kAttnRow = 68;              // partial row: O[64], m, l, 2 pad (272 B)
 constexpr int kAttnMaxRows = 128;         // rows of one query block (the MMA's M)
-constexpr int kAttnMaxCluster = 8;        // items merged inside a cluster
+constexpr int kAttnMaxCluster = 16;       // items merged inside a cluster (16: non-portable size)
 constexpr int kAttnSoftWarps = 8;         // two warps per TMEM lane quarter
 constexpr int kAttnSoftThreads = kAttnSoftWarps * 32;
 constexpr int kAttnThreads = kAttnSoftThreads + 64;   // + TMA warp, MMA warp
@@ -90,7 +90,7 @@ struct AttnArgs {
   int rows_per_page;          // 2 * Hkv * 64
   int split_pages;            // SP: pages per item
   int max_items;              // items per (block, head) the grid covers
-  int cluster;                // 1: the grid's x dimension is one cluster (max_items <= 8)
+  int cluster;                // 1: the grid's x dimension is one cluster (max_items <= 16)
   float* part;                // global merge: [n_blocks][Hkv][max_items][128][kAttnRow]
   int* ticket;                // global merge: [n_blocks][Hkv], zero between launches
   int* err;

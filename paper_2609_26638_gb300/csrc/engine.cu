@@ -85,10 +85,10 @@ AttnGeom attn_geom(int W, int G) {
   return {qs, cdiv(W, qs), kAttnMaxRows};
 }
 
-// Items merge inside a cluster when there are at most 8 of them and the
-// launch is about one wave (clusters of 8 CTAs wait for 8 free SMs of one GPC
-// and fragment larger grids); otherwise through global scratch.  Both give
-// the same bits.
+// Items merge inside a cluster when there are at most 16 of them and the
+// launch is about one wave (a cluster waits for free SMs of one GPC, and
+// clusters fragment larger grids); otherwise through global scratch.  Both
+// give the same bits.
 bool attn_use_cluster(int items, int blocks_x_heads) {
   return items <= kAttnMaxCluster && items * blocks_x_heads <= 2 * kNumSMs;
 }
@@ -299,16 +299,19 @@ size_t carve(gs_handle* h, const gs_config& c, void* base) {
   const int W_max = c.max_K + 1;
   int T_max = std::max(c.max_batch * W_max, c.max_prefill);
   T_max = static_cast<int>(align_up(std::max(T_max, 256), 256));
-  // attention work items (fixed absolute page ranges).  Decode: at most 8
-  // items per sequence (one cluster) unless the config asks for smaller
-  // items; prefill: at least 8 pages per item, at most 8 items.
+  // attention work items (fixed absolute page ranges).  Decode: at most 16
+  // items per sequence (one cluster) when a full batch of them still fits in
+  // about one wave of CTAs, else at most 8, unless the config asks for
+  // smaller items; prefill: at least 8 pages per item, at most 8 items.
   const int r_max = round16(W_max * G);
   const AttnGeom g_dec = attn_geom(W_max, G);
   const int qb_pf = std::max(1, kAttnMaxRows / G);
-  int sp = c.split_pages > 0 ? c.split_pages : std::max(2, cdiv(pt_stride, kAttnMaxCluster));
+  const int items_target =
+      attn_use_cluster(kAttnMaxCluster, c.max_batch * g_dec.n_sub * c.n_kv_heads) ? kAttnMaxCluster : 8;
+  int sp = c.split_pages > 0 ? c.split_pages : std::max(2, cdiv(pt_stride, items_target));
   sp = std::max(sp, cdiv(pt_stride, attn_max_merge_items(g_dec.rows)));
   const int items_dec = cdiv(pt_stride, sp);
-  const int sp_pf = std::max(8, cdiv(pt_stride, kAttnMaxCluster));
+  const int sp_pf = std::max(8, cdiv(pt_stride, 8));
   const int items_pf = cdiv(pt_stride, sp_pf);
   const AttnGeom g_pf = attn_geom(qb_pf, G);
   const int blocks_pf = cdiv(std::min(c.max_prefill, T_max), qb_pf);
@@ -678,6 +681,8 @@ int gs_create(const gs_config* cfg, const gs_weights* w, void* workspace, size_t
     if (e == cudaSuccess)
       e = cudaFuncSetAttribute(attn_paged_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                attn_max_smem_bytes());
+    if (e == cudaSuccess)   // clusters of up to 16 items
+      e = cudaFuncSetAttribute(attn_paged_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
 
     if (e != cudaSuccess)
       return fail(nullptr, GS_ERR_CUDA, std::string("kernel attributes: ") + cudaGetErrorString(e));
@@ -1083,7 +1088,9 @@ int gs_attention(int mode, const void* q, const void* kv, int n_pages, const int
   static bool attr = false;
   if (!attr) {
     if (cudaFuncSetAttribute(attn_paged_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             attn_max_smem_bytes()) != cudaSuccess)
+                             attn_max_smem_bytes()) != cudaSuccess ||
+        cudaFuncSetAttribute(attn_paged_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed,
+                             1) != cudaSuccess)
       return GS_ERR_CUDA;
     attr = true;
   }
