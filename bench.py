@@ -462,7 +462,10 @@ def attention_roofline(cfg, dev, ns=None, K=16):
     out = torch.zeros_like(q)
     ptd = torch.from_numpy(pt).to(dev)
     nd = torch.from_numpy(ns).to(dev)
-    sp = max(2, math.ceil(pt_stride / 8))   # the engine's default: at most 8 items
+    # the engine's default: at most 16 items per sequence when a batch of them
+    # fits about one wave of CTAs, else at most 8
+    items = 16 if B * Hkv * 16 <= 2 * 152 else 8
+    sp = max(2, math.ceil(pt_stride / items))
     sb = gs.gs_attention_scratch_bytes(B, W, Hq, Hkv, pt_stride, sp)
     scratch = torch.zeros(sb, dtype=torch.uint8, device=dev)
     stream = torch.cuda.current_stream(dev)
@@ -565,8 +568,9 @@ def main():
                     help="skip timing plain greedy AR (K = 0 rounds) on the same workload")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--kernel", default=None, choices=["attention", "lm_head"],
-                    help="time one kernel alone at its serving / decode shape and print its "
-                         "roofline line (the single-kernel ncu captures run this)")
+                    help="time one kernel alone and print its roofline line (the single-kernel "
+                         "ncu captures run this): attention at the workload's decode shape "
+                         "(the serving batch for serve_b32), the LM head at 17 rows")
     args = ap.parse_args()
     if args.kernel is not None:
         import torch

@@ -234,19 +234,22 @@ __device__ __forceinline__ bool attn_softmax(const AttnArgs& a, const AttnSync& 
       mx = fmaxf(mx, red[((pp & 1) * 4 + (mr >> 5)) * 32 + (mr & 31)]);
     }
     // 4. a rise by more than 2^8 rescales O and the row sums first
-    if (mx > m + kAttnRescale) {
-      const float alpha = (m == -INFINITY) ? 0.f : exp2f(m - mx);
-      if (cp == 0 && j > 0) {
-        if (!wwait(y.pv_done, (j - 1) & 1)) return false;
-        tc_fence_after();
-        uint32_t o32[32];
-        tmem_ld32_nowait(trow + 128 + half * 32, o32);
-        tmem_wait_ld();
+    //    tcgen05.ld / st are warp-collective: a warp with any rising row
+    //    rescales all its rows, the others by exactly 1.
+    const bool rise = mx > m + kAttnRescale;
+    const float alpha = !rise ? 1.f : ((m == -INFINITY) ? 0.f : exp2f(m - mx));
+    if (cp == 0 && j > 0 && __any_sync(0xFFFFFFFFu, rise)) {
+      if (!wwait(y.pv_done, (j - 1) & 1)) return false;
+      tc_fence_after();
+      uint32_t o32[32];
+      tmem_ld32_nowait(trow + 128 + half * 32, o32);
+      tmem_wait_ld();
 #pragma unroll
-        for (int k = 0; k < 32; ++k) o32[k] = __float_as_uint(alpha * __uint_as_float(o32[k]));
-        tmem_st32(trow + 128 + half * 32, o32);
-        tmem_wait_st();
-      }
+      for (int k = 0; k < 32; ++k) o32[k] = __float_as_uint(alpha * __uint_as_float(o32[k]));
+      tmem_st32(trow + 128 + half * 32, o32);
+      tmem_wait_st();
+    }
+    if (rise) {
 #pragma unroll
       for (int c = 0; c < NCH; ++c) lc[c] *= alpha;
       m = mx;
