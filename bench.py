@@ -322,7 +322,7 @@ def gpu_arm(args, rank: int, world: int):
               "ms_per_step": round(1e3 * ar_s, 3), "steps": n_ar, "rounds_per_step": R_ar}
 
     # per-kernel device times: the forced decode once more, every round
-    # enqueued eagerly with a CUDA event after each launch (gs_round_profile)
+    # replayed as a graph with a CUDA event after each launch (gs_round_profile)
     hbm, bf16_tf, src = load_peaks()
     W = K + 1
     T = B * W
@@ -359,7 +359,8 @@ def gpu_arm(args, rank: int, world: int):
         kernels[name] = k
     dom = max((n for n in kernels if "bound" in kernels[n]), key=lambda n: kernels[n]["total_ms"])
     dk = kernels[dom]
-    timing = "CUDA events around each launch of one eagerly enqueued decode (no launch overlap)"
+    timing = ("CUDA event nodes after every launch of one forced decode, each round captured and "
+              "replayed as a graph (no host gaps; no launch overlap across an event)")
     if dk["bound"] == "tensor":
         roof = {"kernel": f"{dom} (gemm_tc_kernel), {T} rows", "bound": "tensor",
                 "achieved": dk["tflop_s"], "peak": bf16_tf, "unit": "TFLOP/s",
@@ -386,15 +387,29 @@ def gpu_arm(args, rank: int, world: int):
     return res
 
 
-def _time_kernel(fn, stream, iters: int):
+def _time_kernel(fn, iters: int):
+    """Average device seconds of one fn() launch: `iters` launches captured as
+    one CUDA graph and replayed, so no host enqueue time falls between them.
+    fn enqueues on torch's current stream at call time."""
     import torch
-    for _ in range(3):
-        fn()
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):
+        for _ in range(3):
+            fn()
+    torch.cuda.current_stream().wait_stream(side)
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        for _ in range(iters):
+            fn()
+    g.replay()
+    torch.cuda.synchronize()
     a = torch.cuda.Event(enable_timing=True)
     b = torch.cuda.Event(enable_timing=True)
+    stream = torch.cuda.current_stream()
     a.record(stream)
-    for _ in range(iters):
-        fn()
+    g.replay()
     b.record(stream)
     b.synchronize()
     return a.elapsed_time(b) / 1e3 / iters
@@ -403,7 +418,7 @@ def _time_kernel(fn, stream, iters: int):
 def lm_head_roofline(cfg, K, dev):
     """LM-head GEMM + argmax at the decode shape (17 rows x 59392 x 1024), the
     same kernel instantiation the round launches, over rotating weight copies
-    (3 x 121.6 MB > L2)."""
+    (3 x 121.6 MB > L2), 30 launches replayed as one graph."""
     import torch
     from paper_2609_26638_gb300 import gs
     hbm, _, src = load_peaks()
@@ -414,16 +429,15 @@ def lm_head_roofline(cfg, K, dev):
     keys = torch.zeros(M, dtype=torch.int64, device=dev)
     sb = gs.gs_linear_scratch_bytes(M, N, 1)
     scratch = torch.zeros(sb, dtype=torch.uint8, device=dev)
-    stream = torch.cuda.current_stream(dev)
     it = [0]
 
     def fn():
         w = ws[it[0] % 3]
         it[0] += 1
         gs.gs_linear(x.data_ptr(), w.data_ptr(), keys.data_ptr(), M, N, Kd, gs.EPI_ARGMAX, 1,
-                     scratch.data_ptr(), sb, stream.cuda_stream)
+                     scratch.data_ptr(), sb, torch.cuda.current_stream(dev).cuda_stream)
 
-    t = _time_kernel(fn, stream, 30)
+    t = _time_kernel(fn, 30)
     algo = N * Kd * 2 + M * Kd * 2 + M * 8
     achieved = algo / t / 1e9
     return {"kernel": "gemm_tc_kernel<32, argmax> (LM head 17x59392x1024)", "bound": "hbm",
@@ -468,8 +482,6 @@ def attention_roofline(cfg, dev, ns=None, K=16):
     sp = max(2, math.ceil(pt_stride / items))
     sb = gs.gs_attention_scratch_bytes(B, W, Hq, Hkv, pt_stride, sp)
     scratch = torch.zeros(sb, dtype=torch.uint8, device=dev)
-    stream = torch.cuda.current_stream(dev)
-
     it = [0]
 
     def fn():
@@ -477,9 +489,9 @@ def attention_roofline(cfg, dev, ns=None, K=16):
         it[0] += 1
         gs.gs_attention(0, q.data_ptr(), kv.data_ptr(), n_pages, ptd.data_ptr(), pt_stride,
                         nd.data_ptr(), B, W, Hq, Hkv, out.data_ptr(), scratch.data_ptr(), sb, sp,
-                        stream.cuda_stream)
+                        torch.cuda.current_stream(dev).cuda_stream)
 
-    t = _time_kernel(fn, stream, 20)
+    t = _time_kernel(fn, 64 if B == 1 else 20)
     keys = int(sum(int(n) + W for n in ns))
     algo = keys * Hkv * 64 * 2 * 2 + 2 * B * W * Hq * 64 * 2
     achieved = algo / t / 1e9

@@ -206,13 +206,15 @@ enum {
 
 /* Measurement aid: one greedy round, with the same arguments and effects as
  * gs_round(h, slots, n_seq, K, GS_ACCEPT_GREEDY, force, out_tok, out_cnt,
- * out_done, NULL), enqueued eagerly (never from the graph cache) with a CUDA
- * event recorded after every kernel launch.  The paper has no counterpart.
+ * out_done, NULL), captured (never from the graph cache) with a CUDA event
+ * recorded after every kernel launch and replayed as one graph, so the host's
+ * enqueue time never falls between two launches.  The paper has no
+ * counterpart.
  *   ms[i]       device milliseconds between launch i-1's end event and launch
  *               i's end event (for i = 0, from an event recorded before the
  *               round).  An event between two kernels stops the second from
- *               starting early, so each figure is the kernel alone plus the
- *               gap the front end needs to start it.
+ *               starting early, so each figure is the kernel alone, from the
+ *               front end starting it to its last CTA.
  *   kind[i]     GS_KIND_* of launch i.
  *   n_launches  number of launches written.
  * ms and kind are host arrays of max_launches entries.  Synchronises the

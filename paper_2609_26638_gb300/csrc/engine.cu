@@ -261,7 +261,8 @@ void note_launch(gs_handle* h, int kind) {
     }
     h->prof_ev.push_back(e);
   }
-  cudaError_t r = cudaEventRecord(h->prof_ev[i], h->stream);
+  // an event-record node of the captured profiling graph
+  cudaError_t r = cudaEventRecordWithFlags(h->prof_ev[i], h->stream, cudaEventRecordExternal);
   if (r != cudaSuccess && h->prof_err == cudaSuccess) h->prof_err = r;
   h->prof_kind.push_back(kind);
 }
@@ -991,14 +992,34 @@ int gs_round_profile(gs_handle* h, const int32_t* slots, int n_seq, int K, const
   }
   h->prof_kind.clear();
   h->prof_err = cudaSuccess;
-  GS_CUDA(h, cudaEventRecord(h->prof_ev[0], h->stream));
+  // The round with an event after every launch is captured and replayed as
+  // one graph, so the host's enqueue time never separates two launches; an
+  // event node between two kernels turns their programmatic overlap into a
+  // plain dependency, so each interval is one kernel's whole duration.
+  cudaGraph_t g = nullptr;
+  GS_CUDA(h, cudaStreamBeginCapture(h->stream, cudaStreamCaptureModeThreadLocal));
+  cudaError_t e0 = cudaEventRecordWithFlags(h->prof_ev[0], h->stream, cudaEventRecordExternal);
   h->profiling = true;
   const int rc = enqueue_round(h, slots, n_seq, K, force, out_tok, out_cnt, out_done, nullptr);
   h->profiling = false;
-  if (rc) return rc;
-  if (h->prof_err != cudaSuccess)
-    return fail(h, GS_ERR_CUDA, std::string("profile events: ") + cudaGetErrorString(h->prof_err));
-  GS_CUDA(h, cudaStreamSynchronize(h->stream));
+  cudaError_t e1 = cudaStreamEndCapture(h->stream, &g);
+  if (rc) {
+    if (e1 == cudaSuccess) cudaGraphDestroy(g);
+    return rc;
+  }
+  if (e0 != cudaSuccess || e1 != cudaSuccess || h->prof_err != cudaSuccess) {
+    if (e1 == cudaSuccess) cudaGraphDestroy(g);
+    const cudaError_t e = e0 != cudaSuccess ? e0 : (e1 != cudaSuccess ? e1 : h->prof_err);
+    return fail(h, GS_ERR_CUDA, std::string("profile capture: ") + cudaGetErrorString(e));
+  }
+  cudaGraphExec_t ge = nullptr;
+  cudaError_t e2 = cudaGraphInstantiate(&ge, g, 0);
+  cudaGraphDestroy(g);
+  if (e2 != cudaSuccess) return fail(h, GS_ERR_CUDA, std::string("profile graph: ") + cudaGetErrorString(e2));
+  e2 = cudaGraphLaunch(ge, h->stream);
+  if (e2 == cudaSuccess) e2 = cudaStreamSynchronize(h->stream);
+  cudaGraphExecDestroy(ge);
+  if (e2 != cudaSuccess) return fail(h, GS_ERR_CUDA, std::string("profile replay: ") + cudaGetErrorString(e2));
   const int n = static_cast<int>(h->prof_kind.size());
   if (n > max_launches) return fail(h, GS_ERR_INVALID_ARG, "max_launches below the round's launches");
   for (int i = 0; i < n; ++i) {

@@ -97,7 +97,7 @@ class Engine:
     def round_profile(self, slots: torch.Tensor, K: int, out_tok: torch.Tensor,
                       out_cnt: torch.Tensor, out_done: torch.Tensor,
                       force: Optional[gs.gs_force] = None) -> list:
-        """One round enqueued eagerly with an event after every kernel:
+        """One round replayed as a graph with an event after every kernel:
         [(kind name, device ms)] per launch (see gs_round_profile)."""
         prof = gs.gs_round_profile(self.handle, slots.data_ptr(), slots.shape[0], K, force,
                                    out_tok.data_ptr(), out_cnt.data_ptr(), out_done.data_ptr())
