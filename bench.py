@@ -55,6 +55,39 @@ def schedule_rounds(sched: np.ndarray, max_new: int) -> int:
     return r
 
 
+# DRAM traffic per launch (dram__bytes_read.sum + dram__bytes_write.sum) from
+# ncu captures of the kernels as committed (summaries under profiles/), with
+# the algorithmic bytes of the captured launch.  A figure is used only while
+# the kernel's sources hash to the value it was taken with; it is scaled to
+# another launch of the same kernel by its algorithmic bytes (attention
+# traffic grows with the keys read: K and V rows, once each).
+_CSRC = os.path.join(ROOT, "paper_2609_26638_gb300", "csrc")
+NCU_TRAFFIC = {
+    "attention_b1": dict(sources=("attention.cuh", "ptx.cuh"), bytes=5002069, algorithmic=4823040,
+                         sha256="06dec0a6372c8c089f2878d8cc6e2a400cf336f9289bf7cad4281e0c8fe06266"),
+    "attention_serve": dict(sources=("attention.cuh", "ptx.cuh"), bytes=233307904,
+                            algorithmic=225173504,
+                            sha256="06dec0a6372c8c089f2878d8cc6e2a400cf336f9289bf7cad4281e0c8fe06266"),
+    "lm_head_b1": dict(sources=("gemm_tc.cuh", "gemm.cu", "ptx.cuh"), bytes=124822784,
+                       algorithmic=121669768,
+                       sha256="acd78b83a80ba74bcd7c190a8f523f7fc8182269637458b3430e12d923ff8077"),
+}
+
+
+def ncu_traffic(key: str, algorithmic: int):
+    """Measured DRAM bytes for a launch of `algorithmic` bytes, or None once
+    the kernel has changed since its capture."""
+    import hashlib
+    e = NCU_TRAFFIC[key]
+    h = hashlib.sha256()
+    for f in e["sources"]:
+        with open(os.path.join(_CSRC, f), "rb") as fh:
+            h.update(fh.read())
+    if h.hexdigest() != e["sha256"]:
+        return None
+    return int(round(e["bytes"] * algorithmic / e["algorithmic"]))
+
+
 def load_peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
@@ -369,12 +402,18 @@ def gpu_arm(args, rank: int, world: int):
                 "us_per_launch": dk["us_per_launch"], "launches_per_step": dk["launches"],
                 "timing": timing, "traffic": None}
     else:
+        traffic = None
+        if dom == "attention":
+            traffic = ncu_traffic("attention_b1" if B == 1 else "attention_serve",
+                                  dk["bytes_per_launch"])
         roof = {"kernel": f"{dom} (gemm_tc_kernel / attn_paged_kernel by kind), {T} rows",
                 "bound": "hbm", "achieved": dk["gb_s"], "peak": hbm, "unit": "GB/s",
                 "frac": dk["frac_hbm"], "peak_source": src,
                 "algorithmic_bytes_per_launch": dk["bytes_per_launch"],
                 "us_per_launch": dk["us_per_launch"], "launches_per_step": dk["launches"],
-                "timing": timing, "traffic": None}
+                "timing": timing, "traffic": traffic,
+                "traffic_source": "ncu dram bytes of the standalone kernel, scaled by algorithmic bytes"
+                if traffic is not None else None}
     lm = lm_head_roofline(cfg, K, dev) if B == 1 else None
     attn = attention_roofline(cfg, dev)
     res = dict(elapsed=elapsed, e2e_elapsed=e_elapsed, tokens=committed_per_decode * args.steps,
@@ -443,7 +482,7 @@ def lm_head_roofline(cfg, K, dev):
     return {"kernel": "gemm_tc_kernel<32, argmax> (LM head 17x59392x1024)", "bound": "hbm",
             "achieved": round(achieved, 1), "peak": hbm, "unit": "GB/s",
             "frac": round(achieved / hbm, 4), "peak_source": src, "algorithmic_bytes": algo,
-            "us_per_launch": round(t * 1e6, 2), "traffic": None}
+            "us_per_launch": round(t * 1e6, 2), "traffic": ncu_traffic("lm_head_b1", algo)}
 
 
 def attention_roofline(cfg, dev, ns=None, K=16):
@@ -498,7 +537,8 @@ def attention_roofline(cfg, dev, ns=None, K=16):
     return {"kernel": f"attn_paged_kernel (draft, {B} seqs, mean cached {int(ns.mean())}, K={K}, "
                       f"{sp} pages per item)", "bound": "hbm",
             "achieved": round(achieved, 1), "peak": hbm, "unit": "GB/s",
-            "frac": round(achieved / hbm, 4), "kv_bytes": algo, "us_per_launch": round(t * 1e6, 2)}
+            "frac": round(achieved / hbm, 4), "kv_bytes": algo, "us_per_launch": round(t * 1e6, 2),
+            "traffic": ncu_traffic("attention_b1" if B == 1 else "attention_serve", algo)}
 
 
 # ---------------------------------------------------------------------- oracle arm
