@@ -122,18 +122,22 @@ int decode_splits(int weight_rows, int K) {
   return s;
 }
 
-// Decode windows of up to 64 tokens split K across the CTAs of a cluster;
-// wider decode launches reduce the same K chunks inside each CTA (one TMEM
-// accumulator per chunk, summed in chunk order).  The chunks' accumulators
-// take at most 256 TMEM columns, so two CTAs share an SM, and the token tile
-// shrinks until the launch covers about one wave.  Prefill does not split K.
-GemmPlan plan_split(int weight_rows, int T, int S) {
+// Decode windows of up to 64 tokens split K across the CTAs of a cluster.
+// Wider decode launches with at least 8 k-blocks per split keep that (64-token
+// tiles); the others reduce the same K chunks inside each CTA (one TMEM
+// accumulator per chunk, summed in chunk order), with the chunks'
+// accumulators in at most 256 TMEM columns, so two CTAs share an SM, and the
+// token tile shrunk until the launch covers about one wave.  All three give
+// the same sums in the same order.  Prefill does not split K.
+GemmPlan plan_split(int weight_rows, int T, int S, int nkb) {
   GemmPlan p;
   p.feat_tiles = weight_rows / 128;
   p.chunks = 1;
   p.splits = S;
   p.bn = gemm_bn_for(T);
-  if (S > 1 && T > 64 && S * 32 <= 256) {
+  if (S > 1 && T > 64 && nkb / S >= 8 && gemm_cluster_ok(64, S)) {
+    p.bn = 64;
+  } else if (S > 1 && T > 64 && S * 32 <= 256) {
     p.chunks = S;
     p.splits = 1;
     p.bn = std::min(128, 256 / S);
@@ -144,7 +148,7 @@ GemmPlan plan_split(int weight_rows, int T, int S) {
 }
 
 GemmPlan plan_gemm(int weight_rows, int K, int T, bool decode) {
-  return plan_split(weight_rows, T, decode ? decode_splits(weight_rows, K) : 1);
+  return plan_split(weight_rows, T, decode ? decode_splits(weight_rows, K) : 1, K / 64);
 }
 
 // fp32 partials the widest decode tiles (BN > 64, reduced through global
@@ -1168,11 +1172,13 @@ size_t gs_linear_scratch_bytes(int M, int N, int split_k) {
   // the larger of the plans for an N-row and a 2N-row (SwiGLU) weight
   size_t counters = 0, partial = 0;
   for (int w_rows : {N, 2 * N}) {
-    const GemmPlan p = plan_split(w_rows, M, split_k);
-    counters = std::max(counters, static_cast<size_t>(p.tok_tiles) * p.feat_tiles);
-    if (p.splits > 1 && !gemm_cluster_ok(p.bn, p.splits))
-      partial = std::max(partial, static_cast<size_t>(p.splits) * p.tok_tiles * p.feat_tiles *
-                                      p.bn * 128);
+    for (int nkb : {split_k, 8 * split_k}) {   // the plans for short and long K per split
+      const GemmPlan p = plan_split(w_rows, M, split_k, nkb);
+      counters = std::max(counters, static_cast<size_t>(p.tok_tiles) * p.feat_tiles);
+      if (p.splits > 1 && !gemm_cluster_ok(p.bn, p.splits))
+        partial = std::max(partial, static_cast<size_t>(p.splits) * p.tok_tiles * p.feat_tiles *
+                                        p.bn * 128);
+    }
   }
   Carver cv(nullptr);
   cv.take<int>(64);
@@ -1200,7 +1206,7 @@ int gs_linear(const void* x, const void* w, void* y, int M, int N, int K, int ep
   // split-K as the decoder plans it: across the CTAs of a cluster (up to 64
   // rows), as chunks inside each CTA (wider), else through global scratch
   const int w_rows = epilogue == kEpiSwiGLU ? 2 * N : N;
-  const GemmPlan p = plan_split(w_rows, M, split_k);
+  const GemmPlan p = plan_split(w_rows, M, split_k, K / 64);
   const int bn = p.bn, tok_tiles = p.tok_tiles, feat_tiles = p.feat_tiles;
   CUtensorMap tw, tx;
   if (!make_map(&tw, w, w_rows, K, epilogue == kEpiSwiGLU ? 64 : 128)) return GS_ERR_INVALID_ARG;
