@@ -46,7 +46,7 @@ enum {
   GS_OK = 0,
   GS_ERR_INVALID_ARG = 1,   /* bad pointer, size, slot or config value        */
   GS_ERR_OOM = 2,           /* workspace too small / KV page pool exhausted    */
-  GS_ERR_UNSUPPORTED = 3,   /* valid request this build does not implement     */
+  GS_ERR_UNSUPPORTED = 3,   /* valid request the library does not implement   */
   GS_ERR_CUDA = 4,          /* a CUDA runtime call failed                      */
   GS_ERR_DEVICE_CHECK = 5,  /* a kernel's bounds check fired                   */
   GS_ERR_TIMEOUT = 6        /* a kernel's bounded wait ran out                 */
@@ -271,7 +271,11 @@ int gs_attention(int mode, const void *q, const void *kv, int n_pages, const int
  *   [2N, K] (gate rows then up rows), y fp16 [M, N] = silu(gate) * up;
  *   3: argmax: y is uint64 [M] packed (ordered fp32 bits << 32 | ~index),
  *   combined with atomicMax (caller zeroes it first).
- *   split_k: 1 or a divisor of K/64; scratch device >= gs_linear_scratch_bytes.
+ *   split_k S: 1 or a divisor of K/64.  K is reduced as S consecutive chunks,
+ *   each summed from zero in k order, then the chunks summed in order
+ *   0..S-1.  Where the chunks are reduced (across a cluster of CTAs, inside
+ *   one CTA, or through the scratch) depends on M; the sums do not, so a row's
+ *   result is the same for any M.  scratch device >= gs_linear_scratch_bytes.
  *   Requirements: K % 64 == 0, N % 128 == 0 (N % 64 for epilogue 2), M >= 1. */
 size_t gs_linear_scratch_bytes(int M, int N, int split_k);
 int gs_linear(const void *x, const void *w, void *y, int M, int N, int K, int epilogue, int split_k,
