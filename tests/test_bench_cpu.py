@@ -1,0 +1,67 @@
+"""Host logic of bench.py (no GPU): the decode length of a forced schedule,
+the algorithmic-byte model the roofline lines use, and the gating of the
+measured DRAM traffic on the kernels' sources."""
+import json
+import math
+
+import numpy as np
+
+import bench
+import synth
+
+GLM = synth.WORKLOADS["glm_b1"].model
+
+
+def test_schedule_rounds_counts_committed_tokens():
+    # every round commits L + 2 tokens; the boundary token x0 is the first output
+    K, max_new = 16, 512
+    full = np.full(100, K, np.int64)
+    assert bench.schedule_rounds(full, max_new) == math.ceil((max_new - 1) / (K + 2))
+    zero = np.zeros(400, np.int64)
+    assert bench.schedule_rounds(zero, max_new) == math.ceil((max_new - 1) / 2)
+    sched = np.array([3, 0, 16, 5] * 50)
+    n, r = 1, 0
+    while n < max_new:           # brute force
+        n += int(sched[r]) + 2
+        r += 1
+    assert bench.schedule_rounds(sched, max_new) == r
+
+
+def test_weight_bytes_per_forward_match_the_model():
+    # the five projection kinds at any T stream each weight once: summed over
+    # the layers and the LM head they must give the model's matrix bytes
+    T = 17
+    per_layer = sum(bench.gemm_flops(GLM, k, T) // (2 * T) for k in ("qkv", "o_proj", "gate_up", "down"))
+    total = GLM.n_layers * per_layer + bench.gemm_flops(GLM, "lm_head", T) // (2 * T)
+    assert total * 2 == 876_609_536            # 438.3M fp16 weights = 876.6 MB per forward
+    for kind in ("qkv", "o_proj", "gate_up", "down", "lm_head"):
+        b = bench.kernel_bytes(GLM, kind, T, [])
+        w = bench.gemm_flops(GLM, kind, T) // (2 * T) * 2
+        assert w < b < w + 64 * T * GLM.d_ffn, kind   # weights plus per-row activation traffic
+
+
+def test_attention_bytes_count_k_and_v_rows_once():
+    T = 17
+    ctx = [2048 + T, 3000 + T]
+    b = bench.kernel_bytes(GLM, "attention", 2 * T, ctx)
+    kv = sum(ctx) * GLM.n_kv_heads * GLM.head_dim * 2 * 2       # K and V, fp16
+    qo = 2 * (2 * 2 * T * GLM.n_heads * GLM.head_dim)          # q read + out written, fp16
+    assert b == kv + qo
+
+
+def test_measured_traffic_is_gated_on_the_kernel_sources(monkeypatch):
+    e = bench.NCU_TRAFFIC["lm_head_b1"]
+    assert bench.ncu_traffic("lm_head_b1", e["algorithmic"]) == e["bytes"]
+    assert bench.ncu_traffic("lm_head_b1", 2 * e["algorithmic"]) == 2 * e["bytes"]
+    changed = dict(bench.NCU_TRAFFIC)
+    changed["lm_head_b1"] = dict(e, sha256="0" * 64)           # the kernel changed since
+    monkeypatch.setattr(bench, "NCU_TRAFFIC", changed)
+    assert bench.ncu_traffic("lm_head_b1", e["algorithmic"]) is None
+
+
+def test_config_names_the_workload():
+    wl = synth.WORKLOADS["serve_b32"]
+    d = bench.describe(wl, wl.K, wl.accept_mean, 1)
+    json.dumps(d)
+    assert "serve_b32" in d["workload"] and d["global_batch"] == 32 and d["K"] == wl.K
+    assert bench.describe(wl, wl.K, wl.accept_mean, 4)["global_batch"] == 128
