@@ -426,6 +426,21 @@ def gpu_arm(args, rank: int, world: int):
     return res
 
 
+def job_totals(elapsed: float, e2e_elapsed: float, tokens: int, world: int, device):
+    """Whole-job figures over the ranks (replicas, one per GPU): the slowest
+    rank's timed and end-to-end seconds (max) and the tokens every rank
+    committed (sum).  One rank: the inputs."""
+    if world <= 1:
+        return elapsed, e2e_elapsed, tokens
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([elapsed, e2e_elapsed], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    n = torch.tensor([float(tokens)], dtype=torch.float64, device=device)
+    dist.all_reduce(n, op=dist.ReduceOp.SUM)
+    return float(t[0]), float(t[1]), int(round(float(n[0])))
+
+
 def _time_kernel(fn, iters: int):
     """Average device seconds of one fn() launch: `iters` launches captured as
     one CUDA graph and replayed, so no host enqueue time falls between them.
@@ -674,14 +689,7 @@ def main():
         import torch.distributed as dist
         dist.init_process_group("nccl", device_id=torch.device("cuda", int(os.environ["LOCAL_RANK"])))
     res = gpu_arm(args, rank, world)
-    el = res["elapsed"]
-    ee = res["e2e_elapsed"]
-    if world > 1:
-        import torch.distributed as dist
-        t = torch.tensor([el, ee], dtype=torch.float64, device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        el, ee = float(t[0]), float(t[1])
-    tokens_all = res["tokens"] * max(world, 1)
+    el, ee, tokens_all = job_totals(res["elapsed"], res["e2e_elapsed"], res["tokens"], world, "cuda")
     value = tokens_all / el
     rms = res["round_ms"]
     B = res["B"]
