@@ -500,10 +500,11 @@ def lm_head_roofline(cfg, K, dev):
             "us_per_launch": round(t * 1e6, 2), "traffic": ncu_traffic("lm_head_b1", algo)}
 
 
-def attention_roofline(cfg, dev, ns=None, K=16):
-    """Hybrid-mask draft attention alone over a paged pool.  Default shape: the
-    serving one (32 sequences, prefix U[1024, 6144] -> mean ~3600, K = 16, a
-    pool larger than L2); `ns` gives other cached lengths (one per sequence)."""
+def attention_roofline(cfg, dev, ns=None, K=16, mode=0):
+    """Hybrid-mask attention alone over a paged pool (mode 0: draft masks, 1:
+    verify masks).  Default shape: the serving one (32 sequences, prefix
+    U[1024, 6144] -> mean ~3600, K = 16, a pool larger than L2); `ns` gives
+    other cached lengths (one per sequence)."""
     import torch
     from paper_2609_26638_gb300 import gs
     hbm, _, src = load_peaks()
@@ -541,16 +542,16 @@ def attention_roofline(cfg, dev, ns=None, K=16):
     def fn():
         kv = kvs[it[0] % n_copy]
         it[0] += 1
-        gs.gs_attention(0, q.data_ptr(), kv.data_ptr(), n_pages, ptd.data_ptr(), pt_stride,
+        gs.gs_attention(mode, q.data_ptr(), kv.data_ptr(), n_pages, ptd.data_ptr(), pt_stride,
                         nd.data_ptr(), B, W, Hq, Hkv, out.data_ptr(), scratch.data_ptr(), sb, sp,
                         torch.cuda.current_stream(dev).cuda_stream)
 
     t = _time_kernel(fn, 64 if B == 1 else 20)
-    keys = int(sum(int(n) + W for n in ns))
+    keys = int(sum(int(n) + W + mode for n in ns))   # the verify window reaches one slot further
     algo = keys * Hkv * 64 * 2 * 2 + 2 * B * W * Hq * 64 * 2
     achieved = algo / t / 1e9
-    return {"kernel": f"attn_paged_kernel (draft, {B} seqs, mean cached {int(ns.mean())}, K={K}, "
-                      f"{sp} pages per item)", "bound": "hbm",
+    return {"kernel": f"attn_paged_kernel ({'verify' if mode else 'draft'}, {B} seqs, mean cached "
+                      f"{int(ns.mean())}, K={K}, {sp} pages per item)", "bound": "hbm",
             "achieved": round(achieved, 1), "peak": hbm, "unit": "GB/s",
             "frac": round(achieved / hbm, 4), "kv_bytes": algo, "us_per_launch": round(t * 1e6, 2),
             "traffic": ncu_traffic("attention_b1" if B == 1 else "attention_serve", algo)}
@@ -634,10 +635,12 @@ def main():
     ap.add_argument("--no-compare-ar", dest="compare_ar", action="store_false",
                     help="skip timing plain greedy AR (K = 0 rounds) on the same workload")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--kernel", default=None, choices=["attention", "lm_head"],
+    ap.add_argument("--kernel", default=None, choices=["attention", "lm_head", "attention-sweep"],
                     help="time one kernel alone and print its roofline line (the single-kernel "
                          "ncu captures run this): attention at the workload's decode shape "
-                         "(the serving batch for serve_b32), the LM head at 17 rows")
+                         "(the serving batch for serve_b32), the LM head at 17 rows; "
+                         "attention-sweep: one line per point of K {4,8,16,32,64} x batch "
+                         "{1,8,64} x prefix {1024,4096,8192}, draft and verify masks")
     args = ap.parse_args()
     if args.kernel is not None:
         import torch
@@ -646,6 +649,16 @@ def main():
         cfg = synth.WORKLOADS[args.workload].model
         K = synth.WORKLOADS[args.workload].K if args.K is None else args.K
         wl = synth.WORKLOADS[args.workload]
+        if args.kernel == "attention-sweep":
+            for mode in (0, 1):
+                for Ks in (4, 8, 16, 32, 64):
+                    for Bs in (1, 8, 64):
+                        for pre in (1024, 4096, 8192):
+                            r = attention_roofline(cfg, dev, [pre] * Bs, Ks, mode)
+                            r.update(mode="verify" if mode else "draft", K=Ks, batch=Bs, prefix=pre)
+                            print(json.dumps(r), flush=True)
+                            torch.cuda.empty_cache()
+            return
         if args.kernel == "lm_head":
             r = lm_head_roofline(cfg, K, dev)
         elif wl.batch == 1:   # mid-decode of the single-sequence workload
