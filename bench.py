@@ -500,6 +500,49 @@ def lm_head_roofline(cfg, K, dev):
             "us_per_launch": round(t * 1e6, 2), "traffic": ncu_traffic("lm_head_b1", algo)}
 
 
+def gemm_serve_rooflines(cfg, dev, T=544):
+    """The four projections at the serving window (32 sequences x 17 rows) alone,
+    through gs_linear with the decoder's split-K factors (so the same tile plans
+    and kernels as the round), over rotating weight copies larger than L2.
+    Down first (the single-kernel ncu capture takes the first launches)."""
+    import torch
+    from paper_2609_26638_gb300 import gs
+    _, bf16_tf, src = load_peaks()
+    d, F, HD = cfg.d_model, cfg.d_ffn, cfg.n_heads * cfg.head_dim
+    # name, N (output features), K, epilogue, split-K as the decoder plans it
+    shapes = [("down", d, F, gs.EPI_RESID_F32, 8), ("gate_up", F, d, gs.EPI_SWIGLU, 4),
+              ("qkv", cfg.qkv_dim, d, gs.EPI_STORE_F16, 8), ("o_proj", d, HD, gs.EPI_RESID_F32, 8)]
+    g = torch.Generator(device=dev).manual_seed(0)
+    out = []
+    for name, N, Kd, epi, split in shapes:
+        wrows = 2 * N if epi == gs.EPI_SWIGLU else N
+        n_copy = max(1, math.ceil(300e6 / (wrows * Kd * 2)))
+        ws = [(0.02 * torch.randn(wrows, Kd, device=dev, generator=g)).half() for _ in range(n_copy)]
+        x = torch.randn(T, Kd, device=dev, generator=g).half()
+        y = torch.zeros(T, N, dtype=torch.float32 if epi == gs.EPI_RESID_F32 else torch.float16,
+                        device=dev)
+        sb = gs.gs_linear_scratch_bytes(T, N, split)
+        scratch = torch.zeros(sb, dtype=torch.uint8, device=dev)
+        it = [0]
+
+        def fn():
+            w = ws[it[0] % n_copy]
+            it[0] += 1
+            gs.gs_linear(x.data_ptr(), w.data_ptr(), y.data_ptr(), T, N, Kd, epi, split,
+                         scratch.data_ptr(), sb, torch.cuda.current_stream(dev).cuda_stream)
+
+        t = _time_kernel(fn, 20)
+        flops = 2 * T * wrows * Kd
+        tf = flops / t / 1e12
+        out.append({"kernel": f"gemm_tc_kernel ({name}, {T} x {wrows} x {Kd}, split-K {split})",
+                    "bound": "tensor", "achieved": round(tf, 1), "peak": bf16_tf, "unit": "TFLOP/s",
+                    "frac": round(tf / bf16_tf, 4), "peak_source": src + " bf16 burst",
+                    "flops": flops, "us_per_launch": round(t * 1e6, 2)})
+        del ws
+        torch.cuda.empty_cache()
+    return out
+
+
 def attention_roofline(cfg, dev, ns=None, K=16, mode=0):
     """Hybrid-mask attention alone over a paged pool (mode 0: draft masks, 1:
     verify masks).  Default shape: the serving one (32 sequences, prefix
@@ -635,12 +678,14 @@ def main():
     ap.add_argument("--no-compare-ar", dest="compare_ar", action="store_false",
                     help="skip timing plain greedy AR (K = 0 rounds) on the same workload")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--kernel", default=None, choices=["attention", "lm_head", "attention-sweep"],
+    ap.add_argument("--kernel", default=None,
+                    choices=["attention", "lm_head", "attention-sweep", "gemm-serve"],
                     help="time one kernel alone and print its roofline line (the single-kernel "
                          "ncu captures run this): attention at the workload's decode shape "
                          "(the serving batch for serve_b32), the LM head at 17 rows; "
                          "attention-sweep: one line per point of K {4,8,16,32,64} x batch "
-                         "{1,8,64} x prefix {1024,4096,8192}, draft and verify masks")
+                         "{1,8,64} x prefix {1024,4096,8192}, draft and verify masks; "
+                         "gemm-serve: the four projections at the 544-row serving window")
     args = ap.parse_args()
     if args.kernel is not None:
         import torch
@@ -649,6 +694,10 @@ def main():
         cfg = synth.WORKLOADS[args.workload].model
         K = synth.WORKLOADS[args.workload].K if args.K is None else args.K
         wl = synth.WORKLOADS[args.workload]
+        if args.kernel == "gemm-serve":
+            for r in gemm_serve_rooflines(cfg, dev):
+                print(json.dumps(r), flush=True)
+            return
         if args.kernel == "attention-sweep":
             for mode in (0, 1):
                 for Ks in (4, 8, 16, 32, 64):
