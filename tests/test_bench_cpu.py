@@ -50,13 +50,19 @@ def test_attention_bytes_count_k_and_v_rows_once():
 
 
 def test_measured_traffic_is_gated_on_the_kernel_sources(monkeypatch):
-    e = bench.NCU_TRAFFIC["lm_head_b1"]
-    assert bench.ncu_traffic("lm_head_b1", e["algorithmic"]) == e["bytes"]
-    assert bench.ncu_traffic("lm_head_b1", 2 * e["algorithmic"]) == 2 * e["bytes"]
-    changed = dict(bench.NCU_TRAFFIC)
-    changed["lm_head_b1"] = dict(e, sha256="0" * 64)           # the kernel changed since
-    monkeypatch.setattr(bench, "NCU_TRAFFIC", changed)
-    assert bench.ncu_traffic("lm_head_b1", e["algorithmic"]) is None
+    import hashlib
+    import os
+    srcs = ("gemm_tc.cuh", "gemm.cu", "ptx.cuh")
+    h = hashlib.sha256()
+    for f in srcs:
+        with open(os.path.join(bench._CSRC, f), "rb") as fh:
+            h.update(fh.read())
+    cur = dict(sources=srcs, bytes=1000, algorithmic=800, sha256=h.hexdigest())
+    table = dict(bench.NCU_TRAFFIC, probe=cur, stale=dict(cur, sha256="0" * 64))
+    monkeypatch.setattr(bench, "NCU_TRAFFIC", table)
+    assert bench.ncu_traffic("probe", 800) == 1000            # sources as captured
+    assert bench.ncu_traffic("probe", 1600) == 2000           # scaled by algorithmic bytes
+    assert bench.ncu_traffic("stale", 800) is None            # the kernel changed since
 
 
 def test_config_names_the_workload():
