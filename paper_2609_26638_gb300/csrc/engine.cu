@@ -6,6 +6,7 @@
 #include <cstdio>
 #include <cstring>
 #include <map>
+#include <mutex>
 #include <string>
 #include <tuple>
 #include <vector>
@@ -89,6 +90,30 @@ AttnGeom attn_geom(int W, int G) {
 // launch is about one wave (a cluster waits for free SMs of one GPC, and
 // clusters fragment larger grids); otherwise through global scratch.  Both
 // give the same bits.
+}  // namespace
+
+// Kernel attributes (dynamic shared memory above 48 KB, non-portable cluster
+// sizes) are set once per device, under a lock, before the first launch.
+cudaError_t gs::ensure_kernel_attributes() {
+  static std::mutex mu;
+  static uint64_t done = 0;   // bit d: device d configured
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  std::lock_guard<std::mutex> lock(mu);
+  if (dev < 64 && ((done >> dev) & 1)) return cudaSuccess;
+  e = gemm_init_attributes();
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(attn_paged_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             attn_max_smem_bytes());
+  if (e == cudaSuccess)   // clusters of up to 16 attention items
+    e = cudaFuncSetAttribute(attn_paged_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  if (e == cudaSuccess && dev < 64) done |= 1ull << dev;
+  return e;
+}
+
+namespace {
+
 bool attn_use_cluster(int items, int blocks_x_heads) {
   return items <= kAttnMaxCluster && items * blocks_x_heads <= 2 * kNumSMs;
 }
@@ -680,19 +705,8 @@ int gs_create(const gs_config* cfg, const gs_weights* w, void* workspace, size_t
   if (ws_bytes < need)
     return fail(nullptr, GS_ERR_OOM, "workspace too small: need " + std::to_string(need));
   if (!get_encode()) return fail(nullptr, GS_ERR_CUDA, "cuTensorMapEncodeTiled unavailable");
-  static bool attrs_done = false;
-  if (!attrs_done) {
-    cudaError_t e = gemm_init_attributes();
-    if (e == cudaSuccess)
-      e = cudaFuncSetAttribute(attn_paged_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                               attn_max_smem_bytes());
-    if (e == cudaSuccess)   // clusters of up to 16 items
-      e = cudaFuncSetAttribute(attn_paged_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
-
-    if (e != cudaSuccess)
-      return fail(nullptr, GS_ERR_CUDA, std::string("kernel attributes: ") + cudaGetErrorString(e));
-    attrs_done = true;
-  }
+  if (const cudaError_t e = ensure_kernel_attributes(); e != cudaSuccess)
+    return fail(nullptr, GS_ERR_CUDA, std::string("kernel attributes: ") + cudaGetErrorString(e));
 
   gs_handle* h = new gs_handle();
   h->cfg = *cfg;
@@ -1110,15 +1124,7 @@ int gs_attention(int mode, const void* q, const void* kv, int n_pages, const int
     return GS_ERR_OOM;
   if ((reinterpret_cast<uintptr_t>(kv) & 15) || (reinterpret_cast<uintptr_t>(q) & 15))
     return GS_ERR_INVALID_ARG;
-  static bool attr = false;
-  if (!attr) {
-    if (cudaFuncSetAttribute(attn_paged_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             attn_max_smem_bytes()) != cudaSuccess ||
-        cudaFuncSetAttribute(attn_paged_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed,
-                             1) != cudaSuccess)
-      return GS_ERR_CUDA;
-    attr = true;
-  }
+  if (ensure_kernel_attributes() != cudaSuccess) return GS_ERR_CUDA;
   const AttnGeom g = attn_geom(W, G);
   const int items = cdiv(pt_stride, split_pages);
   if (items > attn_max_merge_items(g.rows)) return GS_ERR_UNSUPPORTED;
@@ -1198,11 +1204,7 @@ int gs_linear(const void* x, const void* w, void* y, int M, int N, int K, int ep
   if (scratch_bytes < gs_linear_scratch_bytes(M, N, split_k)) return GS_ERR_OOM;
   if ((reinterpret_cast<uintptr_t>(x) & 15) || (reinterpret_cast<uintptr_t>(w) & 15))
     return GS_ERR_INVALID_ARG;
-  static bool attrs = false;
-  if (!attrs) {
-    if (gemm_init_attributes() != cudaSuccess) return GS_ERR_CUDA;
-    attrs = true;
-  }
+  if (ensure_kernel_attributes() != cudaSuccess) return GS_ERR_CUDA;
   // split-K as the decoder plans it: across the CTAs of a cluster (up to 64
   // rows), as chunks inside each CTA (wider), else through global scratch
   const int w_rows = epilogue == kEpiSwiGLU ? 2 * N : N;

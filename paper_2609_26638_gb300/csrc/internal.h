@@ -66,5 +66,8 @@ cudaError_t launch_gemm(int bn, int epi, const CUtensorMap& tmW, const CUtensorM
 
 // Sets the dynamic shared-memory limit of every GEMM instantiation once.
 cudaError_t gemm_init_attributes();
+// Every kernel's launch attributes on the current device, once per device
+// (thread-safe); call before the first launch.
+cudaError_t ensure_kernel_attributes();
 
 }  // namespace gs

@@ -99,11 +99,7 @@ extern "C" int gs_linear_noalloc(const void* x, const void* w, void* y, int M, i
                   : 0;
   if (err_bytes + cnt_bytes + part_bytes > GS_NOALLOC_SCRATCH_BYTES) return GS_ERR_OOM;
 
-  static bool attrs = false;
-  if (!attrs) {
-    if (gemm_init_attributes() != cudaSuccess) return GS_ERR_CUDA;
-    attrs = true;
-  }
+  if (ensure_kernel_attributes() != cudaSuccess) return GS_ERR_CUDA;
   void* base = nullptr;
   int rc = scratch_for_current_device(&base);
   if (rc != GS_OK) return rc;
