@@ -232,6 +232,16 @@ int gs_release(gs_handle *h, int slot);
  * failure raised since the last call (then clear it). */
 int gs_sync_check(gs_handle *h);
 
+/* Failure-detection self-test (the paper has no counterpart).  Enqueues on
+ * the handle's stream one kernel that waits, through the same bounded
+ * mbarrier wait every pipeline of the library uses, on a barrier nothing
+ * arrives on; the wait gives up after limit_us microseconds of device time
+ * (1 <= limit_us <= 2,000,000) and raises the timeout code in the handle's
+ * error word, so the next gs_sync_check returns GS_ERR_TIMEOUT.  The context
+ * stays usable: nothing else is in flight in the probe's CTA.
+ * Errors: GS_ERR_INVALID_ARG, GS_ERR_CUDA. */
+int gs_wait_probe(gs_handle *h, int limit_us);
+
 /* ---------------------------------------------------------------------------
  * Sub-steps exposed for the attention-only sweep and kernel parity tests.
  * ------------------------------------------------------------------------ */
@@ -248,9 +258,11 @@ int gs_sync_check(gs_handle *h);
  *   page_table device int32 [n_seq, pt_stride]: logical page -> physical page
  *   n        device int32 [n_seq]: n_s
  *   out      device fp16 [n_seq, W, n_heads, 64]
- *   scratch  device, >= gs_attention_scratch_bytes(...) bytes: key limits, the
- *            block -> page-table map, merge tickets and the fp32 partial rows
- *            (O, m, l) of every work item
+ *   scratch  device, >= gs_attention_scratch_bytes(...) bytes: the kernel's
+ *            error word (first int32: 0 = no failure, 1 = bounds check,
+ *            2 = bounded wait ran out, 3 = fp16 range; cleared by each call),
+ *            key limits, the block -> page-table map, merge tickets and the
+ *            fp32 partial rows (O, m, l) of every work item
  *   split_pages pages per work item (>= 1): item i of a sequence covers its
  *            logical pages [i * split_pages, (i + 1) * split_pages); items are
  *            reduced independently and merged in item order, so results depend
@@ -275,7 +287,11 @@ int gs_attention(int mode, const void *q, const void *kv, int n_pages, const int
  *   each summed from zero in k order, then the chunks summed in order
  *   0..S-1.  Where the chunks are reduced (across a cluster of CTAs, inside
  *   one CTA, or through the scratch) depends on M; the sums do not, so a row's
- *   result is the same for any M.  scratch device >= gs_linear_scratch_bytes.
+ *   result is the same for any M.  scratch device >= gs_linear_scratch_bytes,
+ *   any contents: the call clears the parts that must start at zero.  Its
+ *   first int32 is the kernel's error word after the stream reaches the end
+ *   of the call (0 = no failure, 1 = bounds check, 2 = bounded wait ran out,
+ *   3 = a value beyond the fp16 range).
  *   Requirements: K % 64 == 0, N % 128 == 0 (N % 64 for epilogue 2), M >= 1. */
 size_t gs_linear_scratch_bytes(int M, int N, int split_k);
 int gs_linear(const void *x, const void *w, void *y, int M, int N, int K, int epilogue, int split_k,
@@ -296,7 +312,9 @@ int gs_linear(const void *x, const void *w, void *y, int M, int N, int K, int ep
  * makes no cudaMalloc / cudaFree and calls no allocating library routine.
  *   - The first call on a device looks up that array's device address (with
  *     the device current); make that first call before any stream capture.
- *   - Every call clears the counters it uses before its kernel runs.
+ *   - Every call clears the counters it uses and the error word before its
+ *     kernel runs.  gs_linear_noalloc_status reports that call's kernel-side
+ *     checks.
  *   - All calls share the one array: calls whose kernels overlap on the GPU
  *     (two streams, or two host threads on one device) race; serialise them.
  * Errors: as gs_linear; GS_ERR_OOM when split_k x tiles of partials for
@@ -305,6 +323,14 @@ int gs_linear(const void *x, const void *w, void *y, int M, int N, int K, int ep
 #define GS_NOALLOC_SCRATCH_BYTES (8u << 20)
 int gs_linear_noalloc(const void *x, const void *w, void *y, int M, int N, int K, int epilogue,
                       int split_k, void *stream);
+
+/* Kernel-side status of the most recent gs_linear_noalloc on the current
+ * device: synchronises `stream` (the one that call used), then returns GS_OK,
+ * GS_ERR_DEVICE_CHECK (a bounds check fired or a value left the fp16 range)
+ * or GS_ERR_TIMEOUT (a bounded wait ran out), and clears the word.  Call it
+ * before the next gs_linear_noalloc, which clears the word again.  Allocates
+ * nothing.  Errors: GS_ERR_CUDA. */
+int gs_linear_noalloc_status(void *stream);
 
 #ifdef __cplusplus
 }

@@ -28,22 +28,24 @@ typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t,
                                   const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
                                   CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
 
+// The driver's tensor-map encoder, looked up once per process.
 EncodeTiledFn get_encode() {
+  static std::once_flag once;
   static EncodeTiledFn fn = nullptr;
-  if (!fn) {
+  std::call_once(once, [] {
     void* p = nullptr;
     cudaDriverEntryPointQueryResult q;
     if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
                                          &q) == cudaSuccess &&
         q == cudaDriverEntryPointSuccess)
       fn = reinterpret_cast<EncodeTiledFn>(p);
-  }
+  });
   return fn;
 }
+}  // namespace
 
-// 2-D fp16 tensor map over a row-major [rows, cols] array, box {64, box_rows},
-// 128-byte swizzle, zero fill out of bounds.
-bool make_map(CUtensorMap* m, const void* base, uint64_t rows, uint64_t cols, uint32_t box_rows) {
+bool gs::make_map(CUtensorMap* m, const void* base, uint64_t rows, uint64_t cols,
+                  uint32_t box_rows) {
   EncodeTiledFn enc = get_encode();
   if (!enc) return false;
   cuuint64_t dims[2] = {cols, rows};
@@ -55,6 +57,8 @@ bool make_map(CUtensorMap* m, const void* base, uint64_t rows, uint64_t cols, ui
                    CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;
 }
+
+namespace {
 
 inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 inline int cdiv(long long a, long long b) { return static_cast<int>((a + b - 1) / b); }
@@ -1063,6 +1067,14 @@ int gs_seq_state(gs_handle* h, int slot, int* seq_len, int* x0, int* n_out, int*
   return GS_OK;
 }
 
+int gs_wait_probe(gs_handle* h, int limit_us) {
+  if (!h) return GS_ERR_INVALID_ARG;
+  if (limit_us < 1 || limit_us > 2000000) return fail(h, GS_ERR_INVALID_ARG, "limit_us out of range");
+  wait_probe_kernel<<<1, 32, 0, h->stream>>>(h->err_word, static_cast<uint64_t>(limit_us) * 1000u);
+  GS_CUDA(h, cudaGetLastError());
+  return GS_OK;
+}
+
 int gs_sync_check(gs_handle* h) {
   if (!h) return GS_ERR_INVALID_ARG;
   GS_CUDA(h, cudaStreamSynchronize(h->stream));
@@ -1217,6 +1229,9 @@ int gs_linear(const void* x, const void* w, void* y, int M, int N, int K, int ep
   GemmArgs a = {};
   a.err = cv.take<int>(64);
   a.counters = cv.take<int>(static_cast<size_t>(tok_tiles) * feat_tiles);
+  // The error word and the per-tile arrival counters of the global split-K
+  // path must start at zero, whatever the caller's scratch held before.
+  const size_t head_bytes = cv.off;
   a.cluster = p.splits > 1 && gemm_cluster_ok(bn, p.splits) ? 1 : 0;
   a.partial = p.splits > 1 && !a.cluster
                   ? cv.take<float>(static_cast<size_t>(p.splits) * tok_tiles * feat_tiles * bn * 128)
@@ -1231,8 +1246,9 @@ int gs_linear(const void* x, const void* w, void* y, int M, int N, int K, int ep
   a.ldy = N;
   a.logits = nullptr;
   a.w_scale = 1.f;
-  return launch_gemm(bn, epilogue, tw, tx, a, feat_tiles, tok_tiles,
-                     static_cast<cudaStream_t>(stream)) == cudaSuccess
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (cudaMemsetAsync(scratch, 0, head_bytes, s) != cudaSuccess) return GS_ERR_CUDA;
+  return launch_gemm(bn, epilogue, tw, tx, a, feat_tiles, tok_tiles, s) == cudaSuccess
              ? GS_OK
              : GS_ERR_CUDA;
 }

@@ -64,6 +64,12 @@ cudaError_t launch_gemm(int bn, int epi, const CUtensorMap& tmW, const CUtensorM
                         const GemmArgs& args, int feat_tiles, int tok_tiles, cudaStream_t s,
                         bool pdl = false);
 
+// 2-D fp16 tensor map over a row-major [rows, cols] array, box {64 columns,
+// box_rows rows}, 128-byte swizzle, zero fill out of bounds.  The driver's
+// encoder is looked up once per process (thread-safe).  False if the lookup
+// or the encode fails.
+bool make_map(CUtensorMap* m, const void* base, uint64_t rows, uint64_t cols, uint32_t box_rows);
+
 // Sets the dynamic shared-memory limit of every GEMM instantiation once.
 cudaError_t gemm_init_attributes();
 // Every kernel's launch attributes on the current device, once per device

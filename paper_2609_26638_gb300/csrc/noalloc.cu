@@ -47,32 +47,6 @@ int scratch_for_current_device(void** out) {
   return GS_OK;
 }
 
-typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
-                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
-                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
-                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
-
-bool encode_f16_rows(CUtensorMap* m, const void* base, uint64_t rows, uint64_t cols,
-                      uint32_t box_rows) {
-  static EncodeTiledFn fn = nullptr;
-  if (!fn) {
-    void* p = nullptr;
-    cudaDriverEntryPointQueryResult q;
-    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
-                                         &q) != cudaSuccess ||
-        q != cudaDriverEntryPointSuccess)
-      return false;
-    fn = reinterpret_cast<EncodeTiledFn>(p);
-  }
-  cuuint64_t dims[2] = {cols, rows};
-  cuuint64_t strides[1] = {cols * 2};
-  cuuint32_t box[2] = {64, box_rows};
-  cuuint32_t es[2] = {1, 1};
-  return fn(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void*>(base), dims, strides, box, es,
-            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-}
-
 inline size_t up256(size_t x) { return (x + 255) / 256 * 256; }
 
 }  // namespace
@@ -104,9 +78,8 @@ extern "C" int gs_linear_noalloc(const void* x, const void* w, void* y, int M, i
   int rc = scratch_for_current_device(&base);
   if (rc != GS_OK) return rc;
   CUtensorMap tw, tx;
-  if (!encode_f16_rows(&tw, w, w_rows, K, epilogue == kEpiSwiGLU ? 64 : 128))
-    return GS_ERR_INVALID_ARG;
-  if (!encode_f16_rows(&tx, x, M, K, bn)) return GS_ERR_INVALID_ARG;
+  if (!make_map(&tw, w, w_rows, K, epilogue == kEpiSwiGLU ? 64 : 128)) return GS_ERR_INVALID_ARG;
+  if (!make_map(&tx, x, M, K, bn)) return GS_ERR_INVALID_ARG;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   uint8_t* b = static_cast<uint8_t*>(base);
   // the split-K counters must start at zero; the array keeps the last call's contents
@@ -127,4 +100,20 @@ extern "C" int gs_linear_noalloc(const void* x, const void* w, void* y, int M, i
   a.w_scale = 1.f;
   return launch_gemm(bn, epilogue, tw, tx, a, feat_tiles, tok_tiles, s) == cudaSuccess ? GS_OK
                                                                                         : GS_ERR_CUDA;
+}
+
+extern "C" int gs_linear_noalloc_status(void* stream) {
+  using namespace gs;
+  void* base = nullptr;
+  int rc = scratch_for_current_device(&base);
+  if (rc != GS_OK) return rc;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  int word = 0;
+  if (cudaMemcpyAsync(&word, base, sizeof(int), cudaMemcpyDeviceToHost, s) != cudaSuccess ||
+      cudaStreamSynchronize(s) != cudaSuccess)
+    return GS_ERR_CUDA;
+  if (word == kErrNone) return GS_OK;
+  if (cudaMemsetAsync(base, 0, sizeof(int), s) != cudaSuccess || cudaStreamSynchronize(s) != cudaSuccess)
+    return GS_ERR_CUDA;
+  return word == kErrTimeout ? GS_ERR_TIMEOUT : GS_ERR_DEVICE_CHECK;
 }

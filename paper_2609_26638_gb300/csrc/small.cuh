@@ -300,6 +300,19 @@ __global__ void rope_table_kernel(float2* tab, int max_ctx, double theta) {
   tab[idx] = make_float2(static_cast<float>(cos(ang)), static_cast<float>(sin(ang)));
 }
 
+// Failure-detection probe: one thread waits, through the same bounded
+// mbarrier wait every pipeline uses, on a barrier that nothing arrives on, so
+// the wait runs out after limit_ns and raises kErrTimeout in the error word.
+// Nothing else is in flight in this CTA (no copy, no MMA, no TMEM).
+__global__ void wait_probe_kernel(int* err, uint64_t limit_ns) {
+  __shared__ __align__(8) uint64_t bar;
+  if (threadIdx.x != 0) return;
+  mbar_init(smem_u32(&bar), 1);
+  fence_mbar_init();
+  mbar_wait(smem_u32(&bar), 0, err, limit_ns);
+  asm volatile("mbarrier.inval.shared::cta.b64 [%0];" ::"r"(smem_u32(&bar)) : "memory");
+}
+
 __global__ void copy_i32_kernel(const int32_t* src, int32_t* dst, int n) {
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
   if (i < n) dst[i] = src[i];

@@ -87,12 +87,14 @@ def _load():
         "gs_seq_state": (i32, [vp, i32] + [ctypes.POINTER(i32)] * 5),
         "gs_release": (i32, [vp, i32]),
         "gs_sync_check": (i32, [vp]),
+        "gs_wait_probe": (i32, [vp, i32]),
         "gs_attention_scratch_bytes": (sz, [i32] * 6),
         "gs_attention": (i32, [i32, vp, vp, i32, vp, i32, vp, i32, i32, i32, i32, vp, vp, sz, i32,
                                vp]),
         "gs_linear_scratch_bytes": (sz, [i32, i32, i32]),
         "gs_linear": (i32, [vp, vp, vp, i32, i32, i32, i32, i32, vp, sz, vp]),
         "gs_linear_noalloc": (i32, [vp, vp, vp, i32, i32, i32, i32, i32, vp]),
+        "gs_linear_noalloc_status": (i32, [vp]),
     }
     for name, (res, args) in sig.items():
         f = getattr(lib, name)
@@ -104,9 +106,9 @@ def _load():
 _lib = _load()
 EXPORTED = ("gs_workspace_bytes", "gs_create", "gs_destroy", "gs_last_error", "gs_prefill",
             "gs_round", "gs_seq_restore", "gs_round_launches", "gs_round_profile", "gs_seq_state",
-            "gs_release", "gs_sync_check",
+            "gs_release", "gs_sync_check", "gs_wait_probe",
             "gs_attention_scratch_bytes", "gs_attention", "gs_linear_scratch_bytes", "gs_linear",
-            "gs_linear_noalloc")
+            "gs_linear_noalloc", "gs_linear_noalloc_status")
 
 
 def lib():
@@ -192,6 +194,10 @@ def gs_sync_check(h) -> None:
     _check(h, _lib.gs_sync_check(h))
 
 
+def gs_wait_probe(h, limit_us: int) -> None:
+    _check(h, _lib.gs_wait_probe(h, limit_us))
+
+
 def gs_attention_scratch_bytes(n_seq, W, n_heads, n_kv_heads, max_pages, split_pages) -> int:
     return int(_lib.gs_attention_scratch_bytes(n_seq, W, n_heads, n_kv_heads, max_pages, split_pages))
 
@@ -227,3 +233,8 @@ def gs_linear_noalloc(x_ptr, w_ptr, y_ptr, M, N, K, epilogue, split_k, stream_pt
     rc = _lib.gs_linear_noalloc(x_ptr, w_ptr, y_ptr, M, N, K, epilogue, split_k, stream_ptr)
     if rc != GS_OK:
         raise GsError(rc, "gs_linear_noalloc")
+
+
+def gs_linear_noalloc_status(stream_ptr) -> int:
+    """GS_OK or the kernel-side failure code of the last gs_linear_noalloc (synchronises)."""
+    return int(_lib.gs_linear_noalloc_status(stream_ptr))

@@ -54,6 +54,30 @@ def test_linear_store_and_residual(gs, M, N, K, split):
     torch.testing.assert_close(r, base + ref, rtol=1e-4, atol=1e-4 * ref.abs().max().item())
 
 
+@pytest.mark.parametrize("M,N,K,split", [(9, 1024, 4096, 16), (100, 1024, 4096, 32)])
+def test_linear_clears_stale_scratch(gs, M, N, K, split):
+    """Split-K through global scratch (no cluster, no in-CTA chunks): the
+    caller's scratch arrives full of stale bytes (0x7f), as from a caching
+    allocator; the call clears the arrival counters and the error word itself,
+    so every tile is written once from all its partial sums, and the error
+    word (first int32) reads 0 afterwards."""
+    g = torch.Generator(device=DEV).manual_seed(M + split)
+    x = torch.randn(M, K, device=DEV, generator=g).half()
+    w = (0.02 * torch.randn(N, K, device=DEV, generator=g)).half()
+    ref = x.float() @ w.float().T
+    sb = gs.gs_linear_scratch_bytes(M, N, split)
+    stream = torch.cuda.current_stream().cuda_stream
+    for _ in range(2):                     # stale bytes, then the previous call's leftovers
+        y = torch.full((M, N), 7.0, dtype=torch.float16, device=DEV)
+        if _ == 0:
+            scratch = torch.full((sb,), 0x7F, dtype=torch.uint8, device=DEV)
+        gs.gs_linear(x.data_ptr(), w.data_ptr(), y.data_ptr(), M, N, K, gs.EPI_STORE_F16, split,
+                     scratch.data_ptr(), sb, stream)
+        torch.cuda.synchronize()
+        torch.testing.assert_close(y.float(), ref, rtol=2e-3, atol=1e-3 * ref.abs().max().item())
+        assert int(scratch[:4].view(torch.int32).item()) == 0
+
+
 @pytest.mark.parametrize("M,split", [(9, 1), (17, 2), (200, 1)])
 def test_linear_swiglu(gs, M, split):
     F, K = 1024, 256

@@ -181,6 +181,33 @@ def test_bad_requests_raise(tiny):
     eng.close()
 
 
+def test_bounded_wait_times_out_and_context_survives(tiny_gain):
+    """Failure detection without a GPU fault: a probe kernel waits, through the
+    bounded mbarrier wait every pipeline uses, on a barrier nothing arrives on,
+    with a 20 ms limit.  The wait runs out, gs_sync_check reports
+    GS_ERR_TIMEOUT (then the word is clear), and the context stays usable: the
+    rounds that follow commit the same tokens as before the probe."""
+    from paper_2609_26638_gb300 import gs
+    cfg, w, _ = tiny_gain
+    eng = new_engine(cfg, w, max_ctx=512, max_K=8, max_prefill=128)
+    prompt = synth.make_prompt(cfg, 40, 12, index=17)
+    slots = torch.tensor([0], dtype=torch.int32, device=eng.device)
+    eng.prefill(0, prompt.vis, prompt.text, 24)
+    before = decode_all(eng, slots, 8, 12)[0]
+    gs.gs_wait_probe(eng.handle, 20000)
+    with pytest.raises(gs.GsError) as e:
+        eng.check()
+    assert e.value.code == gs.GS_ERR_TIMEOUT
+    eng.check()                                            # cleared
+    with pytest.raises(gs.GsError) as e:
+        gs.gs_wait_probe(eng.handle, 0)
+    assert e.value.code == gs.GS_ERR_INVALID_ARG
+    eng.prefill(0, prompt.vis, prompt.text, 24)
+    after = decode_all(eng, slots, 8, 12)[0]
+    assert after == before
+    eng.close()
+
+
 def test_round_profile_matches_round(tiny_gain):
     """gs_round_profile runs the same round as gs_round (same committed tokens
     and state) and reports one timed entry per kernel launch, in launch order:

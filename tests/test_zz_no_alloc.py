@@ -39,11 +39,42 @@ def test_noalloc_matches_linear_on_two_calls_in_a_row(gs):
         _with_caller_scratch(gs, x, w, M, N, K, epi, split, want)
         got = torch.zeros(M, N, dtype=torch.float16, device=DEV)
         gs.gs_linear_noalloc(x.data_ptr(), w.data_ptr(), got.data_ptr(), M, N, K, epi, split, stream)
-        torch.cuda.synchronize()
+        assert gs.gs_linear_noalloc_status(stream) == gs.GS_OK     # synchronises the stream
         ref = x.float() @ w.float().T
         torch.testing.assert_close(got.float(), want.float(), rtol=1e-2,
                                    atol=1e-2 * ref.abs().max().item())
         torch.testing.assert_close(got.float(), ref, rtol=1e-2, atol=1e-2 * ref.abs().max().item())
+
+
+@pytest.mark.parametrize("M,N,K,epi,split", [
+    (17, 1024, 4096, 1, 8),       # residual add; gs_linear reduces its splits in a cluster
+    (200, 1024, 1024, 1, 2),      # 256-token tile here, 64-token cluster tiles in gs_linear
+    (72, 512, 1024, 2, 4),        # SwiGLU; gs_linear sums the four chunks inside one CTA
+    (100, 4096, 1024, 3, 2),      # LM-head argmax keys
+    (300, 2048, 1024, 0, 1),      # no split: two 256-token tiles
+])
+def test_noalloc_equals_linear_bitwise(gs, M, N, K, epi, split):
+    """Same split-K factor, so the same K chunks summed in the same order:
+    whatever tile width or reduction path each entry point takes, the
+    outputs are identical bit for bit, and the kernel-side status is clean."""
+    stream = torch.cuda.current_stream().cuda_stream
+    g = torch.Generator(device=DEV).manual_seed(M * 31 + epi)
+    wrows = 2 * N if epi == gs.EPI_SWIGLU else N
+    x = torch.randn(M, K, device=DEV, generator=g).half()
+    w = (0.02 * torch.randn(wrows, K, device=DEV, generator=g)).half()
+    if epi == gs.EPI_RESID_F32:
+        base = torch.randn(M, N, device=DEV, generator=g)
+        want, got = base.clone(), base.clone()
+    elif epi == gs.EPI_ARGMAX:
+        want = torch.zeros(M, dtype=torch.int64, device=DEV)
+        got = torch.zeros(M, dtype=torch.int64, device=DEV)
+    else:
+        want = torch.zeros(M, N, dtype=torch.float16, device=DEV)
+        got = torch.zeros(M, N, dtype=torch.float16, device=DEV)
+    _with_caller_scratch(gs, x, w, M, N, K, epi, split, want)
+    gs.gs_linear_noalloc(x.data_ptr(), w.data_ptr(), got.data_ptr(), M, N, K, epi, split, stream)
+    assert gs.gs_linear_noalloc_status(stream) == gs.GS_OK
+    assert torch.equal(got, want)
 
 
 def test_noalloc_rejects_scratch_beyond_its_array(gs):
