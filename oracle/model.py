@@ -17,7 +17,14 @@ exactly as the paper words them.
 """
 from __future__ import annotations
 
+import os
+from concurrent.futures import ThreadPoolExecutor
+
 import numpy as np
+
+# Query rows per block of one head's score matrix (bounds the temporaries at
+# long prefixes; every row's softmax is still taken over all its keys).
+ROW_BLOCK = 2048
 
 from synth import ModelConfig, bf16_bits_to_f32
 
@@ -104,14 +111,28 @@ class Decoder:
         group = cfg.n_heads // cfg.n_kv_heads
         out = np.empty_like(q)
         scale = 1.0 / np.sqrt(cfg.head_dim)
-        for h in range(cfg.n_heads):
+
+        def one_head(h):
             kh = h // group
-            s = (q[:, h, :] @ k[:, kh, :].T) * scale                       # [rows, keys]
-            s = np.where(allowed, s, -np.inf)
-            s = s - np.max(s, axis=1, keepdims=True)
-            p = np.where(allowed, np.exp(s), 0.0)
-            p = p / np.sum(p, axis=1, keepdims=True)
-            out[:, h, :] = p @ v[:, kh, :]
+            for r0 in range(0, q.shape[0], ROW_BLOCK):
+                r1 = min(r0 + ROW_BLOCK, q.shape[0])
+                a = allowed[r0:r1]
+                s = (q[r0:r1, h, :] @ k[:, kh, :].T) * scale               # [rows, keys]
+                s = np.where(a, s, -np.inf)
+                s = s - np.max(s, axis=1, keepdims=True)
+                p = np.where(a, np.exp(s), 0.0)
+                p = p / np.sum(p, axis=1, keepdims=True)
+                out[r0:r1, h, :] = p @ v[:, kh, :]
+
+        # heads are independent; numpy releases the GIL inside these array
+        # operations, so long prefixes evaluate several heads at once
+        workers = min(cfg.n_heads, os.cpu_count() or 1, 8)
+        if workers <= 1 or q.shape[0] * k.shape[0] < (1 << 20):
+            for h in range(cfg.n_heads):
+                one_head(h)
+        else:
+            with ThreadPoolExecutor(max_workers=workers) as ex:
+                list(ex.map(one_head, range(cfg.n_heads)))
         return out
 
     # ------------------------------------------------------------ forward
