@@ -1,24 +1,33 @@
 """Benchmark: greedy self-speculative decoding on one GB300 per rank.
 
-Default workload ``glm_b1``: the GLM-OCR-scale synthetic decoder (24 layers,
-d_model 1024, 16 query / 8 KV heads, SwiGLU 4096, vocab 59392, random bf16
-weights), batch 1, prefix 2048 (1600 visual embeddings + 448 text tokens),
-block size K = 16, 512 output tokens, accepted draft lengths forced to a
-seeded censored-geometric schedule with mean 9.7.  ``--workload serve_b32``
-(32 sequences, prefixes U[1024, 6144]) and ``--workload long_b8`` (8 x prefix
-8192, K = 32, heavy-tailed acceptance) time the other configurations;
-``--K`` and ``--accept-mean`` override the block size and the forced mean
-(``--K 32 --accept-mean 17.4`` is the paper's TPF-9.7 operating point).
+Default workload ``serve_b32``: the GLM-OCR-scale synthetic decoder (24
+layers, d_model 1024, 16 query / 8 KV heads, SwiGLU 4096, vocab 59392, random
+bf16 weights) serving 32 documents at once, prefixes U[1024, 6144] (75 %
+visual embeddings, 64-token KV pages, ragged), block size K = 16, 512 output
+tokens per sequence, accepted draft lengths forced to a seeded
+censored-geometric schedule whose realized mean over the rounds run is 9.7
+(within 0.1).  The same line carries the batch-1 workload ``glm_b1`` (prefix
+2048 = 1600 visual + 448 text) as an extra key.  ``--workload glm_b1`` and
+``--workload long_b8`` (8 x prefix 8192, K = 32, heavy-tailed acceptance) time
+the other configurations as the headline; ``--K`` and ``--accept-mean``
+override the block size and the forced mean (``--K 32 --accept-mean 17.4`` is
+the paper's TPF-9.7 operating point).
 
 A step is one complete decode of every sequence: the sequence states are
 rolled back to the end of the prefill (the prefill itself is untimed, as in
 the paper's TPF accounting) and every round of the schedule runs as one CUDA
 graph (draft forward -> forcing -> verify forward -> accept/commit).  The
 metric is committed tokens per second over all sequences; per-round latencies
-come from CUDA events.  The 876.6 MB of weights every forward streams exceed
-the 129 MB L2, so no flush is needed between steps.  The same decode with
-K = 0 rounds (plain greedy AR, one token per forward) is timed on the same
-kernels for the speed-up the method buys.
+come from CUDA events.  The 876.6 MB of weights and the KV pages every forward
+streams exceed the 129 MB L2, so no flush is needed between steps.  The same
+decode with K = 0 rounds (plain greedy AR, one token per forward) is timed on
+the same kernels for the speed-up the method buys.
+
+After the timed regions (one GPU, rank 0): the float64 oracle runs a bounded
+sample of forced rounds of the workload's shortest sequence on the host cores
+(``cpu_baseline``), and the GPU runs the same rounds with the same teacher and
+schedule; ``parity`` reports the rows compared, the argmax flips at near-ties
+and the largest logit error.
 
 --impl reference times the float64 CPU oracle on this host's cores instead
 (forced rounds of the workload's shortest sequence).  Multi-GPU: replicas
@@ -48,11 +57,8 @@ UNIT = "tokens/s"
 
 
 def schedule_rounds(sched: np.ndarray, max_new: int) -> int:
-    n_out, r = 1, 0
-    while n_out < max_new:
-        n_out += int(sched[r]) + 2
-        r += 1
-    return r
+    """Rounds a forced schedule runs until max_new tokens are committed."""
+    return synth.rounds_used(sched, max_new)
 
 
 # DRAM traffic per launch (dram__bytes_read.sum + dram__bytes_write.sum) from
@@ -192,25 +198,46 @@ def gemm_flops(cfg, kind: str, T: int) -> int | None:
 
 
 def gpu_arm(args, rank: int, world: int):
+    """The GPU arm: the headline workload's timed decode, its end-to-end
+    figure, the per-kernel table and, on rank 0 of a one-GPU run, the oracle
+    sample (cpu_baseline) and the parity of the GPU rounds against it; with
+    the default serving workload also the batch-1 workload's figures."""
     import torch
-    from paper_2609_26638_gb300 import gs
-    from paper_2609_26638_gb300.runtime import Engine
 
     dev = torch.device("cuda", int(os.environ.get("LOCAL_RANK", 0)))
     torch.cuda.set_device(dev)
     wl = synth.WORKLOADS[args.workload]
-    cfg = wl.model
     K = wl.K if args.K is None else args.K
     mean = wl.accept_mean if args.accept_mean is None else args.accept_mean
+    weights = synth.make_weights(wl.model)
+    oracle_leg = rank == 0 and world == 1 and not args.no_cpu_baseline
+    res = run_decode(args, wl, K, mean, weights, dev, world, steps=args.steps, warmup=args.warmup,
+                     compare_ar=args.compare_ar, kernels=True, oracle_leg=oracle_leg)
+    if args.workload == "serve_b32" and args.K is None and args.accept_mean is None \
+            and args.extra_b1:
+        b1 = synth.WORKLOADS["glm_b1"]
+        r1 = run_decode(args, b1, b1.K, b1.accept_mean, weights, dev, world,
+                        steps=max(3, args.steps // 2), warmup=args.warmup, compare_ar=False,
+                        kernels=False, oracle_leg=False)
+        res["glm_b1"] = r1
+    return res
+
+
+def run_decode(args, wl, K, mean, weights, dev, world, *, steps, warmup, compare_ar, kernels,
+               oracle_leg):
+    import torch
+    from paper_2609_26638_gb300 import gs
+    from paper_2609_26638_gb300.runtime import Engine
+
+    cfg = wl.model
     max_new = wl.max_new
     prompts = wl.prompts()
     B = len(prompts)
     P = [p.length for p in prompts]
-    weights = synth.make_weights(cfg)
     extra = K + 4
-    eng = Engine(cfg, weights, max_batch=B, max_ctx=max(P) + max_new + extra + K + 2 + 64, max_K=K,
-                 max_prefill=2048, device=str(dev))
-    del weights
+    # (256 spare slots: the parity leg re-prefills a sequence with its history)
+    eng = Engine(cfg, weights, max_batch=B, max_ctx=max(P) + max_new + extra + K + 2 + 320,
+                 max_K=K, max_prefill=2048, device=str(dev))
     stream = eng.stream
     slots = torch.arange(B, dtype=torch.int32, device=dev)
     out_tok = torch.zeros((B, K + 2), dtype=torch.int32, device=dev)
@@ -237,11 +264,11 @@ def gpu_arm(args, rank: int, world: int):
     teacher = np.full((B, stride), -1, np.int32)
     for i in range(B):
         teacher[i, P[i]:P[i] + len(teacher_toks[i])] = teacher_toks[i]
-    kind = "geometric" if wl.accept in ("geometric", "natural") else wl.accept
-    sched_all = synth.accept_schedule(kind, K, B, wl.max_rounds(), mean)
+    sched_all = wl.schedule(K, mean)
     Rb = [schedule_rounds(sched_all[i], max_new) for i in range(B)]
     R = max(Rb)
     sched = np.ascontiguousarray(sched_all[:, :R + 1])
+    realized = synth.realized_mean(sched_all, max_new)
     t_dev = torch.from_numpy(teacher).to(dev)
     s_dev = torch.from_numpy(sched).to(dev)
     force = gs.gs_force(teacher=t_dev.data_ptr(), teacher_stride=stride, L_sched=s_dev.data_ptr(),
@@ -267,7 +294,7 @@ def gpu_arm(args, rank: int, world: int):
                     rt[r].copy_(out_tok, non_blocking=True)
                     rc[r].copy_(out_cnt, non_blocking=True)
 
-    for _ in range(args.warmup):
+    for _ in range(warmup):
         one_decode()
     stream.synchronize()
     launches_per_round = gs.gs_round_launches(eng.handle)
@@ -279,7 +306,7 @@ def gpu_arm(args, rank: int, world: int):
         torch.cuda.synchronize(dev)
 
     ev = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-           for _ in range(R)] for _ in range(args.steps)]
+           for _ in range(R)] for _ in range(steps)]
     t0 = torch.cuda.Event(enable_timing=True)
     t1 = torch.cuda.Event(enable_timing=True)
     # GS_PROFILE_RANGE=1 marks the first timed decode as the profiler's capture
@@ -288,7 +315,7 @@ def gpu_arm(args, rank: int, world: int):
     barrier()
     with ClockSampler(dev.index) as clk:
         t0.record(stream)
-        for s in range(args.steps):
+        for s in range(steps):
             if prof and s == 0:
                 torch.cuda.profiler.start()
             one_decode(ev[s])
@@ -322,7 +349,7 @@ def gpu_arm(args, rank: int, world: int):
     h_cnt = torch.empty((R, B), dtype=torch.int32).pin_memory()
     barrier()
     e0 = time.perf_counter()
-    for s in range(args.steps):
+    for s in range(steps):
         with torch.cuda.stream(stream):
             t_dev.copy_(h_teacher, non_blocking=True)
             s_dev.copy_(h_sched, non_blocking=True)
@@ -337,13 +364,13 @@ def gpu_arm(args, rank: int, world: int):
     # plain greedy AR on the same kernels (K = 0 rounds: two one-token forwards,
     # two tokens per round), for the speed-up the method buys on this GPU
     ar = None
-    if args.compare_ar:
+    if compare_ar:
         R_ar = (max_new + 1) // 2
         one_decode(Kr=0, frc=None, rounds=R_ar, rt=None)
         stream.synchronize()
         a0 = torch.cuda.Event(enable_timing=True)
         a1 = torch.cuda.Event(enable_timing=True)
-        n_ar = max(1, min(args.steps, 3))
+        n_ar = max(1, min(steps, 3))
         a0.record(stream)
         for _ in range(n_ar):
             one_decode(Kr=0, frc=None, rounds=R_ar, rt=None)
@@ -354,8 +381,30 @@ def gpu_arm(args, rank: int, world: int):
         ar = {"value": round(B * (max_new - 1) / ar_s, 1), "unit": UNIT,
               "ms_per_step": round(1e3 * ar_s, 3), "steps": n_ar, "rounds_per_step": R_ar}
 
-    # per-kernel device times: the forced decode once more, every round
-    # replayed as a graph with a CUDA event after each launch (gs_round_profile)
+    res = dict(elapsed=elapsed, e2e_elapsed=e_elapsed, tokens=committed_per_decode * steps,
+               steps=steps, round_ms=round_ms, rounds=R, launches_per_round=launches_per_round,
+               ok_sched=ok_sched, ok_tokens=ok_tokens, clocks=clk.summary(), ar=ar, B=B, K=K,
+               mean=mean, realized_mean=round(realized, 3),
+               h2d=int(teacher.nbytes + sched.nbytes),
+               d2h=int(R * B * (K + 2) * 4 + R * B * 4), max_new=max_new)
+    if kernels:
+        res.update(kernel_table(eng, cfg, slots, K, B, R, force, out_tok, out_cnt, out_done,
+                                restore_all))
+        res["lm_head"] = lm_head_roofline(cfg, K, dev) if B == 1 else None
+        res["attention"] = attention_roofline(cfg, dev)
+    if oracle_leg:
+        sample = oracle_sample(wl, 6, 1, 25.0, K, mean, weights)
+        res["cpu_sample"] = sample
+        res["parity"] = gpu_oracle_parity(eng, wl, sample, K)
+    eng.close()
+    return res
+
+
+def kernel_table(eng, cfg, slots, K, B, R, force, out_tok, out_cnt, out_done, restore_all):
+    """Per-kernel device times: the forced decode once more, every round
+    replayed as a graph with a CUDA event after each launch (gs_round_profile);
+    per kind the algorithmic bytes and flops per launch, and the roofline line
+    of the kind with the largest total time."""
     hbm, bf16_tf, src = load_peaks()
     W = K + 1
     T = B * W
@@ -414,16 +463,10 @@ def gpu_arm(args, rank: int, world: int):
                 "timing": timing, "traffic": traffic,
                 "traffic_source": "ncu dram bytes of the standalone kernel, scaled by algorithmic bytes"
                 if traffic is not None else None}
-    lm = lm_head_roofline(cfg, K, dev) if B == 1 else None
-    attn = attention_roofline(cfg, dev)
-    res = dict(elapsed=elapsed, e2e_elapsed=e_elapsed, tokens=committed_per_decode * args.steps,
-               round_ms=round_ms, rounds=R, launches_per_round=launches_per_round,
-               ok_sched=ok_sched, ok_tokens=ok_tokens, clocks=clk.summary(), roofline=roof,
-               kernels=kernels, lm_head=lm, attention=attn, ar=ar, B=B, K=K, mean=mean,
-               h2d=int(teacher.nbytes + sched.nbytes),
-               d2h=int(R * B * (K + 2) * 4 + R * B * 4), max_new=max_new)
-    eng.close()
-    return res
+    gemm = {n: {"frac_tensor": kernels[n].get("frac_tensor"), "tflop_s": kernels[n].get("tflop_s"),
+                "frac_hbm": kernels[n].get("frac_hbm"), "bound": kernels[n].get("bound")}
+            for n in ("qkv", "o_proj", "gate_up", "down", "lm_head") if n in kernels}
+    return {"roofline": roof, "kernels": kernels, "gemm_fracs": gemm}
 
 
 def job_totals(elapsed: float, e2e_elapsed: float, tokens: int, world: int, device):
@@ -601,14 +644,17 @@ def attention_roofline(cfg, dev, ns=None, K=16, mode=0):
 
 
 # ---------------------------------------------------------------------- oracle arm
-def oracle_sample(wl, n_rounds: int, warmup: int, budget_s: float, K: int, mean: float):
+def oracle_sample(wl, n_rounds: int, warmup: int, budget_s: float, K: int, mean: float,
+                  weights=None) -> dict:
     """Forced self-speculative rounds of the float64 oracle on this host's cores.
 
     The sample is the workload's shortest-prefix sequence (the oracle decodes
     one sequence at a time, so its tokens/s is the same for any batch): its
-    own greedy AR continuation is the forcing teacher, the timed rounds are the
-    first rounds of its forced decode (prefill and teacher untimed).  Returns
-    (per-round seconds, committed tokens per timed round, prefix length).
+    own greedy AR continuation is the forcing teacher, its forced L are the
+    workload's schedule for that sequence, and the timed rounds are the first
+    rounds of its forced decode (prefill and teacher untimed).  Returns the
+    per-round seconds and committed counts of the timed rounds, and every
+    round's result with the teacher, so the GPU can run the same rounds.
     """
     from oracle import decode as od
     from oracle.model import Decoder
@@ -616,25 +662,25 @@ def oracle_sample(wl, n_rounds: int, warmup: int, budget_s: float, K: int, mean:
     prompts = wl.prompts()
     idx = min(range(len(prompts)), key=lambda i: prompts[i].length)
     prompt = prompts[idx]
-    dec = Decoder(cfg, synth.make_weights(cfg))
-    kind = "geometric" if wl.accept in ("geometric", "natural") else wl.accept
-    sched = synth.accept_schedule(kind, K, len(prompts), wl.max_rounds(), mean)[idx]
+    dec = Decoder(cfg, weights if weights is not None else synth.make_weights(cfg))
+    sched = wl.schedule(K, mean)[idx]
     total = warmup + n_rounds
     need = int(sum(int(sched[r]) + 2 for r in range(total))) + K + 4
     cap = prompt.length + need + K + 8
     ar_state = od.prefill(dec, prompt.vis, prompt.text, cap, need)
     st = od.SeqState(cache=ar_state.cache.copy(), x0=ar_state.x0, out=[ar_state.x0],
-                     max_new=wl.max_new)
+                     max_new=wl.max_new, prefill_gap=ar_state.prefill_gap)
     od.ar_decode(dec, ar_state)
     P = prompt.length
-    teacher = np.full(P + len(ar_state.out) + 8, -1, np.int64)
+    teacher = np.full(P + len(ar_state.out) + 8, -1, np.int32)
     teacher[P:P + len(ar_state.out)] = ar_state.out
-    times, counts = [], []
+    times, counts, results = [], [], []
     t_start = time.perf_counter()
     for r in range(total):
         t0 = time.perf_counter()
         res = od.self_spec_round(dec, st, K, teacher, int(sched[r]))
         dt = time.perf_counter() - t0
+        results.append(res)
         if r >= warmup:
             times.append(dt)
             counts.append(len(res.committed))
@@ -642,7 +688,94 @@ def oracle_sample(wl, n_rounds: int, warmup: int, budget_s: float, K: int, mean:
                 break
         if st.done:
             break
-    return times, counts, P
+    return dict(times=times, counts=counts, P=P, idx=idx, results=results, teacher=teacher,
+                sched=np.asarray(sched[:len(results)], np.int32), x0=st.out[0],
+                prefill_gap=ar_state.prefill_gap, warmup=warmup)
+
+
+NEAR_TIE = 0.1      # nats: top-2 logit gap under which an argmax flip is allowed
+LOGIT_TOL = 3e-2    # max-abs logit error of the 16-bit GPU path against the float64 oracle
+
+
+def gpu_oracle_parity(eng, wl, sample, K) -> dict:
+    """The oracle sample's forced rounds run again on the GPU (untimed, after
+    the timed region): the sequence is prefilled into its own slot, the same
+    teacher and L schedule go through gs_force, and every round's draft and
+    verify argmax rows, logits and committed run are compared with the
+    oracle's.  An argmax may differ only where the oracle's top-2 gap is below
+    0.1 (counted; the GPU sequence then continues from the oracle's history)."""
+    import torch
+    from paper_2609_26638_gb300 import gs
+    dev = eng.device
+    prompt = wl.prompts()[sample["idx"]]
+    slot = sample["idx"]
+    W, V = K + 1, wl.model.vocab
+    max_new = wl.max_new
+    out = dict(rounds=0, rows=0, logit_rows=0, near_tie_flips=0, hard_mismatches=0,
+               max_logit_err=0.0, rounds_equal=0, accepted_equal=0,
+               sequence=f"prefix-{sample['P']} sequence of {wl.name}, the oracle sample's "
+                        f"{len(sample['results'])} forced rounds",
+               near_tie=NEAR_TIE, logit_tol=LOGIT_TOL)
+    x0 = eng.prefill(slot, prompt.vis, prompt.text, max_new)
+    if x0 != sample["x0"]:
+        out["near_tie_flips"] += 1
+        out["hard_mismatches"] += int(sample["prefill_gap"] >= NEAR_TIE)
+        eng.restore(slot, sample["P"], sample["x0"], 1, max_new)
+    t_dev = torch.from_numpy(sample["teacher"]).to(dev)
+    s_dev = torch.from_numpy(np.ascontiguousarray(sample["sched"])).to(dev)
+    force = gs.gs_force(teacher=t_dev.data_ptr(), teacher_stride=int(t_dev.shape[0]),
+                        L_sched=s_dev.data_ptr(), L_stride=int(s_dev.shape[0]))
+    slots = torch.tensor([slot], dtype=torch.int32, device=dev)
+    o_tok = torch.zeros((1, K + 2), dtype=torch.int32, device=dev)
+    o_cnt = torch.zeros(1, dtype=torch.int32, device=dev)
+    o_done = torch.zeros(1, dtype=torch.int32, device=dev)
+    b = [torch.zeros(W, dtype=torch.int32, device=dev) for _ in range(3)]
+    dl = torch.zeros((W, V), dtype=torch.float32, device=dev)
+    vl = torch.zeros((W, V), dtype=torch.float32, device=dev)
+    dbg = gs.gs_debug(draft_tok=b[0].data_ptr(), verify_in=b[1].data_ptr(),
+                      verify_tok=b[2].data_ptr(), draft_logits=dl.data_ptr(),
+                      verify_logits=vl.data_ptr())
+    history = [sample["x0"]]
+    n = sample["P"]
+    for r, res in enumerate(sample["results"]):
+        eng.round(slots, K, o_tok, o_cnt, o_done, force=force, dbg=dbg)
+        eng.stream.synchronize()
+        g_draft, g_vin, g_vt = (x.cpu().numpy() for x in b)
+        got = o_tok.cpu().numpy()[0, :int(o_cnt.cpu()[0])].tolist()
+        out["rounds"] += 1
+        want_draft = np.concatenate([[res.a0], res.d_draft])
+        for i in range(W):
+            out["rows"] += 1
+            if g_draft[i] != want_draft[i]:
+                out["near_tie_flips"] += 1
+                out["hard_mismatches"] += int(res.draft_gap[i] >= NEAR_TIE)
+        err = float(np.max(np.abs(dl.cpu().numpy().astype(np.float64) - res.draft_logits)))
+        out["max_logit_err"] = max(out["max_logit_err"], err)
+        out["logit_rows"] += W
+        if list(g_vin) == [res.a0] + list(res.d):
+            for i in range(W):
+                out["rows"] += 1
+                if g_vt[i] != res.a[i]:
+                    out["near_tie_flips"] += 1
+                    out["hard_mismatches"] += int(res.verify_gap[i] >= NEAR_TIE)
+            err = float(np.max(np.abs(vl.cpu().numpy().astype(np.float64) - res.verify_logits)))
+            out["max_logit_err"] = max(out["max_logit_err"], err)
+            out["logit_rows"] += W
+            A = 0
+            while A < K and g_vin[1 + A] == g_vt[A]:
+                A += 1
+            out["accepted_equal"] += int(A == res.A)
+        n += res.A + 2
+        history.extend(res.committed)
+        if got == res.committed:
+            out["rounds_equal"] += 1
+        else:        # continue from the oracle's history
+            text = np.concatenate([prompt.text, np.asarray(history[:-1], np.int32)])
+            eng.prefill(slot, prompt.vis, text, max_new)
+            eng.restore(slot, n, history[-1], len(history), max_new, 0, r + 1)
+    eng.check()
+    out["max_logit_err"] = round(out["max_logit_err"], 5)
+    return out
 
 
 def describe(wl, K: int, mean: float, world: int) -> dict:
@@ -653,16 +786,43 @@ def describe(wl, K: int, mean: float, world: int) -> dict:
     else:
         prefix = (f"prefixes U[{wl.prefix_min}, {wl.prefix_max}] ({round(100 * wl.vis_frac)}% visual, "
                   f"64-token pages, ragged)")
-    accept = {"geometric": f"censored geometric, mean accepted length {mean}",
-              "heavy": f"10% L=K, 10% L=0, else geometric; mean accepted length {mean}",
-              "natural": f"censored geometric, mean accepted length {mean}"}[wl.accept]
+    accept = {"geometric": f"censored geometric, mean accepted length {mean} realized over the "
+                           f"rounds run (within 0.1)",
+              "heavy": f"10% L=K, 10% L=0, else geometric; mean accepted length {mean} realized "
+                       f"over the rounds run (within 0.1)",
+              "natural": f"censored geometric, mean accepted length {mean} realized over the "
+                         f"rounds run (within 0.1)"}[wl.accept]
     return {"workload": f"{wl.name}: GLM-OCR-scale synthetic decoder L24 d1024 H16/8 F4096 V59392, "
                         f"batch {wl.batch}, {prefix}, K={K}, {wl.max_new} output tokens per "
                         f"sequence, forced acceptance ({accept})",
             "model": "synthetic random-init bf16 weights (seed 0)",
             "global_batch": wl.batch * max(world, 1), "K": K, "max_new": wl.max_new,
-            "l2": "inputs larger than L2: 876.6 MB of weights streamed per forward",
+            "l2": "inputs larger than L2: 876.6 MB of weights (plus the KV pages) streamed per "
+                  "forward, no flush needed",
             "parallelism": f"replicas x{max(world, 1)}"}
+
+
+def decode_line(res, world: int) -> dict:
+    """The figures of one timed decode (whole job over the ranks)."""
+    el, ee, tokens_all = job_totals(res["elapsed"], res["e2e_elapsed"], res["tokens"], world, "cuda")
+    value = tokens_all / el
+    rms = res["round_ms"]
+    B, steps, R = res["B"], res["steps"], res["rounds"]
+    d = {"value": round(value, 1), "ms_per_step": round(1e3 * el / steps, 3),
+         "round_p50_ms": round(rms[len(rms) // 2], 4),
+         "round_p90_ms": round(rms[int(len(rms) * 0.9)], 4),
+         "rounds_per_step": R,
+         "accept_mean_realized": res["realized_mean"],
+         "committed_per_round_per_seq": round(res["tokens"] / (steps * R * B), 3),
+         "tpf": round(res["tokens"] / (steps * R * 2 * B), 3),
+         "forced_schedule_hit": res["ok_sched"], "tokens_match_greedy": res["ok_tokens"],
+         "gpu_launches": res["launches_per_round"] * R * steps + steps * B,
+         "e2e": {"value": round(tokens_all / ee, 1), "unit": UNIT,
+                 "h2d_bytes_per_step": res["h2d"], "d2h_bytes_per_step": res["d2h"]}}
+    if res["ar"] is not None:
+        d["greedy_ar"] = res["ar"]
+        d["speedup_vs_greedy_ar"] = round(value / (res["ar"]["value"] * max(world, 1)), 3)
+    return d
 
 
 def main():
@@ -671,12 +831,14 @@ def main():
     ap.add_argument("--steps", type=int, default=10)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="gpu", choices=["gpu", "reference"])
-    ap.add_argument("--workload", default="glm_b1", choices=sorted(synth.WORKLOADS))
+    ap.add_argument("--workload", default="serve_b32", choices=sorted(synth.WORKLOADS))
     ap.add_argument("--K", type=int, default=None, help="block size (default: the workload's)")
     ap.add_argument("--accept-mean", type=float, default=None,
                     help="mean forced accepted length (default: the workload's)")
     ap.add_argument("--no-compare-ar", dest="compare_ar", action="store_false",
                     help="skip timing plain greedy AR (K = 0 rounds) on the same workload")
+    ap.add_argument("--no-extra-b1", dest="extra_b1", action="store_false",
+                    help="with the serving workload, skip the batch-1 workload's extra figures")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--kernel", default=None,
                     choices=["attention", "lm_head", "attention-sweep", "gemm-serve"],
@@ -727,11 +889,12 @@ def main():
         if rank != 0:
             return
         t0 = time.perf_counter()
-        times, counts, P0 = oracle_sample(wl, args.steps, args.warmup, 240.0, K, mean)
+        smp = oracle_sample(wl, args.steps, args.warmup, 240.0, K, mean)
+        times, counts = smp["times"], smp["counts"]
         value = sum(counts) / sum(times)
         cores = os.cpu_count()
         sample = (f"{len(times)} forced rounds (after {args.warmup} warm-up rounds) of the "
-                  f"prefix-{P0} sequence of {wl.name}, float64 oracle on all host cores "
+                  f"prefix-{smp['P']} sequence of {wl.name}, float64 oracle on all host cores "
                   f"(numpy/OpenBLAS), prefill and teacher untimed")
         line = {"impl": "reference", "metric": METRIC, "value": round(value, 3), "unit": UNIT,
                 "n_gpus": args.gpus, "steps": len(times), "warmup": args.warmup,
@@ -751,40 +914,34 @@ def main():
         import torch.distributed as dist
         dist.init_process_group("nccl", device_id=torch.device("cuda", int(os.environ["LOCAL_RANK"])))
     res = gpu_arm(args, rank, world)
-    el, ee, tokens_all = job_totals(res["elapsed"], res["e2e_elapsed"], res["tokens"], world, "cuda")
-    value = tokens_all / el
-    rms = res["round_ms"]
-    B = res["B"]
-    line = {"metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": max(world, 1),
+    head = decode_line(res, world)
+    line = {"metric": METRIC, "value": head.pop("value"), "unit": UNIT, "n_gpus": max(world, 1),
             "steps": args.steps, "warmup": args.warmup,
-            "ms_per_step": round(1e3 * el / args.steps, 3), "higher_is_better": True,
+            "ms_per_step": head.pop("ms_per_step"), "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f16", "data": "synthetic",
-            "config": config,
-            "round_p50_ms": round(rms[len(rms) // 2], 4),
-            "round_p90_ms": round(rms[int(len(rms) * 0.9)], 4),
-            "rounds_per_step": res["rounds"],
-            "committed_per_round_per_seq": round(res["tokens"] / (args.steps * res["rounds"] * B), 3),
-            "tpf": round(res["tokens"] / (args.steps * res["rounds"] * 2 * B), 3),
-            "forced_schedule_hit": res["ok_sched"], "tokens_match_greedy": res["ok_tokens"],
-            "gpu_launches": res["launches_per_round"] * res["rounds"] * args.steps
-            + args.steps * B,
-            "e2e": {"value": round(tokens_all / ee, 1), "unit": UNIT,
-                    "h2d_bytes_per_step": res["h2d"], "d2h_bytes_per_step": res["d2h"]},
-            "clocks": res["clocks"], "roofline": res["roofline"], "kernels": res["kernels"],
-            "attention_roofline": res["attention"]}
-    if res["lm_head"] is not None:
+            "config": config}
+    line.update(head)
+    line.update({"clocks": res["clocks"], "roofline": res["roofline"],
+                 "gemm_fracs": res["gemm_fracs"], "kernels": res["kernels"],
+                 "attention_roofline": res["attention"]})
+    if res.get("lm_head") is not None:
         line["lm_head_alone"] = res["lm_head"]
-    if res["ar"] is not None:
-        line["greedy_ar"] = res["ar"]
-        line["speedup_vs_greedy_ar"] = round(value / (res["ar"]["value"] * max(world, 1)), 3)
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        times, counts, P0 = oracle_sample(wl, 6, 1, 25.0, K, mean)
+    if "glm_b1" in res:
+        b1 = synth.WORKLOADS["glm_b1"]
+        extra = decode_line(res["glm_b1"], world)
+        extra["config"] = describe(b1, b1.K, b1.accept_mean, world)["workload"]
+        extra["steps"] = res["glm_b1"]["steps"]
+        line["glm_b1"] = extra
+    if "parity" in res:
+        line["parity"] = res["parity"]
+    if "cpu_sample" in res:
+        smp = res["cpu_sample"]
         line["cpu_baseline"] = {
-            "value": round(sum(counts) / sum(times), 3), "unit": UNIT, "cores": os.cpu_count(),
-            "kind": "oracle",
-            "sample": f"{len(times)} forced rounds (after 1 warm-up) of the prefix-{P0} sequence "
-                      f"of the same workload, float64 oracle with numpy/OpenBLAS threads on all "
-                      f"host cores"}
+            "value": round(sum(smp["counts"]) / sum(smp["times"]), 3), "unit": UNIT,
+            "cores": os.cpu_count(), "kind": "oracle",
+            "sample": f"{len(smp['times'])} forced rounds (after {smp['warmup']} warm-up) of the "
+                      f"prefix-{smp['P']} sequence of the same workload, float64 oracle with "
+                      f"numpy/OpenBLAS threads on all host cores"}
     if rank == 0:
         print(json.dumps(line))
     if world > 1:

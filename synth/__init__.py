@@ -182,16 +182,50 @@ def solve_alpha(mean: float, K: int) -> float:
     return 0.5 * (lo + hi)
 
 
+def rounds_used(sched_row: np.ndarray, max_new: int) -> int:
+    """Rounds one sequence runs under a forced schedule: every round commits
+    L + 2 tokens and the prefill's boundary token is the first output, so
+    rounds run until max_new tokens are out (the last one may be cut)."""
+    n_out, r = 1, 0
+    while n_out < max_new:
+        n_out += int(sched_row[r]) + 2
+        r += 1
+    return r
+
+
+def realized_mean(sched: np.ndarray, max_new: int) -> float:
+    """Mean forced L over the rounds the sequences actually run."""
+    used = [sched[i, :rounds_used(sched[i], max_new)] for i in range(sched.shape[0])]
+    return float(np.concatenate(used).mean())
+
+
 def accept_schedule(kind: str, K: int, n_seq: int, n_rounds: int, mean: float = 9.7,
-                    seed: int = ACCEPT_SEED) -> np.ndarray:
+                    seed: int = ACCEPT_SEED, max_new: Optional[int] = None,
+                    tol: float = 0.1) -> np.ndarray:
     """Forced accepted-draft lengths L[seq, round], int32 in [0, K].
 
     kind "geometric": L = min(G, K), P(G >= j) = alpha**j, alpha solved for ``mean``.
     kind "heavy":     10% L = K, 10% L = 0, 80% censored geometric whose mean makes
                       the mixture mean ``mean``.
     kind "full"/"zero": always K / always 0.
+
+    With ``max_new``, the draw is conditioned on the rounds a decode of
+    max_new tokens actually runs: draws (numbered 0, 1, ... in the seed key)
+    are taken until the mean L over those rounds lies within ``tol`` of
+    ``mean``, so a short decode realizes the stated mean.
     """
-    rng = _rng(seed, 200, K)
+    if max_new is None or kind in ("full", "zero"):
+        return _draw_schedule(kind, K, n_seq, n_rounds, mean, seed, 0)
+    for attempt in range(10000):
+        s = _draw_schedule(kind, K, n_seq, n_rounds, mean, seed, attempt)
+        if abs(realized_mean(s, max_new) - mean) <= tol:
+            return s
+    raise RuntimeError("no schedule draw realizes the mean within tol")
+
+
+def _draw_schedule(kind: str, K: int, n_seq: int, n_rounds: int, mean: float, seed: int,
+                   attempt: int) -> np.ndarray:
+    rng = _rng(seed, 200, K) if attempt == 0 else _rng(seed, 200, K, attempt)
     shape = (n_seq, n_rounds)
     if kind == "full":
         return np.full(shape, K, np.int32)
@@ -247,10 +281,17 @@ class Workload:
         # every round commits at least 2 tokens; the prefill commits 1
         return self.max_new // 2 + 1
 
-    def schedule(self) -> Optional[np.ndarray]:
+    def schedule(self, K: Optional[int] = None, mean: Optional[float] = None
+                 ) -> Optional[np.ndarray]:
+        """Forced L per (sequence, round), drawn so that the rounds a decode of
+        max_new tokens runs realize the mean within 0.1 (``accept_schedule``).
+        ``K`` and ``mean`` override the workload's block size and mean."""
         if self.accept == "natural":
             return None
-        return accept_schedule(self.accept, self.K, self.batch, self.max_rounds(), self.accept_mean)
+        K = self.K if K is None else K
+        mean = self.accept_mean if mean is None else mean
+        return accept_schedule(self.accept, K, self.batch, self.max_new // 2 + 1, mean,
+                               max_new=self.max_new)
 
 
 WORKLOADS: Dict[str, Workload] = {
