@@ -19,4 +19,5 @@ from .model import Decoder, KVCache  # noqa: F401
 from .decode import (  # noqa: F401
     SeqState, RoundResult, prefill, draft_forward, verify_forward, accept_length,
     self_spec_round, ar_decode, self_spec_decode, forced_drafts, tokens_per_forward,
+    reveal_positions, denoise_forward, cache_write_forward, diffusion_block, diffusion_decode,
 )

@@ -236,6 +236,125 @@ def ar_decode(dec: Decoder, st: SeqState) -> List[int]:
     return st.out
 
 
+# ------------------------------------------------------------------ direct block diffusion
+def softmax_rows(logits: np.ndarray) -> np.ndarray:
+    """Row-wise softmax in float64."""
+    z = logits - np.max(logits, axis=1, keepdims=True)
+    e = np.exp(z)
+    return e / np.sum(e, axis=1, keepdims=True)
+
+
+def reveal_positions(conf: np.ndarray, masked: List[int], tau: float) -> List[int]:
+    """The confidence rule of direct block-diffusion decoding (Appendix "Direct
+    Block-Diffusion Decoding"): every still-masked position whose predicted
+    token's probability exceeds tau is revealed; if none does, the single most
+    confident masked position is (ties to the lowest position)."""
+    above = [j for j in masked if conf[j] > tau]
+    if above:
+        return above
+    best = masked[0]
+    for j in masked[1:]:
+        if conf[j] > conf[best]:
+            best = j
+    return [best]
+
+
+def denoise_forward(dec: Decoder, cache: KVCache, x0: int, block: List[Optional[int]]
+                    ) -> np.ndarray:
+    """One denoising forward over [x0, block] at slots n..n+B.
+
+    ``block[j-1]`` is the token at block position j (slot n+j), or None while
+    it is still masked (fed as [M]).  The boundary row (slot n) attends
+    causally to the cache (keys 0..n); every block row attends to the cache
+    and to the whole window (keys 0..n+B), the same hybrid mask as the
+    self-speculative draft.  Under the shifted alignment, the row at slot
+    n+j-1 predicts block position j.  Returns logits [B+1, V]; rows 0..B-1
+    are the predictions for positions 1..B.
+    """
+    n = cache.seq_len
+    B = len(block)
+    mask_id = dec.cfg.mask_token_id
+    ids = np.array([x0] + [mask_id if t is None else int(t) for t in block])
+    slots = n + np.arange(B + 1)
+    return dec.forward(dec.embed_tokens(ids), slots, draft_allowed(n, B), cache)
+
+
+def cache_write_forward(dec: Decoder, cache: KVCache, x0: int, block: List[int]) -> None:
+    """The pass that extends the cache once a block is complete: a causal
+    forward over [x0, y_1..y_{B-1}] at slots n..n+B-1 (row i sees keys
+    0..n+i).  It only writes causal KV states; no token is read from it.
+    The block's last token y_B becomes the next boundary, whose state the
+    next block's first denoising forward writes."""
+    n = cache.seq_len
+    B = len(block)
+    ids = np.array([x0] + [int(t) for t in block[:-1]])
+    slots = n + np.arange(B)
+    allowed = np.arange(n + B)[None, :] <= slots[:, None]
+    dec.forward(dec.embed_tokens(ids), slots, allowed, cache)
+    cache.truncate(n + B)
+
+
+@dataclasses.dataclass
+class BlockResult:
+    block: List[int]            # y_1..y_B as revealed
+    committed: List[int]        # tokens this block commits (after stop truncation)
+    steps: int                  # denoising forwards (the cache write not counted)
+    revealed_per_step: List[List[int]]   # block positions (1-based) revealed per step
+    conf_per_step: List[np.ndarray]      # confidence of every position's prediction per step
+    tok_per_step: List[np.ndarray]       # argmax prediction of every position per step
+
+
+def diffusion_block(dec: Decoder, st: SeqState, B: int, tau_c: float) -> BlockResult:
+    """Decode one block of B tokens by direct block diffusion and commit it.
+
+    State as in self-speculative decoding: the cache holds the causal states
+    of every committed token except the boundary x0 (slot n).  The block is
+    initialised with B masks at slots n+1..n+B.  Each denoising step runs
+    one forward and reveals positions by ``reveal_positions``; revealed
+    tokens stay fixed.  Once complete, one cache-write forward extends the
+    cache (slots n..n+B-1) and y_B becomes the boundary.  The committed run is
+    cut at the first stop token or at the output cap, which ends generation.
+    """
+    assert not st.done
+    cache = st.cache
+    block: List[Optional[int]] = [None] * B
+    revealed, confs, toks = [], [], []
+    while any(t is None for t in block):
+        logits = denoise_forward(dec, cache, st.x0, block)
+        probs = softmax_rows(logits[:B])
+        conf = np.max(probs, axis=1)
+        tok = argmax_rows(logits[:B])
+        masked = [j for j in range(B) if block[j] is None]
+        pick = reveal_positions(conf, masked, tau_c)
+        for j in pick:
+            block[j] = int(tok[j])
+        revealed.append([j + 1 for j in pick])
+        confs.append(conf)
+        toks.append(tok)
+    full = [int(t) for t in block]
+    committed = []
+    for t in full:
+        committed.append(t)
+        if t == st.eos or len(st.out) + len(committed) >= st.max_new:
+            st.done = True
+            break
+    st.out.extend(committed)
+    if not st.done:
+        cache_write_forward(dec, cache, st.x0, full)
+        st.x0 = full[-1]
+    return BlockResult(block=full, committed=committed, steps=len(revealed),
+                       revealed_per_step=revealed, conf_per_step=confs, tok_per_step=toks)
+
+
+def diffusion_decode(dec: Decoder, st: SeqState, B: int, tau_c: float,
+                     max_blocks: int = 1 << 30) -> List[BlockResult]:
+    """Direct block-diffusion decoding from a prefill state until a stop."""
+    out = []
+    while not st.done and len(out) < max_blocks:
+        out.append(diffusion_block(dec, st, B, tau_c))
+    return out
+
+
 def tokens_per_forward(committed_per_round: List[int]) -> float:
     """TPF (Sec. 5 "Efficiency Measurement"): committed tokens / forwards, counting
     the draft and the verify forward of every round separately, prefill excluded."""

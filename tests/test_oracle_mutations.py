@@ -92,6 +92,27 @@ def _truncate_one_short(self, n):
     self.seq_len = n
 
 
+def _reveal_at_threshold_too(conf, masked, tau):
+    above = [j for j in masked if conf[j] >= tau]                 # slip: >= instead of >
+    return above if above else [max(masked, key=lambda j: (conf[j], -j))]
+
+
+def _reveal_only_the_best(conf, masked, tau):
+    return [max(masked, key=lambda j: (conf[j], -j))]            # slip: ignores the threshold
+
+
+def _denoise_unshifted(dec, cache, x0, block):
+    n = cache.seq_len
+    B = len(block)
+    ids = np.array([x0] + [dec.cfg.mask_token_id if t is None else int(t) for t in block])
+    logits = dec.forward(dec.embed_tokens(ids), n + np.arange(B + 1), od.draft_allowed(n, B), cache)
+    return np.concatenate([logits[1:], logits[:1]])               # slip: position j read from row j
+
+
+def _cache_write_skipped(dec, cache, x0, block):
+    cache.truncate(cache.seq_len + len(block))                   # slip: no causal rewrite
+
+
 MUTATIONS = [
     ("draft boundary row sees the mask block", od, "draft_forward", _draft_boundary_sees_masks,
      "test_boundary_row_is_the_ar_logit"),
@@ -105,6 +126,14 @@ MUTATIONS = [
     ("softmax scale dropped", Decoder, "attention", _attention_no_scale, "test_causal_forward_matches_torch"),
     ("RMSNorm gain dropped", Decoder, "rmsnorm", _rmsnorm_no_gain, "test_causal_forward_matches_torch"),
     ("cache truncation one short", KVCache, "truncate", _truncate_one_short, "test_self_spec_equals_greedy_ar"),
+    ("reveal at the threshold itself", od, "reveal_positions", _reveal_at_threshold_too,
+     "test_reveal_rule_cases"),
+    ("reveal ignores the threshold", od, "reveal_positions", _reveal_only_the_best,
+     "test_diffusion_first_token_is_ar_and_cache_is_ar"),
+    ("block prediction not shifted", od, "denoise_forward", _denoise_unshifted,
+     "test_diffusion_first_token_is_ar_and_cache_is_ar"),
+    ("block cache write skipped", od, "cache_write_forward", _cache_write_skipped,
+     "test_diffusion_first_token_is_ar_and_cache_is_ar"),
 ]
 
 
@@ -119,6 +148,8 @@ def test_pin_catches_planted_mistake(monkeypatch, name, owner, attr, patched, pi
         caught = _fails(fn, (dec, w), monkeypatch)
     elif pin == "test_self_spec_equals_greedy_ar":
         caught = _fails(fn, (dec, w), 3)
+    elif pin == "test_reveal_rule_cases":
+        caught = _fails(fn)
     else:
         caught = _fails(fn, (dec, w))
     assert caught, f"planted mistake not caught: {name}"

@@ -12,7 +12,13 @@
   "Draft forward"), verify rows equal to incremental AR logits, commit bounds
   2..K+2, KV-cache contents equal to AR's and no surviving draft state
   (Appendix step "Cache update");
-* TPF accounting against the paper's printed tables (tests/golden).
+* TPF accounting against the paper's printed tables (tests/golden);
+* direct block-diffusion decoding (Appendix "Direct Block-Diffusion
+  Decoding"): block size 1 is greedy AR; a threshold above every probability
+  reveals one position per step, the most confident; a threshold below every
+  probability reveals the block in one step, equal to the one-shot draft; a
+  block's first token is the AR prediction; after every block the cache equals
+  AR's cache with no bidirectional state left; output cut at the first EOS.
 """
 import math
 import os
@@ -337,3 +343,106 @@ def test_tpf_accounting_matches_paper_tables(src, accepted, tpf):
     n_rounds = 1000
     got = oracle.tokens_per_forward([accepted + 2] * n_rounds)
     assert abs(got - tpf) <= 0.05 + 1e-9, (src, got, tpf)
+
+
+# ------------------------------------------------------------------ direct block diffusion
+def test_reveal_rule_cases():
+    """Every masked position above the threshold is revealed (strictly above);
+    if none is, the single most confident one, ties to the lowest position."""
+    conf = np.array([0.2, 0.9, 0.5, 0.95, 0.5])
+    assert od.reveal_positions(conf, [0, 1, 2, 3, 4], 0.8) == [1, 3]
+    assert od.reveal_positions(conf, [0, 2, 4], 0.8) == [2]          # none above: the max, lowest
+    assert od.reveal_positions(conf, [0, 2, 4], 0.5) == [2]          # 0.5 is not above 0.5
+    assert od.reveal_positions(conf, [4], 2.0) == [4]
+    assert od.reveal_positions(conf, [0, 1, 2, 3, 4], -1.0) == [0, 1, 2, 3, 4]
+
+
+@pytest.mark.parametrize("tau", [-1.0, 0.5, 2.0])
+def test_diffusion_block_size_one_is_greedy_ar(micro, tau):
+    """B = 1: the only prediction comes from the causal boundary row, so direct
+    block diffusion emits the greedy AR sequence for any threshold."""
+    dec, _ = micro
+    ar = od.ar_decode(dec, _prefill(dec, max_new=24))
+    st = _prefill(dec, max_new=24)
+    blocks = od.diffusion_decode(dec, st, 1, tau)
+    assert st.out == ar
+    assert all(b.steps == 1 for b in blocks)
+
+
+def test_diffusion_threshold_above_one_reveals_the_most_confident(micro):
+    """No probability exceeds 1.5: each step reveals exactly one position, the
+    masked one whose prediction is the most confident (brute force over the
+    recorded confidences), so a block takes B steps."""
+    dec, _ = micro
+    B = 5
+    st = _prefill(dec, max_new=1 + 3 * B)
+    blocks = od.diffusion_decode(dec, st, B, 1.5)
+    assert len(blocks) == 3
+    for b in blocks:
+        assert b.steps == B
+        masked = set(range(1, B + 1))
+        for rev, conf in zip(b.revealed_per_step, b.conf_per_step):
+            assert len(rev) == 1
+            best = max(sorted(masked), key=lambda j: (conf[j - 1], -j))
+            assert rev == [best]
+            masked.remove(best)
+
+
+def test_diffusion_threshold_below_zero_is_the_one_shot_draft(micro):
+    """Every probability exceeds -1: the block is revealed in one step, and it is
+    the self-speculative one-shot draft [a0, d_1..d_{B-1}] of a window of B masks."""
+    dec, _ = micro
+    B = 6
+    st = _prefill(dec, max_new=40)
+    c = st.cache.copy()
+    tok = od.argmax_rows(od.draft_forward(dec, c, st.x0, B))
+    b = od.diffusion_block(dec, st, B, -1.0)
+    assert b.steps == 1 and b.block == [int(t) for t in tok[:B]]
+
+
+def test_diffusion_first_token_is_ar_and_cache_is_ar(micro):
+    """The first position of every block is predicted by the causal boundary
+    row, so it is the AR prediction after the committed prefix; after every
+    block the cache holds exactly AR's causal states of the committed tokens
+    (all but the boundary) and nothing beyond them."""
+    dec, _ = micro
+    B, max_new = 4, 30
+    st = _prefill(dec, max_new=max_new)
+    conf0 = np.max(od.softmax_rows(od.denoise_forward(dec, st.cache.copy(), st.x0, [None] * B)[:B]),
+                   axis=1)
+    tau = float(np.median(conf0))       # about half the first step's predictions above
+    multi = 0
+    while not st.done:
+        c = st.cache.copy()
+        ar_next = int(od.argmax_rows(od.ar_step_forward(dec, c, st.x0))[0])
+        b = od.diffusion_block(dec, st, B, tau)
+        assert b.block[0] == ar_next
+        multi += any(len(r) > 1 for r in b.revealed_per_step)
+        if st.done:
+            break
+        # AR's cache: the prefix, then one causal step per committed token
+        # except the boundary (the last one)
+        ref_cache = _prefill(dec, max_new=max_new).cache
+        for t in st.out[:-1]:
+            od.ar_step_forward(dec, ref_cache, t)
+        assert st.n == ref_cache.seq_len
+        for layer in range(MICRO.n_layers):
+            np.testing.assert_allclose(st.cache.k[layer][:st.n], ref_cache.k[layer][:st.n],
+                                       atol=1e-10)
+            np.testing.assert_allclose(st.cache.v[layer][:st.n], ref_cache.v[layer][:st.n],
+                                       atol=1e-10)
+            assert np.isnan(st.cache.k[layer][st.n:]).all()
+    assert multi >= 1          # the threshold revealed several positions in one step somewhere
+
+
+def test_diffusion_stop_token_truncates(micro):
+    dec, _ = micro
+    B = 4
+    st = _prefill(dec, max_new=40)
+    od.diffusion_decode(dec, st, B, 0.0)
+    free = st.out
+    eos = free[9]
+    cut = free.index(eos) + 1
+    st = _prefill(dec, max_new=40, eos=eos)
+    od.diffusion_decode(dec, st, B, 0.0)
+    assert st.done and st.out == free[:cut]
