@@ -20,4 +20,5 @@ from .decode import (  # noqa: F401
     SeqState, RoundResult, prefill, draft_forward, verify_forward, accept_length,
     self_spec_round, ar_decode, self_spec_decode, forced_drafts, tokens_per_forward,
     reveal_positions, denoise_forward, cache_write_forward, diffusion_block, diffusion_decode,
+    refine_draft, self_spec_round_refined, reveal_margin,
 )

@@ -28,6 +28,7 @@ absolute RoPE positions of mask slots, output cap counting the prefill's x0).
 from __future__ import annotations
 
 import dataclasses
+import math
 from typing import List, Optional
 
 import numpy as np
@@ -193,7 +194,15 @@ def self_spec_round(dec: Decoder, st: SeqState, K: int, teacher: Optional[np.nda
     n = cache.seq_len
     dl = draft_forward(dec, cache, st.x0, K)
     tok = argmax_rows(dl)
-    a0, d_draft = int(tok[0]), tok[1:].copy()
+    return _verify_accept_commit(dec, st, n, K, int(tok[0]), tok[1:].copy(), dl, teacher, L)
+
+
+def _verify_accept_commit(dec: Decoder, st: SeqState, n: int, K: int, a0: int,
+                          d_draft: np.ndarray, dl: np.ndarray, teacher: Optional[np.ndarray],
+                          L: Optional[int]) -> RoundResult:
+    """Verify forward, acceptance, commit and cache update of a round whose
+    draft (a0, d_1..d_K) is given (Appendix steps Verify forward .. Next round)."""
+    cache = st.cache
     d = d_draft if teacher is None else forced_drafts(d_draft, teacher, n, L, dec.cfg.vocab)
     vl = verify_forward(dec, cache, a0, d)
     a = argmax_rows(vl)                                    # a_1..a_{K+1}
@@ -213,6 +222,57 @@ def self_spec_round(dec: Decoder, st: SeqState, K: int, teacher: Optional[np.nda
     return RoundResult(a0=a0, d_draft=d_draft, d=d, a=a, A=A, committed=committed,
                        draft_logits=dl, verify_logits=vl,
                        draft_gap=top2_gap(dl), verify_gap=top2_gap(vl))
+
+
+@dataclasses.dataclass
+class RefinedDraft:
+    steps: int                           # draft forwards
+    fixed_per_step: List[List[int]]      # prediction indices (0 = a0, j = d_j) fixed per step
+    conf_per_step: List[np.ndarray]      # confidence of every prediction per step
+    gap_per_step: List[np.ndarray]       # top-2 logit gap of every prediction row per step
+    tok_per_step: List[np.ndarray]       # argmax of every prediction row per step
+
+
+def refine_draft(dec: Decoder, cache: KVCache, x0: int, K: int, tau_d: float):
+    """Multi-step drafting (Sec. 6 "Draft Schedule", Fig. "Multi-step drafting
+    versus one-shot drafting"): the draft window [x0, [M] x K] is re-run, and
+    at each step the predictions whose confidence exceeds tau_d are fixed; the
+    rest are re-drafted.  Prediction i (a0 for i = 0, d_i otherwise) is read
+    from row i; a fixed prediction i < K is fed back as the input at its own
+    slot n+1+i in place of the mask there (prediction K has no slot in the
+    window).  If no open prediction exceeds tau_d, the single most confident
+    one is fixed, as in direct block diffusion, so the draft completes in at
+    most K+1 forwards.  Returns (a0, d_1..d_K, the last step's logits, record).
+    """
+    fixed: List[Optional[int]] = [None] * (K + 1)
+    rec = RefinedDraft(steps=0, fixed_per_step=[], conf_per_step=[], gap_per_step=[],
+                       tok_per_step=[])
+    logits = None
+    while any(t is None for t in fixed):
+        logits = denoise_forward(dec, cache, x0, fixed[:K])
+        conf = np.max(softmax_rows(logits), axis=1)
+        tok = argmax_rows(logits)
+        masked = [i for i in range(K + 1) if fixed[i] is None]
+        pick = reveal_positions(conf, masked, tau_d)
+        for i in pick:
+            fixed[i] = int(tok[i])
+        rec.steps += 1
+        rec.fixed_per_step.append(pick)
+        rec.conf_per_step.append(conf)
+        rec.gap_per_step.append(top2_gap(logits))
+        rec.tok_per_step.append(tok)
+    return fixed[0], np.array(fixed[1:], dtype=np.int64), logits, rec
+
+
+def self_spec_round_refined(dec: Decoder, st: SeqState, K: int, tau_d: float,
+                            teacher: Optional[np.ndarray] = None, L: Optional[int] = None):
+    """A self-speculative round whose draft is refined over several denoising
+    steps (``refine_draft``), then verified exactly as a one-shot draft.
+    Returns (RoundResult, RefinedDraft)."""
+    assert not st.done
+    n = st.cache.seq_len
+    a0, d_draft, dl, rec = refine_draft(dec, st.cache, st.x0, K, tau_d)
+    return _verify_accept_commit(dec, st, n, K, a0, d_draft, dl, teacher, L), rec
 
 
 def self_spec_decode(dec: Decoder, st: SeqState, K: int, teacher: Optional[np.ndarray] = None,
@@ -302,6 +362,7 @@ class BlockResult:
     revealed_per_step: List[List[int]]   # block positions (1-based) revealed per step
     conf_per_step: List[np.ndarray]      # confidence of every position's prediction per step
     tok_per_step: List[np.ndarray]       # argmax prediction of every position per step
+    gap_per_step: List[np.ndarray]       # top-2 logit gap of every position's row per step
 
 
 def diffusion_block(dec: Decoder, st: SeqState, B: int, tau_c: float) -> BlockResult:
@@ -318,12 +379,13 @@ def diffusion_block(dec: Decoder, st: SeqState, B: int, tau_c: float) -> BlockRe
     assert not st.done
     cache = st.cache
     block: List[Optional[int]] = [None] * B
-    revealed, confs, toks = [], [], []
+    revealed, confs, toks, gaps = [], [], [], []
     while any(t is None for t in block):
         logits = denoise_forward(dec, cache, st.x0, block)
         probs = softmax_rows(logits[:B])
         conf = np.max(probs, axis=1)
         tok = argmax_rows(logits[:B])
+        gaps.append(top2_gap(logits[:B]))
         masked = [j for j in range(B) if block[j] is None]
         pick = reveal_positions(conf, masked, tau_c)
         for j in pick:
@@ -343,7 +405,8 @@ def diffusion_block(dec: Decoder, st: SeqState, B: int, tau_c: float) -> BlockRe
         cache_write_forward(dec, cache, st.x0, full)
         st.x0 = full[-1]
     return BlockResult(block=full, committed=committed, steps=len(revealed),
-                       revealed_per_step=revealed, conf_per_step=confs, tok_per_step=toks)
+                       revealed_per_step=revealed, conf_per_step=confs, tok_per_step=toks,
+                       gap_per_step=gaps)
 
 
 def diffusion_decode(dec: Decoder, st: SeqState, B: int, tau_c: float,
@@ -353,6 +416,26 @@ def diffusion_decode(dec: Decoder, st: SeqState, B: int, tau_c: float,
     while not st.done and len(out) < max_blocks:
         out.append(diffusion_block(dec, st, B, tau_c))
     return out
+
+
+def reveal_margin(conf: np.ndarray, gap: np.ndarray, masked: List[int], picked: List[int],
+                  tau: float) -> float:
+    """How far one reveal step's decisions are from flipping, in log units:
+    the top-2 logit gap of every picked row (its token), the distance of each
+    open confidence from the threshold (log scale), and, when the fallback
+    picked the single most confident, its log-ratio to the runner-up.  A GPU
+    whose logits are within e of these agrees with every decision where the
+    margin exceeds 2e."""
+    m = float("inf")
+    for j in picked:
+        m = min(m, float(gap[j]))
+    if tau > 0:
+        for j in masked:
+            m = min(m, abs(math.log(conf[j]) - math.log(tau)))
+    if len(picked) == 1 and not any(conf[j] > tau for j in masked) and len(masked) > 1:
+        rest = sorted((conf[j] for j in masked if j != picked[0]), reverse=True)
+        m = min(m, math.log(conf[picked[0]]) - math.log(rest[0]))
+    return m
 
 
 def tokens_per_forward(committed_per_round: List[int]) -> float:

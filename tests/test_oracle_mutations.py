@@ -113,6 +113,25 @@ def _cache_write_skipped(dec, cache, x0, block):
     cache.truncate(cache.seq_len + len(block))                   # slip: no causal rewrite
 
 
+def _refine_feedback_off_by_one(dec, cache, x0, K, tau_d):
+    fixed = [None] * (K + 1)
+    rec = od.RefinedDraft(0, [], [], [], [])
+    logits = None
+    while any(t is None for t in fixed):
+        logits = od.denoise_forward(dec, cache, x0, fixed[1:K + 1])   # slip: slot n+i carries pred i
+        conf = np.max(od.softmax_rows(logits), axis=1)
+        tok = od.argmax_rows(logits)
+        pick = od.reveal_positions(conf, [i for i in range(K + 1) if fixed[i] is None], tau_d)
+        for i in pick:
+            fixed[i] = int(tok[i])
+        rec.steps += 1
+        rec.fixed_per_step.append(pick)
+        rec.conf_per_step.append(conf)
+        rec.gap_per_step.append(od.top2_gap(logits))
+        rec.tok_per_step.append(tok)
+    return fixed[0], np.array(fixed[1:], dtype=np.int64), logits, rec
+
+
 MUTATIONS = [
     ("draft boundary row sees the mask block", od, "draft_forward", _draft_boundary_sees_masks,
      "test_boundary_row_is_the_ar_logit"),
@@ -134,6 +153,8 @@ MUTATIONS = [
      "test_diffusion_first_token_is_ar_and_cache_is_ar"),
     ("block cache write skipped", od, "cache_write_forward", _cache_write_skipped,
      "test_diffusion_first_token_is_ar_and_cache_is_ar"),
+    ("refined draft fed back one slot early", od, "refine_draft", _refine_feedback_off_by_one,
+     "test_refined_drafting_feeds_fixed_predictions_back_at_their_slots"),
 ]
 
 
@@ -150,6 +171,8 @@ def test_pin_catches_planted_mistake(monkeypatch, name, owner, attr, patched, pi
         caught = _fails(fn, (dec, w), 3)
     elif pin == "test_reveal_rule_cases":
         caught = _fails(fn)
+    elif pin == "test_refined_drafting_feeds_fixed_predictions_back_at_their_slots":
+        caught = _fails(fn, (dec, w), monkeypatch)
     else:
         caught = _fails(fn, (dec, w))
     assert caught, f"planted mistake not caught: {name}"

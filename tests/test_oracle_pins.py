@@ -18,7 +18,11 @@
   reveals one position per step, the most confident; a threshold below every
   probability reveals the block in one step, equal to the one-shot draft; a
   block's first token is the AR prediction; after every block the cache equals
-  AR's cache with no bidirectional state left; output cut at the first EOS.
+  AR's cache with no bidirectional state left; output cut at the first EOS;
+* multi-step drafting (Sec. 6 "Draft Schedule"): committed output equal to
+  greedy AR for every threshold, tau_d < 0 is the one-shot round, tau_d > 1
+  fixes one prediction per step (the most confident), each fixed prediction
+  is fed back at its own slot, and forcing still hits the schedule.
 """
 import math
 import os
@@ -446,3 +450,100 @@ def test_diffusion_stop_token_truncates(micro):
     st = _prefill(dec, max_new=40, eos=eos)
     od.diffusion_decode(dec, st, B, 0.0)
     assert st.done and st.out == free[:cut]
+
+
+# ------------------------------------------------------------------ multi-step drafting
+def _median_first_conf(dec, st, K):
+    logits = od.denoise_forward(dec, st.cache.copy(), st.x0, [None] * K)
+    return float(np.median(np.max(od.softmax_rows(logits), axis=1)))
+
+
+@pytest.mark.parametrize("tau", [-1.0, "median", 2.0])
+def test_refined_drafting_equals_greedy_ar(micro, tau):
+    """The verifier decides every committed token, so refining the draft
+    changes how many tokens a round commits, never which."""
+    dec, _ = micro
+    K = 5
+    ar = od.ar_decode(dec, _prefill(dec, max_new=36))
+    st = _prefill(dec, max_new=36)
+    t = _median_first_conf(dec, st, K) if tau == "median" else tau
+    while not st.done:
+        r, rec = od.self_spec_round_refined(dec, st, K, t)
+        assert 1 <= rec.steps <= K + 1
+        assert 2 <= len(r.committed) <= K + 2 or st.done
+    assert st.out == ar
+
+
+def test_refined_drafting_below_zero_is_one_shot(micro):
+    dec, _ = micro
+    K = 6
+    a, b = _prefill(dec, max_new=40), _prefill(dec, max_new=40)
+    for _ in range(3):
+        r1 = od.self_spec_round(dec, a, K)
+        r2, rec = od.self_spec_round_refined(dec, b, K, -1.0)
+        assert rec.steps == 1
+        assert (r1.a0, list(r1.d), list(r1.a), r1.A, r1.committed) == \
+            (r2.a0, list(r2.d), list(r2.a), r2.A, r2.committed)
+        np.testing.assert_allclose(r1.draft_logits, r2.draft_logits, rtol=0, atol=1e-12)
+
+
+def test_refined_drafting_above_one_fixes_the_most_confident(micro):
+    dec, _ = micro
+    K = 4
+    st = _prefill(dec, max_new=40)
+    _, rec = od.self_spec_round_refined(dec, st, K, 2.0)
+    assert rec.steps == K + 1
+    open_ = set(range(K + 1))
+    for pick, conf in zip(rec.fixed_per_step, rec.conf_per_step):
+        best = max(sorted(open_), key=lambda i: (conf[i], -i))
+        assert pick == [best]
+        open_.remove(best)
+
+
+def test_refined_drafting_feeds_fixed_predictions_back_at_their_slots(micro, monkeypatch):
+    """Prediction i (a0 for i = 0, d_i otherwise) is the token at slot n+1+i:
+    once fixed, the next draft forward carries it at that slot instead of [M]
+    (prediction K has no slot in the window)."""
+    dec, _ = micro
+    K = 4
+    st = _prefill(dec, max_new=40)
+    n = st.n
+    windows = []
+    real = Decoder.forward
+
+    def spy(self, x, slots, allowed, cache, return_hidden=False):
+        ids = [int(np.argmax(np.all(self.embed == row, axis=1))) for row in x]
+        windows.append((list(np.asarray(slots)), ids))
+        return real(self, x, slots, allowed, cache, return_hidden)
+
+    monkeypatch.setattr(Decoder, "forward", spy)
+    _, _, _, rec = od.refine_draft(dec, st.cache.copy(), st.x0, K, 2.0)
+    M = MICRO.mask_token_id
+    fixed = {}
+    assert len(windows) == rec.steps
+    for step, (slots, ids) in enumerate(windows):
+        assert slots == [n + i for i in range(K + 1)]
+        assert ids[0] == st.x0
+        for i in range(K):                       # slot n+1+i carries prediction i
+            assert ids[1 + i] == fixed.get(i, M), (step, i)
+        for i in rec.fixed_per_step[step]:
+            fixed[i] = int(rec.tok_per_step[step][i])
+    assert sorted(fixed) == list(range(K + 1))
+
+
+def test_refined_drafting_forced_schedule_hit(micro):
+    dec, _ = micro
+    K, max_new = 5, 40
+    ar = od.ar_decode(dec, _prefill(dec, max_new=max_new + K + 4))
+    st = _prefill(dec, max_new=max_new)
+    P = st.n
+    teacher = np.full(P + len(ar) + 1, -1, np.int64)
+    teacher[P:P + len(ar)] = ar
+    sched = [0, K, 2, 4, 1, 3, 0, K, 2, 2, 2, 2, 2, 2, 2]
+    r = 0
+    while not st.done:
+        res, _ = od.self_spec_round_refined(dec, st, K, 0.0, teacher, sched[r])
+        if not st.done:
+            assert res.A == sched[r]
+        r += 1
+    assert st.out == ar[:max_new]
