@@ -173,6 +173,52 @@ int gs_prefill(gs_handle *h, int slot, const void *vis_emb, int n_vis, const int
 int gs_round(gs_handle *h, const int32_t *slots, int n_seq, int K, int rule, const gs_force *force,
              int32_t *out_tok, int32_t *out_cnt, int32_t *out_done, const gs_debug *dbg);
 
+/* Direct block-diffusion decoding of one block per sequence (paper Appendix
+ * "Direct Block-Diffusion Decoding"; Sec. 5 diffusion-vs-self-speculative
+ * comparison).  From the same state as gs_round (the cache holds every
+ * committed token but the boundary x0), a block of B [M] tokens at slots
+ * n+1..n+B is denoised: each step is one forward over [x0, block] with the
+ * draft's hybrid mask (x0 causal, block rows bidirectional in the window),
+ * the prediction for position p read from the row at p-1; every still-masked
+ * position whose argmax probability exceeds tau_c is revealed, or, if none
+ * is, the single most confident one (ties to the lowest position); revealed
+ * tokens stay fixed.  When every sequence's block is complete, one causal
+ * forward over [x0, y_1..y_B] writes the cache (no LM head), and the block is
+ * committed: y_1..y_B cut at the first EOS or at max_new, seq_len += B,
+ * x0 = y_B.  All steps run inside one CUDA graph whose denoising loop is a
+ * conditional (while) node: no host synchronisation; the loop is capped at B
+ * steps (a sequence still open after B steps raises the device check).
+ *   slots     device int32 [n_seq], distinct prefilled slots
+ *   B         block size, 1 <= B <= max_K
+ *   tau_c     confidence threshold (probabilities are in (0, 1]; tau_c >= 1
+ *             reveals one position per step, tau_c < 0 the whole block at once)
+ *   out_tok   device int32 [n_seq, B]: committed tokens of the block
+ *   out_cnt   device int32 [n_seq]: how many (0 for a sequence already done)
+ *   out_done  device int32 [n_seq]: 1 once the sequence hit EOS or max_new
+ *   out_steps device int32 [n_seq] or NULL: denoising forwards of the block
+ *             (the paper's TPF for this mode counts these, not the cache write)
+ * Needs a handle created on a non-default stream.  Graphs are cached per
+ * (n_seq, B, tau_c, pointers).  Errors: GS_ERR_INVALID_ARG, GS_ERR_CUDA. */
+int gs_diffusion_block(gs_handle *h, const int32_t *slots, int n_seq, int B, float tau_c,
+                       int32_t *out_tok, int32_t *out_cnt, int32_t *out_done, int32_t *out_steps);
+
+/* A self-speculative round with multi-step drafting (paper Sec. 6 "Draft
+ * Schedule", Fig. "Multi-step drafting versus one-shot drafting").  The draft
+ * window [x0, [M] x K] is run repeatedly: prediction i (a0 for i = 0, d_i
+ * otherwise, read from row i) is fixed once its argmax probability exceeds
+ * tau_d, or, when no open prediction does, the single most confident one is;
+ * a fixed prediction i < K is fed back at its own slot n+1+i in place of the
+ * mask; after at most K+1 draft forwards the finished draft is verified,
+ * accepted and committed exactly as by gs_round (GS_ACCEPT_GREEDY; the
+ * forcing hook applies to the refined draft).  tau_d < 0 is the one-shot
+ * round.  One graph launch with a conditional loop, no host synchronisation.
+ *   out_tok [n_seq, K+2], out_cnt, out_done: as gs_round
+ *   out_steps device int32 [n_seq] or NULL: draft forwards of the round
+ * Needs a non-default stream.  Errors: GS_ERR_INVALID_ARG, GS_ERR_CUDA. */
+int gs_round_refined(gs_handle *h, const int32_t *slots, int n_seq, int K, float tau_d,
+                     const gs_force *force, int32_t *out_tok, int32_t *out_cnt, int32_t *out_done,
+                     int32_t *out_steps);
+
 /* Overwrite a sequence's per-slot state (resume/checkpoint: with the KV pages,
  * which keep their contents, the state is the cached length, the boundary
  * token, the output count and cap, the done flag and the round counter that

@@ -5,6 +5,7 @@
 #include <cmath>
 #include <cstdio>
 #include <cstring>
+#include <functional>
 #include <map>
 #include <mutex>
 #include <string>
@@ -12,6 +13,7 @@
 #include <vector>
 
 #include "attention.cuh"
+#include "denoise.cuh"
 #include "gemm_tc.cuh"
 #include "internal.h"
 #include "small.cuh"
@@ -257,6 +259,19 @@ struct gs_handle {
   int launches = 0;             // kernel launches counted while enqueueing
   int last_round_launches = 0;
 
+  // programmatic dependent launch on the decoder's launches (off while a
+  // graph with a conditional loop is captured)
+  bool pdl = true;
+  // denoising loops (block diffusion, multi-step drafting): per-slot fixed
+  // predictions, flags and step counts, the loop counter, the LM head's
+  // softmax partials, a side stream for capturing loop bodies, their graphs
+  int32_t *dn_fixed = nullptr, *dn_live = nullptr, *dn_part = nullptr, *dn_steps = nullptr;
+  int32_t* dn_iter = nullptr;
+  float2* lse_part = nullptr;
+  int lse_tiles = 0;
+  cudaStream_t side = nullptr;
+  std::map<std::vector<uint64_t>, cudaGraphExec_t> loop_graphs;
+
   // gs_round_profile: an event after every launch and the launch's kind
   bool profiling = false;
   cudaError_t prof_err = cudaSuccess;
@@ -390,6 +405,13 @@ size_t carve(gs_handle* h, const gs_config& c, void* base) {
   int* gemm_counters = cv.take<int>(kGemmCounters);
   float* attn_part = cv.take<float>(attn_part_floats);
   int* attn_ticket = cv.take<int>(attn_blocks * c.n_kv_heads);
+  int32_t* dn_fixed = cv.take<int32_t>(static_cast<size_t>(c.max_batch) * W_max);
+  int32_t* dn_live = cv.take<int32_t>(c.max_batch);
+  int32_t* dn_part = cv.take<int32_t>(c.max_batch);
+  int32_t* dn_steps = cv.take<int32_t>(c.max_batch);
+  int32_t* dn_iter = cv.take<int32_t>(64);
+  const int lse_tiles = c.vocab / 128;
+  float2* lse_part = cv.take<float2>(static_cast<size_t>(c.max_batch) * W_max * lse_tiles);
   // fp16 weight copies: per layer qkv | o | gate_up | down, then the LM head
   const size_t per_layer = static_cast<size_t>(qkv_dim) * c.d_model +
                            static_cast<size_t>(c.d_model) * c.n_heads * 64 +
@@ -440,6 +462,13 @@ size_t carve(gs_handle* h, const gs_config& c, void* base) {
     h->verify_tok = verify_tok;
     h->gemm_partial = gemm_partial;
     h->gemm_counters = gemm_counters;
+    h->dn_fixed = dn_fixed;
+    h->dn_live = dn_live;
+    h->dn_part = dn_part;
+    h->dn_steps = dn_steps;
+    h->dn_iter = dn_iter;
+    h->lse_part = lse_part;
+    h->lse_tiles = lse_tiles;
   }
   return align_up(cv.off, 256);
 }
@@ -473,7 +502,7 @@ int run_gemm(gs_handle* h, const CUtensorMap& tw, int weight_rows, const CUtenso
        p.feat_tiles * p.tok_tiles > kGemmCounters))
     return fail(h, GS_ERR_OOM, "split-K scratch too small");
   GS_CUDA(h, launch_gemm(p.bn, epi, tw, tx_set[bn_index(p.bn)], a, p.feat_tiles, p.tok_tiles,
-                         h->stream, true));
+                         h->stream, h->pdl));
   note_launch(h, kind);
   return GS_OK;
 }
@@ -518,7 +547,7 @@ int run_attention(gs_handle* h, int layer, int T, const AttnLaunch& L) {
            h->attn_part_floats ||
        L.max_items > attn_max_merge_items(g.rows)))
     return fail(h, GS_ERR_OOM, "attention item scratch too small");
-  GS_CUDA(h, launch_attention(h->tm_kv, a, n_blocks, h->stream, true));
+  GS_CUDA(h, launch_attention(h->tm_kv, a, n_blocks, h->stream, h->pdl));
   note_launch(h, GS_KIND_ATTENTION);
   return GS_OK;
 }
@@ -531,10 +560,10 @@ int run_attention(gs_handle* h, int layer, int T, const AttnLaunch& L) {
 // (+residual, next norm's input).
 int forward(gs_handle* h, int T, const int32_t* tok, const __nv_bfloat16* vis, int n_vis,
             const AttnLaunch& AL, int lm_row0, int n_lm, unsigned long long* packed,
-            float* logits, bool decode) {
+            float* logits, bool decode, float2* lse_part = nullptr) {
   const gs_config& c = h->cfg;
   const int d = c.d_model, F = c.d_ffn, HD = c.n_heads * 64, L = c.n_layers;
-  GS_CUDA(h, launch_ex(embed_kernel, dim3(T), dim3(128), 0, h->stream, true, dim3(1), tok, h->embed, vis,
+  GS_CUDA(h, launch_ex(embed_kernel, dim3(T), dim3(128), 0, h->stream, h->pdl, dim3(1), tok, h->embed, vis,
                        n_vis, T, d, c.vocab, h->hbuf, h->hb, h->attn_norm[0], h->ssp, packed,
                        h->err_word));
   note_launch(h, GS_KIND_EMBED);
@@ -598,6 +627,7 @@ int forward(gs_handle* h, int T, const int32_t* tok, const __nv_bfloat16* vis, i
   lm.N = c.vocab;
   lm.y = packed;
   lm.logits = logits;
+  lm.lse_part = lse_part;
   lm.ssp_in = h->ssp;
   lm.x_row0 = lm_row0;
   return run_gemm(h, h->tm_lm, c.vocab, h->tm_hb, d, n_lm, kEpiArgmax, lm, decode,
@@ -644,12 +674,12 @@ int enqueue_round(gs_handle* h, const int32_t* slots, int n_seq, int K, const gs
   AL.fixed_slot = -1;
 
   h->launches = 0;
-  GS_CUDA(h, launch_ex(window_draft_kernel, dim3(nb), dim3(128), 0, h->stream, true, dim3(1), w));
+  GS_CUDA(h, launch_ex(window_draft_kernel, dim3(nb), dim3(128), 0, h->stream, h->pdl, dim3(1), w));
   note_launch(h, GS_KIND_WINDOW);
   int rc = forward(h, T, h->tok, nullptr, 0, AL, 0, T, h->packed_d,
                    dbg ? dbg->draft_logits : nullptr, true);
   if (rc) return rc;
-  GS_CUDA(h, launch_ex(window_verify_kernel, dim3(nb), dim3(128), 0, h->stream, true, dim3(1), w));
+  GS_CUDA(h, launch_ex(window_verify_kernel, dim3(nb), dim3(128), 0, h->stream, h->pdl, dim3(1), w));
   note_launch(h, GS_KIND_WINDOW);
   rc = forward(h, T, h->tok, nullptr, 0, AL, 0, T, h->packed_v, dbg ? dbg->verify_logits : nullptr,
                true);
@@ -667,7 +697,7 @@ int enqueue_round(gs_handle* h, const int32_t* slots, int n_seq, int K, const gs
   ac.out_tok = out_tok;
   ac.out_cnt = out_cnt;
   ac.out_done = out_done;
-  GS_CUDA(h, launch_ex(accept_commit_kernel, dim3(cdiv(n_seq, 64)), dim3(64), 0, h->stream, true, dim3(1),
+  GS_CUDA(h, launch_ex(accept_commit_kernel, dim3(cdiv(n_seq, 64)), dim3(64), 0, h->stream, h->pdl, dim3(1),
                        ac));
   note_launch(h, GS_KIND_ACCEPT);
   if (dbg) {
@@ -681,6 +711,165 @@ int enqueue_round(gs_handle* h, const int32_t* slots, int n_seq, int K, const gs
   }
   h->last_round_launches = h->launches;
   return GS_OK;
+}
+
+// Capture pre(), then a WHILE conditional node whose body is body(handle)
+// (captured on the side stream), then post(), as one executable graph.  The
+// loop runs while the handle's value is nonzero; it is 1 at every launch and
+// the body's last kernel sets it.  Programmatic dependent launch is off for
+// every launch of such a graph.
+int capture_loop_graph(gs_handle* h, const std::function<int()>& pre,
+                       const std::function<int(cudaGraphConditionalHandle)>& body,
+                       const std::function<int()>& post, cudaGraphExec_t* out) {
+  if (!h->side) GS_CUDA(h, cudaStreamCreateWithFlags(&h->side, cudaStreamNonBlocking));
+  const bool pdl_was = h->pdl;
+  h->pdl = false;
+  cudaGraph_t g = nullptr;
+  auto finish = [&](int code, const char* what, cudaError_t e) {
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    if (cudaStreamIsCapturing(h->stream, &cs) == cudaSuccess && cs != cudaStreamCaptureStatusNone) {
+      cudaGraph_t dead = nullptr;
+      cudaStreamEndCapture(h->stream, &dead);
+      if (dead) cudaGraphDestroy(dead);
+    }
+    h->pdl = pdl_was;
+    if (code == GS_ERR_CUDA)
+      return fail(h, code, std::string(what) + ": " + cudaGetErrorString(e));
+    return code;
+  };
+  cudaError_t e = cudaStreamBeginCapture(h->stream, cudaStreamCaptureModeThreadLocal);
+  if (e != cudaSuccess) return finish(GS_ERR_CUDA, "loop capture", e);
+  int rc = pre();
+  if (rc) return finish(rc, "", cudaSuccess);
+  cudaStreamCaptureStatus cs;
+  cudaGraph_t cg = nullptr;
+  const cudaGraphNode_t* deps = nullptr;
+  const cudaGraphEdgeData* edata = nullptr;
+  size_t ndeps = 0;
+  e = cudaStreamGetCaptureInfo(h->stream, &cs, nullptr, &cg, &deps, &edata, &ndeps);
+  if (e != cudaSuccess) return finish(GS_ERR_CUDA, "capture info", e);
+  cudaGraphConditionalHandle hc;
+  e = cudaGraphConditionalHandleCreate(&hc, cg, 1, cudaGraphCondAssignDefault);
+  if (e != cudaSuccess) return finish(GS_ERR_CUDA, "conditional handle", e);
+  cudaGraphNodeParams np = {};
+  np.type = cudaGraphNodeTypeConditional;
+  np.conditional.handle = hc;
+  np.conditional.type = cudaGraphCondTypeWhile;
+  np.conditional.size = 1;
+  cudaGraphNode_t node;
+  e = cudaGraphAddNode(&node, cg, deps, edata, ndeps, &np);
+  if (e != cudaSuccess) return finish(GS_ERR_CUDA, "conditional node", e);
+  cudaGraph_t body_graph = np.conditional.phGraph_out[0];
+  e = cudaStreamUpdateCaptureDependencies(h->stream, &node, nullptr, 1,
+                                          cudaStreamSetCaptureDependencies);
+  if (e != cudaSuccess) return finish(GS_ERR_CUDA, "capture dependencies", e);
+  e = cudaStreamBeginCaptureToGraph(h->side, body_graph, nullptr, nullptr, 0,
+                                    cudaStreamCaptureModeThreadLocal);
+  if (e != cudaSuccess) return finish(GS_ERR_CUDA, "body capture", e);
+  std::swap(h->stream, h->side);
+  rc = body(hc);
+  std::swap(h->stream, h->side);
+  cudaGraph_t captured_body = nullptr;
+  e = cudaStreamEndCapture(h->side, &captured_body);
+  if (rc) return finish(rc, "", cudaSuccess);
+  if (e != cudaSuccess) return finish(GS_ERR_CUDA, "body capture end", e);
+  rc = post();
+  if (rc) return finish(rc, "", cudaSuccess);
+  e = cudaStreamEndCapture(h->stream, &g);
+  h->pdl = pdl_was;
+  if (e != cudaSuccess) return fail(h, GS_ERR_CUDA, std::string("loop capture end: ") + cudaGetErrorString(e));
+  e = cudaGraphInstantiate(out, g, 0);
+  cudaGraphDestroy(g);
+  if (e != cudaSuccess)
+    return fail(h, GS_ERR_CUDA, std::string("loop graph instantiate: ") + cudaGetErrorString(e));
+  return GS_OK;
+}
+
+DenoiseArgs denoise_args(gs_handle* h, const int32_t* slots, int n_seq, int W, int n_pred,
+                         float tau) {
+  DenoiseArgs d;
+  memset(&d, 0, sizeof(d));
+  d.slots = slots;
+  d.n_seq = n_seq;
+  d.W = W;
+  d.n_pred = n_pred;
+  d.mask_id = h->cfg.mask_token_id;
+  d.vocab = h->cfg.vocab;
+  d.eos = h->cfg.eos_token_id;
+  d.tau = tau;
+  d.st = h->st;
+  d.fixed = h->dn_fixed;
+  d.W_max = h->W_max;
+  d.live = h->dn_live;
+  d.part = h->dn_part;
+  d.steps = h->dn_steps;
+  d.iter = h->dn_iter;
+  d.tok = h->tok;
+  d.pos = h->pos;
+  d.lim = h->lim;
+  d.tok_slot = h->tok_slot;
+  d.blk_slot = h->blk_slot;
+  d.blk_active = h->blk_active;
+  d.packed = h->packed_d;
+  d.lse_part = h->lse_part;
+  d.lse_tiles = h->lse_tiles;
+  d.err = h->err_word;
+  return d;
+}
+
+AttnLaunch decode_attention(gs_handle* h, int n_seq, int W) {
+  AttnLaunch AL;
+  AL.n_seq = n_seq;
+  AL.QB = W;
+  AL.split_pages = h->split_pages;
+  AL.max_items = h->items_dec;
+  AL.blk_slot = h->blk_slot;
+  AL.blk_active = h->blk_active;
+  AL.fixed_slot = -1;
+  return AL;
+}
+
+// One denoising step (the body of the loop): window, forward with the LM
+// head's argmax and softmax partials, reveal, loop condition.
+int enqueue_denoise_step(gs_handle* h, DenoiseArgs d) {
+  const int T = d.n_seq * d.W;
+  GS_CUDA(h, launch_ex(denoise_window_kernel, dim3(cdiv(T, 128)), dim3(128), 0, h->stream, h->pdl,
+                       dim3(1), d));
+  note_launch(h, GS_KIND_WINDOW);
+  int rc = forward(h, T, h->tok, nullptr, 0, decode_attention(h, d.n_seq, d.W), 0, T, h->packed_d,
+                   nullptr, true, h->lse_part);
+  if (rc) return rc;
+  GS_CUDA(h, launch_ex(denoise_reveal_kernel, dim3(d.n_seq), dim3(128), 0, h->stream, h->pdl,
+                       dim3(1), d));
+  note_launch(h, GS_KIND_ACCEPT);
+  GS_CUDA(h, launch_ex(denoise_cond_kernel, dim3(1), dim3(32), 0, h->stream, h->pdl, dim3(1), d));
+  note_launch(h, GS_KIND_ACCEPT);
+  return GS_OK;
+}
+
+int launch_loop_graph(gs_handle* h, const std::vector<uint64_t>& key,
+                      const std::function<int(cudaGraphExec_t*)>& build) {
+  auto it = h->loop_graphs.find(key);
+  if (it == h->loop_graphs.end()) {
+    cudaGraphExec_t ge = nullptr;
+    const int rc = build(&ge);
+    if (rc) return rc;
+    if (h->loop_graphs.size() >= 32) {
+      cudaGraphExecDestroy(h->loop_graphs.begin()->second);
+      h->loop_graphs.erase(h->loop_graphs.begin());
+    }
+    it = h->loop_graphs.emplace(key, ge).first;
+  }
+  GS_CUDA(h, cudaGraphLaunch(it->second, h->stream));
+  return GS_OK;
+}
+
+uint64_t ptr_key(const void* p) { return static_cast<uint64_t>(reinterpret_cast<uintptr_t>(p)); }
+
+uint32_t float_bits(float x) {
+  uint32_t u;
+  std::memcpy(&u, &x, 4);
+  return u;
 }
 
 }  // namespace
@@ -844,6 +1033,8 @@ int gs_create(const gs_config* cfg, const gs_weights* w, void* workspace, size_t
 int gs_destroy(gs_handle* h) {
   if (!h) return GS_ERR_INVALID_ARG;
   for (auto& kv : h->graphs) cudaGraphExecDestroy(kv.second);
+  for (auto& kv : h->loop_graphs) cudaGraphExecDestroy(kv.second);
+  if (h->side) cudaStreamDestroy(h->side);
   for (cudaEvent_t e : h->prof_ev) cudaEventDestroy(e);
   delete h;
   return GS_OK;
@@ -969,6 +1160,152 @@ int gs_round(gs_handle* h, const int32_t* slots, int n_seq, int K, int rule, con
   }
   GS_CUDA(h, cudaGraphLaunch(it->second, h->stream));
   return GS_OK;
+}
+
+int gs_diffusion_block(gs_handle* h, const int32_t* slots, int n_seq, int B, float tau_c,
+                       int32_t* out_tok, int32_t* out_cnt, int32_t* out_done, int32_t* out_steps) {
+  if (!h) return GS_ERR_INVALID_ARG;
+  const gs_config& c = h->cfg;
+  if (!slots || !out_tok || !out_cnt || !out_done)
+    return fail(h, GS_ERR_INVALID_ARG, "null slots or output pointer");
+  if (n_seq < 1 || n_seq > c.max_batch) return fail(h, GS_ERR_INVALID_ARG, "n_seq out of range");
+  if (B < 1 || B > c.max_K) return fail(h, GS_ERR_INVALID_ARG, "B out of range (1..max_K)");
+  if (!(tau_c == tau_c)) return fail(h, GS_ERR_INVALID_ARG, "tau_c is NaN");
+  if (!h->stream) return fail(h, GS_ERR_INVALID_ARG, "block diffusion needs a non-default stream");
+  const int W = B + 1, T = n_seq * W;
+  const std::vector<uint64_t> key = {1, static_cast<uint64_t>(n_seq), static_cast<uint64_t>(B),
+                                     float_bits(tau_c), ptr_key(slots), ptr_key(out_tok),
+                                     ptr_key(out_cnt), ptr_key(out_done), ptr_key(out_steps)};
+  return launch_loop_graph(h, key, [&](cudaGraphExec_t* ge) -> int {
+    DenoiseArgs d = denoise_args(h, slots, n_seq, W, B, tau_c);
+    d.out_tok = out_tok;
+    d.out_cnt = out_cnt;
+    d.out_done = out_done;
+    d.out_steps = out_steps;
+    h->launches = 0;
+    return capture_loop_graph(
+        h,
+        [&]() -> int {
+          GS_CUDA(h, launch_ex(denoise_init_kernel, dim3(n_seq), dim3(32), 0, h->stream, h->pdl,
+                               dim3(1), d));
+          note_launch(h, GS_KIND_WINDOW);
+          return GS_OK;
+        },
+        [&](cudaGraphConditionalHandle hc) -> int {
+          DenoiseArgs db = d;
+          db.cond = hc;
+          return enqueue_denoise_step(h, db);
+        },
+        [&]() -> int {
+          // the cache-write pass of the completed blocks (no LM head), then commit
+          GS_CUDA(h, launch_ex(block_write_window_kernel, dim3(cdiv(T, 128)), dim3(128), 0,
+                               h->stream, h->pdl, dim3(1), d));
+          note_launch(h, GS_KIND_WINDOW);
+          int rc = forward(h, T, h->tok, nullptr, 0, decode_attention(h, n_seq, W), 0, 0,
+                           h->packed_d, nullptr, true);
+          if (rc) return rc;
+          GS_CUDA(h, launch_ex(block_commit_kernel, dim3(cdiv(n_seq, 64)), dim3(64), 0, h->stream,
+                               h->pdl, dim3(1), d));
+          note_launch(h, GS_KIND_ACCEPT);
+          return GS_OK;
+        },
+        ge);
+  });
+}
+
+int gs_round_refined(gs_handle* h, const int32_t* slots, int n_seq, int K, float tau_d,
+                     const gs_force* force, int32_t* out_tok, int32_t* out_cnt, int32_t* out_done,
+                     int32_t* out_steps) {
+  if (!h) return GS_ERR_INVALID_ARG;
+  const gs_config& c = h->cfg;
+  if (!slots || !out_tok || !out_cnt || !out_done)
+    return fail(h, GS_ERR_INVALID_ARG, "null slots or output pointer");
+  if (n_seq < 1 || n_seq > c.max_batch) return fail(h, GS_ERR_INVALID_ARG, "n_seq out of range");
+  if (K < 0 || K > c.max_K) return fail(h, GS_ERR_INVALID_ARG, "K out of range");
+  if (!(tau_d == tau_d)) return fail(h, GS_ERR_INVALID_ARG, "tau_d is NaN");
+  if (force && (!force->teacher || !force->L_sched || force->teacher_stride < 1))
+    return fail(h, GS_ERR_INVALID_ARG, "incomplete force hook");
+  if (!h->stream) return fail(h, GS_ERR_INVALID_ARG, "multi-step drafting needs a non-default stream");
+  const int W = K + 1, T = n_seq * W;
+  const std::vector<uint64_t> key = {
+      2, static_cast<uint64_t>(n_seq), static_cast<uint64_t>(K), float_bits(tau_d), ptr_key(slots),
+      ptr_key(out_tok), ptr_key(out_cnt), ptr_key(out_done), ptr_key(out_steps),
+      ptr_key(force ? force->teacher : nullptr),
+      static_cast<uint64_t>(force ? force->teacher_stride : 0),
+      ptr_key(force ? force->L_sched : nullptr), static_cast<uint64_t>(force ? force->L_stride : 0)};
+  return launch_loop_graph(h, key, [&](cudaGraphExec_t* ge) -> int {
+    DenoiseArgs d = denoise_args(h, slots, n_seq, W, W, tau_d);
+    h->launches = 0;
+    return capture_loop_graph(
+        h,
+        [&]() -> int {
+          GS_CUDA(h, launch_ex(denoise_init_kernel, dim3(n_seq), dim3(32), 0, h->stream, h->pdl,
+                               dim3(1), d));
+          note_launch(h, GS_KIND_WINDOW);
+          return GS_OK;
+        },
+        [&](cudaGraphConditionalHandle hc) -> int {
+          DenoiseArgs db = d;
+          db.cond = hc;
+          return enqueue_denoise_step(h, db);
+        },
+        [&]() -> int {
+          // verify the refined draft exactly as a one-shot draft, then accept
+          WindowArgs w;
+          memset(&w, 0, sizeof(w));
+          w.slots = slots;
+          w.n_seq = n_seq;
+          w.K = K;
+          w.W = W;
+          w.mask_id = c.mask_token_id;
+          w.vocab = c.vocab;
+          w.st = h->st;
+          w.tok = h->tok;
+          w.pos = h->pos;
+          w.lim = h->lim;
+          w.tok_slot = h->tok_slot;
+          w.blk_slot = h->blk_slot;
+          w.blk_active = h->blk_active;
+          w.draft_packed = h->packed_d;
+          w.draft_tok = h->draft_tok;
+          w.verify_in = h->verify_in;
+          w.draft_fixed = h->dn_fixed;
+          w.fixed_stride = h->W_max;
+          w.steps_src = h->dn_steps;
+          w.steps_out = out_steps;
+          if (force) {
+            w.teacher = force->teacher;
+            w.teacher_stride = force->teacher_stride;
+            w.L_sched = force->L_sched;
+            w.L_stride = force->L_stride;
+          }
+          w.err = h->err_word;
+          GS_CUDA(h, launch_ex(window_verify_kernel, dim3(cdiv(T, 128)), dim3(128), 0, h->stream,
+                               h->pdl, dim3(1), w));
+          note_launch(h, GS_KIND_WINDOW);
+          int rc = forward(h, T, h->tok, nullptr, 0, decode_attention(h, n_seq, W), 0, T,
+                           h->packed_v, nullptr, true);
+          if (rc) return rc;
+          AcceptArgs ac;
+          ac.slots = slots;
+          ac.n_seq = n_seq;
+          ac.K = K;
+          ac.W = W;
+          ac.eos = c.eos_token_id;
+          ac.st = h->st;
+          ac.verify_in = h->verify_in;
+          ac.verify_packed = h->packed_v;
+          ac.verify_tok = h->verify_tok;
+          ac.out_tok = out_tok;
+          ac.out_cnt = out_cnt;
+          ac.out_done = out_done;
+          GS_CUDA(h, launch_ex(accept_commit_kernel, dim3(cdiv(n_seq, 64)), dim3(64), 0, h->stream,
+                               h->pdl, dim3(1), ac));
+          note_launch(h, GS_KIND_ACCEPT);
+          return GS_OK;
+        },
+        ge);
+  });
 }
 
 int gs_seq_restore(gs_handle* h, int slot, int seq_len, int x0, int n_out, int max_new, int done,

@@ -64,6 +64,9 @@ struct GemmArgs {
   float* partial;   // global split-K partials [splits][tiles][BN][128] fp32 (cluster == 0)
   int* counters;    // per output tile, zero between launches (cluster == 0)
   float* logits;    // argmax only: optional fp32 [M, N] dump
+  // argmax only, optional: per token and 128-row feature tile, (tile max,
+  // sum over the tile of exp(logit - tile max)) at [token][feature tile]
+  float2* lse_part;
   int* err;
   float w_scale;    // 2^-s of the weight copy (1 for unscaled weights)
   int x_row0;       // X (and ssp_in) row of token 0
@@ -101,8 +104,9 @@ struct GemmShape {
   static constexpr int kXBufBytes = 32 * 128 * 4;  // epilogue exchange (SwiGLU, RoPE, sums)
   static_assert(!(BN <= 64) || kXBufBytes + kRedBytes <= kStagesMin * kStageBytes,
                 "cluster staging smem");
-  // argmax epilogue: keys [128][33] and quarter maxima [4][32], 8 bytes each
-  static_assert((128 * 33 + 4 * 32) * 8 <= kStagesMin * kStageBytes, "argmax smem");
+  // argmax epilogue: keys [128][33] and quarter maxima [4][32], 8 bytes each,
+  // then the softmax partials' tile maxima [32] and warp sums [4][32], 4 bytes each
+  static_assert((128 * 33 + 4 * 32) * 8 + 5 * 32 * 4 <= kStagesMin * kStageBytes, "argmax smem");
   // RoPE cos/sin rows of the tile's tokens, staged while the mainloop runs
   // (QKV launches, decode tiles)
   static constexpr bool kStageRope = BN <= 64;
@@ -309,14 +313,37 @@ __device__ __forceinline__ void gemm_epilogue_chunk(const GemmArgs& a, float (&v
       qb[q * EW + j] = best;
     }
     asm volatile("bar.sync 2, 128;" ::: "memory");
+    float* tmax = reinterpret_cast<float*>(qb + 4 * EW);   // [EW] tile maxima
     if (threadIdx.x < EW) {
       const int j = threadIdx.x;
       unsigned long long best = qb[j];
 #pragma unroll
       for (int q = 1; q < 4; ++q) best = qb[q * EW + j] > best ? qb[q * EW + j] : best;
       if (j >= jlo && j < jhi) atomicMax(out + t0 + j, best);
+      tmax[j] = argmax_key_value(best);
     }
     asm volatile("bar.sync 2, 128;" ::: "memory");
+    if (a.lse_part != nullptr) {
+      // softmax partials of this tile: sum over its 128 rows of exp(v - tile
+      // max), a warp tree then the four warps in order (fixed order: the same
+      // bits for a row whatever the batch)
+      float* wsum = tmax + EW;   // [4][EW]
+#pragma unroll
+      for (int j = 0; j < EW; ++j) {
+        float e = expf(v[j] - tmax[j]);
+#pragma unroll
+        for (int m = 16; m >= 1; m >>= 1) e += __shfl_xor_sync(0xFFFFFFFFu, e, m);
+        if (lane == 0) wsum[warp * EW + j] = e;
+      }
+      asm volatile("bar.sync 2, 128;" ::: "memory");
+      if (threadIdx.x < EW) {
+        const int j = threadIdx.x;
+        if (j >= jlo && j < jhi)
+          a.lse_part[static_cast<size_t>(t0 + j) * gridDim.y + feat_tile] = make_float2(
+              tmax[j], ((wsum[j] + wsum[EW + j]) + wsum[2 * EW + j]) + wsum[3 * EW + j]);
+      }
+      asm volatile("bar.sync 2, 128;" ::: "memory");
+    }
   }
 }
 

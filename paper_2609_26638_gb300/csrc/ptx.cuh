@@ -311,6 +311,12 @@ __device__ __forceinline__ unsigned long long argmax_key(float v, uint32_t idx) 
          static_cast<unsigned long long>(0xFFFFFFFFu - idx);
 }
 
+// The float value an argmax key was made from (inverse of float_order_key).
+__device__ __forceinline__ float argmax_key_value(unsigned long long key) {
+  const uint32_t k = static_cast<uint32_t>(key >> 32);
+  return __uint_as_float((k & 0x80000000u) ? (k & 0x7FFFFFFFu) : ~k);
+}
+
 __device__ __forceinline__ int argmax_key_index(unsigned long long key) {
   return static_cast<int>(0xFFFFFFFFu - static_cast<uint32_t>(key & 0xFFFFFFFFull));
 }

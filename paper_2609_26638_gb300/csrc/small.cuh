@@ -36,6 +36,13 @@ struct WindowArgs {
   const int32_t* L_sched;
   long long L_stride;
   int* err;
+  // multi-step drafting: the refined draft (fixed predictions per slot,
+  // [slot * fixed_stride + i]) replaces the draft argmax; its step counts
+  // are copied to steps_out [n_seq]
+  const int32_t* draft_fixed;
+  int fixed_stride;
+  const int32_t* steps_src;
+  int32_t* steps_out;
 };
 
 // Draft window: [x0, [M] x K] at slots n..n+K; row 0 sees keys 0..n, mask rows 0..n+K.
@@ -68,8 +75,11 @@ __global__ void window_verify_kernel(WindowArgs a) {
   const int b = idx / a.W, i = idx % a.W;
   const int slot = a.slots[b];
   const int n = a.st.seq_len[slot];
-  int t = argmax_key_index(a.draft_packed[idx]);
+  int t = a.draft_fixed != nullptr
+              ? a.draft_fixed[static_cast<size_t>(slot) * a.fixed_stride + i]
+              : argmax_key_index(a.draft_packed[idx]);
   a.draft_tok[idx] = t;
+  if (i == 0 && a.steps_out != nullptr) a.steps_out[b] = a.steps_src[slot];
   if (a.teacher != nullptr && i >= 1 && a.st.done[slot] == 0) {
     const int r = a.st.rounds[slot];
     int L = 0;

@@ -80,6 +80,9 @@ def _load():
         "gs_round": (i32, [vp, vp, i32, i32, i32, ctypes.POINTER(gs_force), vp, vp, vp,
                            ctypes.POINTER(gs_debug)]),
         "gs_seq_restore": (i32, [vp, i32, i32, i32, i32, i32, i32, i32]),
+        "gs_diffusion_block": (i32, [vp, vp, i32, i32, ctypes.c_float, vp, vp, vp, vp]),
+        "gs_round_refined": (i32, [vp, vp, i32, i32, ctypes.c_float, ctypes.POINTER(gs_force), vp,
+                                   vp, vp, vp]),
         "gs_round_launches": (i32, [vp]),
         "gs_round_profile": (i32, [vp, vp, i32, i32, ctypes.POINTER(gs_force), vp, vp, vp, i32,
                                    ctypes.POINTER(ctypes.c_float), ctypes.POINTER(i32),
@@ -105,7 +108,7 @@ def _load():
 
 _lib = _load()
 EXPORTED = ("gs_workspace_bytes", "gs_create", "gs_destroy", "gs_last_error", "gs_prefill",
-            "gs_round", "gs_seq_restore", "gs_round_launches", "gs_round_profile", "gs_seq_state",
+            "gs_round", "gs_diffusion_block", "gs_round_refined", "gs_seq_restore", "gs_round_launches", "gs_round_profile", "gs_seq_state",
             "gs_release", "gs_sync_check", "gs_wait_probe",
             "gs_attention_scratch_bytes", "gs_attention", "gs_linear_scratch_bytes", "gs_linear",
             "gs_linear_noalloc", "gs_linear_noalloc_status")
@@ -155,6 +158,20 @@ def gs_round(h, slots_ptr: int, n_seq: int, K: int, rule: int, force: gs_force |
                             ctypes.byref(force) if force is not None else None,
                             out_tok_ptr, out_cnt_ptr, out_done_ptr,
                             ctypes.byref(dbg) if dbg is not None else None))
+
+
+def gs_diffusion_block(h, slots_ptr: int, n_seq: int, B: int, tau_c: float, out_tok_ptr: int,
+                       out_cnt_ptr: int, out_done_ptr: int, out_steps_ptr: int = 0) -> None:
+    _check(h, _lib.gs_diffusion_block(h, slots_ptr, n_seq, B, tau_c, out_tok_ptr, out_cnt_ptr,
+                                      out_done_ptr, out_steps_ptr or None))
+
+
+def gs_round_refined(h, slots_ptr: int, n_seq: int, K: int, tau_d: float, force: gs_force | None,
+                     out_tok_ptr: int, out_cnt_ptr: int, out_done_ptr: int,
+                     out_steps_ptr: int = 0) -> None:
+    _check(h, _lib.gs_round_refined(h, slots_ptr, n_seq, K, tau_d,
+                                    ctypes.byref(force) if force is not None else None,
+                                    out_tok_ptr, out_cnt_ptr, out_done_ptr, out_steps_ptr or None))
 
 
 def gs_seq_restore(h, slot: int, seq_len: int, x0: int, n_out: int, max_new: int, done: int,

@@ -94,6 +94,21 @@ class Engine:
         gs.gs_round(self.handle, slots.data_ptr(), slots.shape[0], K, gs.GS_ACCEPT_GREEDY, force,
                     out_tok.data_ptr(), out_cnt.data_ptr(), out_done.data_ptr(), dbg)
 
+    def diffusion_block(self, slots: torch.Tensor, B: int, tau_c: float, out_tok: torch.Tensor,
+                        out_cnt: torch.Tensor, out_done: torch.Tensor,
+                        out_steps: Optional[torch.Tensor] = None) -> None:
+        gs.gs_diffusion_block(self.handle, slots.data_ptr(), slots.shape[0], B, tau_c,
+                              out_tok.data_ptr(), out_cnt.data_ptr(), out_done.data_ptr(),
+                              out_steps.data_ptr() if out_steps is not None else 0)
+
+    def round_refined(self, slots: torch.Tensor, K: int, tau_d: float, out_tok: torch.Tensor,
+                      out_cnt: torch.Tensor, out_done: torch.Tensor,
+                      force: Optional[gs.gs_force] = None,
+                      out_steps: Optional[torch.Tensor] = None) -> None:
+        gs.gs_round_refined(self.handle, slots.data_ptr(), slots.shape[0], K, tau_d, force,
+                            out_tok.data_ptr(), out_cnt.data_ptr(), out_done.data_ptr(),
+                            out_steps.data_ptr() if out_steps is not None else 0)
+
     def round_profile(self, slots: torch.Tensor, K: int, out_tok: torch.Tensor,
                       out_cnt: torch.Tensor, out_done: torch.Tensor,
                       force: Optional[gs.gs_force] = None) -> list:

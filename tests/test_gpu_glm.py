@@ -334,3 +334,23 @@ def test_long_b8_lockstep_forced(glm):
         if A_gpu is not None and stats.near_tie_flips == 0:
             assert A_gpu == A_or == L, (r, L, A_or, A_gpu)
     eng.close()
+
+
+def test_glm_diffusion_blocks_vs_oracle(glm, glm_b1_state):
+    """Direct block diffusion at the GLM scale (prefix 2048, B = 16): two blocks
+    revealed in one step each (tau < 0), then a block revealed one position per
+    step (tau = 2), each block's tokens and steps against the oracle's."""
+    from tests.test_gpu_denoise import diffusion_lockstep
+    w, dec = glm
+    wl = synth.WORKLOADS["glm_b1"]
+    prompt = wl.prompts()[0]
+    eng = new_engine(GLM, w, max_ctx=prompt.length + 700, max_K=16, max_prefill=2048)
+    st, blocks, equal, near = diffusion_lockstep(eng, dec, prompt, 16, -1.0, wl.max_new,
+                                                 max_blocks=2, st=_copy_state(glm_b1_state))
+    print(f"\nGLM diffusion tau<0: {blocks} blocks, {equal} equal, {near} near-margin")
+    assert blocks == 2 and equal + near == 2
+    st, blocks, equal, near = diffusion_lockstep(eng, dec, prompt, 16, 2.0, wl.max_new,
+                                                 max_blocks=1, st=_copy_state(glm_b1_state))
+    print(f"GLM diffusion tau=2: {blocks} blocks, {equal} equal, {near} near-margin")
+    assert blocks == 1 and equal + near == 1
+    eng.close()
