@@ -53,8 +53,13 @@ enum {
 };
 
 /* Acceptance rule (paper Sec. 3 "Speculative Decoding"): greedy accepts drafts
- * while they equal the verifier's argmax; stochastic (rejection sampling) is
- * named by the paper but not used in its experiments -> GS_ERR_UNSUPPORTED. */
+ * while they equal the verifier's argmax; stochastic is the standard
+ * acceptance-rejection rule of speculative sampling, which preserves the
+ * target distribution (named by the paper, not used in its experiments):
+ * a0 and the drafts are sampled at the handle's temperature (gs_set_sampling)
+ * from the draft rows, d_j is accepted while r_j < P_j(d_j) / q_j(d_j), the
+ * first rejected position takes a sample of max(0, P_j - q_j), a fully
+ * accepted draft a bonus sample of P_{K+1}. */
 typedef enum { GS_ACCEPT_GREEDY = 0, GS_ACCEPT_STOCHASTIC = 1 } gs_accept_rule;
 
 /* Decoder shape and capacity.  The paper does not print the architecture; the
@@ -162,8 +167,9 @@ int gs_prefill(gs_handle *h, int slot, const void *vis_emb, int n_vis, const int
  * forward / Verify forward / Accept / Cache update / Next round).
  *   slots    device int32 [n_seq], distinct prefilled slots
  *   K        block size, 0 <= K <= max_K (K = 0 is two plain AR steps)
- *   rule     GS_ACCEPT_GREEDY
- *   force    NULL for natural drafting, else the forcing hook above
+ *   rule     GS_ACCEPT_GREEDY, or GS_ACCEPT_STOCHASTIC (sampling at the
+ *            handle's temperature and seed, see gs_set_sampling)
+ *   force    NULL for natural drafting, else the forcing hook above (greedy only)
  *   out_tok  device int32 [n_seq, K+2]: committed tokens of this round
  *   out_cnt  device int32 [n_seq]: how many (0 for a sequence already done)
  *   out_done device int32 [n_seq]: 1 once the sequence hit EOS or max_new
@@ -172,6 +178,19 @@ int gs_prefill(gs_handle *h, int slot, const void *vis_emb, int n_vis, const int
  * host synchronisation happens inside or between rounds. */
 int gs_round(gs_handle *h, const int32_t *slots, int n_seq, int K, int rule, const gs_force *force,
              int32_t *out_tok, int32_t *out_cnt, int32_t *out_done, const gs_debug *dbg);
+
+/* Sampling parameters of GS_ACCEPT_STOCHASTIC rounds (host values, kept by
+ * the handle).  temperature > 0: tokens are sampled from softmax(logits / T).
+ * seed: the 64-bit key of Philox4x32-10 (Salmon et al., SC 2011), whose
+ * counter is (vocabulary entry / 4, window row, round of the sequence,
+ * stream << 24 | slot); word (entry % 4) x gives the uniform
+ * (2 * (x >> 9) + 1) * 2^-24 and token samples are Gumbel-max
+ * (argmax of log-weight - log(-log u)).  Streams: 0 draft samples (a0, d_j),
+ * 2 acceptance uniforms (row j, entry 0), 3 the replacement or bonus sample
+ * (row j of the rejected position, K+1 for the bonus).  A round's draws thus
+ * depend on the seed, the slot and the sequence's round count only.
+ * Defaults: T = 1, seed = 0.  Errors: GS_ERR_INVALID_ARG. */
+int gs_set_sampling(gs_handle *h, float temperature, uint64_t seed);
 
 /* Direct block-diffusion decoding of one block per sequence (paper Appendix
  * "Direct Block-Diffusion Decoding"; Sec. 5 diffusion-vs-self-speculative

@@ -253,7 +253,7 @@ struct gs_handle {
 
   // graphs keyed by (n_seq, K, pointers)
   typedef std::tuple<int, int, const void*, const void*, long long, const void*, long long,
-                     const void*, const void*, const void*>
+                     const void*, const void*, const void*, long long>
       GraphKey;
   std::map<GraphKey, cudaGraphExec_t> graphs;
   int launches = 0;             // kernel launches counted while enqueueing
@@ -271,6 +271,15 @@ struct gs_handle {
   int lse_tiles = 0;
   cudaStream_t side = nullptr;
   std::map<std::vector<uint64_t>, cudaGraphExec_t> loop_graphs;
+
+  // stochastic rounds: temperature and seed (gs_set_sampling), the two LM
+  // heads' logits and the verify head's softmax partials, the draft rows'
+  // sampling counters
+  float temperature = 1.f;
+  uint64_t seed = 0;
+  float *logits_d = nullptr, *logits_v = nullptr;
+  float2* lse_v = nullptr;
+  uint4* rng_row = nullptr;
 
   // gs_round_profile: an event after every launch and the launch's kind
   bool profiling = false;
@@ -412,6 +421,10 @@ size_t carve(gs_handle* h, const gs_config& c, void* base) {
   int32_t* dn_iter = cv.take<int32_t>(64);
   const int lse_tiles = c.vocab / 128;
   float2* lse_part = cv.take<float2>(static_cast<size_t>(c.max_batch) * W_max * lse_tiles);
+  float2* lse_v = cv.take<float2>(static_cast<size_t>(c.max_batch) * W_max * lse_tiles);
+  float* logits_d = cv.take<float>(static_cast<size_t>(c.max_batch) * W_max * c.vocab);
+  float* logits_v = cv.take<float>(static_cast<size_t>(c.max_batch) * W_max * c.vocab);
+  uint4* rng_row = cv.take<uint4>(static_cast<size_t>(c.max_batch) * W_max);
   // fp16 weight copies: per layer qkv | o | gate_up | down, then the LM head
   const size_t per_layer = static_cast<size_t>(qkv_dim) * c.d_model +
                            static_cast<size_t>(c.d_model) * c.n_heads * 64 +
@@ -469,6 +482,10 @@ size_t carve(gs_handle* h, const gs_config& c, void* base) {
     h->dn_iter = dn_iter;
     h->lse_part = lse_part;
     h->lse_tiles = lse_tiles;
+    h->lse_v = lse_v;
+    h->logits_d = logits_d;
+    h->logits_v = logits_v;
+    h->rng_row = rng_row;
   }
   return align_up(cv.off, 256);
 }
@@ -485,6 +502,7 @@ GemmArgs gemm_base(gs_handle* h) {
   a.inv_d = 1.0f / static_cast<float>(h->cfg.d_model);
   a.eps = h->cfg.rms_eps;
   a.w_scale = 1.f;
+  a.inv_temp = 1.f;
   return a;
 }
 
@@ -558,9 +576,18 @@ int run_attention(gs_handle* h, int layer, int T, const AttnLaunch& L) {
 // `packed`.  Per layer: QKV (+norm scale, RoPE, KV write) -> attention ->
 // O (+residual, next norm's input) -> gate/up (+norm scale, SwiGLU) -> down
 // (+residual, next norm's input).
+// LM-head options of a forward beyond the argmax: softmax partials at a
+// temperature, and Gumbel-max sampling with per-row counters.
+struct LmHeadOpts {
+  float2* lse_part = nullptr;
+  float inv_temp = 1.f;
+  const uint4* rng_row = nullptr;
+  uint64_t seed = 0;
+};
+
 int forward(gs_handle* h, int T, const int32_t* tok, const __nv_bfloat16* vis, int n_vis,
             const AttnLaunch& AL, int lm_row0, int n_lm, unsigned long long* packed,
-            float* logits, bool decode, float2* lse_part = nullptr) {
+            float* logits, bool decode, const LmHeadOpts& lmo = LmHeadOpts()) {
   const gs_config& c = h->cfg;
   const int d = c.d_model, F = c.d_ffn, HD = c.n_heads * 64, L = c.n_layers;
   GS_CUDA(h, launch_ex(embed_kernel, dim3(T), dim3(128), 0, h->stream, h->pdl, dim3(1), tok, h->embed, vis,
@@ -627,7 +654,11 @@ int forward(gs_handle* h, int T, const int32_t* tok, const __nv_bfloat16* vis, i
   lm.N = c.vocab;
   lm.y = packed;
   lm.logits = logits;
-  lm.lse_part = lse_part;
+  lm.lse_part = lmo.lse_part;
+  lm.inv_temp = lmo.inv_temp;
+  lm.rng_row = lmo.rng_row;
+  lm.seed_lo = static_cast<uint32_t>(lmo.seed);
+  lm.seed_hi = static_cast<uint32_t>(lmo.seed >> 32);
   lm.ssp_in = h->ssp;
   lm.x_row0 = lm_row0;
   return run_gemm(h, h->tm_lm, c.vocab, h->tm_hb, d, n_lm, kEpiArgmax, lm, decode,
@@ -635,7 +666,9 @@ int forward(gs_handle* h, int T, const int32_t* tok, const __nv_bfloat16* vis, i
 }
 
 int enqueue_round(gs_handle* h, const int32_t* slots, int n_seq, int K, const gs_force* force,
-                  int32_t* out_tok, int32_t* out_cnt, int32_t* out_done, const gs_debug* dbg) {
+                  int32_t* out_tok, int32_t* out_cnt, int32_t* out_done, const gs_debug* dbg,
+                  int rule = GS_ACCEPT_GREEDY) {
+  const bool stoch = rule == GS_ACCEPT_STOCHASTIC;
   const gs_config& c = h->cfg;
   const int W = K + 1, T = n_seq * W;
   WindowArgs w;
@@ -663,6 +696,7 @@ int enqueue_round(gs_handle* h, const int32_t* slots, int n_seq, int K, const gs
     w.L_stride = force->L_stride;
   }
   w.err = h->err_word;
+  if (stoch) w.rng_row = h->rng_row;
   const int nb = cdiv(T, 128);
   AttnLaunch AL;
   AL.n_seq = n_seq;
@@ -676,14 +710,61 @@ int enqueue_round(gs_handle* h, const int32_t* slots, int n_seq, int K, const gs
   h->launches = 0;
   GS_CUDA(h, launch_ex(window_draft_kernel, dim3(nb), dim3(128), 0, h->stream, h->pdl, dim3(1), w));
   note_launch(h, GS_KIND_WINDOW);
+  // stochastic rounds sample the draft rows and keep both heads' logits and
+  // softmax partials at the temperature for the acceptance test
+  LmHeadOpts lo_d, lo_v;
+  if (stoch) {
+    lo_d.lse_part = h->lse_part;
+    lo_d.inv_temp = lo_v.inv_temp = 1.0f / h->temperature;
+    lo_d.rng_row = h->rng_row;
+    lo_d.seed = h->seed;
+    lo_v.lse_part = h->lse_v;
+  }
   int rc = forward(h, T, h->tok, nullptr, 0, AL, 0, T, h->packed_d,
-                   dbg ? dbg->draft_logits : nullptr, true);
+                   stoch ? h->logits_d : (dbg ? dbg->draft_logits : nullptr), true, lo_d);
   if (rc) return rc;
   GS_CUDA(h, launch_ex(window_verify_kernel, dim3(nb), dim3(128), 0, h->stream, h->pdl, dim3(1), w));
   note_launch(h, GS_KIND_WINDOW);
-  rc = forward(h, T, h->tok, nullptr, 0, AL, 0, T, h->packed_v, dbg ? dbg->verify_logits : nullptr,
-               true);
+  rc = forward(h, T, h->tok, nullptr, 0, AL, 0, T, h->packed_v,
+               stoch ? h->logits_v : (dbg ? dbg->verify_logits : nullptr), true, lo_v);
   if (rc) return rc;
+  if (stoch) {
+    AcceptStochArgs as;
+    memset(&as, 0, sizeof(as));
+    as.slots = slots;
+    as.n_seq = n_seq;
+    as.K = K;
+    as.W = W;
+    as.eos = c.eos_token_id;
+    as.vocab = c.vocab;
+    as.lse_tiles = h->lse_tiles;
+    as.st = h->st;
+    as.verify_in = h->verify_in;
+    as.logits_d = h->logits_d;
+    as.logits_v = h->logits_v;
+    as.lse_d = h->lse_part;
+    as.lse_v = h->lse_v;
+    as.inv_temp = 1.0f / h->temperature;
+    as.seed_lo = static_cast<uint32_t>(h->seed);
+    as.seed_hi = static_cast<uint32_t>(h->seed >> 32);
+    as.verify_tok = h->verify_tok;
+    as.out_tok = out_tok;
+    as.out_cnt = out_cnt;
+    as.out_done = out_done;
+    as.err = h->err_word;
+    GS_CUDA(h, launch_ex(accept_stochastic_kernel, dim3(n_seq), dim3(256), 0, h->stream, h->pdl,
+                         dim3(1), as));
+    note_launch(h, GS_KIND_ACCEPT);
+    if (dbg) {
+      const size_t bytes = static_cast<size_t>(T) * c.vocab * sizeof(float);
+      if (dbg->draft_logits)
+        GS_CUDA(h, cudaMemcpyAsync(dbg->draft_logits, h->logits_d, bytes, cudaMemcpyDeviceToDevice,
+                                   h->stream));
+      if (dbg->verify_logits)
+        GS_CUDA(h, cudaMemcpyAsync(dbg->verify_logits, h->logits_v, bytes,
+                                   cudaMemcpyDeviceToDevice, h->stream));
+    }
+  } else {
   AcceptArgs ac;
   ac.slots = slots;
   ac.n_seq = n_seq;
@@ -700,6 +781,7 @@ int enqueue_round(gs_handle* h, const int32_t* slots, int n_seq, int K, const gs
   GS_CUDA(h, launch_ex(accept_commit_kernel, dim3(cdiv(n_seq, 64)), dim3(64), 0, h->stream, h->pdl, dim3(1),
                        ac));
   note_launch(h, GS_KIND_ACCEPT);
+  }
   if (dbg) {
     if (dbg->draft_tok) copy_i32_kernel<<<nb, 128, 0, h->stream>>>(h->draft_tok, dbg->draft_tok, T);
     if (dbg->verify_in) copy_i32_kernel<<<nb, 128, 0, h->stream>>>(h->verify_in, dbg->verify_in, T);
@@ -836,8 +918,10 @@ int enqueue_denoise_step(gs_handle* h, DenoiseArgs d) {
   GS_CUDA(h, launch_ex(denoise_window_kernel, dim3(cdiv(T, 128)), dim3(128), 0, h->stream, h->pdl,
                        dim3(1), d));
   note_launch(h, GS_KIND_WINDOW);
+  LmHeadOpts lmo;
+  lmo.lse_part = h->lse_part;
   int rc = forward(h, T, h->tok, nullptr, 0, decode_attention(h, d.n_seq, d.W), 0, T, h->packed_d,
-                   nullptr, true, h->lse_part);
+                   nullptr, true, lmo);
   if (rc) return rc;
   GS_CUDA(h, launch_ex(denoise_reveal_kernel, dim3(d.n_seq), dim3(128), 0, h->stream, h->pdl,
                        dim3(1), d));
@@ -1122,9 +1206,10 @@ int gs_round(gs_handle* h, const int32_t* slots, int n_seq, int K, int rule, con
              int32_t* out_tok, int32_t* out_cnt, int32_t* out_done, const gs_debug* dbg) {
   if (!h) return GS_ERR_INVALID_ARG;
   const gs_config& c = h->cfg;
-  if (rule == GS_ACCEPT_STOCHASTIC)
-    return fail(h, GS_ERR_UNSUPPORTED, "stochastic acceptance is not implemented");
-  if (rule != GS_ACCEPT_GREEDY) return fail(h, GS_ERR_INVALID_ARG, "unknown acceptance rule");
+  if (rule != GS_ACCEPT_GREEDY && rule != GS_ACCEPT_STOCHASTIC)
+    return fail(h, GS_ERR_INVALID_ARG, "unknown acceptance rule");
+  if (rule == GS_ACCEPT_STOCHASTIC && force)
+    return fail(h, GS_ERR_INVALID_ARG, "forcing applies to greedy rounds only");
   if (!slots || !out_tok || !out_cnt || !out_done)
     return fail(h, GS_ERR_INVALID_ARG, "null slots or output pointer");
   if (n_seq < 1 || n_seq > c.max_batch) return fail(h, GS_ERR_INVALID_ARG, "n_seq out of range");
@@ -1132,15 +1217,21 @@ int gs_round(gs_handle* h, const int32_t* slots, int n_seq, int K, int rule, con
   if (force && (!force->teacher || !force->L_sched || force->teacher_stride < 1))
     return fail(h, GS_ERR_INVALID_ARG, "incomplete force hook");
   if (dbg || h->stream == nullptr)
-    return enqueue_round(h, slots, n_seq, K, force, out_tok, out_cnt, out_done, dbg);
+    return enqueue_round(h, slots, n_seq, K, force, out_tok, out_cnt, out_done, dbg, rule);
+  // stochastic rounds are keyed by their temperature and seed as well (the
+  // kernels take them as arguments)
+  const long long samp = rule == GS_ACCEPT_STOCHASTIC
+                             ? static_cast<long long>(float_bits(h->temperature)) ^
+                                   static_cast<long long>(h->seed * 0x9E3779B97F4A7C15ull) ^ 1ll
+                             : 0ll;
   gs_handle::GraphKey key(n_seq, K, slots, force ? force->teacher : nullptr,
                           force ? force->teacher_stride : 0, force ? force->L_sched : nullptr,
-                          force ? force->L_stride : 0, out_tok, out_cnt, out_done);
+                          force ? force->L_stride : 0, out_tok, out_cnt, out_done, samp);
   auto it = h->graphs.find(key);
   if (it == h->graphs.end()) {
     cudaGraph_t g;
     GS_CUDA(h, cudaStreamBeginCapture(h->stream, cudaStreamCaptureModeThreadLocal));
-    const int rc = enqueue_round(h, slots, n_seq, K, force, out_tok, out_cnt, out_done, nullptr);
+    const int rc = enqueue_round(h, slots, n_seq, K, force, out_tok, out_cnt, out_done, nullptr, rule);
     cudaError_t e = cudaStreamEndCapture(h->stream, &g);
     if (rc) {
       if (e == cudaSuccess) cudaGraphDestroy(g);
@@ -1306,6 +1397,15 @@ int gs_round_refined(gs_handle* h, const int32_t* slots, int n_seq, int K, float
         },
         ge);
   });
+}
+
+int gs_set_sampling(gs_handle* h, float temperature, uint64_t seed) {
+  if (!h) return GS_ERR_INVALID_ARG;
+  if (!(temperature > 0.f) || !std::isfinite(1.0f / temperature))
+    return fail(h, GS_ERR_INVALID_ARG, "temperature must be positive and finite");
+  h->temperature = temperature;
+  h->seed = seed;
+  return GS_OK;
 }
 
 int gs_seq_restore(gs_handle* h, int slot, int seq_len, int x0, int n_out, int max_new, int done,

@@ -65,8 +65,15 @@ struct GemmArgs {
   int* counters;    // per output tile, zero between launches (cluster == 0)
   float* logits;    // argmax only: optional fp32 [M, N] dump
   // argmax only, optional: per token and 128-row feature tile, (tile max,
-  // sum over the tile of exp(logit - tile max)) at [token][feature tile]
+  // sum over the tile of exp(logit - tile max)) at [token][feature tile],
+  // of the logits times inv_temp
   float2* lse_part;
+  float inv_temp;   // 1 / temperature of the softmax partials and the samples
+  // argmax only, optional: sample instead of argmax (Gumbel-max over
+  // logit * inv_temp, Philox stream kStreamDraft); rng_row[token] =
+  // (unused, window row, round, slot)
+  const uint4* rng_row;
+  uint32_t seed_lo, seed_hi;
   int* err;
   float w_scale;    // 2^-s of the weight copy (1 for unscaled weights)
   int x_row0;       // X (and ssp_in) row of token 0
@@ -105,8 +112,9 @@ struct GemmShape {
   static_assert(!(BN <= 64) || kXBufBytes + kRedBytes <= kStagesMin * kStageBytes,
                 "cluster staging smem");
   // argmax epilogue: keys [128][33] and quarter maxima [4][32], 8 bytes each,
-  // then the softmax partials' tile maxima [32] and warp sums [4][32], 4 bytes each
-  static_assert((128 * 33 + 4 * 32) * 8 + 5 * 32 * 4 <= kStagesMin * kStageBytes, "argmax smem");
+  // then the softmax partials' tile maxima [32] and warp maxima and sums
+  // [2][4][32], 4 bytes each
+  static_assert((128 * 33 + 4 * 32) * 8 + 9 * 32 * 4 <= kStagesMin * kStageBytes, "argmax smem");
   // RoPE cos/sin rows of the tile's tokens, staged while the mainloop runs
   // (QKV launches, decode tiles)
   static constexpr bool kStageRope = BN <= 64;
@@ -299,8 +307,22 @@ __device__ __forceinline__ void gemm_epilogue_chunk(const GemmArgs& a, float (&v
     // warp the max over the four quarters: one atomicMax per token per CTA
     unsigned long long* kb = reinterpret_cast<unsigned long long*>(xbuf);
     constexpr int LD = EW + 1;
+    if (a.rng_row != nullptr) {
+      // sample: argmax of logit / T + Gumbel noise of this (row, vocabulary entry)
 #pragma unroll
-    for (int j = 0; j < EW; ++j) kb[row * LD + j] = argmax_key(v[j], f);
+      for (int j = 0; j < EW; ++j) {
+        float sc = -INFINITY;
+        if (j >= jlo && j < jhi) {
+          const uint4 c = a.rng_row[t0 + j];
+          sc = v[j] * a.inv_temp +
+               gumbel_of(philox_uniform(a.seed_lo, a.seed_hi, c.w, c.z, kStreamDraft, c.y, f));
+        }
+        kb[row * LD + j] = argmax_key(sc, f);
+      }
+    } else {
+#pragma unroll
+      for (int j = 0; j < EW; ++j) kb[row * LD + j] = argmax_key(v[j], f);
+    }
     asm volatile("bar.sync 2, 128;" ::: "memory");
     unsigned long long* qb = kb + 128 * LD;   // [4][EW] quarter maxima
     if (threadIdx.x < 4 * EW) {
@@ -313,24 +335,38 @@ __device__ __forceinline__ void gemm_epilogue_chunk(const GemmArgs& a, float (&v
       qb[q * EW + j] = best;
     }
     asm volatile("bar.sync 2, 128;" ::: "memory");
-    float* tmax = reinterpret_cast<float*>(qb + 4 * EW);   // [EW] tile maxima
     if (threadIdx.x < EW) {
       const int j = threadIdx.x;
       unsigned long long best = qb[j];
 #pragma unroll
       for (int q = 1; q < 4; ++q) best = qb[q * EW + j] > best ? qb[q * EW + j] : best;
       if (j >= jlo && j < jhi) atomicMax(out + t0 + j, best);
-      tmax[j] = argmax_key_value(best);
     }
     asm volatile("bar.sync 2, 128;" ::: "memory");
     if (a.lse_part != nullptr) {
-      // softmax partials of this tile: sum over its 128 rows of exp(v - tile
-      // max), a warp tree then the four warps in order (fixed order: the same
-      // bits for a row whatever the batch)
-      float* wsum = tmax + EW;   // [4][EW]
+      // softmax partials of this tile over logit / T: the tile max (warp tree,
+      // then the four warps), then the sum over its 128 rows of exp(x - max),
+      // a warp tree then the four warps in order (fixed order: the same bits
+      // for a row whatever the batch)
+      float* tmax = reinterpret_cast<float*>(qb + 4 * EW);   // [EW]
+      float* wmax = tmax + EW;                               // [4][EW]
+      float* wsum = wmax + 4 * EW;                           // [4][EW]
 #pragma unroll
       for (int j = 0; j < EW; ++j) {
-        float e = expf(v[j] - tmax[j]);
+        float m = v[j] * a.inv_temp;
+#pragma unroll
+        for (int o = 16; o >= 1; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xFFFFFFFFu, m, o));
+        if (lane == 0) wmax[warp * EW + j] = m;
+      }
+      asm volatile("bar.sync 2, 128;" ::: "memory");
+      if (threadIdx.x < EW) {
+        const int j = threadIdx.x;
+        tmax[j] = fmaxf(fmaxf(wmax[j], wmax[EW + j]), fmaxf(wmax[2 * EW + j], wmax[3 * EW + j]));
+      }
+      asm volatile("bar.sync 2, 128;" ::: "memory");
+#pragma unroll
+      for (int j = 0; j < EW; ++j) {
+        float e = expf(v[j] * a.inv_temp - tmax[j]);
 #pragma unroll
         for (int m = 16; m >= 1; m >>= 1) e += __shfl_xor_sync(0xFFFFFFFFu, e, m);
         if (lane == 0) wsum[warp * EW + j] = e;

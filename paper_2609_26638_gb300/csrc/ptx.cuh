@@ -298,6 +298,45 @@ __device__ __forceinline__ __half to_f16(float x, int* err) {
   return __float2half_rn(x);
 }
 
+// ---------------------------------------------------------------- sampling
+// Philox4x32-10 (Salmon, Moraes, Dror and Shaw, "Parallel random numbers: as
+// easy as 1, 2, 3", SC 2011): ten rounds of two 32x32 -> 64-bit products with
+// the round multipliers, the counter words permuted and xored with the key,
+// the key advanced by the Weyl increments between rounds.
+__host__ __device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint32_t k0, uint32_t k1) {
+  constexpr uint32_t kM0 = 0xD2511F53u, kM1 = 0xCD9E8D57u;
+  constexpr uint32_t kW0 = 0x9E3779B9u, kW1 = 0xBB67AE85u;
+#pragma unroll
+  for (int r = 0; r < 10; ++r) {
+    const uint64_t p0 = static_cast<uint64_t>(kM0) * c.x;
+    const uint64_t p1 = static_cast<uint64_t>(kM1) * c.z;
+    const uint32_t hi0 = static_cast<uint32_t>(p0 >> 32), lo0 = static_cast<uint32_t>(p0);
+    const uint32_t hi1 = static_cast<uint32_t>(p1 >> 32), lo1 = static_cast<uint32_t>(p1);
+    c = make_uint4(hi1 ^ c.y ^ k0, lo1, hi0 ^ c.w ^ k1, lo0);
+    k0 += kW0;
+    k1 += kW1;
+  }
+  return c;
+}
+
+// Random streams of a stochastic round (the oracle uses the same numbering).
+enum : uint32_t { kStreamDraft = 0, kStreamAccept = 2, kStreamSample = 3 };
+
+// Uniform for vocabulary entry v of (seed, slot, round, stream, row):
+// word v % 4 of Philox at counter (v / 4, row, round, stream << 24 | slot),
+// mapped to (2 * (x >> 9) + 1) * 2^-24, exact in float32, in (0, 1).
+__device__ __forceinline__ float philox_uniform(uint32_t seed_lo, uint32_t seed_hi, uint32_t slot,
+                                                uint32_t rnd, uint32_t stream, uint32_t row,
+                                                uint32_t v) {
+  const uint4 w = philox4x32_10(make_uint4(v >> 2, row, rnd, (stream << 24) | slot), seed_lo, seed_hi);
+  const uint32_t x = (v & 3) == 0 ? w.x : ((v & 3) == 1 ? w.y : ((v & 3) == 2 ? w.z : w.w));
+  return __uint2float_rn(((x >> 9) << 1) | 1u) * 5.9604644775390625e-08f;
+}
+
+// Gumbel noise -log(-log u): added to log-weights, the argmax samples an
+// entry with probability proportional to its weight (Gumbel-max).
+__device__ __forceinline__ float gumbel_of(float u) { return -logf(-logf(u)); }
+
 // ---------------------------------------------------------------- misc
 // Total order on floats as unsigned keys (larger float -> larger key).
 __device__ __forceinline__ uint32_t float_order_key(float v) {

@@ -43,6 +43,9 @@ struct WindowArgs {
   int fixed_stride;
   const int32_t* steps_src;
   int32_t* steps_out;
+  // stochastic rounds: per draft row, the sampling counter words
+  // (unused, window row, round, slot) read by the LM head
+  uint4* rng_row;
 };
 
 // Draft window: [x0, [M] x K] at slots n..n+K; row 0 sees keys 0..n, mask rows 0..n+K.
@@ -59,6 +62,9 @@ __global__ void window_draft_kernel(WindowArgs a) {
   a.pos[idx] = n + i;
   a.lim[idx] = i == 0 ? n : n + a.K;
   a.tok_slot[idx] = active ? slot : -1;
+  if (a.rng_row != nullptr)
+    a.rng_row[idx] = make_uint4(0u, static_cast<uint32_t>(i), static_cast<uint32_t>(a.st.rounds[slot]),
+                                static_cast<uint32_t>(slot));
   if (i == 0) {
     a.blk_slot[b] = slot;
     a.blk_active[b] = active ? 1 : 0;
@@ -153,6 +159,162 @@ __global__ void accept_commit_kernel(AcceptArgs a) {
   }
   a.st.seq_len[slot] = a.st.seq_len[slot] + A + 2;
   a.st.x0[slot] = vt[A];
+  a.st.n_out[slot] = n_out;
+  a.st.done[slot] = done;
+  a.st.rounds[slot] = a.st.rounds[slot] + 1;
+  a.out_cnt[b] = cnt;
+  a.out_done[b] = done;
+}
+
+// Stochastic acceptance (paper Sec. 3 "Speculative Decoding": the standard
+// acceptance-rejection rule, which preserves the target distribution).  The
+// draft forward sampled a0 from the causal boundary row and d_j from mask row
+// j (draft distribution q_j); the verify forward's row j-1 is the target P_j
+// of the token at d_j's slot.  With logits dumped by both LM heads and their
+// softmax partials at temperature T:
+//   P_j(d_j) = exp(lv[j-1][d_j] / T - lse_v[j-1]),  q_j(d_j) = exp(ld[j][d_j] / T - lse_d[j]);
+//   d_j is accepted while r_j * q_j(d_j) < P_j(d_j) (r_j: stream kStreamAccept,
+//   row j, word 0 of group 0); at the first rejection j the next token is the
+//   Gumbel-max sample of max(0, P_j - q_j) (stream kStreamSample, row j), after
+//   K acceptances of P_{K+1} (row K+1).
+// Commit a0, d_1..d_A and that token (EOS / cap cut), seq_len <- n + A + 2.
+// One CTA of 256 threads per sequence.
+struct AcceptStochArgs {
+  const int32_t* slots;
+  int n_seq, K, W, eos, vocab, lse_tiles;
+  SeqStateDev st;
+  const int32_t* verify_in;     // [n_seq * W] a0, d_1..d_K
+  const float* logits_d;        // [n_seq * W, vocab]
+  const float* logits_v;        // [n_seq * W, vocab]
+  const float2* lse_d;          // [n_seq * W, lse_tiles] partials of logit / T
+  const float2* lse_v;
+  float inv_temp;
+  uint32_t seed_lo, seed_hi;
+  int32_t* verify_tok;          // [n_seq * W] diagnostics: the sampled next tokens
+  int32_t* out_tok;
+  int32_t* out_cnt;
+  int32_t* out_done;
+  int* err;
+};
+
+__device__ __forceinline__ float row_lse(const float2* part, int tiles, float* red) {
+  // log-sum-exp of one row from its tile partials: max over tiles, then the
+  // rescaled sums, each reduced in a fixed order (thread-strided, then a tree)
+  float m = -INFINITY;
+  for (int t = threadIdx.x; t < tiles; t += blockDim.x) m = fmaxf(m, part[t].x);
+  red[threadIdx.x] = m;
+  __syncthreads();
+  for (int o = blockDim.x / 2; o >= 1; o >>= 1) {
+    if (threadIdx.x < o) red[threadIdx.x] = fmaxf(red[threadIdx.x], red[threadIdx.x + o]);
+    __syncthreads();
+  }
+  const float M = red[0];
+  __syncthreads();
+  float s = 0.f;
+  for (int t = threadIdx.x; t < tiles; t += blockDim.x) s += part[t].y * expf(part[t].x - M);
+  red[threadIdx.x] = s;
+  __syncthreads();
+  for (int o = blockDim.x / 2; o >= 1; o >>= 1) {
+    if (threadIdx.x < o) red[threadIdx.x] += red[threadIdx.x + o];
+    __syncthreads();
+  }
+  const float r = M + logf(red[0]);
+  __syncthreads();
+  return r;
+}
+
+__global__ void __launch_bounds__(256) accept_stochastic_kernel(AcceptStochArgs a) {
+  __shared__ float red[256];
+  __shared__ unsigned long long bestk[256];
+  __shared__ float lse_v_s[257], lse_d_s[257];
+  __shared__ int A_s;
+  pdl_wait();
+  pdl_trigger();
+  const int b = blockIdx.x;
+  if (b >= a.n_seq) return;
+  const int slot = a.slots[b];
+  const int K = a.K, W = a.W;
+  if (a.st.done[slot]) {
+    if (threadIdx.x == 0) {
+      a.out_cnt[b] = 0;
+      a.out_done[b] = 1;
+    }
+    return;
+  }
+  const uint32_t rnd = static_cast<uint32_t>(a.st.rounds[slot]);
+  const int row0 = b * W;
+  for (int i = 0; i <= K; ++i) {
+    const float lv = row_lse(a.lse_v + static_cast<size_t>(row0 + i) * a.lse_tiles, a.lse_tiles, red);
+    const float ld = row_lse(a.lse_d + static_cast<size_t>(row0 + i) * a.lse_tiles, a.lse_tiles, red);
+    if (threadIdx.x == 0) {
+      lse_v_s[i] = lv;
+      lse_d_s[i] = ld;
+    }
+  }
+  __syncthreads();
+  const int* vin = a.verify_in + row0;   // a0, d_1..d_K
+  if (threadIdx.x == 0) {
+    int A = 0;
+    while (A < K) {
+      const int j = A + 1, dj = vin[j];
+      const float P = expf(a.logits_v[static_cast<size_t>(row0 + j - 1) * a.vocab + dj] * a.inv_temp -
+                           lse_v_s[j - 1]);
+      const float q = expf(a.logits_d[static_cast<size_t>(row0 + j) * a.vocab + dj] * a.inv_temp -
+                           lse_d_s[j]);
+      const float r = philox_uniform(a.seed_lo, a.seed_hi, slot, rnd, kStreamAccept, j, 0);
+      if (!(r * q < P)) break;
+      ++A;
+    }
+    A_s = A;
+  }
+  __syncthreads();
+  const int A = A_s;
+  // the next token: Gumbel-max over max(0, P_j - q_j) (rejection at j = A+1)
+  // or over P_{K+1}; entries with zero weight never win; ties to the lowest id
+  const bool bonus = A == K;
+  const int j = A + 1;
+  const float* lv = a.logits_v + static_cast<size_t>(row0 + j - 1) * a.vocab;
+  const float* ld = bonus ? nullptr : a.logits_d + static_cast<size_t>(row0 + j) * a.vocab;
+  const float lsev = lse_v_s[j - 1], lsed = bonus ? 0.f : lse_d_s[j];
+  unsigned long long best = 0;
+  for (int v = threadIdx.x; v < a.vocab; v += blockDim.x) {
+    float w = expf(lv[v] * a.inv_temp - lsev);
+    if (!bonus) w = fmaxf(w - expf(ld[v] * a.inv_temp - lsed), 0.f);
+    if (w > 0.f) {
+      const float sc = logf(w) + gumbel_of(philox_uniform(a.seed_lo, a.seed_hi, slot, rnd,
+                                                          kStreamSample, j, v));
+      const unsigned long long k = argmax_key(sc, static_cast<uint32_t>(v));
+      best = k > best ? k : best;
+    }
+  }
+  bestk[threadIdx.x] = best;
+  __syncthreads();
+  for (int o = blockDim.x / 2; o >= 1; o >>= 1) {
+    if (threadIdx.x < o && bestk[threadIdx.x + o] > bestk[threadIdx.x])
+      bestk[threadIdx.x] = bestk[threadIdx.x + o];
+    __syncthreads();
+  }
+  if (threadIdx.x != 0) return;
+  int tok = bestk[0] == 0 ? -1 : argmax_key_index(bestk[0]);
+  if (tok < 0 || tok >= a.vocab) {   // no positive weight: cannot happen for a distribution
+    atomicExch(a.err, kErrBounds);
+    tok = 0;
+  }
+  for (int i = 0; i < W; ++i) a.verify_tok[row0 + i] = i == A ? tok : -1;
+  int n_out = a.st.n_out[slot];
+  const int cap = a.st.max_new[slot];
+  int cnt = 0, done = 0;
+  for (int i = 0; i < A + 2; ++i) {
+    const int t = i <= A ? vin[i] : tok;
+    a.out_tok[b * (K + 2) + cnt++] = t;
+    ++n_out;
+    if (t == a.eos || n_out >= cap) {
+      done = 1;
+      break;
+    }
+  }
+  a.st.seq_len[slot] = a.st.seq_len[slot] + A + 2;
+  a.st.x0[slot] = tok;
   a.st.n_out[slot] = n_out;
   a.st.done[slot] = done;
   a.st.rounds[slot] = a.st.rounds[slot] + 1;

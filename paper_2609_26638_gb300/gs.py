@@ -80,6 +80,7 @@ def _load():
         "gs_round": (i32, [vp, vp, i32, i32, i32, ctypes.POINTER(gs_force), vp, vp, vp,
                            ctypes.POINTER(gs_debug)]),
         "gs_seq_restore": (i32, [vp, i32, i32, i32, i32, i32, i32, i32]),
+        "gs_set_sampling": (i32, [vp, ctypes.c_float, ctypes.c_uint64]),
         "gs_diffusion_block": (i32, [vp, vp, i32, i32, ctypes.c_float, vp, vp, vp, vp]),
         "gs_round_refined": (i32, [vp, vp, i32, i32, ctypes.c_float, ctypes.POINTER(gs_force), vp,
                                    vp, vp, vp]),
@@ -108,7 +109,7 @@ def _load():
 
 _lib = _load()
 EXPORTED = ("gs_workspace_bytes", "gs_create", "gs_destroy", "gs_last_error", "gs_prefill",
-            "gs_round", "gs_diffusion_block", "gs_round_refined", "gs_seq_restore", "gs_round_launches", "gs_round_profile", "gs_seq_state",
+            "gs_round", "gs_set_sampling", "gs_diffusion_block", "gs_round_refined", "gs_seq_restore", "gs_round_launches", "gs_round_profile", "gs_seq_state",
             "gs_release", "gs_sync_check", "gs_wait_probe",
             "gs_attention_scratch_bytes", "gs_attention", "gs_linear_scratch_bytes", "gs_linear",
             "gs_linear_noalloc", "gs_linear_noalloc_status")
@@ -158,6 +159,10 @@ def gs_round(h, slots_ptr: int, n_seq: int, K: int, rule: int, force: gs_force |
                             ctypes.byref(force) if force is not None else None,
                             out_tok_ptr, out_cnt_ptr, out_done_ptr,
                             ctypes.byref(dbg) if dbg is not None else None))
+
+
+def gs_set_sampling(h, temperature: float, seed: int) -> None:
+    _check(h, _lib.gs_set_sampling(h, temperature, seed))
 
 
 def gs_diffusion_block(h, slots_ptr: int, n_seq: int, B: int, tau_c: float, out_tok_ptr: int,

@@ -90,9 +90,12 @@ class Engine:
 
     def round(self, slots: torch.Tensor, K: int, out_tok: torch.Tensor, out_cnt: torch.Tensor,
               out_done: torch.Tensor, force: Optional[gs.gs_force] = None,
-              dbg: Optional[gs.gs_debug] = None) -> None:
-        gs.gs_round(self.handle, slots.data_ptr(), slots.shape[0], K, gs.GS_ACCEPT_GREEDY, force,
+              dbg: Optional[gs.gs_debug] = None, rule: int = gs.GS_ACCEPT_GREEDY) -> None:
+        gs.gs_round(self.handle, slots.data_ptr(), slots.shape[0], K, rule, force,
                     out_tok.data_ptr(), out_cnt.data_ptr(), out_done.data_ptr(), dbg)
+
+    def set_sampling(self, temperature: float, seed: int) -> None:
+        gs.gs_set_sampling(self.handle, temperature, seed)
 
     def diffusion_block(self, slots: torch.Tensor, B: int, tau_c: float, out_tok: torch.Tensor,
                         out_cnt: torch.Tensor, out_done: torch.Tensor,

@@ -354,3 +354,20 @@ def test_glm_diffusion_blocks_vs_oracle(glm, glm_b1_state):
     print(f"GLM diffusion tau=2: {blocks} blocks, {equal} equal, {near} near-margin")
     assert blocks == 1 and equal + near == 1
     eng.close()
+
+
+def test_glm_stochastic_rounds_vs_oracle(glm, glm_b1_state):
+    """Stochastic rounds (T = 1, the standard acceptance-rejection rule) at the
+    GLM scale: sampled drafts, acceptance, the replacement or bonus sample and
+    the logits of three rounds against the oracle's same Philox draws."""
+    from tests.test_gpu_sampling import stochastic_lockstep
+    w, dec = glm
+    wl = synth.WORKLOADS["glm_b1"]
+    prompt = wl.prompts()[0]
+    eng = new_engine(GLM, w, max_ctx=prompt.length + 700, max_K=16, max_prefill=2048)
+    st, rounds, equal, near = stochastic_lockstep(eng, dec, prompt, 16, 1.0, 2024, wl.max_new,
+                                                  check_logits=True, st=_copy_state(glm_b1_state),
+                                                  max_rounds=3)
+    print(f"\nGLM stochastic: {rounds} rounds, {equal} equal, {near} near-margin")
+    assert rounds == 3 and equal + near == 3
+    eng.close()

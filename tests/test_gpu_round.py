@@ -156,10 +156,18 @@ def test_bad_requests_raise(tiny):
     with pytest.raises(gs.GsError) as e:
         eng.round(slots, 5, o, c, d)                         # K > max_K
     assert e.value.code == gs.GS_ERR_INVALID_ARG
-    with pytest.raises(gs.GsError) as e:
-        gs.gs_round(eng.handle, slots.data_ptr(), 1, 2, gs.GS_ACCEPT_STOCHASTIC, None,
+    force = gs.gs_force(teacher=o.data_ptr(), teacher_stride=8, L_sched=c.data_ptr(), L_stride=1)
+    with pytest.raises(gs.GsError) as e:                     # forcing is a greedy-only hook
+        gs.gs_round(eng.handle, slots.data_ptr(), 1, 2, gs.GS_ACCEPT_STOCHASTIC, force,
                     o.data_ptr(), c.data_ptr(), d.data_ptr())
-    assert e.value.code == gs.GS_ERR_UNSUPPORTED
+    assert e.value.code == gs.GS_ERR_INVALID_ARG
+    with pytest.raises(gs.GsError) as e:
+        gs.gs_round(eng.handle, slots.data_ptr(), 1, 2, 7, None, o.data_ptr(), c.data_ptr(),
+                    d.data_ptr())
+    assert e.value.code == gs.GS_ERR_INVALID_ARG
+    with pytest.raises(gs.GsError) as e:
+        eng.set_sampling(0.0, 1)
+    assert e.value.code == gs.GS_ERR_INVALID_ARG
     p = synth.make_prompt(cfg, 200, 10)
     with pytest.raises(gs.GsError) as e:
         eng.prefill(0, p.vis, p.text, 100)                   # 210 + 100 + 6 > 256
