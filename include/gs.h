@@ -357,7 +357,8 @@ int gs_attention(int mode, const void *q, const void *kv, int n_pages, const int
  *   first int32 is the kernel's error word after the stream reaches the end
  *   of the call (0 = no failure, 1 = bounds check, 2 = bounded wait ran out,
  *   3 = a value beyond the fp16 range).
- *   Requirements: K % 64 == 0, N % 128 == 0 (N % 64 for epilogue 2), M >= 1. */
+ *   Requirements: K % 64 == 0, N % 128 == 0 (N % 64 for epilogue 2), M >= 1;
+ *   x, w and y 16-byte aligned. */
 size_t gs_linear_scratch_bytes(int M, int N, int split_k);
 int gs_linear(const void *x, const void *w, void *y, int M, int N, int K, int epilogue, int split_k,
               void *scratch, size_t scratch_bytes, void *stream);

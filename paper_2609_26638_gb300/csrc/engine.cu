@@ -155,11 +155,11 @@ int decode_splits(int weight_rows, int K) {
 
 // Decode windows of up to 64 tokens split K across the CTAs of a cluster.
 // Wider decode launches with at least 8 k-blocks per split keep that (64-token
-// tiles); the others reduce the same K chunks inside each CTA (one TMEM
-// accumulator per chunk, summed in chunk order), with the chunks'
-// accumulators in at most 256 TMEM columns, so two CTAs share an SM, and the
-// token tile shrunk until the launch covers about one wave.  All three give
-// the same sums in the same order.  Prefill does not split K.
+// tiles); the others reduce the same K chunks inside each CTA
+// (gemm_chunk_kernel: each chunk summed from zero in a TMEM buffer, then added
+// in chunk order to a running sum in TMEM), with the token tile the widest of
+// 128 / 64 / 32 with the fewest waves x operand bytes per CTA.  All three
+// give the same sums in the same order.  Prefill does not split K.
 GemmPlan plan_split(int weight_rows, int T, int S, int nkb) {
   GemmPlan p;
   p.feat_tiles = weight_rows / 128;
@@ -168,11 +168,22 @@ GemmPlan plan_split(int weight_rows, int T, int S, int nkb) {
   p.bn = gemm_bn_for(T);
   if (S > 1 && T > 64 && nkb / S >= 8 && gemm_cluster_ok(64, S)) {
     p.bn = 64;
-  } else if (S > 1 && T > 64 && S * 32 <= 256) {
+  } else if (S > 1 && T > 64) {
+    // chunked K inside each CTA (gemm_chunk_kernel, two CTAs per SM).  A CTA
+    // streams K x (128 + BN) operand bytes, and the launch takes ceil(CTAs /
+    // slots) rounds of them: pick the token tile of 128 / 64 / 32 with the
+    // least waves x (128 + BN), the wider on a tie.
     p.chunks = S;
     p.splits = 1;
-    p.bn = std::min(128, 256 / S);
-    while (p.bn > 32 && p.feat_tiles * cdiv(T, p.bn) < 148) p.bn /= 2;
+    long best = -1;
+    for (int bn : {128, 64, 32}) {
+      const long waves = cdiv(static_cast<long long>(p.feat_tiles) * cdiv(T, bn), 2 * kNumSMs);
+      const long cost = waves * (128 + bn);
+      if (best < 0 || cost < best) {
+        best = cost;
+        p.bn = bn;
+      }
+    }
   }
   p.tok_tiles = cdiv(T, p.bn);
   return p;
@@ -1651,7 +1662,8 @@ int gs_linear(const void* x, const void* w, void* y, int M, int N, int K, int ep
   if (epilogue == kEpiSwiGLU ? (N % 64) : (N % 128)) return GS_ERR_INVALID_ARG;
   if (M > 65536) return GS_ERR_UNSUPPORTED;
   if (scratch_bytes < gs_linear_scratch_bytes(M, N, split_k)) return GS_ERR_OOM;
-  if ((reinterpret_cast<uintptr_t>(x) & 15) || (reinterpret_cast<uintptr_t>(w) & 15))
+  if ((reinterpret_cast<uintptr_t>(x) & 15) || (reinterpret_cast<uintptr_t>(w) & 15) ||
+      (reinterpret_cast<uintptr_t>(y) & 15))
     return GS_ERR_INVALID_ARG;
   if (ensure_kernel_attributes() != cudaSuccess) return GS_ERR_CUDA;
   // split-K as the decoder plans it: across the CTAs of a cluster (up to 64

@@ -28,15 +28,38 @@ static cudaError_t launch_one(const CUtensorMap& tmW, const CUtensorMap& tmX, Ge
                    pdl, dim3(1, 1, cz), tmW, tmX, a);
 }
 
+// Chunked-K launches (wide decode windows): two CTAs per SM, the deepest
+// pipeline that still fits them, never more stages than k-blocks.
+template <int BN, int EPI>
+static cudaError_t launch_chunk_one(const CUtensorMap& tmW, const CUtensorMap& tmX, GemmArgs a,
+                                    int feat_tiles, int tok_tiles, cudaStream_t s, bool pdl) {
+  using S = GemmShape<BN>;
+  const int want = S::stages_fitting(2, EPI, false);
+  const int kb = a.K / 64;
+  a.stages = kb < S::kStagesMin ? S::kStagesMin : (kb > want ? want : kb);
+  dim3 grid(tok_tiles, feat_tiles, 1);
+  return launch_ex(gemm_chunk_kernel<BN, EPI>, grid, dim3(192), S::smem_bytes(a.stages, EPI, false),
+                   s, pdl, dim3(1, 1, 1), tmW, tmX, a);
+}
+
+template <int BN, int EPI>
+static cudaError_t launch_one_or_chunk(const CUtensorMap& tmW, const CUtensorMap& tmX,
+                                       const GemmArgs& a, int ft, int tt, cudaStream_t s, bool pdl) {
+  if constexpr (BN <= 128) {
+    if (a.chunks > 1 && a.splits == 1) return launch_chunk_one<BN, EPI>(tmW, tmX, a, ft, tt, s, pdl);
+  }
+  return launch_one<BN, EPI>(tmW, tmX, a, ft, tt, s, pdl);
+}
+
 template <int BN>
 static cudaError_t launch_bn(int epi, const CUtensorMap& tmW, const CUtensorMap& tmX,
                              const GemmArgs& a, int ft, int tt, cudaStream_t s, bool pdl) {
   switch (epi) {
-    case kEpiStoreF16: return launch_one<BN, kEpiStoreF16>(tmW, tmX, a, ft, tt, s, pdl);
-    case kEpiResidF32: return launch_one<BN, kEpiResidF32>(tmW, tmX, a, ft, tt, s, pdl);
-    case kEpiSwiGLU: return launch_one<BN, kEpiSwiGLU>(tmW, tmX, a, ft, tt, s, pdl);
-    case kEpiArgmax: return launch_one<BN, kEpiArgmax>(tmW, tmX, a, ft, tt, s, pdl);
-    case kEpiQKV: return launch_one<BN, kEpiQKV>(tmW, tmX, a, ft, tt, s, pdl);
+    case kEpiStoreF16: return launch_one_or_chunk<BN, kEpiStoreF16>(tmW, tmX, a, ft, tt, s, pdl);
+    case kEpiResidF32: return launch_one_or_chunk<BN, kEpiResidF32>(tmW, tmX, a, ft, tt, s, pdl);
+    case kEpiSwiGLU: return launch_one_or_chunk<BN, kEpiSwiGLU>(tmW, tmX, a, ft, tt, s, pdl);
+    case kEpiArgmax: return launch_one_or_chunk<BN, kEpiArgmax>(tmW, tmX, a, ft, tt, s, pdl);
+    case kEpiQKV: return launch_one_or_chunk<BN, kEpiQKV>(tmW, tmX, a, ft, tt, s, pdl);
   }
   return cudaErrorInvalidValue;
 }
@@ -54,9 +77,32 @@ cudaError_t launch_gemm(int bn, int epi, const CUtensorMap& tmW, const CUtensorM
 }
 
 template <int BN>
+static cudaError_t set_attr_chunk() {
+  const int bytes = GemmShape<BN>::kSmemMax;
+  cudaError_t e;
+  if ((e = cudaFuncSetAttribute(gemm_chunk_kernel<BN, kEpiStoreF16>,
+                                cudaFuncAttributeMaxDynamicSharedMemorySize, bytes)) != cudaSuccess)
+    return e;
+  if ((e = cudaFuncSetAttribute(gemm_chunk_kernel<BN, kEpiResidF32>,
+                                cudaFuncAttributeMaxDynamicSharedMemorySize, bytes)) != cudaSuccess)
+    return e;
+  if ((e = cudaFuncSetAttribute(gemm_chunk_kernel<BN, kEpiSwiGLU>,
+                                cudaFuncAttributeMaxDynamicSharedMemorySize, bytes)) != cudaSuccess)
+    return e;
+  if ((e = cudaFuncSetAttribute(gemm_chunk_kernel<BN, kEpiArgmax>,
+                                cudaFuncAttributeMaxDynamicSharedMemorySize, bytes)) != cudaSuccess)
+    return e;
+  return cudaFuncSetAttribute(gemm_chunk_kernel<BN, kEpiQKV>,
+                              cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+}
+
+template <int BN>
 static cudaError_t set_attr_bn() {
   const int bytes = GemmShape<BN>::kSmemMax;
   cudaError_t e;
+  if constexpr (BN <= 128) {
+    if ((e = set_attr_chunk<BN>()) != cudaSuccess) return e;
+  }
   if ((e = cudaFuncSetAttribute(gemm_tc_kernel<BN, kEpiStoreF16>,
                                 cudaFuncAttributeMaxDynamicSharedMemorySize, bytes)) != cudaSuccess)
     return e;

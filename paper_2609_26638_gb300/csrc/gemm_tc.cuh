@@ -111,6 +111,8 @@ struct GemmShape {
   static constexpr int kXBufBytes = 32 * 128 * 4;  // epilogue exchange (SwiGLU, RoPE, sums)
   static_assert(!(BN <= 64) || kXBufBytes + kRedBytes <= kStagesMin * kStageBytes,
                 "cluster staging smem");
+  // transposed epilogue slice [32][132] fp32 and per-token partial sums [32][16]
+  static_assert((32 * 132 + 32 * 16) * 4 <= kStagesMin * kStageBytes, "epilogue slice smem");
   // argmax epilogue: keys [128][33] and quarter maxima [4][32], 8 bytes each,
   // then the softmax partials' tile maxima [32] and warp maxima and sums
   // [2][4][32], 4 bytes each
@@ -159,6 +161,28 @@ struct TokMeta {
 // Epilogue of EW consecutive token slots t0 .. t0+EW-1 of feature row `row`;
 // slots q in [jlo, jhi) with t0 + q < M are produced.  Split CTAs own at most
 // 8 tokens and use EW = 8; whole tiles use EW = 32.
+// Eight fp32 values -> eight fp16 bit patterns in one 16-byte word; `bad` is
+// raised for a value beyond the fp16 range or a NaN (no branch per value).
+__device__ __forceinline__ uint4 pack8_f16(const float (&x)[8], bool& bad) {
+  uint32_t w[4];
+#pragma unroll
+  for (int e = 0; e < 4; ++e) {
+    bad |= !(fabsf(x[2 * e]) <= 65504.0f) || !(fabsf(x[2 * e + 1]) <= 65504.0f);
+    __half2 h = __floats2half2_rn(x[2 * e], x[2 * e + 1]);
+    w[e] = *reinterpret_cast<uint32_t*>(&h);
+  }
+  return make_uint4(w[0], w[1], w[2], w[3]);
+}
+
+// Epilogue of EW consecutive token slots t0 .. t0+EW-1 of the 128 rows of one
+// feature tile; thread `row` (0..127, the four epilogue warps) holds row
+// `row` of those tokens in v.  Slots q in [jlo, jhi) with t0 + q < M are
+// produced.  Split CTAs own at most 8 tokens and use EW = 8; whole tiles use
+// EW = 32.  The slice is first transposed through shared memory (xs[token][row],
+// row stride 132 floats), then each work item -- one token and 8 consecutive
+// rows -- reads, computes and writes 16-byte vectors, so global traffic is
+// contiguous.  A value's arithmetic is the same for every EW and every token
+// tile.  Values beyond the fp16 range raise kErrRange once per thread.
 template <int BN, int EPI, int EW>
 __device__ __forceinline__ void gemm_epilogue_chunk(const GemmArgs& a, float (&v)[EW], int row,
                                                     int feat_tile, int t0, int jlo, int jhi,
@@ -174,126 +198,143 @@ __device__ __forceinline__ void gemm_epilogue_chunk(const GemmArgs& a, float (&v
 #pragma unroll
     for (int j = 0; j < EW; ++j) v[j] *= a.w_scale;
   }
-  if constexpr (EPI == kEpiStoreF16) {
-    __half* y = static_cast<__half*>(a.y);
-    const int f = feat_tile * 128 + row;
+  if constexpr (EPI != kEpiArgmax) {
+    constexpr int LDX = 132;
+    float* xs = xbuf;   // [EW][LDX]
 #pragma unroll
-    for (int j = 0; j < EW; ++j)
-      if (j >= jlo && j < jhi) y[static_cast<size_t>(t0 + j) * a.ldy + f] = to_f16(v[j], a.err);
-  } else if constexpr (EPI == kEpiResidF32) {
-    float* y = static_cast<float*>(a.y);
-    const int f = feat_tile * 128 + row;
-    const float g = a.hb_out ? __bfloat162float(a.g_next[f]) : 0.f;
-    float hv[EW];
-#pragma unroll
-    for (int j = 0; j < EW; ++j)   // all loads first: one round trip, not 32
-      hv[j] = (j >= jlo && j < jhi) ? y[static_cast<size_t>(t0 + j) * a.ldy + f] : 0.f;
-#pragma unroll
-    for (int j = 0; j < EW; ++j) {
-      float hsq = 0.f;
-      if (j >= jlo && j < jhi) {
-        const float hn = hv[j] + v[j];
-        y[static_cast<size_t>(t0 + j) * a.ldy + f] = hn;
-        if (a.hb_out) a.hb_out[static_cast<size_t>(t0 + j) * a.ldy + f] = to_f16(hn * g, a.err);
-        hsq = hn * hn;
-      }
-      v[j] = hsq;
-    }
-    if (a.ssp_out != nullptr) {
-      // sum of h^2 over the tile's 128 features per token: warp tree, then 4 warps in order
-#pragma unroll
-      for (int j = 0; j < EW; ++j) {
-        if (j >= jlo && j < jhi) {   // uniform across the CTA
-          float t = v[j];
-#pragma unroll
-          for (int m = 16; m >= 1; m >>= 1) t += __shfl_xor_sync(0xFFFFFFFFu, t, m);
-          if (lane == 0) xbuf[warp * 32 + j] = t;
-        }
-      }
-      asm volatile("bar.sync 2, 128;" ::: "memory");
-      if (threadIdx.x < 32) {
-        const int j = threadIdx.x;
-        if (j >= jlo && j < jhi)
-          a.ssp_out[static_cast<size_t>(t0 + j) * a.n_ssp + feat_tile] =
-              ((xbuf[j] + xbuf[32 + j]) + xbuf[64 + j]) + xbuf[96 + j];
-      }
-      asm volatile("bar.sync 2, 128;" ::: "memory");
-    }
-  } else if constexpr (EPI == kEpiQKV) {
-    // rows of this tile: two heads of 64; RoPE pairs row r with row r ^ 32
-    const int rbase = feat_tile * 128;
-    const int region = rbase < a.Hq * 64 ? 0 : (rbase < (a.Hq + a.Hkv) * 64 ? 1 : 2);
-    const int d = row & 63;
-    if (region < 2) {
-#pragma unroll
-      for (int j = 0; j < EW; ++j)
-        if (j >= jlo && j < jhi) xbuf[j * 128 + row] = v[j];
-      asm volatile("bar.sync 1, 128;" ::: "memory");
-      float2 cs[EW];
-#pragma unroll
-      for (int j = 0; j < EW; ++j) {   // staged rows, else all table loads first
-        const int p = tm.pos[j];
-        const bool ok = j >= jlo && j < jhi && p >= 0 && p < a.max_ctx;
-        cs[j] = !ok ? make_float2(1.f, 0.f)
-                    : (tm.cs ? tm.cs[j * 32 + (d & 31)]
-                             : a.rope[static_cast<size_t>(p) * 32 + (d & 31)]);
-      }
-#pragma unroll
-      for (int j = 0; j < EW; ++j) {
-        if (j >= jlo && j < jhi) {
-          const float pr = xbuf[j * 128 + (row ^ 32)];
-          v[j] = d < 32 ? v[j] * cs[j].x - pr * cs[j].y : v[j] * cs[j].x + pr * cs[j].y;
-        }
-      }
-      asm volatile("bar.sync 1, 128;" ::: "memory");
-    }
-    const int head = (rbase + row) / 64 - (region == 0 ? 0 : (region == 1 ? a.Hq : a.Hq + a.Hkv));
-    if (region == 0) {
-#pragma unroll
-      for (int j = 0; j < EW; ++j)
-        if (j >= jlo && j < jhi)
-          a.q_out[(static_cast<size_t>(t0 + j) * a.Hq + head) * 64 + d] = to_f16(v[j], a.err);
-    } else if (region == 1) {
-      // K: kvdst[j] = offset of (page, K, head 0, token p & 63, dim 0); K is [token][dim]
-      const long long off = static_cast<long long>(head) * 4096 + d;
-#pragma unroll
-      for (int j = 0; j < EW; ++j) {
-        const long long base = tm.kvdst[j];
-        if (j >= jlo && j < jhi && base >= 0) a.kv_layer[base + off] = to_f16(v[j], a.err);
-      }
-    } else {
-      // V is stored transposed, [dim][token]: (page, V, head, dim d, token p & 63)
-      const long long off = (static_cast<long long>(a.Hkv) + head) * 4096 + d * 64;
-#pragma unroll
-      for (int j = 0; j < EW; ++j) {
-        const long long base = tm.kvdst[j];
-        if (j >= jlo && j < jhi && base >= 0) {
-          const int tok = tm.pos[j] & 63;
-          a.kv_layer[base - tok * 64 + off + tok] = to_f16(v[j], a.err);
-        }
-      }
-    }
-  } else if constexpr (EPI == kEpiSwiGLU) {
-    // rows 0..63: gate of features f0..f0+63; rows 64..127: up of the same features
-    if (warp >= 2) {
-#pragma unroll
-      for (int j = 0; j < EW; ++j)
-        if (j >= jlo && j < jhi) xbuf[j * 64 + (row - 64)] = v[j];
-    }
+    for (int j = 0; j < EW; ++j) xs[j * LDX + row] = v[j];
     asm volatile("bar.sync 1, 128;" ::: "memory");
-    if (warp < 2) {
+    bool bad = false;
+    const int tid = row;
+    if constexpr (EPI == kEpiStoreF16) {
       __half* y = static_cast<__half*>(a.y);
-      const int f = feat_tile * 64 + row;
+      for (int it = tid; it < EW * 16; it += 128) {
+        const int j = it >> 4, g = it & 15;
+        if (j < jlo || j >= jhi) continue;
+        const float4 a0 = *reinterpret_cast<const float4*>(xs + j * LDX + 8 * g);
+        const float4 a1 = *reinterpret_cast<const float4*>(xs + j * LDX + 8 * g + 4);
+        const float x[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
+        *reinterpret_cast<uint4*>(y + static_cast<size_t>(t0 + j) * a.ldy + feat_tile * 128 + 8 * g) =
+            pack8_f16(x, bad);
+      }
+    } else if constexpr (EPI == kEpiResidF32) {
+      // h = h + acc (fp32), the next norm's input hb = fp16(h * g), and the sum
+      // of h^2 over the tile's 128 features per token: each item sums its 8
+      // features in order, then the 16 items of a token in order
+      float* y = static_cast<float*>(a.y);
+      float* part = xs + EW * LDX;   // [EW][16]
+      for (int it = tid; it < EW * 16; it += 128) {
+        const int j = it >> 4, g = it & 15;
+        if (j < jlo || j >= jhi) continue;
+        const int f = feat_tile * 128 + 8 * g;
+        float* yr = y + static_cast<size_t>(t0 + j) * a.ldy + f;
+        const float4 h0 = *reinterpret_cast<const float4*>(yr);
+        const float4 h1 = *reinterpret_cast<const float4*>(yr + 4);
+        const float4 a0 = *reinterpret_cast<const float4*>(xs + j * LDX + 8 * g);
+        const float4 a1 = *reinterpret_cast<const float4*>(xs + j * LDX + 8 * g + 4);
+        const float hn[8] = {h0.x + a0.x, h0.y + a0.y, h0.z + a0.z, h0.w + a0.w,
+                             h1.x + a1.x, h1.y + a1.y, h1.z + a1.z, h1.w + a1.w};
+        *reinterpret_cast<float4*>(yr) = make_float4(hn[0], hn[1], hn[2], hn[3]);
+        *reinterpret_cast<float4*>(yr + 4) = make_float4(hn[4], hn[5], hn[6], hn[7]);
+        if (a.hb_out != nullptr) {
+          const uint4 graw = *reinterpret_cast<const uint4*>(a.g_next + f);
+          const __nv_bfloat162* gp = reinterpret_cast<const __nv_bfloat162*>(&graw);
+          float x[8];
 #pragma unroll
-      for (int j = 0; j < EW; ++j)
-        if (j >= jlo && j < jhi) {
-          const float g = v[j];
-          const float u = xbuf[j * 64 + row];
-          const float s = g / (1.0f + __expf(-g));
-          y[static_cast<size_t>(t0 + j) * a.ldy + f] = to_f16(s * u, a.err);
+          for (int e = 0; e < 4; ++e) {
+            const float2 gg = __bfloat1622float2(gp[e]);
+            x[2 * e] = hn[2 * e] * gg.x;
+            x[2 * e + 1] = hn[2 * e + 1] * gg.y;
+          }
+          *reinterpret_cast<uint4*>(a.hb_out + static_cast<size_t>(t0 + j) * a.ldy + f) =
+              pack8_f16(x, bad);
         }
+        float sq = 0.f;
+#pragma unroll
+        for (int e = 0; e < 8; ++e) sq += hn[e] * hn[e];
+        part[j * 16 + g] = sq;
+      }
+      if (a.ssp_out != nullptr) {
+        asm volatile("bar.sync 2, 128;" ::: "memory");
+        if (tid < EW) {
+          const int j = tid;
+          if (j >= jlo && j < jhi) {
+            const float* pp = part + j * 16;
+            float t = 0.f;
+#pragma unroll
+            for (int g = 0; g < 16; ++g) t += pp[g];
+            a.ssp_out[static_cast<size_t>(t0 + j) * a.n_ssp + feat_tile] = t;
+          }
+        }
+      }
+    } else if constexpr (EPI == kEpiSwiGLU) {
+      // rows 0..63: gate of output features f0..f0+63; rows 64..127: up of the same
+      __half* y = static_cast<__half*>(a.y);
+      for (int it = tid; it < EW * 8; it += 128) {
+        const int j = it >> 3, g = it & 7;
+        if (j < jlo || j >= jhi) continue;
+        float x[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+          const float gt = xs[j * LDX + 8 * g + e];
+          const float up = xs[j * LDX + 64 + 8 * g + e];
+          x[e] = gt / (1.0f + __expf(-gt)) * up;
+        }
+        *reinterpret_cast<uint4*>(y + static_cast<size_t>(t0 + j) * a.ldy + feat_tile * 64 + 8 * g) =
+            pack8_f16(x, bad);
+      }
+    } else {   // kEpiQKV
+      // rows of this tile: two heads of 64; RoPE rotates dims d and d ^ 32
+      // with angle index d & 31 at the token's position; q to its buffer, k
+      // and v into the token's KV page (V stored transposed, [dim][token])
+      const int rbase = feat_tile * 128;
+      const int region = rbase < a.Hq * 64 ? 0 : (rbase < (a.Hq + a.Hkv) * 64 ? 1 : 2);
+      const int head0 = rbase / 64 - (region == 0 ? 0 : (region == 1 ? a.Hq : a.Hq + a.Hkv));
+      for (int it = tid; it < EW * 16; it += 128) {
+        const int j = it >> 4, hh = (it >> 3) & 1, g = it & 7;
+        if (j < jlo || j >= jhi) continue;
+        const int head = head0 + hh;
+        const float* xr = xs + j * LDX + hh * 64;
+        float x[8];
+        if (region < 2) {
+          const int p = tm.pos[j];
+          const bool okp = p >= 0 && p < a.max_ctx;
+#pragma unroll
+          for (int e = 0; e < 8; ++e) {
+            const int d = 8 * g + e;
+            const float2 cs = !okp ? make_float2(1.f, 0.f)
+                                   : (tm.cs ? tm.cs[j * 32 + (d & 31)]
+                                            : a.rope[static_cast<size_t>(p) * 32 + (d & 31)]);
+            const float pr = xr[d ^ 32];
+            x[e] = d < 32 ? xr[d] * cs.x - pr * cs.y : xr[d] * cs.x + pr * cs.y;
+          }
+        } else {
+#pragma unroll
+          for (int e = 0; e < 8; ++e) x[e] = xr[8 * g + e];
+        }
+        if (region == 0) {
+          *reinterpret_cast<uint4*>(a.q_out + (static_cast<size_t>(t0 + j) * a.Hq + head) * 64 + 8 * g) =
+              pack8_f16(x, bad);
+        } else {
+          const long long base = tm.kvdst[j];
+          if (base < 0) continue;
+          if (region == 1) {   // K: [token][dim]
+            *reinterpret_cast<uint4*>(a.kv_layer + base + static_cast<long long>(head) * 4096 + 8 * g) =
+                pack8_f16(x, bad);
+          } else {             // V^T: [dim][token]
+            const int tok = tm.pos[j] & 63;
+            __half* vt = a.kv_layer + base - tok * 64 + (static_cast<long long>(a.Hkv) + head) * 4096 + tok;
+            const uint4 w = pack8_f16(x, bad);
+            const __half* hv = reinterpret_cast<const __half*>(&w);
+#pragma unroll
+            for (int e = 0; e < 8; ++e) vt[(8 * g + e) * 64] = hv[e];
+          }
+        }
+      }
     }
-    asm volatile("bar.sync 1, 128;" ::: "memory");
+    if (bad) atomicExch(a.err, kErrRange);
+    asm volatile("bar.sync 1, 128;" ::: "memory");   // xs is reused by the next slice
+    return;
   } else {  // argmax over the vocabulary rows of this tile, per token
     const uint32_t f = static_cast<uint32_t>(feat_tile * 128 + row);
     unsigned long long* out = static_cast<unsigned long long*>(a.y);
@@ -646,10 +687,10 @@ __global__ void __launch_bounds__(128, 1)
         bulk_commit();
       }
       const bool got = __syncthreads_and(mbar_wait(smem_u32(recv_bar), 0, a.err)) != 0;
-      if constexpr (EPI == kEpiArgmax) {   // its key table overlaps `stage`
-        if (threadIdx.x == 0) bulk_wait_read_all();
-        __syncthreads();
-      }
+      // the epilogue's exchange buffer overlaps `stage`: our outgoing slices
+      // must have left it
+      if (threadIdx.x == 0) bulk_wait_read_all();
+      __syncthreads();
       const int lo = split * per, hi = min(lo + per, ntok);
       if (hi > lo && !failed && got) {
         const int nq = hi - lo;
@@ -678,7 +719,6 @@ __global__ void __launch_bounds__(128, 1)
                                            rs_of(c));
         }
       }
-      if (threadIdx.x == 0) bulk_wait_read_all();   // our outgoing slices have left `stage`
       return;
     }
   }
@@ -722,6 +762,253 @@ __global__ void __launch_bounds__(128, 1)
     }
     gemm_epilogue_chunk<BN, EPI, 32>(a, v, row, feat_tile, tok0 + c * 32, 0, 32, xbuf, rs_of(c));
   }
+}
+
+// ---------------------------------------------------------------------------
+// Chunked-K GEMM for wide decode windows.  K is reduced as `chunks` chunks of
+// kpc k-blocks, each summed from zero, then the chunks summed in order
+// 0..chunks-1 -- the same sums, in the same order, as split-K across CTAs --
+// but with one running sum instead of one accumulator per chunk, so the token
+// tile can be wide: TMEM holds the running sum (BN columns) and NB = 256 / BN
+// - 1 chunk buffers, 256 columns in all, so two CTAs share an SM.
+//   warp 4 lane 0   TMA producer (k-blocks in chunk order through the ring)
+//   warp 5 lane 0   MMA issuer: chunk c into buffer c % NB, fresh at its first
+//                   k-block, then a commit on acc_full[buffer]; a buffer is
+//                   reused once the epilogue warps have drained it
+//   warps 0-3       drain each chunk as it completes: sum = sum + chunk (the
+//                   first chunk: 0 + chunk) in TMEM, then release the buffer;
+//                   the last chunk goes from registers to the fused epilogue
+// The epilogue warps also stage the per-token epilogue data while the first
+// chunk runs.  Every wait is bounded; a failure is made uniform across the
+// epilogue warps before their first named barrier.
+template <int BN, int EPI>
+__global__ void __launch_bounds__(192, 2)
+    gemm_chunk_kernel(const __grid_constant__ CUtensorMap tmW,
+                      const __grid_constant__ CUtensorMap tmX, const GemmArgs a) {
+  using S = GemmShape<BN>;
+  constexpr int NB = 256 / BN - 1;            // chunk buffers
+  constexpr uint32_t kCols = 256;             // sum at column 0, buffer b at (1 + b) * BN
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  uint8_t* smA = smem;
+  const int NS = a.stages;
+  uint8_t* smB = smem + NS * S::kABytes;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + NS * S::kStageBytes);
+  uint64_t* full = bars;                      // [NS]
+  uint64_t* empty = bars + NS;                // [NS]
+  uint64_t* acc_full = bars + 2 * NS;         // [NB] chunk in its buffer
+  uint64_t* acc_free = acc_full + NB;         // [NB] buffer drained (4 warp arrivals)
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(acc_free + NB);
+  int* fail_flag = reinterpret_cast<int*>(tmem_slot + 1);
+  static_assert((2 * S::kStagesMax + 2 * NB) * 8 + 8 <= 256, "gemm_chunk barriers");
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const int tok_tile = blockIdx.x;
+  const int feat_tile = blockIdx.y;
+  const int nkb = a.K / 64;
+  const int nchunk = a.chunks;
+  const int kpc = nkb / nchunk;
+
+  if (threadIdx.x == 0) {
+    tma_prefetch_desc(&tmW);
+    tma_prefetch_desc(&tmX);
+    for (int s = 0; s < NS; ++s) {
+      mbar_init(smem_u32(&full[s]), 1);
+      mbar_init(smem_u32(&empty[s]), 1);
+    }
+    for (int b = 0; b < NB; ++b) {
+      mbar_init(smem_u32(&acc_full[b]), 1);
+      mbar_init(smem_u32(&acc_free[b]), 4);
+    }
+    *fail_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 4) tmem_alloc(smem_u32(tmem_slot), kCols);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 4) {
+    if (lane == 0) {
+      // TMA producer: the first stages' weight tiles before the dependency wait
+      const uint64_t pol_w = l2_policy_evict_first();
+      const uint64_t pol_x = l2_policy_evict_last();
+      auto load_w = [&](int i, int s) {
+        const uint32_t fb = smem_u32(&full[s]);
+        if constexpr (EPI == kEpiSwiGLU) {
+          tma_load_2d(smem_u32(smA + s * S::kABytes), &tmW, i * 64, feat_tile * 64, fb, pol_w);
+          tma_load_2d(smem_u32(smA + s * S::kABytes + 64 * 128), &tmW, i * 64, a.N + feat_tile * 64,
+                      fb, pol_w);
+        } else {
+          tma_load_2d(smem_u32(smA + s * S::kABytes), &tmW, i * 64, feat_tile * 128, fb, pol_w);
+        }
+      };
+      auto load_x = [&](int i, int s) {
+        tma_load_2d(smem_u32(smB + s * S::kBBytes), &tmX, i * 64, a.x_row0 + tok_tile * BN,
+                    smem_u32(&full[s]), pol_x);
+      };
+      const int npre = nkb < NS ? nkb : NS;
+      for (int i = 0; i < npre; ++i) {
+        mbar_arrive_expect_tx(smem_u32(&full[i]), S::kStageBytes);
+        load_w(i, i);
+      }
+      pdl_wait();
+      pdl_trigger();
+      for (int i = 0; i < npre; ++i) load_x(i, i);
+      for (int i = npre; i < nkb; ++i) {
+        const int s = i % NS;
+        if (!mbar_wait(smem_u32(&empty[s]), ((i / NS) & 1) ^ 1, a.err)) break;
+        mbar_arrive_expect_tx(smem_u32(&full[s]), S::kStageBytes);
+        load_w(i, s);
+        load_x(i, s);
+      }
+    } else {
+      pdl_wait();
+      pdl_trigger();
+    }
+  } else if (warp == 5) {
+    pdl_wait();
+    pdl_trigger();
+    if (lane == 0) {
+      // MMA issuer, N = the tile's rows rounded up to 16 (a ragged last tile
+      // issues narrower MMAs; its columns past M are never read)
+      const int rows = min(BN, a.M - tok_tile * BN);
+      const int n_mma = BN <= 16 ? BN : ((rows + 15) / 16) * 16;
+      const uint32_t idesc = umma_idesc_f16(128, n_mma < 16 ? 16 : n_mma);
+      bool ok = true;
+      for (int c = 0; c < nchunk && ok; ++c) {
+        const int b = c % NB, u = c / NB;
+        if (c >= NB && !mbar_wait(smem_u32(&acc_free[b]), (u - 1) & 1, a.err)) break;
+        tc_fence_after();
+        const uint32_t dst = tmem + static_cast<uint32_t>((1 + b) * BN);
+        for (int k = 0; k < kpc; ++k) {
+          const int i = c * kpc + k;
+          const int s = i % NS;
+          if (!mbar_wait(smem_u32(&full[s]), (i / NS) & 1, a.err)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint64_t ad = umma_desc_sw128(smem_u32(smA + s * S::kABytes));
+          const uint64_t bd = umma_desc_sw128(smem_u32(smB + s * S::kBBytes));
+#pragma unroll
+          for (int q = 0; q < 4; ++q)
+            umma_f16(dst, ad + 2 * q, bd + 2 * q, idesc, (k > 0 || q > 0) ? 1u : 0u);
+          umma_commit(smem_u32(&empty[s]));
+        }
+        if (ok) umma_commit(smem_u32(&acc_full[b]));
+      }
+    }
+  } else {
+    // ---- warps 0-3: per-token epilogue data, then drain the chunks
+    float* rs_s = reinterpret_cast<float*>(smem + NS * S::kStageBytes + 256);
+    long long* kvdst_s = reinterpret_cast<long long*>(rs_s + BN);
+    int* pos_s = reinterpret_cast<int*>(kvdst_s + BN);
+    float2* cs_s = S::kStageRope ? reinterpret_cast<float2*>(pos_s + BN) : nullptr;
+    const int tok0 = tok_tile * BN;
+    if constexpr (EPI == kEpiQKV) {
+      for (int t = threadIdx.x; t < BN; t += 128) {
+        long long dst = -1;
+        int p = -1;
+        if (tok0 + t < a.M) {
+          p = a.pos[tok0 + t];
+          const int slot = a.tok_slot[tok0 + t];
+          if (slot >= 0) {
+            const int lp = p >> 6;
+            const int phys = (p >= 0 && p < a.max_ctx && lp < a.pt_stride)
+                                 ? a.page_table[static_cast<size_t>(slot) * a.pt_stride + lp] : -1;
+            if (phys < 0 || phys >= a.n_pages) atomicExch(a.err, kErrBounds);
+            else dst = static_cast<long long>(phys) * 2 * a.Hkv * 4096 + (p & 63) * 64;
+          }
+        }
+        kvdst_s[t] = dst;
+        pos_s[t] = p;
+        if constexpr (S::kStageRope) {
+          if (p >= 0 && p < a.max_ctx) {
+            const float4* src = reinterpret_cast<const float4*>(a.rope + static_cast<size_t>(p) * 32);
+            float4* dstv = reinterpret_cast<float4*>(cs_s + t * 32);
+#pragma unroll 4
+            for (int q = 0; q < 16; ++q) dstv[q] = src[q];
+          }
+        }
+      }
+    }
+    pdl_wait();
+    pdl_trigger();
+    if (a.ssp_in != nullptr) {
+      for (int t = threadIdx.x; t < BN; t += 128) {
+        float ss = 0.f;
+        if (tok0 + t < a.M) {
+          const float* sp = a.ssp_in + static_cast<size_t>(a.x_row0 + tok0 + t) * a.n_ssp;
+          float part[16];
+#pragma unroll
+          for (int q = 0; q < 16; ++q) part[q] = q < a.n_ssp ? sp[q] : 0.f;
+#pragma unroll
+          for (int q = 0; q < 16; ++q) ss += part[q];
+          for (int q = 16; q < a.n_ssp; ++q) ss += sp[q];
+        }
+        rs_s[t] = rsqrtf(ss * a.inv_d + a.eps);
+      }
+    }
+    const uint32_t trow = tmem + (static_cast<uint32_t>(warp * 32) << 16);
+    const int npiece = min(BN / 32, (a.M - tok0 + 31) / 32);   // 32-token pieces with rows
+    bool ok = true;
+    for (int c = 0; c + 1 < nchunk && ok; ++c) {
+      const int b = c % NB, u = c / NB;
+      ok = __all_sync(0xFFFFFFFFu, mbar_wait(smem_u32(&acc_full[b]), u & 1, a.err)) != 0;
+      if (!ok) break;
+      tc_fence_after();
+      const uint32_t buf = trow + static_cast<uint32_t>((1 + b) * BN);
+      for (int pc = 0; pc < npiece; ++pc) {
+        uint32_t ch[32], sm[32];
+        tmem_ld32_nowait(buf + pc * 32, ch);
+        if (c > 0) tmem_ld32_nowait(trow + pc * 32, sm);
+        tmem_wait_ld();
+#pragma unroll
+        for (int j = 0; j < 32; ++j)
+          sm[j] = __float_as_uint((c > 0 ? __uint_as_float(sm[j]) : 0.0f) + __uint_as_float(ch[j]));
+        tmem_st32(trow + pc * 32, sm);
+      }
+      tmem_wait_st();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(smem_u32(&acc_free[b]));
+    }
+    if (ok) {
+      const int c = nchunk - 1, b = c % NB, u = c / NB;
+      ok = __all_sync(0xFFFFFFFFu, mbar_wait(smem_u32(&acc_full[b]), u & 1, a.err)) != 0;
+    }
+    if (!ok && lane == 0) atomicExch(fail_flag, 1);
+    asm volatile("bar.sync 3, 128;" ::: "memory");
+    const bool failed = *reinterpret_cast<volatile int*>(fail_flag) != 0;
+    if (!failed) {
+      tc_fence_after();
+      const int c = nchunk - 1, b = c % NB;
+      const uint32_t buf = trow + static_cast<uint32_t>((1 + b) * BN);
+      float* xbuf = reinterpret_cast<float*>(smA);   // every MMA has retired: the ring is free
+      const float* rs_c = a.ssp_in ? rs_s : nullptr;
+      for (int pc = 0; pc < npiece; ++pc) {
+        uint32_t ch[32], sm[32];
+        tmem_ld32_nowait(buf + pc * 32, ch);
+        if (c > 0) tmem_ld32_nowait(trow + pc * 32, sm);
+        tmem_wait_ld();
+        float v[32];
+#pragma unroll
+        for (int j = 0; j < 32; ++j)
+          v[j] = (c > 0 ? __uint_as_float(sm[j]) : 0.0f) + __uint_as_float(ch[j]);
+        const TokMeta tm{rs_c ? rs_c + pc * 32 : nullptr, kvdst_s + pc * 32, pos_s + pc * 32,
+                         cs_s ? cs_s + pc * 32 * 32 : nullptr};
+        gemm_epilogue_chunk<BN, EPI, 32>(a, v, warp * 32 + lane, feat_tile, tok0 + pc * 32, 0, 32,
+                                         xbuf, tm);
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 4) tmem_dealloc(tmem, kCols);
 }
 
 }  // namespace gs

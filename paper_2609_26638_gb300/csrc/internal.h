@@ -70,6 +70,7 @@ cudaError_t launch_gemm(int bn, int epi, const CUtensorMap& tmW, const CUtensorM
 // or the encode fails.
 bool make_map(CUtensorMap* m, const void* base, uint64_t rows, uint64_t cols, uint32_t box_rows);
 
+
 // Sets the dynamic shared-memory limit of every GEMM instantiation once.
 cudaError_t gemm_init_attributes();
 // Every kernel's launch attributes on the current device, once per device

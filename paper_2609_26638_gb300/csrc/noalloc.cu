@@ -59,7 +59,8 @@ extern "C" int gs_linear_noalloc(const void* x, const void* w, void* y, int M, i
   if (epilogue < 0 || epilogue > 3) return GS_ERR_INVALID_ARG;
   if (epilogue == kEpiSwiGLU ? (N % 64) : (N % 128)) return GS_ERR_INVALID_ARG;
   if (M > 65536) return GS_ERR_UNSUPPORTED;
-  if ((reinterpret_cast<uintptr_t>(x) & 15) || (reinterpret_cast<uintptr_t>(w) & 15))
+  if ((reinterpret_cast<uintptr_t>(x) & 15) || (reinterpret_cast<uintptr_t>(w) & 15) ||
+      (reinterpret_cast<uintptr_t>(y) & 15))
     return GS_ERR_INVALID_ARG;
   const int bn = gemm_bn_for(M);
   const int tok_tiles = (M + bn - 1) / bn;
