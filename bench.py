@@ -778,6 +778,180 @@ def gpu_oracle_parity(eng, wl, sample, K) -> dict:
     return out
 
 
+# ---------------------------------------------------------------------- the other decoding modes
+MODE_PARAMS = {
+    # stochastic acceptance (Sec. 3): temperature 1, block size K of the workload
+    "stochastic": dict(temperature=1.0, seed=2024),
+    # direct block diffusion (decoding appendix): block B = K, tau_c = 0.9 (the paper's sweep value)
+    "diffusion": dict(tau=0.9),
+    # multi-step drafting (Sec. 6): tau_d = 0.9
+    "refined": dict(tau=0.9),
+}
+MODE_METRIC = {
+    "stochastic": "committed tokens/s (stochastic self-speculative decode, T=1, 1 GB300 per rank)",
+    "diffusion": "committed tokens/s (direct block-diffusion decode, tau_c=0.9, 1 GB300 per rank)",
+    "refined": "committed tokens/s (multi-step drafting self-speculative decode, tau_d=0.9, "
+               "1 GB300 per rank)",
+}
+
+
+def forward_bytes(cfg, ctx_total: int) -> int:
+    """Algorithmic HBM bytes of one decoder forward over a batch whose
+    sequences see ctx_total keys in all: every weight matrix once (fp16
+    copies), the KV rows read once per layer (K and V, fp16)."""
+    return synth.weight_bytes(cfg) + ctx_total * cfg.n_layers * cfg.n_kv_heads * cfg.head_dim * 2 * 2
+
+
+def mode_arm(args, world: int):
+    """One complete decode of every sequence of the workload per step in the
+    given mode, each call one CUDA graph (a round, or a block with its
+    conditional denoising loop).  The draws and thresholds are deterministic,
+    so the calls a decode needs are counted once and then replayed without a
+    host synchronisation; per call, its forwards and their context lengths
+    give the algorithmic bytes of the step."""
+    import torch
+    from paper_2609_26638_gb300 import gs
+    from paper_2609_26638_gb300.runtime import Engine
+    dev = torch.device("cuda", int(os.environ.get("LOCAL_RANK", 0)))
+    torch.cuda.set_device(dev)
+    wl = synth.WORKLOADS[args.workload]
+    cfg, K, max_new, mode = wl.model, (wl.K if args.K is None else args.K), wl.max_new, args.mode
+    prm = MODE_PARAMS[mode]
+    prompts = wl.prompts()
+    B = len(prompts)
+    P = [p.length for p in prompts]
+    weights = synth.make_weights(cfg)
+    eng = Engine(cfg, weights, max_batch=B, max_ctx=max(P) + max_new + 2 * K + 64, max_K=K,
+                 max_prefill=2048, device=str(dev))
+    stream = eng.stream
+    slots = torch.arange(B, dtype=torch.int32, device=dev)
+    width = K if mode == "diffusion" else K + 2
+    out_tok = torch.zeros((B, width), dtype=torch.int32, device=dev)
+    out_cnt = torch.zeros(B, dtype=torch.int32, device=dev)
+    out_done = torch.zeros(B, dtype=torch.int32, device=dev)
+    out_steps = torch.zeros(B, dtype=torch.int32, device=dev)
+    x0 = [eng.prefill(i, p.vis, p.text, max_new) for i, p in enumerate(prompts)]
+    if mode == "stochastic":
+        eng.set_sampling(prm["temperature"], prm["seed"])
+
+    def call():
+        if mode == "stochastic":
+            eng.round(slots, K, out_tok, out_cnt, out_done, rule=gs.GS_ACCEPT_STOCHASTIC)
+        elif mode == "diffusion":
+            eng.diffusion_block(slots, K, prm["tau"], out_tok, out_cnt, out_done, out_steps)
+        else:
+            eng.round_refined(slots, K, prm["tau"], out_tok, out_cnt, out_done, out_steps=out_steps)
+
+    def restore_all():
+        for i in range(B):
+            eng.restore(i, P[i], x0[i], 1, max_new, 0, 0)
+
+    # count the calls and forwards of one decode (host-synchronised, untimed)
+    restore_all()
+    calls, forwards, fwd_bytes, committed, launches = 0, 0, 0, 0, 0
+    while True:
+        ctx = [eng.state(i)["seq_len"] for i in range(B)]
+        live = [not eng.state(i)["done"] for i in range(B)]
+        call()
+        stream.synchronize()
+        calls += 1
+        c = out_cnt.cpu().numpy()
+        committed += int(c.sum())
+        W = K + 1
+        ctx_total = sum(n + W for n, lv in zip(ctx, live) if lv)
+        # kernel launches of the call: a forward is embed + 5 per layer + the LM
+        # head; a loop step adds its window, reveal and condition kernels
+        per_fwd = 2 + 5 * cfg.n_layers
+        if mode == "stochastic":
+            nf = 2
+            launches += 2 * per_fwd + 3                     # two windows, accept
+        else:
+            steps = int(out_steps.cpu().numpy().max())
+            nf = steps + 1                                  # the loop's steps + verify / cache write
+            launches += 1 + steps * (per_fwd + 3) + 2 + per_fwd - (1 if mode == "diffusion" else 0)
+        forwards += nf
+        fwd_bytes += nf * forward_bytes(cfg, ctx_total)
+        if out_done.cpu().numpy().all():
+            break
+    eng.check()
+
+    def one_decode():
+        restore_all()
+        for _ in range(calls):
+            call()
+
+    for _ in range(args.warmup):
+        one_decode()
+    stream.synchronize()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize(dev)
+    with ClockSampler(dev.index) as clk:
+        t0.record(stream)
+        for _ in range(args.steps):
+            one_decode()
+        t1.record(stream)
+        stream.synchronize()
+    elapsed = t0.elapsed_time(t1) / 1e3
+    eng.check()
+    # end to end: every call's committed tokens copied back to pinned host memory
+    h_tok = torch.empty((B, width), dtype=torch.int32).pin_memory()
+    h_cnt = torch.empty(B, dtype=torch.int32).pin_memory()
+    torch.cuda.synchronize(dev)
+    e0 = time.perf_counter()
+    for _ in range(args.steps):
+        restore_all()
+        for _ in range(calls):
+            call()
+            with torch.cuda.stream(stream):
+                h_tok.copy_(out_tok, non_blocking=True)
+                h_cnt.copy_(out_cnt, non_blocking=True)
+        stream.synchronize()
+    e_elapsed = time.perf_counter() - e0
+    eng.close()
+    hbm, _, src = load_peaks()
+    achieved = fwd_bytes * args.steps / elapsed / 1e9
+    return dict(elapsed=elapsed, e2e_elapsed=e_elapsed, tokens=committed * args.steps, calls=calls,
+                launches=launches * args.steps + args.steps * B,
+                forwards=forwards, committed=committed, clocks=clk.summary(),
+                roofline={"kernel": f"whole {mode} decode step (all kernels of every forward)",
+                          "bound": "hbm", "achieved": round(achieved, 1), "peak": hbm,
+                          "unit": "GB/s", "frac": round(achieved / hbm, 4), "peak_source": src,
+                          "algorithmic_bytes_per_step": int(fwd_bytes),
+                          "traffic": None},
+                d2h=int(calls * (B * width * 4 + B * 4)), B=B, K=K)
+
+
+def oracle_mode_sample(wl, mode: str, K: int, budget_s: float, weights=None) -> dict:
+    """The oracle in the same mode on this host's cores: the workload's
+    shortest-prefix sequence from its prefill (untimed), calls timed until the
+    budget is spent.  Returns committed tokens and seconds."""
+    from oracle import decode as od
+    from oracle import sampling as sm
+    from oracle.model import Decoder
+    cfg = wl.model
+    prompts = wl.prompts()
+    idx = min(range(len(prompts)), key=lambda i: prompts[i].length)
+    prompt = prompts[idx]
+    dec = Decoder(cfg, weights if weights is not None else synth.make_weights(cfg))
+    st = od.prefill(dec, prompt.vis, prompt.text, prompt.length + wl.max_new + 2 * K + 8, wl.max_new)
+    prm = MODE_PARAMS[mode]
+    tokens, secs, calls = 0, 0.0, 0
+    while not st.done and secs < budget_s:
+        t0 = time.perf_counter()
+        if mode == "stochastic":
+            r = sm.self_spec_round_stochastic(dec, st, K, prm["temperature"], prm["seed"], idx, calls)
+            n = len(r.committed)
+        elif mode == "diffusion":
+            n = len(od.diffusion_block(dec, st, K, prm["tau"]).committed)
+        else:
+            n = len(od.self_spec_round_refined(dec, st, K, prm["tau"])[0].committed)
+        secs += time.perf_counter() - t0
+        tokens += n
+        calls += 1
+    return dict(tokens=tokens, secs=secs, calls=calls, P=prompt.length)
+
+
 def describe(wl, K: int, mean: float, world: int) -> dict:
     prompts = wl.prompts()
     if wl.prefix_min == wl.prefix_max:
@@ -825,6 +999,60 @@ def decode_line(res, world: int) -> dict:
     return d
 
 
+def mode_main(args, wl, world: int, rank: int) -> None:
+    """The bench line of a decoding mode other than the forced greedy decode."""
+    K = wl.K if args.K is None else args.K
+    config = describe(wl, K, wl.accept_mean, world)
+    prm = MODE_PARAMS[args.mode]
+    config["workload"] = (f"{wl.name} ({args.mode} mode, {prm}): GLM-OCR-scale synthetic decoder, "
+                          f"batch {wl.batch}, K (or block size) {K}, {wl.max_new} output tokens per "
+                          f"sequence, natural drafting (no forcing)")
+    config["mode"] = args.mode
+    if args.impl == "reference":
+        if rank != 0:
+            return
+        smp = oracle_mode_sample(wl, args.mode, K, 120.0)
+        value = smp["tokens"] / smp["secs"]
+        cpu = {"value": round(value, 3), "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
+               "sample": f"{smp['calls']} {args.mode} calls of the prefix-{smp['P']} sequence, float64 "
+                         f"oracle on all host cores"}
+        print(json.dumps({"impl": "reference", "metric": MODE_METRIC[args.mode],
+                          "value": round(value, 3), "unit": UNIT, "n_gpus": args.gpus, "steps": smp["calls"],
+                          "warmup": 0, "ms_per_step": round(1e3 * smp["secs"] / max(1, smp["calls"]), 2),
+                          "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+                          "dtype": "f64", "data": "synthetic", "config": config, "cpu_baseline": cpu,
+                          "e2e": {"value": round(value, 3), "unit": UNIT, "h2d_bytes_per_step": 0,
+                                  "d2h_bytes_per_step": 0}}))
+        return
+    import torch
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", int(os.environ["LOCAL_RANK"])))
+    res = mode_arm(args, world)
+    el, ee, tokens_all = job_totals(res["elapsed"], res["e2e_elapsed"], res["tokens"], world, "cuda")
+    line = {"metric": MODE_METRIC[args.mode], "value": round(tokens_all / el, 1), "unit": UNIT,
+            "n_gpus": max(world, 1), "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": round(1e3 * el / args.steps, 3), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f16", "data": "synthetic",
+            "config": config, "calls_per_step": res["calls"], "forwards_per_step": res["forwards"],
+            "tokens_per_forward": round(res["committed"] / (res["forwards"] * res["B"]), 3),
+            "gpu_launches": res["launches"],
+            "e2e": {"value": round(tokens_all / ee, 1), "unit": UNIT, "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": res["d2h"]},
+            "clocks": res["clocks"], "roofline": res["roofline"]}
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        smp = oracle_mode_sample(wl, args.mode, res["K"], 25.0)
+        line["cpu_baseline"] = {
+            "value": round(smp["tokens"] / smp["secs"], 3), "unit": UNIT, "cores": os.cpu_count(),
+            "kind": "oracle", "sample": f"{smp['calls']} {args.mode} calls of the prefix-{smp['P']} "
+                                        f"sequence of the same workload, float64 oracle"}
+    if rank == 0:
+        print(json.dumps(line))
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -840,6 +1068,12 @@ def main():
     ap.add_argument("--no-extra-b1", dest="extra_b1", action="store_false",
                     help="with the serving workload, skip the batch-1 workload's extra figures")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--mode", default="greedy", choices=["greedy", "stochastic", "diffusion", "refined"],
+                    help="greedy: the forced self-speculative decode (the headline); stochastic: "
+                         "GS_ACCEPT_STOCHASTIC rounds at T = 1; diffusion: direct block-diffusion "
+                         "decoding, B = K, tau_c = 0.9; refined: multi-step drafting, tau_d = 0.9")
+    ap.add_argument("--max-new", type=int, default=None,
+                    help="output tokens per sequence (default: the workload's)")
     ap.add_argument("--kernel", default=None,
                     choices=["attention", "lm_head", "attention-sweep", "gemm-serve"],
                     help="time one kernel alone and print its roofline line (the single-kernel "
@@ -880,7 +1114,14 @@ def main():
         return
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
+    if args.max_new is not None:
+        import dataclasses
+        synth.WORKLOADS[args.workload] = dataclasses.replace(synth.WORKLOADS[args.workload],
+                                                             max_new=args.max_new)
     wl = synth.WORKLOADS[args.workload]
+    if args.mode != "greedy":
+        mode_main(args, wl, world, rank)
+        return
     K = wl.K if args.K is None else args.K
     mean = wl.accept_mean if args.accept_mean is None else args.accept_mean
     config = describe(wl, K, mean, world)

@@ -71,3 +71,21 @@ def test_config_names_the_workload():
     json.dumps(d)
     assert "serve_b32" in d["workload"] and d["global_batch"] == 32 and d["K"] == wl.K
     assert bench.describe(wl, wl.K, wl.accept_mean, 4)["global_batch"] == 128
+
+
+def test_mode_oracle_sample_commits_tokens():
+    """The oracle leg of the other decoding modes runs on the small workload
+    and reports committed tokens, calls and the sequence it sampled."""
+    wl = synth.WORKLOADS["tiny"]
+    for mode in ("stochastic", "diffusion", "refined"):
+        smp = bench.oracle_mode_sample(wl, mode, 4, 0.5)
+        assert smp["calls"] >= 1 and smp["tokens"] >= smp["calls"] and smp["secs"] > 0
+        assert smp["P"] == min(p.length for p in wl.prompts())
+        assert bench.MODE_METRIC[mode].startswith("committed tokens/s")
+
+
+def test_forward_bytes_grow_with_context():
+    """One forward reads every weight once and each sequence's cached K and V."""
+    a, b = bench.forward_bytes(GLM, 0), bench.forward_bytes(GLM, 1000)
+    per_key = GLM.n_layers * GLM.n_kv_heads * GLM.head_dim * 2 * 2
+    assert a > 0 and b - a == 1000 * per_key
