@@ -86,3 +86,21 @@ def test_noalloc_rejects_scratch_beyond_its_array(gs):
         gs.gs_linear_noalloc(x.data_ptr(), w.data_ptr(), y.data_ptr(), 17, 8192, 4096,
                              gs.EPI_STORE_F16, 64, torch.cuda.current_stream().cuda_stream)
     assert e.value.code == gs.GS_ERR_OOM
+
+
+def test_noalloc_status_reports_a_range_overflow_then_clears(gs):
+    """Outputs beyond the fp16 range set the private error word; the status
+    query reports it once (GS_ERR_DEVICE_CHECK) and clears it."""
+    stream = torch.cuda.current_stream().cuda_stream
+    x = torch.full((17, 1024), 256.0, dtype=torch.float16, device=DEV)
+    w = torch.full((256, 1024), 256.0, dtype=torch.float16, device=DEV)
+    y = torch.zeros(17, 256, dtype=torch.float16, device=DEV)
+    gs.gs_linear_noalloc(x.data_ptr(), w.data_ptr(), y.data_ptr(), 17, 256, 1024,
+                         gs.EPI_STORE_F16, 1, stream)
+    assert gs.gs_linear_noalloc_status(stream) == gs.GS_ERR_DEVICE_CHECK
+    assert gs.gs_linear_noalloc_status(stream) == gs.GS_OK
+    x.fill_(1.0 / 64)
+    gs.gs_linear_noalloc(x.data_ptr(), w.data_ptr(), y.data_ptr(), 17, 256, 1024,
+                         gs.EPI_STORE_F16, 1, stream)
+    assert gs.gs_linear_noalloc_status(stream) == gs.GS_OK
+    assert torch.all(y == 4096.0)                       # 1024 * 256 / 64, exact in fp16
