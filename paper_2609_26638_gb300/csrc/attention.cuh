@@ -54,7 +54,7 @@ constexpr int kAttnStageBytes = 2 * kAttnPageBytes;
 constexpr int kAttnRow = 68;              // partial row: O[64], m, l, 2 pad (272 B)
 constexpr int kAttnMaxRows = 128;         // rows of one query block (the MMA's M)
 constexpr int kAttnMaxCluster = 16;       // items merged inside a cluster (16: non-portable size)
-constexpr int kAttnSoftWarps = 8;         // two warps per TMEM lane quarter
+constexpr int kAttnSoftWarps = 4;         // one warp per TMEM lane quarter
 constexpr int kAttnSoftThreads = kAttnSoftWarps * 32;
 constexpr int kAttnThreads = kAttnSoftThreads + 64;   // + TMA warp, MMA warp
 constexpr int kAttnTmaWarp = kAttnSoftWarps, kAttnMmaWarp = kAttnSoftWarps + 1;
@@ -119,117 +119,129 @@ __device__ __forceinline__ void tmem_ld16_nowait(uint32_t taddr, uint32_t (&r)[1
 // Barriers and buffers the softmax warps share with the MMA warp.
 struct AttnSync {
   uint64_t *s_full, *s_free, *p_full, *pv_done;
-  uint64_t* mx_bar;  // [2] every thread of a row-holding warp posted its page max
   uint8_t* sP;       // [2][128][128 B]
-  float* red;        // [2][128] per-thread page maxima
+  float* red;        // [128] per-thread page maxima (exchanged only when a max rises)
 };
 
-__device__ __forceinline__ void tmem_ld8_nowait(uint32_t taddr, uint32_t (&r)[8]) {
+// Named barriers of the softmax warps (barrier 0 is __syncthreads).
+constexpr int kAttnBarVote = 1, kAttnBarMax = 2;
+
+// OR of a predicate over the softmax threads: one hardware barrier.
+__device__ __forceinline__ bool softmax_vote_or(bool v) {
+  uint32_t r;
   asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%8];"
-      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
-        "=r"(r[7])
-      : "r"(taddr));
+      "{\n\t.reg .pred p, q;\n\t"
+      "setp.ne.u32 q, %1, 0;\n\t"
+      "bar.red.or.pred p, %2, %3, q;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(r)
+      : "r"(v ? 1u : 0u), "n"(kAttnBarVote), "n"(kAttnSoftThreads)
+      : "memory");
+  return r != 0;
 }
 
-// Online softmax over the item's pages for the rows one thread sees.  DUP
-// copies of each block row sit in the MMA's 128 rows (copy k of row rr at MMA
-// row k * 128 / DUP + rr, so every TMEM lane quarter -- and every SM
-// sub-partition -- holds rows), and two warps share each lane quarter: the
-// thread of (copy k, warp half s) takes the columns of part 2k + s, NC =
-// 64 / (2 DUP) columns of every page.  Per page: S from TMEM, mask and scale,
-// the row max over its parts (shared memory), an O rescale when the max rises
-// by more than 2^8 (the two copy-0 threads of the row, 32 columns each; the
-// previous O += P V must have retired), P into shared memory, and the row sum
-// kept as eight 8-column partials, so the arithmetic of a row is the same for
-// every DUP.  Returns false if a wait ran out.
+__device__ __forceinline__ void softmax_bar_max() {
+  asm volatile("bar.sync %0, %1;" ::"n"(kAttnBarMax), "n"(kAttnSoftThreads) : "memory");
+}
+
+// Online softmax over the item's pages, one thread per TMEM lane.  DUP copies
+// of each block row sit in the MMA's 128 rows (copy k of row rr at MMA row
+// k * 128 / DUP + rr, so every lane quarter -- and every SM sub-partition --
+// holds rows); the thread of copy k takes the NC = 64 / DUP columns
+// [k NC, (k + 1) NC) of every page.  Per page: S from TMEM, mask and scale,
+// this thread's maximum; the row's running max m (log2 units) only moves when
+// a page raises it by more than 2^8, so one vote over the softmax threads (a
+// hardware barrier) decides whether any row of the block rises, and only then
+// are the copies' page maxima exchanged through shared memory (always on the
+// first page, rarely after).  A rise rescales O (the copy-0 thread of the row;
+// the previous O += P V must have retired) and the row sums; then P_j =
+// exp2(s - m) as fp16 into row rr of the P tile and the row sum kept as eight
+// 8-column partials.  m, P, the partials and the rescale are the same for every
+// DUP.  Waits are bounded; a warp whose wait ran out keeps passing the named
+// barriers and arriving on the MMA warp's barriers to the last page, so no
+// thread is left at a barrier.  Returns false if a wait ran out.
 template <int DUP>
 __device__ __forceinline__ bool attn_softmax(const AttnArgs& a, const AttnSync& y, uint32_t tmem,
                                              int np, int p_begin, int R, int tok0, float& m,
                                              float (&lc)[8]) {
   constexpr int RPC = kAttnMaxRows / DUP;   // MMA rows per copy
-  constexpr int NC = 64 / (2 * DUP);        // columns per thread
+  constexpr int NC = 64 / DUP;              // columns per thread
   constexpr int NCH = NC / 8;               // 8-column chunks per thread
-  const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
-  const int quarter = warp & 3, half = warp >> 2;
-  const int mrow = quarter * 32 + lane;     // MMA row = TMEM lane
+  const int mrow = threadIdx.x, warp = mrow >> 5, lane = mrow & 31;   // MMA row = TMEM lane
   const int cp = mrow / RPC, rr = mrow % RPC;
-  const int part = 2 * cp + half, col0 = part * NC;
-  const bool busy = ((quarter * 32) % RPC) < R;   // the warp holds at least one real row
+  const int col0 = cp * NC;
+  const bool busy = ((warp * 32) % RPC) < R;   // the warp holds at least one real row
   const int lim_r = rr < R ? a.lim[tok0 + rr / a.G] : -1;
-  const uint32_t trow = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
+  const uint32_t trow = tmem + (static_cast<uint32_t>(warp * 32) << 16);
   const float kScaleLog2 = 0.125f * 1.4426950408889634f;   // 1/sqrt(64) in log2 units
-  // waits are warp-uniform, so a warp that gives up leaves together
+  bool ok = true;
+  // waits are warp-uniform; after a failure the warp stops waiting
   auto wwait = [&](uint64_t* bar, uint32_t parity) {
-    return __all_sync(0xFFFFFFFFu, mbar_wait(smem_u32(bar), parity, a.err)) != 0;
+    if (ok) ok = __all_sync(0xFFFFFFFFu, mbar_wait(smem_u32(bar), parity, a.err)) != 0;
+    return ok;
   };
   for (int j = 0; j < np; ++j) {
     const int buf = j & 1;
-    if (!wwait(&y.s_full[buf], (j >> 1) & 1)) return false;
-    if (!busy) {   // padding rows only: release S, hand over an (unused) P
-      if (lane == 0) {
-        mbar_arrive(smem_u32(&y.s_free[buf]));
-        mbar_arrive(smem_u32(&y.p_full[buf]));
-      }
-      continue;
-    }
+    const bool have = wwait(&y.s_full[buf], (j >> 1) & 1) && busy;
     // 1. this thread's columns of S_j; the buffer is free once every warp has read
-    tc_fence_after();
-    uint32_t sr[NC];
-    if constexpr (NC == 8) {
-      tmem_ld8_nowait(trow + buf * 64 + col0, *reinterpret_cast<uint32_t(*)[8]>(sr));
-    } else if constexpr (NC == 16) {
-      tmem_ld16_nowait(trow + buf * 64 + col0, *reinterpret_cast<uint32_t(*)[16]>(sr));
-    } else {
-      tmem_ld32_nowait(trow + buf * 64 + col0, *reinterpret_cast<uint32_t(*)[32]>(sr));
+    float sv[NC];
+    float pm = -INFINITY;
+    if (have) {
+      tc_fence_after();
+      uint32_t sr[NC];
+      if constexpr (NC == 16) {
+        tmem_ld16_nowait(trow + buf * 64 + col0, *reinterpret_cast<uint32_t(*)[16]>(sr));
+      } else if constexpr (NC == 32) {
+        tmem_ld32_nowait(trow + buf * 64 + col0, *reinterpret_cast<uint32_t(*)[32]>(sr));
+      } else {
+        tmem_ld32_nowait(trow + buf * 64, *reinterpret_cast<uint32_t(*)[32]>(sr));
+        tmem_ld32_nowait(trow + buf * 64 + 32, *reinterpret_cast<uint32_t(*)[32]>(sr + 32));
+      }
+      tmem_wait_ld();
+      // 2. mask (keys past the row's limit), scale, this thread's maximum
+      const int key0 = (p_begin + j) * 64 + col0;
+#pragma unroll
+      for (int k = 0; k < NC; ++k)
+        sv[k] = key0 + k <= lim_r ? __uint_as_float(sr[k]) * kScaleLog2 : -INFINITY;
+      float mt[8];   // max as a tree (a chain of NC dependent fmax would dominate the page)
+#pragma unroll
+      for (int e = 0; e < 8; ++e) {
+        mt[e] = sv[e];
+#pragma unroll
+        for (int k = e + 8; k < NC; k += 8) mt[e] = fmaxf(mt[e], sv[k]);
+      }
+      pm = fmaxf(fmaxf(fmaxf(mt[0], mt[1]), fmaxf(mt[2], mt[3])),
+                 fmaxf(fmaxf(mt[4], mt[5]), fmaxf(mt[6], mt[7])));
     }
-    tmem_wait_ld();
     tc_fence_before();
     __syncwarp();
     if (lane == 0) mbar_arrive(smem_u32(&y.s_free[buf]));
-    // 2. mask (keys past the row's limit), scale, this thread's maximum
-    const int key0 = (p_begin + j) * 64 + col0;
-    float sv[NC];
-#pragma unroll
-    for (int k = 0; k < NC; ++k)
-      sv[k] = key0 + k <= lim_r ? __uint_as_float(sr[k]) * kScaleLog2 : -INFINITY;
-    // max as a tree (a chain of NC dependent fmax would dominate the page)
-    float mt[8];
-#pragma unroll
-    for (int e = 0; e < 8; ++e) {
-      mt[e] = sv[e];
-#pragma unroll
-      for (int k = e + 8; k < NC; k += 8) mt[e] = fmaxf(mt[e], sv[k]);
-    }
-    const float pmx = fmaxf(fmaxf(fmaxf(mt[0], mt[1]), fmaxf(mt[2], mt[3])),
-                            fmaxf(fmaxf(mt[4], mt[5]), fmaxf(mt[6], mt[7])));
-    // 3. the row's page max over its 2 DUP parts (thread of part p: MMA row
-    //    (p / 2) * RPC + rr, warp half p % 2)
-    float* red = y.red + buf * kAttnSoftThreads;
-    red[t] = pmx;
-    __syncwarp();
-    if (lane == 0) mbar_arrive(smem_u32(&y.mx_bar[buf]));
-    if (!wwait(&y.mx_bar[buf], (j >> 1) & 1)) return false;
+    // 3. does any row rise by more than 2^8?  Then the row's page max over its
+    //    DUP copies (copy k at MMA row k * RPC + rr).
+    const bool any = softmax_vote_or(pm > m + kAttnRescale);
     float mx = -INFINITY;
+    if (any) {
+      y.red[mrow] = pm;
+      softmax_bar_max();
 #pragma unroll
-    for (int pp = 0; pp < 2 * DUP; ++pp) {
-      const int mr = (pp >> 1) * RPC + rr;
-      mx = fmaxf(mx, red[((pp & 1) * 4 + (mr >> 5)) * 32 + (mr & 31)]);
+      for (int k = 0; k < DUP; ++k) mx = fmaxf(mx, y.red[k * RPC + rr]);
     }
-    // 4. a rise by more than 2^8 rescales O and the row sums first
-    //    tcgen05.ld / st are warp-collective: a warp with any rising row
-    //    rescales all its rows, the others by exactly 1.
-    const bool rise = mx > m + kAttnRescale;
+    // 4. a rise rescales O and the row sums first.  tcgen05.ld / st are
+    //    warp-collective: a warp with any rising row rescales all its rows,
+    //    the others by exactly 1.
+    const bool rise = any && mx > m + kAttnRescale;
     const float alpha = !rise ? 1.f : ((m == -INFINITY) ? 0.f : exp2f(m - mx));
-    if (cp == 0 && j > 0 && __any_sync(0xFFFFFFFFu, rise)) {
-      if (!wwait(y.pv_done, (j - 1) & 1)) return false;
+    if (cp == 0 && j > 0 && __any_sync(0xFFFFFFFFu, rise) && wwait(y.pv_done, (j - 1) & 1)) {
       tc_fence_after();
-      uint32_t o32[32];
-      tmem_ld32_nowait(trow + 128 + half * 32, o32);
-      tmem_wait_ld();
 #pragma unroll
-      for (int k = 0; k < 32; ++k) o32[k] = __float_as_uint(alpha * __uint_as_float(o32[k]));
-      tmem_st32(trow + 128 + half * 32, o32);
+      for (int hh = 0; hh < 2; ++hh) {
+        uint32_t o32[32];
+        tmem_ld32_nowait(trow + 128 + hh * 32, o32);
+        tmem_wait_ld();
+#pragma unroll
+        for (int k = 0; k < 32; ++k) o32[k] = __float_as_uint(alpha * __uint_as_float(o32[k]));
+        tmem_st32(trow + 128 + hh * 32, o32);
+      }
       tmem_wait_st();
     }
     if (rise) {
@@ -238,29 +250,31 @@ __device__ __forceinline__ bool attn_softmax(const AttnArgs& a, const AttnSync& 
       m = mx;
     }
     // 5. P_j = exp2(s - m) (fp16) into row rr of the P tile; 8-column sums
-    const float sub = (m == -INFINITY) ? 0.f : m;
-    uint8_t* prow = y.sP + buf * kAttnMaxRows * 128;
+    if (have) {
+      const float sub = (m == -INFINITY) ? 0.f : m;
+      uint8_t* prow = y.sP + buf * kAttnMaxRows * 128;
 #pragma unroll
-    for (int c = 0; c < NCH; ++c) {
-      float p[8];
+      for (int c = 0; c < NCH; ++c) {
+        float p[8];
 #pragma unroll
-      for (int e = 0; e < 8; ++e) p[e] = exp2f(sv[8 * c + e] - sub);
-      lc[c] += ((p[0] + p[1]) + (p[2] + p[3])) + ((p[4] + p[5]) + (p[6] + p[7]));
-      uint32_t w4[4];
+        for (int e = 0; e < 8; ++e) p[e] = exp2f(sv[8 * c + e] - sub);
+        lc[c] += ((p[0] + p[1]) + (p[2] + p[3])) + ((p[4] + p[5]) + (p[6] + p[7]));
+        uint32_t w4[4];
 #pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        __half2 hv = __floats2half2_rn(p[2 * e], p[2 * e + 1]);
-        w4[e] = *reinterpret_cast<uint32_t*>(&hv);
+        for (int e = 0; e < 4; ++e) {
+          __half2 hv = __floats2half2_rn(p[2 * e], p[2 * e + 1]);
+          w4[e] = *reinterpret_cast<uint32_t*>(&hv);
+        }
+        *reinterpret_cast<uint4*>(prow + sw128(rr, col0 / 8 + c)) =
+            make_uint4(w4[0], w4[1], w4[2], w4[3]);
       }
-      *reinterpret_cast<uint4*>(prow + sw128(rr, col0 / 8 + c)) =
-          make_uint4(w4[0], w4[1], w4[2], w4[3]);
+      fence_proxy_async_smem();
     }
-    fence_proxy_async_smem();
     tc_fence_before();
     __syncwarp();
     if (lane == 0) mbar_arrive(smem_u32(&y.p_full[buf]));
   }
-  return true;
+  return ok;
 }
 
 __global__ void __launch_bounds__(kAttnThreads, 2)
@@ -283,7 +297,6 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
   uint64_t* mma_done = s_full + 7;                       // every MMA of this CTA retired
   uint64_t* recv_bar = s_full + 8;
   uint64_t* q_full = s_full + 9;                         // Q tile in smem (4 warp arrivals)
-  uint64_t* mx_bar = s_full + 10;                        // [2] page maxima exchanged
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(s_full + 12);
   // [0] max limit, [1] last-item flag, [2] pages the MMA warp took, [3] pages issued
   int* s_int = reinterpret_cast<int*>(s_full + 13);
@@ -340,13 +353,6 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
     mbar_init(smem_u32(pv_done), 1);
     mbar_init(smem_u32(mma_done), 1);
     mbar_init(smem_u32(q_full), kAttnSoftWarps);
-    {
-      const int rpc = kAttnMaxRows / (R <= 32 ? 4 : (R <= 64 ? 2 : 1));
-      int nbusy = 0;   // softmax warps that hold rows
-      for (int w = 0; w < kAttnSoftWarps; ++w) nbusy += (((w & 3) * 32) % rpc) < R ? 1 : 0;
-      mbar_init(smem_u32(&mx_bar[0]), nbusy);
-      mbar_init(smem_u32(&mx_bar[1]), nbusy);
-    }
     if (in_cluster) {
       mbar_init(smem_u32(recv_bar), 1);
       // nitems sources, ceil(128 / nitems) rows each, arrive by bulk copy
@@ -369,7 +375,7 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
   bool ok = true;
   float m = -INFINITY, l = 0.f;   // the row's running max (log2 units) and sum
   float lc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};   // row sum, 8-column partials
-  float* red = reinterpret_cast<float*>(s_int + 8);        // [2][softmax threads] page maxima
+  float* red = reinterpret_cast<float*>(s_int + 8);        // [softmax threads] page maxima
   float* lsum = red + 2 * kAttnSoftThreads;                // [8][128] partial sums
 
   if (warp == kAttnTmaWarp) {
@@ -470,14 +476,14 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
     fence_proxy_async_smem();
     __syncwarp();
     if (lane == 0) mbar_arrive(smem_u32(q_full));
-    AttnSync y{s_full, s_free, p_full, pv_done, mx_bar, sP, red};
+    AttnSync y{s_full, s_free, p_full, pv_done, sP, red};
     if (dup == 4) ok = attn_softmax<4>(a, y, tmem, np, p_begin, R, tok0, m, lc);
     else if (dup == 2) ok = attn_softmax<2>(a, y, tmem, np, p_begin, R, tok0, m, lc);
     else ok = attn_softmax<1>(a, y, tmem, np, p_begin, R, tok0, m, lc);
     // the row's eight 8-column partial sums -> shared memory [chunk][row]
-    const int mrow = (warp & 3) * 32 + lane;
-    const int part = 2 * (mrow / rpc) + (warp >> 2), nch = 8 / (2 * dup);
-    for (int cc = 0; cc < nch; ++cc) lsum[(part * nch + cc) * kAttnMaxRows + mrow % rpc] = lc[cc];  }
+    const int mrow = threadIdx.x, nch = 8 / dup;
+    for (int cc = 0; cc < nch; ++cc) lsum[((mrow / rpc) * nch + cc) * kAttnMaxRows + mrow % rpc] = lc[cc];
+  }
 
   const bool all_ok = __syncthreads_and(ok);
   // every MMA retired and every TMA copy landed before TMEM and the ring are reused
