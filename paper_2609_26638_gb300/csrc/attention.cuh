@@ -116,6 +116,14 @@ __device__ __forceinline__ void tmem_ld16_nowait(uint32_t taddr, uint32_t (&r)[1
       : "r"(taddr));
 }
 
+// 2^x on the SFU (PTX ex2.approx.ftz.f32, one instruction): the P values are
+// 2^(s - m) <= 2^8, and a result below the fp32 normal range is an fp16 zero.
+__device__ __forceinline__ float ex2_sfu(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
 // Barriers and buffers the softmax warps share with the MMA warp.
 struct AttnSync {
   uint64_t *s_full, *s_free, *p_full, *pv_done;
@@ -257,7 +265,7 @@ __device__ __forceinline__ bool attn_softmax(const AttnArgs& a, const AttnSync& 
       for (int c = 0; c < NCH; ++c) {
         float p[8];
 #pragma unroll
-        for (int e = 0; e < 8; ++e) p[e] = exp2f(sv[8 * c + e] - sub);
+        for (int e = 0; e < 8; ++e) p[e] = ex2_sfu(sv[8 * c + e] - sub);
         lc[c] += ((p[0] + p[1]) + (p[2] + p[3])) + ((p[4] + p[5]) + (p[6] + p[7]));
         uint32_t w4[4];
 #pragma unroll
