@@ -206,11 +206,16 @@ __device__ __forceinline__ bool attn_softmax(const AttnArgs& a, const AttnSync& 
         tmem_ld32_nowait(trow + buf * 64 + 32, *reinterpret_cast<uint32_t(*)[32]>(sr + 32));
       }
       tmem_wait_ld();
-      // 2. mask (keys past the row's limit), scale, this thread's maximum
+      // 2. mask (keys past the row's limit: only on the window's last pages),
+      //    this thread's maximum (of the unscaled scores; the scale is positive)
       const int key0 = (p_begin + j) * 64 + col0;
+      if (__all_sync(0xFFFFFFFFu, rr >= R || key0 + NC - 1 <= lim_r)) {
 #pragma unroll
-      for (int k = 0; k < NC; ++k)
-        sv[k] = key0 + k <= lim_r ? __uint_as_float(sr[k]) * kScaleLog2 : -INFINITY;
+        for (int k = 0; k < NC; ++k) sv[k] = __uint_as_float(sr[k]);
+      } else {
+#pragma unroll
+        for (int k = 0; k < NC; ++k) sv[k] = key0 + k <= lim_r ? __uint_as_float(sr[k]) : -INFINITY;
+      }
       float mt[8];   // max as a tree (a chain of NC dependent fmax would dominate the page)
 #pragma unroll
       for (int e = 0; e < 8; ++e) {
@@ -219,7 +224,7 @@ __device__ __forceinline__ bool attn_softmax(const AttnArgs& a, const AttnSync& 
         for (int k = e + 8; k < NC; k += 8) mt[e] = fmaxf(mt[e], sv[k]);
       }
       pm = fmaxf(fmaxf(fmaxf(mt[0], mt[1]), fmaxf(mt[2], mt[3])),
-                 fmaxf(fmaxf(mt[4], mt[5]), fmaxf(mt[6], mt[7])));
+                 fmaxf(fmaxf(mt[4], mt[5]), fmaxf(mt[6], mt[7]))) * kScaleLog2;
     }
     tc_fence_before();
     __syncwarp();
@@ -265,7 +270,7 @@ __device__ __forceinline__ bool attn_softmax(const AttnArgs& a, const AttnSync& 
       for (int c = 0; c < NCH; ++c) {
         float p[8];
 #pragma unroll
-        for (int e = 0; e < 8; ++e) p[e] = ex2_sfu(sv[8 * c + e] - sub);
+        for (int e = 0; e < 8; ++e) p[e] = ex2_sfu(fmaf(sv[8 * c + e], kScaleLog2, -sub));
         lc[c] += ((p[0] + p[1]) + (p[2] + p[3])) + ((p[4] + p[5]) + (p[6] + p[7]));
         uint32_t w4[4];
 #pragma unroll
