@@ -124,6 +124,13 @@ __device__ __forceinline__ float ex2_sfu(float x) {
   return y;
 }
 
+// max of three (PTX max.f32 with three sources, sm_100 and later)
+__device__ __forceinline__ float fmax3(float x, float y, float z) {
+  float r;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(x), "f"(y), "f"(z));
+  return r;
+}
+
 // Barriers and buffers the softmax warps share with the MMA warp.
 struct AttnSync {
   uint64_t *s_full, *s_free, *p_full, *pv_done;
@@ -216,15 +223,19 @@ __device__ __forceinline__ bool attn_softmax(const AttnArgs& a, const AttnSync& 
 #pragma unroll
         for (int k = 0; k < NC; ++k) sv[k] = key0 + k <= lim_r ? __uint_as_float(sr[k]) : -INFINITY;
       }
-      float mt[8];   // max as a tree (a chain of NC dependent fmax would dominate the page)
+      // max as a tree of three-way maxima (a chain of NC dependent fmax
+      // would dominate the page)
+      float mt[8];
 #pragma unroll
       for (int e = 0; e < 8; ++e) {
         mt[e] = sv[e];
+        int k = e + 8;
 #pragma unroll
-        for (int k = e + 8; k < NC; k += 8) mt[e] = fmaxf(mt[e], sv[k]);
+        for (; k + 8 < NC; k += 16) mt[e] = fmax3(mt[e], sv[k], sv[k + 8]);
+        if (k < NC) mt[e] = fmaxf(mt[e], sv[k]);
       }
-      pm = fmaxf(fmaxf(fmaxf(mt[0], mt[1]), fmaxf(mt[2], mt[3])),
-                 fmaxf(fmaxf(mt[4], mt[5]), fmaxf(mt[6], mt[7]))) * kScaleLog2;
+      pm = fmax3(fmax3(mt[0], mt[1], mt[2]), fmax3(mt[3], mt[4], mt[5]), fmaxf(mt[6], mt[7])) *
+           kScaleLog2;
     }
     tc_fence_before();
     __syncwarp();
