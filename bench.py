@@ -71,9 +71,9 @@ _CSRC = os.path.join(ROOT, "paper_2609_26638_gb300", "csrc")
 NCU_TRAFFIC = {
     "attention_b1": dict(sources=("attention.cuh", "ptx.cuh"), bytes=5002069, algorithmic=4823040,
                          sha256="06dec0a6372c8c089f2878d8cc6e2a400cf336f9289bf7cad4281e0c8fe06266"),
-    "attention_serve": dict(sources=("attention.cuh", "ptx.cuh"), bytes=234571520,
+    "attention_serve": dict(sources=("attention.cuh", "ptx.cuh"), bytes=233819648,
                             algorithmic=225173504,
-                            sha256="5a1604b895b865f33bd8f3b60594178814d09693337068d869d94c94d3450f33"),
+                            sha256="c4154e97724194c54884ba6a96d4f34400276927858e81f4dd4810b09e00183e"),
     "lm_head_b1": dict(sources=("gemm_tc.cuh", "gemm.cu", "ptx.cuh"), bytes=124822784,
                        algorithmic=121669768,
                        sha256="acd78b83a80ba74bcd7c190a8f523f7fc8182269637458b3430e12d923ff8077"),
