@@ -69,8 +69,8 @@ def schedule_rounds(sched: np.ndarray, max_new: int) -> int:
 # traffic grows with the keys read: K and V rows, once each).
 _CSRC = os.path.join(ROOT, "paper_2609_26638_gb300", "csrc")
 NCU_TRAFFIC = {
-    "attention_b1": dict(sources=("attention.cuh", "ptx.cuh"), bytes=5002069, algorithmic=4823040,
-                         sha256="06dec0a6372c8c089f2878d8cc6e2a400cf336f9289bf7cad4281e0c8fe06266"),
+    "attention_b1": dict(sources=("attention.cuh", "ptx.cuh"), bytes=4990976, algorithmic=4823040,
+                         sha256="c4154e97724194c54884ba6a96d4f34400276927858e81f4dd4810b09e00183e"),
     "attention_serve": dict(sources=("attention.cuh", "ptx.cuh"), bytes=233819648,
                             algorithmic=225173504,
                             sha256="c4154e97724194c54884ba6a96d4f34400276927858e81f4dd4810b09e00183e"),
