@@ -133,7 +133,8 @@ __device__ __forceinline__ float fmax3(float x, float y, float z) {
 
 // Barriers and buffers the softmax warps share with the MMA warp.
 struct AttnSync {
-  uint64_t *s_full, *s_free, *p_full, *pv_done;
+  uint64_t *s_full, *s_free, *p_full;
+  uint64_t* empty;   // [stages] O += P V of the stage's page retired
   uint8_t* sP;       // [2][128][128 B]
   float* red;        // [128] per-thread page maxima (exchanged only when a max rises)
 };
@@ -255,7 +256,8 @@ __device__ __forceinline__ bool attn_softmax(const AttnArgs& a, const AttnSync& 
     //    the others by exactly 1.
     const bool rise = any && mx > m + kAttnRescale;
     const float alpha = !rise ? 1.f : ((m == -INFINITY) ? 0.f : exp2f(m - mx));
-    if (cp == 0 && j > 0 && __any_sync(0xFFFFFFFFu, rise) && wwait(y.pv_done, (j - 1) & 1)) {
+    if (cp == 0 && j > 0 && __any_sync(0xFFFFFFFFu, rise) &&
+        wwait(&y.empty[(j - 1) % kAttnStages], ((j - 1) / kAttnStages) & 1)) {
       tc_fence_after();
 #pragma unroll
       for (int hh = 0; hh < 2; ++hh) {
@@ -317,7 +319,6 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
   uint64_t* s_full = bars + 2 * kAttnStages;             // [2] S in TMEM
   uint64_t* s_free = s_full + 2;                         // [2] S read by the 4 softmax warps
   uint64_t* p_full = s_full + 4;                         // [2] P in smem (4 warp arrivals)
-  uint64_t* pv_done = s_full + 6;                        // O += P_j V_j retired (phase j)
   uint64_t* mma_done = s_full + 7;                       // every MMA of this CTA retired
   uint64_t* recv_bar = s_full + 8;
   uint64_t* q_full = s_full + 9;                         // Q tile in smem (4 warp arrivals)
@@ -374,7 +375,6 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
       mbar_init(smem_u32(&s_free[i]), kAttnSoftWarps);   // one arrival per softmax warp
       mbar_init(smem_u32(&p_full[i]), kAttnSoftWarps);
     }
-    mbar_init(smem_u32(pv_done), 1);
     mbar_init(smem_u32(mma_done), 1);
     mbar_init(smem_u32(q_full), kAttnSoftWarps);
     if (in_cluster) {
@@ -475,7 +475,6 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
 #pragma unroll
         for (int k = 0; k < 4; ++k)
           umma_f16(tmem + 128, pdesc + 2 * k, vdesc + 2 * k, idesc, (j > 0 || k > 0) ? 1u : 0u);
-        umma_commit(smem_u32(pv_done));
         umma_commit(smem_u32(&empty[s]));
       }
       umma_commit(smem_u32(mma_done));   // retires once every MMA above has
@@ -500,7 +499,7 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
     fence_proxy_async_smem();
     __syncwarp();
     if (lane == 0) mbar_arrive(smem_u32(q_full));
-    AttnSync y{s_full, s_free, p_full, pv_done, sP, red};
+    AttnSync y{s_full, s_free, p_full, empty, sP, red};
     if (dup == 4) ok = attn_softmax<4>(a, y, tmem, np, p_begin, R, tok0, m, lc);
     else if (dup == 2) ok = attn_softmax<2>(a, y, tmem, np, p_begin, R, tok0, m, lc);
     else ok = attn_softmax<1>(a, y, tmem, np, p_begin, R, tok0, m, lc);
