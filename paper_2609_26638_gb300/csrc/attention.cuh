@@ -15,12 +15,14 @@
 // transposed, [64 dims][64 tokens] (8 KB each), so both are K-major operands.
 // Per page j:
 //   S_j = Q K_j^T       tcgen05.mma M=128 (rows) N=64 (keys) K=64 into TMEM
-//   softmax             one thread per row: running max m (log2 units) and
-//                       sum l in fp32, P_j = exp2(s*scale - m) as fp16 into
-//                       shared memory (the A operand of the next MMA)
-//   O += P_j V_j        tcgen05.mma M=128 N=64 (dims) K=64 (keys), O in TMEM
+//   softmax             per row: running max m (log2 units), P_j =
+//                       exp2(s*scale - m) as fp16 into shared memory (the A
+//                       operand of the next MMA)
+//   O += P_j [V_j | 1]  tcgen05.mma M=128 N=80 K=64 (keys), O in TMEM: 64 dims
+//                       and, from 16 rows of ones kept after every V^T page,
+//                       the row sum l in O's column 64 (fp32 on the tensor core)
 // The max only moves when a page raises it by more than 2^8: then the thread
-// first rescales its O row in TMEM (and l) by exp2(m_old - m_new).  Smaller
+// first rescales its O row in TMEM (and l with it) by exp2(m_old - m_new).  Smaller
 // rises keep the old m, so P stays <= 2^8 (well inside fp16).  Either way
 // O / l is the softmax-weighted sum.  Warps 0-3 own rows 0-127 (TMEM lanes;
 // warps whose rows are all padding only keep the barriers' pace); warp 4
@@ -50,7 +52,8 @@ namespace gs {
 
 constexpr int kAttnStages = 3;             // K/V page pairs in flight
 constexpr int kAttnPageBytes = 64 * 128;  // 64 x 64 fp16
-constexpr int kAttnStageBytes = 2 * kAttnPageBytes;
+constexpr int kAttnOnesBytes = 16 * 128;  // 16 rows of fp16 ones after each V^T page
+constexpr int kAttnStageBytes = 2 * kAttnPageBytes + kAttnOnesBytes;
 constexpr int kAttnRow = 68;              // partial row: O[64], m, l, 2 pad (272 B)
 constexpr int kAttnMaxRows = 128;         // rows of one query block (the MMA's M)
 constexpr int kAttnMaxCluster = 16;       // items merged inside a cluster (16: non-portable size)
@@ -68,7 +71,7 @@ constexpr int kAttnQOff = 0;
 constexpr int kAttnPOff = kAttnMaxRows * 128;
 constexpr int kAttnRingOff = kAttnPOff + 2 * kAttnMaxRows * 128;
 constexpr int kAttnBarOff = kAttnRingOff + kAttnRingBytes;
-constexpr int kAttnSmemBytes = 1024 + kAttnBarOff + 256 + (2 * kAttnSoftThreads + 8 * kAttnMaxRows) * 4;
+constexpr int kAttnSmemBytes = 1024 + kAttnBarOff + 256 + 2 * kAttnSoftThreads * 4;
 constexpr int kAttnRowsFloats = (kAttnMaxRows + kAttnMaxCluster) * kAttnRow;
 static_assert(kAttnRingOff >= kAttnRowsFloats * 4 && kAttnRingBytes >= kAttnRowsFloats * 4,
               "Q + P hold the owner-grouped rows, the ring the received rows");
@@ -114,6 +117,16 @@ __device__ __forceinline__ void tmem_ld16_nowait(uint32_t taddr, uint32_t (&r)[1
         "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
         "=r"(r[14]), "=r"(r[15])
       : "r"(taddr));
+}
+
+__device__ __forceinline__ uint32_t tmem_ld1(uint32_t taddr) {
+  uint32_t r;
+  asm volatile("tcgen05.ld.sync.aligned.32x32b.x1.b32 {%0}, [%1];" : "=r"(r) : "r"(taddr));
+  return r;
+}
+
+__device__ __forceinline__ void tmem_st1(uint32_t taddr, uint32_t v) {
+  asm volatile("tcgen05.st.sync.aligned.32x32b.x1.b32 [%0], {%1};" ::"r"(taddr), "r"(v) : "memory");
 }
 
 // 2^x on the SFU (PTX ex2.approx.ftz.f32, one instruction): the P values are
@@ -169,17 +182,15 @@ __device__ __forceinline__ void softmax_bar_max() {
 // a page raises it by more than 2^8, so one vote over the softmax threads (a
 // hardware barrier) decides whether any row of the block rises, and only then
 // are the copies' page maxima exchanged through shared memory (always on the
-// first page, rarely after).  A rise rescales O (the copy-0 thread of the row;
-// the previous O += P V must have retired) and the row sums; then P_j =
-// exp2(s - m) as fp16 into row rr of the P tile and the row sum kept as eight
-// 8-column partials.  m, P, the partials and the rescale are the same for every
-// DUP.  Waits are bounded; a warp whose wait ran out keeps passing the named
+// first page, rarely after).  A rise rescales O and the row sum in O's column
+// 64 (the copy-0 thread of the row; the previous O += P V must have retired);
+// then P_j = exp2(s - m) as fp16 into row rr of the P tile.  m, P and the
+// rescale are the same for every DUP.  Waits are bounded; a warp whose wait ran out keeps passing the named
 // barriers and arriving on the MMA warp's barriers to the last page, so no
 // thread is left at a barrier.  Returns false if a wait ran out.
 template <int DUP>
 __device__ __forceinline__ bool attn_softmax(const AttnArgs& a, const AttnSync& y, uint32_t tmem,
-                                             int np, int p_begin, int R, int tok0, float& m,
-                                             float (&lc)[8]) {
+                                             int np, int p_begin, int R, int tok0, float& m) {
   constexpr int RPC = kAttnMaxRows / DUP;   // MMA rows per copy
   constexpr int NC = 64 / DUP;              // columns per thread
   constexpr int NCH = NC / 8;               // 8-column chunks per thread
@@ -251,7 +262,7 @@ __device__ __forceinline__ bool attn_softmax(const AttnArgs& a, const AttnSync& 
 #pragma unroll
       for (int k = 0; k < DUP; ++k) mx = fmaxf(mx, y.red[k * RPC + rr]);
     }
-    // 4. a rise rescales O and the row sums first.  tcgen05.ld / st are
+    // 4. a rise rescales O and the row sum first.  tcgen05.ld / st are
     //    warp-collective: a warp with any rising row rescales all its rows,
     //    the others by exactly 1.
     const bool rise = any && mx > m + kAttnRescale;
@@ -268,14 +279,14 @@ __device__ __forceinline__ bool attn_softmax(const AttnArgs& a, const AttnSync& 
         for (int k = 0; k < 32; ++k) o32[k] = __float_as_uint(alpha * __uint_as_float(o32[k]));
         tmem_st32(trow + 128 + hh * 32, o32);
       }
+      // and the row sum, O's column 64
+      const uint32_t l1 = tmem_ld1(trow + 192);
+      tmem_wait_ld();
+      tmem_st1(trow + 192, __float_as_uint(alpha * __uint_as_float(l1)));
       tmem_wait_st();
     }
-    if (rise) {
-#pragma unroll
-      for (int c = 0; c < NCH; ++c) lc[c] *= alpha;
-      m = mx;
-    }
-    // 5. P_j = exp2(s - m) (fp16) into row rr of the P tile; 8-column sums
+    if (rise) m = mx;
+    // 5. P_j = exp2(s - m) (fp16) into row rr of the P tile
     if (have) {
       const float sub = (m == -INFINITY) ? 0.f : m;
       uint8_t* prow = y.sP + buf * kAttnMaxRows * 128;
@@ -284,7 +295,6 @@ __device__ __forceinline__ bool attn_softmax(const AttnArgs& a, const AttnSync& 
         float p[8];
 #pragma unroll
         for (int e = 0; e < 8; ++e) p[e] = ex2_sfu(fmaf(sv[8 * c + e], kScaleLog2, -sub));
-        lc[c] += ((p[0] + p[1]) + (p[2] + p[3])) + ((p[4] + p[5]) + (p[6] + p[7]));
         uint32_t w4[4];
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
@@ -387,6 +397,13 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
     s_int[3] = 0;
     fence_mbar_init();
   }
+  // the ones rows after every V^T page: O += P [V | 1] puts the row sum in O's column 64
+  for (int i = threadIdx.x; i < kAttnStages * kAttnOnesBytes / 16; i += blockDim.x) {
+    const int st = i / (kAttnOnesBytes / 16), off = i % (kAttnOnesBytes / 16);
+    *reinterpret_cast<uint4*>(ring + st * kAttnStageBytes + 2 * kAttnPageBytes + off * 16) =
+        make_uint4(0x3C003C00u, 0x3C003C00u, 0x3C003C00u, 0x3C003C00u);
+  }
+  fence_proxy_async_smem();
   if (warp == kAttnMmaWarp) tmem_alloc(smem_u32(tmem_slot), kAttnTmemCols);
   tc_fence_before();
   __syncthreads();
@@ -398,9 +415,7 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
   const int32_t* pt = a.page_table + static_cast<size_t>(slot) * a.pt_stride;
   bool ok = true;
   float m = -INFINITY, l = 0.f;   // the row's running max (log2 units) and sum
-  float lc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};   // row sum, 8-column partials
   float* red = reinterpret_cast<float*>(s_int + 8);        // [softmax threads] page maxima
-  float* lsum = red + 2 * kAttnSoftThreads;                // [8][128] partial sums
 
   if (warp == kAttnTmaWarp) {
     // ---- TMA producer: K and V^T pages of the item, in order
@@ -417,7 +432,7 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
         }
         const long long row = a.kv_row_base + static_cast<long long>(phys) * a.rows_per_page;
         const uint32_t fb = smem_u32(&full[s]);
-        mbar_arrive_expect_tx(fb, kAttnStageBytes);
+        mbar_arrive_expect_tx(fb, 2 * kAttnPageBytes);   // K and V^T (the ones rows stay)
         uint8_t* st = ring + s * kAttnStageBytes;
         tma_load_2d(smem_u32(st), &tmKV, 0, static_cast<int>(row + h * 64), fb, pol);
         tma_load_2d(smem_u32(st + kAttnPageBytes), &tmKV, 0, static_cast<int>(row + (a.Hkv + h) * 64),
@@ -446,6 +461,7 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
     pdl_trigger();
     if (lane == 0) {
       constexpr uint32_t idesc = umma_idesc_f16(128, 64);
+      constexpr uint32_t idesc_pv = umma_idesc_f16(128, 80);   // V^T page and its 16 ones rows
       const uint64_t qdesc = umma_desc_sw128(smem_u32(sQ));
       auto issue_s = [&](int j) -> bool {
         const int s = j % kAttnStages, buf = j & 1;
@@ -474,7 +490,7 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
         const uint64_t vdesc = umma_desc_sw128(smem_u32(ring + s * kAttnStageBytes + kAttnPageBytes));
 #pragma unroll
         for (int k = 0; k < 4; ++k)
-          umma_f16(tmem + 128, pdesc + 2 * k, vdesc + 2 * k, idesc, (j > 0 || k > 0) ? 1u : 0u);
+          umma_f16(tmem + 128, pdesc + 2 * k, vdesc + 2 * k, idesc_pv, (j > 0 || k > 0) ? 1u : 0u);
         umma_commit(smem_u32(&empty[s]));
       }
       umma_commit(smem_u32(mma_done));   // retires once every MMA above has
@@ -500,12 +516,9 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
     __syncwarp();
     if (lane == 0) mbar_arrive(smem_u32(q_full));
     AttnSync y{s_full, s_free, p_full, empty, sP, red};
-    if (dup == 4) ok = attn_softmax<4>(a, y, tmem, np, p_begin, R, tok0, m, lc);
-    else if (dup == 2) ok = attn_softmax<2>(a, y, tmem, np, p_begin, R, tok0, m, lc);
-    else ok = attn_softmax<1>(a, y, tmem, np, p_begin, R, tok0, m, lc);
-    // the row's eight 8-column partial sums -> shared memory [chunk][row]
-    const int mrow = threadIdx.x, nch = 8 / dup;
-    for (int cc = 0; cc < nch; ++cc) lsum[((mrow / rpc) * nch + cc) * kAttnMaxRows + mrow % rpc] = lc[cc];
+    if (dup == 4) ok = attn_softmax<4>(a, y, tmem, np, p_begin, R, tok0, m);
+    else if (dup == 2) ok = attn_softmax<2>(a, y, tmem, np, p_begin, R, tok0, m);
+    else ok = attn_softmax<1>(a, y, tmem, np, p_begin, R, tok0, m);
   }
 
   const bool all_ok = __syncthreads_and(ok);
@@ -516,21 +529,18 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
       mbar_wait(smem_u32(&full[i % kAttnStages]), (i / kAttnStages) & 1, a.err);
   }
   __syncthreads();
-  // the row's O from TMEM and its sum from the four partials (rows < R)
+  // the row's O and its sum (O's column 64) from TMEM (rows < R)
   const int r = threadIdx.x;
   const bool row_thread = r < R;
-  if (row_thread) {
-    const float* ls = lsum + r;
-    l = ((ls[0 * kAttnMaxRows] + ls[1 * kAttnMaxRows]) + (ls[2 * kAttnMaxRows] + ls[3 * kAttnMaxRows])) +
-        ((ls[4 * kAttnMaxRows] + ls[5 * kAttnMaxRows]) + (ls[6 * kAttnMaxRows] + ls[7 * kAttnMaxRows]));
-  }
   float o[64];
   if (warp < 4) {
     tc_fence_after();
     uint32_t o0[32], o1[32];
     tmem_ld32_nowait(tmem + (static_cast<uint32_t>(warp * 32) << 16) + 128, o0);
     tmem_ld32_nowait(tmem + (static_cast<uint32_t>(warp * 32) << 16) + 128 + 32, o1);
+    const uint32_t l1 = tmem_ld1(tmem + (static_cast<uint32_t>(warp * 32) << 16) + 192);
     tmem_wait_ld();
+    l = __uint_as_float(l1);
 #pragma unroll
     for (int k = 0; k < 32; ++k) {
       o[k] = __uint_as_float(o0[k]);
