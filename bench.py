@@ -71,9 +71,9 @@ _CSRC = os.path.join(ROOT, "paper_2609_26638_gb300", "csrc")
 NCU_TRAFFIC = {
     "attention_b1": dict(sources=("attention.cuh", "ptx.cuh"), bytes=4990976, algorithmic=4823040,
                          sha256="c4154e97724194c54884ba6a96d4f34400276927858e81f4dd4810b09e00183e"),
-    "attention_serve": dict(sources=("attention.cuh", "ptx.cuh"), bytes=233819648,
+    "attention_serve": dict(sources=("attention.cuh", "ptx.cuh"), bytes=233378304,
                             algorithmic=225173504,
-                            sha256="c4154e97724194c54884ba6a96d4f34400276927858e81f4dd4810b09e00183e"),
+                            sha256="f2eb4e50dce5541dd1624732eca164b8f2d58dde484e3e6a86061e1e6dbac85a"),
     "lm_head_b1": dict(sources=("gemm_tc.cuh", "gemm.cu", "ptx.cuh"), bytes=124897280,
                        algorithmic=121669768,
                        sha256="cf843ef01b07ec00b2c8f45ea0314bd187665ee6d84ddb19be137f33e3a34ecb"),
