@@ -332,9 +332,9 @@ int gs_wait_probe(gs_handle *h, int limit_us);
  *            logical pages [i * split_pages, (i + 1) * split_pages); items are
  *            reduced independently and merged in item order, so results depend
  *            on split_pages but not on n_seq, W or the other sequences.
- *            GS_ERR_UNSUPPORTED if ceil(pt_stride / split_pages) > 48 (the
- *            merge keeps each item's running max and sum of every row in
- *            shared memory).
+ *            GS_ERR_UNSUPPORTED if ceil(pt_stride / split_pages) > 54 (the
+ *            merge keeps each item's running max and sum of every row in the
+ *            kernel's idle page ring, 54 KB).
  *   stream   cudaStream_t */
 size_t gs_attention_scratch_bytes(int n_seq, int W, int n_heads, int n_kv_heads, int max_pages,
                                   int split_pages);
